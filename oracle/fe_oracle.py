@@ -1,0 +1,207 @@
+"""CPU oracle for FlashEvaluator joint evaluation (test infrastructure only).
+
+This is a plain, slow restatement in float64 numpy of what the evaluator of
+Section 4 computes.  It exists to check the CUDA path: only the test suite,
+the smoke check and the benchmark's CPU-baseline leg may import it, and it
+shares no code with the CUDA path.
+
+Model, in the paper's order (Section 4.1: H = Enc(x, U(z)) -> c = Idx(H, L) ->
+s = Inter(c), then Eq. 1's argmax):
+
+* Query Context Module (Section 4.2): X = LN(context); per layer l the
+  context keys/values K_l = X W_K^l, V_l = X W_V^l, computed once per request
+  (the K/V half of the QKV-Cache).
+* Distinct-element encoding (Section 4.2): for each element of
+  U(z) = union of the K sequences (Section 4.1), h = pool row; per layer
+  h += MHA(LN(h) W_Q^l, K_l, V_l) W_O^l;  h += FFN^l(LN(h)); output LN(h).
+  Each distinct element is encoded once (the Q-Cache).
+* Index-based assembly (Section 4.3): x_0 = [CLS], x_j = H[i_{k,j}] + P[j-1];
+  one CLS-pooled SeqEnc block gives c_k.
+* Cross-sequence interaction (Section 4.4): C' = C + MHA(LN(C)W_Qx,
+  LN(C)W_Kx, LN(C)W_Vx) W_Ox over the K sequences; score head
+  s_k = ReLU(LN(C'_k) W1h + b1h) . w2h + b2h.
+* Selection (Eq. 1): the smallest k attaining max_k s_k (the smallest-index
+  rule the paper uses for its listwise labels, Appendix B.1).
+
+The paper leaves the block internals open (norm placement, FFN, pooling, head
+shape).  The readings taken here: pre-LN blocks with LayerNorm without affine
+parameters, eps 1e-5, biased variance; FFN width 4d with ReLU; projections
+without bias, FFN and head with bias; attention scale 1/sqrt(d_h) with heads
+as contiguous column blocks; no position embedding on [CLS]; no masking.
+
+`evaluate(..., mode="no_reuse")` recomputes the context K/V for every sequence
+and every element occurrence independently (the candidate-factorized cost
+structure of Appendix A.3); `mode="reuse"` computes them once per request and
+once per distinct element.  Both must give the same numbers.
+
+Requests whose candidate indices fall outside [0, M) get NaN scores and best
+index -1 (the boundary's per-request error behaviour).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+__all__ = ["layer_norm", "softmax", "mha", "context_kv", "encode_elements",
+           "seq_encode", "cross_sequence", "score_head", "select_best",
+           "distinct_layout", "evaluate_request", "evaluate"]
+
+
+# -- building blocks --------------------------------------------------------
+
+def layer_norm(x, eps=1e-5):
+    """Per-row LayerNorm without affine parameters: (x - mean) / sqrt(var + eps),
+    var the biased variance over the last axis."""
+    x = np.asarray(x, dtype=np.float64)
+    mu = x.mean(axis=-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=-1, keepdims=True)
+    return (x - mu) / np.sqrt(var + eps)
+
+
+def softmax(z):
+    """Softmax over the last axis, with the row maximum subtracted first."""
+    z = np.asarray(z, dtype=np.float64)
+    e = np.exp(z - z.max(axis=-1, keepdims=True))
+    return e / e.sum(axis=-1, keepdims=True)
+
+
+def mha(q, k, v, n_heads):
+    """Multi-head scaled dot-product attention of query rows q [n, d] over key
+    rows k [m, d] with values v [m, d].  Head h uses columns
+    [h*d_h, (h+1)*d_h), d_h = d / n_heads; weights softmax(q_h k_h^T / sqrt(d_h))."""
+    n, d = q.shape
+    dh = d // n_heads
+    out = np.empty((n, d), dtype=np.float64)
+    for h in range(n_heads):
+        cols = slice(h * dh, (h + 1) * dh)
+        w = softmax(q[:, cols] @ k[:, cols].T / np.sqrt(dh))
+        out[:, cols] = w @ v[:, cols]
+    return out
+
+
+def _relu(x):
+    return np.maximum(x, 0.0)
+
+
+def _w(W, name):
+    return np.asarray(W[name], dtype=np.float64)
+
+
+# -- Section 4.2: request context and distinct elements ----------------------
+
+def context_kv(context_b, W, n_layers, eps):
+    """Query Context Module: per-layer context keys and values of one request,
+    [(K_1, V_1), ..., (K_Ly, V_Ly)], each [C, d]."""
+    X = layer_norm(context_b, eps)
+    return [(X @ _w(W, f"WK.{l}"), X @ _w(W, f"WV.{l}")) for l in range(n_layers)]
+
+
+def encode_elements(h0, kv, W, n_heads, eps):
+    """Request-conditioned representation of each element row of h0 [n, d]:
+    the cross-attention stack over the context K/V, then a final LN."""
+    h = np.array(h0, dtype=np.float64)
+    for l, (Kl, Vl) in enumerate(kv):
+        q = layer_norm(h, eps) @ _w(W, f"WQ.{l}")
+        h = h + mha(q, Kl, Vl, n_heads) @ _w(W, f"WO.{l}")
+        f = _relu(layer_norm(h, eps) @ _w(W, f"W1.{l}") + _w(W, f"b1.{l}"))
+        h = h + f @ _w(W, f"W2.{l}") + _w(W, f"b2.{l}")
+    return layer_norm(h, eps)
+
+
+# -- Section 4.3: index-based assembly and intra-sequence aggregation --------
+
+def seq_encode(elem_rows, W, n_heads, eps):
+    """c_k for one sequence whose element representations are elem_rows [L, d]:
+    tokens [CLS; rows + P[0..L-1]], one attention block whose output is the
+    [CLS] row, residual on [CLS], then a pre-LN FFN with residual."""
+    L = elem_rows.shape[0]
+    cls = _w(W, "cls")
+    x = np.vstack([cls[None, :], elem_rows + _w(W, "P")[:L]])
+    o = mha(x @ _w(W, "WQs"), x @ _w(W, "WKs"), x @ _w(W, "WVs"), n_heads)[0]
+    c = cls + o @ _w(W, "WOs")
+    f = _relu(layer_norm(c, eps) @ _w(W, "W1s") + _w(W, "b1s"))
+    return c + f @ _w(W, "W2s") + _w(W, "b2s")
+
+
+# -- Section 4.4: cross-sequence interaction and score head ------------------
+
+def cross_sequence(Cm, W, n_heads, eps):
+    """C' = C + MHA(Z W_Qx, Z W_Kx, Z W_Vx) W_Ox with Z = LN(C), over the K rows."""
+    Z = layer_norm(Cm, eps)
+    a = mha(Z @ _w(W, "WQx"), Z @ _w(W, "WKx"), Z @ _w(W, "WVx"), n_heads)
+    return Cm + a @ _w(W, "WOx")
+
+
+def score_head(Cp, W, eps):
+    """Shared prediction head s_k = ReLU(LN(C'_k) W1h + b1h) . w2h + b2h."""
+    f = _relu(layer_norm(Cp, eps) @ _w(W, "W1h") + _w(W, "b1h"))
+    return f @ _w(W, "w2h") + _w(W, "b2h")[0]
+
+
+def select_best(s):
+    """Eq. 1 argmax over k, ties resolved to the smallest index; -1 when any
+    score is NaN."""
+    s = np.asarray(s, dtype=np.float64)
+    if s.size == 0 or np.isnan(s).any():
+        return -1
+    return int(np.flatnonzero(s == s.max())[0])
+
+
+def distinct_layout(cand_b):
+    """U(z) of one request (Section 4.1) as the ascending list of distinct pool
+    rows, and slot[k, j] = position of cand_b[k, j] in that list."""
+    cand_b = np.asarray(cand_b)
+    uniq = np.unique(cand_b)
+    slots = np.searchsorted(uniq, cand_b).astype(np.int32)
+    return uniq.astype(np.int32), slots
+
+
+# -- whole evaluator ---------------------------------------------------------
+
+def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse"):
+    """Scores [K] of one request's K candidate sequences."""
+    H, Ly, eps = cfg.n_heads, cfg.n_layers, cfg.ln_eps
+    K, L = cand_b.shape
+    if mode == "reuse":
+        kv = context_kv(context_b, W, Ly, eps)
+        uniq, slots = distinct_layout(cand_b)
+        Henc = encode_elements(np.asarray(pool_b, np.float64)[uniq], kv, W, H, eps)
+        rows = [Henc[slots[k]] for k in range(K)]
+    elif mode == "no_reuse":
+        rows = []
+        for k in range(K):
+            kv = context_kv(context_b, W, Ly, eps)          # per sequence
+            r = np.vstack([encode_elements(np.asarray(pool_b, np.float64)[[m]], kv, W, H, eps)
+                           for m in cand_b[k]])             # per occurrence
+            rows.append(r)
+    else:
+        raise ValueError(mode)
+    Cm = np.vstack([seq_encode(rows[k], W, H, eps) for k in range(K)])
+    Cp = cross_sequence(Cm, W, H, eps)
+    return score_head(Cp, W, eps)
+
+
+def evaluate(context, pool, cand_idx, W, cfg, mode="reuse", requests=None):
+    """E_theta over a batch.  Returns (scores [B, K] float64, best [B] int32,
+    U [B] int32, slots [B, K, L] int32).  `requests` restricts the work to a
+    subset of request indices (the other rows stay NaN / -1)."""
+    context = np.asarray(context)
+    pool = np.asarray(pool)
+    cand_idx = np.asarray(cand_idx)
+    B, K, L = cand_idx.shape
+    M = pool.shape[1]
+    scores = np.full((B, K), np.nan)
+    best = np.full(B, -1, dtype=np.int32)
+    U = np.zeros(B, dtype=np.int32)
+    slots = np.full((B, K, L), -1, dtype=np.int32)
+    for b in (range(B) if requests is None else requests):
+        cb = cand_idx[b]
+        if cb.size and (cb.min() < 0 or cb.max() >= M):
+            continue
+        uniq, sl = distinct_layout(cb)
+        U[b] = len(uniq)
+        slots[b] = sl
+        if K == 0:
+            continue
+        scores[b] = evaluate_request(context[b], pool[b], cb, W, cfg, mode)
+        best[b] = select_best(scores[b])
+    return scores, best, U, slots
