@@ -1,0 +1,187 @@
+/*
+ * fe.h -- C-ABI of the GB300 joint evaluator (FlashEvaluator, arXiv 2603.02565).
+ *
+ * The library scores all K candidate sequences of each request in one pass
+ * (the joint mapping E_theta(z) in R^K of Section 3) and selects
+ * argmax_k s_k (Eq. 1).  It follows the QKV-Cache structure of Section 4:
+ *   1. the request context is encoded once into per-layer keys/values
+ *      (Section 4.2, "context-side key and value representations ... computed
+ *      only once");
+ *   2. every DISTINCT element of U(z) = union of the K sequences
+ *      (Section 4.1) gets its request-conditioned representation once
+ *      (cross-attention to the context + FFN; the Q-Cache of Section 4.2);
+ *   3. sequences are assembled by integer index plus position embeddings added
+ *      after indexing, prefixed with [CLS] and pooled by SeqEnc (Section 4.3);
+ *   4. self-attention across the K sequence vectors, then a shared score head
+ *      (Section 4.4), then the argmax of Eq. 1 (ties -> smallest k).
+ *
+ * Model definition (the paper leaves block internals open; these are the
+ * readings this library implements):
+ *   LN(x)   = (x - mean) / sqrt(var + ln_eps), biased var, no affine params.
+ *   MHA     = per head softmax(q_h k_h^T / sqrt(d_h)) v_h, heads are
+ *             contiguous column blocks of width d_h = d / n_heads.
+ *   context : X = LN(context); K_l = X WK_l, V_l = X WV_l       (l < n_layers)
+ *   element : h = pool row; per layer: h += MHA(LN(h) WQ_l, K_l, V_l) WO_l;
+ *             h += ReLU(LN(h) W1_l + b1_l) W2_l + b2_l;  H = LN(h)
+ *   SeqEnc  : x_0 = cls, x_j = H[i_{k,j}] + P[j-1];  o = MHA(x_0 WQs, x WKs, x WVs)
+ *             c = cls + o WOs;  c += ReLU(LN(c) W1s + b1s) W2s + b2s
+ *   cross   : C' = C + MHA(Z WQx, Z WKx, Z WVx) WOx,  Z = LN(C)  (over the K rows)
+ *   head    : s_k = ReLU(LN(C'_k) W1h + b1h) . w2h + b2h
+ *
+ * Arithmetic: bf16 tensor-core products with fp32 accumulation.  Activations
+ * feeding a product are carried as an unevaluated pair of bf16 values
+ * (hi + lo), so each product is hi*W + lo*W (plus hi*W_lo when the weights
+ * are not exactly bf16); softmax, LayerNorm and residual streams are fp32.
+ *
+ * Threading: a context is not thread-safe; calls on one context must be
+ * serialised (one in flight at a time per context).  Different contexts are
+ * independent.
+ */
+#ifndef FE_H_
+#define FE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Return codes.  No exception ever crosses this boundary. */
+enum {
+  FE_OK = 0,
+  FE_ERR_INVALID_ARG = 1,   /* null pointer, negative or zero size where >0 is required  */
+  FE_ERR_UNSUPPORTED = 2,   /* shape outside the limits listed below                     */
+  FE_ERR_INDEX = 3,         /* some cand_idx outside [0, M): those requests get NaN / -1 */
+  FE_ERR_WORKSPACE = 4,     /* workspace could not be sized for the call                 */
+  FE_ERR_OOM = 5,           /* device allocation failed                                  */
+  FE_ERR_CUDA = 6,          /* a CUDA call failed (message in fe_last_error_message)     */
+  FE_ERR_NUMERIC = 7,       /* a request produced a NaN score: its best index is -1      */
+  FE_ERR_TIMEOUT = 8        /* a bounded device-side wait gave up; results are invalid   */
+};
+
+/* Element type of the context / pool inputs. */
+enum { FE_IO_BF16 = 0, FE_IO_F32 = 1 };
+
+typedef struct fe_config {
+  int32_t d;          /* model width; multiple of 32, 32 <= d <= 512                  */
+  int32_t n_heads;    /* heads; d / n_heads must be 32 or 64                          */
+  int32_t n_layers;   /* depth of the element cross-attention stack, 1..8            */
+  int32_t ffn_mult;   /* FFN width F = ffn_mult * d, 1..8 (the readings use 4)        */
+  int32_t max_L;      /* rows of the position table P; sequences have L <= max_L     */
+  int32_t io_dtype;   /* FE_IO_BF16 or FE_IO_F32 for context and pool                 */
+  float   ln_eps;     /* LayerNorm epsilon (1e-5)                                     */
+} fe_config;
+
+typedef struct fe_ctx fe_ctx;
+
+/*
+ * Number of floats fe_init expects in `weights`, for this configuration.
+ * Returns 0 for an invalid configuration.
+ *
+ * Weight order (all fp32, row-major, y = x W with W stored [in, out]):
+ *   for l in 0..n_layers-1:
+ *     WQ_l[d,d] WK_l[d,d] WV_l[d,d] WO_l[d,d] W1_l[d,F] b1_l[F] W2_l[F,d] b2_l[d]
+ *   P[max_L,d] cls[d] WQs[d,d] WKs[d,d] WVs[d,d] WOs[d,d] W1s[d,F] b1s[F] W2s[F,d] b2s[d]
+ *   WQx[d,d] WKx[d,d] WVx[d,d] WOx[d,d]
+ *   W1h[d,d] b1h[d] w2h[d] b2h[1]
+ */
+size_t fe_weight_count(const fe_config* cfg);
+
+/*
+ * Create a context on the current CUDA device: validates `cfg`, copies the
+ * weights (host memory, fe_weight_count(cfg) floats, caller keeps ownership)
+ * to the device and precomputes the weight-only products of SeqEnc
+ * ([CLS] WQs, [CLS] WKs, [CLS] WVs, P WKs, P WVs).  Weights whose values are
+ * all bf16-representable are stored as one bf16 plane, others as a hi/lo pair.
+ * On success *out owns device memory until fe_destroy.
+ * Errors: FE_ERR_INVALID_ARG, FE_ERR_UNSUPPORTED, FE_ERR_OOM, FE_ERR_CUDA.
+ */
+int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx** out);
+
+/*
+ * Size the device workspace for batches up to (B, C, M, K, L) and build the
+ * TMA descriptors for it.  Optional: fe_evaluate grows the workspace itself
+ * when a call exceeds the reserved shape (that call then allocates).
+ * Limits: 1 <= C <= 65536, M <= 262144, K <= 4096, L <= max_L, B <= 65535.
+ * Errors: FE_ERR_INVALID_ARG, FE_ERR_UNSUPPORTED, FE_ERR_OOM, FE_ERR_CUDA.
+ */
+int fe_reserve(fe_ctx* ctx, int B, int C, int M, int K, int L);
+
+/*
+ * Score a batch of B requests (device pointers, contiguous row-major):
+ *   context  [B, C, d]  io_dtype     request contexts (x of Section 3)
+ *   pool     [B, M, d]  io_dtype     candidate pools C(x), one row per element
+ *   cand_idx [B, K, L]  int32        sequence k of request b is the pool rows
+ *                                    cand_idx[b,k,0..L-1] (L_k of Section 3)
+ *   scores_out [B, K]   float32      s_k of Section 4.4
+ *   best_out   [B]      int32        argmax_k s_k, smallest k on ties (Eq. 1)
+ * The work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ * stream) and the call waits for it, then returns the batch status:
+ *   FE_ERR_INDEX   some request had an index outside [0, M): that request's
+ *                  scores are NaN and its best index -1; others are valid.
+ *   FE_ERR_NUMERIC some request produced a NaN score (best index -1).
+ * Inputs must be 16-byte aligned.  The caller owns every buffer.  Repeated
+ * calls with the same shape and pointers replay one captured CUDA graph.
+ */
+int fe_evaluate(fe_ctx* ctx, int B, int C, int M, int K, int L,
+                const void* context, const void* pool, const int32_t* cand_idx,
+                float* scores_out, int32_t* best_out, void* stream);
+
+/*
+ * As fe_evaluate, but returns right after enqueueing (argument errors are
+ * still reported immediately).  The batch status of the most recent call is
+ * returned by fe_last_status, which waits for that call to finish.
+ */
+int fe_evaluate_async(fe_ctx* ctx, int B, int C, int M, int K, int L,
+                      const void* context, const void* pool, const int32_t* cand_idx,
+                      float* scores_out, int32_t* best_out, void* stream);
+int fe_last_status(fe_ctx* ctx);
+
+/*
+ * As fe_evaluate, for callers whose buffers live in HOST memory (same shapes
+ * and types).  Copies the inputs to library-owned device buffers on `stream`,
+ * evaluates, copies scores and best indices back and waits.  Page-locked host
+ * buffers give the fastest copies; pageable ones work.
+ */
+int fe_evaluate_host(fe_ctx* ctx, int B, int C, int M, int K, int L,
+                     const void* context, const void* pool, const int32_t* cand_idx,
+                     float* scores_out, int32_t* best_out, void* stream);
+
+/*
+ * Test hook: the distinct-element layout of the last evaluated batch, copied
+ * to host memory.  U_out[B] = |U(z_b)| (Section 4.1); slot_out[B,K,L] = rank of
+ * cand_idx[b,k,j] among the distinct indices of request b in ascending order
+ * (-1 for requests rejected with FE_ERR_INDEX).  Waits for the last call.
+ */
+int fe_debug_layout(fe_ctx* ctx, int32_t* slot_out, int32_t* U_out);
+
+/*
+ * Test hook: copy an intermediate of the last batch to host memory as fp32,
+ * row-major.  `name` is one of:
+ *   "ctx_ln"  [B*C, d]      LN(context)
+ *   "ctx_kv"  [B*C, 2*n_layers*d]  K_0 | V_0 | K_1 | V_1 ...
+ *   "elem"    [sum U, d]    H, the final element representations, requests in
+ *                           order, each request's elements in ascending pool index
+ *   "seq"     [B*K, d]      c_k, the SeqEnc output
+ *   "cross"   [B*K, d]      C', the cross-sequence output
+ * `max_floats` is the capacity of `dst`; *n_floats receives the element count
+ * (also when dst is NULL).  Waits for the last call.
+ */
+int fe_debug_fetch(fe_ctx* ctx, const char* name, float* dst, size_t max_floats,
+                   size_t* n_floats);
+
+/* Release every device resource owned by ctx (waits for its work first). */
+int fe_destroy(fe_ctx* ctx);
+
+/* Static description of a return code. */
+const char* fe_strerror(int code);
+
+/* Thread-local detail of the last FE_ERR_CUDA / FE_ERR_UNSUPPORTED on this thread. */
+const char* fe_last_error_message(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FE_H_ */

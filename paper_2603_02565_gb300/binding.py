@@ -1,0 +1,224 @@
+"""Python binding of libfe.so: argument marshalling only.
+
+Every step of the evaluation runs in the library's CUDA kernels; this module
+packs the weights in the order fe.h documents, passes device pointers of torch
+tensors (or host buffers) through ctypes and turns return codes into
+exceptions.  It never computes anything itself and has no fallback: without
+the built library every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libfe.so")
+
+FE_OK = 0
+FE_ERR_INVALID_ARG = 1
+FE_ERR_UNSUPPORTED = 2
+FE_ERR_INDEX = 3
+FE_ERR_WORKSPACE = 4
+FE_ERR_OOM = 5
+FE_ERR_CUDA = 6
+FE_ERR_NUMERIC = 7
+FE_ERR_TIMEOUT = 8
+FE_IO_BF16 = 0
+FE_IO_F32 = 1
+
+EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evaluate_async", "fe_last_status",
+           "fe_evaluate_host", "fe_debug_layout", "fe_debug_fetch", "fe_destroy", "fe_strerror",
+           "fe_last_error_message"]
+
+
+class FeConfig(ctypes.Structure):
+    _fields_ = [("d", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("n_layers", ctypes.c_int32),
+                ("ffn_mult", ctypes.c_int32), ("max_L", ctypes.c_int32), ("io_dtype", ctypes.c_int32),
+                ("ln_eps", ctypes.c_float)]
+
+
+class FeError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__(f"fe error {code}: {msg}")
+        self.code = code
+
+
+_lib = None
+
+
+def load_library(path: str = LIB_PATH):
+    """Load libfe.so and declare every entry point of fe.h."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise ImportError(f"{path} is not built; run paper_2603_02565_gb300.build.build()")
+    L = ctypes.CDLL(path)
+    vp, i32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+    L.fe_weight_count.argtypes = [ctypes.POINTER(FeConfig)]
+    L.fe_weight_count.restype = sz
+    L.fe_init.argtypes = [ctypes.POINTER(FeConfig), ctypes.POINTER(ctypes.c_float), sz, ctypes.POINTER(vp)]
+    L.fe_init.restype = i32
+    L.fe_reserve.argtypes = [vp, i32, i32, i32, i32, i32]
+    L.fe_reserve.restype = i32
+    for name in ("fe_evaluate", "fe_evaluate_async", "fe_evaluate_host"):
+        f = getattr(L, name)
+        f.argtypes = [vp, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp]
+        f.restype = i32
+    L.fe_last_status.argtypes = [vp]
+    L.fe_last_status.restype = i32
+    L.fe_debug_layout.argtypes = [vp, vp, vp]
+    L.fe_debug_layout.restype = i32
+    L.fe_debug_fetch.argtypes = [vp, ctypes.c_char_p, vp, sz, ctypes.POINTER(sz)]
+    L.fe_debug_fetch.restype = i32
+    L.fe_destroy.argtypes = [vp]
+    L.fe_destroy.restype = i32
+    L.fe_strerror.argtypes = [i32]
+    L.fe_strerror.restype = ctypes.c_char_p
+    L.fe_last_error_message.argtypes = []
+    L.fe_last_error_message.restype = ctypes.c_char_p
+    _lib = L
+    return L
+
+
+def _check(rc, allowed=(FE_OK,)):
+    if rc not in allowed:
+        L = load_library()
+        raise FeError(rc, f"{L.fe_strerror(rc).decode()} ({L.fe_last_error_message().decode()})")
+    return rc
+
+
+def weight_order(n_layers: int):
+    """Tensor names in the order fe.h documents for fe_init."""
+    names = []
+    for l in range(n_layers):
+        names += [f"WQ.{l}", f"WK.{l}", f"WV.{l}", f"WO.{l}", f"W1.{l}", f"b1.{l}", f"W2.{l}", f"b2.{l}"]
+    names += ["P", "cls", "WQs", "WKs", "WVs", "WOs", "W1s", "b1s", "W2s", "b2s",
+              "WQx", "WKx", "WVx", "WOx", "W1h", "b1h", "w2h", "b2h"]
+    return names
+
+
+def make_config(cfg) -> FeConfig:
+    """fe_config from any object with d, n_heads, n_layers, ffn_mult, max_L, io_bf16, ln_eps."""
+    return FeConfig(cfg.d, cfg.n_heads, cfg.n_layers, cfg.ffn_mult, cfg.max_L,
+                    FE_IO_BF16 if cfg.io_bf16 else FE_IO_F32, cfg.ln_eps)
+
+
+def pack_weights(cfg, weights: dict) -> np.ndarray:
+    parts = [np.ascontiguousarray(weights[n], dtype=np.float32).ravel() for n in weight_order(cfg.n_layers)]
+    return np.concatenate(parts)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(0 if t is None else t.data_ptr())
+
+
+class Evaluator:
+    """One library context: weights on the device plus a reusable workspace."""
+
+    def __init__(self, cfg, weights: dict):
+        L = load_library()
+        self.cfg = cfg
+        self._c = make_config(cfg)
+        flat = pack_weights(cfg, weights)
+        need = L.fe_weight_count(ctypes.byref(self._c))
+        if need != flat.size:
+            raise FeError(FE_ERR_INVALID_ARG, f"weights have {flat.size} floats, library expects {need}")
+        h = ctypes.c_void_p()
+        _check(L.fe_init(ctypes.byref(self._c), flat.ctypes.data_as(ctypes.POINTER(ctypes.c_float)),
+                         flat.size, ctypes.byref(h)))
+        self._h = h
+        self.last_status = FE_OK
+
+    # -- lifetime -------------------------------------------------------------
+    def close(self):
+        if getattr(self, "_h", None):
+            load_library().fe_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def reserve(self, B, C, M, K, L):
+        _check(load_library().fe_reserve(self._h, B, C, M, K, L))
+
+    # -- evaluation -------------------------------------------------------------
+    def evaluate(self, context, pool, cand_idx, scores=None, best=None, stream=None, sync=True,
+                 allowed=(FE_OK, FE_ERR_INDEX, FE_ERR_NUMERIC)):
+        """context [B,C,d], pool [B,M,d] (bf16 or fp32 per the config), cand_idx [B,K,L]
+        int32, all CUDA tensors.  Returns (scores [B,K] fp32, best [B] int32)."""
+        import torch
+        B, C, _ = context.shape
+        M = pool.shape[1]
+        K, L = cand_idx.shape[1], cand_idx.shape[2]
+        dev = context.device
+        if scores is None:
+            scores = torch.empty((B, K), dtype=torch.float32, device=dev)
+        if best is None:
+            best = torch.empty((B,), dtype=torch.int32, device=dev)
+        for t in (context, pool, cand_idx, scores, best):
+            if not t.is_cuda or not t.is_contiguous():
+                raise ValueError("evaluate expects contiguous CUDA tensors")
+        if cand_idx.dtype != torch.int32:
+            raise ValueError("cand_idx must be int32")
+        want = torch.bfloat16 if self.cfg.io_bf16 else torch.float32
+        if context.dtype != want or pool.dtype != want:
+            raise ValueError(f"context and pool must be {want}")
+        if stream is None:
+            stream = torch.cuda.current_stream(dev).cuda_stream
+        Lb = load_library()
+        fn = Lb.fe_evaluate if sync else Lb.fe_evaluate_async
+        rc = fn(self._h, B, C, M, K, L, _ptr(context), _ptr(pool), _ptr(cand_idx), _ptr(scores), _ptr(best),
+                ctypes.c_void_p(stream))
+        self.last_status = _check(rc, allowed)
+        return scores, best
+
+    def wait(self, allowed=(FE_OK, FE_ERR_INDEX, FE_ERR_NUMERIC)):
+        """Status of the last evaluate(..., sync=False), after waiting for it."""
+        self.last_status = _check(load_library().fe_last_status(self._h), allowed)
+        return self.last_status
+
+    def evaluate_host(self, context, pool, cand_idx, scores=None, best=None, stream=0,
+                      allowed=(FE_OK, FE_ERR_INDEX, FE_ERR_NUMERIC)):
+        """Same as evaluate for host buffers (numpy arrays or CPU tensors, pinned or
+        not); the library copies in and out.  context/pool must already hold the
+        config's element type (uint16 bf16 bits, a bfloat16 tensor, or float32)."""
+        B, C, _ = context.shape
+        M = pool.shape[1]
+        K, L = cand_idx.shape[1], cand_idx.shape[2]
+        if scores is None:
+            scores = np.empty((B, K), dtype=np.float32)
+        if best is None:
+            best = np.empty((B,), dtype=np.int32)
+
+        def hp(a):
+            if hasattr(a, "data_ptr"):
+                return ctypes.c_void_p(a.data_ptr())
+            return ctypes.c_void_p(a.ctypes.data)
+
+        rc = load_library().fe_evaluate_host(self._h, B, C, M, K, L, hp(context), hp(pool), hp(cand_idx),
+                                             hp(scores), hp(best), ctypes.c_void_p(stream))
+        self.last_status = _check(rc, allowed)
+        return scores, best
+
+    # -- test hooks ---------------------------------------------------------------
+    def layout(self, B, K, L):
+        slots = np.empty((B, K, L), dtype=np.int32)
+        U = np.empty((B,), dtype=np.int32)
+        _check(load_library().fe_debug_layout(self._h, ctypes.c_void_p(slots.ctypes.data),
+                                              ctypes.c_void_p(U.ctypes.data)))
+        return slots, U
+
+    def fetch(self, name: str, cols: int | None = None):
+        Lb = load_library()
+        n = ctypes.c_size_t()
+        _check(Lb.fe_debug_fetch(self._h, name.encode(), None, 0, ctypes.byref(n)))
+        out = np.empty(n.value, dtype=np.float32)
+        _check(Lb.fe_debug_fetch(self._h, name.encode(), ctypes.c_void_p(out.ctypes.data), out.size,
+                                 ctypes.byref(n)))
+        c = cols or self.cfg.d
+        return out.reshape(-1, c) if out.size else out.reshape(0, c)

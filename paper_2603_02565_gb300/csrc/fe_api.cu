@@ -1,0 +1,966 @@
+// C-ABI of the joint evaluator: weights, workspace, TMA descriptors, the
+// launch sequence of one evaluation and its CUDA-graph cache.
+#include <algorithm>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "fe.h"
+#include "fe_kernels.h"
+
+using fe::bf16;
+
+namespace {
+
+thread_local std::string g_msg;
+
+int set_cuda_err(cudaError_t e, const char* what) {
+  g_msg = std::string(what) + ": " + cudaGetErrorString(e);
+  return FE_ERR_CUDA;
+}
+
+#define FE_CK(call)                                                     \
+  do {                                                                  \
+    cudaError_t e_ = (call);                                            \
+    if (e_ != cudaSuccess) return set_cuda_err(e_, #call);              \
+  } while (0)
+
+inline int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+// ---------------------------------------------------------------------------
+// TMA descriptor encoding (driver entry point, no link-time libcuda dependency)
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// A bf16 matrix stored as one or two planes (hi, lo), row-major [rows, ld].
+struct Planes {
+  bf16* h = nullptr;
+  bf16* l = nullptr;
+  int ld = 0;
+  int rows = 0;
+  CUtensorMap th{}, tl{};
+};
+
+int alloc_planes(Planes& p, int rows, int ld, bool two, std::vector<void*>& owned) {
+  p.rows = rows < 128 ? 128 : rows;  // TMA boxes of 128 rows stay inside every allocation
+  p.ld = ld;
+  const size_t bytes = (size_t)p.rows * ld * sizeof(bf16);
+  if (cudaMalloc(&p.h, bytes) != cudaSuccess) return FE_ERR_OOM;
+  owned.push_back(p.h);
+  FE_CK(cudaMemset(p.h, 0, bytes));
+  if (two) {
+    if (cudaMalloc(&p.l, bytes) != cudaSuccess) return FE_ERR_OOM;
+    owned.push_back(p.l);
+    FE_CK(cudaMemset(p.l, 0, bytes));
+  }
+  return FE_OK;
+}
+
+int encode_map(CUtensorMap* m, const bf16* base, int cols, int rows, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) {
+    g_msg = "cuTensorMapEncodeTiled is unavailable";
+    return FE_ERR_CUDA;
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * sizeof(bf16)};
+  cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
+  cuuint32_t es[2] = {1u, 1u};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<bf16*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    g_msg = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+    return FE_ERR_CUDA;
+  }
+  return FE_OK;
+}
+
+// Descriptors of an activation (A operand): 128-row boxes on both planes.
+int map_act(Planes& p) {
+  int rc = encode_map(&p.th, p.h, p.ld, p.rows, 128);
+  if (rc == FE_OK) rc = encode_map(&p.tl, p.l, p.ld, p.rows, 128);
+  return rc;
+}
+
+// A weight matrix W[K, N] stored transposed as B operand [N, K_pad] plus its GEMM tiling.
+struct Weight {
+  Planes p;
+  int N = 0, K_pad = 0, BN = 0, stages = 0;
+};
+
+int largest_bn(int N, int cap) {
+  for (int bn = cap; bn >= 32; bn -= 32)
+    if (N % bn == 0) return bn;
+  return 0;
+}
+
+struct Shape {
+  int B = 0, C = 0, M = 0, K = 0, L = 0;
+  bool operator==(const Shape& o) const { return B == o.B && C == o.C && M == o.M && K == o.K && L == o.L; }
+};
+
+struct IoPtrs {
+  const void* ctx;
+  const void* pool;
+  const int32_t* idx;
+  float* scores;
+  int32_t* best;
+  bool operator==(const IoPtrs& o) const {
+    return ctx == o.ctx && pool == o.pool && idx == o.idx && scores == o.scores && best == o.best;
+  }
+};
+
+struct GraphEntry {
+  Shape s;
+  IoPtrs io;
+  cudaGraphExec_t exec = nullptr;
+  unsigned long long last_use = 0;
+};
+
+}  // namespace
+
+struct fe_ctx {
+  fe_config cfg{};
+  int device = 0;
+  int d = 0, H = 0, dh = 0, Ly = 0, F = 0, dpad = 0, Fpad = 0, nb = 1;
+  std::vector<void*> owned_w;  // weight allocations
+  std::vector<void*> owned_ws; // workspace allocations
+  float* w32 = nullptr;        // every weight in fp32, fe_weight_count order
+  std::vector<size_t> woff;    // offsets into w32, by tensor index
+  // transposed bf16 weights
+  Weight ctx_kv;
+  std::vector<Weight> wq, wo, w1, w2;
+  Weight kvs, os, w1s, w2s, qkvx, ox, w1h;
+  float *q0 = nullptr, *k0 = nullptr, *v0 = nullptr, *kP = nullptr, *vP = nullptr;
+  // workspace
+  Shape cap_shape;  // reserved maxima
+  int cap_rows = 0; // B * min(M, K*L) of the reservation
+  int *status = nullptr, *U = nullptr, *off = nullptr, *bad = nullptr, *slot = nullptr, *list = nullptr;
+  unsigned* ticket = nullptr;
+  Planes X, KV, xln, q, a, mid, kvI, o, cln, mids, z, qkv, ax, lncp;
+  float *h = nullptr, *c = nullptr, *cp = nullptr;
+  void* in_ctx = nullptr;
+  void* in_pool = nullptr;
+  int32_t* in_idx = nullptr;
+  float* out_scores = nullptr;
+  int32_t* out_best = nullptr;
+  int* host_status = nullptr;  // page-locked
+  cudaEvent_t done_ev = nullptr;
+  cudaStream_t cap_stream = nullptr;
+  std::vector<GraphEntry> graphs;
+  unsigned long long use_clock = 0;
+  bool use_graph = true;
+  Shape last_shape;
+  bool have_last = false;
+};
+
+namespace {
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+bool config_ok(const fe_config* c) {
+  if (!c) return false;
+  const int d = c->d;
+  if (d != 32 && d != 64 && d != 128 && d != 256 && d != 512) return false;
+  if (c->n_heads <= 0 || d % c->n_heads) return false;
+  const int dh = d / c->n_heads;
+  if (dh != 32 && dh != 64) return false;
+  if (c->n_layers < 1 || c->n_layers > 8) return false;
+  if (c->ffn_mult < 1 || c->ffn_mult > 8) return false;
+  if (c->max_L < 1 || c->max_L > 4096) return false;
+  if (c->io_dtype != FE_IO_BF16 && c->io_dtype != FE_IO_F32) return false;
+  if (!(c->ln_eps >= 0.f)) return false;
+  return true;
+}
+
+// sizes of the weight tensors in fe_weight_count order
+std::vector<size_t> weight_sizes(const fe_config* c) {
+  const size_t d = c->d, F = (size_t)c->ffn_mult * c->d;
+  std::vector<size_t> s;
+  for (int l = 0; l < c->n_layers; ++l) {
+    s.push_back(d * d);  // WQ
+    s.push_back(d * d);  // WK
+    s.push_back(d * d);  // WV
+    s.push_back(d * d);  // WO
+    s.push_back(d * F);  // W1
+    s.push_back(F);      // b1
+    s.push_back(F * d);  // W2
+    s.push_back(d);      // b2
+  }
+  s.push_back((size_t)c->max_L * d);  // P
+  s.push_back(d);                     // cls
+  for (int i = 0; i < 4; ++i) s.push_back(d * d);  // WQs WKs WVs WOs
+  s.push_back(d * F);                 // W1s
+  s.push_back(F);                     // b1s
+  s.push_back(F * d);                 // W2s
+  s.push_back(d);                     // b2s
+  for (int i = 0; i < 4; ++i) s.push_back(d * d);  // WQx WKx WVx WOx
+  s.push_back(d * d);                 // W1h
+  s.push_back(d);                     // b1h
+  s.push_back(d);                     // w2h
+  s.push_back(1);                     // b2h
+  return s;
+}
+
+// tensor indices into weight_sizes()
+enum { T_WQ = 0, T_WK, T_WV, T_WO, T_W1, T_B1, T_W2, T_B2, T_PER_LAYER };
+int t_tail(const fe_ctx* c, int i) { return T_PER_LAYER * c->Ly + i; }
+enum { T_P = 0, T_CLS, T_WQS, T_WKS, T_WVS, T_WOS, T_W1S, T_B1S, T_W2S, T_B2S, T_WQX, T_WKX, T_WVX, T_WOX, T_W1H,
+       T_B1H, T_W2H, T_B2H };
+
+const float* wptr(const fe_ctx* c, int tensor) { return c->w32 + c->woff[tensor]; }
+const float* lw(const fe_ctx* c, int l, int i) { return wptr(c, T_PER_LAYER * l + i); }
+const float* tw(const fe_ctx* c, int i) { return wptr(c, t_tail(c, i)); }
+
+// Allocate the transposed weight [N, K_pad] and pick its tiling.
+int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
+  w.N = N;
+  w.K_pad = round_up(Kin, 64);
+  w.BN = largest_bn(N, bn_cap);
+  if (w.BN == 0) {
+    g_msg = "no column tile divides N";
+    return FE_ERR_UNSUPPORTED;
+  }
+  w.stages = fe::gemm_max_stages(w.BN, c->nb, w.K_pad);
+  int rc = alloc_planes(w.p, N, w.K_pad, c->nb > 1, c->owned_w);
+  if (rc != FE_OK) return rc;
+  const int box = w.BN > 256 ? 256 : w.BN;
+  rc = encode_map(&w.p.th, w.p.h, w.p.ld, w.p.rows, box);
+  if (rc == FE_OK) rc = encode_map(&w.p.tl, c->nb > 1 ? w.p.l : w.p.h, w.p.ld, w.p.rows, box);
+  return rc;
+}
+
+int fill_weight(Weight& w, const float* W, int Kin, int N, int row0) {
+  FE_CK(fe::transpose_split_launch(W, Kin, N, w.p.h, w.p.l, w.p.ld, row0, 0));
+  return FE_OK;
+}
+
+void free_list(std::vector<void*>& v) {
+  for (void* p : v) cudaFree(p);
+  v.clear();
+}
+
+void clear_graphs(fe_ctx* c) {
+  for (auto& g : c->graphs)
+    if (g.exec) cudaGraphExecDestroy(g.exec);
+  c->graphs.clear();
+}
+
+int gemm(fe_ctx* c, int epi, const Planes& A, const Weight& W, int rows, const int* rows_dev,
+         fe::GemmParams p, cudaStream_t s) {
+  p.rows = rows;
+  p.rows_dev = rows_dev;
+  p.N = W.N;
+  p.BN = (epi == fe::EPI_STORE) ? W.BN : W.N;
+  p.K_pad = W.K_pad;
+  p.nb = c->nb;
+  p.stages = (epi == fe::EPI_STORE) ? W.stages : fe::gemm_max_stages(p.BN, c->nb, W.K_pad);
+  p.status = c->status;
+  p.eps = c->cfg.ln_eps;
+  FE_CK(fe::gemm_launch(epi, &A.th, &A.tl, &W.p.th, &W.p.tl, p, s));
+  return FE_OK;
+}
+
+#define FE_RC(call)              \
+  do {                           \
+    int rc_ = (call);            \
+    if (rc_ != FE_OK) return rc_; \
+  } while (0)
+
+// The whole evaluation of one batch, enqueued on s (captured into a graph by the caller).
+int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) {
+  const int B = sh.B, C = sh.C, M = sh.M, K = sh.K, L = sh.L;
+  const int d = c->d, Ly = c->Ly;
+  const int io_f32 = c->cfg.io_dtype == FE_IO_F32;
+  const int cap = (M < K * L) ? M : K * L;
+  const int R = B * cap;
+  const int S = B * K;
+  FE_CK(cudaMemsetAsync(c->status, 0, sizeof(int), s));
+  if (K == 0) {
+    FE_CK(cudaMemsetAsync(io.best, 0xFF, (size_t)B * sizeof(int32_t), s));
+    FE_CK(cudaMemcpyAsync(c->host_status, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+    return FE_OK;
+  }
+  const int* sumU = c->off + B;  // device: number of distinct elements of the batch
+
+  // (a0) distinct-element compaction of every request
+  FE_CK(fe::compact_launch(io.idx, B, M, K, L, cap, c->U, c->off, c->bad, c->slot, c->list, c->status, c->ticket,
+                           s));
+  // (a1) context keys/values, once per request
+  FE_CK(fe::ctx_ln_launch(io.ctx, io_f32, B * C, d, c->cfg.ln_eps, c->X.h, c->X.l, c->X.ld, s));
+  {
+    fe::GemmParams p{};
+    p.out_h = c->KV.h;
+    p.out_l = c->KV.l;
+    p.ldo = c->KV.ld;
+    FE_RC(gemm(c, fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, s));
+  }
+  // (a2) distinct elements: gather + LN, then the cross-attention stack
+  FE_CK(fe::gather_ln_launch(io.pool, io_f32, B, M, d, cap, c->off, c->list, R, c->cfg.ln_eps, c->h, d, c->xln.h,
+                             c->xln.l, c->xln.ld, s));
+  for (int l = 0; l < Ly; ++l) {
+    fe::GemmParams p{};
+    p.out_h = c->q.h;
+    p.out_l = c->q.l;
+    p.ldo = c->q.ld;
+    FE_RC(gemm(c, fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, s));
+
+    fe::AttnParams ap{};
+    ap.q_h = c->q.h;
+    ap.q_l = c->q.l;
+    ap.ldq = c->q.ld;
+    ap.k_h = c->KV.h + (size_t)(2 * l) * d;
+    ap.k_l = c->KV.l + (size_t)(2 * l) * d;
+    ap.v_h = c->KV.h + (size_t)(2 * l + 1) * d;
+    ap.v_l = c->KV.l + (size_t)(2 * l + 1) * d;
+    ap.ldkv = c->KV.ld;
+    ap.o_h = c->a.h;
+    ap.o_l = c->a.l;
+    ap.ldo = c->a.ld;
+    ap.q_off_dev = c->off;
+    ap.q_cnt_dev = c->U;
+    ap.kv_stride = C;
+    ap.kv_cnt = C;
+    ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
+    FE_CK(fe::attn_launch(c->dh, c->H, B, cap, ap, s));
+
+    fe::GemmParams po{};
+    po.resid = c->h;
+    po.ldr = d;
+    po.x_out = c->h;
+    po.ldx = d;
+    po.ln_h = c->xln.h;
+    po.ln_l = c->xln.l;
+    po.ldln = c->xln.ld;
+    FE_RC(gemm(c, fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, s));
+
+    fe::GemmParams p1{};
+    p1.bias = lw(c, l, T_B1);
+    p1.relu = 1;
+    p1.out_h = c->mid.h;
+    p1.out_l = c->mid.l;
+    p1.ldo = c->mid.ld;
+    FE_RC(gemm(c, fe::EPI_STORE, c->xln, c->w1[l], R, sumU, p1, s));
+
+    fe::GemmParams p2{};
+    p2.bias = lw(c, l, T_B2);
+    p2.resid = c->h;
+    p2.ldr = d;
+    p2.x_out = c->h;
+    p2.ldx = d;
+    p2.ln_h = c->xln.h;
+    p2.ln_l = c->xln.l;
+    p2.ldln = c->xln.ld;
+    FE_RC(gemm(c, fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, s));
+  }
+  // element projections of SeqEnc: H WKs | H WVs
+  {
+    fe::GemmParams p{};
+    p.out_h = c->kvI.h;
+    p.out_l = c->kvI.l;
+    p.ldo = c->kvI.ld;
+    FE_RC(gemm(c, fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, s));
+  }
+  // (a3, a4) index-based assembly + [CLS] attention, then c = cls + o WOs, FFN
+  {
+    fe::ClsParams cp{};
+    cp.B = B;
+    cp.K = K;
+    cp.L = L;
+    cp.d = d;
+    cp.H = c->H;
+    cp.off = c->off;
+    cp.bad = c->bad;
+    cp.slot_local = c->slot;
+    cp.kv_h = c->kvI.h;
+    cp.kv_l = c->kvI.l;
+    cp.ldkv = c->kvI.ld;
+    cp.q0 = c->q0;
+    cp.k0 = c->k0;
+    cp.v0 = c->v0;
+    cp.kP = c->kP;
+    cp.vP = c->vP;
+    cp.o_h = c->o.h;
+    cp.o_l = c->o.l;
+    cp.ldo = c->o.ld;
+    cp.scale = 1.0f / sqrtf((float)c->dh);
+    FE_CK(fe::cls_attn_launch(cp, s));
+  }
+  {
+    fe::GemmParams p{};
+    p.resid = tw(c, T_CLS);
+    p.ldr = 0;
+    p.x_out = c->c;
+    p.ldx = d;
+    p.ln_h = c->cln.h;
+    p.ln_l = c->cln.l;
+    p.ldln = c->cln.ld;
+    FE_RC(gemm(c, fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, s));
+  }
+  {
+    fe::GemmParams p{};
+    p.bias = tw(c, T_B1S);
+    p.relu = 1;
+    p.out_h = c->mids.h;
+    p.out_l = c->mids.l;
+    p.ldo = c->mids.ld;
+    FE_RC(gemm(c, fe::EPI_STORE, c->cln, c->w1s, S, nullptr, p, s));
+  }
+  {
+    fe::GemmParams p{};
+    p.bias = tw(c, T_B2S);
+    p.resid = c->c;
+    p.ldr = d;
+    p.x_out = c->c;
+    p.ldx = d;
+    p.ln_h = c->z.h;
+    p.ln_l = c->z.l;
+    p.ldln = c->z.ld;
+    FE_RC(gemm(c, fe::EPI_RESID_LN, c->mids, c->w2s, S, nullptr, p, s));
+  }
+  // (a5) cross-sequence attention over the K sequence vectors of each request
+  {
+    fe::GemmParams p{};
+    p.out_h = c->qkv.h;
+    p.out_l = c->qkv.l;
+    p.ldo = c->qkv.ld;
+    FE_RC(gemm(c, fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, s));
+    fe::AttnParams ap{};
+    ap.q_h = c->qkv.h;
+    ap.q_l = c->qkv.l;
+    ap.ldq = c->qkv.ld;
+    ap.k_h = c->qkv.h + d;
+    ap.k_l = c->qkv.l + d;
+    ap.v_h = c->qkv.h + 2 * d;
+    ap.v_l = c->qkv.l + 2 * d;
+    ap.ldkv = c->qkv.ld;
+    ap.o_h = c->ax.h;
+    ap.o_l = c->ax.l;
+    ap.ldo = c->ax.ld;
+    ap.q_stride = K;
+    ap.q_cnt_fixed = K;
+    ap.kv_stride = K;
+    ap.kv_cnt = K;
+    ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
+    FE_CK(fe::attn_launch(c->dh, c->H, B, K, ap, s));
+    fe::GemmParams po{};
+    po.resid = c->c;
+    po.ldr = d;
+    po.x_out = c->cp;
+    po.ldx = d;
+    po.ln_h = c->lncp.h;
+    po.ln_l = c->lncp.l;
+    po.ldln = c->lncp.ld;
+    FE_RC(gemm(c, fe::EPI_RESID_LN, c->ax, c->ox, S, nullptr, po, s));
+  }
+  // (a6) score head and selection
+  {
+    fe::GemmParams p{};
+    p.bias = tw(c, T_B1H);
+    p.w2 = tw(c, T_W2H);
+    p.b2 = tw(c, T_B2H);
+    p.scores = io.scores;
+    FE_RC(gemm(c, fe::EPI_HEAD, c->lncp, c->w1h, S, nullptr, p, s));
+  }
+  FE_CK(fe::select_launch(io.scores, B, K, c->bad, io.best, c->status, s));
+  FE_CK(cudaMemcpyAsync(c->host_status, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  return FE_OK;
+}
+
+int status_to_rc(int st) {
+  if (st & fe::ST_TIMEOUT) return FE_ERR_TIMEOUT;
+  if (st & fe::ST_INDEX) return FE_ERR_INDEX;
+  if (st & fe::ST_NUMERIC) return FE_ERR_NUMERIC;
+  return FE_OK;
+}
+
+int check_shape(const fe_ctx* c, int B, int C, int M, int K, int L) {
+  if (B < 0 || C < 1 || M < 0 || K < 0 || L < 0) {
+    g_msg = "negative size or C < 1";
+    return FE_ERR_INVALID_ARG;
+  }
+  if (C > 65536 || M > 262144 || K > 4096 || L > c->cfg.max_L || B > 65535) {
+    g_msg = "shape outside the supported limits";
+    return FE_ERR_UNSUPPORTED;
+  }
+  const long long cap = (M < (long long)K * L) ? M : (long long)K * L;
+  if ((long long)B * cap > (1ll << 30) || (long long)B * C > (1ll << 30) || (long long)B * K > (1ll << 30)) {
+    g_msg = "batch too large";
+    return FE_ERR_UNSUPPORTED;
+  }
+  return FE_OK;
+}
+
+int reserve_impl(fe_ctx* c, Shape s) {
+  FE_RC(check_shape(c, s.B, s.C, s.M, s.K, s.L));
+  // grow monotonically
+  s.B = std::max(s.B, c->cap_shape.B);
+  s.C = std::max(s.C, c->cap_shape.C);
+  s.M = std::max(s.M, c->cap_shape.M);
+  s.K = std::max(s.K, c->cap_shape.K);
+  s.L = std::max(s.L, c->cap_shape.L);
+  FE_CK(cudaDeviceSynchronize());
+  clear_graphs(c);
+  free_list(c->owned_ws);
+  c->have_last = false;
+  const int d = c->d, Ly = c->Ly;
+  const long long capL = (long long)s.K * s.L;
+  const int cap = (int)((s.M < capL) ? s.M : capL);
+  const int B = s.B > 0 ? s.B : 1;
+  const int R = B * (cap > 0 ? cap : 1);
+  const int S = B * (s.K > 0 ? s.K : 1);
+  const int BC = B * s.C;
+  auto dalloc = [&](void** p, size_t bytes) -> int {
+    if (bytes == 0) bytes = 16;
+    if (cudaMalloc(p, bytes) != cudaSuccess) {
+      g_msg = "cudaMalloc of " + std::to_string(bytes) + " bytes failed";
+      return FE_ERR_OOM;
+    }
+    c->owned_ws.push_back(*p);
+    if (cudaMemset(*p, 0, bytes) != cudaSuccess) return set_cuda_err(cudaGetLastError(), "cudaMemset");
+    return FE_OK;
+  };
+  FE_RC(dalloc((void**)&c->status, sizeof(int)));
+  FE_RC(dalloc((void**)&c->ticket, sizeof(unsigned)));
+  FE_RC(dalloc((void**)&c->U, (size_t)B * sizeof(int)));
+  FE_RC(dalloc((void**)&c->off, (size_t)(B + 1) * sizeof(int)));
+  FE_RC(dalloc((void**)&c->bad, (size_t)B * sizeof(int)));
+  FE_RC(dalloc((void**)&c->slot, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int)));
+  FE_RC(dalloc((void**)&c->list, (size_t)R * sizeof(int)));
+  FE_RC(dalloc((void**)&c->h, (size_t)R * d * sizeof(float)));
+  FE_RC(dalloc((void**)&c->c, (size_t)S * d * sizeof(float)));
+  FE_RC(dalloc((void**)&c->cp, (size_t)S * d * sizeof(float)));
+  const size_t esz = c->cfg.io_dtype == FE_IO_F32 ? 4 : 2;
+  FE_RC(dalloc(&c->in_ctx, (size_t)BC * d * esz));
+  FE_RC(dalloc(&c->in_pool, (size_t)B * (s.M > 0 ? s.M : 1) * d * esz));
+  FE_RC(dalloc((void**)&c->in_idx, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int32_t)));
+  FE_RC(dalloc((void**)&c->out_scores, (size_t)S * sizeof(float)));
+  FE_RC(dalloc((void**)&c->out_best, (size_t)B * sizeof(int32_t)));
+  FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->KV, BC, 2 * Ly * d, true, c->owned_ws));
+  FE_RC(alloc_planes(c->xln, R, c->dpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->q, R, d, true, c->owned_ws));
+  FE_RC(alloc_planes(c->a, R, c->dpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->mid, R, c->Fpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->kvI, R, 2 * d, true, c->owned_ws));
+  FE_RC(alloc_planes(c->o, S, c->dpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->cln, S, c->dpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->mids, S, c->Fpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->z, S, c->dpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->qkv, S, 3 * d, true, c->owned_ws));
+  FE_RC(alloc_planes(c->ax, S, c->dpad, true, c->owned_ws));
+  FE_RC(alloc_planes(c->lncp, S, c->dpad, true, c->owned_ws));
+  for (Planes* p : {&c->X, &c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp})
+    FE_RC(map_act(*p));
+  c->cap_shape = s;
+  c->cap_rows = R;
+  return FE_OK;
+}
+
+bool fits(const fe_ctx* c, const Shape& s) {
+  const Shape& r = c->cap_shape;
+  return r.B > 0 && s.B <= r.B && s.C <= r.C && s.M <= r.M && s.K <= r.K && s.L <= r.L;
+}
+
+int launch_batch(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t stream) {
+  if (!fits(c, s)) FE_RC(reserve_impl(c, s));
+  c->last_shape = s;
+  c->have_last = true;
+  if (!c->use_graph) {
+    FE_RC(enqueue_batch(c, s, io, stream));
+    FE_CK(cudaEventRecord(c->done_ev, stream));
+    return FE_OK;
+  }
+  GraphEntry* hit = nullptr;
+  for (auto& g : c->graphs)
+    if (g.s == s && g.io == io) hit = &g;
+  if (!hit) {
+    if (c->graphs.size() >= 16) {
+      size_t oldest = 0;
+      for (size_t i = 1; i < c->graphs.size(); ++i)
+        if (c->graphs[i].last_use < c->graphs[oldest].last_use) oldest = i;
+      cudaGraphExecDestroy(c->graphs[oldest].exec);
+      c->graphs.erase(c->graphs.begin() + oldest);
+    }
+    cudaGraph_t graph = nullptr;
+    FE_CK(cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal));
+    int rc = enqueue_batch(c, s, io, c->cap_stream);
+    cudaError_t e = cudaStreamEndCapture(c->cap_stream, &graph);
+    if (rc != FE_OK) {
+      if (graph) cudaGraphDestroy(graph);
+      return rc;
+    }
+    if (e != cudaSuccess) return set_cuda_err(e, "cudaStreamEndCapture");
+    GraphEntry g;
+    g.s = s;
+    g.io = io;
+    e = cudaGraphInstantiate(&g.exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) return set_cuda_err(e, "cudaGraphInstantiate");
+    c->graphs.push_back(g);
+    hit = &c->graphs.back();
+  }
+  hit->last_use = ++c->use_clock;
+  FE_CK(cudaGraphLaunch(hit->exec, stream));
+  FE_CK(cudaEventRecord(c->done_ev, stream));
+  return FE_OK;
+}
+
+int wait_status(fe_ctx* c) {
+  FE_CK(cudaEventSynchronize(c->done_ev));
+  FE_CK(cudaGetLastError());
+  return status_to_rc(*c->host_status);
+}
+
+int check_io(const void* ctx, const void* pool, const int32_t* idx, const float* scores, const int32_t* best, int B,
+             int M, int K, int L) {
+  if (B == 0) return FE_OK;
+  if (!ctx || !best || (K > 0 && !scores) || (K * L > 0 && !idx) || (K * L > 0 && M > 0 && !pool)) {
+    g_msg = "null pointer";
+    return FE_ERR_INVALID_ARG;
+  }
+  auto mis = [](const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u); };
+  if (mis(ctx) || mis(pool) || mis(idx) || mis(scores) || mis(best)) {
+    g_msg = "buffers must be 16-byte aligned";
+    return FE_ERR_INVALID_ARG;
+  }
+  return FE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t fe_weight_count(const fe_config* cfg) {
+  if (!config_ok(cfg)) return 0;
+  size_t n = 0;
+  for (size_t s : weight_sizes(cfg)) n += s;
+  return n;
+}
+
+int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx** out) {
+  if (!out || !cfg || !weights) {
+    g_msg = "null argument";
+    return FE_ERR_INVALID_ARG;
+  }
+  *out = nullptr;
+  if (!config_ok(cfg)) {
+    g_msg = "unsupported configuration (d in {32,64,128,256,512}, d/n_heads in {32,64})";
+    return FE_ERR_UNSUPPORTED;
+  }
+  const size_t need = fe_weight_count(cfg);
+  if (n_floats != need) {
+    g_msg = "weight count " + std::to_string(n_floats) + " != " + std::to_string(need);
+    return FE_ERR_INVALID_ARG;
+  }
+  fe_ctx* c = new fe_ctx();
+  c->cfg = *cfg;
+  if (cudaGetDevice(&c->device) != cudaSuccess) {
+    delete c;
+    g_msg = "no CUDA device";
+    return FE_ERR_CUDA;
+  }
+  c->d = cfg->d;
+  c->H = cfg->n_heads;
+  c->dh = cfg->d / cfg->n_heads;
+  c->Ly = cfg->n_layers;
+  c->F = cfg->ffn_mult * cfg->d;
+  c->dpad = round_up(c->d, 64);
+  c->Fpad = round_up(c->F, 64);
+  const char* ng = std::getenv("FE_NO_GRAPH");
+  c->use_graph = !(ng && ng[0] == '1');
+  // one bf16 plane when every weight is bf16-representable, else hi + lo
+  c->nb = 1;
+  for (size_t i = 0; i < n_floats; ++i) {
+    uint32_t u;
+    std::memcpy(&u, weights + i, 4);
+    if (u & 0xFFFFu) {
+      c->nb = 2;
+      break;
+    }
+  }
+  auto fail = [&](int rc) {
+    fe_destroy(c);
+    return rc;
+  };
+  int rc = FE_OK;
+  if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess)
+    return fail(set_cuda_err(cudaGetLastError(), "kernel attributes"));
+  {
+    size_t o = 0;
+    for (size_t s : weight_sizes(cfg)) {
+      c->woff.push_back(o);
+      o += s;
+    }
+  }
+  if (cudaMalloc(&c->w32, n_floats * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+  c->owned_w.push_back(c->w32);
+  if (cudaMemcpy(c->w32, weights, n_floats * sizeof(float), cudaMemcpyHostToDevice) != cudaSuccess)
+    return fail(set_cuda_err(cudaGetLastError(), "weight copy"));
+  const int d = c->d, F = c->F, Ly = c->Ly;
+  if ((rc = make_weight(c, c->ctx_kv, 2 * Ly * d, d, 256)) != FE_OK) return fail(rc);
+  for (int l = 0; l < Ly; ++l) {
+    if ((rc = fill_weight(c->ctx_kv, lw(c, l, T_WK), d, d, 2 * l * d)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->ctx_kv, lw(c, l, T_WV), d, d, (2 * l + 1) * d)) != FE_OK) return fail(rc);
+  }
+  c->wq.resize(Ly);
+  c->wo.resize(Ly);
+  c->w1.resize(Ly);
+  c->w2.resize(Ly);
+  for (int l = 0; l < Ly; ++l) {
+    if ((rc = make_weight(c, c->wq[l], d, d, 256)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->wq[l], lw(c, l, T_WQ), d, d, 0)) != FE_OK) return fail(rc);
+    if ((rc = make_weight(c, c->wo[l], d, d, 512)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->wo[l], lw(c, l, T_WO), d, d, 0)) != FE_OK) return fail(rc);
+    if ((rc = make_weight(c, c->w1[l], F, d, 256)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->w1[l], lw(c, l, T_W1), d, F, 0)) != FE_OK) return fail(rc);
+    if ((rc = make_weight(c, c->w2[l], d, F, 512)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->w2[l], lw(c, l, T_W2), F, d, 0)) != FE_OK) return fail(rc);
+  }
+  if ((rc = make_weight(c, c->kvs, 2 * d, d, 256)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->kvs, tw(c, T_WKS), d, d, 0)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->kvs, tw(c, T_WVS), d, d, d)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->os, d, d, 512)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->os, tw(c, T_WOS), d, d, 0)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->w1s, F, d, 256)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->w1s, tw(c, T_W1S), d, F, 0)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->w2s, d, F, 512)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->w2s, tw(c, T_W2S), F, d, 0)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->qkvx, 3 * d, d, 256)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->qkvx, tw(c, T_WQX), d, d, 0)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->qkvx, tw(c, T_WKX), d, d, d)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->qkvx, tw(c, T_WVX), d, d, 2 * d)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->ox, d, d, 512)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->ox, tw(c, T_WOX), d, d, 0)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->w1h, d, d, 512)) != FE_OK) return fail(rc);
+  if ((rc = fill_weight(c->w1h, tw(c, T_W1H), d, d, 0)) != FE_OK) return fail(rc);
+  // weight-only products of SeqEnc: [CLS] W and P W
+  const int mL = cfg->max_L;
+  float* consts = nullptr;
+  if (cudaMalloc(&consts, (size_t)(3 + 2 * mL) * d * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+  c->owned_w.push_back(consts);
+  c->q0 = consts;
+  c->k0 = consts + d;
+  c->v0 = consts + 2 * d;
+  c->kP = consts + 3 * d;
+  c->vP = consts + (size_t)(3 + mL) * d;
+  if (fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WQS), d, c->q0, 0) != cudaSuccess ||
+      fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WKS), d, c->k0, 0) != cudaSuccess ||
+      fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WVS), d, c->v0, 0) != cudaSuccess ||
+      fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WKS), d, c->kP, 0) != cudaSuccess ||
+      fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WVS), d, c->vP, 0) != cudaSuccess)
+    return fail(set_cuda_err(cudaGetLastError(), "SeqEnc constants"));
+  if (cudaMallocHost(&c->host_status, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
+  *c->host_status = 0;
+  if (cudaEventCreateWithFlags(&c->done_ev, cudaEventDisableTiming) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
+    return fail(set_cuda_err(cudaGetLastError(), "stream/event"));
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return fail(set_cuda_err(e, "fe_init"));
+  *out = c;
+  return FE_OK;
+}
+
+int fe_reserve(fe_ctx* c, int B, int C, int M, int K, int L) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  Shape s{B, C, M, K, L};
+  return reserve_impl(c, s);
+}
+
+int fe_evaluate_async(fe_ctx* c, int B, int C, int M, int K, int L, const void* context, const void* pool,
+                      const int32_t* cand_idx, float* scores_out, int32_t* best_out, void* stream) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  FE_RC(check_shape(c, B, C, M, K, L));
+  FE_RC(check_io(context, pool, cand_idx, scores_out, best_out, B, M, K, L));
+  if (B == 0) {
+    *c->host_status = 0;
+    FE_CK(cudaEventRecord(c->done_ev, (cudaStream_t)stream));
+    return FE_OK;
+  }
+  Shape s{B, C, M, K, L};
+  IoPtrs io{context, pool, cand_idx, scores_out, best_out};
+  return launch_batch(c, s, io, (cudaStream_t)stream);
+}
+
+int fe_last_status(fe_ctx* c) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  return wait_status(c);
+}
+
+int fe_evaluate(fe_ctx* c, int B, int C, int M, int K, int L, const void* context, const void* pool,
+                const int32_t* cand_idx, float* scores_out, int32_t* best_out, void* stream) {
+  FE_RC(fe_evaluate_async(c, B, C, M, K, L, context, pool, cand_idx, scores_out, best_out, stream));
+  return fe_last_status(c);
+}
+
+int fe_evaluate_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* context, const void* pool,
+                     const int32_t* cand_idx, float* scores_out, int32_t* best_out, void* stream) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  FE_RC(check_shape(c, B, C, M, K, L));
+  if (B == 0) return FE_OK;
+  if (!context || !best_out || (K > 0 && !scores_out) || (K * L > 0 && !cand_idx) || (K * L > 0 && M > 0 && !pool)) {
+    g_msg = "null pointer";
+    return FE_ERR_INVALID_ARG;
+  }
+  Shape s{B, C, M, K, L};
+  if (!fits(c, s)) FE_RC(reserve_impl(c, s));
+  cudaStream_t st = (cudaStream_t)stream;
+  const size_t esz = c->cfg.io_dtype == FE_IO_F32 ? 4 : 2;
+  FE_CK(cudaMemcpyAsync(c->in_ctx, context, (size_t)B * C * c->d * esz, cudaMemcpyHostToDevice, st));
+  if (M > 0 && pool)
+    FE_CK(cudaMemcpyAsync(c->in_pool, pool, (size_t)B * M * c->d * esz, cudaMemcpyHostToDevice, st));
+  if (K * L > 0)
+    FE_CK(cudaMemcpyAsync(c->in_idx, cand_idx, (size_t)B * K * L * sizeof(int32_t), cudaMemcpyHostToDevice, st));
+  IoPtrs io{c->in_ctx, c->in_pool, c->in_idx, c->out_scores, c->out_best};
+  FE_RC(launch_batch(c, s, io, st));
+  if (K > 0) FE_CK(cudaMemcpyAsync(scores_out, c->out_scores, (size_t)B * K * sizeof(float), cudaMemcpyDeviceToHost, st));
+  FE_CK(cudaMemcpyAsync(best_out, c->out_best, (size_t)B * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  FE_CK(cudaEventRecord(c->done_ev, st));
+  return wait_status(c);
+}
+
+int fe_debug_layout(fe_ctx* c, int32_t* slot_out, int32_t* U_out) {
+  if (!c || !slot_out || !U_out) return FE_ERR_INVALID_ARG;
+  if (!c->have_last) {
+    g_msg = "no evaluated batch";
+    return FE_ERR_INVALID_ARG;
+  }
+  DeviceGuard g(c->device);
+  FE_CK(cudaEventSynchronize(c->done_ev));
+  const Shape& s = c->last_shape;
+  FE_CK(cudaMemcpy(U_out, c->U, (size_t)s.B * sizeof(int), cudaMemcpyDeviceToHost));
+  FE_CK(cudaMemcpy(slot_out, c->slot, (size_t)s.B * s.K * s.L * sizeof(int), cudaMemcpyDeviceToHost));
+  return FE_OK;
+}
+
+int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, size_t* n_floats) {
+  if (!c || !name || !n_floats) return FE_ERR_INVALID_ARG;
+  if (!c->have_last) {
+    g_msg = "no evaluated batch";
+    return FE_ERR_INVALID_ARG;
+  }
+  DeviceGuard g(c->device);
+  FE_CK(cudaEventSynchronize(c->done_ev));
+  const Shape& s = c->last_shape;
+  const int d = c->d;
+  const Planes* pl = nullptr;
+  const float* f32 = nullptr;
+  size_t rows = 0, cols = 0;
+  const std::string n(name);
+  if (n == "ctx_ln") {
+    pl = &c->X;
+    rows = (size_t)s.B * s.C;
+    cols = d;
+  } else if (n == "ctx_kv") {
+    pl = &c->KV;
+    rows = (size_t)s.B * s.C;
+    cols = 2 * c->Ly * d;
+  } else if (n == "elem") {
+    int sum = 0;
+    FE_CK(cudaMemcpy(&sum, c->off + s.B, sizeof(int), cudaMemcpyDeviceToHost));
+    pl = &c->xln;
+    rows = (size_t)sum;
+    cols = d;
+  } else if (n == "seq") {
+    f32 = c->c;
+    rows = (size_t)s.B * s.K;
+    cols = d;
+  } else if (n == "cross") {
+    f32 = c->cp;
+    rows = (size_t)s.B * s.K;
+    cols = d;
+  } else {
+    g_msg = "unknown buffer name";
+    return FE_ERR_INVALID_ARG;
+  }
+  *n_floats = rows * cols;
+  if (!dst) return FE_OK;
+  if (max_floats < rows * cols) {
+    g_msg = "destination too small";
+    return FE_ERR_INVALID_ARG;
+  }
+  if (f32) {
+    FE_CK(cudaMemcpy(dst, f32, rows * cols * sizeof(float), cudaMemcpyDeviceToHost));
+    return FE_OK;
+  }
+  std::vector<uint16_t> hh((size_t)rows * pl->ld), ll((size_t)rows * pl->ld);
+  if (rows) {
+    FE_CK(cudaMemcpy(hh.data(), pl->h, hh.size() * 2, cudaMemcpyDeviceToHost));
+    FE_CK(cudaMemcpy(ll.data(), pl->l, ll.size() * 2, cudaMemcpyDeviceToHost));
+  }
+  for (size_t r = 0; r < rows; ++r)
+    for (size_t j = 0; j < cols; ++j) {
+      const uint32_t a = (uint32_t)hh[r * pl->ld + j] << 16, b = (uint32_t)ll[r * pl->ld + j] << 16;
+      float fa, fb;
+      std::memcpy(&fa, &a, 4);
+      std::memcpy(&fb, &b, 4);
+      dst[r * cols + j] = fa + fb;
+    }
+  return FE_OK;
+}
+
+int fe_destroy(fe_ctx* c) {
+  if (!c) return FE_OK;
+  {
+    DeviceGuard g(c->device);
+    cudaDeviceSynchronize();
+    clear_graphs(c);
+    free_list(c->owned_ws);
+    free_list(c->owned_w);
+    if (c->host_status) cudaFreeHost(c->host_status);
+    if (c->done_ev) cudaEventDestroy(c->done_ev);
+    if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+  }
+  delete c;
+  return FE_OK;
+}
+
+const char* fe_strerror(int code) {
+  switch (code) {
+    case FE_OK: return "ok";
+    case FE_ERR_INVALID_ARG: return "invalid argument";
+    case FE_ERR_UNSUPPORTED: return "unsupported shape or configuration";
+    case FE_ERR_INDEX: return "candidate index outside [0, M)";
+    case FE_ERR_WORKSPACE: return "workspace could not be sized";
+    case FE_ERR_OOM: return "device allocation failed";
+    case FE_ERR_CUDA: return "CUDA error";
+    case FE_ERR_NUMERIC: return "NaN score";
+    case FE_ERR_TIMEOUT: return "device-side wait timed out";
+    default: return "unknown error";
+  }
+}
+
+const char* fe_last_error_message(void) { return g_msg.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,135 @@
+// Internal interface between the host orchestration (fe_api.cu) and the
+// kernels (fe_gemm.cu, fe_attn.cu, fe_misc.cu).  Not part of the C-ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace fe {
+
+typedef __nv_bfloat16 bf16;
+
+// Device status bits, OR-ed into the per-batch status word.
+enum : int {
+  ST_INDEX = 1,    // a request had an out-of-range candidate index
+  ST_NUMERIC = 2,  // a request produced a NaN score
+  ST_TIMEOUT = 4,  // a bounded wait gave up
+};
+
+// ---------------------------------------------------------------------------
+// tcgen05 GEMM:  D[r, n] = sum over planes  A_p[r, :] . B_q[n, :]
+// A: activation as two bf16 planes (hi, lo), row-major [rows, K_pad]
+// B: weights transposed, [N, K_pad], one or two bf16 planes (hi[, lo])
+// One CTA computes a 128 x BN tile; BN <= 512 (two N=256 MMAs above 256).
+// ---------------------------------------------------------------------------
+enum GemmEpilogue : int {
+  EPI_STORE = 0,    // out = [ReLU](acc + bias) as split planes
+  EPI_RESID_LN = 1, // x = resid + acc + bias -> x_out (fp32) and LN(x) as split planes; BN == N
+  EPI_HEAD = 2,     // s = ReLU(acc + bias) . w2 + b2 -> scores (fp32); BN == N
+};
+
+struct GemmParams {
+  int rows;             // row extent of the A descriptors
+  const int* rows_dev;  // when set: number of valid rows, read on the device
+  int N;                // output columns
+  int BN;               // columns per CTA (multiple of 32, <= 512)
+  int K_pad;            // reduction length, multiple of 64
+  int nb;               // weight planes: 1 (exact bf16) or 2 (hi + lo)
+  int stages;           // shared-memory pipeline depth
+  const float* bias;    // [N] or null
+  int relu;
+  // EPI_STORE
+  bf16* out_h;
+  bf16* out_l;
+  int ldo;
+  // EPI_RESID_LN
+  const float* resid;   // residual rows (ldr == 0: one row broadcast to every row)
+  int ldr;
+  float* x_out;
+  int ldx;
+  bf16* ln_h;
+  bf16* ln_l;
+  int ldln;
+  float eps;
+  // EPI_HEAD
+  const float* w2;
+  const float* b2;
+  float* scores;
+  int* status;
+};
+
+// Raises the dynamic shared-memory limit of the GEMM kernels (call once per device, outside capture).
+cudaError_t gemm_prepare();
+size_t gemm_smem_bytes(int BN, int nb, int stages);
+int gemm_max_stages(int BN, int nb, int K_pad);
+cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* b_h,
+                        const CUtensorMap* b_l, const GemmParams& p, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// Flash-style multi-head attention over request segments (split-bf16 operands)
+// segment b: query rows [q_off(b), q_off(b) + q_cnt(b)), key rows
+// [b * kv_stride, b * kv_stride + kv_cnt); grid (q tiles of 64, heads, segments)
+// ---------------------------------------------------------------------------
+struct AttnParams {
+  const bf16 *q_h, *q_l;
+  int ldq;
+  const bf16 *k_h, *k_l, *v_h, *v_l;
+  int ldkv;
+  bf16 *o_h, *o_l;
+  int ldo;
+  const int* q_off_dev;  // null: q_off = b * q_stride
+  const int* q_cnt_dev;  // null: q_cnt = q_cnt_fixed
+  int q_stride;
+  int q_cnt_fixed;
+  int kv_stride;
+  int kv_cnt;
+  float scale_log2;      // log2(e) / sqrt(d_h)
+};
+cudaError_t attn_prepare();
+cudaError_t attn_launch(int dh, int n_heads, int n_segments, int max_q, const AttnParams& p, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// element-wise / gather / selection kernels (fe_misc.cu)
+// ---------------------------------------------------------------------------
+// Raises the dynamic shared-memory limit of the compaction kernel (once per device).
+cudaError_t misc_prepare();
+// Distinct-element compaction of every request: bitmap over the pool, ranks,
+// distinct list, |U(z_b)|, bad-request flags; the last CTA scans U into offsets.
+cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int cap, int* U, int* off,
+                           int* bad, int* slot_local, int* list, int* status, unsigned* ticket,
+                           cudaStream_t s);
+// Per-row LN of the context -> split planes [rows, ldo]
+cudaError_t ctx_ln_launch(const void* x, int io_f32, int rows, int d, float eps, bf16* out_h, bf16* out_l,
+                          int ldo, cudaStream_t s);
+// Gather distinct pool rows of every request -> residual stream h (fp32) and LN(h) planes
+cudaError_t gather_ln_launch(const void* pool, int io_f32, int B, int M, int d, int cap, const int* off,
+                             const int* list, int max_rows, float eps, float* h, int ldh, bf16* ln_h,
+                             bf16* ln_l, int ldln, cudaStream_t s);
+// [CLS]-query attention of SeqEnc over [CLS; elements + P]; one warp per sequence
+struct ClsParams {
+  int B, K, L, d, H;
+  const int* off;
+  const int* bad;
+  const int* slot_local;  // [B, K, L]
+  const bf16 *kv_h, *kv_l;  // element projections [rows, 2d]: keys | values
+  int ldkv;
+  const float *q0, *k0, *v0;  // [CLS] WQs, [CLS] WKs, [CLS] WVs
+  const float *kP, *vP;       // P WKs, P WVs  [max_L, d]
+  bf16 *o_h, *o_l;
+  int ldo;
+  float scale;                // 1 / sqrt(d_h)
+};
+cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s);
+// argmax with smallest-index ties; NaN / bad requests -> -1 (+ status bits)
+cudaError_t select_launch(float* scores, int B, int K, const int* bad, int32_t* best, int* status,
+                          cudaStream_t s);
+// weight preparation: out[(row0 + n) * ldo + k] = split(W[k * N + n]) for k < Kin, n < N
+cudaError_t transpose_split_launch(const float* W, int Kin, int N, bf16* out_h, bf16* out_l, int ldo,
+                                   int row0, cudaStream_t s);
+// out[r, n] = sum_k X[r, k] W[k, n]  (fp32; init-time weight-only products)
+cudaError_t small_matmul_launch(const float* X, int R, int Kd, const float* W, int N, float* out,
+                                cudaStream_t s);
+
+}  // namespace fe

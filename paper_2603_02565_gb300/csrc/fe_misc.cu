@@ -1,0 +1,502 @@
+// Memory-bound kernels of the joint evaluator: distinct-element compaction
+// (Section 4.1), LayerNorm / gather of the element rows (Section 4.2),
+// index-based assembly with the [CLS]-pooled SeqEnc attention (Section 4.3),
+// the argmax of Eq. 1, and init-time weight preparation.
+#include <climits>
+
+#include "fe_common.cuh"
+#include "fe_kernels.h"
+
+namespace fe {
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// small helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Block-wide exclusive scan of one int per thread (blockDim.x == 256).
+__device__ int block_excl_scan_256(int v, int* total) {
+  __shared__ int warp_tot[8];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tot[warp] = x;
+  __syncthreads();
+  int base = 0, all = 0;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) {
+    if (w < warp) base += warp_tot[w];
+    all += warp_tot[w];
+  }
+  __syncthreads();
+  *total = all;
+  return base + x - v;
+}
+
+// DPL consecutive elements of type T -> float
+template <int DPL, typename T>
+__device__ __forceinline__ void load_vec(const T* src, float* out) {
+  if constexpr (sizeof(T) == 4) {
+    if constexpr (DPL % 4 == 0) {
+#pragma unroll
+      for (int i = 0; i < DPL; i += 4) {
+        const float4 q = *reinterpret_cast<const float4*>(src + i);
+        out[i] = q.x;
+        out[i + 1] = q.y;
+        out[i + 2] = q.z;
+        out[i + 3] = q.w;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) out[i] = reinterpret_cast<const float*>(src)[i];
+    }
+  } else {
+    if constexpr (DPL % 8 == 0) {
+#pragma unroll
+      for (int i = 0; i < DPL; i += 8) {
+        const uint4 q = *reinterpret_cast<const uint4*>(src + i);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          out[i + 2 * j] = bf16lo_f(w[j]);
+          out[i + 2 * j + 1] = bf16hi_f(w[j]);
+        }
+      }
+    } else if constexpr (DPL % 2 == 0) {
+#pragma unroll
+      for (int i = 0; i < DPL; i += 2) {
+        const uint32_t w = *reinterpret_cast<const uint32_t*>(src + i);
+        out[i] = bf16lo_f(w);
+        out[i + 1] = bf16hi_f(w);
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) out[i] = __bfloat162float(src[i]);
+    }
+  }
+}
+
+// split pair of DPL consecutive bf16 (hi plane + lo plane) -> float
+template <int DPL>
+__device__ __forceinline__ void load_split(const bf16* h, const bf16* l, float* out) {
+  float a[DPL], b[DPL];
+  load_vec<DPL>(h, a);
+  load_vec<DPL>(l, b);
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) out[i] = a[i] + b[i];
+}
+
+// DPL floats -> split planes
+template <int DPL>
+__device__ __forceinline__ void store_split(const float* x, bf16* h, bf16* l) {
+  if constexpr (DPL % 2 == 0) {
+    uint32_t hw[DPL / 2], lw[DPL / 2];
+#pragma unroll
+    for (int i = 0; i < DPL; i += 2) split2(x[i], x[i + 1], hw[i / 2], lw[i / 2]);
+    if constexpr (DPL % 8 == 0) {
+#pragma unroll
+      for (int i = 0; i < DPL / 2; i += 4) {
+        *reinterpret_cast<uint4*>(h + 2 * i) = make_uint4(hw[i], hw[i + 1], hw[i + 2], hw[i + 3]);
+        *reinterpret_cast<uint4*>(l + 2 * i) = make_uint4(lw[i], lw[i + 1], lw[i + 2], lw[i + 3]);
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < DPL / 2; ++i) {
+        *reinterpret_cast<uint32_t*>(h + 2 * i) = hw[i];
+        *reinterpret_cast<uint32_t*>(l + 2 * i) = lw[i];
+      }
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < DPL; ++i) split_bf16(x[i], h[i], l[i]);
+  }
+}
+
+// LN of a row distributed over a warp, DPL values per lane (biased variance, two passes)
+template <int DPL>
+__device__ __forceinline__ void warp_layer_norm(float* x, int d, float eps) {
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) s += x[i];
+  const float mean = warp_sum(s) / (float)d;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) {
+    const float t = x[i] - mean;
+    q = fmaf(t, t, q);
+  }
+  const float rstd = 1.0f / sqrtf(warp_sum(q) / (float)d + eps);
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) x[i] = (x[i] - mean) * rstd;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// distinct-element compaction, one CTA (256 threads) per request
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) compact_kernel(const int32_t* __restrict__ cand, int B, int M, int K,
+                                                      int L, int cap, int* U, int* off, int* bad, int* slot_local,
+                                                      int* list, int* status, unsigned* ticket) {
+  extern __shared__ uint32_t csm[];
+  const int W = (M + 31) >> 5;
+  uint32_t* bits = csm;
+  int* pre = reinterpret_cast<int*>(csm + W);
+  __shared__ int s_bad;
+  __shared__ int s_last;
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const int n = K * L;
+  const int32_t* cb = cand + (size_t)b * n;
+
+  for (int w = tid; w < W; w += 256) bits[w] = 0u;
+  if (tid == 0) s_bad = 0;
+  __syncthreads();
+  for (int i = tid; i < n; i += 256) {
+    const int m = cb[i];
+    if (m < 0 || m >= M)
+      s_bad = 1;
+    else
+      atomicOr(&bits[m >> 5], 1u << (m & 31));
+  }
+  __syncthreads();
+  if (s_bad) {
+    for (int i = tid; i < n; i += 256) slot_local[(size_t)b * n + i] = -1;
+    if (tid == 0) {
+      U[b] = 0;
+      bad[b] = 1;
+      atomicOr(status, ST_INDEX);
+    }
+  } else {
+    const int per = (W + 255) / 256;
+    const int w0 = min(W, tid * per), w1 = min(W, w0 + per);
+    int local = 0;
+    for (int w = w0; w < w1; ++w) local += __popc(bits[w]);
+    int total;
+    int run = block_excl_scan_256(local, &total);
+    for (int w = w0; w < w1; ++w) {
+      pre[w] = run;
+      run += __popc(bits[w]);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      U[b] = total;
+      bad[b] = 0;
+    }
+    for (int w = tid; w < W; w += 256) {
+      uint32_t x = bits[w];
+      int r = pre[w];
+      while (x) {
+        const int bit = __ffs(x) - 1;
+        list[(size_t)b * cap + r++] = w * 32 + bit;
+        x &= x - 1;
+      }
+    }
+    for (int i = tid; i < n; i += 256) {
+      const int m = cb[i];
+      slot_local[(size_t)b * n + i] = pre[m >> 5] + __popc(bits[m >> 5] & ((1u << (m & 31)) - 1u));
+    }
+  }
+  // the last CTA to finish turns the counts into offsets (no CTA waits on another)
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = (atomicAdd(ticket, 1u) == gridDim.x - 1);
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    const int per = (B + 255) / 256;
+    const int b0 = min(B, tid * per), b1 = min(B, b0 + per);
+    int local = 0;
+    for (int i = b0; i < b1; ++i) local += __ldcg(U + i);
+    int total;
+    int run = block_excl_scan_256(local, &total);
+    for (int i = b0; i < b1; ++i) {
+      off[i] = run;
+      run += __ldcg(U + i);
+    }
+    if (tid == 0) {
+      off[B] = total;
+      *ticket = 0u;
+    }
+  }
+}
+
+cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int cap, int* U, int* off,
+                           int* bad, int* slot_local, int* list, int* status, unsigned* ticket,
+                           cudaStream_t s) {
+  const size_t smem = (size_t)2 * ((M + 31) / 32) * sizeof(uint32_t);
+  compact_kernel<<<B, 256, smem, s>>>(cand, B, M, K, L, cap, U, off, bad, slot_local, list, status, ticket);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// LN of context rows -> split planes (one warp per row)
+// ---------------------------------------------------------------------------
+template <int DPL, typename T>
+__global__ void __launch_bounds__(256) ctx_ln_kernel(const T* __restrict__ x, int rows, float eps,
+                                                     bf16* out_h, bf16* out_l, int ldo) {
+  constexpr int d = DPL * 32;
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (r >= rows) return;
+  float v[DPL];
+  load_vec<DPL>(x + (size_t)r * d + lane * DPL, v);
+  warp_layer_norm<DPL>(v, d, eps);
+  store_split<DPL>(v, out_h + (size_t)r * ldo + lane * DPL, out_l + (size_t)r * ldo + lane * DPL);
+}
+
+// ---------------------------------------------------------------------------
+// gather the distinct pool rows -> h (fp32) and LN(h) planes (one warp per row)
+// ---------------------------------------------------------------------------
+template <int DPL, typename T>
+__global__ void __launch_bounds__(256) gather_ln_kernel(const T* __restrict__ pool, int B, int M, int cap,
+                                                        const int* __restrict__ off, const int* __restrict__ list,
+                                                        int max_rows, float eps, float* h, int ldh, bf16* ln_h,
+                                                        bf16* ln_l, int ldln) {
+  constexpr int d = DPL * 32;
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (r >= max_rows || r >= off[B]) return;
+  int lo = 0, hi = B - 1;  // largest b with off[b] <= r
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (off[mid] <= r)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  const int b = lo;
+  const int m = list[(size_t)b * cap + (r - off[b])];
+  float v[DPL];
+  load_vec<DPL>(pool + ((size_t)b * M + m) * d + lane * DPL, v);
+  float* hr = h + (size_t)r * ldh + lane * DPL;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) hr[i] = v[i];
+  warp_layer_norm<DPL>(v, d, eps);
+  store_split<DPL>(v, ln_h + (size_t)r * ldln + lane * DPL, ln_l + (size_t)r * ldln + lane * DPL);
+}
+
+template <typename T>
+static cudaError_t ctx_ln_t(const T* x, int rows, int d, float eps, bf16* oh, bf16* ol, int ldo, cudaStream_t s) {
+  const unsigned g = (unsigned)((rows + 7) / 8);
+  switch (d) {
+    case 32: ctx_ln_kernel<1, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
+    case 64: ctx_ln_kernel<2, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
+    case 128: ctx_ln_kernel<4, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
+    case 256: ctx_ln_kernel<8, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
+    case 512: ctx_ln_kernel<16, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t ctx_ln_launch(const void* x, int io_f32, int rows, int d, float eps, bf16* out_h, bf16* out_l,
+                          int ldo, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  if (io_f32) return ctx_ln_t(static_cast<const float*>(x), rows, d, eps, out_h, out_l, ldo, s);
+  return ctx_ln_t(static_cast<const bf16*>(x), rows, d, eps, out_h, out_l, ldo, s);
+}
+
+template <typename T>
+static cudaError_t gather_t(const T* pool, int B, int M, int d, int cap, const int* off, const int* list,
+                            int max_rows, float eps, float* h, int ldh, bf16* lh, bf16* ll, int ldln,
+                            cudaStream_t s) {
+  const unsigned g = (unsigned)((max_rows + 7) / 8);
+#define FE_GATHER(DPL) \
+  gather_ln_kernel<DPL, T><<<g, 256, 0, s>>>(pool, B, M, cap, off, list, max_rows, eps, h, ldh, lh, ll, ldln)
+  switch (d) {
+    case 32: FE_GATHER(1); break;
+    case 64: FE_GATHER(2); break;
+    case 128: FE_GATHER(4); break;
+    case 256: FE_GATHER(8); break;
+    case 512: FE_GATHER(16); break;
+    default: return cudaErrorInvalidValue;
+  }
+#undef FE_GATHER
+  return cudaGetLastError();
+}
+
+cudaError_t gather_ln_launch(const void* pool, int io_f32, int B, int M, int d, int cap, const int* off,
+                             const int* list, int max_rows, float eps, float* h, int ldh, bf16* ln_h,
+                             bf16* ln_l, int ldln, cudaStream_t s) {
+  if (max_rows <= 0) return cudaSuccess;
+  if (io_f32)
+    return gather_t(static_cast<const float*>(pool), B, M, d, cap, off, list, max_rows, eps, h, ldh, ln_h, ln_l,
+                    ldln, s);
+  return gather_t(static_cast<const bf16*>(pool), B, M, d, cap, off, list, max_rows, eps, h, ldh, ln_h, ln_l,
+                  ldln, s);
+}
+
+// ---------------------------------------------------------------------------
+// SeqEnc [CLS] attention: one warp per sequence (b, k).  Tokens are [CLS]
+// (key/value = [CLS] WKs / WVs) and the L indexed elements, whose keys/values
+// are the cached element projections plus the position projections
+// (x_j W = H[i] W + P[j-1] W; positions added after indexing).
+// ---------------------------------------------------------------------------
+template <int DPL>
+__global__ void __launch_bounds__(256) cls_attn_kernel(const ClsParams p) {
+  const int lane = threadIdx.x & 31;
+  const int seq = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (seq >= p.B * p.K) return;
+  const int b = seq / p.K;
+  const int d = p.d;
+  const int lph = 32 / p.H;  // lanes per head
+  const int d0 = lane * DPL;
+  float q[DPL], kx[DPL], vx[DPL], o[DPL];
+  load_vec<DPL>(p.q0 + d0, q);
+  load_vec<DPL>(p.k0 + d0, kx);
+  load_vec<DPL>(p.v0 + d0, vx);
+  // token 0: [CLS]
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) s = fmaf(q[i], kx[i], s);
+  for (int o2 = 1; o2 < lph; o2 <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o2);
+  float m = s * p.scale, l = 1.f;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) o[i] = vx[i];
+  const int L = p.bad[b] ? 0 : p.L;
+  const int base = p.off[b];
+  const int* sl = p.slot_local + (size_t)seq * p.L;
+  for (int j = 0; j < L; ++j) {
+    const size_t row = (size_t)(base + sl[j]) * p.ldkv;
+    float kp[DPL], vp[DPL];
+    load_split<DPL>(p.kv_h + row + d0, p.kv_l + row + d0, kx);
+    load_split<DPL>(p.kv_h + row + d + d0, p.kv_l + row + d + d0, vx);
+    load_vec<DPL>(p.kP + (size_t)j * d + d0, kp);
+    load_vec<DPL>(p.vP + (size_t)j * d + d0, vp);
+    s = 0.f;
+#pragma unroll
+    for (int i = 0; i < DPL; ++i) s = fmaf(q[i], kx[i] + kp[i], s);
+    for (int o2 = 1; o2 < lph; o2 <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o2);
+    s *= p.scale;
+    const float mn = fmaxf(m, s);
+    const float c = expf(m - mn);
+    const float e = expf(s - mn);
+    l = l * c + e;
+#pragma unroll
+    for (int i = 0; i < DPL; ++i) o[i] = o[i] * c + e * (vx[i] + vp[i]);
+    m = mn;
+  }
+  const float inv = 1.f / l;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) o[i] *= inv;
+  store_split<DPL>(o, p.o_h + (size_t)seq * p.ldo + d0, p.o_l + (size_t)seq * p.ldo + d0);
+}
+
+cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s) {
+  const int n = p.B * p.K;
+  if (n <= 0) return cudaSuccess;
+  const unsigned g = (unsigned)((n + 7) / 8);
+  switch (p.d) {
+    case 32: cls_attn_kernel<1><<<g, 256, 0, s>>>(p); break;
+    case 64: cls_attn_kernel<2><<<g, 256, 0, s>>>(p); break;
+    case 128: cls_attn_kernel<4><<<g, 256, 0, s>>>(p); break;
+    case 256: cls_attn_kernel<8><<<g, 256, 0, s>>>(p); break;
+    case 512: cls_attn_kernel<16><<<g, 256, 0, s>>>(p); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Eq. 1 selection: one warp per request; first maximal index; NaN -> -1
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) select_kernel(float* scores, int B, int K, const int* bad, int32_t* best,
+                                                     int* status) {
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (b >= B) return;
+  float* sb = scores + (size_t)b * K;
+  if (bad[b]) {
+    for (int k = lane; k < K; k += 32) sb[k] = __int_as_float(0x7fc00000);
+    if (lane == 0) best[b] = -1;
+    return;
+  }
+  float bv = -INFINITY;
+  int bi = INT_MAX;
+  bool nan = false;
+  for (int k = lane; k < K; k += 32) {
+    const float v = sb[k];
+    if (v != v)
+      nan = true;
+    else if (bi == INT_MAX || v > bv) {
+      bv = v;
+      bi = k;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (oi != INT_MAX && (bi == INT_MAX || ov > bv || (ov == bv && oi < bi))) {
+      bv = ov;
+      bi = oi;
+    }
+  }
+  nan = __any_sync(0xffffffffu, nan);
+  if (lane == 0) {
+    best[b] = nan ? -1 : bi;
+    if (nan) atomicOr(status, ST_NUMERIC);
+  }
+}
+
+cudaError_t select_launch(float* scores, int B, int K, const int* bad, int32_t* best, int* status,
+                          cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  select_kernel<<<(unsigned)((B + 7) / 8), 256, 0, s>>>(scores, B, K, bad, best, status);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// init-time weight preparation
+// ---------------------------------------------------------------------------
+__global__ void transpose_split_kernel(const float* __restrict__ W, int Kin, int N, bf16* out_h, bf16* out_l,
+                                       int ldo, int row0) {
+  const size_t total = (size_t)Kin * N;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
+    const int n = (int)(i % N), k = (int)(i / N);
+    bf16 h, l;
+    split_bf16(W[i], h, l);
+    const size_t o = (size_t)(row0 + n) * ldo + k;
+    out_h[o] = h;
+    if (out_l) out_l[o] = l;
+  }
+}
+
+cudaError_t transpose_split_launch(const float* W, int Kin, int N, bf16* out_h, bf16* out_l, int ldo, int row0,
+                                   cudaStream_t s) {
+  transpose_split_kernel<<<256, 256, 0, s>>>(W, Kin, N, out_h, out_l, ldo, row0);
+  return cudaGetLastError();
+}
+
+__global__ void small_matmul_kernel(const float* __restrict__ X, int R, int Kd, const float* __restrict__ W, int N,
+                                    float* out) {
+  const size_t total = (size_t)R * N;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
+    const int n = (int)(i % N), r = (int)(i / N);
+    float acc = 0.f;
+    for (int k = 0; k < Kd; ++k) acc = fmaf(X[(size_t)r * Kd + k], W[(size_t)k * N + n], acc);
+    out[i] = acc;
+  }
+}
+
+cudaError_t small_matmul_launch(const float* X, int R, int Kd, const float* W, int N, float* out, cudaStream_t s) {
+  if (R <= 0) return cudaSuccess;
+  small_matmul_kernel<<<128, 256, 0, s>>>(X, R, Kd, W, N, out);
+  return cudaGetLastError();
+}
+
+cudaError_t misc_prepare() {
+  return cudaFuncSetAttribute(compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 65536 + 1024);
+}
+
+}  // namespace fe

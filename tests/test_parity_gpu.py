@@ -1,0 +1,166 @@
+"""CUDA path vs the CPU oracle, through the C-ABI (needs a GB300)."""
+import numpy as np
+import pytest
+
+import oracle.fe_oracle as O
+from oracle import compare
+from paper_2603_02565_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def dev():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2603_02565_gb300 import build
+    build.build()
+    return torch.device("cuda:0")
+
+
+def to_dev(w, dev):
+    dt = torch.bfloat16 if w.cfg.io_bf16 else torch.float32
+    return (torch.from_numpy(w.context).to(dev, dt), torch.from_numpy(w.pool).to(dev, dt),
+            torch.from_numpy(np.ascontiguousarray(w.cand_idx)).to(dev))
+
+
+def run_gpu(w, dev, ev=None):
+    from paper_2603_02565_gb300.binding import Evaluator
+    ev = ev or Evaluator(w.cfg, w.weights)
+    ctx, pool, idx = to_dev(w, dev)
+    s, b = ev.evaluate(ctx, pool, idx)
+    return ev, s.cpu().numpy(), b.cpu().numpy()
+
+
+def check(w, gs, gb, requests=None):
+    o_s, o_b, o_U, o_sl = O.evaluate(w.context, w.pool, w.cand_idx, w.weights, w.cfg, requests=requests)
+    rq = list(range(w.shape[0])) if requests is None else list(requests)
+    err = compare.score_error(gs[rq], o_s[rq])
+    ok, exact = compare.best_ok(gb[rq], o_s[rq], o_b[rq])
+    assert err <= compare.REL_TOL, f"{w.name}: max rel err {err:.3e}"
+    assert ok, f"{w.name}: best index mismatch beyond near-ties (exact {exact:.3f})"
+    return o_s, o_b, o_U, o_sl, err
+
+
+def check_layout(ev, w, o_U, o_sl, requests=None):
+    B, C, M, K, L = w.shape
+    sl, U = ev.layout(B, K, L)
+    rq = list(range(B)) if requests is None else list(requests)
+    np.testing.assert_array_equal(U[rq], o_U[rq])
+    np.testing.assert_array_equal(sl[rq], o_sl[rq])
+
+
+def test_tiny(dev):
+    w = wl.make_workload("tiny")
+    ev, gs, gb = run_gpu(w, dev)
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb)
+    check_layout(ev, w, o_U, o_sl)
+    assert gb[0] == o_b[0]
+
+
+@pytest.mark.parametrize("B", [3, 8])
+def test_serving_small_batches(dev, B):
+    w = wl.make_workload("serving", B=B)
+    ev, gs, gb = run_gpu(w, dev)
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb)
+    check_layout(ev, w, o_U, o_sl)
+
+
+def test_stagewise_serving(dev):
+    """Intermediates: context LN, element cache, SeqEnc and cross-sequence outputs."""
+    w = wl.make_workload("serving", B=2)
+    ev, gs, gb = run_gpu(w, dev)
+    cfg, W = w.cfg, w.weights
+    eps = cfg.ln_eps
+    X = np.vstack([O.layer_norm(w.context[b], eps) for b in range(2)])
+    np.testing.assert_allclose(ev.fetch("ctx_ln"), X, rtol=0, atol=2e-5)
+    elem, seq, cross = [], [], []
+    for b in range(2):
+        kv = O.context_kv(w.context[b], W, cfg.n_layers, eps)
+        uniq, slots = O.distinct_layout(w.cand_idx[b])
+        Hb = O.encode_elements(w.pool[b][uniq], kv, W, cfg.n_heads, eps)
+        elem.append(Hb)
+        Cm = np.vstack([O.seq_encode(Hb[slots[k]], W, cfg.n_heads, eps) for k in range(w.shape[3])])
+        seq.append(Cm)
+        cross.append(O.cross_sequence(Cm, W, cfg.n_heads, eps))
+    np.testing.assert_allclose(ev.fetch("elem"), np.vstack(elem), rtol=0, atol=2e-4)
+    np.testing.assert_allclose(ev.fetch("seq"), np.vstack(seq), rtol=1e-3, atol=2e-5)
+    np.testing.assert_allclose(ev.fetch("cross"), np.vstack(cross), rtol=1e-3, atol=2e-5)
+
+
+@pytest.mark.parametrize("K", [10, 100, 1000])
+def test_ksweep_small(dev, K):
+    w = wl.make_workload("ksweep", K=K, B=3)
+    ev, gs, gb = run_gpu(w, dev)
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb)
+    check_layout(ev, w, o_U, o_sl)
+
+
+def test_summarisation_small(dev):
+    w = wl.summarisation(B=2)
+    ev, gs, gb = run_gpu(w, dev)
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb)
+    check_layout(ev, w, o_U, o_sl)
+
+
+def test_stress_small(dev):
+    w = wl.make_workload("stress", B=3)
+    ev, gs, gb = run_gpu(w, dev)
+    check(w, gs, gb)
+
+
+def test_bad_index_isolated(dev):
+    from paper_2603_02565_gb300 import binding
+    w = wl.make_workload("serving", B=4)
+    w.cand_idx = w.cand_idx.copy()
+    w.cand_idx[2, 7, 3] = w.shape[2]          # == M
+    w.cand_idx[3, 0, 0] = -1
+    ev, gs, gb = run_gpu(w, dev)
+    assert ev.last_status == binding.FE_ERR_INDEX
+    assert np.isnan(gs[2:]).all() and (gb[2:] == -1).all()
+    check(w, gs, gb, requests=[0, 1])
+
+
+def test_edge_shapes(dev):
+    """K = 1, L = 1, M = 1, and a sequence repeating one element."""
+    for kw in [dict(K=1), dict(L=1), dict(M=1, L=1, K=3), dict(K=2, L=3, M=3)]:
+        w = wl.make_workload("serving", B=2, **kw)
+        ev, gs, gb = run_gpu(w, dev)
+        check(w, gs, gb)
+    w = wl.make_workload("serving", B=2, K=3, L=4)
+    w.cand_idx = w.cand_idx.copy()
+    w.cand_idx[0, 1, :] = w.cand_idx[0, 1, 0]  # one element four times
+    ev, gs, gb = run_gpu(w, dev)
+    check(w, gs, gb)
+
+
+def test_repeat_calls_and_host_entry_agree(dev):
+    w = wl.make_workload("serving", B=5)
+    ev, gs1, gb1 = run_gpu(w, dev)
+    _, gs2, gb2 = run_gpu(w, dev, ev)
+    np.testing.assert_array_equal(gs1, gs2)
+    ctx = torch.from_numpy(w.context).to(torch.bfloat16).pin_memory()
+    pool = torch.from_numpy(w.pool).to(torch.bfloat16).pin_memory()
+    idx = torch.from_numpy(w.cand_idx).pin_memory()
+    hs, hb = ev.evaluate_host(ctx, pool, idx)
+    np.testing.assert_array_equal(hs, gs1)
+    np.testing.assert_array_equal(hb, gb1)
+
+
+def test_serving_full_batch(dev):
+    """The benchmark's serving batch (B=256, K=50), every request checked."""
+    w = wl.make_workload("serving")
+    ev, gs, gb = run_gpu(w, dev)
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb)
+    check_layout(ev, w, o_U, o_sl)
+
+
+def test_stress_full_batch_sampled(dev):
+    """Throughput-stress batch at full size (B=1024), 6 sampled requests checked."""
+    w = wl.make_workload("stress")
+    ev, gs, gb = run_gpu(w, dev)
+    rq = [0, 1, 511, 777, 1022, 1023]
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb, requests=rq)
+    check_layout(ev, w, o_U, o_sl, requests=rq)
