@@ -13,7 +13,7 @@
 namespace fe {
 
 // A bounded wait gives up after this many nanoseconds of %globaltimer.
-constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;
 
 // ---------------------------------------------------------------------------
 // split bf16: x ~= hi + lo with hi = bf16(x), lo = bf16(x - hi)
@@ -79,11 +79,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 
 // Wait for the completion of the phase with the given parity.  Gives up after
 // kWaitLimitNs, sets ST_TIMEOUT in *status and returns false.
+// Also gives up at once when another CTA of the batch has already timed out.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, int* status) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
-  while (true) {
+  for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 0u && (*reinterpret_cast<volatile int*>(status) & ST_TIMEOUT)) return false;
     if (globaltimer_ns() - t0 > kWaitLimitNs) {
       atomicOr(status, ST_TIMEOUT);
       return false;
