@@ -1,0 +1,478 @@
+#!/usr/bin/env python3
+"""Throughput benchmark of the joint evaluator on GB300.
+
+One step = one joint evaluation of a whole batch (every stage of the hot
+path: compaction, context K/V, distinct-element encoding, assembly + SeqEnc,
+cross-sequence attention, head, argmax).  Default workload: the serving shape
+(B=256 requests, C=256, d=128, 4 heads, 2 layers, M=100, K=50, L=6, Zipf 1.1).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload serving]
+  python bench.py --impl reference ...   (the CPU oracle on the same workload)
+
+Prints one JSON line.  Multi-GPU runs (torchrun, one rank per GPU) give every
+rank its own batch of requests (requests are independent: weak scaling, no
+collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import datetime as _dt
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "requests/s and candidate sequences scored/s at K=50; p50 batch latency; % roofline"
+UNIT = "requests/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+# ----------------------------------------------------------------------------------------------
+# workload
+# ----------------------------------------------------------------------------------------------
+def make_workload(args, seed_offset=0):
+    from paper_2603_02565_gb300 import workloads as wl
+    kw = {}
+    if args.batch:
+        kw["B"] = args.batch
+    if args.workload == "serving":
+        return wl.serving(seed=1 + seed_offset, **kw)
+    if args.workload == "ksweep":
+        return wl.ksweep(args.K, seed=2 + seed_offset, **kw)
+    if args.workload == "stress":
+        return wl.stress(seed=4 + seed_offset, **kw)
+    if args.workload == "summarisation":
+        return wl.summarisation(seed=3 + seed_offset, **kw)
+    if args.workload == "tiny":
+        return wl.tiny(seed=0 + seed_offset)
+    raise SystemExit(f"unknown workload {args.workload}")
+
+
+def describe(w):
+    B, C, M, K, L = w.shape
+    c = w.cfg
+    return (f"{w.name}: B={B} requests, C={C}, d={c.d}, {c.n_heads} heads, {c.n_layers} layers, "
+            f"M={M}, K={K}, L={L}")
+
+
+# ----------------------------------------------------------------------------------------------
+# algorithmic work per launch site (flops, bytes); split activations are 4 B/element
+# ----------------------------------------------------------------------------------------------
+def site_work(site, cfg, B, C, M, K, L, R):
+    d, F, Ly = cfg.d, cfg.F, cfg.n_layers
+    S, n = B * K, B * C
+    esz = 2 if cfg.io_bf16 else 4
+    A = 4
+    t = {
+        "compact": (0, 4 * B * K * L * 2 + 4 * R + 12 * B),
+        "ctx_ln": (0, n * d * (esz + A)),
+        "gemm_ctx_kv": (2 * n * d * 2 * Ly * d, n * d * A + n * 2 * Ly * d * A),
+        "gather_ln": (0, R * d * (esz + 4 + A)),
+        "gemm_item_q": (2 * R * d * d, 2 * R * d * A),
+        "attn_item_ctx": (4 * R * C * d, 2 * R * d * A + 2 * n * d * A),
+        "gemm_item_o_ln": (2 * R * d * d, R * d * (A + 8 + A)),
+        "gemm_item_ffn1": (2 * R * d * F, R * d * A + R * F * A),
+        "gemm_item_ffn2_ln": (2 * R * F * d, R * F * A + R * d * (8 + A)),
+        "gemm_item_seq_kv": (4 * R * d * d, R * d * A + 2 * R * d * A),
+        "seq_cls_attn": (4 * S * (L + 1) * d, 2 * R * d * A + 4 * S * L + S * d * A),
+        "gemm_seq_o_ln": (2 * S * d * d, S * d * (A + 4 + A)),
+        "gemm_seq_ffn1": (2 * S * d * F, S * d * A + S * F * A),
+        "gemm_seq_ffn2_ln": (2 * S * F * d, S * F * A + S * d * (8 + A)),
+        "gemm_cross_qkv": (6 * S * d * d, S * d * A + 3 * S * d * A),
+        "attn_cross_seq": (4 * B * K * K * d, 3 * S * d * A + S * d * A),
+        "gemm_cross_o_ln": (2 * S * d * d, S * d * (A + 8 + A)),
+        "gemm_head": (2 * S * d * d + 3 * S * d, S * d * A + 4 * S),
+        "select": (0, 4 * S + 4 * B),
+    }
+    return t.get(site, (0, 0))
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index, interval_ms=20):
+        self.gpu = gpu_index
+        self.interval = interval_ms
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="fe_clocks_", suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", str(self.interval), "-f", self.path],
+                stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self, t0, t1):
+        if self.proc is None:
+            return None
+        time.sleep(0.05)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        try:
+            for line in open(self.path):
+                f = [x.strip() for x in line.split(",")]
+                if len(f) < 10:
+                    continue
+                try:
+                    ts = _dt.datetime.strptime(f[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                    rows.append((ts, float(f[2]), float(f[3]), f[6:10]))
+                except ValueError:
+                    continue
+        finally:
+            try:
+                os.remove(self.path)
+            except OSError:
+                pass
+        inside = [r for r in rows if t0 - 0.05 <= r[0] <= t1 + 0.05] or rows
+        if not inside:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i, v in enumerate(r[3]) if v.lower() == "active"})
+        return {"sm_mhz": float(np.median([r[1] for r in inside])), "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": reasons, "samples": len(inside), "samples_in_window": len(
+                    [r for r in rows if t0 <= r[0] <= t1])}
+
+
+# ----------------------------------------------------------------------------------------------
+# CPU baseline: the oracle as it stands, on a bounded sample of the workload
+# ----------------------------------------------------------------------------------------------
+def blas_threads():
+    for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(var):
+            try:
+                return int(os.environ[var])
+            except ValueError:
+                pass
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads", 0) for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def oracle_requests_per_s(w, budget_s=12.0, max_requests=None):
+    import oracle.fe_oracle as O
+    B = w.shape[0]
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        b = n % B
+        O.evaluate(w.context[b:b + 1], w.pool[b:b + 1], w.cand_idx[b:b + 1], w.weights, w.cfg)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s or (max_requests and n >= max_requests):
+            break
+    return n / el, n, el
+
+
+# ----------------------------------------------------------------------------------------------
+# GPU arm
+# ----------------------------------------------------------------------------------------------
+def run_ours(args):
+    import torch
+    from paper_2603_02565_gb300 import build
+    from paper_2603_02565_gb300.binding import FE_OK, Evaluator
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if rank == 0:
+        build.build()
+    if dist:
+        dist.barrier()
+    else:
+        build.build()
+
+    w = make_workload(args, seed_offset=0)
+    B, C, M, K, L = w.shape
+    cfg = w.cfg
+    ev = Evaluator(cfg, w.weights)
+    dt = torch.bfloat16 if cfg.io_bf16 else torch.float32
+    in_bytes = w.context.nbytes // (2 if cfg.io_bf16 else 1) + w.pool.nbytes // (2 if cfg.io_bf16 else 1) \
+        + w.cand_idx.nbytes
+    L2 = 126 * 2 ** 20
+    n_copies = int(min(16, max(2, math.ceil(2 * L2 / max(in_bytes, 1)))))
+    copies = []
+    for i in range(n_copies):
+        sh = (7 * i + 3 * rank) % B
+        ctx = torch.from_numpy(np.roll(w.context, sh, axis=0)).to(dev, dt)
+        pool = torch.from_numpy(np.roll(w.pool, sh, axis=0)).to(dev, dt)
+        idx = torch.from_numpy(np.ascontiguousarray(np.roll(w.cand_idx, sh, axis=0))).to(dev)
+        sc = torch.empty((B, K), dtype=torch.float32, device=dev)
+        be = torch.empty((B,), dtype=torch.int32, device=dev)
+        copies.append((ctx, pool, idx, sc, be))
+    stream = torch.cuda.current_stream(dev)
+    sh_ = stream.cuda_stream
+
+    def step(i):
+        c = copies[i % n_copies]
+        ev.evaluate(c[0], c[1], c[2], c[3], c[4], stream=sh_, sync=False)
+
+    # first pass: distinct-element statistics of the batch (layout hook)
+    step(0)
+    assert ev.wait() == FE_OK
+    slots, U = ev.layout(B, K, L)
+    sumU = int(U.sum())
+
+    # capture the graph of every input copy before timing anything
+    for i in range(n_copies):
+        step(i)
+    torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.start()
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_wall0 = time.time()
+    e0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    e1.record(stream)
+    e1.synchronize()
+    t_wall1 = time.time()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clocks = sampler.stop(t_wall0, t_wall1)
+    st = ev.wait()
+    if st != FE_OK:
+        raise SystemExit(f"batch status {st}")
+    launches = ev.kernels_per_batch()
+    total_ms = e0.elapsed_time(e1)
+    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    if dist:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * B * args.steps / (total_ms / 1e3)
+
+    # single-batch latency distribution (back to back, graph replay)
+    lat = []
+    n_lat = min(args.steps, 200)
+    for i in range(n_lat):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        step(i)
+        b.record(stream)
+        lat.append((a, b))
+    torch.cuda.synchronize()
+    lat_ms = sorted(a.elapsed_time(b) for a, b in lat)
+    p50 = float(np.percentile(lat_ms, 50))
+    p90 = float(np.percentile(lat_ms, 90))
+
+    # per-kernel times: the same steps launched kernel by kernel with events on this stream
+    ev.profile(True)
+    n_prof = min(args.steps, 50)
+    for i in range(n_prof):
+        step(i)
+    sites = ev.profile_read()
+    ev.profile(False)
+    peaks, peak_src = load_peaks()
+    kern = []
+    step_total = sum(s[2] for s in sites) / n_prof
+    for name, nl, tot in sites:
+        per_launch_ms = tot / nl
+        flops, byts = site_work(name, cfg, B, C, M, K, L, sumU)
+        kern.append({"site": name, "launches_per_step": nl / n_prof, "us_per_launch": per_launch_ms * 1e3,
+                     "share": (tot / n_prof) / step_total if step_total else 0.0,
+                     "gbs": byts / (per_launch_ms * 1e-3) / 1e9 if byts else 0.0,
+                     "tflops": flops / (per_launch_ms * 1e-3) / 1e12 if flops else 0.0})
+    dom = max(kern, key=lambda k: k["share"])
+    flops, byts = site_work(dom["site"], cfg, B, C, M, K, L, sumU)
+    t_launch = dom["us_per_launch"] * 1e-6
+    tensor_bound = flops / (peaks["bf16_tflops"] * 1e12) > byts / (peaks["hbm_gbs"] * 1e9)
+    if tensor_bound:
+        ach = flops / t_launch / 1e12
+        roof = {"bound": "tensor", "achieved": ach, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s"}
+    else:
+        ach = byts / t_launch / 1e9
+        roof = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["traffic"] = recorded_traffic(dom["site"], w.name)
+    roof["kernel"] = dom["site"]
+    roof["peak_source"] = peak_src
+    roof["algorithmic_per_launch"] = {"flops": flops, "bytes": byts}
+
+    # end to end through the C-ABI host entry: H2D of the inputs and D2H of the results timed
+    e2e = None
+    if not args.no_e2e:
+        hctx = torch.from_numpy(w.context).to(dt).pin_memory()
+        hpool = torch.from_numpy(w.pool).to(dt).pin_memory()
+        hidx = torch.from_numpy(np.ascontiguousarray(w.cand_idx)).pin_memory()
+        hsc = torch.empty((B, K), dtype=torch.float32).pin_memory()
+        hbe = torch.empty((B,), dtype=torch.int32).pin_memory()
+        for _ in range(3):
+            ev.evaluate_host(hctx, hpool, hidx, hsc, hbe, stream=sh_)
+        n_e2e = min(args.steps, 100)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(n_e2e):
+            ev.evaluate_host(hctx, hpool, hidx, hsc, hbe, stream=sh_)
+        el = time.perf_counter() - t0
+        te = torch.tensor([el], dtype=torch.float64, device=dev)
+        if dist:
+            dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        el = float(te.item())
+        e2e = {"value": world * B * n_e2e / el, "unit": UNIT,
+               "h2d_bytes_per_step": int(hctx.numel() * hctx.element_size() + hpool.numel() * hpool.element_size()
+                                         + hidx.numel() * 4),
+               "d2h_bytes_per_step": int(hsc.numel() * 4 + hbe.numel() * 4), "steps": n_e2e}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rps, n, el = oracle_requests_per_s(w, budget_s=args.cpu_seconds)
+        cpu = {"value": rps, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+               "sample": f"{n} requests of the {w.name} batch, one at a time (float64 numpy, reuse mode), "
+                         f"{el:.1f} s"}
+
+    if rank == 0:
+        out = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": describe(w), "global_batch": world * B, "K": K, "L": L,
+                       "parallelism": f"dp{world} (requests sharded, no collective)",
+                       "precision": "bf16 MMA operands, activations split hi+lo bf16, fp32 accumulate",
+                       "l2": f"inputs rotate over {n_copies} copies ({n_copies * in_bytes / 2**20:.0f} MB) "
+                             f"and each step writes {B * C * 2 * cfg.n_layers * cfg.d * 4 / 2**20:.0f} MB "
+                             f"of context K/V: > L2",
+                       "sum_U": sumU, "U_mean": sumU / B, "rho": K * L * B / max(sumU, 1)},
+            "seq_per_s": value * K, "p50_ms": p50, "p90_ms": p90,
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+            "gpu_launches": launches * args.steps, "kernels_per_step": launches,
+            "kernels": [{k: (round(v, 4) if isinstance(v, float) else v) for k, v in x.items()} for x in kern],
+        }
+        print(json.dumps(out))
+    ev.close()
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def recorded_traffic(site, workload_name):
+    """DRAM bytes per launch from a committed ncu capture of the same kernel
+    source, scaled to this workload; None when absent or the source changed."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(p) as f:
+            rec = json.load(f)
+    except Exception:
+        return None
+    r = rec.get(site)
+    if not r or r.get("workload") != workload_name:
+        return None
+    import hashlib
+    h = hashlib.sha256()
+    for src in r.get("sources", []):
+        with open(os.path.join(ROOT, src), "rb") as f:
+            h.update(f.read())
+    if h.hexdigest() != r.get("sources_sha256"):
+        return None
+    return r.get("bytes_per_launch")
+
+
+# ----------------------------------------------------------------------------------------------
+# reference arm: the oracle, timed on the host cores
+# ----------------------------------------------------------------------------------------------
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = make_workload(args)
+    B = w.shape[0]
+    import oracle.fe_oracle as O
+    for i in range(args.warmup):
+        b = i % B
+        O.evaluate(w.context[b:b + 1], w.pool[b:b + 1], w.cand_idx[b:b + 1], w.weights, w.cfg)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        b = i % B
+        O.evaluate(w.context[b:b + 1], w.pool[b:b + 1], w.cand_idx[b:b + 1], w.weights, w.cfg)
+    el = time.perf_counter() - t0
+    value = args.steps / el
+    out = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": describe(w), "global_batch": B, "K": w.shape[3], "L": w.shape[4],
+                   "parallelism": "host cores (oracle)"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+                         "sample": f"one request of the {w.name} batch per step, {args.steps} steps"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out))
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="serving",
+                    choices=["serving", "ksweep", "stress", "summarisation", "tiny"])
+    ap.add_argument("--K", type=int, default=50, help="sequences per request for --workload ksweep")
+    ap.add_argument("--batch", type=int, default=0, help="override B")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

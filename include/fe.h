@@ -171,6 +171,21 @@ int fe_debug_layout(fe_ctx* ctx, int32_t* slot_out, int32_t* U_out);
 int fe_debug_fetch(fe_ctx* ctx, const char* name, float* dst, size_t max_floats,
                    size_t* n_floats);
 
+/*
+ * Tracing.  fe_profile(ctx, 1) makes later evaluations launch kernel by kernel
+ * (no graph) with a pair of CUDA events on the caller's stream around every
+ * launch; fe_profile(ctx, 0) returns to graph replay.  fe_profile_read waits
+ * for the recorded work and reports, per launch site (in launch order):
+ *   names     site names, max_sites x 32 chars, NUL-terminated
+ *   launches  launches recorded at the site
+ *   total_ms  summed event time of those launches
+ * and clears the counters.  *n_sites receives the number of sites.
+ * fe_kernels_per_batch returns how many kernels the last batch launched.
+ */
+int fe_profile(fe_ctx* ctx, int enable);
+int fe_profile_read(fe_ctx* ctx, int max_sites, char* names, int* launches, double* total_ms, int* n_sites);
+int fe_kernels_per_batch(fe_ctx* ctx);
+
 /* Release every device resource owned by ctx (waits for its work first). */
 int fe_destroy(fe_ctx* ctx);
 

@@ -28,8 +28,8 @@ FE_IO_BF16 = 0
 FE_IO_F32 = 1
 
 EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evaluate_async", "fe_last_status",
-           "fe_evaluate_host", "fe_debug_layout", "fe_debug_fetch", "fe_destroy", "fe_strerror",
-           "fe_last_error_message"]
+           "fe_evaluate_host", "fe_debug_layout", "fe_debug_fetch", "fe_profile", "fe_profile_read",
+           "fe_kernels_per_batch", "fe_destroy", "fe_strerror", "fe_last_error_message"]
 
 
 class FeConfig(ctypes.Structure):
@@ -72,6 +72,12 @@ def load_library(path: str = LIB_PATH):
     L.fe_debug_layout.restype = i32
     L.fe_debug_fetch.argtypes = [vp, ctypes.c_char_p, vp, sz, ctypes.POINTER(sz)]
     L.fe_debug_fetch.restype = i32
+    L.fe_profile.argtypes = [vp, i32]
+    L.fe_profile.restype = i32
+    L.fe_profile_read.argtypes = [vp, i32, vp, vp, vp, ctypes.POINTER(i32)]
+    L.fe_profile_read.restype = i32
+    L.fe_kernels_per_batch.argtypes = [vp]
+    L.fe_kernels_per_batch.restype = i32
     L.fe_destroy.argtypes = [vp]
     L.fe_destroy.restype = i32
     L.fe_strerror.argtypes = [i32]
@@ -204,6 +210,28 @@ class Evaluator:
                                              hp(scores), hp(best), ctypes.c_void_p(stream))
         self.last_status = _check(rc, allowed)
         return scores, best
+
+    # -- tracing ----------------------------------------------------------------------
+    def profile(self, enable: bool):
+        _check(load_library().fe_profile(self._h, 1 if enable else 0))
+
+    def profile_read(self, max_sites: int = 64):
+        """[(site, launches, total_ms)] since the last read, in launch order."""
+        names = ctypes.create_string_buffer(32 * max_sites)
+        launches = np.zeros(max_sites, dtype=np.int32)
+        total = np.zeros(max_sites, dtype=np.float64)
+        n = ctypes.c_int()
+        _check(load_library().fe_profile_read(self._h, max_sites, names, ctypes.c_void_p(launches.ctypes.data),
+                                              ctypes.c_void_p(total.ctypes.data), ctypes.byref(n)))
+        raw = names.raw
+        out = []
+        for i in range(min(n.value, max_sites)):
+            nm = raw[32 * i:32 * (i + 1)].split(b"\0", 1)[0].decode()
+            out.append((nm, int(launches[i]), float(total[i])))
+        return out
+
+    def kernels_per_batch(self) -> int:
+        return int(load_library().fe_kernels_per_batch(self._h))
 
     # -- test hooks ---------------------------------------------------------------
     def layout(self, B, K, L):

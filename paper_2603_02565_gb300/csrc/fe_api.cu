@@ -131,6 +131,7 @@ struct IoPtrs {
 struct GraphEntry {
   Shape s;
   IoPtrs io;
+  int launches = 0;
   cudaGraphExec_t exec = nullptr;
   unsigned long long last_use = 0;
 };
@@ -170,6 +171,17 @@ struct fe_ctx {
   bool use_graph = true;
   Shape last_shape;
   bool have_last = false;
+  // tracing
+  struct Site {
+    std::string name;
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> pending, spare;
+    double total_ms = 0.0;
+    int launches = 0;
+  };
+  bool profiling = false;
+  std::vector<Site> sites;
+  int launches_batch = 0;  // kernels launched by the batch being enqueued
+  int launches_last = 0;
 };
 
 namespace {
@@ -182,6 +194,39 @@ struct DeviceGuard {
   ~DeviceGuard() {
     int cur;
     if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+// Counts a kernel launch of the batch and, while tracing, brackets it with events.
+struct Prof {
+  fe_ctx* c;
+  cudaStream_t s;
+  std::pair<cudaEvent_t, cudaEvent_t> ev{nullptr, nullptr};
+  fe_ctx::Site* site = nullptr;
+  Prof(fe_ctx* c_, const char* name, cudaStream_t s_) : c(c_), s(s_) {
+    ++c->launches_batch;
+    if (!c->profiling) return;
+    for (auto& x : c->sites)
+      if (x.name == name) site = &x;
+    if (!site) {
+      c->sites.emplace_back();
+      site = &c->sites.back();
+      site->name = name;
+    }
+    if (!site->spare.empty()) {
+      ev = site->spare.back();
+      site->spare.pop_back();
+    } else {
+      cudaEventCreate(&ev.first);
+      cudaEventCreate(&ev.second);
+    }
+    cudaEventRecord(ev.first, s);
+  }
+  ~Prof() {
+    if (site) {
+      cudaEventRecord(ev.second, s);
+      site->pending.push_back(ev);
+    }
   }
 };
 
@@ -273,8 +318,10 @@ void clear_graphs(fe_ctx* c) {
   c->graphs.clear();
 }
 
-int gemm(fe_ctx* c, int epi, const Planes& A, const Weight& W, int rows, const int* rows_dev,
+int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W, int rows, const int* rows_dev,
          fe::GemmParams p, cudaStream_t s) {
+  if (rows <= 0) return FE_OK;
+  Prof pf(c, site, s);
   p.rows = rows;
   p.rows_dev = rows_dev;
   p.N = W.N;
@@ -302,6 +349,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   const int cap = (M < K * L) ? M : K * L;
   const int R = B * cap;
   const int S = B * K;
+  c->launches_batch = 0;
   FE_CK(cudaMemsetAsync(c->status, 0, sizeof(int), s));
   if (K == 0) {
     FE_CK(cudaMemsetAsync(io.best, 0xFF, (size_t)B * sizeof(int32_t), s));
@@ -311,26 +359,35 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   const int* sumU = c->off + B;  // device: number of distinct elements of the batch
 
   // (a0) distinct-element compaction of every request
-  FE_CK(fe::compact_launch(io.idx, B, M, K, L, cap, c->U, c->off, c->bad, c->slot, c->list, c->status, c->ticket,
+  {
+    Prof pf(c, "compact", s);
+    FE_CK(fe::compact_launch(io.idx, B, M, K, L, cap, c->U, c->off, c->bad, c->slot, c->list, c->status, c->ticket,
                            s));
+  }
   // (a1) context keys/values, once per request
-  FE_CK(fe::ctx_ln_launch(io.ctx, io_f32, B * C, d, c->cfg.ln_eps, c->X.h, c->X.l, c->X.ld, s));
+  {
+    Prof pf(c, "ctx_ln", s);
+    FE_CK(fe::ctx_ln_launch(io.ctx, io_f32, B * C, d, c->cfg.ln_eps, c->X.h, c->X.l, c->X.ld, s));
+  }
   {
     fe::GemmParams p{};
     p.out_h = c->KV.h;
     p.out_l = c->KV.l;
     p.ldo = c->KV.ld;
-    FE_RC(gemm(c, fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, s));
   }
   // (a2) distinct elements: gather + LN, then the cross-attention stack
-  FE_CK(fe::gather_ln_launch(io.pool, io_f32, B, M, d, cap, c->off, c->list, R, c->cfg.ln_eps, c->h, d, c->xln.h,
+  {
+    Prof pf(c, "gather_ln", s);
+    FE_CK(fe::gather_ln_launch(io.pool, io_f32, B, M, d, cap, c->off, c->list, R, c->cfg.ln_eps, c->h, d, c->xln.h,
                              c->xln.l, c->xln.ld, s));
+  }
   for (int l = 0; l < Ly; ++l) {
     fe::GemmParams p{};
     p.out_h = c->q.h;
     p.out_l = c->q.l;
     p.ldo = c->q.ld;
-    FE_RC(gemm(c, fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, s));
+    FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, s));
 
     fe::AttnParams ap{};
     ap.q_h = c->q.h;
@@ -349,7 +406,10 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.kv_stride = C;
     ap.kv_cnt = C;
     ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
-    FE_CK(fe::attn_launch(c->dh, c->H, B, cap, ap, s));
+    {
+      Prof pf(c, "attn_item_ctx", s);
+      FE_CK(fe::attn_launch(c->dh, c->H, B, cap, ap, s));
+    }
 
     fe::GemmParams po{};
     po.resid = c->h;
@@ -359,7 +419,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     po.ln_h = c->xln.h;
     po.ln_l = c->xln.l;
     po.ldln = c->xln.ld;
-    FE_RC(gemm(c, fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, s));
+    FE_RC(gemm(c, "gemm_item_o_ln", fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, s));
 
     fe::GemmParams p1{};
     p1.bias = lw(c, l, T_B1);
@@ -367,7 +427,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p1.out_h = c->mid.h;
     p1.out_l = c->mid.l;
     p1.ldo = c->mid.ld;
-    FE_RC(gemm(c, fe::EPI_STORE, c->xln, c->w1[l], R, sumU, p1, s));
+    FE_RC(gemm(c, "gemm_item_ffn1", fe::EPI_STORE, c->xln, c->w1[l], R, sumU, p1, s));
 
     fe::GemmParams p2{};
     p2.bias = lw(c, l, T_B2);
@@ -378,7 +438,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p2.ln_h = c->xln.h;
     p2.ln_l = c->xln.l;
     p2.ldln = c->xln.ld;
-    FE_RC(gemm(c, fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, s));
+    FE_RC(gemm(c, "gemm_item_ffn2_ln", fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, s));
   }
   // element projections of SeqEnc: H WKs | H WVs
   {
@@ -386,7 +446,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.out_h = c->kvI.h;
     p.out_l = c->kvI.l;
     p.ldo = c->kvI.ld;
-    FE_RC(gemm(c, fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, s));
+    FE_RC(gemm(c, "gemm_item_seq_kv", fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, s));
   }
   // (a3, a4) index-based assembly + [CLS] attention, then c = cls + o WOs, FFN
   {
@@ -411,7 +471,10 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     cp.o_l = c->o.l;
     cp.ldo = c->o.ld;
     cp.scale = 1.0f / sqrtf((float)c->dh);
+    {
+    Prof pf(c, "seq_cls_attn", s);
     FE_CK(fe::cls_attn_launch(cp, s));
+  }
   }
   {
     fe::GemmParams p{};
@@ -422,7 +485,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.ln_h = c->cln.h;
     p.ln_l = c->cln.l;
     p.ldln = c->cln.ld;
-    FE_RC(gemm(c, fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_seq_o_ln", fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, s));
   }
   {
     fe::GemmParams p{};
@@ -431,7 +494,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.out_h = c->mids.h;
     p.out_l = c->mids.l;
     p.ldo = c->mids.ld;
-    FE_RC(gemm(c, fe::EPI_STORE, c->cln, c->w1s, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_seq_ffn1", fe::EPI_STORE, c->cln, c->w1s, S, nullptr, p, s));
   }
   {
     fe::GemmParams p{};
@@ -443,7 +506,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.ln_h = c->z.h;
     p.ln_l = c->z.l;
     p.ldln = c->z.ld;
-    FE_RC(gemm(c, fe::EPI_RESID_LN, c->mids, c->w2s, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_seq_ffn2_ln", fe::EPI_RESID_LN, c->mids, c->w2s, S, nullptr, p, s));
   }
   // (a5) cross-sequence attention over the K sequence vectors of each request
   {
@@ -451,7 +514,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.out_h = c->qkv.h;
     p.out_l = c->qkv.l;
     p.ldo = c->qkv.ld;
-    FE_RC(gemm(c, fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_cross_qkv", fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, s));
     fe::AttnParams ap{};
     ap.q_h = c->qkv.h;
     ap.q_l = c->qkv.l;
@@ -469,7 +532,10 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.kv_stride = K;
     ap.kv_cnt = K;
     ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
-    FE_CK(fe::attn_launch(c->dh, c->H, B, K, ap, s));
+    {
+      Prof pf(c, "attn_cross_seq", s);
+      FE_CK(fe::attn_launch(c->dh, c->H, B, K, ap, s));
+    }
     fe::GemmParams po{};
     po.resid = c->c;
     po.ldr = d;
@@ -478,7 +544,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     po.ln_h = c->lncp.h;
     po.ln_l = c->lncp.l;
     po.ldln = c->lncp.ld;
-    FE_RC(gemm(c, fe::EPI_RESID_LN, c->ax, c->ox, S, nullptr, po, s));
+    FE_RC(gemm(c, "gemm_cross_o_ln", fe::EPI_RESID_LN, c->ax, c->ox, S, nullptr, po, s));
   }
   // (a6) score head and selection
   {
@@ -487,10 +553,14 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.w2 = tw(c, T_W2H);
     p.b2 = tw(c, T_B2H);
     p.scores = io.scores;
-    FE_RC(gemm(c, fe::EPI_HEAD, c->lncp, c->w1h, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_head", fe::EPI_HEAD, c->lncp, c->w1h, S, nullptr, p, s));
   }
-  FE_CK(fe::select_launch(io.scores, B, K, c->bad, io.best, c->status, s));
+  {
+    Prof pf(c, "select", s);
+    FE_CK(fe::select_launch(io.scores, B, K, c->bad, io.best, c->status, s));
+  }
   FE_CK(cudaMemcpyAsync(c->host_status, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  c->launches_last = c->launches_batch;
   return FE_OK;
 }
 
@@ -593,7 +663,7 @@ int launch_batch(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t strea
   if (!fits(c, s)) FE_RC(reserve_impl(c, s));
   c->last_shape = s;
   c->have_last = true;
-  if (!c->use_graph) {
+  if (!c->use_graph || c->profiling) {
     FE_RC(enqueue_batch(c, s, io, stream));
     FE_CK(cudaEventRecord(c->done_ev, stream));
     return FE_OK;
@@ -621,6 +691,7 @@ int launch_batch(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t strea
     GraphEntry g;
     g.s = s;
     g.io = io;
+    g.launches = c->launches_last;
     e = cudaGraphInstantiate(&g.exec, graph, 0);
     cudaGraphDestroy(graph);
     if (e != cudaSuccess) return set_cuda_err(e, "cudaGraphInstantiate");
@@ -628,6 +699,7 @@ int launch_batch(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t strea
     hit = &c->graphs.back();
   }
   hit->last_use = ++c->use_clock;
+  c->launches_last = hit->launches;
   FE_CK(cudaGraphLaunch(hit->exec, stream));
   FE_CK(cudaEventRecord(c->done_ev, stream));
   return FE_OK;
@@ -930,12 +1002,59 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
   return FE_OK;
 }
 
+int fe_profile(fe_ctx* c, int enable) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  c->profiling = enable != 0;
+  return FE_OK;
+}
+
+int fe_profile_read(fe_ctx* c, int max_sites, char* names, int* launches, double* total_ms, int* n_sites) {
+  if (!c || !n_sites || max_sites < 0) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  FE_CK(cudaDeviceSynchronize());
+  for (auto& site : c->sites) {
+    for (auto& ev : site.pending) {
+      float ms = 0.f;
+      FE_CK(cudaEventElapsedTime(&ms, ev.first, ev.second));
+      site.total_ms += ms;
+      site.launches += 1;
+      site.spare.push_back(ev);
+    }
+    site.pending.clear();
+  }
+  *n_sites = (int)c->sites.size();
+  for (int i = 0; i < (int)c->sites.size() && i < max_sites; ++i) {
+    auto& site = c->sites[i];
+    if (names) {
+      std::strncpy(names + 32 * i, site.name.c_str(), 31);
+      names[32 * i + 31] = 0;
+    }
+    if (launches) launches[i] = site.launches;
+    if (total_ms) total_ms[i] = site.total_ms;
+    site.launches = 0;
+    site.total_ms = 0.0;
+  }
+  return FE_OK;
+}
+
+int fe_kernels_per_batch(fe_ctx* c) { return c ? c->launches_last : 0; }
+
 int fe_destroy(fe_ctx* c) {
   if (!c) return FE_OK;
   {
     DeviceGuard g(c->device);
     cudaDeviceSynchronize();
     clear_graphs(c);
+    for (auto& site : c->sites) {
+      for (auto& ev : site.pending) {
+        cudaEventDestroy(ev.first);
+        cudaEventDestroy(ev.second);
+      }
+      for (auto& ev : site.spare) {
+        cudaEventDestroy(ev.first);
+        cudaEventDestroy(ev.second);
+      }
+    }
     free_list(c->owned_ws);
     free_list(c->owned_w);
     if (c->host_status) cudaFreeHost(c->host_status);
