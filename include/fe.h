@@ -186,6 +186,38 @@ int fe_profile(fe_ctx* ctx, int enable);
 int fe_profile_read(fe_ctx* ctx, int max_sites, char* names, int* launches, double* total_ms, int* n_sites);
 int fe_kernels_per_batch(fe_ctx* ctx);
 
+/*
+ * Distinct-element layout without any device allocation.  The paper has no
+ * counterpart: this entry point exists for callers that are not allowed to
+ * allocate GPU memory -- for example a serving runtime whose memory pool owns
+ * the device and forbids cudaMalloc after start-up, or code that must not
+ * trigger the implicit synchronisation an allocation can cause.
+ *
+ * It computes what the first stage of fe_evaluate computes, with no fe_ctx:
+ *   U_out    [B]        int32, device: number of distinct pool rows of request b
+ *                       (0 for a request with an index outside [0, M))
+ *   slot_out [B, K, L]  int32, device: rank of cand_idx[b,k,j] among request b's
+ *                       distinct rows in ascending order (-1 for such a request)
+ * from cand_idx [B, K, L] int32 on the device.  The work is enqueued on
+ * `stream` and the call returns without waiting.
+ *
+ * Scratch (offsets, flags, distinct lists, a status word and a counter) lives
+ * in a fixed file-scope device array of 4.5 MiB that every GPU loading
+ * the library holds until the process exits.  Limits: B <= 65536,
+ * M <= 262144 and B * min(M, K*L) <= 1048576; larger batches are rejected with
+ * FE_ERR_UNSUPPORTED before anything is enqueued.  The call allocates nothing:
+ * no cudaMalloc, no cudaFree, no allocating library routine.
+ *
+ * The first call on a device looks up the array's device address and sets a
+ * kernel attribute on that device; make that first call before any stream
+ * capture.  All calls on a device share the one array and each call clears
+ * the part that must start at zero, so calls whose work overlaps on the GPU
+ * (different streams, no ordering between them) race and corrupt each other.
+ * Returns FE_OK, FE_ERR_INVALID_ARG, FE_ERR_UNSUPPORTED or FE_ERR_CUDA.
+ */
+int fe_distinct_layout_noalloc(const int32_t* cand_idx, int B, int M, int K, int L,
+                               int32_t* U_out, int32_t* slot_out, void* stream);
+
 /* Release every device resource owned by ctx (waits for its work first). */
 int fe_destroy(fe_ctx* ctx);
 

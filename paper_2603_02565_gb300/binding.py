@@ -29,7 +29,8 @@ FE_IO_F32 = 1
 
 EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evaluate_async", "fe_last_status",
            "fe_evaluate_host", "fe_debug_layout", "fe_debug_fetch", "fe_profile", "fe_profile_read",
-           "fe_kernels_per_batch", "fe_destroy", "fe_strerror", "fe_last_error_message"]
+           "fe_kernels_per_batch", "fe_distinct_layout_noalloc", "fe_destroy", "fe_strerror",
+           "fe_last_error_message"]
 
 
 class FeConfig(ctypes.Structure):
@@ -78,6 +79,8 @@ def load_library(path: str = LIB_PATH):
     L.fe_profile_read.restype = i32
     L.fe_kernels_per_batch.argtypes = [vp]
     L.fe_kernels_per_batch.restype = i32
+    L.fe_distinct_layout_noalloc.argtypes = [vp, i32, i32, i32, i32, vp, vp, vp]
+    L.fe_distinct_layout_noalloc.restype = i32
     L.fe_destroy.argtypes = [vp]
     L.fe_destroy.restype = i32
     L.fe_strerror.argtypes = [i32]
