@@ -55,7 +55,16 @@ struct Planes {
   bf16* l = nullptr;
   int ld = 0;
   int rows = 0;
-  CUtensorMap th{}, tl{};
+  CUtensorMap th{}, tl{};  // operand loads: 64 x 128 boxes, 128-byte swizzle
+  CUtensorMap sh{}, sl{};  // epilogue stores: 32 x 32 boxes, 64-byte swizzle
+};
+
+// fp32 rows (the residual streams), with the epilogue's store descriptor.
+struct F32Rows {
+  float* p = nullptr;
+  int ld = 0;
+  int rows = 0;
+  CUtensorMap sx{};  // 32 x 32 boxes, 128-byte swizzle
 };
 
 int alloc_planes(Planes& p, int rows, int ld, bool two, std::vector<void*>& owned) {
@@ -73,19 +82,19 @@ int alloc_planes(Planes& p, int rows, int ld, bool two, std::vector<void*>& owne
   return FE_OK;
 }
 
-int encode_map(CUtensorMap* m, const bf16* base, int cols, int rows, int box_rows) {
+int encode_map_t(CUtensorMap* m, CUtensorMapDataType dt, size_t esz, const void* base, int cols, int rows,
+                 int box_cols, int box_rows, CUtensorMapSwizzle sw) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) {
     g_msg = "cuTensorMapEncodeTiled is unavailable";
     return FE_ERR_CUDA;
   }
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)cols * sizeof(bf16)};
-  cuuint32_t box[2] = {64u, (cuuint32_t)box_rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * esz};
+  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   cuuint32_t es[2] = {1u, 1u};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<bf16*>(base), dims, strides, box, es,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, sw,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     g_msg = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
     return FE_ERR_CUDA;
@@ -93,11 +102,37 @@ int encode_map(CUtensorMap* m, const bf16* base, int cols, int rows, int box_row
   return FE_OK;
 }
 
+// Operand tiles: 64 bf16 (128 B) x box_rows, 128-byte swizzle.
+int encode_map(CUtensorMap* m, const bf16* base, int cols, int rows, int box_rows) {
+  return encode_map_t(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, cols, rows, 64, box_rows,
+                      CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
 // Descriptors of an activation (A operand): 128-row boxes on both planes.
 int map_act(Planes& p) {
   int rc = encode_map(&p.th, p.h, p.ld, p.rows, 128);
   if (rc == FE_OK) rc = encode_map(&p.tl, p.l, p.ld, p.rows, 128);
   return rc;
+}
+
+// Descriptors of a GEMM output written by the epilogue.
+int map_out(Planes& p) {
+  int rc = encode_map_t(&p.sh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.h, p.ld, p.rows, 32, 32,
+                        CU_TENSOR_MAP_SWIZZLE_64B);
+  if (rc == FE_OK)
+    rc = encode_map_t(&p.sl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.l, p.ld, p.rows, 32, 32,
+                      CU_TENSOR_MAP_SWIZZLE_64B);
+  return rc;
+}
+
+int alloc_f32(F32Rows& f, int rows, int ld, std::vector<void*>& owned) {
+  f.rows = rows < 128 ? 128 : rows;
+  f.ld = ld;
+  const size_t bytes = (size_t)f.rows * ld * sizeof(float);
+  if (cudaMalloc(&f.p, bytes) != cudaSuccess) return FE_ERR_OOM;
+  owned.push_back(f.p);
+  FE_CK(cudaMemset(f.p, 0, bytes));
+  return encode_map_t(&f.sx, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, f.p, ld, f.rows, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 // A weight matrix W[K, N] stored transposed as B operand [N, K_pad] plus its GEMM tiling.
@@ -157,7 +192,7 @@ struct fe_ctx {
   int *status = nullptr, *U = nullptr, *off = nullptr, *bad = nullptr, *slot = nullptr, *list = nullptr;
   unsigned* ticket = nullptr;
   Planes X, KV, xln, q, a, mid, kvI, o, cln, mids, z, qkv, ax, lncp;
-  float *h = nullptr, *c = nullptr, *cp = nullptr;
+  F32Rows h, c, cp;
   void* in_ctx = nullptr;
   void* in_pool = nullptr;
   int32_t* in_idx = nullptr;
@@ -319,7 +354,7 @@ void clear_graphs(fe_ctx* c) {
 }
 
 int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W, int rows, const int* rows_dev,
-         fe::GemmParams p, cudaStream_t s) {
+         fe::GemmParams p, const Planes* out, const F32Rows* xout, cudaStream_t s) {
   if (rows <= 0) return FE_OK;
   Prof pf(c, site, s);
   p.rows = rows;
@@ -328,10 +363,12 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   p.BN = (epi == fe::EPI_STORE) ? W.BN : W.N;
   p.K_pad = W.K_pad;
   p.nb = c->nb;
-  p.stages = (epi == fe::EPI_STORE) ? W.stages : fe::gemm_max_stages(p.BN, c->nb, W.K_pad);
+  p.stages = 0;  // chosen by gemm_launch
+  p.nacc = 0;
   p.status = c->status;
   p.eps = c->cfg.ln_eps;
-  FE_CK(fe::gemm_launch(epi, &A.th, &A.tl, &W.p.th, &W.p.tl, p, s));
+  FE_CK(fe::gemm_launch(epi, &A.th, &A.tl, &W.p.th, &W.p.tl, out ? &out->sh : nullptr, out ? &out->sl : nullptr,
+                        xout ? &xout->sx : nullptr, p, s));
   return FE_OK;
 }
 
@@ -371,23 +408,17 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   }
   {
     fe::GemmParams p{};
-    p.out_h = c->KV.h;
-    p.out_l = c->KV.l;
-    p.ldo = c->KV.ld;
-    FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, &c->KV, nullptr, s));
   }
   // (a2) distinct elements: gather + LN, then the cross-attention stack
   {
     Prof pf(c, "gather_ln", s);
-    FE_CK(fe::gather_ln_launch(io.pool, io_f32, B, M, d, cap, c->off, c->list, R, c->cfg.ln_eps, c->h, d, c->xln.h,
+    FE_CK(fe::gather_ln_launch(io.pool, io_f32, B, M, d, cap, c->off, c->list, R, c->cfg.ln_eps, c->h.p, d, c->xln.h,
                              c->xln.l, c->xln.ld, s));
   }
   for (int l = 0; l < Ly; ++l) {
     fe::GemmParams p{};
-    p.out_h = c->q.h;
-    p.out_l = c->q.l;
-    p.ldo = c->q.ld;
-    FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, s));
+    FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
 
     fe::AttnParams ap{};
     ap.q_h = c->q.h;
@@ -412,41 +443,25 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     }
 
     fe::GemmParams po{};
-    po.resid = c->h;
+    po.resid = c->h.p;
     po.ldr = d;
-    po.x_out = c->h;
-    po.ldx = d;
-    po.ln_h = c->xln.h;
-    po.ln_l = c->xln.l;
-    po.ldln = c->xln.ld;
-    FE_RC(gemm(c, "gemm_item_o_ln", fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, s));
+    FE_RC(gemm(c, "gemm_item_o_ln", fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, &c->xln, &c->h, s));
 
     fe::GemmParams p1{};
     p1.bias = lw(c, l, T_B1);
     p1.relu = 1;
-    p1.out_h = c->mid.h;
-    p1.out_l = c->mid.l;
-    p1.ldo = c->mid.ld;
-    FE_RC(gemm(c, "gemm_item_ffn1", fe::EPI_STORE, c->xln, c->w1[l], R, sumU, p1, s));
+    FE_RC(gemm(c, "gemm_item_ffn1", fe::EPI_STORE, c->xln, c->w1[l], R, sumU, p1, &c->mid, nullptr, s));
 
     fe::GemmParams p2{};
     p2.bias = lw(c, l, T_B2);
-    p2.resid = c->h;
+    p2.resid = c->h.p;
     p2.ldr = d;
-    p2.x_out = c->h;
-    p2.ldx = d;
-    p2.ln_h = c->xln.h;
-    p2.ln_l = c->xln.l;
-    p2.ldln = c->xln.ld;
-    FE_RC(gemm(c, "gemm_item_ffn2_ln", fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, s));
+    FE_RC(gemm(c, "gemm_item_ffn2_ln", fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, &c->xln, &c->h, s));
   }
   // element projections of SeqEnc: H WKs | H WVs
   {
     fe::GemmParams p{};
-    p.out_h = c->kvI.h;
-    p.out_l = c->kvI.l;
-    p.ldo = c->kvI.ld;
-    FE_RC(gemm(c, "gemm_item_seq_kv", fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, s));
+    FE_RC(gemm(c, "gemm_item_seq_kv", fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, &c->kvI, nullptr, s));
   }
   // (a3, a4) index-based assembly + [CLS] attention, then c = cls + o WOs, FFN
   {
@@ -471,50 +486,32 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     cp.o_l = c->o.l;
     cp.ldo = c->o.ld;
     cp.scale = 1.0f / sqrtf((float)c->dh);
-    {
     Prof pf(c, "seq_cls_attn", s);
     FE_CK(fe::cls_attn_launch(cp, s));
-  }
   }
   {
     fe::GemmParams p{};
     p.resid = tw(c, T_CLS);
     p.ldr = 0;
-    p.x_out = c->c;
-    p.ldx = d;
-    p.ln_h = c->cln.h;
-    p.ln_l = c->cln.l;
-    p.ldln = c->cln.ld;
-    FE_RC(gemm(c, "gemm_seq_o_ln", fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_seq_o_ln", fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, &c->cln, &c->c, s));
   }
   {
     fe::GemmParams p{};
     p.bias = tw(c, T_B1S);
     p.relu = 1;
-    p.out_h = c->mids.h;
-    p.out_l = c->mids.l;
-    p.ldo = c->mids.ld;
-    FE_RC(gemm(c, "gemm_seq_ffn1", fe::EPI_STORE, c->cln, c->w1s, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_seq_ffn1", fe::EPI_STORE, c->cln, c->w1s, S, nullptr, p, &c->mids, nullptr, s));
   }
   {
     fe::GemmParams p{};
     p.bias = tw(c, T_B2S);
-    p.resid = c->c;
+    p.resid = c->c.p;
     p.ldr = d;
-    p.x_out = c->c;
-    p.ldx = d;
-    p.ln_h = c->z.h;
-    p.ln_l = c->z.l;
-    p.ldln = c->z.ld;
-    FE_RC(gemm(c, "gemm_seq_ffn2_ln", fe::EPI_RESID_LN, c->mids, c->w2s, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_seq_ffn2_ln", fe::EPI_RESID_LN, c->mids, c->w2s, S, nullptr, p, &c->z, &c->c, s));
   }
   // (a5) cross-sequence attention over the K sequence vectors of each request
   {
     fe::GemmParams p{};
-    p.out_h = c->qkv.h;
-    p.out_l = c->qkv.l;
-    p.ldo = c->qkv.ld;
-    FE_RC(gemm(c, "gemm_cross_qkv", fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_cross_qkv", fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, &c->qkv, nullptr, s));
     fe::AttnParams ap{};
     ap.q_h = c->qkv.h;
     ap.q_l = c->qkv.l;
@@ -537,14 +534,9 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
       FE_CK(fe::attn_launch(c->dh, c->H, B, K, ap, s));
     }
     fe::GemmParams po{};
-    po.resid = c->c;
+    po.resid = c->c.p;
     po.ldr = d;
-    po.x_out = c->cp;
-    po.ldx = d;
-    po.ln_h = c->lncp.h;
-    po.ln_l = c->lncp.l;
-    po.ldln = c->lncp.ld;
-    FE_RC(gemm(c, "gemm_cross_o_ln", fe::EPI_RESID_LN, c->ax, c->ox, S, nullptr, po, s));
+    FE_RC(gemm(c, "gemm_cross_o_ln", fe::EPI_RESID_LN, c->ax, c->ox, S, nullptr, po, &c->lncp, &c->cp, s));
   }
   // (a6) score head and selection
   {
@@ -553,7 +545,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.w2 = tw(c, T_W2H);
     p.b2 = tw(c, T_B2H);
     p.scores = io.scores;
-    FE_RC(gemm(c, "gemm_head", fe::EPI_HEAD, c->lncp, c->w1h, S, nullptr, p, s));
+    FE_RC(gemm(c, "gemm_head", fe::EPI_HEAD, c->lncp, c->w1h, S, nullptr, p, nullptr, nullptr, s));
   }
   {
     Prof pf(c, "select", s);
@@ -624,9 +616,9 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->bad, (size_t)B * sizeof(int)));
   FE_RC(dalloc((void**)&c->slot, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int)));
   FE_RC(dalloc((void**)&c->list, (size_t)R * sizeof(int)));
-  FE_RC(dalloc((void**)&c->h, (size_t)R * d * sizeof(float)));
-  FE_RC(dalloc((void**)&c->c, (size_t)S * d * sizeof(float)));
-  FE_RC(dalloc((void**)&c->cp, (size_t)S * d * sizeof(float)));
+  FE_RC(alloc_f32(c->h, R, d, c->owned_ws));
+  FE_RC(alloc_f32(c->c, S, d, c->owned_ws));
+  FE_RC(alloc_f32(c->cp, S, d, c->owned_ws));
   const size_t esz = c->cfg.io_dtype == FE_IO_F32 ? 4 : 2;
   FE_RC(dalloc(&c->in_ctx, (size_t)BC * d * esz));
   FE_RC(dalloc(&c->in_pool, (size_t)B * (s.M > 0 ? s.M : 1) * d * esz));
@@ -649,6 +641,8 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(alloc_planes(c->lncp, S, c->dpad, true, c->owned_ws));
   for (Planes* p : {&c->X, &c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp})
     FE_RC(map_act(*p));
+  for (Planes* p : {&c->KV, &c->q, &c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->qkv, &c->lncp})
+    FE_RC(map_out(*p));
   c->cap_shape = s;
   c->cap_rows = R;
   return FE_OK;
@@ -797,7 +791,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if (cudaMemcpy(c->w32, weights, n_floats * sizeof(float), cudaMemcpyHostToDevice) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "weight copy"));
   const int d = c->d, F = c->F, Ly = c->Ly;
-  if ((rc = make_weight(c, c->ctx_kv, 2 * Ly * d, d, 256)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->ctx_kv, 2 * Ly * d, d, 128)) != FE_OK) return fail(rc);
   for (int l = 0; l < Ly; ++l) {
     if ((rc = fill_weight(c->ctx_kv, lw(c, l, T_WK), d, d, 2 * l * d)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->ctx_kv, lw(c, l, T_WV), d, d, (2 * l + 1) * d)) != FE_OK) return fail(rc);
@@ -807,25 +801,25 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   c->w1.resize(Ly);
   c->w2.resize(Ly);
   for (int l = 0; l < Ly; ++l) {
-    if ((rc = make_weight(c, c->wq[l], d, d, 256)) != FE_OK) return fail(rc);
+    if ((rc = make_weight(c, c->wq[l], d, d, 128)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->wq[l], lw(c, l, T_WQ), d, d, 0)) != FE_OK) return fail(rc);
     if ((rc = make_weight(c, c->wo[l], d, d, 512)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->wo[l], lw(c, l, T_WO), d, d, 0)) != FE_OK) return fail(rc);
-    if ((rc = make_weight(c, c->w1[l], F, d, 256)) != FE_OK) return fail(rc);
+    if ((rc = make_weight(c, c->w1[l], F, d, 128)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->w1[l], lw(c, l, T_W1), d, F, 0)) != FE_OK) return fail(rc);
     if ((rc = make_weight(c, c->w2[l], d, F, 512)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->w2[l], lw(c, l, T_W2), F, d, 0)) != FE_OK) return fail(rc);
   }
-  if ((rc = make_weight(c, c->kvs, 2 * d, d, 256)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->kvs, 2 * d, d, 128)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->kvs, tw(c, T_WKS), d, d, 0)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->kvs, tw(c, T_WVS), d, d, d)) != FE_OK) return fail(rc);
   if ((rc = make_weight(c, c->os, d, d, 512)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->os, tw(c, T_WOS), d, d, 0)) != FE_OK) return fail(rc);
-  if ((rc = make_weight(c, c->w1s, F, d, 256)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->w1s, F, d, 128)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w1s, tw(c, T_W1S), d, F, 0)) != FE_OK) return fail(rc);
   if ((rc = make_weight(c, c->w2s, d, F, 512)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w2s, tw(c, T_W2S), F, d, 0)) != FE_OK) return fail(rc);
-  if ((rc = make_weight(c, c->qkvx, 3 * d, d, 256)) != FE_OK) return fail(rc);
+  if ((rc = make_weight(c, c->qkvx, 3 * d, d, 128)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->qkvx, tw(c, T_WQX), d, d, 0)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->qkvx, tw(c, T_WKX), d, d, d)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->qkvx, tw(c, T_WVX), d, d, 2 * d)) != FE_OK) return fail(rc);
@@ -965,11 +959,11 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
     rows = (size_t)sum;
     cols = d;
   } else if (n == "seq") {
-    f32 = c->c;
+    f32 = c->c.p;
     rows = (size_t)s.B * s.K;
     cols = d;
   } else if (n == "cross") {
-    f32 = c->cp;
+    f32 = c->cp.p;
     rows = (size_t)s.B * s.K;
     cols = d;
   } else {

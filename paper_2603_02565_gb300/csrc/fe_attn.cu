@@ -67,6 +67,8 @@ __global__ void __launch_bounds__(128) attn_kernel(const AttnParams p) {
   bf16* sKV = sQl + BQ * P;  // [buffer 2][plane 4: Kh Kl Vh Vl][BKV * P]
 
   const int b = blockIdx.z, head = blockIdx.y;
+  pdl_wait();
+  pdl_trigger();
   const int q_cnt = p.q_cnt_dev ? p.q_cnt_dev[b] : p.q_cnt_fixed;
   const int q_begin = blockIdx.x * BQ;
   if (q_begin >= q_cnt) return;
@@ -253,11 +255,8 @@ cudaError_t attn_prepare() {
 cudaError_t attn_launch(int dh, int n_heads, int n_segments, int max_q, const AttnParams& p, cudaStream_t s) {
   if (n_segments <= 0 || max_q <= 0 || p.kv_cnt <= 0) return cudaSuccess;
   dim3 grid((unsigned)((max_q + BQ - 1) / BQ), (unsigned)n_heads, (unsigned)n_segments);
-  if (dh == 32)
-    attn_kernel<32><<<grid, 128, attn_smem<32>(), s>>>(p);
-  else
-    attn_kernel<64><<<grid, 128, attn_smem<64>(), s>>>(p);
-  return cudaGetLastError();
+  if (dh == 32) return launch_k(attn_kernel<32>, grid, dim3(128), attn_smem<32>(), s, p);
+  return launch_k(attn_kernel<64>, grid, dim3(128), attn_smem<64>(), s, p);
 }
 
 }  // namespace fe

@@ -3,10 +3,15 @@
 // Every dense product of the model (context K/V projection and element
 // WQ / WO / FFN of Section 4.2, SeqEnc and cross-sequence projections of
 // Sections 4.3-4.4, the score head) is  act[rows, K] x W[K, N]  with a small
-// K (d or F).  One CTA computes a 128-row x BN-column tile:
-//   warp 0 lane 0  : TMA producer (A hi/lo tiles + weight tiles per 64-wide k block)
-//   warp 1 lane 0  : tcgen05.mma issuer, fp32 accumulator in TMEM
-//   warps 0-3      : epilogue, thread t owns tile row t (TMEM lane t)
+// K (d or F).  The kernel is persistent and warp-specialised; each CTA walks
+// 128-row x BN-column tiles (column tile fastest, so concurrently running CTAs
+// share activation rows in L2):
+//   warp 0 lane 0  : TMA producer, a ring of shared-memory stages that runs
+//                    ahead across tile boundaries
+//   warp 1 lane 0  : tcgen05.mma issuer into one of two TMEM accumulators
+//   warps 2-5      : epilogue of the previous tile while the next one is
+//                    multiplied; thread (warp % 4) * 32 + lane owns tile row
+//                    = TMEM lane (warp % 4) * 32 + lane
 // The activation is a split pair (hi + lo bf16); the product is
 // A_hi W_hi + A_lo W_hi (+ A_hi W_lo when the weights carry a lo plane).
 #include "fe_common.cuh"
@@ -20,10 +25,15 @@ constexpr int BK = 64;                               // one 128-byte swizzle row
 constexpr uint32_t kATile = BM * BK * 2;             // 16 KB per activation plane
 constexpr size_t kSmemPerSM = 233472;                // 228 KB
 constexpr size_t kSmemMaxBlock = 232448;             // 227 KB opt-in per block
-constexpr size_t kSmemExtra = 1024 + 256;            // alignment slack + barriers
+constexpr uint32_t kStageOut = 4096;                 // per epilogue warp: 32 rows x 128 B output staging
+constexpr size_t kSmemExtra = 1024 + 256 + 1024 + 4 * kStageOut;  // align + barriers + align + staging
+constexpr int kThreads = 192;
+constexpr int kMaxStages = 8;
 
-uint32_t tmem_cols_for(int BN) {
-  return BN <= 32 ? 32u : BN <= 64 ? 64u : BN <= 128 ? 128u : BN <= 256 ? 256u : 512u;
+int g_num_sms = 0;
+
+__host__ __device__ inline uint32_t pow2_cols(int n) {
+  return n <= 32 ? 32u : n <= 64 ? 64u : n <= 128 ? 128u : n <= 256 ? 256u : 512u;
 }
 }  // namespace
 
@@ -33,45 +43,57 @@ size_t gemm_smem_bytes(int BN, int nb, int stages) {
 }
 
 int gemm_max_stages(int BN, int nb, int K_pad) {
+  (void)K_pad;  // stages run ahead across tiles, so the ring is not capped by one tile's k blocks
   const size_t stage = 2 * (size_t)kATile + (size_t)nb * BN * BK * 2;
   int s = (int)((kSmemMaxBlock - kSmemExtra) / stage);
-  const int nk = K_pad / BK;
-  if (s > 4) s = 4;
-  if (s > nk) s = nk;
+  if (s > kMaxStages) s = kMaxStages;
   return s < 1 ? 1 : s;
 }
 
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
 template <int EPI>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tA_h, const __grid_constant__ CUtensorMap tA_l,
                 const __grid_constant__ CUtensorMap tB_h, const __grid_constant__ CUtensorMap tB_l,
-                const GemmParams p) {
+                const __grid_constant__ CUtensorMap tO_h, const __grid_constant__ CUtensorMap tO_l,
+                const __grid_constant__ CUtensorMap tO_x, const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_s = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
 
   const int BN = p.BN, nb = p.nb, S = p.stages;
+  const int nacc = p.nacc;
   const uint32_t b_bytes = (uint32_t)BN * BK * 2;
   const uint32_t stage_bytes = 2 * kATile + (uint32_t)nb * b_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
   uint64_t* empty = full + S;
-  uint64_t* done = empty + S;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* tfull = empty + S;  // [2] accumulator ready for the epilogue
+  uint64_t* tempty = tfull + 2; // [2] accumulator drained by the epilogue
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  // output staging, one 4 KB buffer per epilogue warp, 1024-byte aligned
+  uint8_t* stg_base = smem + (((size_t)S * stage_bytes + 256 + 1023) & ~(size_t)1023);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row0 = blockIdx.x * BM;
-  const int n0 = blockIdx.y * BN;
+  pdl_wait();
   int rows_valid = p.rows;
   if (p.rows_dev) rows_valid = min(*p.rows_dev, p.rows);
-  if (row0 >= rows_valid) return;  // whole CTA past the valid rows
+  const int nt = p.N / BN;
+  const int tiles = ((rows_valid + BM - 1) / BM) * nt;
+  if ((int)blockIdx.x >= tiles) return;  // nothing for this CTA
 
-  const uint32_t ncols = BN <= 32 ? 32u : BN <= 64 ? 64u : BN <= 128 ? 128u : BN <= 256 ? 256u : 512u;
+  const uint32_t ncols = pow2_cols(nacc * BN);
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(full + s, 1);
       mbar_init(empty + s, 1);
     }
-    mbar_init(done, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull + a, 1);
+      mbar_init(tempty + a, 4);  // one arrival per epilogue warp
+    }
     fence_mbar_init();
     prefetch_tmap(&tA_h);
     prefetch_tmap(&tA_l);
@@ -84,163 +106,213 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int nk = p.K_pad / BK;
+  pdl_trigger();
 
-  if (warp == 0 && lane == 0) {
-    // ---------------- TMA producer ----------------
-    for (int kb = 0; kb < nk; ++kb) {
-      const int s = kb % S;
-      if (kb >= S && !mbar_wait_bounded(empty + s, ((kb / S) & 1) ^ 1, p.status)) break;
-      uint8_t* st = smem + (size_t)s * stage_bytes;
-      mbar_arrive_expect_tx(full + s, stage_bytes);
-      tma_load_2d(st, &tA_h, kb * BK, row0, full + s);
-      tma_load_2d(st + kATile, &tA_l, kb * BK, row0, full + s);
-      for (int q = 0; q < nb; ++q) {
-        const CUtensorMap* tb = q ? &tB_l : &tB_h;
-        for (int h = 0; h < BN; h += 256)
-          tma_load_2d(st + 2 * kATile + q * b_bytes + (uint32_t)h * BK * 2, tb, kb * BK, n0 + h, full + s);
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      int it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        const int m0 = (t / nt) * BM, n0 = (t % nt) * BN;
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int s = it % S;
+          if (it >= S && !mbar_wait_bounded(empty + s, ((it / S) & 1) ^ 1, p.status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + (size_t)s * stage_bytes;
+          mbar_arrive_expect_tx(full + s, stage_bytes);
+          tma_load_2d(st, &tA_h, kb * BK, m0, full + s);
+          tma_load_2d(st + kATile, &tA_l, kb * BK, m0, full + s);
+          for (int q = 0; q < nb; ++q) {
+            const CUtensorMap* tb = q ? &tB_l : &tB_h;
+            for (int h = 0; h < BN; h += 256)
+              tma_load_2d(st + 2 * kATile + q * b_bytes + (uint32_t)h * BK * 2, tb, kb * BK, n0 + h, full + s);
+          }
+        }
       }
     }
-  } else if (warp == 1 && lane == 0) {
-    // ---------------- MMA issuer ----------------
-    const int nmma = BN > 256 ? 256 : BN;
-    const uint32_t idesc = umma_idesc_bf16(BM, nmma);
-    for (int kb = 0; kb < nk; ++kb) {
-      const int s = kb % S;
-      if (!mbar_wait_bounded(full + s, (kb / S) & 1, p.status)) break;
-      tc_fence_after();
-      const uint32_t st = smem_u32(smem + (size_t)s * stage_bytes);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const int nmma = BN > 256 ? 256 : BN;
+      const uint32_t idesc = umma_idesc_bf16(BM, nmma);
+      int it = 0, tl = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+        const int acc = tl % nacc, use = tl / nacc;
+        if (use > 0 && !mbar_wait_bounded(tempty + acc, (use - 1) & 1, p.status)) break;
+        tc_fence_after();
+        const uint32_t dst = tmem + (uint32_t)(acc * BN);
+        for (int kb = 0; kb < nk; ++kb, ++it) {
+          const int s = it % S;
+          if (!mbar_wait_bounded(full + s, (it / S) & 1, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(smem + (size_t)s * stage_bytes);
 #pragma unroll 1
-      for (int kk = 0; kk < BK / 16; ++kk) {
-        // (A_hi, W_hi), (A_lo, W_hi), (A_hi, W_lo)
-        for (int pr = 0; pr < 1 + nb; ++pr) {
-          const uint32_t a = st + (pr == 1 ? kATile : 0u) + (uint32_t)kk * 32;
-          const uint32_t b = st + 2 * kATile + (pr == 2 ? b_bytes : 0u) + (uint32_t)kk * 32;
-          const uint64_t ad = umma_desc_sw128(a);
-          for (int h = 0; h < BN; h += 256) {
-            const uint64_t bd = umma_desc_sw128(b + (uint32_t)h * BK * 2);
-            umma_bf16(tmem + (uint32_t)h, ad, bd, idesc, (kb | kk | pr) != 0 ? 1u : 0u);
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            // (A_hi, W_hi), (A_lo, W_hi), (A_hi, W_lo)
+            for (int pr = 0; pr < 1 + nb; ++pr) {
+              const uint32_t a = st + (pr == 1 ? kATile : 0u) + (uint32_t)kk * 32;
+              const uint32_t b = st + 2 * kATile + (pr == 2 ? b_bytes : 0u) + (uint32_t)kk * 32;
+              const uint64_t ad = umma_desc_sw128(a);
+              for (int h = 0; h < BN; h += 256) {
+                const uint64_t bd = umma_desc_sw128(b + (uint32_t)h * BK * 2);
+                umma_bf16(dst + (uint32_t)h, ad, bd, idesc, (kb | kk | pr) != 0 ? 1u : 0u);
+              }
+            }
           }
+          umma_commit(empty + s);  // frees this stage once its MMAs complete
         }
+        umma_commit(tfull + acc);  // accumulator complete (or abandoned after a timeout)
       }
-      umma_commit(empty + s);  // frees this stage once its MMAs complete
     }
-    umma_commit(done);
-  }
-  __syncwarp();
+  } else {
+    // ---------------- epilogue (warps 2..5) ----------------
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int r = q * 32 + lane;
+    int tl = 0;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tl) {
+      const int acc = tl % nacc, use = tl / nacc;
+      if (!mbar_wait_bounded(tfull + acc, use & 1, p.status)) break;
+      tc_fence_after();
+      const int m0 = (t / nt) * BM, n0 = (t % nt) * BN;
+      const int grow = m0 + r;
+      const bool valid = grow < rows_valid;
+      const uint32_t trow = tmem + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
 
-  // ---------------- epilogue ----------------
-  mbar_wait_bounded(done, 0, p.status);
-  tc_fence_after();
-  const int r = warp * 32 + lane;
-  const int grow = row0 + r;
-  const bool valid = grow < rows_valid;
-  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-
-  if (EPI == EPI_STORE) {
-    for (int c = 0; c < BN; c += 32) {
-      float v[32];
-      tmem_ld32(trow + (uint32_t)c, v);
-      const int col = n0 + c;
-      if (valid) {
-        uint32_t hi[16], lo[16];
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) {
-          float x0 = v[i], x1 = v[i + 1];
-          if (p.bias) {
-            x0 += p.bias[col + i];
-            x1 += p.bias[col + i + 1];
-          }
-          if (p.relu) {
-            x0 = fmaxf(x0, 0.f);
-            x1 = fmaxf(x1, 0.f);
-          }
-          split2(x0, x1, hi[i / 2], lo[i / 2]);
-        }
-        uint4* dh = reinterpret_cast<uint4*>(p.out_h + (size_t)grow * p.ldo + col);
-        uint4* dl = reinterpret_cast<uint4*>(p.out_l + (size_t)grow * p.ldo + col);
+      // 32 rows x 32 columns of this warp go out through its staging buffer as
+      // TMA tensor stores: bf16 planes with the 64-byte swizzle (2 KB each),
+      // fp32 rows with the 128-byte swizzle (4 KB); rows past the tensor
+      // extent are clipped by the TMA unit
+      uint8_t* stg = stg_base + (size_t)q * kStageOut;
+      const int srow = m0 + q * 32;
+      auto stage_split = [&](const uint32_t* hi, const uint32_t* lo, const CUtensorMap* mh,
+                             const CUtensorMap* ml, int col) {
+        if (lane == 0) bulk_wait_read0();
+        __syncwarp();
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          dh[j] = make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
-          dl[j] = make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
+          const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
+          *reinterpret_cast<uint4*>(stg + o) = make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
+          *reinterpret_cast<uint4*>(stg + 2048 + o) =
+              make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
         }
-      }
-    }
-  } else if (EPI == EPI_RESID_LN) {
-    // pass 1: x = resid + acc + bias, written out and kept in TMEM
-    float sum = 0.f;
-    const float* rrow = p.resid + (p.ldr ? (size_t)grow * p.ldr : (size_t)0);
-    for (int c = 0; c < BN; c += 32) {
-      float v[32];
-      tmem_ld32(trow + (uint32_t)c, v);
-      if (valid) {
-        const float4* rr = reinterpret_cast<const float4*>(rrow + c);
-        float4* xo = reinterpret_cast<float4*>(p.x_out + (size_t)grow * p.ldx + c);
+        fence_async_shared();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_2d(mh, stg, col, srow);
+          tma_store_2d(ml, stg + 2048, col, srow);
+          bulk_commit();
+        }
+      };
+
+      if (EPI == EPI_STORE) {
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
+          const int col = n0 + c;
+          uint32_t hi[16], lo[16];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float4 q = rr[j];
-          float4 x;
-          x.x = v[4 * j + 0] + q.x;
-          x.y = v[4 * j + 1] + q.y;
-          x.z = v[4 * j + 2] + q.z;
-          x.w = v[4 * j + 3] + q.w;
-          if (p.bias) {
-            x.x += p.bias[c + 4 * j + 0];
-            x.y += p.bias[c + 4 * j + 1];
-            x.z += p.bias[c + 4 * j + 2];
-            x.w += p.bias[c + 4 * j + 3];
+          for (int i = 0; i < 32; i += 2) {
+            float x0 = v[i], x1 = v[i + 1];
+            if (p.bias) {
+              x0 += p.bias[col + i];
+              x1 += p.bias[col + i + 1];
+            }
+            if (p.relu) {
+              x0 = fmaxf(x0, 0.f);
+              x1 = fmaxf(x1, 0.f);
+            }
+            split2(x0, x1, hi[i / 2], lo[i / 2]);
           }
-          v[4 * j + 0] = x.x;
-          v[4 * j + 1] = x.y;
-          v[4 * j + 2] = x.z;
-          v[4 * j + 3] = x.w;
-          sum += (x.x + x.y) + (x.z + x.w);
-          xo[j] = x;
+          stage_split(hi, lo, &tO_h, &tO_l, col);
         }
-      }
-      tmem_st32(trow + (uint32_t)c, v);
-    }
-    const float mean = sum / (float)BN;
-    // pass 2: biased variance about the mean
-    float var = 0.f;
-    for (int c = 0; c < BN; c += 32) {
-      float v[32];
-      tmem_ld32(trow + (uint32_t)c, v);
+      } else if (EPI == EPI_RESID_LN) {
+        // pass 1: x = resid + acc + bias, written out and kept in TMEM
+        float sum = 0.f;
+        const float* rrow = p.resid + (p.ldr ? (size_t)grow * p.ldr : (size_t)0);
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
+          if (valid) {
+            const float4* rr = reinterpret_cast<const float4*>(rrow + c);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float dv = v[i] - mean;
-        var = fmaf(dv, dv, var);
-      }
-    }
-    const float rstd = 1.0f / sqrtf(var / (float)BN + p.eps);
-    // pass 3: LN(x) as split planes
-    for (int c = 0; c < BN; c += 32) {
-      float v[32];
-      tmem_ld32(trow + (uint32_t)c, v);
-      if (valid) {
-        uint32_t hi[16], lo[16];
+            for (int j = 0; j < 8; ++j) {
+              const float4 qv = rr[j];
+              v[4 * j + 0] += qv.x;
+              v[4 * j + 1] += qv.y;
+              v[4 * j + 2] += qv.z;
+              v[4 * j + 3] += qv.w;
+            }
+          }
+          if (p.bias) {
 #pragma unroll
-        for (int i = 0; i < 32; i += 2) split2((v[i] - mean) * rstd, (v[i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
-        uint4* dh = reinterpret_cast<uint4*>(p.ln_h + (size_t)grow * p.ldln + c);
-        uint4* dl = reinterpret_cast<uint4*>(p.ln_l + (size_t)grow * p.ldln + c);
+            for (int i = 0; i < 32; ++i) v[i] += p.bias[c + i];
+          }
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          dh[j] = make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
-          dl[j] = make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
+          for (int i = 0; i < 32; i += 4) sum += (v[i] + v[i + 1]) + (v[i + 2] + v[i + 3]);
+          tmem_st32(trow + (uint32_t)c, v);
+          if (lane == 0) bulk_wait_read0();
+          __syncwarp();
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const uint32_t o = (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4);
+            *reinterpret_cast<float4*>(stg + o) = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+          }
+          fence_async_shared();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tO_x, stg, c, srow);
+            bulk_commit();
+          }
         }
-      }
-    }
-  } else {  // EPI_HEAD
-    float acc = 0.f;
-    for (int c = 0; c < BN; c += 32) {
-      float v[32];
-      tmem_ld32(trow + (uint32_t)c, v);
+        const float mean = sum / (float)BN;
+        // pass 2: biased variance about the mean
+        float var = 0.f;
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float x = fmaxf(v[i] + p.bias[c + i], 0.f);
-        acc = fmaf(x, p.w2[c + i], acc);
+          for (int i = 0; i < 32; ++i) {
+            const float dv = v[i] - mean;
+            var = fmaf(dv, dv, var);
+          }
+        }
+        const float rstd = 1.0f / sqrtf(var / (float)BN + p.eps);
+        // pass 3: LN(x) as split planes
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
+          uint32_t hi[16], lo[16];
+#pragma unroll
+          for (int i = 0; i < 32; i += 2)
+            split2((v[i] - mean) * rstd, (v[i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
+          stage_split(hi, lo, &tO_h, &tO_l, c);
+        }
+      } else {  // EPI_HEAD
+        float accv = 0.f;
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float x = fmaxf(v[i] + p.bias[c + i], 0.f);
+            accv = fmaf(x, p.w2[c + i], accv);
+          }
+        }
+        if (valid) p.scores[grow] = accv + p.b2[0];
       }
+      // every TMEM read of this accumulator has completed (tcgen05.wait::ld)
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty + acc);
     }
-    if (valid) p.scores[grow] = acc + p.b2[0];
+    if (lane == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
   }
 
   tc_fence_before();
@@ -248,29 +320,47 @@ __global__ void __launch_bounds__(128, 1)
   if (warp == 0) tmem_dealloc(tmem, ncols);
 }
 
-static size_t gemm_launch_smem(int BN, int nb, int stages) {
-  size_t smem = gemm_smem_bytes(BN, nb, stages);
-  // Keep (CTAs resident per SM) x (TMEM columns per CTA) <= 512 so that no CTA
-  // waits in tcgen05.alloc for a co-resident CTA.
-  const size_t max_ctas = 512 / tmem_cols_for(BN);
+template <int EPI>
+static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* b_h,
+                            const CUtensorMap* b_l, const CUtensorMap* o_h, const CUtensorMap* o_l,
+                            const CUtensorMap* o_x, const GemmParams& p0, cudaStream_t s) {
+  GemmParams p = p0;
+  const int sms = g_num_sms > 0 ? g_num_sms : 148;
+  const long long tiles = (long long)((p.rows + BM - 1) / BM) * (p.N / p.BN);
+  const size_t stage = 2 * (size_t)kATile + (size_t)p.nb * p.BN * BK * 2;
+  // At most two waves of tiles: two CTAs per SM, one accumulator each, so the
+  // co-resident CTAs overlap each other's loads, MMAs and epilogues.
+  // Otherwise: one persistent CTA per SM with a double-buffered accumulator.
+  int per_sm = 1;
+  const int st2 = (int)((kSmemPerSM / 2 - 1024 - kSmemExtra) / stage);
+  if (tiles <= 2LL * sms && st2 >= 1 && 2 * pow2_cols(p.BN) <= 512) {
+    per_sm = 2;
+    p.nacc = 1;
+    p.stages = st2 < kMaxStages ? st2 : kMaxStages;
+  } else {
+    p.nacc = 2 * p.BN <= 512 ? 2 : 1;
+    p.stages = gemm_max_stages(p.BN, p.nb, p.K_pad);
+  }
+  size_t smem = gemm_smem_bytes(p.BN, p.nb, p.stages);
+  // (CTAs resident per SM) x (TMEM columns per CTA) <= 512: no CTA ever waits in
+  // tcgen05.alloc for a co-resident one
+  const size_t max_ctas = 512 / pow2_cols(p.nacc * p.BN);
   const size_t floor_bytes = kSmemPerSM / (max_ctas + 1) + 1;
   if (smem < floor_bytes) smem = floor_bytes;
   if (smem > kSmemMaxBlock) smem = kSmemMaxBlock;
-  return smem;
-}
-
-template <int EPI>
-static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* b_h,
-                            const CUtensorMap* b_l, const GemmParams& p, cudaStream_t s) {
-  const size_t smem = gemm_launch_smem(p.BN, p.nb, p.stages);
-  dim3 grid((unsigned)((p.rows + BM - 1) / BM), (unsigned)(p.N / p.BN));
-  gemm_kernel<EPI><<<grid, 128, smem, s>>>(*a_h, *a_l, *b_h, *b_l, p);
-  return cudaGetLastError();
+  long long grid = (long long)sms * per_sm;
+  if (grid > tiles) grid = tiles;
+  return launch_k(gemm_kernel<EPI>, dim3((unsigned)grid), dim3(kThreads), smem, s, *a_h, *a_l, *b_h, *b_l,
+                  o_h ? *o_h : *a_h, o_l ? *o_l : *a_l, o_x ? *o_x : *a_h, p);
 }
 
 cudaError_t gemm_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(gemm_kernel<EPI_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kSmemMaxBlock);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(gemm_kernel<EPI_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kSmemMaxBlock);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(gemm_kernel<EPI_RESID_LN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)kSmemMaxBlock);
@@ -281,12 +371,13 @@ cudaError_t gemm_prepare() {
 }
 
 cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* b_h,
-                        const CUtensorMap* b_l, const GemmParams& p, cudaStream_t s) {
+                        const CUtensorMap* b_l, const CUtensorMap* o_h, const CUtensorMap* o_l,
+                        const CUtensorMap* o_x, const GemmParams& p, cudaStream_t s) {
   if (p.rows <= 0) return cudaSuccess;
   switch (epi) {
-    case EPI_STORE: return launch_t<EPI_STORE>(a_h, a_l, b_h, b_l, p, s);
-    case EPI_RESID_LN: return launch_t<EPI_RESID_LN>(a_h, a_l, b_h, b_l, p, s);
-    default: return launch_t<EPI_HEAD>(a_h, a_l, b_h, b_l, p, s);
+    case EPI_STORE: return launch_t<EPI_STORE>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
+    case EPI_RESID_LN: return launch_t<EPI_RESID_LN>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
+    default: return launch_t<EPI_HEAD>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
   }
 }
 

@@ -18,11 +18,32 @@ enum : int {
   ST_TIMEOUT = 4,  // a bounded wait gave up
 };
 
+// Whether batch kernels are launched with programmatic stream serialisation
+// (overlapping each kernel's launch and prologue with its predecessor's tail).
+// On unless the environment sets FE_NO_PDL=1.
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                            Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // ---------------------------------------------------------------------------
 // tcgen05 GEMM:  D[r, n] = sum over planes  A_p[r, :] . B_q[n, :]
 // A: activation as two bf16 planes (hi, lo), row-major [rows, K_pad]
 // B: weights transposed, [N, K_pad], one or two bf16 planes (hi[, lo])
-// One CTA computes a 128 x BN tile; BN <= 512 (two N=256 MMAs above 256).
+// Persistent CTAs walk 128 x BN tiles; BN <= 512 (two N=256 MMAs above 256).
 // ---------------------------------------------------------------------------
 enum GemmEpilogue : int {
   EPI_STORE = 0,    // out = [ReLU](acc + bias) as split planes
@@ -37,21 +58,13 @@ struct GemmParams {
   int BN;               // columns per CTA (multiple of 32, <= 512)
   int K_pad;            // reduction length, multiple of 64
   int nb;               // weight planes: 1 (exact bf16) or 2 (hi + lo)
-  int stages;           // shared-memory pipeline depth
+  int stages;           // shared-memory pipeline depth (chosen by gemm_launch)
+  int nacc;             // TMEM accumulators, 1 or 2 (chosen by gemm_launch)
   const float* bias;    // [N] or null
   int relu;
-  // EPI_STORE
-  bf16* out_h;
-  bf16* out_l;
-  int ldo;
-  // EPI_RESID_LN
+  // EPI_RESID_LN (outputs through the o_x / o_h / o_l tensor maps)
   const float* resid;   // residual rows (ldr == 0: one row broadcast to every row)
   int ldr;
-  float* x_out;
-  int ldx;
-  bf16* ln_h;
-  bf16* ln_l;
-  int ldln;
   float eps;
   // EPI_HEAD
   const float* w2;
@@ -64,8 +77,12 @@ struct GemmParams {
 cudaError_t gemm_prepare();
 size_t gemm_smem_bytes(int BN, int nb, int stages);
 int gemm_max_stages(int BN, int nb, int K_pad);
+// o_h / o_l: output bf16 planes (EPI_STORE: the product, EPI_RESID_LN: LN(x)), tensor maps with
+// 32 x 32 boxes and the 64-byte swizzle; o_x: the fp32 x_out rows of EPI_RESID_LN, 32 x 32 boxes,
+// 128-byte swizzle.  Unused maps may be null.
 cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* b_h,
-                        const CUtensorMap* b_l, const GemmParams& p, cudaStream_t s);
+                        const CUtensorMap* b_l, const CUtensorMap* o_h, const CUtensorMap* o_l,
+                        const CUtensorMap* o_x, const GemmParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Flash-style multi-head attention over request segments (split-bf16 operands)

@@ -3,6 +3,7 @@
 // index-based assembly with the [CLS]-pooled SeqEnc attention (Section 4.3),
 // the argmax of Eq. 1, and init-time weight preparation.
 #include <climits>
+#include <cstdlib>
 
 #include "fe_common.cuh"
 #include "fe_kernels.h"
@@ -157,6 +158,8 @@ __global__ void __launch_bounds__(256) compact_kernel(const int32_t* __restrict_
   const int b = blockIdx.x, tid = threadIdx.x;
   const int n = K * L;
   const int32_t* cb = cand + (size_t)b * n;
+  pdl_wait();
+  pdl_trigger();
 
   for (int w = tid; w < W; w += 256) bits[w] = 0u;
   if (tid == 0) s_bad = 0;
@@ -234,8 +237,8 @@ cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int 
                            int* bad, int* slot_local, int* list, int* status, unsigned* ticket,
                            cudaStream_t s) {
   const size_t smem = (size_t)2 * ((M + 31) / 32) * sizeof(uint32_t);
-  compact_kernel<<<B, 256, smem, s>>>(cand, B, M, K, L, cap, U, off, bad, slot_local, list, status, ticket);
-  return cudaGetLastError();
+  return launch_k(compact_kernel, dim3(B), dim3(256), smem, s, cand, B, M, K, L, cap, U, off, bad, slot_local, list,
+                  status, ticket);
 }
 
 // ---------------------------------------------------------------------------
@@ -247,6 +250,8 @@ __global__ void __launch_bounds__(256) ctx_ln_kernel(const T* __restrict__ x, in
   constexpr int d = DPL * 32;
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  pdl_wait();
+  pdl_trigger();
   if (r >= rows) return;
   float v[DPL];
   load_vec<DPL>(x + (size_t)r * d + lane * DPL, v);
@@ -265,6 +270,8 @@ __global__ void __launch_bounds__(256) gather_ln_kernel(const T* __restrict__ po
   constexpr int d = DPL * 32;
   const int lane = threadIdx.x & 31;
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  pdl_wait();
+  pdl_trigger();
   if (r >= max_rows || r >= off[B]) return;
   int lo = 0, hi = B - 1;  // largest b with off[b] <= r
   while (lo < hi) {
@@ -289,11 +296,11 @@ template <typename T>
 static cudaError_t ctx_ln_t(const T* x, int rows, int d, float eps, bf16* oh, bf16* ol, int ldo, cudaStream_t s) {
   const unsigned g = (unsigned)((rows + 7) / 8);
   switch (d) {
-    case 32: ctx_ln_kernel<1, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
-    case 64: ctx_ln_kernel<2, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
-    case 128: ctx_ln_kernel<4, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
-    case 256: ctx_ln_kernel<8, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
-    case 512: ctx_ln_kernel<16, T><<<g, 256, 0, s>>>(x, rows, eps, oh, ol, ldo); break;
+    case 32: return launch_k(ctx_ln_kernel<1, T>, dim3(g), dim3(256), 0, s, x, rows, eps, oh, ol, ldo);
+    case 64: return launch_k(ctx_ln_kernel<2, T>, dim3(g), dim3(256), 0, s, x, rows, eps, oh, ol, ldo);
+    case 128: return launch_k(ctx_ln_kernel<4, T>, dim3(g), dim3(256), 0, s, x, rows, eps, oh, ol, ldo);
+    case 256: return launch_k(ctx_ln_kernel<8, T>, dim3(g), dim3(256), 0, s, x, rows, eps, oh, ol, ldo);
+    case 512: return launch_k(ctx_ln_kernel<16, T>, dim3(g), dim3(256), 0, s, x, rows, eps, oh, ol, ldo);
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
@@ -311,8 +318,9 @@ static cudaError_t gather_t(const T* pool, int B, int M, int d, int cap, const i
                             int max_rows, float eps, float* h, int ldh, bf16* lh, bf16* ll, int ldln,
                             cudaStream_t s) {
   const unsigned g = (unsigned)((max_rows + 7) / 8);
-#define FE_GATHER(DPL) \
-  gather_ln_kernel<DPL, T><<<g, 256, 0, s>>>(pool, B, M, cap, off, list, max_rows, eps, h, ldh, lh, ll, ldln)
+#define FE_GATHER(DPL)                                                                                      \
+  return launch_k(gather_ln_kernel<DPL, T>, dim3(g), dim3(256), 0, s, pool, B, M, cap, off, list, max_rows, eps, h, \
+                  ldh, lh, ll, ldln)
   switch (d) {
     case 32: FE_GATHER(1); break;
     case 64: FE_GATHER(2); break;
@@ -346,6 +354,8 @@ template <int DPL>
 __global__ void __launch_bounds__(256) cls_attn_kernel(const ClsParams p) {
   const int lane = threadIdx.x & 31;
   const int seq = blockIdx.x * 8 + (threadIdx.x >> 5);
+  pdl_wait();
+  pdl_trigger();
   if (seq >= p.B * p.K) return;
   const int b = seq / p.K;
   const int d = p.d;
@@ -397,11 +407,11 @@ cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const unsigned g = (unsigned)((n + 7) / 8);
   switch (p.d) {
-    case 32: cls_attn_kernel<1><<<g, 256, 0, s>>>(p); break;
-    case 64: cls_attn_kernel<2><<<g, 256, 0, s>>>(p); break;
-    case 128: cls_attn_kernel<4><<<g, 256, 0, s>>>(p); break;
-    case 256: cls_attn_kernel<8><<<g, 256, 0, s>>>(p); break;
-    case 512: cls_attn_kernel<16><<<g, 256, 0, s>>>(p); break;
+    case 32: return launch_k(cls_attn_kernel<1>, dim3(g), dim3(256), 0, s, p);
+    case 64: return launch_k(cls_attn_kernel<2>, dim3(g), dim3(256), 0, s, p);
+    case 128: return launch_k(cls_attn_kernel<4>, dim3(g), dim3(256), 0, s, p);
+    case 256: return launch_k(cls_attn_kernel<8>, dim3(g), dim3(256), 0, s, p);
+    case 512: return launch_k(cls_attn_kernel<16>, dim3(g), dim3(256), 0, s, p);
     default: return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
@@ -414,6 +424,8 @@ __global__ void __launch_bounds__(256) select_kernel(float* scores, int B, int K
                                                      int* status) {
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
+  pdl_wait();
+  pdl_trigger();
   if (b >= B) return;
   float* sb = scores + (size_t)b * K;
   if (bad[b]) {
@@ -452,8 +464,7 @@ __global__ void __launch_bounds__(256) select_kernel(float* scores, int B, int K
 cudaError_t select_launch(float* scores, int B, int K, const int* bad, int32_t* best, int* status,
                           cudaStream_t s) {
   if (B <= 0) return cudaSuccess;
-  select_kernel<<<(unsigned)((B + 7) / 8), 256, 0, s>>>(scores, B, K, bad, best, status);
-  return cudaGetLastError();
+  return launch_k(select_kernel, dim3((unsigned)((B + 7) / 8)), dim3(256), 0, s, scores, B, K, bad, best, status);
 }
 
 // ---------------------------------------------------------------------------
@@ -493,6 +504,14 @@ cudaError_t small_matmul_launch(const float* X, int R, int Kd, const float* W, i
   if (R <= 0) return cudaSuccess;
   small_matmul_kernel<<<128, 256, 0, s>>>(X, R, Kd, W, N, out);
   return cudaGetLastError();
+}
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("FE_NO_PDL");
+    return !(v && v[0] == '1');
+  }();
+  return on;
 }
 
 cudaError_t misc_prepare() {
