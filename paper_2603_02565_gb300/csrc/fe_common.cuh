@@ -27,13 +27,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(bf16 a, bf16 b) {
   return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
 }
 
-// two floats -> packed hi pair and packed lo pair
+// two floats -> packed hi pair and packed lo pair (x0 in the low half);
+// the same round-to-nearest-even values as split_bf16, two lanes per cvt
 __device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
-  bf16 h0, l0, h1, l1;
-  split_bf16(x0, h0, l0);
-  split_bf16(x1, h1, l1);
-  hi = pack_bf16x2(h0, h1);
-  lo = pack_bf16x2(l0, l1);
+  __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+  const uint32_t hu = *reinterpret_cast<uint32_t*>(&h);
+  __nv_bfloat162 l = __floats2bfloat162_rn(x0 - __uint_as_float(hu << 16), x1 - __uint_as_float(hu & 0xFFFF0000u));
+  hi = hu;
+  lo = *reinterpret_cast<uint32_t*>(&l);
 }
 
 __device__ __forceinline__ float bf16lo_f(uint32_t v) { return __uint_as_float(v << 16); }

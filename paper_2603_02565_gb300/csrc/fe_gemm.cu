@@ -9,9 +9,10 @@
 //   warp 0 lane 0  : TMA producer, a ring of shared-memory stages that runs
 //                    ahead across tile boundaries
 //   warp 1 lane 0  : tcgen05.mma issuer into one of two TMEM accumulators
-//   warps 2-5      : epilogue of the previous tile while the next one is
-//                    multiplied; thread (warp % 4) * 32 + lane owns tile row
-//                    = TMEM lane (warp % 4) * 32 + lane
+//   warps 2-9      : epilogue of the previous tile while the next one is
+//                    multiplied; warps w and w+4 share TMEM lane quadrant
+//                    w % 4 (tile rows (w % 4) * 32 + lane) and take
+//                    alternate 32-column chunks
 // The activation is a split pair (hi + lo bf16); the product is
 // A_hi W_hi + A_lo W_hi (+ A_hi W_lo when the weights carry a lo plane).
 #include "fe_common.cuh"
@@ -25,9 +26,11 @@ constexpr int BK = 64;                               // one 128-byte swizzle row
 constexpr uint32_t kATile = BM * BK * 2;             // 16 KB per activation plane
 constexpr size_t kSmemPerSM = 233472;                // 228 KB
 constexpr size_t kSmemMaxBlock = 232448;             // 227 KB opt-in per block
-constexpr uint32_t kStageOut = 4096;                 // per epilogue warp: 32 rows x 128 B output staging
-constexpr size_t kSmemExtra = 1024 + 256 + 1024 + 4 * kStageOut;  // align + barriers + align + staging
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;                         // two per TMEM lane quadrant, alternating 32-column chunks
+constexpr uint32_t kStageOut = 4096;                 // one staging buffer: 32 rows x 128 B
+constexpr uint32_t kRedBytes = 4 * 2 * 128 * 4;      // row-reduction exchange: [parity][sum|var][half][128]
+constexpr size_t kSmemExtra = 1024 + 256 + 1024 + kEpiWarps * 2 * kStageOut + kRedBytes;
+constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kMaxStages = 8;
 
 int g_num_sms = 0;
@@ -73,8 +76,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tfull = empty + S;  // [2] accumulator ready for the epilogue
   uint64_t* tempty = tfull + 2; // [2] accumulator drained by the epilogue
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
-  // output staging, one 4 KB buffer per epilogue warp, 1024-byte aligned
+  // output staging: two 4 KB buffers per epilogue warp, 1024-byte aligned; then
+  // the row-reduction exchange of the two warps sharing a lane quadrant
   uint8_t* stg_base = smem + (((size_t)S * stage_bytes + 256 + 1023) & ~(size_t)1023);
+  float* red = reinterpret_cast<float*>(stg_base + (size_t)kEpiWarps * 2 * kStageOut);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   pdl_wait();
@@ -92,7 +97,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull + a, 1);
-      mbar_init(tempty + a, 4);  // one arrival per epilogue warp
+      mbar_init(tempty + a, kEpiWarps);  // one arrival per epilogue warp
     }
     fence_mbar_init();
     prefetch_tmap(&tA_h);
@@ -172,9 +177,48 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
-    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    // ---------------- epilogue (warps 2..9) ----------------
+    const int ew = warp - 2;     // 0..7
+    const int q = warp & 3;      // TMEM lane quadrant this warp may access
+    const int half = ew >> 2;    // which alternate 32-column chunks
     const int r = q * 32 + lane;
+    uint8_t* stg0 = stg_base + (size_t)ew * 2 * kStageOut;
+    int nstore = 0;              // bulk-store groups issued by this warp (selects the staging buffer)
+    // the two warps of a lane quadrant meet at named barrier 1 + q (64 threads)
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory"); };
+    // 32 rows x 32 columns of this warp leave through a staging buffer as TMA
+    // tensor stores: bf16 planes with the 64-byte swizzle (2 KB each), fp32
+    // rows with the 128-byte swizzle (4 KB); the TMA unit clips rows past the
+    // tensor extent.  Two buffers alternate so one store drains while the
+    // next chunk is written.
+    auto next_stage = [&]() -> uint8_t* {
+      uint8_t* b = stg0 + (size_t)(nstore & 1) * kStageOut;
+      if (lane == 0 && nstore >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+      __syncwarp();
+      return b;
+    };
+    auto issue = [&](const CUtensorMap* m0p, const void* s0, const CUtensorMap* m1p, const void* s1, int col,
+                     int row) {
+      fence_async_shared();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(m0p, s0, col, row);
+        if (m1p) tma_store_2d(m1p, s1, col, row);
+        bulk_commit();
+      }
+      ++nstore;
+    };
+    auto stage_split = [&](const uint32_t* hi, const uint32_t* lo, int col, int row) {
+      uint8_t* b = next_stage();
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
+        *reinterpret_cast<uint4*>(b + o) = make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
+        *reinterpret_cast<uint4*>(b + 2048 + o) = make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
+      }
+      issue(&tO_h, b, &tO_l, b + 2048, col, row);
+    };
+
     int tl = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tl) {
       const int acc = tl % nacc, use = tl / nacc;
@@ -183,36 +227,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int m0 = (t / nt) * BM, n0 = (t % nt) * BN;
       const int grow = m0 + r;
       const bool valid = grow < rows_valid;
-      const uint32_t trow = tmem + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
-
-      // 32 rows x 32 columns of this warp go out through its staging buffer as
-      // TMA tensor stores: bf16 planes with the 64-byte swizzle (2 KB each),
-      // fp32 rows with the 128-byte swizzle (4 KB); rows past the tensor
-      // extent are clipped by the TMA unit
-      uint8_t* stg = stg_base + (size_t)q * kStageOut;
       const int srow = m0 + q * 32;
-      auto stage_split = [&](const uint32_t* hi, const uint32_t* lo, const CUtensorMap* mh,
-                             const CUtensorMap* ml, int col) {
-        if (lane == 0) bulk_wait_read0();
-        __syncwarp();
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
-          *reinterpret_cast<uint4*>(stg + o) = make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
-          *reinterpret_cast<uint4*>(stg + 2048 + o) =
-              make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
-        }
-        fence_async_shared();
-        __syncwarp();
-        if (lane == 0) {
-          tma_store_2d(mh, stg, col, srow);
-          tma_store_2d(ml, stg + 2048, col, srow);
-          bulk_commit();
-        }
-      };
+      const uint32_t trow = tmem + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
+      float* red_sum = red + (size_t)(tl & 1) * 512;  // [half][128]
+      float* red_var = red_sum + 256;
 
       if (EPI == EPI_STORE) {
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 32 * half; c < BN; c += 64) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
           const int col = n0 + c;
@@ -230,13 +251,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             split2(x0, x1, hi[i / 2], lo[i / 2]);
           }
-          stage_split(hi, lo, &tO_h, &tO_l, col);
+          stage_split(hi, lo, col, srow);
         }
       } else if (EPI == EPI_RESID_LN) {
-        // pass 1: x = resid + acc + bias, written out and kept in TMEM
+        // pass 1: x = resid + acc + bias, stored out and kept in TMEM
         float sum = 0.f;
         const float* rrow = p.resid + (p.ldr ? (size_t)grow * p.ldr : (size_t)0);
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 32 * half; c < BN; c += 64) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
           if (valid) {
@@ -257,24 +278,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int i = 0; i < 32; i += 4) sum += (v[i] + v[i + 1]) + (v[i + 2] + v[i + 3]);
           tmem_st32(trow + (uint32_t)c, v);
-          if (lane == 0) bulk_wait_read0();
-          __syncwarp();
+          uint8_t* b = next_stage();
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const uint32_t o = (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4);
-            *reinterpret_cast<float4*>(stg + o) = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+            *reinterpret_cast<float4*>(b + o) = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
           }
-          fence_async_shared();
-          __syncwarp();
-          if (lane == 0) {
-            tma_store_2d(&tO_x, stg, c, srow);
-            bulk_commit();
-          }
+          issue(&tO_x, b, nullptr, nullptr, c, srow);
         }
-        const float mean = sum / (float)BN;
+        red_sum[half * 128 + r] = sum;
+        pair_sync();
+        const float mean = (red_sum[r] + red_sum[128 + r]) / (float)BN;
         // pass 2: biased variance about the mean
         float var = 0.f;
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 32 * half; c < BN; c += 64) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
 #pragma unroll
@@ -283,20 +300,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             var = fmaf(dv, dv, var);
           }
         }
-        const float rstd = 1.0f / sqrtf(var / (float)BN + p.eps);
+        red_var[half * 128 + r] = var;
+        pair_sync();
+        const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)BN + p.eps);
         // pass 3: LN(x) as split planes
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 32 * half; c < BN; c += 64) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
           uint32_t hi[16], lo[16];
 #pragma unroll
           for (int i = 0; i < 32; i += 2)
             split2((v[i] - mean) * rstd, (v[i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
-          stage_split(hi, lo, &tO_h, &tO_l, c);
+          stage_split(hi, lo, c, srow);
         }
       } else {  // EPI_HEAD
         float accv = 0.f;
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 32 * half; c < BN; c += 64) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
 #pragma unroll
@@ -305,7 +324,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             accv = fmaf(x, p.w2[c + i], accv);
           }
         }
-        if (valid) p.scores[grow] = accv + p.b2[0];
+        red_sum[half * 128 + r] = accv;
+        pair_sync();
+        if (half == 0 && valid) p.scores[grow] = (red_sum[r] + red_sum[128 + r]) + p.b2[0];
       }
       // every TMEM read of this accumulator has completed (tcgen05.wait::ld)
       tc_fence_before();
