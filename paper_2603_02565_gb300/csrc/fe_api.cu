@@ -57,6 +57,8 @@ struct Planes {
   int rows = 0;
   CUtensorMap th{}, tl{};  // operand loads: 64 x 128 boxes, 128-byte swizzle
   CUtensorMap sh{}, sl{};  // epilogue stores: 32 x 32 boxes, 64-byte swizzle
+  CUtensorMap ah{}, al{};  // attention queries: d_h x 128 boxes
+  CUtensorMap kh{}, kl{};  // attention keys / values: d_h x (64 for d_h = 32, else 128) boxes
 };
 
 // fp32 rows (the residual streams), with the epilogue's store descriptor.
@@ -122,6 +124,17 @@ int map_out(Planes& p) {
   if (rc == FE_OK)
     rc = encode_map_t(&p.sl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.l, p.ld, p.rows, 32, 32,
                       CU_TENSOR_MAP_SWIZZLE_64B);
+  return rc;
+}
+
+// Descriptors of an attention operand (Q, K or V head slices).
+int map_attn(Planes& p, int dh) {
+  const CUtensorMapSwizzle sw = dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
+  const int kv_rows = dh == 32 ? 64 : 128;
+  int rc = encode_map_t(&p.ah, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.h, p.ld, p.rows, dh, 128, sw);
+  if (rc == FE_OK) rc = encode_map_t(&p.al, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.l, p.ld, p.rows, dh, 128, sw);
+  if (rc == FE_OK) rc = encode_map_t(&p.kh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.h, p.ld, p.rows, dh, kv_rows, sw);
+  if (rc == FE_OK) rc = encode_map_t(&p.kl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.l, p.ld, p.rows, dh, kv_rows, sw);
   return rc;
 }
 
@@ -421,25 +434,25 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
 
     fe::AttnParams ap{};
-    ap.q_h = c->q.h;
-    ap.q_l = c->q.l;
-    ap.ldq = c->q.ld;
-    ap.k_h = c->KV.h + (size_t)(2 * l) * d;
-    ap.k_l = c->KV.l + (size_t)(2 * l) * d;
-    ap.v_h = c->KV.h + (size_t)(2 * l + 1) * d;
-    ap.v_l = c->KV.l + (size_t)(2 * l + 1) * d;
-    ap.ldkv = c->KV.ld;
-    ap.o_h = c->a.h;
-    ap.o_l = c->a.l;
-    ap.ldo = c->a.ld;
+    ap.n_segments = B;
+    ap.n_heads = c->H;
+    ap.max_q = cap;
     ap.q_off_dev = c->off;
     ap.q_cnt_dev = c->U;
     ap.kv_stride = C;
     ap.kv_cnt = C;
+    ap.q_col = 0;
+    ap.k_col = 2 * l * d;
+    ap.v_col = (2 * l + 1) * d;
+    ap.o_col = 0;
+    ap.o_h = c->a.h;
+    ap.o_l = c->a.l;
+    ap.ldo = c->a.ld;
     ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
+    ap.status = c->status;
     {
       Prof pf(c, "attn_item_ctx", s);
-      FE_CK(fe::attn_launch(c->dh, c->H, B, cap, ap, s));
+      FE_CK(fe::attn_launch(c->dh, &c->q.ah, &c->q.al, &c->KV.kh, &c->KV.kl, &c->KV.kh, &c->KV.kl, ap, s));
     }
 
     fe::GemmParams po{};
@@ -513,25 +526,25 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     fe::GemmParams p{};
     FE_RC(gemm(c, "gemm_cross_qkv", fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, &c->qkv, nullptr, s));
     fe::AttnParams ap{};
-    ap.q_h = c->qkv.h;
-    ap.q_l = c->qkv.l;
-    ap.ldq = c->qkv.ld;
-    ap.k_h = c->qkv.h + d;
-    ap.k_l = c->qkv.l + d;
-    ap.v_h = c->qkv.h + 2 * d;
-    ap.v_l = c->qkv.l + 2 * d;
-    ap.ldkv = c->qkv.ld;
-    ap.o_h = c->ax.h;
-    ap.o_l = c->ax.l;
-    ap.ldo = c->ax.ld;
+    ap.n_segments = B;
+    ap.n_heads = c->H;
+    ap.max_q = K;
     ap.q_stride = K;
     ap.q_cnt_fixed = K;
     ap.kv_stride = K;
     ap.kv_cnt = K;
+    ap.q_col = 0;
+    ap.k_col = d;
+    ap.v_col = 2 * d;
+    ap.o_col = 0;
+    ap.o_h = c->ax.h;
+    ap.o_l = c->ax.l;
+    ap.ldo = c->ax.ld;
     ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
+    ap.status = c->status;
     {
       Prof pf(c, "attn_cross_seq", s);
-      FE_CK(fe::attn_launch(c->dh, c->H, B, K, ap, s));
+      FE_CK(fe::attn_launch(c->dh, &c->qkv.ah, &c->qkv.al, &c->qkv.kh, &c->qkv.kl, &c->qkv.kh, &c->qkv.kl, ap, s));
     }
     fe::GemmParams po{};
     po.resid = c->c.p;
@@ -643,6 +656,7 @@ int reserve_impl(fe_ctx* c, Shape s) {
     FE_RC(map_act(*p));
   for (Planes* p : {&c->KV, &c->q, &c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->qkv, &c->lncp})
     FE_RC(map_out(*p));
+  for (Planes* p : {&c->KV, &c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
   c->cap_shape = s;
   c->cap_rows = R;
   return FE_OK;

@@ -1,14 +1,25 @@
-// Flash-style multi-head attention over request segments.
+// Flash-style multi-head attention over request segments, on tcgen05.
 //
-// Used twice per layer structure of the evaluator:
+// Used twice in the evaluator:
 //  * element -> context cross-attention (Section 4.2): the query rows are the
 //    distinct elements of request b, the keys/values its C context rows, so
 //    the context K/V computed once per request serve every element;
 //  * cross-sequence self-attention (Section 4.4) over the K sequence vectors.
-// One CTA = 4 warps = 64 query rows of one (segment, head); the keys stream
-// through shared memory in blocks of 64 with an online softmax in fp32.
-// Operands are split pairs (hi + lo bf16); S = Qh Kh + Qh Kl + Ql Kh and
-// O = Ph Vh + Ph Vl + Pl Vh, fp32 accumulation.
+//
+// Persistent CTAs walk units (segment b, head h, 128-row query tile).  Per
+// unit the keys stream in chunks of CK (64 for d_h = 32, 128 for d_h = 64):
+//   warp 0 lane 0 : TMA producer -- Q tile (two buffers, one per unit in
+//                   flight) and K/V chunks of CK keys (two stages)
+//   warp 1 lane 0 : tcgen05.mma -- S = Q K^T into one of two TMEM tiles
+//                   (S_{j+1} overlaps the softmax of chunk j), then
+//                   PV = P V into a third TMEM region
+//   warps 2..     : online softmax from TMEM, one query row per lane; with
+//                   d_h = 64, warps w and w+4 share TMEM lane quadrant w % 4
+//                   and each take half of the chunk's keys and half of the
+//                   output columns; P is written to shared memory as a split
+//                   pair and the running output is rescaled in registers
+// Operands are split pairs (hi + lo bf16): S = Qh Kh + Ql Kh + Qh Kl and
+// PV = Ph Vh + Pl Vh + Ph Vl, fp32 accumulation; softmax in fp32.
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -16,247 +27,370 @@ namespace fe {
 
 namespace {
 
-constexpr int BQ = 64;
-constexpr int BKV = 64;
+constexpr int BQ = 128;     // query rows per unit (TMEM lanes)
 
-__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
-               "r"(valid ? 16 : 0)
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t* r, const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_u32(p)));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t* r, const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_u32(p)));
-}
-
-__device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-      "{%0,%1,%2,%3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
+// d_h = 32: 64-key chunks and 4 softmax warps, small enough for two CTAs per SM.
+// d_h = 64: 128-key chunks and 8 softmax warps (two per TMEM lane quadrant).
 template <int DH>
-__host__ __device__ constexpr int pitch() { return DH + 8; }  // bf16 per shared row (16 B pad: conflict-free ldmatrix)
+struct AttnCfg {
+  static constexpr int CK = DH == 32 ? 64 : 128;                // keys per chunk
+  static constexpr int kSoftmaxWarps = DH == 32 ? 4 : 8;
+  static constexpr int kHalves = kSoftmaxWarps / 4;              // warps sharing one lane quadrant
+  static constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
+  static constexpr int kCtasPerSM = DH == 32 ? 2 : 1;
+  static constexpr uint32_t kTmemCols = DH == 32 ? 256 : 512;  // 2 S tiles + PV
+  static constexpr uint32_t kRowBytes = DH * 2;                 // one row of a Q/K/V tile
+  static constexpr uint32_t kTile = 128 * kRowBytes;            // Q tile: 128 rows, one plane
+  static constexpr uint32_t kKVTile = CK * kRowBytes;           // K or V chunk: CK rows, one plane
+  static constexpr uint32_t kSwz = DH == 32 ? 4u : 2u;          // descriptor swizzle code (64 B / 128 B)
+  static constexpr uint32_t kSbo = 8 * kRowBytes;               // 8-row swizzle atom
+  static constexpr uint32_t kQBytes = 2 * kTile;                // hi + lo
+  static constexpr uint32_t kKVBytes = 4 * kKVTile;             // Kh Kl Vh Vl
+  static constexpr uint32_t kPBlock = 128 * 128;                // 128 rows x 64 keys x 2 B
+  static constexpr uint32_t kPBytes = 2 * (CK / 64) * kPBlock;  // 2 planes x key blocks
+  static constexpr int kKVStages = DH == 32 ? 2 : 1;
+  static constexpr uint32_t kRed = 2 * 2 * 2 * 128 * 4;       // [max|sum][parity][half][row]
+  static constexpr size_t kSmem = 1024 + 2 * kQBytes + kKVStages * kKVBytes + kPBytes + 256 + kRed;
+};
 
-template <int DH>
-constexpr size_t attn_smem() { return (size_t)(2 * BQ + 8 * BKV) * pitch<DH>() * 2; }
+__device__ __forceinline__ uint64_t desc_sw(uint32_t saddr, uint32_t sbo, uint32_t swz) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;                       // leading byte offset (unused: one atom wide)
+  d |= (uint64_t)(sbo >> 4) << 32;              // stride byte offset: next 8-row atom
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)swz << 61;
+  return d;
+}
+
+__device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
 
 }  // namespace
 
 template <int DH>
-__global__ void __launch_bounds__(128) attn_kernel(const AttnParams p) {
-  constexpr int P = pitch<DH>();
-  constexpr int CH = DH / 8;  // 16-byte chunks per row
-  extern __shared__ __align__(16) uint8_t smem_raw[];
-  bf16* sQh = reinterpret_cast<bf16*>(smem_raw);
-  bf16* sQl = sQh + BQ * P;
-  bf16* sKV = sQl + BQ * P;  // [buffer 2][plane 4: Kh Kl Vh Vl][BKV * P]
+__global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM)
+    attn_kernel(const __grid_constant__ CUtensorMap tQh, const __grid_constant__ CUtensorMap tQl,
+                const __grid_constant__ CUtensorMap tKh, const __grid_constant__ CUtensorMap tKl,
+                const __grid_constant__ CUtensorMap tVh, const __grid_constant__ CUtensorMap tVl,
+                const AttnParams p) {
+  using Cfg = AttnCfg<DH>;
+  constexpr int CK = Cfg::CK;
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_s = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
+  uint8_t* sQ = smem;                                   // [2 buffers][hi, lo]
+  uint8_t* sKV = sQ + 2 * Cfg::kQBytes;                 // [stages][Kh, Kl, Vh, Vl]
+  uint8_t* sP = sKV + Cfg::kKVStages * Cfg::kKVBytes;   // [hi, lo][key block 0, 1]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + Cfg::kPBytes);
+  uint64_t* q_full = bars;        // [2]
+  uint64_t* q_empty = bars + 2;   // [2]
+  uint64_t* kv_full = bars + 4;   // [2]
+  uint64_t* kv_empty = bars + 6;  // [2]
+  uint64_t* s_full = bars + 8;    // [2]
+  uint64_t* p_full = bars + 10;
+  uint64_t* pv_full = bars + 11;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // row-statistic exchange
 
-  const int b = blockIdx.z, head = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   pdl_wait();
+  const int qtiles = p.max_q_tiles;
+  const int units = p.n_segments * p.n_heads * qtiles;
+  const int nch = (p.kv_cnt + CK - 1) / CK;
+  if ((int)blockIdx.x >= units) return;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(q_full + i, 1);
+      mbar_init(q_empty + i, 1);
+      mbar_init(kv_full + i, 1);
+      mbar_init(kv_empty + i, 1);
+      mbar_init(s_full + i, 1);
+    }
+    mbar_init(p_full, 32 * Cfg::kSoftmaxWarps);
+    mbar_init(pv_full, 1);
+    fence_mbar_init();
+    prefetch_tmap(&tQh);
+    prefetch_tmap(&tKh);
+    prefetch_tmap(&tVh);
+  }
+  if (warp == 0) tmem_alloc(tmem_slot, Cfg::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;  // S tiles at columns [0,CK) and [CK,2CK), PV at [2CK, 2CK+DH)
   pdl_trigger();
-  const int q_cnt = p.q_cnt_dev ? p.q_cnt_dev[b] : p.q_cnt_fixed;
-  const int q_begin = blockIdx.x * BQ;
-  if (q_begin >= q_cnt) return;
-  const int q_off = p.q_off_dev ? p.q_off_dev[b] : b * p.q_stride;
-  const int kv_off = b * p.kv_stride;
-  const int kv_cnt = p.kv_cnt;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int col0 = head * DH;
 
-  for (int i = tid; i < BQ * CH; i += 128) {
-    const int r = i / CH, c = i % CH;
-    const bool v = q_begin + r < q_cnt;
-    const size_t go = (size_t)(q_off + q_begin + (v ? r : 0)) * p.ldq + col0 + c * 8;
-    cp_async16(sQh + r * P + c * 8, p.q_h + go, v);
-    cp_async16(sQl + r * P + c * 8, p.q_l + go, v);
-  }
-  auto load_kv = [&](int kb, int buf) {
-    bf16* base = sKV + buf * 4 * BKV * P;
-    for (int i = tid; i < BKV * CH; i += 128) {
-      const int r = i / CH, c = i % CH;
-      const int key = kb * BKV + r;
-      const bool v = key < kv_cnt;
-      const size_t go = (size_t)(kv_off + (v ? key : 0)) * p.ldkv + col0 + c * 8;
-      const int so = r * P + c * 8;
-      cp_async16(base + 0 * BKV * P + so, p.k_h + go, v);
-      cp_async16(base + 1 * BKV * P + so, p.k_l + go, v);
-      cp_async16(base + 2 * BKV * P + so, p.v_h + go, v);
-      cp_async16(base + 3 * BKV * P + so, p.v_l + go, v);
-    }
+  // unit u -> (segment, head, query tile); query tile fastest
+  auto unit_info = [&](int u, int& b, int& h, int& q0, int& qcnt, int& qoff) {
+    const int qt = u % qtiles;
+    h = (u / qtiles) % p.n_heads;
+    b = u / (qtiles * p.n_heads);
+    qcnt = p.q_cnt_dev ? p.q_cnt_dev[b] : p.q_cnt_fixed;
+    qoff = p.q_off_dev ? p.q_off_dev[b] : b * p.q_stride;
+    q0 = qt * BQ;
   };
-  load_kv(0, 0);
-  cp_async_commit();
 
-  const int nkb = (kv_cnt + BKV - 1) / BKV;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-  float o[DH / 8][4];
-#pragma unroll
-  for (int i = 0; i < DH / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-  uint32_t qh[DH / 16][4], ql[DH / 16][4];
-
-  for (int kb = 0; kb < nkb; ++kb) {
-    const int buf = kb & 1;
-    if (kb + 1 < nkb) {
-      load_kv(kb + 1, buf ^ 1);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
-    __syncthreads();
-    if (kb == 0) {
-#pragma unroll
-      for (int kc = 0; kc < DH / 16; ++kc) {
-        const int off = (warp * 16 + (lane & 15)) * P + kc * 16 + (lane >> 4) * 8;
-        ldsm_x4(qh[kc], sQh + off);
-        ldsm_x4(ql[kc], sQl + off);
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      int ui = 0, gc = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        int b, h, q0, qcnt, qoff;
+        unit_info(u, b, h, q0, qcnt, qoff);
+        if (q0 >= qcnt) continue;
+        const int qb = ui & 1;
+        if (ui >= 2 && !mbar_wait_bounded(q_empty + qb, ((ui >> 1) - 1) & 1, p.status)) break;
+        uint8_t* q = sQ + qb * Cfg::kQBytes;
+        mbar_arrive_expect_tx(q_full + qb, Cfg::kQBytes);
+        tma_load_2d(q, &tQh, p.q_col + h * DH, qoff + q0, q_full + qb);
+        tma_load_2d(q + Cfg::kTile, &tQl, p.q_col + h * DH, qoff + q0, q_full + qb);
+        for (int j = 0; j < nch; ++j, ++gc) {
+          const int ks = gc % Cfg::kKVStages;
+          if (gc >= Cfg::kKVStages &&
+              !mbar_wait_bounded(kv_empty + ks, ((gc / Cfg::kKVStages) - 1) & 1, p.status)) {
+            ok = false;
+            break;
+          }
+          uint8_t* kv = sKV + ks * Cfg::kKVBytes;
+          const int row = b * p.kv_stride + j * CK;
+          mbar_arrive_expect_tx(kv_full + ks, Cfg::kKVBytes);
+          tma_load_2d(kv, &tKh, p.k_col + h * DH, row, kv_full + ks);
+          tma_load_2d(kv + Cfg::kKVTile, &tKl, p.k_col + h * DH, row, kv_full + ks);
+          tma_load_2d(kv + 2 * Cfg::kKVTile, &tVh, p.v_col + h * DH, row, kv_full + ks);
+          tma_load_2d(kv + 3 * Cfg::kKVTile, &tVl, p.v_col + h * DH, row, kv_full + ks);
+        }
+        ++ui;
       }
     }
-    const bf16* sKh = sKV + buf * 4 * BKV * P;
-    const bf16* sKl = sKh + BKV * P;
-    const bf16* sVh = sKl + BKV * P;
-    const bf16* sVl = sVh + BKV * P;
-
-    // S = Q K^T over 64 keys: 8 n-blocks of 8 keys
-    float s[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
-#pragma unroll
-    for (int kc = 0; kc < DH / 16; ++kc) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        const int off = (np * 16 + (lane & 7) + ((lane >> 4) << 3)) * P + kc * 16 + ((lane >> 3) & 1) * 8;
-        uint32_t kh[4], kl[4];
-        ldsm_x4(kh, sKh + off);
-        ldsm_x4(kl, sKl + off);
-        mma16816(s[2 * np], qh[kc], kh[0], kh[1]);
-        mma16816(s[2 * np], qh[kc], kl[0], kl[1]);
-        mma16816(s[2 * np], ql[kc], kh[0], kh[1]);
-        mma16816(s[2 * np + 1], qh[kc], kh[2], kh[3]);
-        mma16816(s[2 * np + 1], qh[kc], kl[2], kl[3]);
-        mma16816(s[2 * np + 1], ql[kc], kh[2], kh[3]);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const uint32_t idesc_s = umma_idesc_bf16(BQ, CK);
+      const uint32_t idesc_pv = umma_idesc_bf16(BQ, DH) | (1u << 16);  // B (V) is MN-major
+      int ui = 0, gc = 0;
+      bool ok = true;
+      // S = Q K^T of global chunk gcc, the unit's Q in buffer qb
+      auto issue_s = [&](int qb, int gcc) -> bool {
+        const int ks = gcc % Cfg::kKVStages;
+        if (!mbar_wait_bounded(kv_full + ks, (gcc / Cfg::kKVStages) & 1, p.status)) return false;
+        tc_fence_after();
+        const uint32_t q = smem_u32(sQ + qb * Cfg::kQBytes);
+        const uint32_t k = smem_u32(sKV + ks * Cfg::kKVBytes);
+        const uint32_t dst = tmem + (uint32_t)((gcc & 1) * CK);
+#pragma unroll 1
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          // (Qh, Kh), (Ql, Kh), (Qh, Kl)
+          for (int pr = 0; pr < 3; ++pr) {
+            const uint32_t a = q + (pr == 1 ? Cfg::kTile : 0u) + (uint32_t)kk * 32;
+            const uint32_t bb = k + (pr == 2 ? Cfg::kKVTile : 0u) + (uint32_t)kk * 32;
+            umma_bf16(dst, desc_sw(a, Cfg::kSbo, Cfg::kSwz), desc_sw(bb, Cfg::kSbo, Cfg::kSwz), idesc_s,
+                      (kk | pr) != 0 ? 1u : 0u);
+          }
+        }
+        umma_commit(s_full + (gcc & 1));
+        return true;
+      };
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        int b, h, q0, qcnt, qoff;
+        unit_info(u, b, h, q0, qcnt, qoff);
+        if (q0 >= qcnt) continue;
+        const int qb = ui & 1;
+        if (!mbar_wait_bounded(q_full + qb, (ui >> 1) & 1, p.status)) break;
+        for (int j = 0; j < nch; ++j, ++gc) {
+          if (j == 0 && !issue_s(qb, gc)) {
+            ok = false;
+            break;
+          }
+          // with two K/V stages S_{j+1} overlaps the softmax of chunk j; with one
+          // stage chunk j+1 can only load after PV_j, so S_{j+1} follows PV_j
+          if (Cfg::kKVStages == 2 && j + 1 < nch && !issue_s(qb, gc + 1)) {
+            ok = false;
+            break;
+          }
+          if (j + 1 == nch) umma_commit(q_empty + qb);  // every S of this unit issued: Q buffer frees on completion
+          // PV = P V once the softmax has written P for this chunk
+          if (!mbar_wait_bounded(p_full, gc & 1, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const int ks = gc % Cfg::kKVStages;
+          const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + 2 * Cfg::kKVTile);
+          const uint32_t pp = smem_u32(sP);
+#pragma unroll 1
+          for (int kk = 0; kk < CK / 16; ++kk) {
+            const uint32_t pa = pp + (uint32_t)(kk >> 2) * Cfg::kPBlock + (uint32_t)(kk & 3) * 32;
+            const uint32_t vb = v + (uint32_t)kk * 16 * Cfg::kRowBytes;
+            // (Ph, Vh), (Pl, Vh), (Ph, Vl)
+            for (int pr = 0; pr < 3; ++pr) {
+              const uint32_t a = pa + (pr == 1 ? (uint32_t)(CK / 64) * Cfg::kPBlock : 0u);
+              const uint32_t bb = vb + (pr == 2 ? Cfg::kKVTile : 0u);
+              umma_bf16(tmem + 2 * CK, desc_sw(a, 1024, 2), desc_sw(bb, Cfg::kSbo, Cfg::kSwz), idesc_pv,
+                        (kk | pr) != 0 ? 1u : 0u);
+            }
+          }
+          umma_commit(pv_full);
+          umma_commit(kv_empty + ks);
+          if (Cfg::kKVStages == 1 && j + 1 < nch && !issue_s(qb, gc + 1)) {
+            ok = false;
+            break;
+          }
+        }
+        ++ui;
       }
     }
-    // scale (log2 domain) and mask keys past the segment
-    float mx0 = -INFINITY, mx1 = -INFINITY;
+  } else {
+    // ---------------- softmax / output (warps 2..9) ----------------
+    constexpr int DO = DH / Cfg::kHalves;  // output columns per warp
+    constexpr int KW = CK / Cfg::kHalves;  // keys per warp and chunk (64)
+    const int sw = warp - 2;
+    const int q4 = warp & 3;
+    const int half = sw >> 2;     // keys [KW half, KW half + KW) of each chunk, output columns [DO half, DO half + DO)
+    const int r = q4 * 32 + lane; // query row of the tile = TMEM lane
+    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    float* red_max = red;         // [parity][half][128]
+    float* red_sum = red + 512;
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q4) : "memory"); };
+    uint8_t* pH = sP + (uint32_t)half * Cfg::kPBlock;
+    uint8_t* pL = sP + (uint32_t)(CK / 64) * Cfg::kPBlock + (uint32_t)half * Cfg::kPBlock;
+    int gc = 0, ui = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      int b, h, q0, qcnt, qoff;
+      unit_info(u, b, h, q0, qcnt, qoff);
+      if (q0 >= qcnt) continue;
+      float m = -INFINITY, l = 0.f;
+      float o[DO];
 #pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-      const int key = kb * BKV + nb * 8 + 2 * (lane & 3);
+      for (int i = 0; i < DO; ++i) o[i] = 0.f;
+      for (int j = 0; j < nch; ++j, ++gc) {
+        if (!mbar_wait_bounded(s_full + (gc & 1), (gc >> 1) & 1, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float v[64];
+        tmem_ld64(tmem + lane_off + (uint32_t)((gc & 1) * CK + half * KW), v);
+        const int kvalid = p.kv_cnt - j * CK - half * KW;  // valid keys among this warp's 64
+        float mx = -INFINITY;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const bool v = key + (e & 1) < kv_cnt;
-        s[nb][e] = v ? s[nb][e] * p.scale_log2 : -INFINITY;
+        for (int i = 0; i < 64; ++i) {
+          v[i] *= p.scale_log2;
+          if (i < kvalid) mx = fmaxf(mx, v[i]);
+        }
+        if (Cfg::kHalves == 2) {
+          float* rm = red_max + (gc & 1) * 256;
+          rm[half * 128 + r] = mx;
+          pair_sync();
+          mx = fmaxf(rm[r], rm[128 + r]);
+        }
+        const float mn = fmaxf(m, mx);
+        const float corr = ex2_approx(m - mn);
+        m = mn;
+        // P = 2^(s - m) as split pairs in the 128-byte-swizzled K-major tile (key block = half)
+        float sum = 0.f;
+#pragma unroll
+        for (int g = 0; g < 8; ++g) {
+          uint32_t hi[4], lo[4];
+#pragma unroll
+          for (int i = 0; i < 8; i += 2) {
+            const int k = 8 * g + i;
+            const float p0 = (k < kvalid) ? ex2_approx(v[k] - mn) : 0.f;
+            const float p1 = (k + 1 < kvalid) ? ex2_approx(v[k + 1] - mn) : 0.f;
+            sum += p0 + p1;
+            split2(p0, p1, hi[i / 2], lo[i / 2]);
+          }
+          const uint32_t off = (uint32_t)r * 128u + (((uint32_t)g ^ (uint32_t)(r & 7)) << 4);
+          *reinterpret_cast<uint4*>(pH + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          *reinterpret_cast<uint4*>(pL + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        }
+        l = l * corr + sum;
+        fence_async_shared();
+        tc_fence_before();
+        mbar_arrive1(p_full);
+        // fold this chunk's P V into this warp's output columns
+        if (!mbar_wait_bounded(pv_full, gc & 1, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float pv[DO];
+        if (DO == 16) {
+          tmem_ld16(tmem + lane_off + (uint32_t)(2 * CK + half * DO), pv);
+        } else {
+#pragma unroll
+          for (int c = 0; c < DO; c += 32) tmem_ld32(tmem + lane_off + (uint32_t)(2 * CK + half * DO + c), pv + c);
+        }
+#pragma unroll
+        for (int i = 0; i < DO; ++i) o[i] = o[i] * corr + pv[i];
       }
-      mx0 = fmaxf(mx0, fmaxf(s[nb][0], s[nb][1]));
-      mx1 = fmaxf(mx1, fmaxf(s[nb][2], s[nb][3]));
-    }
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-    const float c0 = exp2f(m0 - mn0), c1 = exp2f(m1 - mn1);
-    m0 = mn0;
-    m1 = mn1;
-    float rs0 = 0.f, rs1 = 0.f;
+      if (!ok) break;
+      // row sum over both halves, then O / l as a split pair
+      float ltot = l;
+      if (Cfg::kHalves == 2) {
+        float* rs = red_sum + (ui & 1) * 256;
+        rs[half * 128 + r] = l;
+        pair_sync();
+        ltot = rs[r] + rs[128 + r];
+      }
+      ++ui;
+      if (q0 + r < qcnt) {
+        const float inv = 1.f / ltot;
+        const size_t go = (size_t)(qoff + q0 + r) * p.ldo + p.o_col + h * DH + half * DO;
 #pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-      s[nb][0] = exp2f(s[nb][0] - mn0);
-      s[nb][1] = exp2f(s[nb][1] - mn0);
-      s[nb][2] = exp2f(s[nb][2] - mn1);
-      s[nb][3] = exp2f(s[nb][3] - mn1);
-      rs0 += s[nb][0] + s[nb][1];
-      rs1 += s[nb][2] + s[nb][3];
-    }
-    l0 = l0 * c0 + rs0;
-    l1 = l1 * c1 + rs1;
+        for (int c = 0; c < DO; c += 8) {
+          uint32_t hi[4], lo[4];
 #pragma unroll
-    for (int i = 0; i < DH / 8; ++i) {
-      o[i][0] *= c0;
-      o[i][1] *= c0;
-      o[i][2] *= c1;
-      o[i][3] *= c1;
-    }
-    // O += P V, P as split A fragments (16 keys per k-chunk)
-#pragma unroll
-    for (int kc = 0; kc < 4; ++kc) {
-      uint32_t ph[4], pl[4];
-      split2(s[2 * kc][0], s[2 * kc][1], ph[0], pl[0]);
-      split2(s[2 * kc][2], s[2 * kc][3], ph[1], pl[1]);
-      split2(s[2 * kc + 1][0], s[2 * kc + 1][1], ph[2], pl[2]);
-      split2(s[2 * kc + 1][2], s[2 * kc + 1][3], ph[3], pl[3]);
-#pragma unroll
-      for (int dp = 0; dp < DH / 16; ++dp) {
-        const int off = (kc * 16 + (lane & 7) + ((lane >> 3) & 1) * 8) * P + dp * 16 + (lane >> 4) * 8;
-        uint32_t vh[4], vl[4];
-        ldsm_x4_t(vh, sVh + off);
-        ldsm_x4_t(vl, sVl + off);
-        mma16816(o[2 * dp], ph, vh[0], vh[1]);
-        mma16816(o[2 * dp], ph, vl[0], vl[1]);
-        mma16816(o[2 * dp], pl, vh[0], vh[1]);
-        mma16816(o[2 * dp + 1], ph, vh[2], vh[3]);
-        mma16816(o[2 * dp + 1], ph, vl[2], vl[3]);
-        mma16816(o[2 * dp + 1], pl, vh[2], vh[3]);
+          for (int i = 0; i < 8; i += 2) split2(o[c + i] * inv, o[c + i + 1] * inv, hi[i / 2], lo[i / 2]);
+          *reinterpret_cast<uint4*>(p.o_h + go + c) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          *reinterpret_cast<uint4*>(p.o_l + go + c) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        }
       }
     }
-    __syncthreads();  // buffer `buf` is refilled two iterations later
   }
 
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
-  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
-  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
-  const float i0 = 1.f / l0, i1 = 1.f / l1;
-  const int r0 = q_begin + warp * 16 + (lane >> 2);
-  const int r1 = r0 + 8;
-#pragma unroll
-  for (int nb = 0; nb < DH / 8; ++nb) {
-    const int c = col0 + nb * 8 + 2 * (lane & 3);
-    uint32_t hi, lo;
-    if (r0 < q_cnt) {
-      split2(o[nb][0] * i0, o[nb][1] * i0, hi, lo);
-      const size_t go = (size_t)(q_off + r0) * p.ldo + c;
-      *reinterpret_cast<uint32_t*>(p.o_h + go) = hi;
-      *reinterpret_cast<uint32_t*>(p.o_l + go) = lo;
-    }
-    if (r1 < q_cnt) {
-      split2(o[nb][2] * i1, o[nb][3] * i1, hi, lo);
-      const size_t go = (size_t)(q_off + r1) * p.ldo + c;
-      *reinterpret_cast<uint32_t*>(p.o_h + go) = hi;
-      *reinterpret_cast<uint32_t*>(p.o_l + go) = lo;
-    }
-  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, Cfg::kTmemCols);
+}
+
+namespace {
+int g_attn_sms = 0;
 }
 
 cudaError_t attn_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(attn_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)attn_smem<32>());
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_attn_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)AttnCfg<32>::kSmem);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)attn_smem<64>());
+                             (int)AttnCfg<64>::kSmem);
   return e;
 }
 
-cudaError_t attn_launch(int dh, int n_heads, int n_segments, int max_q, const AttnParams& p, cudaStream_t s) {
-  if (n_segments <= 0 || max_q <= 0 || p.kv_cnt <= 0) return cudaSuccess;
-  dim3 grid((unsigned)((max_q + BQ - 1) / BQ), (unsigned)n_heads, (unsigned)n_segments);
-  if (dh == 32) return launch_k(attn_kernel<32>, grid, dim3(128), attn_smem<32>(), s, p);
-  return launch_k(attn_kernel<64>, grid, dim3(128), attn_smem<64>(), s, p);
+cudaError_t attn_launch(int dh, const CUtensorMap* q_h, const CUtensorMap* q_l, const CUtensorMap* k_h,
+                        const CUtensorMap* k_l, const CUtensorMap* v_h, const CUtensorMap* v_l, const AttnParams& p0,
+                        cudaStream_t s) {
+  if (p0.n_segments <= 0 || p0.max_q <= 0 || p0.kv_cnt <= 0) return cudaSuccess;
+  AttnParams p = p0;
+  p.max_q_tiles = (p.max_q + BQ - 1) / BQ;
+  const long long units = (long long)p.n_segments * p.n_heads * p.max_q_tiles;
+  const long long sms = g_attn_sms > 0 ? g_attn_sms : 148;
+  if (dh == 32) {
+    const long long grid = units < sms * AttnCfg<32>::kCtasPerSM ? units : sms * AttnCfg<32>::kCtasPerSM;
+    return launch_k(attn_kernel<32>, dim3((unsigned)grid), dim3(AttnCfg<32>::kThreads), AttnCfg<32>::kSmem, s, *q_h,
+                    *q_l, *k_h, *k_l, *v_h, *v_l, p);
+  }
+  const long long grid = units < sms * AttnCfg<64>::kCtasPerSM ? units : sms * AttnCfg<64>::kCtasPerSM;
+  return launch_k(attn_kernel<64>, dim3((unsigned)grid), dim3(AttnCfg<64>::kThreads), AttnCfg<64>::kSmem, s, *q_h,
+                  *q_l, *k_h, *k_l, *v_h, *v_l, p);
 }
 
 }  // namespace fe

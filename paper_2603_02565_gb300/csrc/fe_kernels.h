@@ -85,27 +85,33 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l,
                         const CUtensorMap* o_x, const GemmParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
-// Flash-style multi-head attention over request segments (split-bf16 operands)
-// segment b: query rows [q_off(b), q_off(b) + q_cnt(b)), key rows
-// [b * kv_stride, b * kv_stride + kv_cnt); grid (q tiles of 64, heads, segments)
+// Flash-style multi-head attention over request segments (tcgen05, split-bf16
+// operands).  Segment b: query rows [q_off(b), q_off(b) + q_cnt(b)), key and
+// value rows [b * kv_stride, b * kv_stride + kv_cnt).  Head h reads columns
+// q_col + h*dh of Q, k_col + h*dh of K, v_col + h*dh of V and writes columns
+// o_col + h*dh of the output planes.  The Q/K/V tensor maps have boxes of
+// dh x 128 with the 64-byte (dh = 32) or 128-byte (dh = 64) swizzle.
 // ---------------------------------------------------------------------------
 struct AttnParams {
-  const bf16 *q_h, *q_l;
-  int ldq;
-  const bf16 *k_h, *k_l, *v_h, *v_l;
-  int ldkv;
-  bf16 *o_h, *o_l;
-  int ldo;
+  int n_segments, n_heads;
+  int max_q;             // largest q_cnt of any segment (grid sizing)
+  int max_q_tiles;       // set by attn_launch
   const int* q_off_dev;  // null: q_off = b * q_stride
   const int* q_cnt_dev;  // null: q_cnt = q_cnt_fixed
   int q_stride;
   int q_cnt_fixed;
   int kv_stride;
   int kv_cnt;
+  int q_col, k_col, v_col, o_col;
+  bf16 *o_h, *o_l;
+  int ldo;
   float scale_log2;      // log2(e) / sqrt(d_h)
+  int* status;
 };
 cudaError_t attn_prepare();
-cudaError_t attn_launch(int dh, int n_heads, int n_segments, int max_q, const AttnParams& p, cudaStream_t s);
+cudaError_t attn_launch(int dh, const CUtensorMap* q_h, const CUtensorMap* q_l, const CUtensorMap* k_h,
+                        const CUtensorMap* k_l, const CUtensorMap* v_h, const CUtensorMap* v_l, const AttnParams& p,
+                        cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // element-wise / gather / selection kernels (fe_misc.cu)
