@@ -201,6 +201,25 @@ def oracle_requests_per_s(w, budget_s=12.0, max_requests=None):
 
 
 # ----------------------------------------------------------------------------------------------
+# multi-rank bookkeeping (requests are independent: each rank scores its own batch)
+# ----------------------------------------------------------------------------------------------
+def rank_copy_shift(rank, copy, B):
+    """Request rotation of input copy `copy` on rank `rank` (distinct batches per rank)."""
+    return (7 * copy + 3 * rank) % B
+
+
+def weak_scaling_value(local_ms, world, B, steps, dist=None, device=None):
+    """Whole-job requests/s: every rank scored `steps` batches of B requests; the
+    job time is the slowest rank's (max over ranks)."""
+    import torch
+    t = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    if dist is not None and world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    return world * B * steps / (total_ms / 1e3), total_ms
+
+
+# ----------------------------------------------------------------------------------------------
 # GPU arm
 # ----------------------------------------------------------------------------------------------
 def run_ours(args):
@@ -237,7 +256,7 @@ def run_ours(args):
     n_copies = int(min(16, max(2, math.ceil(2 * L2 / max(in_bytes, 1)))))
     copies = []
     for i in range(n_copies):
-        sh = (7 * i + 3 * rank) % B
+        sh = rank_copy_shift(rank, i, B)
         ctx = torch.from_numpy(np.roll(w.context, sh, axis=0)).to(dev, dt)
         pool = torch.from_numpy(np.roll(w.pool, sh, axis=0)).to(dev, dt)
         idx = torch.from_numpy(np.ascontiguousarray(np.roll(w.cand_idx, sh, axis=0))).to(dev)
@@ -285,13 +304,8 @@ def run_ours(args):
     if st != FE_OK:
         raise SystemExit(f"batch status {st}")
     launches = ev.kernels_per_batch()
-    total_ms = e0.elapsed_time(e1)
-    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-    if dist:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms = float(t.item())
+    value, total_ms = weak_scaling_value(e0.elapsed_time(e1), world, B, args.steps, dist, dev)
     ms_per_step = total_ms / args.steps
-    value = world * B * args.steps / (total_ms / 1e3)
 
     # single-batch latency distribution (back to back, graph replay)
     lat = []
