@@ -95,7 +95,6 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // row-statistic exchange
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  pdl_wait();
   const int qtiles = p.max_q_tiles;
   const int units = p.n_segments * p.n_heads * qtiles;
   const int nch = (p.kv_cnt + CK - 1) / CK;
@@ -121,7 +120,10 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;  // S tiles at columns [0,CK) and [CK,2CK), PV at [2CK, 2CK+DH)
+  // the set-up above reads nothing written by earlier kernels; from here on
+  // the segment offsets, counts and operands are
   pdl_trigger();
+  pdl_wait();
 
   // unit u -> (segment, head, query tile); query tile fastest
   auto unit_info = [&](int u, int& b, int& h, int& q0, int& qcnt, int& qoff) {

@@ -82,13 +82,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* red = reinterpret_cast<float*>(stg_base + (size_t)kEpiWarps * 2 * kStageOut);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  pdl_wait();
-  int rows_valid = p.rows;
-  if (p.rows_dev) rows_valid = min(*p.rows_dev, p.rows);
-  const int nt = p.N / BN;
-  const int tiles = ((rows_valid + BM - 1) / BM) * nt;
-  if ((int)blockIdx.x >= tiles) return;  // nothing for this CTA
-
+  // set-up needs nothing from earlier kernels, so it runs before the
+  // programmatic wait and overlaps the tail of the previous kernel
   const uint32_t ncols = pow2_cols(nacc * BN);
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -112,6 +107,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
   const int nk = p.K_pad / BK;
   pdl_trigger();
+  pdl_wait();
+  int rows_valid = p.rows;
+  if (p.rows_dev) rows_valid = min(*p.rows_dev, p.rows);
+  const int nt = p.N / BN;
+  const int tiles = ((rows_valid + BM - 1) / BM) * nt;
+  if ((int)blockIdx.x >= tiles) {  // nothing for this CTA (uniform)
+    if (warp == 0) tmem_dealloc(tmem, ncols);
+    return;
+  }
 
   if (warp == 0) {
     if (lane == 0) {
@@ -220,13 +224,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
 
     int tl = 0;
+    float xr[64];  // EPI_RESID_LN with BN <= 128: this warp's chunks of the row
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tl) {
       const int acc = tl % nacc, use = tl / nacc;
-      if (!mbar_wait_bounded(tfull + acc, use & 1, p.status)) break;
-      tc_fence_after();
       const int m0 = (t / nt) * BM, n0 = (t % nt) * BN;
       const int grow = m0 + r;
       const bool valid = grow < rows_valid;
+      if (EPI == EPI_RESID_LN && BN <= 128) {
+        // residual rows, loaded while the MMAs of this tile run
+        const float* rrow = p.resid + (p.ldr ? (size_t)grow * p.ldr : (size_t)0);
+#pragma unroll
+        for (int ci = 0; ci < 2; ++ci) {
+          const int c = 32 * half + 64 * ci;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float4 qv = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (valid && c < BN) qv = reinterpret_cast<const float4*>(rrow + c)[j];
+            xr[32 * ci + 4 * j] = qv.x;
+            xr[32 * ci + 4 * j + 1] = qv.y;
+            xr[32 * ci + 4 * j + 2] = qv.z;
+            xr[32 * ci + 4 * j + 3] = qv.w;
+          }
+        }
+      }
+      if (!mbar_wait_bounded(tfull + acc, use & 1, p.status)) break;
+      tc_fence_after();
       const int srow = m0 + q * 32;
       const uint32_t trow = tmem + (uint32_t)(acc * BN) + ((uint32_t)(q * 32) << 16);
       float* red_sum = red + (size_t)(tl & 1) * 512;  // [half][128]
@@ -237,14 +259,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
           const int col = n0 + c;
+          if (p.bias) {
+            const float4* b4 = reinterpret_cast<const float4*>(p.bias + col);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 bb = __ldg(b4 + j);
+              v[4 * j] += bb.x;
+              v[4 * j + 1] += bb.y;
+              v[4 * j + 2] += bb.z;
+              v[4 * j + 3] += bb.w;
+            }
+          }
           uint32_t hi[16], lo[16];
 #pragma unroll
           for (int i = 0; i < 32; i += 2) {
             float x0 = v[i], x1 = v[i + 1];
-            if (p.bias) {
-              x0 += p.bias[col + i];
-              x1 += p.bias[col + i + 1];
-            }
             if (p.relu) {
               x0 = fmaxf(x0, 0.f);
               x1 = fmaxf(x1, 0.f);
@@ -253,8 +282,74 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           stage_split(hi, lo, col, srow);
         }
+      } else if (EPI == EPI_RESID_LN && BN <= 128) {
+        // rows of at most 128 columns: each warp holds its (at most two) chunks of
+        // x = resid + acc + bias in registers; the residual was loaded before the
+        // accumulator was ready, TMEM is read once
+        float sum = 0.f;
+#pragma unroll
+        for (int ci = 0; ci < 2; ++ci) {
+          const int c = 32 * half + 64 * ci;
+          if (c < BN) {
+            float v[32];
+            tmem_ld32(trow + (uint32_t)c, v);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) xr[32 * ci + i] += v[i];
+            if (p.bias) {
+              const float4* b4 = reinterpret_cast<const float4*>(p.bias + c);
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const float4 bb = __ldg(b4 + j);
+                xr[32 * ci + 4 * j] += bb.x;
+                xr[32 * ci + 4 * j + 1] += bb.y;
+                xr[32 * ci + 4 * j + 2] += bb.z;
+                xr[32 * ci + 4 * j + 3] += bb.w;
+              }
+            }
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+              sum += (xr[32 * ci + i] + xr[32 * ci + i + 1]) + (xr[32 * ci + i + 2] + xr[32 * ci + i + 3]);
+            uint8_t* b = next_stage();
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const uint32_t o = (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4);
+              *reinterpret_cast<float4*>(b + o) =
+                  make_float4(xr[32 * ci + 4 * j], xr[32 * ci + 4 * j + 1], xr[32 * ci + 4 * j + 2],
+                              xr[32 * ci + 4 * j + 3]);
+            }
+            issue(&tO_x, b, nullptr, nullptr, c, srow);
+          }
+        }
+        red_sum[half * 128 + r] = sum;
+        pair_sync();
+        const float mean = (red_sum[r] + red_sum[128 + r]) / (float)BN;
+        float var = 0.f;
+#pragma unroll
+        for (int ci = 0; ci < 2; ++ci) {
+          if (32 * half + 64 * ci < BN) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float dv = xr[32 * ci + i] - mean;
+              var = fmaf(dv, dv, var);
+            }
+          }
+        }
+        red_var[half * 128 + r] = var;
+        pair_sync();
+        const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)BN + p.eps);
+#pragma unroll
+        for (int ci = 0; ci < 2; ++ci) {
+          const int c = 32 * half + 64 * ci;
+          if (c < BN) {
+            uint32_t hi[16], lo[16];
+#pragma unroll
+            for (int i = 0; i < 32; i += 2)
+              split2((xr[32 * ci + i] - mean) * rstd, (xr[32 * ci + i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
+            stage_split(hi, lo, c, srow);
+          }
+        }
       } else if (EPI == EPI_RESID_LN) {
-        // pass 1: x = resid + acc + bias, stored out and kept in TMEM
+        // wider rows: x kept in TMEM between the passes
         float sum = 0.f;
         const float* rrow = p.resid + (p.ldr ? (size_t)grow * p.ldr : (size_t)0);
         for (int c = 32 * half; c < BN; c += 64) {
@@ -289,7 +384,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         red_sum[half * 128 + r] = sum;
         pair_sync();
         const float mean = (red_sum[r] + red_sum[128 + r]) / (float)BN;
-        // pass 2: biased variance about the mean
         float var = 0.f;
         for (int c = 32 * half; c < BN; c += 64) {
           float v[32];
@@ -303,7 +397,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         red_var[half * 128 + r] = var;
         pair_sync();
         const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)BN + p.eps);
-        // pass 3: LN(x) as split planes
         for (int c = 32 * half; c < BN; c += 64) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
