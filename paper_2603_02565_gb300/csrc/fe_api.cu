@@ -152,6 +152,7 @@ int alloc_f32(F32Rows& f, int rows, int ld, std::vector<void*>& owned) {
 struct Weight {
   Planes p;
   int N = 0, K_pad = 0, BN = 0, stages = 0;
+  CUtensorMap fh{}, fl{};  // W1 of the fused FFN: 64 x 64 boxes
 };
 
 int largest_bn(int N, int cap) {
@@ -190,6 +191,7 @@ struct fe_ctx {
   fe_config cfg{};
   int device = 0;
   int d = 0, H = 0, dh = 0, Ly = 0, F = 0, dpad = 0, Fpad = 0, nb = 1;
+  bool fused_ffn = false;  // FFN1 + FFN2 in one kernel (d <= 128)
   std::vector<void*> owned_w;  // weight allocations
   std::vector<void*> owned_ws; // workspace allocations
   float* w32 = nullptr;        // every weight in fp32, fe_weight_count order
@@ -350,6 +352,12 @@ int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
   return rc;
 }
 
+int map_fused_w1(Weight& w, bool two) {
+  int rc = encode_map(&w.fh, w.p.h, w.p.ld, w.p.rows, 64);
+  if (rc == FE_OK) rc = encode_map(&w.fl, two ? w.p.l : w.p.h, w.p.ld, w.p.rows, 64);
+  return rc;
+}
+
 int fill_weight(Weight& w, const float* W, int Kin, int N, int row0) {
   FE_CK(fe::transpose_split_launch(W, Kin, N, w.p.h, w.p.l, w.p.ld, row0, 0));
   return FE_OK;
@@ -382,6 +390,27 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   p.eps = c->cfg.ln_eps;
   FE_CK(fe::gemm_launch(epi, &A.th, &A.tl, &W.p.th, &W.p.tl, out ? &out->sh : nullptr, out ? &out->sl : nullptr,
                         xout ? &xout->sx : nullptr, p, s));
+  return FE_OK;
+}
+
+int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& W1, const Weight& W2, const float* b1,
+        const float* b2, const F32Rows& x, const Planes& ln_out, int rows, const int* rows_dev, cudaStream_t s) {
+  if (rows <= 0) return FE_OK;
+  Prof pf(c, site, s);
+  fe::FfnParams p{};
+  p.rows = rows;
+  p.rows_dev = rows_dev;
+  p.d = c->d;
+  p.d_pad = c->dpad;
+  p.F = c->F;
+  p.nb = c->nb;
+  p.b1 = b1;
+  p.b2 = b2;
+  p.resid = x.p;
+  p.ldr = x.ld;
+  p.eps = c->cfg.ln_eps;
+  p.status = c->status;
+  FE_CK(fe::ffn_launch(&A.th, &A.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.sh, &ln_out.sl, &x.sx, p, s));
   return FE_OK;
 }
 
@@ -460,16 +489,20 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     po.ldr = d;
     FE_RC(gemm(c, "gemm_item_o_ln", fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, &c->xln, &c->h, s));
 
-    fe::GemmParams p1{};
-    p1.bias = lw(c, l, T_B1);
-    p1.relu = 1;
-    FE_RC(gemm(c, "gemm_item_ffn1", fe::EPI_STORE, c->xln, c->w1[l], R, sumU, p1, &c->mid, nullptr, s));
+    if (c->fused_ffn) {
+      FE_RC(ffn(c, "ffn_item", c->xln, c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), c->h, c->xln, R, sumU, s));
+    } else {
+      fe::GemmParams p1{};
+      p1.bias = lw(c, l, T_B1);
+      p1.relu = 1;
+      FE_RC(gemm(c, "gemm_item_ffn1", fe::EPI_STORE, c->xln, c->w1[l], R, sumU, p1, &c->mid, nullptr, s));
 
-    fe::GemmParams p2{};
-    p2.bias = lw(c, l, T_B2);
-    p2.resid = c->h.p;
-    p2.ldr = d;
-    FE_RC(gemm(c, "gemm_item_ffn2_ln", fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, &c->xln, &c->h, s));
+      fe::GemmParams p2{};
+      p2.bias = lw(c, l, T_B2);
+      p2.resid = c->h.p;
+      p2.ldr = d;
+      FE_RC(gemm(c, "gemm_item_ffn2_ln", fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, &c->xln, &c->h, s));
+    }
   }
   // element projections of SeqEnc: H WKs | H WVs
   {
@@ -508,18 +541,22 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.ldr = 0;
     FE_RC(gemm(c, "gemm_seq_o_ln", fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, &c->cln, &c->c, s));
   }
-  {
-    fe::GemmParams p{};
-    p.bias = tw(c, T_B1S);
-    p.relu = 1;
-    FE_RC(gemm(c, "gemm_seq_ffn1", fe::EPI_STORE, c->cln, c->w1s, S, nullptr, p, &c->mids, nullptr, s));
-  }
-  {
-    fe::GemmParams p{};
-    p.bias = tw(c, T_B2S);
-    p.resid = c->c.p;
-    p.ldr = d;
-    FE_RC(gemm(c, "gemm_seq_ffn2_ln", fe::EPI_RESID_LN, c->mids, c->w2s, S, nullptr, p, &c->z, &c->c, s));
+  if (c->fused_ffn) {
+    FE_RC(ffn(c, "ffn_seq", c->cln, c->w1s, c->w2s, tw(c, T_B1S), tw(c, T_B2S), c->c, c->z, S, nullptr, s));
+  } else {
+    {
+      fe::GemmParams p{};
+      p.bias = tw(c, T_B1S);
+      p.relu = 1;
+      FE_RC(gemm(c, "gemm_seq_ffn1", fe::EPI_STORE, c->cln, c->w1s, S, nullptr, p, &c->mids, nullptr, s));
+    }
+    {
+      fe::GemmParams p{};
+      p.bias = tw(c, T_B2S);
+      p.resid = c->c.p;
+      p.ldr = d;
+      FE_RC(gemm(c, "gemm_seq_ffn2_ln", fe::EPI_RESID_LN, c->mids, c->w2s, S, nullptr, p, &c->z, &c->c, s));
+    }
   }
   // (a5) cross-sequence attention over the K sequence vectors of each request
   {
@@ -791,7 +828,8 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     return rc;
   };
   int rc = FE_OK;
-  if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess)
+  if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess ||
+      fe::ffn_prepare() != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "kernel attributes"));
   {
     size_t o = 0;
@@ -824,6 +862,11 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     if ((rc = make_weight(c, c->w2[l], d, F, 512)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->w2[l], lw(c, l, T_W2), F, d, 0)) != FE_OK) return fail(rc);
   }
+  c->fused_ffn = fe::ffn_supported(d, c->dpad, F, c->nb);
+  if (c->fused_ffn) {
+    for (int l = 0; l < Ly; ++l)
+      if ((rc = map_fused_w1(c->w1[l], c->nb > 1)) != FE_OK) return fail(rc);
+  }
   if ((rc = make_weight(c, c->kvs, 2 * d, d, 128)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->kvs, tw(c, T_WKS), d, d, 0)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->kvs, tw(c, T_WVS), d, d, d)) != FE_OK) return fail(rc);
@@ -831,6 +874,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if ((rc = fill_weight(c->os, tw(c, T_WOS), d, d, 0)) != FE_OK) return fail(rc);
   if ((rc = make_weight(c, c->w1s, F, d, 128)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w1s, tw(c, T_W1S), d, F, 0)) != FE_OK) return fail(rc);
+  if (c->fused_ffn && (rc = map_fused_w1(c->w1s, c->nb > 1)) != FE_OK) return fail(rc);
   if ((rc = make_weight(c, c->w2s, d, F, 512)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w2s, tw(c, T_W2S), F, d, 0)) != FE_OK) return fail(rc);
   if ((rc = make_weight(c, c->qkvx, 3 * d, d, 128)) != FE_OK) return fail(rc);

@@ -1,0 +1,432 @@
+// Fused position-wise FFN block of the evaluator (element layers of Section
+// 4.2 and the SeqEnc block of Section 4.3):
+//     x_out = x + ReLU(LN(x) W1 + b1) W2 + b2,   also LN(x_out)
+// for rows of width d <= 128, without writing the F-wide intermediate to
+// memory.  A persistent CTA walks 128-row tiles:
+//   warp 0 lane 0 : TMA producer -- the LN(x) tile (hi/lo, held for the whole
+//                   tile) and a ring of weight slots in consumption order
+//                   W1_0, W1_1, W2_0, W1_2, W2_1, ...
+//   warp 1 lane 0 : tcgen05.mma -- FFN1 chunk f (64 columns of F) into one
+//                   of two TMEM buffers, then FFN2 of chunk f-1 accumulating
+//                   all chunks into a d-column TMEM accumulator
+//   warps 2-9     : per chunk: bias + ReLU, split into hi/lo bf16, written to
+//                   a 128-byte-swizzled K-major shared tile that FFN2 reads
+//                   as its A operand; per tile: residual + b2 + LayerNorm,
+//                   stored with TMA tensor stores
+#include "fe_common.cuh"
+#include "fe_kernels.h"
+
+namespace fe {
+
+namespace {
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int FC = 64;                         // FFN columns per chunk
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
+constexpr uint32_t kAPlane = BM * BK * 2;      // 16 KB: 128 rows x 64 bf16
+constexpr uint32_t kMidPlane = BM * FC * 2;    // 16 KB
+constexpr uint32_t kStageOut = 4096;           // final-epilogue staging per warp
+constexpr size_t kSmemMaxBlock = 232448;
+
+struct FfnLayout {
+  uint32_t a_bytes, slot_bytes, w1_chunk, w2_chunk;
+  int ring;
+  size_t smem;
+};
+
+__host__ __device__ inline FfnLayout ffn_layout(int d, int d_pad, int nb) {
+  FfnLayout L;
+  L.a_bytes = (uint32_t)(d_pad / BK) * 2u * kAPlane;
+  L.w1_chunk = (uint32_t)nb * (uint32_t)(d_pad / BK) * (FC * BK * 2);  // [kb][plane][64 x 64]
+  L.w2_chunk = (uint32_t)nb * (uint32_t)d * (FC * 2);                  // [plane][d x 64]
+  L.slot_bytes = L.w1_chunk > L.w2_chunk ? L.w1_chunk : L.w2_chunk;
+  L.slot_bytes = (L.slot_bytes + 1023u) & ~1023u;
+  const size_t fixed = 1024 + L.a_bytes + 4 * kMidPlane + 256 + 4096 + kEpiWarps * kStageOut;
+  L.ring = fixed < kSmemMaxBlock ? (int)((kSmemMaxBlock - fixed) / L.slot_bytes) : 0;
+  if (L.ring > 4) L.ring = 4;
+  L.smem = fixed + (size_t)L.ring * L.slot_bytes;
+  return L;
+}
+
+__device__ __forceinline__ void mbar_arrive_one(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+}  // namespace
+
+__global__ void __launch_bounds__(kThreads, 1)
+    ffn_kernel(const __grid_constant__ CUtensorMap tA_h, const __grid_constant__ CUtensorMap tA_l,
+               const __grid_constant__ CUtensorMap tW1_h, const __grid_constant__ CUtensorMap tW1_l,
+               const __grid_constant__ CUtensorMap tW2_h, const __grid_constant__ CUtensorMap tW2_l,
+               const __grid_constant__ CUtensorMap tO_h, const __grid_constant__ CUtensorMap tO_l,
+               const __grid_constant__ CUtensorMap tO_x, const FfnParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_s = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
+  const int d = p.d, nb = p.nb;
+  const FfnLayout LY = ffn_layout(d, p.d_pad, nb);
+  const int nkb = p.d_pad / BK;
+  const int nf = p.F / FC;
+  uint8_t* sA = smem;
+  uint8_t* sW = sA + LY.a_bytes;
+  uint8_t* sMid = sW + (size_t)LY.ring * LY.slot_bytes;  // [buffer 2][plane 2][16 KB]
+  uint8_t* sStg = sMid + 4 * kMidPlane;                   // [epilogue warp][4 KB]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + kEpiWarps * kStageOut);
+  uint64_t* a_full = bars;
+  uint64_t* a_empty = bars + 1;
+  uint64_t* w_full = bars + 2;       // [4]
+  uint64_t* w_empty = bars + 6;      // [4]
+  uint64_t* acc1_full = bars + 10;   // [2]
+  uint64_t* acc1_empty = bars + 12;  // [2]
+  uint64_t* mid_full = bars + 14;    // [2]
+  uint64_t* mid_empty = bars + 16;   // [2]
+  uint64_t* acc2_full = bars + 18;
+  uint64_t* acc2_empty = bars + 19;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 20);
+  float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [parity][sum|var][half][128]
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(a_full, 1);
+    mbar_init(a_empty, 1);
+    for (int i = 0; i < 4; ++i) {
+      mbar_init(w_full + i, 1);
+      mbar_init(w_empty + i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(acc1_full + i, 1);
+      mbar_init(acc1_empty + i, kEpiWarps);
+      mbar_init(mid_full + i, 32 * kEpiWarps);
+      mbar_init(mid_empty + i, 1);
+    }
+    mbar_init(acc2_full, 1);
+    mbar_init(acc2_empty, kEpiWarps);
+    fence_mbar_init();
+    prefetch_tmap(&tA_h);
+    prefetch_tmap(&tW1_h);
+    prefetch_tmap(&tW2_h);
+  }
+  // TMEM: FFN1 chunk buffers at columns [0,64) and [64,128), FFN2 accumulator at [128, 128+d)
+  if (warp == 0) tmem_alloc(tmem_slot, 256);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
+  int rows_valid = p.rows;
+  if (p.rows_dev) rows_valid = min(*p.rows_dev, p.rows);
+  const int tiles = (rows_valid + BM - 1) / BM;
+  if ((int)blockIdx.x >= tiles) {
+    if (warp == 0) tmem_dealloc(tmem, 256);
+    return;
+  }
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      int tl = 0, ws = 0;
+      bool ok = true;
+      auto load_slot = [&](bool first, int f) -> bool {
+        const int slot = ws % LY.ring;
+        if (ws >= LY.ring && !mbar_wait_bounded(w_empty + slot, ((ws / LY.ring) - 1) & 1, p.status)) return false;
+        uint8_t* dst = sW + (size_t)slot * LY.slot_bytes;
+        if (first) {  // W1 rows [f*64, f*64+64), all k blocks
+          mbar_arrive_expect_tx(w_full + slot, LY.w1_chunk);
+          for (int kb = 0; kb < nkb; ++kb)
+            for (int q = 0; q < nb; ++q)
+              tma_load_2d(dst + (size_t)(kb * nb + q) * (FC * BK * 2), q ? &tW1_l : &tW1_h, kb * BK, f * FC,
+                          w_full + slot);
+        } else {  // W2 columns [f*64, f*64+64), all d rows
+          mbar_arrive_expect_tx(w_full + slot, LY.w2_chunk);
+          for (int q = 0; q < nb; ++q)
+            tma_load_2d(dst + (size_t)q * d * (FC * 2), q ? &tW2_l : &tW2_h, f * FC, 0, w_full + slot);
+        }
+        ++ws;
+        return true;
+      };
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+        if (tl > 0 && !mbar_wait_bounded(a_empty, (tl - 1) & 1, p.status)) break;
+        mbar_arrive_expect_tx(a_full, LY.a_bytes);
+        for (int kb = 0; kb < nkb; ++kb) {
+          tma_load_2d(sA + (size_t)(kb * 2) * kAPlane, &tA_h, kb * BK, t * BM, a_full);
+          tma_load_2d(sA + (size_t)(kb * 2 + 1) * kAPlane, &tA_l, kb * BK, t * BM, a_full);
+        }
+        for (int s = 0; s <= nf && ok; ++s) {
+          if (s < nf && !load_slot(true, s)) ok = false;
+          if (ok && s >= 1 && !load_slot(false, s - 1)) ok = false;
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const uint32_t idesc1 = umma_idesc_bf16(BM, FC);
+      const uint32_t idesc2 = umma_idesc_bf16(BM, d);
+      int tl = 0, ws = 0, gf = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+        if (!mbar_wait_bounded(a_full, tl & 1, p.status)) break;
+        tc_fence_after();
+        const int gf0 = gf;
+        for (int s = 0; s <= nf && ok; ++s) {
+          if (s < nf) {
+            // FFN1 chunk s -> acc1 buffer (gf0 + s) % 2
+            const int g = gf0 + s, b = g & 1;
+            if (g >= 2 && !mbar_wait_bounded(acc1_empty + b, ((g >> 1) - 1) & 1, p.status)) {
+              ok = false;
+              break;
+            }
+            const int slot = ws % LY.ring;
+            if (!mbar_wait_bounded(w_full + slot, (ws / LY.ring) & 1, p.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t a0 = smem_u32(sA), w0 = smem_u32(sW + (size_t)slot * LY.slot_bytes);
+            const uint32_t dst = tmem + (uint32_t)(b * FC);
+            for (int kb = 0; kb < nkb; ++kb)
+              for (int kk = 0; kk < BK / 16; ++kk)
+                for (int pr = 0; pr < 1 + nb; ++pr) {
+                  const uint32_t a = a0 + (uint32_t)(kb * 2 + (pr == 1 ? 1 : 0)) * kAPlane + (uint32_t)kk * 32;
+                  const uint32_t w = w0 + (uint32_t)(kb * nb + (pr == 2 ? 1 : 0)) * (FC * BK * 2) + (uint32_t)kk * 32;
+                  umma_bf16(dst, umma_desc_sw128(a), umma_desc_sw128(w), idesc1, (kb | kk | pr) != 0 ? 1u : 0u);
+                }
+            umma_commit(w_empty + slot);
+            umma_commit(acc1_full + b);
+            ++ws;
+            if (s == nf - 1) umma_commit(a_empty);  // every FFN1 of this tile issued
+          }
+          if (s >= 1) {
+            // FFN2 chunk s-1: acc2 += mid (s-1) . W2 chunk
+            const int g = gf0 + s - 1, b = g & 1;
+            if (s == 1 && tl > 0 && !mbar_wait_bounded(acc2_empty, (tl - 1) & 1, p.status)) {
+              ok = false;
+              break;
+            }
+            if (!mbar_wait_bounded(mid_full + b, (g >> 1) & 1, p.status)) {
+              ok = false;
+              break;
+            }
+            const int slot = ws % LY.ring;
+            if (!mbar_wait_bounded(w_full + slot, (ws / LY.ring) & 1, p.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t m0 = smem_u32(sMid + (size_t)(b * 2) * kMidPlane);
+            const uint32_t w0 = smem_u32(sW + (size_t)slot * LY.slot_bytes);
+            for (int kk = 0; kk < FC / 16; ++kk)
+              for (int pr = 0; pr < 1 + nb; ++pr) {
+                const uint32_t a = m0 + (pr == 1 ? kMidPlane : 0u) + (uint32_t)kk * 32;
+                const uint32_t w = w0 + (pr == 2 ? (uint32_t)d * (FC * 2) : 0u) + (uint32_t)kk * 32;
+                umma_bf16(tmem + 2 * FC, umma_desc_sw128(a), umma_desc_sw128(w), idesc2,
+                          (s > 1 || kk > 0 || pr > 0) ? 1u : 0u);
+              }
+            umma_commit(w_empty + slot);
+            umma_commit(mid_empty + b);
+            ++ws;
+            if (s == nf) umma_commit(acc2_full);
+          }
+        }
+        gf = gf0 + nf;
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..9) ----------------
+    const int ew = warp - 2, q = warp & 3, half = ew >> 2;
+    const int r = q * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    uint8_t* stg = sStg + (size_t)ew * kStageOut;
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory"); };
+    auto issue = [&](const CUtensorMap* m0p, const void* s0, const CUtensorMap* m1p, const void* s1, int col,
+                     int row) {
+      fence_async_shared();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_2d(m0p, s0, col, row);
+        if (m1p) tma_store_2d(m1p, s1, col, row);
+        bulk_commit();
+        bulk_wait_read0();  // the staging is reused right away
+      }
+      __syncwarp();
+    };
+    int tl = 0, gf = 0;
+    bool ok = true;
+    float xr[64];
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+      const int m0 = t * BM;
+      const int grow = m0 + r, srow = m0 + q * 32;
+      const bool valid = grow < rows_valid;
+      // residual row chunks for the final epilogue, loaded while the FFN runs
+      const float* rrow = p.resid + (size_t)grow * p.ldr;
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        const int c = 32 * half + 64 * ci;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4 qv = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (valid && c < d) qv = reinterpret_cast<const float4*>(rrow + c)[j];
+          xr[32 * ci + 4 * j] = qv.x;
+          xr[32 * ci + 4 * j + 1] = qv.y;
+          xr[32 * ci + 4 * j + 2] = qv.z;
+          xr[32 * ci + 4 * j + 3] = qv.w;
+        }
+      }
+      // ---- per chunk: mid = split(ReLU(acc1 + b1)) into the shared A tile of FFN2
+      for (int f = 0; f < nf; ++f, ++gf) {
+        const int b = gf & 1;
+        if (!mbar_wait_bounded(acc1_full + b, (gf >> 1) & 1, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        float v[32];
+        tmem_ld32(tmem + lane_off + (uint32_t)(b * FC + 32 * half), v);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_one(acc1_empty + b);
+        const float4* b4 = reinterpret_cast<const float4*>(p.b1 + f * FC + 32 * half);
+        uint32_t hi[16], lo[16];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float4 bb = __ldg(b4 + j);
+          split2(fmaxf(v[4 * j] + bb.x, 0.f), fmaxf(v[4 * j + 1] + bb.y, 0.f), hi[2 * j], lo[2 * j]);
+          split2(fmaxf(v[4 * j + 2] + bb.z, 0.f), fmaxf(v[4 * j + 3] + bb.w, 0.f), hi[2 * j + 1], lo[2 * j + 1]);
+        }
+        if (gf >= 2 && !mbar_wait_bounded(mid_empty + b, ((gf >> 1) - 1) & 1, p.status)) {
+          ok = false;
+          break;
+        }
+        uint8_t* mh = sMid + (size_t)(b * 2) * kMidPlane;
+        uint8_t* ml = mh + kMidPlane;
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+          const uint32_t off = (uint32_t)r * 128u + ((uint32_t)((4 * half + g) ^ (r & 7)) << 4);
+          *reinterpret_cast<uint4*>(mh + off) = make_uint4(hi[4 * g], hi[4 * g + 1], hi[4 * g + 2], hi[4 * g + 3]);
+          *reinterpret_cast<uint4*>(ml + off) = make_uint4(lo[4 * g], lo[4 * g + 1], lo[4 * g + 2], lo[4 * g + 3]);
+        }
+        fence_async_shared();
+        mbar_arrive_one(mid_full + b);
+      }
+      if (!ok) break;
+      // ---- final: x = resid + acc2 + b2, LayerNorm, stores
+      if (!mbar_wait_bounded(acc2_full, tl & 1, p.status)) break;
+      tc_fence_after();
+      float* red_sum = red + (size_t)(tl & 1) * 512;
+      float* red_var = red_sum + 256;
+      float sum = 0.f;
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        if (c < d) {
+          float v[32];
+          tmem_ld32(tmem + lane_off + (uint32_t)(2 * FC + c), v);
+          const float4* b4 = reinterpret_cast<const float4*>(p.b2 + c);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 bb = __ldg(b4 + j);
+            xr[32 * ci + 4 * j] += v[4 * j] + bb.x;
+            xr[32 * ci + 4 * j + 1] += v[4 * j + 1] + bb.y;
+            xr[32 * ci + 4 * j + 2] += v[4 * j + 2] + bb.z;
+            xr[32 * ci + 4 * j + 3] += v[4 * j + 3] + bb.w;
+          }
+#pragma unroll
+          for (int i = 0; i < 32; i += 4)
+            sum += (xr[32 * ci + i] + xr[32 * ci + i + 1]) + (xr[32 * ci + i + 2] + xr[32 * ci + i + 3]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_one(acc2_empty);  // accumulator read
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        if (c < d) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const uint32_t o = (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4);
+            *reinterpret_cast<float4*>(stg + o) =
+                make_float4(xr[32 * ci + 4 * j], xr[32 * ci + 4 * j + 1], xr[32 * ci + 4 * j + 2],
+                            xr[32 * ci + 4 * j + 3]);
+          }
+          issue(&tO_x, stg, nullptr, nullptr, c, srow);
+        }
+      }
+      red_sum[half * 128 + r] = sum;
+      pair_sync();
+      const float mean = (red_sum[r] + red_sum[128 + r]) / (float)d;
+      float var = 0.f;
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        if (32 * half + 64 * ci < d) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float dv = xr[32 * ci + i] - mean;
+            var = fmaf(dv, dv, var);
+          }
+        }
+      }
+      red_var[half * 128 + r] = var;
+      pair_sync();
+      const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)d + p.eps);
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        if (c < d) {
+          uint32_t hi[16], lo[16];
+#pragma unroll
+          for (int i = 0; i < 32; i += 2)
+            split2((xr[32 * ci + i] - mean) * rstd, (xr[32 * ci + i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
+            *reinterpret_cast<uint4*>(stg + o) = make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
+            *reinterpret_cast<uint4*>(stg + 2048 + o) =
+                make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
+          }
+          issue(&tO_h, stg, &tO_l, stg + 2048, c, srow);
+        }
+      }
+    }
+    if (lane == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, 256);
+}
+
+namespace {
+int g_ffn_sms = 0;
+}
+
+bool ffn_supported(int d, int d_pad, int F, int nb) {
+  if (d > 128 || d % 32 || F % FC || F < FC) return false;
+  const FfnLayout L = ffn_layout(d, d_pad, nb);
+  return L.ring >= 2 && L.smem <= kSmemMaxBlock;
+}
+
+cudaError_t ffn_prepare() {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_ffn_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(ffn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+  return e;
+}
+
+cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* w1_h,
+                       const CUtensorMap* w1_l, const CUtensorMap* w2_h, const CUtensorMap* w2_l,
+                       const CUtensorMap* o_h, const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p,
+                       cudaStream_t s) {
+  if (p.rows <= 0) return cudaSuccess;
+  const FfnLayout LY = ffn_layout(p.d, p.d_pad, p.nb);
+  const long long tiles = (p.rows + BM - 1) / BM;
+  long long grid = g_ffn_sms > 0 ? g_ffn_sms : 148;
+  if (grid > tiles) grid = tiles;
+  return launch_k(ffn_kernel, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *a_h, *a_l, *w1_h,
+                  p.nb > 1 ? *w1_l : *w1_h, *w2_h, p.nb > 1 ? *w2_l : *w2_h, *o_h, *o_l, *o_x, p);
+}
+
+}  // namespace fe

@@ -85,6 +85,31 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l,
                         const CUtensorMap* o_x, const GemmParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
+// Fused FFN block for rows of width d <= 128 (fe_ffn.cu):
+//   x_out = x + ReLU(LN(x) W1 + b1) W2 + b2, and LN(x_out)
+// A: LN(x) planes (64 x 128 boxes, 128-byte swizzle); W1^T [F, d_pad] planes
+// with 64 x 64 boxes; W2^T [d, F_pad] planes with 64 x d boxes; outputs
+// through the same store descriptors as the GEMM epilogue.
+// ---------------------------------------------------------------------------
+struct FfnParams {
+  int rows;             // row extent of the A descriptors
+  const int* rows_dev;  // when set: number of valid rows, read on the device
+  int d, d_pad, F, nb;
+  const float* b1;      // [F]
+  const float* b2;      // [d]
+  const float* resid;   // x rows
+  int ldr;
+  float eps;
+  int* status;
+};
+bool ffn_supported(int d, int d_pad, int F, int nb);
+cudaError_t ffn_prepare();
+cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* w1_h,
+                       const CUtensorMap* w1_l, const CUtensorMap* w2_h, const CUtensorMap* w2_l,
+                       const CUtensorMap* o_h, const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p,
+                       cudaStream_t s);
+
+// ---------------------------------------------------------------------------
 // Flash-style multi-head attention over request segments (tcgen05, split-bf16
 // operands).  Segment b: query rows [q_off(b), q_off(b) + q_cnt(b)), key and
 // value rows [b * kv_stride, b * kv_stride + kv_cnt).  Head h reads columns
