@@ -183,15 +183,15 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         const uint32_t q = smem_u32(sQ + qb * Cfg::kQBytes);
         const uint32_t k = smem_u32(sKV + ks * Cfg::kKVBytes);
         const uint32_t dst = tmem + (uint32_t)((gcc & 1) * CK);
-#pragma unroll 1
+        const uint64_t qh0 = desc_sw(q, Cfg::kSbo, Cfg::kSwz), ql0 = desc_sw(q + Cfg::kTile, Cfg::kSbo, Cfg::kSwz);
+        const uint64_t kh0 = desc_sw(k, Cfg::kSbo, Cfg::kSwz), kl0 = desc_sw(k + Cfg::kKVTile, Cfg::kSbo, Cfg::kSwz);
+#pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk) {
           // (Qh, Kh), (Ql, Kh), (Qh, Kl)
-          for (int pr = 0; pr < 3; ++pr) {
-            const uint32_t a = q + (pr == 1 ? Cfg::kTile : 0u) + (uint32_t)kk * 32;
-            const uint32_t bb = k + (pr == 2 ? Cfg::kKVTile : 0u) + (uint32_t)kk * 32;
-            umma_bf16(dst, desc_sw(a, Cfg::kSbo, Cfg::kSwz), desc_sw(bb, Cfg::kSbo, Cfg::kSwz), idesc_s,
-                      (kk | pr) != 0 ? 1u : 0u);
-          }
+          const uint64_t qh = desc_adv(qh0, kk * 32), kh = desc_adv(kh0, kk * 32);
+          umma_bf16(dst, qh, kh, idesc_s, kk != 0 ? 1u : 0u);
+          umma_bf16(dst, desc_adv(ql0, kk * 32), kh, idesc_s, 1u);
+          umma_bf16(dst, qh, desc_adv(kl0, kk * 32), idesc_s, 1u);
         }
         umma_commit(s_full + (gcc & 1));
         return true;
@@ -223,17 +223,17 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           const int ks = gc % Cfg::kKVStages;
           const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + 2 * Cfg::kKVTile);
           const uint32_t pp = smem_u32(sP);
-#pragma unroll 1
+          const uint64_t ph0 = desc_sw(pp, 1024, 2), pl0 = desc_sw(pp + (uint32_t)(CK / 64) * Cfg::kPBlock, 1024, 2);
+          const uint64_t vh0 = desc_sw(v, Cfg::kSbo, Cfg::kSwz), vl0 = desc_sw(v + Cfg::kKVTile, Cfg::kSbo, Cfg::kSwz);
+#pragma unroll
           for (int kk = 0; kk < CK / 16; ++kk) {
-            const uint32_t pa = pp + (uint32_t)(kk >> 2) * Cfg::kPBlock + (uint32_t)(kk & 3) * 32;
-            const uint32_t vb = v + (uint32_t)kk * 16 * Cfg::kRowBytes;
+            const uint32_t pa = (uint32_t)(kk >> 2) * Cfg::kPBlock + (uint32_t)(kk & 3) * 32;
+            const uint32_t vb = (uint32_t)kk * 16 * Cfg::kRowBytes;
             // (Ph, Vh), (Pl, Vh), (Ph, Vl)
-            for (int pr = 0; pr < 3; ++pr) {
-              const uint32_t a = pa + (pr == 1 ? (uint32_t)(CK / 64) * Cfg::kPBlock : 0u);
-              const uint32_t bb = vb + (pr == 2 ? Cfg::kKVTile : 0u);
-              umma_bf16(tmem + 2 * CK, desc_sw(a, 1024, 2), desc_sw(bb, Cfg::kSbo, Cfg::kSwz), idesc_pv,
-                        (kk | pr) != 0 ? 1u : 0u);
-            }
+            const uint64_t ph = desc_adv(ph0, pa), vh = desc_adv(vh0, vb);
+            umma_bf16(tmem + 2 * CK, ph, vh, idesc_pv, kk != 0 ? 1u : 0u);
+            umma_bf16(tmem + 2 * CK, desc_adv(pl0, pa), vh, idesc_pv, 1u);
+            umma_bf16(tmem + 2 * CK, ph, desc_adv(vl0, vb), idesc_pv, 1u);
           }
           umma_commit(pv_full);
           umma_commit(kv_empty + ks);

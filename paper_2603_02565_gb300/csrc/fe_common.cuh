@@ -165,6 +165,10 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
   return d;
 }
 
+// A descriptor advanced by `bytes` (a multiple of 16) inside the same tile:
+// the start-address field counts 16-byte units and never carries here.
+__device__ __forceinline__ uint64_t desc_adv(uint64_t desc, uint32_t bytes) { return desc + (uint64_t)(bytes >> 4); }
+
 // Instruction descriptor: kind::f16, A = B = bf16, D = f32, both K-major.
 __device__ __forceinline__ uint32_t umma_idesc_bf16(int M, int N) {
   return (1u << 4)                       // D format f32

@@ -7,8 +7,9 @@
 //                   tile) and a ring of weight slots in consumption order
 //                   W1_0, W1_1, W2_0, W1_2, W2_1, ...
 //   warp 1 lane 0 : tcgen05.mma -- FFN1 chunk f (64 columns of F) into one
-//                   of two TMEM buffers, then FFN2 of chunk f-1 accumulating
-//                   all chunks into a d-column TMEM accumulator
+//                   of four TMEM buffers, two chunks ahead of FFN2 of chunk
+//                   f-2, which accumulates all chunks into a d-column TMEM
+//                   accumulator
 //   warps 2-9     : per chunk: bias + ReLU, split into hi/lo bf16, written to
 //                   a 128-byte-swizzled K-major shared tile that FFN2 reads
 //                   as its A operand; per tile: residual + b2 + LayerNorm,
@@ -22,6 +23,8 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int FC = 64;                         // FFN columns per chunk
+constexpr int NA1 = 4;                         // TMEM buffers for FFN1 chunks
+constexpr int LA = 2;                          // FFN1 chunks issued ahead of the FFN2 that consumes them
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
 constexpr uint32_t kAPlane = BM * BK * 2;      // 16 KB: 128 rows x 64 bf16
@@ -76,13 +79,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* a_empty = bars + 1;
   uint64_t* w_full = bars + 2;       // [4]
   uint64_t* w_empty = bars + 6;      // [4]
-  uint64_t* acc1_full = bars + 10;   // [2]
-  uint64_t* acc1_empty = bars + 12;  // [2]
-  uint64_t* mid_full = bars + 14;    // [2]
-  uint64_t* mid_empty = bars + 16;   // [2]
-  uint64_t* acc2_full = bars + 18;
-  uint64_t* acc2_empty = bars + 19;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 20);
+  uint64_t* acc1_full = bars + 10;   // [4]
+  uint64_t* acc1_empty = bars + 14;  // [4]
+  uint64_t* mid_full = bars + 18;    // [2]
+  uint64_t* mid_empty = bars + 20;   // [2]
+  uint64_t* acc2_full = bars + 22;
+  uint64_t* acc2_empty = bars + 23;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [parity][sum|var][half][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -93,9 +96,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(w_full + i, 1);
       mbar_init(w_empty + i, 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < NA1; ++i) {
       mbar_init(acc1_full + i, 1);
       mbar_init(acc1_empty + i, kEpiWarps);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(mid_full + i, 32 * kEpiWarps);
       mbar_init(mid_empty + i, 1);
     }
@@ -106,8 +111,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tW1_h);
     prefetch_tmap(&tW2_h);
   }
-  // TMEM: FFN1 chunk buffers at columns [0,64) and [64,128), FFN2 accumulator at [128, 128+d)
-  if (warp == 0) tmem_alloc(tmem_slot, 256);
+  // TMEM: FFN1 chunk buffers at columns [64 i, 64 i + 64), i < 4; FFN2 accumulator at [256, 256+d)
+  if (warp == 0) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -118,7 +123,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (p.rows_dev) rows_valid = min(*p.rows_dev, p.rows);
   const int tiles = (rows_valid + BM - 1) / BM;
   if ((int)blockIdx.x >= tiles) {
-    if (warp == 0) tmem_dealloc(tmem, 256);
+    if (warp == 0) tmem_dealloc(tmem, 512);
     return;
   }
 
@@ -152,9 +157,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_2d(sA + (size_t)(kb * 2) * kAPlane, &tA_h, kb * BK, t * BM, a_full);
           tma_load_2d(sA + (size_t)(kb * 2 + 1) * kAPlane, &tA_l, kb * BK, t * BM, a_full);
         }
-        for (int s = 0; s <= nf && ok; ++s) {
+        for (int s = 0; s < nf + LA && ok; ++s) {
           if (s < nf && !load_slot(true, s)) ok = false;
-          if (ok && s >= 1 && !load_slot(false, s - 1)) ok = false;
+          if (ok && s >= LA && !load_slot(false, s - LA)) ok = false;
         }
       }
     }
@@ -169,11 +174,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait_bounded(a_full, tl & 1, p.status)) break;
         tc_fence_after();
         const int gf0 = gf;
-        for (int s = 0; s <= nf && ok; ++s) {
+        for (int s = 0; s < nf + LA && ok; ++s) {
           if (s < nf) {
-            // FFN1 chunk s -> acc1 buffer (gf0 + s) % 2
-            const int g = gf0 + s, b = g & 1;
-            if (g >= 2 && !mbar_wait_bounded(acc1_empty + b, ((g >> 1) - 1) & 1, p.status)) {
+            // FFN1 chunk s -> acc1 buffer (gf0 + s) % NA1
+            const int g = gf0 + s, b = g % NA1;
+            if (g >= NA1 && !mbar_wait_bounded(acc1_empty + b, ((g / NA1) - 1) & 1, p.status)) {
               ok = false;
               break;
             }
@@ -183,24 +188,28 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            const uint32_t a0 = smem_u32(sA), w0 = smem_u32(sW + (size_t)slot * LY.slot_bytes);
             const uint32_t dst = tmem + (uint32_t)(b * FC);
-            for (int kb = 0; kb < nkb; ++kb)
-              for (int kk = 0; kk < BK / 16; ++kk)
-                for (int pr = 0; pr < 1 + nb; ++pr) {
-                  const uint32_t a = a0 + (uint32_t)(kb * 2 + (pr == 1 ? 1 : 0)) * kAPlane + (uint32_t)kk * 32;
-                  const uint32_t w = w0 + (uint32_t)(kb * nb + (pr == 2 ? 1 : 0)) * (FC * BK * 2) + (uint32_t)kk * 32;
-                  umma_bf16(dst, umma_desc_sw128(a), umma_desc_sw128(w), idesc1, (kb | kk | pr) != 0 ? 1u : 0u);
-                }
+            const uint64_t a0 = umma_desc_sw128(smem_u32(sA));
+            const uint64_t w0 = umma_desc_sw128(smem_u32(sW + (size_t)slot * LY.slot_bytes));
+            for (int kb = 0; kb < nkb; ++kb) {
+#pragma unroll
+              for (int kk = 0; kk < BK / 16; ++kk) {
+                const uint64_t ah = desc_adv(a0, (uint32_t)(kb * 2) * kAPlane + kk * 32);
+                const uint64_t wh = desc_adv(w0, (uint32_t)(kb * nb) * (FC * BK * 2) + kk * 32);
+                umma_bf16(dst, ah, wh, idesc1, (kb | kk) != 0 ? 1u : 0u);
+                umma_bf16(dst, desc_adv(ah, kAPlane), wh, idesc1, 1u);
+                if (nb > 1) umma_bf16(dst, ah, desc_adv(wh, FC * BK * 2), idesc1, 1u);
+              }
+            }
             umma_commit(w_empty + slot);
             umma_commit(acc1_full + b);
             ++ws;
             if (s == nf - 1) umma_commit(a_empty);  // every FFN1 of this tile issued
           }
-          if (s >= 1) {
-            // FFN2 chunk s-1: acc2 += mid (s-1) . W2 chunk
-            const int g = gf0 + s - 1, b = g & 1;
-            if (s == 1 && tl > 0 && !mbar_wait_bounded(acc2_empty, (tl - 1) & 1, p.status)) {
+          if (s >= LA) {
+            // FFN2 chunk c = s - LA: acc2 += mid(c) . W2 chunk c
+            const int c = s - LA, g = gf0 + c, b = g & 1;
+            if (c == 0 && tl > 0 && !mbar_wait_bounded(acc2_empty, (tl - 1) & 1, p.status)) {
               ok = false;
               break;
             }
@@ -214,19 +223,19 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            const uint32_t m0 = smem_u32(sMid + (size_t)(b * 2) * kMidPlane);
-            const uint32_t w0 = smem_u32(sW + (size_t)slot * LY.slot_bytes);
-            for (int kk = 0; kk < FC / 16; ++kk)
-              for (int pr = 0; pr < 1 + nb; ++pr) {
-                const uint32_t a = m0 + (pr == 1 ? kMidPlane : 0u) + (uint32_t)kk * 32;
-                const uint32_t w = w0 + (pr == 2 ? (uint32_t)d * (FC * 2) : 0u) + (uint32_t)kk * 32;
-                umma_bf16(tmem + 2 * FC, umma_desc_sw128(a), umma_desc_sw128(w), idesc2,
-                          (s > 1 || kk > 0 || pr > 0) ? 1u : 0u);
-              }
+            const uint64_t m0 = umma_desc_sw128(smem_u32(sMid + (size_t)(b * 2) * kMidPlane));
+            const uint64_t w0 = umma_desc_sw128(smem_u32(sW + (size_t)slot * LY.slot_bytes));
+#pragma unroll
+            for (int kk = 0; kk < FC / 16; ++kk) {
+              const uint64_t mh = desc_adv(m0, kk * 32), wh = desc_adv(w0, kk * 32);
+              umma_bf16(tmem + NA1 * FC, mh, wh, idesc2, (c > 0 || kk > 0) ? 1u : 0u);
+              umma_bf16(tmem + NA1 * FC, desc_adv(mh, kMidPlane), wh, idesc2, 1u);
+              if (nb > 1) umma_bf16(tmem + NA1 * FC, mh, desc_adv(wh, (uint32_t)d * (FC * 2)), idesc2, 1u);
+            }
             umma_commit(w_empty + slot);
             umma_commit(mid_empty + b);
             ++ws;
-            if (s == nf) umma_commit(acc2_full);
+            if (c == nf - 1) umma_commit(acc2_full);
           }
         }
         gf = gf0 + nf;
@@ -275,17 +284,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // ---- per chunk: mid = split(ReLU(acc1 + b1)) into the shared A tile of FFN2
       for (int f = 0; f < nf; ++f, ++gf) {
-        const int b = gf & 1;
-        if (!mbar_wait_bounded(acc1_full + b, (gf >> 1) & 1, p.status)) {
+        const int ba = gf % NA1, b = gf & 1;
+        if (!mbar_wait_bounded(acc1_full + ba, (gf / NA1) & 1, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
         float v[32];
-        tmem_ld32(tmem + lane_off + (uint32_t)(b * FC + 32 * half), v);
+        tmem_ld32(tmem + lane_off + (uint32_t)(ba * FC + 32 * half), v);
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_one(acc1_empty + b);
+        if (lane == 0) mbar_arrive_one(acc1_empty + ba);
         const float4* b4 = reinterpret_cast<const float4*>(p.b1 + f * FC + 32 * half);
         uint32_t hi[16], lo[16];
 #pragma unroll
@@ -321,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int c = 32 * half + 64 * ci;
         if (c < d) {
           float v[32];
-          tmem_ld32(tmem + lane_off + (uint32_t)(2 * FC + c), v);
+          tmem_ld32(tmem + lane_off + (uint32_t)(NA1 * FC + c), v);
           const float4* b4 = reinterpret_cast<const float4*>(p.b2 + c);
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -394,7 +403,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) tmem_dealloc(tmem, 256);
+  if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
 namespace {

@@ -162,17 +162,19 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
           const uint32_t st = smem_u32(smem + (size_t)s * stage_bytes);
-#pragma unroll 1
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            // (A_hi, W_hi), (A_lo, W_hi), (A_hi, W_lo)
-            for (int pr = 0; pr < 1 + nb; ++pr) {
-              const uint32_t a = st + (pr == 1 ? kATile : 0u) + (uint32_t)kk * 32;
-              const uint32_t b = st + 2 * kATile + (pr == 2 ? b_bytes : 0u) + (uint32_t)kk * 32;
-              const uint64_t ad = umma_desc_sw128(a);
-              for (int h = 0; h < BN; h += 256) {
-                const uint64_t bd = umma_desc_sw128(b + (uint32_t)h * BK * 2);
-                umma_bf16(dst + (uint32_t)h, ad, bd, idesc, (kb | kk | pr) != 0 ? 1u : 0u);
-              }
+          // descriptors built once per stage; the k steps only add 32-byte offsets
+          const uint64_t ah0 = umma_desc_sw128(st), al0 = umma_desc_sw128(st + kATile);
+          const uint64_t bh0 = umma_desc_sw128(st + 2 * kATile), bl0 = umma_desc_sw128(st + 2 * kATile + b_bytes);
+          for (int h = 0; h < BN; h += 256) {
+            const uint32_t hb = (uint32_t)h * BK * 2;
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+              // (A_hi, W_hi), (A_lo, W_hi), (A_hi, W_lo)
+              const uint64_t ah = desc_adv(ah0, kk * 32), al = desc_adv(al0, kk * 32);
+              const uint64_t bh = desc_adv(bh0, hb + kk * 32);
+              umma_bf16(dst + (uint32_t)h, ah, bh, idesc, (kb | kk) != 0 ? 1u : 0u);
+              umma_bf16(dst + (uint32_t)h, al, bh, idesc, 1u);
+              if (nb > 1) umma_bf16(dst + (uint32_t)h, ah, desc_adv(bl0, hb + kk * 32), idesc, 1u);
             }
           }
           umma_commit(empty + s);  // frees this stage once its MMAs complete
