@@ -269,66 +269,88 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       float o[DO];
 #pragma unroll
       for (int i = 0; i < DO; ++i) o[i] = 0.f;
+      // a warp whose 32 query rows all lie past the segment's end only keeps
+      // the barrier protocol; those rows of P and of the output are never used
+      const bool active = q0 + q4 * 32 < qcnt;
       for (int j = 0; j < nch; ++j, ++gc) {
         if (!mbar_wait_bounded(s_full + (gc & 1), (gc >> 1) & 1, p.status)) {
           ok = false;
           break;
         }
-        tc_fence_after();
-        float v[64];
-        tmem_ld64(tmem + lane_off + (uint32_t)((gc & 1) * CK + half * KW), v);
-        const int kvalid = p.kv_cnt - j * CK - half * KW;  // valid keys among this warp's 64
-        float mx = -INFINITY;
+        float corr = 1.f;
+        if (active) {
+          tc_fence_after();
+          float v[64];
+          tmem_ld64(tmem + lane_off + (uint32_t)((gc & 1) * CK + half * KW), v);
+          const int kvalid = p.kv_cnt - j * CK - half * KW;  // valid keys among this warp's 64
+          float mx = -INFINITY;
+          if (kvalid >= 64) {
 #pragma unroll
-        for (int i = 0; i < 64; ++i) {
-          v[i] *= p.scale_log2;
-          if (i < kvalid) mx = fmaxf(mx, v[i]);
-        }
-        if (Cfg::kHalves == 2) {
-          float* rm = red_max + (gc & 1) * 256;
-          rm[half * 128 + r] = mx;
-          pair_sync();
-          mx = fmaxf(rm[r], rm[128 + r]);
-        }
-        const float mn = fmaxf(m, mx);
-        const float corr = ex2_approx(m - mn);
-        m = mn;
-        // P = 2^(s - m) as split pairs in the 128-byte-swizzled K-major tile (key block = half)
-        float sum = 0.f;
+            for (int i = 0; i < 64; ++i) mx = fmaxf(mx, v[i]);
+          } else {
 #pragma unroll
-        for (int g = 0; g < 8; ++g) {
-          uint32_t hi[4], lo[4];
-#pragma unroll
-          for (int i = 0; i < 8; i += 2) {
-            const int k = 8 * g + i;
-            const float p0 = (k < kvalid) ? ex2_approx(v[k] - mn) : 0.f;
-            const float p1 = (k + 1 < kvalid) ? ex2_approx(v[k + 1] - mn) : 0.f;
-            sum += p0 + p1;
-            split2(p0, p1, hi[i / 2], lo[i / 2]);
+            for (int i = 0; i < 64; ++i)
+              if (i < kvalid) mx = fmaxf(mx, v[i]);
           }
-          const uint32_t off = (uint32_t)r * 128u + (((uint32_t)g ^ (uint32_t)(r & 7)) << 4);
-          *reinterpret_cast<uint4*>(pH + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-          *reinterpret_cast<uint4*>(pL + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+          mx *= p.scale_log2;
+          if (Cfg::kHalves == 2) {
+            float* rm = red_max + (gc & 1) * 256;
+            rm[half * 128 + r] = mx;
+            pair_sync();
+            mx = fmaxf(rm[r], rm[128 + r]);
+          }
+          const float mn = fmaxf(m, mx);
+          corr = ex2_approx(m - mn);
+          m = mn;
+          // P = 2^(s * scale - m) as split pairs in the 128-byte-swizzled K-major
+          // tile (key block = half); keys past kv_cnt get 0
+          const float sc = p.scale_log2, nm = -mn;
+          float sum = 0.f;
+          auto emit = [&](auto full) {
+#pragma unroll
+            for (int g = 0; g < 8; ++g) {
+              uint32_t hi[4], lo[4];
+#pragma unroll
+              for (int i = 0; i < 8; i += 2) {
+                const int k = 8 * g + i;
+                float p0 = ex2_approx(fmaf(v[k], sc, nm));
+                float p1 = ex2_approx(fmaf(v[k + 1], sc, nm));
+                if (!decltype(full)::value) {
+                  p0 = k < kvalid ? p0 : 0.f;
+                  p1 = k + 1 < kvalid ? p1 : 0.f;
+                }
+                sum += p0 + p1;
+                split2_trunc(p0, p1, hi[i / 2], lo[i / 2]);
+              }
+              const uint32_t off = (uint32_t)r * 128u + (((uint32_t)g ^ (uint32_t)(r & 7)) << 4);
+              *reinterpret_cast<uint4*>(pH + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+              *reinterpret_cast<uint4*>(pL + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            }
+          };
+          if (kvalid >= 64) emit(std::true_type{});
+          else emit(std::false_type{});
+          l = l * corr + sum;
+          fence_async_shared();
+          tc_fence_before();
         }
-        l = l * corr + sum;
-        fence_async_shared();
-        tc_fence_before();
         mbar_arrive1(p_full);
         // fold this chunk's P V into this warp's output columns
         if (!mbar_wait_bounded(pv_full, gc & 1, p.status)) {
           ok = false;
           break;
         }
-        tc_fence_after();
-        float pv[DO];
-        if (DO == 16) {
-          tmem_ld16(tmem + lane_off + (uint32_t)(2 * CK + half * DO), pv);
-        } else {
+        if (active) {
+          tc_fence_after();
+          float pv[DO];
+          if (DO == 16) {
+            tmem_ld16(tmem + lane_off + (uint32_t)(2 * CK + half * DO), pv);
+          } else {
 #pragma unroll
-          for (int c = 0; c < DO; c += 32) tmem_ld32(tmem + lane_off + (uint32_t)(2 * CK + half * DO + c), pv + c);
+            for (int c = 0; c < DO; c += 32) tmem_ld32(tmem + lane_off + (uint32_t)(2 * CK + half * DO + c), pv + c);
+          }
+#pragma unroll
+          for (int i = 0; i < DO; ++i) o[i] = o[i] * corr + pv[i];
         }
-#pragma unroll
-        for (int i = 0; i < DO; ++i) o[i] = o[i] * corr + pv[i];
       }
       if (!ok) break;
       // row sum over both halves, then O / l as a split pair

@@ -6,6 +6,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <type_traits>
 
 #include "fe.h"
 #include "fe_kernels.h"
@@ -35,6 +36,18 @@ __device__ __forceinline__ void split2(float x0, float x1, uint32_t& hi, uint32_
   __nv_bfloat162 l = __floats2bfloat162_rn(x0 - __uint_as_float(hu << 16), x1 - __uint_as_float(hu & 0xFFFF0000u));
   hi = hu;
   lo = *reinterpret_cast<uint32_t*>(&l);
+}
+
+// Split pair by truncation, for on-chip intermediates (softmax P, the FFN
+// hidden activation): hi keeps the top 16 bits of x, r = x - hi is exact in
+// fp32, lo keeps the top 16 bits of r, so |x - hi - lo| < 2^-14 |x|.  Byte
+// permutes and two subtractions, no conversion instructions.
+__device__ __forceinline__ void split2_trunc(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const uint32_t u0 = __float_as_uint(x0), u1 = __float_as_uint(x1);
+  hi = __byte_perm(u0, u1, 0x7632);
+  const float r0 = x0 - __uint_as_float(u0 & 0xFFFF0000u);
+  const float r1 = x1 - __uint_as_float(u1 & 0xFFFF0000u);
+  lo = __byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x7632);
 }
 
 __device__ __forceinline__ float bf16lo_f(uint32_t v) { return __uint_as_float(v << 16); }

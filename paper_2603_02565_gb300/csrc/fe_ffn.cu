@@ -300,8 +300,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const float4 bb = __ldg(b4 + j);
-          split2(fmaxf(v[4 * j] + bb.x, 0.f), fmaxf(v[4 * j + 1] + bb.y, 0.f), hi[2 * j], lo[2 * j]);
-          split2(fmaxf(v[4 * j + 2] + bb.z, 0.f), fmaxf(v[4 * j + 3] + bb.w, 0.f), hi[2 * j + 1], lo[2 * j + 1]);
+          split2_trunc(fmaxf(v[4 * j] + bb.x, 0.f), fmaxf(v[4 * j + 1] + bb.y, 0.f), hi[2 * j], lo[2 * j]);
+          split2_trunc(fmaxf(v[4 * j + 2] + bb.z, 0.f), fmaxf(v[4 * j + 3] + bb.w, 0.f), hi[2 * j + 1], lo[2 * j + 1]);
         }
         if (gf >= 2 && !mbar_wait_bounded(mid_empty + b, ((gf >> 1) - 1) & 1, p.status)) {
           ok = false;
