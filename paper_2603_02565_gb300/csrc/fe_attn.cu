@@ -9,15 +9,18 @@
 // Persistent CTAs walk units (segment b, head h, 128-row query tile).  Per
 // unit the keys stream in chunks of CK (64 for d_h = 32, 128 for d_h = 64):
 //   warp 0 lane 0 : TMA producer -- Q tile (two buffers, one per unit in
-//                   flight) and K/V chunks of CK keys (two stages)
-//   warp 1 lane 0 : tcgen05.mma -- S = Q K^T into one of two TMEM tiles
-//                   (S_{j+1} overlaps the softmax of chunk j), then
-//                   PV = P V into a third TMEM region
+//                   flight) and K/V chunks of CK keys (4 stages for d_h = 32,
+//                   2 for d_h = 64)
+//   warp 1 lane 0 : tcgen05.mma -- S_j = Q K_j^T into TMEM tile j % 2, then
+//                   PV_j = P_j V_j with P_j read from that same TMEM tile
+//                   into PV buffer j % 2
 //   warps 2..     : online softmax from TMEM, one query row per lane; with
 //                   d_h = 64, warps w and w+4 share TMEM lane quadrant w % 4
 //                   and each take half of the chunk's keys and half of the
-//                   output columns; P is written to shared memory as a split
-//                   pair and the running output is rescaled in registers
+//                   output columns.  P_j is written back over S_j as split
+//                   bf16 pairs; PV_{j-1} is folded into the register output
+//                   after P_j is handed over, so the softmax never waits for
+//                   the PV product of the chunk it has just finished
 // Operands are split pairs (hi + lo bf16): S = Qh Kh + Ql Kh + Qh Kl and
 // PV = Ph Vh + Pl Vh + Ph Vl, fp32 accumulation; softmax in fp32.
 #include "fe_common.cuh"
@@ -38,7 +41,8 @@ struct AttnCfg {
   static constexpr int kHalves = kSoftmaxWarps / 4;              // warps sharing one lane quadrant
   static constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
   static constexpr int kCtasPerSM = DH == 32 ? 2 : 1;
-  static constexpr uint32_t kTmemCols = DH == 32 ? 256 : 512;  // 2 S tiles + PV
+  // TMEM: S/P tiles at [0, CK) and [CK, 2CK), PV buffers at [2CK, 2CK + 2DH)
+  static constexpr uint32_t kTmemCols = DH == 32 ? 256 : 512;
   static constexpr uint32_t kRowBytes = DH * 2;                 // one row of a Q/K/V tile
   static constexpr uint32_t kTile = 128 * kRowBytes;            // Q tile: 128 rows, one plane
   static constexpr uint32_t kKVTile = CK * kRowBytes;           // K or V chunk: CK rows, one plane
@@ -46,11 +50,9 @@ struct AttnCfg {
   static constexpr uint32_t kSbo = 8 * kRowBytes;               // 8-row swizzle atom
   static constexpr uint32_t kQBytes = 2 * kTile;                // hi + lo
   static constexpr uint32_t kKVBytes = 4 * kKVTile;             // Kh Kl Vh Vl
-  static constexpr uint32_t kPBlock = 128 * 128;                // 128 rows x 64 keys x 2 B
-  static constexpr uint32_t kPBytes = 2 * (CK / 64) * kPBlock;  // 2 planes x key blocks
-  static constexpr int kKVStages = DH == 32 ? 2 : 1;
+  static constexpr int kKVStages = DH == 32 ? 4 : 2;
   static constexpr uint32_t kRed = 2 * 2 * 2 * 128 * 4;       // [max|sum][parity][half][row]
-  static constexpr size_t kSmem = 1024 + 2 * kQBytes + kKVStages * kKVBytes + kPBytes + 256 + kRed;
+  static constexpr size_t kSmem = 1024 + 2 * kQBytes + kKVStages * kKVBytes + 256 + kRed;
 };
 
 __device__ __forceinline__ uint64_t desc_sw(uint32_t saddr, uint32_t sbo, uint32_t swz) {
@@ -82,16 +84,15 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
   uint8_t* sQ = smem;                                   // [2 buffers][hi, lo]
   uint8_t* sKV = sQ + 2 * Cfg::kQBytes;                 // [stages][Kh, Kl, Vh, Vl]
-  uint8_t* sP = sKV + Cfg::kKVStages * Cfg::kKVBytes;   // [hi, lo][key block 0, 1]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + Cfg::kPBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + Cfg::kKVStages * Cfg::kKVBytes);
   uint64_t* q_full = bars;        // [2]
   uint64_t* q_empty = bars + 2;   // [2]
-  uint64_t* kv_full = bars + 4;   // [2]
-  uint64_t* kv_empty = bars + 6;  // [2]
-  uint64_t* s_full = bars + 8;    // [2]
-  uint64_t* p_full = bars + 10;
-  uint64_t* pv_full = bars + 11;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  uint64_t* kv_full = bars + 4;   // [stages]
+  uint64_t* kv_empty = bars + 8;  // [stages]
+  uint64_t* s_full = bars + 12;   // [2] S_j complete in TMEM tile j % 2
+  uint64_t* p_full = bars + 14;   // [2] P_j written over S_j
+  uint64_t* pv_full = bars + 16;  // [2] PV_j complete in PV buffer j % 2
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // row-statistic exchange
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -104,12 +105,14 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     for (int i = 0; i < 2; ++i) {
       mbar_init(q_full + i, 1);
       mbar_init(q_empty + i, 1);
+      mbar_init(s_full + i, 1);
+      mbar_init(p_full + i, 32 * Cfg::kSoftmaxWarps);
+      mbar_init(pv_full + i, 1);
+    }
+    for (int i = 0; i < Cfg::kKVStages; ++i) {
       mbar_init(kv_full + i, 1);
       mbar_init(kv_empty + i, 1);
-      mbar_init(s_full + i, 1);
     }
-    mbar_init(p_full, 32 * Cfg::kSoftmaxWarps);
-    mbar_init(pv_full, 1);
     fence_mbar_init();
     prefetch_tmap(&tQh);
     prefetch_tmap(&tKh);
@@ -119,7 +122,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *tmem_slot;  // S tiles at columns [0,CK) and [CK,2CK), PV at [2CK, 2CK+DH)
+  const uint32_t tmem = *tmem_slot;
   // the set-up above reads nothing written by earlier kernels; from here on
   // the segment offsets, counts and operands are
   pdl_trigger();
@@ -175,8 +178,10 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       const uint32_t idesc_pv = umma_idesc_bf16(BQ, DH) | (1u << 16);  // B (V) is MN-major
       int ui = 0, gc = 0;
       bool ok = true;
-      // S = Q K^T of global chunk gcc, the unit's Q in buffer qb
+      // S = Q K^T of global chunk gcc into TMEM tile gcc % 2, the unit's Q in buffer qb
       auto issue_s = [&](int qb, int gcc) -> bool {
+        // the tile is free once PV_{gcc-2}, which reads P_{gcc-2} from it, has completed
+        if (gcc >= 2 && !mbar_wait_bounded(pv_full + (gcc & 1), ((gcc - 2) >> 1) & 1, p.status)) return false;
         const int ks = gcc % Cfg::kKVStages;
         if (!mbar_wait_bounded(kv_full + ks, (gcc / Cfg::kKVStages) & 1, p.status)) return false;
         tc_fence_after();
@@ -203,44 +208,36 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         const int qb = ui & 1;
         if (!mbar_wait_bounded(q_full + qb, (ui >> 1) & 1, p.status)) break;
         for (int j = 0; j < nch; ++j, ++gc) {
-          if (j == 0 && !issue_s(qb, gc)) {
-            ok = false;
-            break;
-          }
-          // with two K/V stages S_{j+1} overlaps the softmax of chunk j; with one
-          // stage chunk j+1 can only load after PV_j, so S_{j+1} follows PV_j
-          if (Cfg::kKVStages == 2 && j + 1 < nch && !issue_s(qb, gc + 1)) {
+          // S_{j+1} is issued ahead so that it overlaps the softmax of chunk j
+          if ((j == 0 && !issue_s(qb, gc)) || (j + 1 < nch && !issue_s(qb, gc + 1))) {
             ok = false;
             break;
           }
           if (j + 1 == nch) umma_commit(q_empty + qb);  // every S of this unit issued: Q buffer frees on completion
-          // PV = P V once the softmax has written P for this chunk
-          if (!mbar_wait_bounded(p_full, gc & 1, p.status)) {
+          if (!mbar_wait_bounded(p_full + (gc & 1), (gc >> 1) & 1, p.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
+          // PV_j: A = P_j from TMEM tile j % 2, where each key block of 64 holds
+          // its hi plane in 32 columns followed by its lo plane in 32 columns
           const int ks = gc % Cfg::kKVStages;
           const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + 2 * Cfg::kKVTile);
-          const uint32_t pp = smem_u32(sP);
-          const uint64_t ph0 = desc_sw(pp, 1024, 2), pl0 = desc_sw(pp + (uint32_t)(CK / 64) * Cfg::kPBlock, 1024, 2);
+          const uint32_t pt = tmem + (uint32_t)((gc & 1) * CK);
+          const uint32_t dst = tmem + (uint32_t)(2 * CK + (gc & 1) * DH);
           const uint64_t vh0 = desc_sw(v, Cfg::kSbo, Cfg::kSwz), vl0 = desc_sw(v + Cfg::kKVTile, Cfg::kSbo, Cfg::kSwz);
 #pragma unroll
           for (int kk = 0; kk < CK / 16; ++kk) {
-            const uint32_t pa = (uint32_t)(kk >> 2) * Cfg::kPBlock + (uint32_t)(kk & 3) * 32;
+            const uint32_t ph = pt + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8), pl = ph + 32;
             const uint32_t vb = (uint32_t)kk * 16 * Cfg::kRowBytes;
             // (Ph, Vh), (Pl, Vh), (Ph, Vl)
-            const uint64_t ph = desc_adv(ph0, pa), vh = desc_adv(vh0, vb);
-            umma_bf16(tmem + 2 * CK, ph, vh, idesc_pv, kk != 0 ? 1u : 0u);
-            umma_bf16(tmem + 2 * CK, desc_adv(pl0, pa), vh, idesc_pv, 1u);
-            umma_bf16(tmem + 2 * CK, ph, desc_adv(vl0, vb), idesc_pv, 1u);
+            const uint64_t vh = desc_adv(vh0, vb);
+            umma_bf16_tmem_a(dst, ph, vh, idesc_pv, kk != 0 ? 1u : 0u);
+            umma_bf16_tmem_a(dst, pl, vh, idesc_pv, 1u);
+            umma_bf16_tmem_a(dst, ph, desc_adv(vl0, vb), idesc_pv, 1u);
           }
-          umma_commit(pv_full);
+          umma_commit(pv_full + (gc & 1));
           umma_commit(kv_empty + ks);
-          if (Cfg::kKVStages == 1 && j + 1 < nch && !issue_s(qb, gc + 1)) {
-            ok = false;
-            break;
-          }
         }
         ++ui;
       }
@@ -257,15 +254,29 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     float* red_max = red;         // [parity][half][128]
     float* red_sum = red + 512;
     auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q4) : "memory"); };
-    uint8_t* pH = sP + (uint32_t)half * Cfg::kPBlock;
-    uint8_t* pL = sP + (uint32_t)(CK / 64) * Cfg::kPBlock + (uint32_t)half * Cfg::kPBlock;
+    // fold PV_g (PV buffer g % 2) into the register output: o = o * c + PV_g
+    auto fold = [&](int g, float c, float* o) -> bool {
+      if (!mbar_wait_bounded(pv_full + (g & 1), (g >> 1) & 1, p.status)) return false;
+      tc_fence_after();
+      float pv[DO];
+      const uint32_t src = tmem + lane_off + (uint32_t)(2 * CK + (g & 1) * DH + half * DO);
+      if (DO == 16) {
+        tmem_ld16(src, pv);
+      } else {
+#pragma unroll
+        for (int cc = 0; cc < DO; cc += 32) tmem_ld32(src + (uint32_t)cc, pv + cc);
+      }
+#pragma unroll
+      for (int i = 0; i < DO; ++i) o[i] = o[i] * c + pv[i];
+      return true;
+    };
     int gc = 0, ui = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
       int b, h, q0, qcnt, qoff;
       unit_info(u, b, h, q0, qcnt, qoff);
       if (q0 >= qcnt) continue;
-      float m = -INFINITY, l = 0.f;
+      float m = -INFINITY, l = 0.f, corr_prev = 1.f;
       float o[DO];
 #pragma unroll
       for (int i = 0; i < DO; ++i) o[i] = 0.f;
@@ -280,8 +291,9 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         float corr = 1.f;
         if (active) {
           tc_fence_after();
+          const uint32_t tile = tmem + lane_off + (uint32_t)((gc & 1) * CK + half * KW);
           float v[64];
-          tmem_ld64(tmem + lane_off + (uint32_t)((gc & 1) * CK + half * KW), v);
+          tmem_ld64(tile, v);
           const int kvalid = p.kv_cnt - j * CK - half * KW;  // valid keys among this warp's 64
           float mx = -INFINITY;
           if (kvalid >= 64) {
@@ -302,17 +314,18 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           const float mn = fmaxf(m, mx);
           corr = ex2_approx(m - mn);
           m = mn;
-          // P = 2^(s * scale - m) as split pairs in the 128-byte-swizzled K-major
-          // tile (key block = half); keys past kv_cnt get 0
+          // P = 2^(s * scale - m) as split bf16 pairs over this warp's 64 S
+          // columns (already in registers): hi plane of keys 2c, 2c+1 in
+          // column c, lo plane in column 32 + c; keys past kv_cnt get 0
           const float sc = p.scale_log2, nm = -mn;
           float sum = 0.f;
           auto emit = [&](auto full) {
 #pragma unroll
-            for (int g = 0; g < 8; ++g) {
-              uint32_t hi[4], lo[4];
+            for (int hb = 0; hb < 2; ++hb) {
+              uint32_t hi[16], lo[16];
 #pragma unroll
-              for (int i = 0; i < 8; i += 2) {
-                const int k = 8 * g + i;
+              for (int i = 0; i < 32; i += 2) {
+                const int k = 32 * hb + i;
                 float p0 = ex2_approx(fmaf(v[k], sc, nm));
                 float p1 = ex2_approx(fmaf(v[k + 1], sc, nm));
                 if (!decltype(full)::value) {
@@ -322,37 +335,26 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
                 sum += p0 + p1;
                 split2_trunc(p0, p1, hi[i / 2], lo[i / 2]);
               }
-              const uint32_t off = (uint32_t)r * 128u + (((uint32_t)g ^ (uint32_t)(r & 7)) << 4);
-              *reinterpret_cast<uint4*>(pH + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-              *reinterpret_cast<uint4*>(pL + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+              tmem_st16_nowait(tile + (uint32_t)(16 * hb), hi);
+              tmem_st16_nowait(tile + (uint32_t)(32 + 16 * hb), lo);
             }
           };
           if (kvalid >= 64) emit(std::true_type{});
           else emit(std::false_type{});
           l = l * corr + sum;
-          fence_async_shared();
+          tmem_st_wait();
           tc_fence_before();
         }
-        mbar_arrive1(p_full);
-        // fold this chunk's P V into this warp's output columns
-        if (!mbar_wait_bounded(pv_full, gc & 1, p.status)) {
+        mbar_arrive1(p_full + (gc & 1));
+        // the previous chunk's PV is folded while PV_j runs
+        if (j > 0 && active && !fold(gc - 1, corr_prev, o)) {
           ok = false;
           break;
         }
-        if (active) {
-          tc_fence_after();
-          float pv[DO];
-          if (DO == 16) {
-            tmem_ld16(tmem + lane_off + (uint32_t)(2 * CK + half * DO), pv);
-          } else {
-#pragma unroll
-            for (int c = 0; c < DO; c += 32) tmem_ld32(tmem + lane_off + (uint32_t)(2 * CK + half * DO + c), pv + c);
-          }
-#pragma unroll
-          for (int i = 0; i < DO; ++i) o[i] = o[i] * corr + pv[i];
-        }
+        corr_prev = corr;
       }
       if (!ok) break;
+      if (active && !fold(gc - 1, corr_prev, o)) break;
       // row sum over both halves, then O / l as a split pair
       float ltot = l;
       if (Cfg::kHalves == 2) {
