@@ -8,12 +8,11 @@
 //                   W1_0, W1_1, W2_0, W1_2, W2_1, ...
 //   warp 1 lane 0 : tcgen05.mma -- FFN1 chunk f (64 columns of F) into one
 //                   of four TMEM buffers, two chunks ahead of FFN2 of chunk
-//                   f-2, which accumulates all chunks into a d-column TMEM
-//                   accumulator
-//   warps 2-9     : per chunk: bias + ReLU, split into hi/lo bf16, written to
-//                   a 128-byte-swizzled K-major shared tile that FFN2 reads
-//                   as its A operand; per tile: residual + b2 + LayerNorm,
-//                   stored with TMA tensor stores
+//                   f-2, which reads its A operand from that TMEM buffer and
+//                   accumulates all chunks into a d-column TMEM accumulator
+//   warps 2-9     : per chunk: bias + ReLU, split into hi/lo bf16 and written
+//                   back over the chunk's fp32 columns in TMEM; per tile:
+//                   residual + b2 + LayerNorm, stored with TMA tensor stores
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -28,9 +27,10 @@ constexpr int LA = 2;                          // FFN1 chunks issued ahead of th
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
 constexpr uint32_t kAPlane = BM * BK * 2;      // 16 KB: 128 rows x 64 bf16
-constexpr uint32_t kMidPlane = BM * FC * 2;    // 16 KB
 constexpr uint32_t kStageOut = 4096;           // final-epilogue staging per warp
 constexpr size_t kSmemMaxBlock = 232448;
+constexpr int kMaxRing = 8;                    // weight slots
+constexpr uint32_t kBarBytes = 512;
 
 struct FfnLayout {
   uint32_t a_bytes, slot_bytes, w1_chunk, w2_chunk;
@@ -45,9 +45,9 @@ __host__ __device__ inline FfnLayout ffn_layout(int d, int d_pad, int nb) {
   L.w2_chunk = (uint32_t)nb * (uint32_t)d * (FC * 2);                  // [plane][d x 64]
   L.slot_bytes = L.w1_chunk > L.w2_chunk ? L.w1_chunk : L.w2_chunk;
   L.slot_bytes = (L.slot_bytes + 1023u) & ~1023u;
-  const size_t fixed = 1024 + L.a_bytes + 4 * kMidPlane + 256 + 4096 + kEpiWarps * kStageOut;
+  const size_t fixed = 1024 + L.a_bytes + kBarBytes + 4096 + kEpiWarps * kStageOut;
   L.ring = fixed < kSmemMaxBlock ? (int)((kSmemMaxBlock - fixed) / L.slot_bytes) : 0;
-  if (L.ring > 4) L.ring = 4;
+  if (L.ring > kMaxRing) L.ring = kMaxRing;
   L.smem = fixed + (size_t)L.ring * L.slot_bytes;
   return L;
 }
@@ -57,6 +57,9 @@ __device__ __forceinline__ void mbar_arrive_one(uint64_t* bar) {
 }
 }  // namespace
 
+// NKB: 64-wide k blocks of d (1 or 2); NB: weight planes (1 or 2).  Both are
+// compile-time constants so that the MMA issue sequences have no branches.
+template <int NKB, int NB>
 __global__ void __launch_bounds__(kThreads, 1)
     ffn_kernel(const __grid_constant__ CUtensorMap tA_h, const __grid_constant__ CUtensorMap tA_l,
                const __grid_constant__ CUtensorMap tW1_h, const __grid_constant__ CUtensorMap tW1_l,
@@ -66,43 +69,38 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_s = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
-  const int d = p.d, nb = p.nb;
-  const FfnLayout LY = ffn_layout(d, p.d_pad, nb);
-  const int nkb = p.d_pad / BK;
+  constexpr int nb = NB, nkb = NKB;
+  const int d = p.d;
+  const FfnLayout LY = ffn_layout(d, NKB * BK, nb);
   const int nf = p.F / FC;
   uint8_t* sA = smem;
   uint8_t* sW = sA + LY.a_bytes;
-  uint8_t* sMid = sW + (size_t)LY.ring * LY.slot_bytes;  // [buffer 2][plane 2][16 KB]
-  uint8_t* sStg = sMid + 4 * kMidPlane;                   // [epilogue warp][4 KB]
+  uint8_t* sStg = sW + (size_t)LY.ring * LY.slot_bytes;  // [epilogue warp][4 KB]
   uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + kEpiWarps * kStageOut);
   uint64_t* a_full = bars;
   uint64_t* a_empty = bars + 1;
-  uint64_t* w_full = bars + 2;       // [4]
-  uint64_t* w_empty = bars + 6;      // [4]
-  uint64_t* acc1_full = bars + 10;   // [4]
-  uint64_t* acc1_empty = bars + 14;  // [4]
-  uint64_t* mid_full = bars + 18;    // [2]
-  uint64_t* mid_empty = bars + 20;   // [2]
-  uint64_t* acc2_full = bars + 22;
-  uint64_t* acc2_empty = bars + 23;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 24);
-  float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [parity][sum|var][half][128]
+  uint64_t* w_full = bars + 2;       // [kMaxRing]
+  uint64_t* w_empty = bars + 10;     // [kMaxRing]
+  uint64_t* acc1_full = bars + 18;   // [NA1] FFN1 chunk complete in TMEM buffer
+  uint64_t* acc1_empty = bars + 22;  // [NA1] FFN2 has read the buffer's hidden activation
+  uint64_t* mid_full = bars + 26;    // [NA1] hidden activation written over the buffer
+  uint64_t* acc2_full = bars + 30;
+  uint64_t* acc2_empty = bars + 31;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 32);
+  float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + kBarBytes);  // [parity][sum|var][half][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     mbar_init(a_full, 1);
     mbar_init(a_empty, 1);
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < kMaxRing; ++i) {
       mbar_init(w_full + i, 1);
       mbar_init(w_empty + i, 1);
     }
     for (int i = 0; i < NA1; ++i) {
       mbar_init(acc1_full + i, 1);
-      mbar_init(acc1_empty + i, kEpiWarps);
-    }
-    for (int i = 0; i < 2; ++i) {
+      mbar_init(acc1_empty + i, 1);
       mbar_init(mid_full + i, 32 * kEpiWarps);
-      mbar_init(mid_empty + i, 1);
     }
     mbar_init(acc2_full, 1);
     mbar_init(acc2_empty, kEpiWarps);
@@ -191,6 +189,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t dst = tmem + (uint32_t)(b * FC);
             const uint64_t a0 = umma_desc_sw128(smem_u32(sA));
             const uint64_t w0 = umma_desc_sw128(smem_u32(sW + (size_t)slot * LY.slot_bytes));
+#pragma unroll
             for (int kb = 0; kb < nkb; ++kb) {
 #pragma unroll
               for (int kk = 0; kk < BK / 16; ++kk) {
@@ -207,13 +206,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (s == nf - 1) umma_commit(a_empty);  // every FFN1 of this tile issued
           }
           if (s >= LA) {
-            // FFN2 chunk c = s - LA: acc2 += mid(c) . W2 chunk c
-            const int c = s - LA, g = gf0 + c, b = g & 1;
+            // FFN2 chunk c = s - LA: acc2 += mid(c) . W2 chunk c, mid(c) from TMEM buffer g % NA1
+            const int c = s - LA, g = gf0 + c, b = g % NA1;
             if (c == 0 && tl > 0 && !mbar_wait_bounded(acc2_empty, (tl - 1) & 1, p.status)) {
               ok = false;
               break;
             }
-            if (!mbar_wait_bounded(mid_full + b, (g >> 1) & 1, p.status)) {
+            if (!mbar_wait_bounded(mid_full + b, (g / NA1) & 1, p.status)) {
               ok = false;
               break;
             }
@@ -223,17 +222,20 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            const uint64_t m0 = umma_desc_sw128(smem_u32(sMid + (size_t)(b * 2) * kMidPlane));
+            // each 32-column half of the buffer holds 32 hidden units: hi plane in
+            // its first 16 columns, lo plane in the next 16 (two bf16 per column)
+            const uint32_t mt = tmem + (uint32_t)(b * FC);
             const uint64_t w0 = umma_desc_sw128(smem_u32(sW + (size_t)slot * LY.slot_bytes));
 #pragma unroll
             for (int kk = 0; kk < FC / 16; ++kk) {
-              const uint64_t mh = desc_adv(m0, kk * 32), wh = desc_adv(w0, kk * 32);
-              umma_bf16(tmem + NA1 * FC, mh, wh, idesc2, (c > 0 || kk > 0) ? 1u : 0u);
-              umma_bf16(tmem + NA1 * FC, desc_adv(mh, kMidPlane), wh, idesc2, 1u);
-              if (nb > 1) umma_bf16(tmem + NA1 * FC, mh, desc_adv(wh, (uint32_t)d * (FC * 2)), idesc2, 1u);
+              const uint32_t mh = mt + (uint32_t)((kk >> 1) * 32 + (kk & 1) * 8), ml = mh + 16;
+              const uint64_t wh = desc_adv(w0, kk * 32);
+              umma_bf16_tmem_a(tmem + NA1 * FC, mh, wh, idesc2, (c > 0 || kk > 0) ? 1u : 0u);
+              umma_bf16_tmem_a(tmem + NA1 * FC, ml, wh, idesc2, 1u);
+              if (nb > 1) umma_bf16_tmem_a(tmem + NA1 * FC, mh, desc_adv(wh, (uint32_t)d * (FC * 2)), idesc2, 1u);
             }
             umma_commit(w_empty + slot);
-            umma_commit(mid_empty + b);
+            umma_commit(acc1_empty + b);
             ++ws;
             if (c == nf - 1) umma_commit(acc2_full);
           }
@@ -282,19 +284,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           xr[32 * ci + 4 * j + 3] = qv.w;
         }
       }
-      // ---- per chunk: mid = split(ReLU(acc1 + b1)) into the shared A tile of FFN2
+      // ---- per chunk: mid = split(ReLU(acc1 + b1)) written back over this
+      // warp's 32 columns of the chunk's TMEM buffer as FFN2's A operand
       for (int f = 0; f < nf; ++f, ++gf) {
-        const int ba = gf % NA1, b = gf & 1;
+        const int ba = gf % NA1;
         if (!mbar_wait_bounded(acc1_full + ba, (gf / NA1) & 1, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
+        const uint32_t col = tmem + lane_off + (uint32_t)(ba * FC + 32 * half);
         float v[32];
-        tmem_ld32(tmem + lane_off + (uint32_t)(ba * FC + 32 * half), v);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive_one(acc1_empty + ba);
+        tmem_ld32(col, v);
         const float4* b4 = reinterpret_cast<const float4*>(p.b1 + f * FC + 32 * half);
         uint32_t hi[16], lo[16];
 #pragma unroll
@@ -303,20 +304,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           split2_trunc(fmaxf(v[4 * j] + bb.x, 0.f), fmaxf(v[4 * j + 1] + bb.y, 0.f), hi[2 * j], lo[2 * j]);
           split2_trunc(fmaxf(v[4 * j + 2] + bb.z, 0.f), fmaxf(v[4 * j + 3] + bb.w, 0.f), hi[2 * j + 1], lo[2 * j + 1]);
         }
-        if (gf >= 2 && !mbar_wait_bounded(mid_empty + b, ((gf >> 1) - 1) & 1, p.status)) {
-          ok = false;
-          break;
-        }
-        uint8_t* mh = sMid + (size_t)(b * 2) * kMidPlane;
-        uint8_t* ml = mh + kMidPlane;
-#pragma unroll
-        for (int g = 0; g < 4; ++g) {
-          const uint32_t off = (uint32_t)r * 128u + ((uint32_t)((4 * half + g) ^ (r & 7)) << 4);
-          *reinterpret_cast<uint4*>(mh + off) = make_uint4(hi[4 * g], hi[4 * g + 1], hi[4 * g + 2], hi[4 * g + 3]);
-          *reinterpret_cast<uint4*>(ml + off) = make_uint4(lo[4 * g], lo[4 * g + 1], lo[4 * g + 2], lo[4 * g + 3]);
-        }
-        fence_async_shared();
-        mbar_arrive_one(mid_full + b);
+        tmem_st16_nowait(col, hi);
+        tmem_st16_nowait(col + 16, lo);
+        tmem_st_wait();
+        tc_fence_before();
+        mbar_arrive_one(mid_full + ba);
       }
       if (!ok) break;
       // ---- final: x = resid + acc2 + b2, LayerNorm, stores
@@ -420,8 +412,13 @@ cudaError_t ffn_prepare() {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_ffn_sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(ffn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+  auto attr = [&](const void* f) {
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+  };
+  attr((const void*)ffn_kernel<1, 1>);
+  attr((const void*)ffn_kernel<1, 2>);
+  attr((const void*)ffn_kernel<2, 1>);
+  attr((const void*)ffn_kernel<2, 2>);
   return e;
 }
 
@@ -434,7 +431,9 @@ cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUt
   const long long tiles = (p.rows + BM - 1) / BM;
   long long grid = g_ffn_sms > 0 ? g_ffn_sms : 148;
   if (grid > tiles) grid = tiles;
-  return launch_k(ffn_kernel, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *a_h, *a_l, *w1_h,
+  auto kern = p.d_pad > BK ? (p.nb > 1 ? ffn_kernel<2, 2> : ffn_kernel<2, 1>)
+                           : (p.nb > 1 ? ffn_kernel<1, 2> : ffn_kernel<1, 1>);
+  return launch_k(kern, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *a_h, *a_l, *w1_h,
                   p.nb > 1 ? *w1_l : *w1_h, *w2_h, p.nb > 1 ? *w2_l : *w2_h, *o_h, *o_l, *o_x, p);
 }
 

@@ -57,7 +57,9 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
-template <int EPI>
+// NB: weight planes (1 when the weights are exact in bf16, else 2); a
+// compile-time constant so that the MMA issue sequence has no branches
+template <int EPI, int NB>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tA_h, const __grid_constant__ CUtensorMap tA_l,
                 const __grid_constant__ CUtensorMap tB_h, const __grid_constant__ CUtensorMap tB_l,
@@ -67,7 +69,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t raw_s = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
 
-  const int BN = p.BN, nb = p.nb, S = p.stages;
+  constexpr int nb = NB;
+  const int BN = p.BN, S = p.stages;
   const int nacc = p.nacc;
   const uint32_t b_bytes = (uint32_t)BN * BK * 2;
   const uint32_t stage_bytes = 2 * kATile + (uint32_t)nb * b_bytes;
@@ -436,7 +439,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) tmem_dealloc(tmem, ncols);
 }
 
-template <int EPI>
+template <int EPI, int NB>
 static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* b_h,
                             const CUtensorMap* b_l, const CUtensorMap* o_h, const CUtensorMap* o_l,
                             const CUtensorMap* o_x, const GemmParams& p0, cudaStream_t s) {
@@ -466,7 +469,7 @@ static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, cons
   if (smem > kSmemMaxBlock) smem = kSmemMaxBlock;
   long long grid = (long long)sms * per_sm;
   if (grid > tiles) grid = tiles;
-  return launch_k(gemm_kernel<EPI>, dim3((unsigned)grid), dim3(kThreads), smem, s, *a_h, *a_l, *b_h, *b_l,
+  return launch_k(gemm_kernel<EPI, NB>, dim3((unsigned)grid), dim3(kThreads), smem, s, *a_h, *a_l, *b_h, *b_l,
                   o_h ? *o_h : *a_h, o_l ? *o_l : *a_l, o_x ? *o_x : *a_h, p);
 }
 
@@ -474,15 +477,15 @@ cudaError_t gemm_prepare() {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(gemm_kernel<EPI_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kSmemMaxBlock);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(gemm_kernel<EPI_RESID_LN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kSmemMaxBlock);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(gemm_kernel<EPI_HEAD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kSmemMaxBlock);
+  auto attr = [&](const void* f) {
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+  };
+  attr((const void*)gemm_kernel<EPI_STORE, 1>);
+  attr((const void*)gemm_kernel<EPI_STORE, 2>);
+  attr((const void*)gemm_kernel<EPI_RESID_LN, 1>);
+  attr((const void*)gemm_kernel<EPI_RESID_LN, 2>);
+  attr((const void*)gemm_kernel<EPI_HEAD, 1>);
+  attr((const void*)gemm_kernel<EPI_HEAD, 2>);
   return e;
 }
 
@@ -490,10 +493,17 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l,
                         const CUtensorMap* b_l, const CUtensorMap* o_h, const CUtensorMap* o_l,
                         const CUtensorMap* o_x, const GemmParams& p, cudaStream_t s) {
   if (p.rows <= 0) return cudaSuccess;
+  const bool two = p.nb > 1;
   switch (epi) {
-    case EPI_STORE: return launch_t<EPI_STORE>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
-    case EPI_RESID_LN: return launch_t<EPI_RESID_LN>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
-    default: return launch_t<EPI_HEAD>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
+    case EPI_STORE:
+      return two ? launch_t<EPI_STORE, 2>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s)
+                 : launch_t<EPI_STORE, 1>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
+    case EPI_RESID_LN:
+      return two ? launch_t<EPI_RESID_LN, 2>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s)
+                 : launch_t<EPI_RESID_LN, 1>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
+    default:
+      return two ? launch_t<EPI_HEAD, 2>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s)
+                 : launch_t<EPI_HEAD, 1>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
   }
 }
 
