@@ -4,8 +4,8 @@
 // for rows of width d <= 128, without writing the F-wide intermediate to
 // memory.  A persistent CTA walks 128-row tiles:
 //   warp 0 lane 0 : TMA producer -- the LN(x) tile (hi/lo, held for the whole
-//                   tile) and a ring of weight slots in consumption order
-//                   W1_0, W1_1, W2_0, W1_2, W2_1, ...
+//                   tile), the fp32 residual tile x, and a ring of weight
+//                   slots in consumption order W1_0, W1_1, W1_2, W2_0, ...
 //   warp 1 lane 0 : tcgen05.mma -- FFN1 chunk f (64 columns of F) into one
 //                   of four TMEM buffers, two chunks ahead of FFN2 of chunk
 //                   f-2, which reads its A operand from that TMEM buffer and
@@ -13,6 +13,10 @@
 //   warps 2-9     : per chunk: bias + ReLU, split into hi/lo bf16 and written
 //                   back over the chunk's fp32 columns in TMEM; per tile:
 //                   residual + b2 + LayerNorm, stored with TMA tensor stores
+//                   staged in the residual tile's own 4 KB blocks
+// The residual arrives by TMA rather than by register loads: plain global
+// loads in flight hold up the shared-memory and mbarrier operations of the
+// producer and MMA warps until HBM answers.
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -27,7 +31,7 @@ constexpr int LA = 2;                          // FFN1 chunks issued ahead of th
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
 constexpr uint32_t kAPlane = BM * BK * 2;      // 16 KB: 128 rows x 64 bf16
-constexpr uint32_t kStageOut = 4096;           // final-epilogue staging per warp
+constexpr uint32_t kResBlock = 4096;           // residual block: 32 rows x 32 fp32, 128-byte swizzle
 constexpr size_t kSmemMaxBlock = 232448;
 constexpr int kMaxRing = 8;                    // weight slots
 constexpr uint32_t kBarBytes = 512;
@@ -45,7 +49,7 @@ __host__ __device__ inline FfnLayout ffn_layout(int d, int d_pad, int nb) {
   L.w2_chunk = (uint32_t)nb * (uint32_t)d * (FC * 2);                  // [plane][d x 64]
   L.slot_bytes = L.w1_chunk > L.w2_chunk ? L.w1_chunk : L.w2_chunk;
   L.slot_bytes = (L.slot_bytes + 1023u) & ~1023u;
-  const size_t fixed = 1024 + L.a_bytes + kBarBytes + 4096 + kEpiWarps * kStageOut;
+  const size_t fixed = 1024 + L.a_bytes + (size_t)(d_pad / 32) * 4 * kResBlock + kBarBytes + 4096;
   L.ring = fixed < kSmemMaxBlock ? (int)((kSmemMaxBlock - fixed) / L.slot_bytes) : 0;
   if (L.ring > kMaxRing) L.ring = kMaxRing;
   L.smem = fixed + (size_t)L.ring * L.slot_bytes;
@@ -75,8 +79,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nf = p.F / FC;
   uint8_t* sA = smem;
   uint8_t* sW = sA + LY.a_bytes;
-  uint8_t* sStg = sW + (size_t)LY.ring * LY.slot_bytes;  // [epilogue warp][4 KB]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + kEpiWarps * kStageOut);
+  uint8_t* sRes = sW + (size_t)LY.ring * LY.slot_bytes;  // [32-column chunk][row quadrant][4 KB]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sRes + (size_t)(NKB * BK / 32) * 4 * kResBlock);
   uint64_t* a_full = bars;
   uint64_t* a_empty = bars + 1;
   uint64_t* w_full = bars + 2;       // [kMaxRing]
@@ -86,7 +90,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* mid_full = bars + 26;    // [NA1] hidden activation written over the buffer
   uint64_t* acc2_full = bars + 30;
   uint64_t* acc2_empty = bars + 31;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 32);
+  uint64_t* r_full = bars + 32;      // residual tile loaded
+  uint64_t* r_empty = bars + 33;     // residual blocks free again (their last store has read them)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 34);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + kBarBytes);  // [parity][sum|var][half][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -104,6 +110,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(acc2_full, 1);
     mbar_init(acc2_empty, kEpiWarps);
+    mbar_init(r_full, 1);
+    mbar_init(r_empty, kEpiWarps);
     fence_mbar_init();
     prefetch_tmap(&tA_h);
     prefetch_tmap(&tW1_h);
@@ -155,6 +163,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           tma_load_2d(sA + (size_t)(kb * 2) * kAPlane, &tA_h, kb * BK, t * BM, a_full);
           tma_load_2d(sA + (size_t)(kb * 2 + 1) * kAPlane, &tA_l, kb * BK, t * BM, a_full);
         }
+        // residual x rows of the tile, 32 x 32 fp32 blocks (rows past the
+        // tensor extent arrive as zeros)
+        if (tl > 0 && !mbar_wait_bounded(r_empty, (tl - 1) & 1, p.status)) break;
+        mbar_arrive_expect_tx(r_full, (uint32_t)(d / 32) * 4 * kResBlock);
+        for (int c = 0; c < d / 32; ++c)
+          for (int q = 0; q < 4; ++q)
+            tma_load_2d(sRes + (size_t)(c * 4 + q) * kResBlock, &tO_x, 32 * c, t * BM + 32 * q, r_full);
         for (int s = 0; s < nf + LA && ok; ++s) {
           if (s < nf && !load_slot(true, s)) ok = false;
           if (ok && s >= LA && !load_slot(false, s - LA)) ok = false;
@@ -248,7 +263,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ew = warp - 2, q = warp & 3, half = ew >> 2;
     const int r = q * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    uint8_t* stg = sStg + (size_t)ew * kStageOut;
     auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory"); };
     auto issue = [&](const CUtensorMap* m0p, const void* s0, const CUtensorMap* m1p, const void* s1, int col,
                      int row) {
@@ -269,21 +283,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int m0 = t * BM;
       const int grow = m0 + r, srow = m0 + q * 32;
       const bool valid = grow < rows_valid;
-      // residual row chunks for the final epilogue, loaded while the FFN runs
-      const float* rrow = p.resid + (size_t)grow * p.ldr;
-#pragma unroll
-      for (int ci = 0; ci < 2; ++ci) {
-        const int c = 32 * half + 64 * ci;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          float4 qv = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (valid && c < d) qv = reinterpret_cast<const float4*>(rrow + c)[j];
-          xr[32 * ci + 4 * j] = qv.x;
-          xr[32 * ci + 4 * j + 1] = qv.y;
-          xr[32 * ci + 4 * j + 2] = qv.z;
-          xr[32 * ci + 4 * j + 3] = qv.w;
-        }
-      }
       // ---- per chunk: mid = split(ReLU(acc1 + b1)) written back over this
       // warp's 32 columns of the chunk's TMEM buffer as FFN2's A operand
       for (int f = 0; f < nf; ++f, ++gf) {
@@ -316,11 +315,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       float* red_sum = red + (size_t)(tl & 1) * 512;
       float* red_var = red_sum + 256;
+      if (!mbar_wait_bounded(r_full, tl & 1, p.status)) break;
+      // this warp's residual blocks: column chunks half and half + 2 of row quadrant q
+      auto blk = [&](int ci) { return sRes + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
       float sum = 0.f;
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
         if (c < d) {
+          // residual row (rows past the valid count are taken as 0)
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float4 qv = *reinterpret_cast<const float4*>(blk(ci) + (uint32_t)lane * 128u +
+                                                         ((uint32_t)(j ^ (lane & 7)) << 4));
+            if (!valid) qv = make_float4(0.f, 0.f, 0.f, 0.f);
+            xr[32 * ci + 4 * j] = qv.x;
+            xr[32 * ci + 4 * j + 1] = qv.y;
+            xr[32 * ci + 4 * j + 2] = qv.z;
+            xr[32 * ci + 4 * j + 3] = qv.w;
+          }
           float v[32];
           tmem_ld32(tmem + lane_off + (uint32_t)(NA1 * FC + c), v);
           const float4* b4 = reinterpret_cast<const float4*>(p.b2 + c);
@@ -347,11 +360,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const uint32_t o = (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4);
-            *reinterpret_cast<float4*>(stg + o) =
+            *reinterpret_cast<float4*>(blk(ci) + o) =
                 make_float4(xr[32 * ci + 4 * j], xr[32 * ci + 4 * j + 1], xr[32 * ci + 4 * j + 2],
                             xr[32 * ci + 4 * j + 3]);
           }
-          issue(&tO_x, stg, nullptr, nullptr, c, srow);
+          issue(&tO_x, blk(ci), nullptr, nullptr, c, srow);
         }
       }
       red_sum[half * 128 + r] = sum;
@@ -382,13 +395,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
-            *reinterpret_cast<uint4*>(stg + o) = make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
-            *reinterpret_cast<uint4*>(stg + 2048 + o) =
+            *reinterpret_cast<uint4*>(blk(ci) + o) =
+                make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
+            *reinterpret_cast<uint4*>(blk(ci) + 2048 + o) =
                 make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
           }
-          issue(&tO_h, stg, &tO_l, stg + 2048, c, srow);
+          issue(&tO_h, blk(ci), &tO_l, blk(ci) + 2048, c, srow);
         }
       }
+      // every store of this warp has read its blocks (issue() waits for that)
+      if (lane == 0) mbar_arrive_one(r_empty);
     }
     if (lane == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
   }
