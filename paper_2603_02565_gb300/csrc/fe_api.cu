@@ -152,7 +152,7 @@ int alloc_f32(F32Rows& f, int rows, int ld, std::vector<void*>& owned) {
 struct Weight {
   Planes p;
   int N = 0, K_pad = 0, BN = 0, stages = 0;
-  CUtensorMap fh{}, fl{};  // W1 of the fused FFN: 64 x 64 boxes
+  CUtensorMap fh{}, fl{};  // W1 of the fused FFN: 64 x 128 boxes
 };
 
 int largest_bn(int N, int cap) {
@@ -353,8 +353,8 @@ int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
 }
 
 int map_fused_w1(Weight& w, bool two) {
-  int rc = encode_map(&w.fh, w.p.h, w.p.ld, w.p.rows, 64);
-  if (rc == FE_OK) rc = encode_map(&w.fl, two ? w.p.l : w.p.h, w.p.ld, w.p.rows, 64);
+  int rc = encode_map(&w.fh, w.p.h, w.p.ld, w.p.rows, 128);
+  if (rc == FE_OK) rc = encode_map(&w.fl, two ? w.p.l : w.p.h, w.p.ld, w.p.rows, 128);
   return rc;
 }
 

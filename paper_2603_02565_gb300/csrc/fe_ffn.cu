@@ -2,21 +2,25 @@
 // 4.2 and the SeqEnc block of Section 4.3):
 //     x_out = x + ReLU(LN(x) W1 + b1) W2 + b2,   also LN(x_out)
 // for rows of width d <= 128, without writing the F-wide intermediate to
-// memory.  A persistent CTA walks 128-row tiles:
-//   warp 0 lane 0 : TMA producer -- the LN(x) tile (hi/lo, held for the whole
-//                   tile), the fp32 residual tile x, and a ring of weight
-//                   slots in consumption order W1_0, W1_1, W1_2, W2_0, ...
-//   warp 1 lane 0 : tcgen05.mma -- FFN1 chunk f (64 columns of F) into one
-//                   of four TMEM buffers, two chunks ahead of FFN2 of chunk
-//                   f-2, which reads its A operand from that TMEM buffer and
-//                   accumulates all chunks into a d-column TMEM accumulator
+// memory.  A persistent CTA walks 128-row tiles, F in chunks of 128 columns:
+//   warp 0 lane 0 : TMA producer -- the LN(x) tile (hi/lo, held while FFN1
+//                   runs), a ring of weight slots in consumption order
+//                   W1_0, W1_1, W1_2, W2_0, W1_3, W2_1, ..., and, once every
+//                   FFN1 of the tile has completed, the fp32 residual tile x
+//                   into the space the LN(x) tile held
+//   warp 1 lane 0 : tcgen05.mma -- FFN1 chunk f (N = 128) into one of three
+//                   TMEM buffers, two chunks ahead of FFN2 of chunk f-2, which
+//                   reads its A operand from that TMEM buffer and accumulates
+//                   every chunk into a d-column TMEM accumulator
 //   warps 2-9     : per chunk: bias + ReLU, split into hi/lo bf16 and written
 //                   back over the chunk's fp32 columns in TMEM; per tile:
 //                   residual + b2 + LayerNorm, stored with TMA tensor stores
 //                   staged in the residual tile's own 4 KB blocks
-// The residual arrives by TMA rather than by register loads: plain global
-// loads in flight hold up the shared-memory and mbarrier operations of the
-// producer and MMA warps until HBM answers.
+// The MMA groups are 16 instructions of N >= 128 so that the tensor pipe has
+// queued work while the issuing thread polls its barriers; the residual
+// arrives by TMA rather than by register loads (global loads in flight hold up
+// the shared-memory and mbarrier operations of the other warps); the biases
+// sit in shared memory.
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -25,8 +29,8 @@ namespace fe {
 namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int FC = 64;                         // FFN columns per chunk
-constexpr int NA1 = 4;                         // TMEM buffers for FFN1 chunks
+constexpr int FC = 128;                        // FFN columns per chunk
+constexpr int NA1 = 3;                         // TMEM buffers for FFN1 chunks
 constexpr int LA = 2;                          // FFN1 chunks issued ahead of the FFN2 that consumes them
 constexpr int kEpiWarps = 8;
 constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
@@ -35,21 +39,23 @@ constexpr uint32_t kResBlock = 4096;           // residual block: 32 rows x 32 f
 constexpr size_t kSmemMaxBlock = 232448;
 constexpr int kMaxRing = 8;                    // weight slots
 constexpr uint32_t kBarBytes = 512;
+constexpr uint32_t kRedBytes = 2 * 2 * 128 * 4;  // [sum|var][half][row]
 
 struct FfnLayout {
-  uint32_t a_bytes, slot_bytes, w1_chunk, w2_chunk;
+  uint32_t a_bytes, slot_bytes, w1_chunk, w2_chunk, bias_bytes;
   int ring;
   size_t smem;
 };
 
-__host__ __device__ inline FfnLayout ffn_layout(int d, int d_pad, int nb) {
+__host__ __device__ inline FfnLayout ffn_layout(int d, int d_pad, int F, int nb) {
   FfnLayout L;
   L.a_bytes = (uint32_t)(d_pad / BK) * 2u * kAPlane;
-  L.w1_chunk = (uint32_t)nb * (uint32_t)(d_pad / BK) * (FC * BK * 2);  // [kb][plane][64 x 64]
-  L.w2_chunk = (uint32_t)nb * (uint32_t)d * (FC * 2);                  // [plane][d x 64]
+  L.w1_chunk = (uint32_t)nb * (uint32_t)(d_pad / BK) * (FC * BK * 2);  // [kb][plane][128 rows x 64]
+  L.w2_chunk = (uint32_t)nb * 2u * (uint32_t)d * (BK * 2);             // [plane][half][d rows x 64]
   L.slot_bytes = L.w1_chunk > L.w2_chunk ? L.w1_chunk : L.w2_chunk;
   L.slot_bytes = (L.slot_bytes + 1023u) & ~1023u;
-  const size_t fixed = 1024 + L.a_bytes + (size_t)(d_pad / 32) * 4 * kResBlock + kBarBytes + 4096;
+  L.bias_bytes = ((uint32_t)(F + d) * 4u + 127u) & ~127u;
+  const size_t fixed = 1024 + L.a_bytes + L.bias_bytes + kBarBytes + kRedBytes;
   L.ring = fixed < kSmemMaxBlock ? (int)((kSmemMaxBlock - fixed) / L.slot_bytes) : 0;
   if (L.ring > kMaxRing) L.ring = kMaxRing;
   L.smem = fixed + (size_t)L.ring * L.slot_bytes;
@@ -74,26 +80,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t raw_s = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
   constexpr int nb = NB, nkb = NKB;
-  const int d = p.d;
-  const FfnLayout LY = ffn_layout(d, NKB * BK, nb);
-  const int nf = p.F / FC;
-  uint8_t* sA = smem;
+  const int d = p.d, F = p.F;
+  const FfnLayout LY = ffn_layout(d, NKB * BK, F, nb);
+  const int nf = F / FC;
+  uint8_t* sA = smem;  // LN(x) tile [kb][plane]; later the residual tile [32-column chunk][row quadrant][4 KB]
   uint8_t* sW = sA + LY.a_bytes;
-  uint8_t* sRes = sW + (size_t)LY.ring * LY.slot_bytes;  // [32-column chunk][row quadrant][4 KB]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sRes + (size_t)(NKB * BK / 32) * 4 * kResBlock);
-  uint64_t* a_full = bars;
-  uint64_t* a_empty = bars + 1;
+  float* sB1 = reinterpret_cast<float*>(sW + (size_t)LY.ring * LY.slot_bytes);
+  float* sB2 = sB1 + F;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(sB1) + LY.bias_bytes);
+  uint64_t* a_full = bars;           // LN(x) tile loaded
+  uint64_t* a_empty = bars + 1;      // every FFN1 of the tile complete
   uint64_t* w_full = bars + 2;       // [kMaxRing]
   uint64_t* w_empty = bars + 10;     // [kMaxRing]
   uint64_t* acc1_full = bars + 18;   // [NA1] FFN1 chunk complete in TMEM buffer
-  uint64_t* acc1_empty = bars + 22;  // [NA1] FFN2 has read the buffer's hidden activation
-  uint64_t* mid_full = bars + 26;    // [NA1] hidden activation written over the buffer
-  uint64_t* acc2_full = bars + 30;
-  uint64_t* acc2_empty = bars + 31;
-  uint64_t* r_full = bars + 32;      // residual tile loaded
-  uint64_t* r_empty = bars + 33;     // residual blocks free again (their last store has read them)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 34);
-  float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + kBarBytes);  // [parity][sum|var][half][128]
+  uint64_t* acc1_empty = bars + 21;  // [NA1] FFN2 has read the buffer's hidden activation
+  uint64_t* mid_full = bars + 24;    // [NA1] hidden activation written over the buffer
+  uint64_t* acc2_full = bars + 27;
+  uint64_t* acc2_empty = bars + 28;
+  uint64_t* r_full = bars + 29;      // residual tile loaded
+  uint64_t* r_empty = bars + 30;     // residual blocks free again (their last store has read them)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 31);
+  float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + kBarBytes);  // [sum|var][half][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -116,8 +123,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tA_h);
     prefetch_tmap(&tW1_h);
     prefetch_tmap(&tW2_h);
+    prefetch_tmap(&tO_x);
   }
-  // TMEM: FFN1 chunk buffers at columns [64 i, 64 i + 64), i < 4; FFN2 accumulator at [256, 256+d)
+  // biases are parameters, not outputs of an earlier kernel: read before the dependency wait
+  for (int i = threadIdx.x; i < F; i += kThreads) sB1[i] = p.b1[i];
+  for (int i = threadIdx.x; i < d; i += kThreads) sB2[i] = p.b2[i];
+  // TMEM: FFN1 chunk buffers at columns [128 i, 128 i + 128), i < 3; FFN2 accumulator at [384, 384 + d)
   if (warp == 0) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
@@ -142,38 +153,42 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int slot = ws % LY.ring;
         if (ws >= LY.ring && !mbar_wait_bounded(w_empty + slot, ((ws / LY.ring) - 1) & 1, p.status)) return false;
         uint8_t* dst = sW + (size_t)slot * LY.slot_bytes;
-        if (first) {  // W1 rows [f*64, f*64+64), all k blocks
+        if (first) {  // W1 rows [f*128, f*128+128), every k block
           mbar_arrive_expect_tx(w_full + slot, LY.w1_chunk);
           for (int kb = 0; kb < nkb; ++kb)
             for (int q = 0; q < nb; ++q)
               tma_load_2d(dst + (size_t)(kb * nb + q) * (FC * BK * 2), q ? &tW1_l : &tW1_h, kb * BK, f * FC,
                           w_full + slot);
-        } else {  // W2 columns [f*64, f*64+64), all d rows
+        } else {  // W2 columns [f*128, f*128+128) as two 64-column halves, every d row
           mbar_arrive_expect_tx(w_full + slot, LY.w2_chunk);
           for (int q = 0; q < nb; ++q)
-            tma_load_2d(dst + (size_t)q * d * (FC * 2), q ? &tW2_l : &tW2_h, f * FC, 0, w_full + slot);
+            for (int hh = 0; hh < 2; ++hh)
+              tma_load_2d(dst + (size_t)(q * 2 + hh) * d * (BK * 2), q ? &tW2_l : &tW2_h, f * FC + BK * hh, 0,
+                          w_full + slot);
         }
         ++ws;
         return true;
       };
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
-        if (tl > 0 && !mbar_wait_bounded(a_empty, (tl - 1) & 1, p.status)) break;
+        // sA holds the previous tile's residual until that tile's stores have read it
+        if (tl > 0 && !mbar_wait_bounded(r_empty, (tl - 1) & 1, p.status)) break;
         mbar_arrive_expect_tx(a_full, LY.a_bytes);
         for (int kb = 0; kb < nkb; ++kb) {
           tma_load_2d(sA + (size_t)(kb * 2) * kAPlane, &tA_h, kb * BK, t * BM, a_full);
           tma_load_2d(sA + (size_t)(kb * 2 + 1) * kAPlane, &tA_l, kb * BK, t * BM, a_full);
         }
-        // residual x rows of the tile, 32 x 32 fp32 blocks (rows past the
-        // tensor extent arrive as zeros)
-        if (tl > 0 && !mbar_wait_bounded(r_empty, (tl - 1) & 1, p.status)) break;
-        mbar_arrive_expect_tx(r_full, (uint32_t)(d / 32) * 4 * kResBlock);
-        for (int c = 0; c < d / 32; ++c)
-          for (int q = 0; q < 4; ++q)
-            tma_load_2d(sRes + (size_t)(c * 4 + q) * kResBlock, &tO_x, 32 * c, t * BM + 32 * q, r_full);
         for (int s = 0; s < nf + LA && ok; ++s) {
           if (s < nf && !load_slot(true, s)) ok = false;
           if (ok && s >= LA && !load_slot(false, s - LA)) ok = false;
         }
+        if (!ok) break;
+        // residual x rows of the tile in 32 x 32 fp32 blocks, into sA once the
+        // last FFN1 has read it (rows past the tensor extent arrive as zeros)
+        if (!mbar_wait_bounded(a_empty, tl & 1, p.status)) break;
+        mbar_arrive_expect_tx(r_full, (uint32_t)(d / 32) * 4 * kResBlock);
+        for (int c = 0; c < d / 32; ++c)
+          for (int q = 0; q < 4; ++q)
+            tma_load_2d(sA + (size_t)(c * 4 + q) * kResBlock, &tO_x, 32 * c, t * BM + 32 * q, r_full);
       }
     }
   } else if (warp == 1) {
@@ -181,6 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---------------- MMA issuer ----------------
       const uint32_t idesc1 = umma_idesc_bf16(BM, FC);
       const uint32_t idesc2 = umma_idesc_bf16(BM, d);
+      const uint32_t acc2 = tmem + (uint32_t)(NA1 * FC);
       int tl = 0, ws = 0, gf = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
@@ -237,17 +253,19 @@ __global__ void __launch_bounds__(kThreads, 1)
               break;
             }
             tc_fence_after();
-            // each 32-column half of the buffer holds 32 hidden units: hi plane in
-            // its first 16 columns, lo plane in the next 16 (two bf16 per column)
+            // each 32-column piece of the buffer holds 32 hidden units: hi plane in
+            // its first 16 columns, lo plane in the next 16 (two bf16 per column);
+            // the W2 slot holds 64-column halves of the chunk, d rows each
             const uint32_t mt = tmem + (uint32_t)(b * FC);
             const uint64_t w0 = umma_desc_sw128(smem_u32(sW + (size_t)slot * LY.slot_bytes));
 #pragma unroll
             for (int kk = 0; kk < FC / 16; ++kk) {
-              const uint32_t mh = mt + (uint32_t)((kk >> 1) * 32 + (kk & 1) * 8), ml = mh + 16;
-              const uint64_t wh = desc_adv(w0, kk * 32);
-              umma_bf16_tmem_a(tmem + NA1 * FC, mh, wh, idesc2, (c > 0 || kk > 0) ? 1u : 0u);
-              umma_bf16_tmem_a(tmem + NA1 * FC, ml, wh, idesc2, 1u);
-              if (nb > 1) umma_bf16_tmem_a(tmem + NA1 * FC, mh, desc_adv(wh, (uint32_t)d * (FC * 2)), idesc2, 1u);
+              const int hh = kk >> 2, k4 = kk & 3;
+              const uint32_t mh = mt + (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1)), ml = mh + 16;
+              const uint64_t wh = desc_adv(w0, (uint32_t)hh * (uint32_t)d * (BK * 2) + k4 * 32);
+              umma_bf16_tmem_a(acc2, mh, wh, idesc2, (c > 0 || kk > 0) ? 1u : 0u);
+              umma_bf16_tmem_a(acc2, ml, wh, idesc2, 1u);
+              if (nb > 1) umma_bf16_tmem_a(acc2, mh, desc_adv(wh, 2u * (uint32_t)d * (BK * 2)), idesc2, 1u);
             }
             umma_commit(w_empty + slot);
             umma_commit(acc1_empty + b);
@@ -263,7 +281,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ew = warp - 2, q = warp & 3, half = ew >> 2;
     const int r = q * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    float* red_sum = red;
+    float* red_var = red + 256;
     auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory"); };
+    // tensor stores of this warp's staged blocks; the reads are awaited separately
     auto issue = [&](const CUtensorMap* m0p, const void* s0, const CUtensorMap* m1p, const void* s1, int col,
                      int row) {
       fence_async_shared();
@@ -272,19 +293,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_store_2d(m0p, s0, col, row);
         if (m1p) tma_store_2d(m1p, s1, col, row);
         bulk_commit();
-        bulk_wait_read0();  // the staging is reused right away
       }
+      __syncwarp();
+    };
+    auto stores_read = [&]() {
+      if (lane == 0) bulk_wait_read0();
       __syncwarp();
     };
     int tl = 0, gf = 0;
     bool ok = true;
-    float xr[64];
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
       const int m0 = t * BM;
-      const int grow = m0 + r, srow = m0 + q * 32;
-      const bool valid = grow < rows_valid;
+      const int srow = m0 + q * 32;
+      const bool valid = m0 + r < rows_valid;
       // ---- per chunk: mid = split(ReLU(acc1 + b1)) written back over this
-      // warp's 32 columns of the chunk's TMEM buffer as FFN2's A operand
+      // warp's 64 columns of the chunk's TMEM buffer as FFN2's A operand
       for (int f = 0; f < nf; ++f, ++gf) {
         const int ba = gf % NA1;
         if (!mbar_wait_bounded(acc1_full + ba, (gf / NA1) & 1, p.status)) {
@@ -292,19 +315,23 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t col = tmem + lane_off + (uint32_t)(ba * FC + 32 * half);
-        float v[32];
-        tmem_ld32(col, v);
-        const float4* b4 = reinterpret_cast<const float4*>(p.b1 + f * FC + 32 * half);
-        uint32_t hi[16], lo[16];
+        // this warp's 64 columns as two 32-column pieces, each read whole and
+        // then overwritten by its own hi (16 columns) and lo (16 columns) planes
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float4 bb = __ldg(b4 + j);
-          split2_trunc(fmaxf(v[4 * j] + bb.x, 0.f), fmaxf(v[4 * j + 1] + bb.y, 0.f), hi[2 * j], lo[2 * j]);
-          split2_trunc(fmaxf(v[4 * j + 2] + bb.z, 0.f), fmaxf(v[4 * j + 3] + bb.w, 0.f), hi[2 * j + 1], lo[2 * j + 1]);
+        for (int hp = 0; hp < 2; ++hp) {
+          const uint32_t col = tmem + lane_off + (uint32_t)(ba * FC + 64 * half + 32 * hp);
+          const float* bias = sB1 + f * FC + 64 * half + 32 * hp;
+          float v[32];
+          tmem_ld32(col, v);
+          uint32_t hi[16], lo[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float2 bb = *reinterpret_cast<const float2*>(bias + 2 * j);
+            split2_trunc(fmaxf(v[2 * j] + bb.x, 0.f), fmaxf(v[2 * j + 1] + bb.y, 0.f), hi[j], lo[j]);
+          }
+          tmem_st16_nowait(col, hi);
+          tmem_st16_nowait(col + 16, lo);
         }
-        tmem_st16_nowait(col, hi);
-        tmem_st16_nowait(col + 16, lo);
         tmem_st_wait();
         tc_fence_before();
         mbar_arrive_one(mid_full + ba);
@@ -312,42 +339,33 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       // ---- final: x = resid + acc2 + b2, LayerNorm, stores
       if (!mbar_wait_bounded(acc2_full, tl & 1, p.status)) break;
-      tc_fence_after();
-      float* red_sum = red + (size_t)(tl & 1) * 512;
-      float* red_var = red_sum + 256;
       if (!mbar_wait_bounded(r_full, tl & 1, p.status)) break;
+      tc_fence_after();
       // this warp's residual blocks: column chunks half and half + 2 of row quadrant q
-      auto blk = [&](int ci) { return sRes + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
+      auto blk = [&](int ci) { return sA + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
+      // row chunk of 32 fp32 in a block: 16-byte piece j of row `lane`, 128-byte swizzle
+      auto xoff = [&](int j) { return (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4); };
+      // x = resid + acc2 + b2, written in place over the residual (rows past the
+      // valid count take resid = 0)
       float sum = 0.f;
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
         if (c < d) {
-          // residual row (rows past the valid count are taken as 0)
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            float4 qv = *reinterpret_cast<const float4*>(blk(ci) + (uint32_t)lane * 128u +
-                                                         ((uint32_t)(j ^ (lane & 7)) << 4));
-            if (!valid) qv = make_float4(0.f, 0.f, 0.f, 0.f);
-            xr[32 * ci + 4 * j] = qv.x;
-            xr[32 * ci + 4 * j + 1] = qv.y;
-            xr[32 * ci + 4 * j + 2] = qv.z;
-            xr[32 * ci + 4 * j + 3] = qv.w;
-          }
           float v[32];
           tmem_ld32(tmem + lane_off + (uint32_t)(NA1 * FC + c), v);
-          const float4* b4 = reinterpret_cast<const float4*>(p.b2 + c);
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            const float4 bb = __ldg(b4 + j);
-            xr[32 * ci + 4 * j] += v[4 * j] + bb.x;
-            xr[32 * ci + 4 * j + 1] += v[4 * j + 1] + bb.y;
-            xr[32 * ci + 4 * j + 2] += v[4 * j + 2] + bb.z;
-            xr[32 * ci + 4 * j + 3] += v[4 * j + 3] + bb.w;
+            float4* px = reinterpret_cast<float4*>(blk(ci) + xoff(j));
+            float4 x = valid ? *px : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 bb = *reinterpret_cast<const float4*>(sB2 + c + 4 * j);
+            x.x += v[4 * j] + bb.x;
+            x.y += v[4 * j + 1] + bb.y;
+            x.z += v[4 * j + 2] + bb.z;
+            x.w += v[4 * j + 3] + bb.w;
+            sum += (x.x + x.y) + (x.z + x.w);
+            *px = x;
           }
-#pragma unroll
-          for (int i = 0; i < 32; i += 4)
-            sum += (xr[32 * ci + i] + xr[32 * ci + i + 1]) + (xr[32 * ci + i + 2] + xr[32 * ci + i + 3]);
         }
       }
       tc_fence_before();
@@ -356,16 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
-        if (c < d) {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const uint32_t o = (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4);
-            *reinterpret_cast<float4*>(blk(ci) + o) =
-                make_float4(xr[32 * ci + 4 * j], xr[32 * ci + 4 * j + 1], xr[32 * ci + 4 * j + 2],
-                            xr[32 * ci + 4 * j + 3]);
-          }
-          issue(&tO_x, blk(ci), nullptr, nullptr, c, srow);
-        }
+        if (c < d) issue(&tO_x, blk(ci), nullptr, nullptr, c, srow);
       }
       red_sum[half * 128 + r] = sum;
       pair_sync();
@@ -375,8 +384,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int ci = 0; ci < 2; ++ci) {
         if (32 * half + 64 * ci < d) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float dv = xr[32 * ci + i] - mean;
+          for (int j = 0; j < 8; ++j) {
+            const float4 x = *reinterpret_cast<const float4*>(blk(ci) + xoff(j));
+            float dv = x.x - mean;
+            var = fmaf(dv, dv, var);
+            dv = x.y - mean;
+            var = fmaf(dv, dv, var);
+            dv = x.z - mean;
+            var = fmaf(dv, dv, var);
+            dv = x.w - mean;
             var = fmaf(dv, dv, var);
           }
         }
@@ -384,14 +400,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       red_var[half * 128 + r] = var;
       pair_sync();
       const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)d + p.eps);
+      stores_read();  // the x stores have read the blocks
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
         if (c < d) {
           uint32_t hi[16], lo[16];
 #pragma unroll
-          for (int i = 0; i < 32; i += 2)
-            split2((xr[32 * ci + i] - mean) * rstd, (xr[32 * ci + i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
+          for (int j = 0; j < 8; ++j) {
+            const float4 x = *reinterpret_cast<const float4*>(blk(ci) + xoff(j));
+            split2((x.x - mean) * rstd, (x.y - mean) * rstd, hi[2 * j], lo[2 * j]);
+            split2((x.z - mean) * rstd, (x.w - mean) * rstd, hi[2 * j + 1], lo[2 * j + 1]);
+          }
+          __syncwarp();  // every row of the block is read before the planes overwrite it
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
@@ -403,8 +424,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue(&tO_h, blk(ci), &tO_l, blk(ci) + 2048, c, srow);
         }
       }
-      // every store of this warp has read its blocks (issue() waits for that)
-      if (lane == 0) mbar_arrive_one(r_empty);
+      stores_read();
+      if (lane == 0) mbar_arrive_one(r_empty);  // sA may take the next tile's LN(x)
     }
     if (lane == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
   }
@@ -419,8 +440,8 @@ int g_ffn_sms = 0;
 }
 
 bool ffn_supported(int d, int d_pad, int F, int nb) {
-  if (d > 128 || d % 32 || F % FC || F < FC) return false;
-  const FfnLayout L = ffn_layout(d, d_pad, nb);
+  if (d > 128 || d % 32 || F % FC || F < FC || NA1 * FC + d > 512) return false;
+  const FfnLayout L = ffn_layout(d, d_pad, F, nb);
   return L.ring >= 2 && L.smem <= kSmemMaxBlock;
 }
 
@@ -443,7 +464,7 @@ cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUt
                        const CUtensorMap* o_h, const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p,
                        cudaStream_t s) {
   if (p.rows <= 0) return cudaSuccess;
-  const FfnLayout LY = ffn_layout(p.d, p.d_pad, p.nb);
+  const FfnLayout LY = ffn_layout(p.d, p.d_pad, p.F, p.nb);
   const long long tiles = (p.rows + BM - 1) / BM;
   long long grid = g_ffn_sms > 0 ? g_ffn_sms : 148;
   if (grid > tiles) grid = tiles;
