@@ -1,6 +1,8 @@
 // C-ABI of the joint evaluator: weights, workspace, TMA descriptors, the
 // launch sequence of one evaluation and its CUDA-graph cache.
 #include <algorithm>
+#include <cmath>
+#include <limits>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -50,8 +52,10 @@ EncodeTiledFn encode_fn() {
 }
 
 // A bf16 matrix stored as one or two planes (hi, lo), row-major [rows, ld].
+// A bf16 hi/lo pair of row-major planes, or (attention operands: context K/V,
+// element queries, cross-sequence Q/K/V) a single f16 plane in h.
 struct Planes {
-  bf16* h = nullptr;
+  bf16* h = nullptr;  // f16 bits for the single-plane attention operands
   bf16* l = nullptr;
   int ld = 0;
   int rows = 0;
@@ -127,14 +131,15 @@ int map_out(Planes& p) {
   return rc;
 }
 
-// Descriptors of an attention operand (Q, K or V head slices).
+// Descriptors of a single-plane f16 attention operand: the GEMM epilogue's
+// store map and the attention kernel's Q and K/V head-slice maps.
 int map_attn(Planes& p, int dh) {
   const CUtensorMapSwizzle sw = dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
   const int kv_rows = dh == 32 ? 64 : 128;
-  int rc = encode_map_t(&p.ah, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.h, p.ld, p.rows, dh, 128, sw);
-  if (rc == FE_OK) rc = encode_map_t(&p.al, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.l, p.ld, p.rows, dh, 128, sw);
-  if (rc == FE_OK) rc = encode_map_t(&p.kh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.h, p.ld, p.rows, dh, kv_rows, sw);
-  if (rc == FE_OK) rc = encode_map_t(&p.kl, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p.l, p.ld, p.rows, dh, kv_rows, sw);
+  int rc = encode_map_t(&p.sh, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.h, p.ld, p.rows, 32, 32,
+                        CU_TENSOR_MAP_SWIZZLE_64B);
+  if (rc == FE_OK) rc = encode_map_t(&p.ah, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.h, p.ld, p.rows, dh, 128, sw);
+  if (rc == FE_OK) rc = encode_map_t(&p.kh, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.h, p.ld, p.rows, dh, kv_rows, sw);
   return rc;
 }
 
@@ -450,6 +455,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   }
   {
     fe::GemmParams p{};
+    p.out_f16 = 1;
     FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, &c->KV, nullptr, s));
   }
   // (a2) distinct elements: gather + LN, then the cross-attention stack
@@ -460,6 +466,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   }
   for (int l = 0; l < Ly; ++l) {
     fe::GemmParams p{};
+    p.out_f16 = 1;
     FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
 
     fe::AttnParams ap{};
@@ -481,7 +488,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.status = c->status;
     {
       Prof pf(c, "attn_item_ctx", s);
-      FE_CK(fe::attn_launch(c->dh, &c->q.ah, &c->q.al, &c->KV.kh, &c->KV.kl, &c->KV.kh, &c->KV.kl, ap, s));
+      FE_CK(fe::attn_launch(c->dh, &c->q.ah, &c->KV.kh, &c->KV.kh, ap, s));
     }
 
     fe::GemmParams po{};
@@ -561,6 +568,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   // (a5) cross-sequence attention over the K sequence vectors of each request
   {
     fe::GemmParams p{};
+    p.out_f16 = 1;
     FE_RC(gemm(c, "gemm_cross_qkv", fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, &c->qkv, nullptr, s));
     fe::AttnParams ap{};
     ap.n_segments = B;
@@ -581,7 +589,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.status = c->status;
     {
       Prof pf(c, "attn_cross_seq", s);
-      FE_CK(fe::attn_launch(c->dh, &c->qkv.ah, &c->qkv.al, &c->qkv.kh, &c->qkv.kl, &c->qkv.kh, &c->qkv.kl, ap, s));
+      FE_CK(fe::attn_launch(c->dh, &c->qkv.ah, &c->qkv.kh, &c->qkv.kh, ap, s));
     }
     fe::GemmParams po{};
     po.resid = c->c.p;
@@ -676,9 +684,9 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->out_scores, (size_t)S * sizeof(float)));
   FE_RC(dalloc((void**)&c->out_best, (size_t)B * sizeof(int32_t)));
   FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
-  FE_RC(alloc_planes(c->KV, BC, 2 * Ly * d, true, c->owned_ws));
+  FE_RC(alloc_planes(c->KV, BC, 2 * Ly * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->xln, R, c->dpad, true, c->owned_ws));
-  FE_RC(alloc_planes(c->q, R, d, true, c->owned_ws));
+  FE_RC(alloc_planes(c->q, R, d, false, c->owned_ws));
   FE_RC(alloc_planes(c->a, R, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->mid, R, c->Fpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->kvI, R, 2 * d, true, c->owned_ws));
@@ -686,13 +694,12 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(alloc_planes(c->cln, S, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->mids, S, c->Fpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->z, S, c->dpad, true, c->owned_ws));
-  FE_RC(alloc_planes(c->qkv, S, 3 * d, true, c->owned_ws));
+  FE_RC(alloc_planes(c->qkv, S, 3 * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->ax, S, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->lncp, S, c->dpad, true, c->owned_ws));
   for (Planes* p : {&c->X, &c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp})
     FE_RC(map_act(*p));
-  for (Planes* p : {&c->KV, &c->q, &c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->qkv, &c->lncp})
-    FE_RC(map_out(*p));
+  for (Planes* p : {&c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->lncp}) FE_RC(map_out(*p));
   for (Planes* p : {&c->KV, &c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
   c->cap_shape = s;
   c->cap_rows = R;
@@ -988,6 +995,25 @@ int fe_debug_layout(fe_ctx* c, int32_t* slot_out, int32_t* U_out) {
   return FE_OK;
 }
 
+// IEEE binary16 bits -> float (normal, subnormal, zero, infinity, NaN)
+static float f16_to_float(uint16_t h) {
+  const uint32_t sign = (uint32_t)(h & 0x8000u) << 16;
+  const uint32_t ex = (h >> 10) & 0x1Fu, man = h & 0x3FFu;
+  float mag;
+  if (ex == 0) {
+    mag = std::ldexp((float)man, -24);
+  } else if (ex == 31) {
+    mag = man ? std::numeric_limits<float>::quiet_NaN() : std::numeric_limits<float>::infinity();
+  } else {
+    mag = std::ldexp((float)(man | 0x400u), (int)ex - 25);
+  }
+  uint32_t u;
+  std::memcpy(&u, &mag, 4);
+  u |= sign;
+  std::memcpy(&mag, &u, 4);
+  return mag;
+}
+
 int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, size_t* n_floats) {
   if (!c || !name || !n_floats) return FE_ERR_INVALID_ARG;
   if (!c->have_last) {
@@ -1039,10 +1065,13 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
     return FE_OK;
   }
   std::vector<uint16_t> hh((size_t)rows * pl->ld), ll((size_t)rows * pl->ld);
-  if (rows) {
-    FE_CK(cudaMemcpy(hh.data(), pl->h, hh.size() * 2, cudaMemcpyDeviceToHost));
-    FE_CK(cudaMemcpy(ll.data(), pl->l, ll.size() * 2, cudaMemcpyDeviceToHost));
+  if (rows) FE_CK(cudaMemcpy(hh.data(), pl->h, hh.size() * 2, cudaMemcpyDeviceToHost));
+  if (!pl->l) {  // single f16 plane
+    for (size_t r = 0; r < rows; ++r)
+      for (size_t j = 0; j < cols; ++j) dst[r * cols + j] = f16_to_float(hh[r * pl->ld + j]);
+    return FE_OK;
   }
+  if (rows) FE_CK(cudaMemcpy(ll.data(), pl->l, ll.size() * 2, cudaMemcpyDeviceToHost));
   for (size_t r = 0; r < rows; ++r)
     for (size_t j = 0; j < cols; ++j) {
       const uint32_t a = (uint32_t)hh[r * pl->ld + j] << 16, b = (uint32_t)ll[r * pl->ld + j] << 16;

@@ -9,20 +9,22 @@
 // Persistent CTAs walk units (segment b, head h, 128-row query tile).  Per
 // unit the keys stream in chunks of CK (64 for d_h = 32, 128 for d_h = 64):
 //   warp 0 lane 0 : TMA producer -- Q tile (two buffers, one per unit in
-//                   flight) and K/V chunks of CK keys (4 stages for d_h = 32,
-//                   2 for d_h = 64)
+//                   flight) and K/V chunks of CK keys (8 stages for d_h = 32,
+//                   4 for d_h = 64)
 //   warp 1 lane 0 : tcgen05.mma -- S_j = Q K_j^T into TMEM tile j % 2, then
 //                   PV_j = P_j V_j with P_j read from that same TMEM tile
 //                   into PV buffer j % 2
 //   warps 2..     : online softmax from TMEM, one query row per lane; with
 //                   d_h = 64, warps w and w+4 share TMEM lane quadrant w % 4
 //                   and each take half of the chunk's keys and half of the
-//                   output columns.  P_j is written back over S_j as split
-//                   bf16 pairs; PV_{j-1} is folded into the register output
-//                   after P_j is handed over, so the softmax never waits for
-//                   the PV product of the chunk it has just finished
-// Operands are split pairs (hi + lo bf16): S = Qh Kh + Ql Kh + Qh Kl and
-// PV = Ph Vh + Pl Vh + Ph Vl, fp32 accumulation; softmax in fp32.
+//                   output columns.  P_j is written back over S_j as f16;
+//                   PV_{j-1} is folded into the register output after P_j is
+//                   handed over, so the softmax never waits for the PV
+//                   product of the chunk it has just finished
+// Q, K, V and P are single f16 planes (unit roundoff 2^-11; Q and K come
+// from LayerNorm'd rows times weights of magnitude well inside the f16
+// range, P lies in [0, 1]); accumulation, softmax statistics and the output
+// are fp32, the output leaves as a bf16 hi/lo pair.
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -44,13 +46,12 @@ struct AttnCfg {
   // TMEM: S/P tiles at [0, CK) and [CK, 2CK), PV buffers at [2CK, 2CK + 2DH)
   static constexpr uint32_t kTmemCols = DH == 32 ? 256 : 512;
   static constexpr uint32_t kRowBytes = DH * 2;                 // one row of a Q/K/V tile
-  static constexpr uint32_t kTile = 128 * kRowBytes;            // Q tile: 128 rows, one plane
-  static constexpr uint32_t kKVTile = CK * kRowBytes;           // K or V chunk: CK rows, one plane
+  static constexpr uint32_t kQBytes = 128 * kRowBytes;          // Q tile: 128 rows
+  static constexpr uint32_t kKVTile = CK * kRowBytes;           // K or V chunk: CK rows
   static constexpr uint32_t kSwz = DH == 32 ? 4u : 2u;          // descriptor swizzle code (64 B / 128 B)
   static constexpr uint32_t kSbo = 8 * kRowBytes;               // 8-row swizzle atom
-  static constexpr uint32_t kQBytes = 2 * kTile;                // hi + lo
-  static constexpr uint32_t kKVBytes = 4 * kKVTile;             // Kh Kl Vh Vl
-  static constexpr int kKVStages = DH == 32 ? 4 : 2;
+  static constexpr uint32_t kKVBytes = 2 * kKVTile;             // K, V
+  static constexpr int kKVStages = DH == 32 ? 8 : 4;
   static constexpr uint32_t kRed = 2 * 2 * 2 * 128 * 4;       // [max|sum][parity][half][row]
   static constexpr size_t kSmem = 1024 + 2 * kQBytes + kKVStages * kKVBytes + 256 + kRed;
 };
@@ -73,26 +74,24 @@ __device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
 
 template <int DH>
 __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM)
-    attn_kernel(const __grid_constant__ CUtensorMap tQh, const __grid_constant__ CUtensorMap tQl,
-                const __grid_constant__ CUtensorMap tKh, const __grid_constant__ CUtensorMap tKl,
-                const __grid_constant__ CUtensorMap tVh, const __grid_constant__ CUtensorMap tVl,
-                const AttnParams p) {
+    attn_kernel(const __grid_constant__ CUtensorMap tQ, const __grid_constant__ CUtensorMap tK,
+                const __grid_constant__ CUtensorMap tV, const AttnParams p) {
   using Cfg = AttnCfg<DH>;
   constexpr int CK = Cfg::CK;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_s = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
-  uint8_t* sQ = smem;                                   // [2 buffers][hi, lo]
-  uint8_t* sKV = sQ + 2 * Cfg::kQBytes;                 // [stages][Kh, Kl, Vh, Vl]
+  uint8_t* sQ = smem;                                   // [2 buffers]
+  uint8_t* sKV = sQ + 2 * Cfg::kQBytes;                 // [stages][K, V]
   uint64_t* bars = reinterpret_cast<uint64_t*>(sKV + Cfg::kKVStages * Cfg::kKVBytes);
   uint64_t* q_full = bars;        // [2]
   uint64_t* q_empty = bars + 2;   // [2]
   uint64_t* kv_full = bars + 4;   // [stages]
-  uint64_t* kv_empty = bars + 8;  // [stages]
-  uint64_t* s_full = bars + 12;   // [2] S_j complete in TMEM tile j % 2
-  uint64_t* p_full = bars + 14;   // [2] P_j written over S_j
-  uint64_t* pv_full = bars + 16;  // [2] PV_j complete in PV buffer j % 2
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+  uint64_t* kv_empty = bars + 12; // [stages]
+  uint64_t* s_full = bars + 20;   // [2] S_j complete in TMEM tile j % 2
+  uint64_t* p_full = bars + 22;   // [2] P_j written over S_j
+  uint64_t* pv_full = bars + 24;  // [2] PV_j complete in PV buffer j % 2
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 26);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // row-statistic exchange
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -114,9 +113,9 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       mbar_init(kv_empty + i, 1);
     }
     fence_mbar_init();
-    prefetch_tmap(&tQh);
-    prefetch_tmap(&tKh);
-    prefetch_tmap(&tVh);
+    prefetch_tmap(&tQ);
+    prefetch_tmap(&tK);
+    prefetch_tmap(&tV);
   }
   if (warp == 0) tmem_alloc(tmem_slot, Cfg::kTmemCols);
   tc_fence_before();
@@ -151,8 +150,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         if (ui >= 2 && !mbar_wait_bounded(q_empty + qb, ((ui >> 1) - 1) & 1, p.status)) break;
         uint8_t* q = sQ + qb * Cfg::kQBytes;
         mbar_arrive_expect_tx(q_full + qb, Cfg::kQBytes);
-        tma_load_2d(q, &tQh, p.q_col + h * DH, qoff + q0, q_full + qb);
-        tma_load_2d(q + Cfg::kTile, &tQl, p.q_col + h * DH, qoff + q0, q_full + qb);
+        tma_load_2d(q, &tQ, p.q_col + h * DH, qoff + q0, q_full + qb);
         for (int j = 0; j < nch; ++j, ++gc) {
           const int ks = gc % Cfg::kKVStages;
           if (gc >= Cfg::kKVStages &&
@@ -163,10 +161,8 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           uint8_t* kv = sKV + ks * Cfg::kKVBytes;
           const int row = b * p.kv_stride + j * CK;
           mbar_arrive_expect_tx(kv_full + ks, Cfg::kKVBytes);
-          tma_load_2d(kv, &tKh, p.k_col + h * DH, row, kv_full + ks);
-          tma_load_2d(kv + Cfg::kKVTile, &tKl, p.k_col + h * DH, row, kv_full + ks);
-          tma_load_2d(kv + 2 * Cfg::kKVTile, &tVh, p.v_col + h * DH, row, kv_full + ks);
-          tma_load_2d(kv + 3 * Cfg::kKVTile, &tVl, p.v_col + h * DH, row, kv_full + ks);
+          tma_load_2d(kv, &tK, p.k_col + h * DH, row, kv_full + ks);
+          tma_load_2d(kv + Cfg::kKVTile, &tV, p.v_col + h * DH, row, kv_full + ks);
         }
         ++ui;
       }
@@ -174,8 +170,8 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
-      const uint32_t idesc_s = umma_idesc_bf16(BQ, CK);
-      const uint32_t idesc_pv = umma_idesc_bf16(BQ, DH) | (1u << 16);  // B (V) is MN-major
+      const uint32_t idesc_s = umma_idesc_f16(BQ, CK);
+      const uint32_t idesc_pv = umma_idesc_f16(BQ, DH) | (1u << 16);  // B (V) is MN-major
       int ui = 0, gc = 0;
       bool ok = true;
       // S = Q K^T of global chunk gcc into TMEM tile gcc % 2, the unit's Q in buffer qb
@@ -188,16 +184,10 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         const uint32_t q = smem_u32(sQ + qb * Cfg::kQBytes);
         const uint32_t k = smem_u32(sKV + ks * Cfg::kKVBytes);
         const uint32_t dst = tmem + (uint32_t)((gcc & 1) * CK);
-        const uint64_t qh0 = desc_sw(q, Cfg::kSbo, Cfg::kSwz), ql0 = desc_sw(q + Cfg::kTile, Cfg::kSbo, Cfg::kSwz);
-        const uint64_t kh0 = desc_sw(k, Cfg::kSbo, Cfg::kSwz), kl0 = desc_sw(k + Cfg::kKVTile, Cfg::kSbo, Cfg::kSwz);
+        const uint64_t q0d = desc_sw(q, Cfg::kSbo, Cfg::kSwz), k0d = desc_sw(k, Cfg::kSbo, Cfg::kSwz);
 #pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          // (Qh, Kh), (Ql, Kh), (Qh, Kl)
-          const uint64_t qh = desc_adv(qh0, kk * 32), kh = desc_adv(kh0, kk * 32);
-          umma_bf16(dst, qh, kh, idesc_s, kk != 0 ? 1u : 0u);
-          umma_bf16(dst, desc_adv(ql0, kk * 32), kh, idesc_s, 1u);
-          umma_bf16(dst, qh, desc_adv(kl0, kk * 32), idesc_s, 1u);
-        }
+        for (int kk = 0; kk < DH / 16; ++kk)
+          umma_bf16(dst, desc_adv(q0d, kk * 32), desc_adv(k0d, kk * 32), idesc_s, kk != 0 ? 1u : 0u);
         umma_commit(s_full + (gcc & 1));
         return true;
       };
@@ -219,23 +209,17 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
             break;
           }
           tc_fence_after();
-          // PV_j: A = P_j from TMEM tile j % 2, where each key block of 64 holds
-          // its hi plane in 32 columns followed by its lo plane in 32 columns
+          // PV_j: A = P_j from TMEM tile j % 2, each key block of 64 as 32
+          // columns of f16 pairs at the start of its 64 S columns
           const int ks = gc % Cfg::kKVStages;
-          const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + 2 * Cfg::kKVTile);
+          const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile);
           const uint32_t pt = tmem + (uint32_t)((gc & 1) * CK);
           const uint32_t dst = tmem + (uint32_t)(2 * CK + (gc & 1) * DH);
-          const uint64_t vh0 = desc_sw(v, Cfg::kSbo, Cfg::kSwz), vl0 = desc_sw(v + Cfg::kKVTile, Cfg::kSbo, Cfg::kSwz);
+          const uint64_t v0d = desc_sw(v, Cfg::kSbo, Cfg::kSwz);
 #pragma unroll
-          for (int kk = 0; kk < CK / 16; ++kk) {
-            const uint32_t ph = pt + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8), pl = ph + 32;
-            const uint32_t vb = (uint32_t)kk * 16 * Cfg::kRowBytes;
-            // (Ph, Vh), (Pl, Vh), (Ph, Vl)
-            const uint64_t vh = desc_adv(vh0, vb);
-            umma_bf16_tmem_a(dst, ph, vh, idesc_pv, kk != 0 ? 1u : 0u);
-            umma_bf16_tmem_a(dst, pl, vh, idesc_pv, 1u);
-            umma_bf16_tmem_a(dst, ph, desc_adv(vl0, vb), idesc_pv, 1u);
-          }
+          for (int kk = 0; kk < CK / 16; ++kk)
+            umma_bf16_tmem_a(dst, pt + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8),
+                             desc_adv(v0d, (uint32_t)kk * 16 * Cfg::kRowBytes), idesc_pv, kk != 0 ? 1u : 0u);
           umma_commit(pv_full + (gc & 1));
           umma_commit(kv_empty + ks);
         }
@@ -314,15 +298,15 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           const float mn = fmaxf(m, mx);
           corr = ex2_approx(m - mn);
           m = mn;
-          // P = 2^(s * scale - m) as split bf16 pairs over this warp's 64 S
-          // columns (already in registers): hi plane of keys 2c, 2c+1 in
-          // column c, lo plane in column 32 + c; keys past kv_cnt get 0
+          // P = 2^(s * scale - m) as f16 over the first 32 of this warp's 64
+          // S columns (all 64 already in registers): keys 2c, 2c+1 in column
+          // c; keys past kv_cnt get 0
           const float sc = p.scale_log2, nm = -mn;
           float sum = 0.f;
           auto emit = [&](auto full) {
 #pragma unroll
             for (int hb = 0; hb < 2; ++hb) {
-              uint32_t hi[16], lo[16];
+              uint32_t pk[16];
 #pragma unroll
               for (int i = 0; i < 32; i += 2) {
                 const int k = 32 * hb + i;
@@ -333,10 +317,9 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
                   p1 = k + 1 < kvalid ? p1 : 0.f;
                 }
                 sum += p0 + p1;
-                split2_trunc(p0, p1, hi[i / 2], lo[i / 2]);
+                pk[i / 2] = pack_f16x2(p0, p1);
               }
-              tmem_st16_nowait(tile + (uint32_t)(16 * hb), hi);
-              tmem_st16_nowait(tile + (uint32_t)(32 + 16 * hb), lo);
+              tmem_st16_nowait(tile + (uint32_t)(16 * hb), pk);
             }
           };
           if (kvalid >= 64) emit(std::true_type{});
@@ -401,8 +384,7 @@ cudaError_t attn_prepare() {
   return e;
 }
 
-cudaError_t attn_launch(int dh, const CUtensorMap* q_h, const CUtensorMap* q_l, const CUtensorMap* k_h,
-                        const CUtensorMap* k_l, const CUtensorMap* v_h, const CUtensorMap* v_l, const AttnParams& p0,
+cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, const CUtensorMap* v, const AttnParams& p0,
                         cudaStream_t s) {
   if (p0.n_segments <= 0 || p0.max_q <= 0 || p0.kv_cnt <= 0) return cudaSuccess;
   AttnParams p = p0;
@@ -411,12 +393,12 @@ cudaError_t attn_launch(int dh, const CUtensorMap* q_h, const CUtensorMap* q_l, 
   const long long sms = g_attn_sms > 0 ? g_attn_sms : 148;
   if (dh == 32) {
     const long long grid = units < sms * AttnCfg<32>::kCtasPerSM ? units : sms * AttnCfg<32>::kCtasPerSM;
-    return launch_k(attn_kernel<32>, dim3((unsigned)grid), dim3(AttnCfg<32>::kThreads), AttnCfg<32>::kSmem, s, *q_h,
-                    *q_l, *k_h, *k_l, *v_h, *v_l, p);
+    return launch_k(attn_kernel<32>, dim3((unsigned)grid), dim3(AttnCfg<32>::kThreads), AttnCfg<32>::kSmem, s, *q, *k,
+                    *v, p);
   }
   const long long grid = units < sms * AttnCfg<64>::kCtasPerSM ? units : sms * AttnCfg<64>::kCtasPerSM;
-  return launch_k(attn_kernel<64>, dim3((unsigned)grid), dim3(AttnCfg<64>::kThreads), AttnCfg<64>::kSmem, s, *q_h,
-                  *q_l, *k_h, *k_l, *v_h, *v_l, p);
+  return launch_k(attn_kernel<64>, dim3((unsigned)grid), dim3(AttnCfg<64>::kThreads), AttnCfg<64>::kSmem, s, *q, *k,
+                  *v, p);
 }
 
 }  // namespace fe

@@ -4,6 +4,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <type_traits>
@@ -189,6 +190,19 @@ __device__ __forceinline__ uint32_t umma_idesc_bf16(int M, int N) {
          | (1u << 10)                    // B format bf16
          | ((uint32_t)(N >> 3) << 17)    // N / 8
          | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+
+// Instruction descriptor: kind::f16, A = B = f16, D = f32, both K-major.
+__device__ __forceinline__ uint32_t umma_idesc_f16(int M, int N) {
+  return (1u << 4)                       // D format f32 (A, B formats 0: f16)
+         | ((uint32_t)(N >> 3) << 17)    // N / 8
+         | ((uint32_t)(M >> 4) << 24);   // M / 16
+}
+
+// Two floats as an f16x2 word (x0 in the low half), round to nearest.
+__device__ __forceinline__ uint32_t pack_f16x2(float x0, float x1) {
+  __half2 h = __floats2half2_rn(x0, x1);
+  return *reinterpret_cast<uint32_t*>(&h);
 }
 
 __device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,

@@ -275,17 +275,27 @@ __global__ void __launch_bounds__(kThreads, 1)
               v[4 * j + 3] += bb.w;
             }
           }
-          uint32_t hi[16], lo[16];
+          if (p.relu) {
 #pragma unroll
-          for (int i = 0; i < 32; i += 2) {
-            float x0 = v[i], x1 = v[i + 1];
-            if (p.relu) {
-              x0 = fmaxf(x0, 0.f);
-              x1 = fmaxf(x1, 0.f);
-            }
-            split2(x0, x1, hi[i / 2], lo[i / 2]);
+            for (int i = 0; i < 32; ++i) v[i] = fmaxf(v[i], 0.f);
           }
-          stage_split(hi, lo, col, srow);
+          if (p.out_f16) {
+            // one f16 plane (an attention operand)
+            uint8_t* b = next_stage();
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
+              *reinterpret_cast<uint4*>(b + o) =
+                  make_uint4(pack_f16x2(v[8 * j], v[8 * j + 1]), pack_f16x2(v[8 * j + 2], v[8 * j + 3]),
+                             pack_f16x2(v[8 * j + 4], v[8 * j + 5]), pack_f16x2(v[8 * j + 6], v[8 * j + 7]));
+            }
+            issue(&tO_h, b, nullptr, nullptr, col, srow);
+          } else {
+            uint32_t hi[16], lo[16];
+#pragma unroll
+            for (int i = 0; i < 32; i += 2) split2(v[i], v[i + 1], hi[i / 2], lo[i / 2]);
+            stage_split(hi, lo, col, srow);
+          }
         }
       } else if (EPI == EPI_RESID_LN && BN <= 128) {
         // rows of at most 128 columns: each warp holds its (at most two) chunks of

@@ -62,6 +62,7 @@ struct GemmParams {
   int nacc;             // TMEM accumulators, 1 or 2 (chosen by gemm_launch)
   const float* bias;    // [N] or null
   int relu;
+  int out_f16;          // EPI_STORE: one f16 plane through o_h (attention operands) instead of bf16 hi/lo
   // EPI_RESID_LN (outputs through the o_x / o_h / o_l tensor maps)
   const float* resid;   // residual rows (ldr == 0: one row broadcast to every row)
   int ldr;
@@ -110,12 +111,14 @@ cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUt
                        cudaStream_t s);
 
 // ---------------------------------------------------------------------------
-// Flash-style multi-head attention over request segments (tcgen05, split-bf16
-// operands).  Segment b: query rows [q_off(b), q_off(b) + q_cnt(b)), key and
-// value rows [b * kv_stride, b * kv_stride + kv_cnt).  Head h reads columns
-// q_col + h*dh of Q, k_col + h*dh of K, v_col + h*dh of V and writes columns
-// o_col + h*dh of the output planes.  The Q/K/V tensor maps have boxes of
-// dh x 128 with the 64-byte (dh = 32) or 128-byte (dh = 64) swizzle.
+// Flash-style multi-head attention over request segments (tcgen05, f16
+// operands, fp32 accumulation and softmax).  Segment b: query rows
+// [q_off(b), q_off(b) + q_cnt(b)), key and value rows
+// [b * kv_stride, b * kv_stride + kv_cnt).  Head h reads columns q_col + h*dh
+// of Q, k_col + h*dh of K, v_col + h*dh of V (each one f16 plane) and writes
+// columns o_col + h*dh of the bf16 hi/lo output planes.  The Q map has boxes
+// of dh x 128, the K/V maps dh x (64 for dh = 32, else 128), with the 64-byte
+// (dh = 32) or 128-byte (dh = 64) swizzle.
 // ---------------------------------------------------------------------------
 struct AttnParams {
   int n_segments, n_heads;
@@ -134,8 +137,7 @@ struct AttnParams {
   int* status;
 };
 cudaError_t attn_prepare();
-cudaError_t attn_launch(int dh, const CUtensorMap* q_h, const CUtensorMap* q_l, const CUtensorMap* k_h,
-                        const CUtensorMap* k_l, const CUtensorMap* v_h, const CUtensorMap* v_l, const AttnParams& p,
+cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, const CUtensorMap* v, const AttnParams& p,
                         cudaStream_t s);
 
 // ---------------------------------------------------------------------------
