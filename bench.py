@@ -64,20 +64,22 @@ def describe(w):
 
 
 # ----------------------------------------------------------------------------------------------
-# algorithmic work per launch site (flops, bytes); split activations are 4 B/element
+# algorithmic work per launch site (flops, bytes); split activations are 4 B/element, the
+# single-plane f16 attention operands (context K/V, element Q, cross Q/K/V) 2 B/element
 # ----------------------------------------------------------------------------------------------
 def site_work(site, cfg, B, C, M, K, L, R):
     d, F, Ly = cfg.d, cfg.F, cfg.n_layers
     S, n = B * K, B * C
     esz = 2 if cfg.io_bf16 else 4
     A = 4
+    H = 2
     t = {
         "compact": (0, 4 * B * K * L * 2 + 4 * R + 12 * B),
         "ctx_ln": (0, n * d * (esz + A)),
-        "gemm_ctx_kv": (2 * n * d * 2 * Ly * d, n * d * A + n * 2 * Ly * d * A),
+        "gemm_ctx_kv": (2 * n * d * 2 * Ly * d, n * d * A + n * 2 * Ly * d * H),
         "gather_ln": (0, R * d * (esz + 4 + A)),
-        "gemm_item_q": (2 * R * d * d, 2 * R * d * A),
-        "attn_item_ctx": (4 * R * C * d, 2 * R * d * A + 2 * n * d * A),
+        "gemm_item_q": (2 * R * d * d, R * d * A + R * d * H),
+        "attn_item_ctx": (4 * R * C * d, R * d * (H + A) + 2 * n * d * H),
         "gemm_item_o_ln": (2 * R * d * d, R * d * (A + 8 + A)),
         "gemm_item_ffn1": (2 * R * d * F, R * d * A + R * F * A),
         "gemm_item_ffn2_ln": (2 * R * F * d, R * F * A + R * d * (8 + A)),
@@ -88,8 +90,8 @@ def site_work(site, cfg, B, C, M, K, L, R):
         "gemm_seq_ffn1": (2 * S * d * F, S * d * A + S * F * A),
         "gemm_seq_ffn2_ln": (2 * S * F * d, S * F * A + S * d * (8 + A)),
         "ffn_seq": (4 * S * d * F, S * d * (A + 8 + A)),
-        "gemm_cross_qkv": (6 * S * d * d, S * d * A + 3 * S * d * A),
-        "attn_cross_seq": (4 * B * K * K * d, 3 * S * d * A + S * d * A),
+        "gemm_cross_qkv": (6 * S * d * d, S * d * A + 3 * S * d * H),
+        "attn_cross_seq": (4 * B * K * K * d, 3 * S * d * H + S * d * A),
         "gemm_cross_o_ln": (2 * S * d * d, S * d * (A + 8 + A)),
         "gemm_head": (2 * S * d * d + 3 * S * d, S * d * A + 4 * S),
         "select": (0, 4 * S + 4 * B),
@@ -397,9 +399,10 @@ def run_ours(args):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": describe(w), "global_batch": world * B, "K": K, "L": L,
                        "parallelism": f"dp{world} (requests sharded, no collective)",
-                       "precision": "bf16 MMA operands, activations split hi+lo bf16, fp32 accumulate",
+                       "precision": "bf16 MMA operands with activations split hi+lo bf16; attention Q, K, V, "
+                                    "P single f16; fp32 accumulate, softmax, LayerNorm and residuals",
                        "l2": f"inputs rotate over {n_copies} copies ({n_copies * in_bytes / 2**20:.0f} MB) "
-                             f"and each step writes {B * C * 2 * cfg.n_layers * cfg.d * 4 / 2**20:.0f} MB "
+                             f"and each step writes {B * C * 2 * cfg.n_layers * cfg.d * 2 / 2**20:.0f} MB "
                              f"of context K/V: > L2",
                        "sum_U": sumU, "U_mean": sumU / B, "rho": K * L * B / max(sumU, 1)},
             "seq_per_s": value * K, "p50_ms": p50, "p90_ms": p90,
