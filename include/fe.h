@@ -160,7 +160,8 @@ int fe_debug_layout(fe_ctx* ctx, int32_t* slot_out, int32_t* U_out);
  * Test hook: copy an intermediate of the last batch to host memory as fp32,
  * row-major.  `name` is one of:
  *   "ctx_ln"  [B*C, d]      LN(context)
- *   "ctx_kv"  [B*C, 2*n_layers*d]  K_0 | V_0 | K_1 | V_1 ...
+ *   "ctx_kv"  [B*C, 2*n_layers*d]  K_0 | V_0 | K_1 | V_1 ... (held as f16, the
+ *                           attention operand precision)
  *   "elem"    [sum U, d]    H, the final element representations, requests in
  *                           order, each request's elements in ascending pool index
  *   "seq"     [B*K, d]      c_k, the SeqEnc output
