@@ -77,6 +77,7 @@ def site_work(site, cfg, B, C, M, K, L, R):
         "compact": (0, 4 * B * K * L * 2 + 4 * R + 12 * B),
         "ctx_ln": (0, n * d * (esz + A)),
         "gemm_ctx_kv": (2 * n * d * 2 * Ly * d, n * d * A + n * 2 * Ly * d * H),
+        "ctx_ln_kv": (2 * n * d * 2 * Ly * d, n * d * esz + n * 2 * Ly * d * H),
         "gather_ln": (0, R * d * (esz + 4 + A)),
         "gemm_item_q": (2 * R * d * d, R * d * A + R * d * H),
         "attn_item_ctx": (4 * R * C * d, R * d * (H + A) + 2 * n * d * H),

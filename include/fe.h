@@ -159,7 +159,10 @@ int fe_debug_layout(fe_ctx* ctx, int32_t* slot_out, int32_t* U_out);
 /*
  * Test hook: copy an intermediate of the last batch to host memory as fp32,
  * row-major.  `name` is one of:
- *   "ctx_ln"  [B*C, d]      LN(context)
+ *   "ctx_ln"  [B*C, d]      LN(context); only where it is materialised: with
+ *                           d <= 128, bf16 inputs and bf16-exact weights the
+ *                           context LayerNorm and K/V projection run as one
+ *                           kernel and this name returns FE_ERR_UNSUPPORTED
  *   "ctx_kv"  [B*C, 2*n_layers*d]  K_0 | V_0 | K_1 | V_1 ... (held as f16, the
  *                           attention operand precision)
  *   "elem"    [sum U, d]    H, the final element representations, requests in

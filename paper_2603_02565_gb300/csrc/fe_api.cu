@@ -197,6 +197,8 @@ struct fe_ctx {
   int device = 0;
   int d = 0, H = 0, dh = 0, Ly = 0, F = 0, dpad = 0, Fpad = 0, nb = 1;
   bool fused_ffn = false;  // FFN1 + FFN2 in one kernel (d <= 128)
+  bool fused_ctxkv = false;  // context LN + K/V projection in one kernel (d <= 128, bf16 inputs)
+  CUtensorMap ctxkv_w{};     // W^T of the K/V projection, 64 x 128 boxes, for the fused kernel
   std::vector<void*> owned_w;  // weight allocations
   std::vector<void*> owned_ws; // workspace allocations
   float* w32 = nullptr;        // every weight in fp32, fe_weight_count order
@@ -449,11 +451,22 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
                            s));
   }
   // (a1) context keys/values, once per request
-  {
-    Prof pf(c, "ctx_ln", s);
-    FE_CK(fe::ctx_ln_launch(io.ctx, io_f32, B * C, d, c->cfg.ln_eps, c->X.h, c->X.l, c->X.ld, s));
-  }
-  {
+  if (c->fused_ctxkv) {
+    CUtensorMap tx{};
+    FE_RC(encode_map(&tx, static_cast<const bf16*>(io.ctx), d, B * C, 128));
+    fe::CtxKvParams p{};
+    p.rows = B * C;
+    p.d = d;
+    p.N = 2 * Ly * d;
+    p.eps = c->cfg.ln_eps;
+    p.status = c->status;
+    Prof pf(c, "ctx_ln_kv", s);
+    FE_CK(fe::ctxkv_launch(&tx, &c->ctxkv_w, &c->KV.sh, c->dpad, p, s));
+  } else {
+    {
+      Prof pf(c, "ctx_ln", s);
+      FE_CK(fe::ctx_ln_launch(io.ctx, io_f32, B * C, d, c->cfg.ln_eps, c->X.h, c->X.l, c->X.ld, s));
+    }
     fe::GemmParams p{};
     p.out_f16 = 1;
     FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, &c->KV, nullptr, s));
@@ -683,7 +696,7 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->in_idx, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int32_t)));
   FE_RC(dalloc((void**)&c->out_scores, (size_t)S * sizeof(float)));
   FE_RC(dalloc((void**)&c->out_best, (size_t)B * sizeof(int32_t)));
-  FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
+  if (!c->fused_ctxkv) FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->KV, BC, 2 * Ly * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->xln, R, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->q, R, d, false, c->owned_ws));
@@ -697,8 +710,8 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(alloc_planes(c->qkv, S, 3 * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->ax, S, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->lncp, S, c->dpad, true, c->owned_ws));
-  for (Planes* p : {&c->X, &c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp})
-    FE_RC(map_act(*p));
+  if (!c->fused_ctxkv) FE_RC(map_act(c->X));
+  for (Planes* p : {&c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp}) FE_RC(map_act(*p));
   for (Planes* p : {&c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->lncp}) FE_RC(map_out(*p));
   for (Planes* p : {&c->KV, &c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
   c->cap_shape = s;
@@ -836,7 +849,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   };
   int rc = FE_OK;
   if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess ||
-      fe::ffn_prepare() != cudaSuccess)
+      fe::ffn_prepare() != cudaSuccess || fe::ctxkv_prepare() != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "kernel attributes"));
   {
     size_t o = 0;
@@ -855,6 +868,9 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     if ((rc = fill_weight(c->ctx_kv, lw(c, l, T_WK), d, d, 2 * l * d)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->ctx_kv, lw(c, l, T_WV), d, d, (2 * l + 1) * d)) != FE_OK) return fail(rc);
   }
+  c->fused_ctxkv = fe::ctxkv_supported(d, c->dpad, 2 * Ly * d, c->nb, c->cfg.io_dtype == FE_IO_F32);
+  if (c->fused_ctxkv && (rc = encode_map(&c->ctxkv_w, c->ctx_kv.p.h, c->ctx_kv.p.ld, c->ctx_kv.p.rows, 128)) != FE_OK)
+    return fail(rc);
   c->wq.resize(Ly);
   c->wo.resize(Ly);
   c->w1.resize(Ly);
@@ -1029,6 +1045,10 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
   size_t rows = 0, cols = 0;
   const std::string n(name);
   if (n == "ctx_ln") {
+    if (c->fused_ctxkv) {
+      g_msg = "ctx_ln is not materialised: the fused context kernel keeps LN(context) on chip";
+      return FE_ERR_UNSUPPORTED;
+    }
     pl = &c->X;
     rows = (size_t)s.B * s.C;
     cols = d;

@@ -111,6 +111,23 @@ cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUt
                        cudaStream_t s);
 
 // ---------------------------------------------------------------------------
+// Context LayerNorm + K/V projection in one kernel (d <= 128, bf16 inputs,
+// bf16-exact weights, N = 2 * n_layers * d in {256, 512}).
+// x: raw context rows [rows, d] bf16, 64 x 128 boxes, 128-byte swizzle;
+// w: W^T [N, d_pad] bf16, 64 x 128 boxes, 128-byte swizzle;
+// o: the f16 K/V rows [rows, N], 32 x 32 boxes, 64-byte swizzle.
+// ---------------------------------------------------------------------------
+struct CtxKvParams {
+  int rows, d, N;
+  float eps;
+  int* status;
+};
+bool ctxkv_supported(int d, int d_pad, int N, int nb, int io_f32);
+cudaError_t ctxkv_prepare();
+cudaError_t ctxkv_launch(const CUtensorMap* x, const CUtensorMap* w, const CUtensorMap* o, int d_pad,
+                         const CtxKvParams& p, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
 // Flash-style multi-head attention over request segments (tcgen05, f16
 // operands, fp32 accumulation and softmax).  Segment b: query rows
 // [q_off(b), q_off(b) + q_cnt(b)), key and value rows
