@@ -376,8 +376,12 @@ __global__ void __launch_bounds__(256) cls_attn_kernel(const ClsParams p) {
   const int L = p.bad[b] ? 0 : p.L;
   const int base = p.off[b];
   const int* sl = p.slot_local + (size_t)seq * p.L;
+  // lane j holds slot j (one load for the first 32 keys), so a key's rows are
+  // requested without first waiting for its slot index
+  const int my_slot = lane < L ? sl[lane] : 0;
   for (int j = 0; j < L; ++j) {
-    const size_t row = (size_t)(base + sl[j]) * p.ldkv;
+    const int slot = j < 32 ? __shfl_sync(0xffffffffu, my_slot, j) : sl[j];
+    const size_t row = (size_t)(base + slot) * p.ldkv;
     float kp[DPL], vp[DPL];
     load_split<DPL>(p.kv_h + row + d0, p.kv_l + row + d0, kx);
     load_split<DPL>(p.kv_h + row + d + d0, p.kv_l + row + d + d0, vx);
