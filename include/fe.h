@@ -149,6 +149,31 @@ int fe_evaluate_host(fe_ctx* ctx, int B, int C, int M, int K, int L,
                      float* scores_out, int32_t* best_out, void* stream);
 
 /*
+ * Pipelined form of fe_evaluate_host for serving loops whose inputs arrive in
+ * host memory.  fe_submit_host enqueues one batch and returns at once: the
+ * inputs are copied to one of two library-owned device staging slots on the
+ * library's own copy stream, the batch runs on the library's own compute
+ * stream once its copy is complete, and scores/best are copied back into the
+ * caller's host buffers.  The copy of one batch therefore overlaps the
+ * evaluation of the previous one; every batch still moves its own inputs and
+ * results across the host link.  fe_wait_host waits for the oldest
+ * outstanding submission and returns its batch status (as fe_evaluate).
+ * At most two submissions may be outstanding (a third returns
+ * FE_ERR_INVALID_ARG); the host buffers of a submission must stay valid and
+ * unchanged until its fe_wait_host returns (page-locked buffers for overlap).
+ * While submissions are outstanding, fe_evaluate, fe_evaluate_async and
+ * fe_evaluate_host return FE_ERR_INVALID_ARG (they share the workspace), and a
+ * batch larger than the reserved workspace is refused until every submission
+ * has been waited for.  Same shapes, types and status codes as fe_evaluate.
+ * The paper evaluates one request batch at a time; this overlap of transfer
+ * and compute across batches is the library's own.
+ */
+int fe_submit_host(fe_ctx* ctx, int B, int C, int M, int K, int L,
+                   const void* context, const void* pool, const int32_t* cand_idx,
+                   float* scores_out, int32_t* best_out);
+int fe_wait_host(fe_ctx* ctx);
+
+/*
  * Test hook: the distinct-element layout of the last evaluated batch, copied
  * to host memory.  U_out[B] = |U(z_b)| (Section 4.1); slot_out[B,K,L] = rank of
  * cand_idx[b,k,j] among the distinct indices of request b in ascending order

@@ -28,7 +28,8 @@ FE_IO_BF16 = 0
 FE_IO_F32 = 1
 
 EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evaluate_async", "fe_last_status",
-           "fe_evaluate_host", "fe_debug_layout", "fe_debug_fetch", "fe_profile", "fe_profile_read",
+           "fe_evaluate_host", "fe_submit_host", "fe_wait_host", "fe_debug_layout", "fe_debug_fetch", "fe_profile",
+           "fe_profile_read",
            "fe_kernels_per_batch", "fe_distinct_layout_noalloc", "fe_destroy", "fe_strerror",
            "fe_last_error_message"]
 
@@ -69,6 +70,10 @@ def load_library(path: str = LIB_PATH):
         f.restype = i32
     L.fe_last_status.argtypes = [vp]
     L.fe_last_status.restype = i32
+    L.fe_submit_host.argtypes = [vp, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp]
+    L.fe_submit_host.restype = i32
+    L.fe_wait_host.argtypes = [vp]
+    L.fe_wait_host.restype = i32
     L.fe_debug_layout.argtypes = [vp, vp, vp]
     L.fe_debug_layout.restype = i32
     L.fe_debug_fetch.argtypes = [vp, ctypes.c_char_p, vp, sz, ctypes.POINTER(sz)]
@@ -213,6 +218,28 @@ class Evaluator:
                                              hp(scores), hp(best), ctypes.c_void_p(stream))
         self.last_status = _check(rc, allowed)
         return scores, best
+
+    def submit_host(self, context, pool, cand_idx, scores, best):
+        """Pipelined host entry: enqueue one batch whose buffers live in host memory
+        and return at once (fe_submit_host).  scores [B, K] float32 and best [B]
+        int32 are host buffers the results are copied into; every buffer must stay
+        alive and unchanged until the matching wait_host() returns."""
+        B, C, _ = context.shape
+        M = pool.shape[1]
+        K, L = cand_idx.shape[1], cand_idx.shape[2]
+
+        def hp(a):
+            if hasattr(a, "data_ptr"):
+                return ctypes.c_void_p(a.data_ptr())
+            return ctypes.c_void_p(a.ctypes.data)
+
+        _check(load_library().fe_submit_host(self._h, B, C, M, K, L, hp(context), hp(pool), hp(cand_idx),
+                                             hp(scores), hp(best)))
+
+    def wait_host(self, allowed=(FE_OK, FE_ERR_INDEX, FE_ERR_NUMERIC)):
+        """Wait for the oldest outstanding submit_host batch; returns its status."""
+        self.last_status = _check(load_library().fe_wait_host(self._h), allowed)
+        return self.last_status
 
     # -- tracing ----------------------------------------------------------------------
     def profile(self, enable: bool):

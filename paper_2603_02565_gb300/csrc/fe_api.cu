@@ -177,9 +177,24 @@ struct IoPtrs {
   const int32_t* idx;
   float* scores;
   int32_t* best;
+  int* hstatus;  // page-locked word that receives the batch status
   bool operator==(const IoPtrs& o) const {
-    return ctx == o.ctx && pool == o.pool && idx == o.idx && scores == o.scores && best == o.best;
+    return ctx == o.ctx && pool == o.pool && idx == o.idx && scores == o.scores && best == o.best &&
+           hstatus == o.hstatus;
   }
+};
+
+// One staging slot of the pipelined host entry (fe_submit_host): device copies
+// of a batch's inputs and outputs, its status word and its events.
+struct HostSlot {
+  void* ctx = nullptr;
+  void* pool = nullptr;
+  int32_t* idx = nullptr;
+  float* scores = nullptr;
+  int32_t* best = nullptr;
+  int* hstatus = nullptr;      // page-locked
+  cudaEvent_t in_ev = nullptr;   // inputs copied in
+  cudaEvent_t done_ev = nullptr; // batch and copy-out complete (the slot is free again)
 };
 
 struct GraphEntry {
@@ -223,6 +238,11 @@ struct fe_ctx {
   int* host_status = nullptr;  // page-locked
   cudaEvent_t done_ev = nullptr;
   cudaStream_t cap_stream = nullptr;
+  // pipelined host entry: two slots, a copy-in stream and a compute stream
+  HostSlot slots[2];
+  cudaStream_t copy_stream = nullptr, sub_stream = nullptr;
+  int next_slot = 0;       // slot of the next submission; slots alternate
+  int n_outstanding = 0;   // submissions not yet waited for (the oldest is next_slot - n_outstanding)
   std::vector<GraphEntry> graphs;
   unsigned long long use_clock = 0;
   bool use_graph = true;
@@ -439,7 +459,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   FE_CK(cudaMemsetAsync(c->status, 0, sizeof(int), s));
   if (K == 0) {
     FE_CK(cudaMemsetAsync(io.best, 0xFF, (size_t)B * sizeof(int32_t), s));
-    FE_CK(cudaMemcpyAsync(c->host_status, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+    FE_CK(cudaMemcpyAsync(io.hstatus, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
     return FE_OK;
   }
   const int* sumU = c->off + B;  // device: number of distinct elements of the batch
@@ -622,7 +642,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     Prof pf(c, "select", s);
     FE_CK(fe::select_launch(io.scores, B, K, c->bad, io.best, c->status, s));
   }
-  FE_CK(cudaMemcpyAsync(c->host_status, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  FE_CK(cudaMemcpyAsync(io.hstatus, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
   c->launches_last = c->launches_batch;
   return FE_OK;
 }
@@ -696,6 +716,17 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->in_idx, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int32_t)));
   FE_RC(dalloc((void**)&c->out_scores, (size_t)S * sizeof(float)));
   FE_RC(dalloc((void**)&c->out_best, (size_t)B * sizeof(int32_t)));
+  // pipelined host entry: slot 0 uses the staging above, slot 1 its own copy
+  c->slots[0].ctx = c->in_ctx;
+  c->slots[0].pool = c->in_pool;
+  c->slots[0].idx = c->in_idx;
+  c->slots[0].scores = c->out_scores;
+  c->slots[0].best = c->out_best;
+  FE_RC(dalloc(&c->slots[1].ctx, (size_t)BC * d * esz));
+  FE_RC(dalloc(&c->slots[1].pool, (size_t)B * (s.M > 0 ? s.M : 1) * d * esz));
+  FE_RC(dalloc((void**)&c->slots[1].idx, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int32_t)));
+  FE_RC(dalloc((void**)&c->slots[1].scores, (size_t)S * sizeof(float)));
+  FE_RC(dalloc((void**)&c->slots[1].best, (size_t)B * sizeof(int32_t)));
   if (!c->fused_ctxkv) FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->KV, BC, 2 * Ly * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->xln, R, c->dpad, true, c->owned_ws));
@@ -786,6 +817,16 @@ int check_io(const void* ctx, const void* pool, const int32_t* idx, const float*
   auto mis = [](const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u); };
   if (mis(ctx) || mis(pool) || mis(idx) || mis(scores) || mis(best)) {
     g_msg = "buffers must be 16-byte aligned";
+    return FE_ERR_INVALID_ARG;
+  }
+  return FE_OK;
+}
+
+// The workspace is shared by every call: while pipelined host submissions are
+// in flight, no other evaluation may be enqueued.
+int no_outstanding(fe_ctx* c) {
+  if (c->n_outstanding > 0) {
+    g_msg = "host submissions are outstanding: call fe_wait_host first";
     return FE_ERR_INVALID_ARG;
   }
   return FE_OK;
@@ -927,8 +968,17 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if (cudaMallocHost(&c->host_status, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
   *c->host_status = 0;
   if (cudaEventCreateWithFlags(&c->done_ev, cudaEventDisableTiming) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess)
+      cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&c->sub_stream, cudaStreamNonBlocking) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "stream/event"));
+  for (HostSlot& hs : c->slots) {
+    if (cudaMallocHost(&hs.hstatus, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
+    *hs.hstatus = 0;
+    if (cudaEventCreateWithFlags(&hs.in_ev, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&hs.done_ev, cudaEventDisableTiming) != cudaSuccess)
+      return fail(set_cuda_err(cudaGetLastError(), "stream/event"));
+  }
   cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return fail(set_cuda_err(e, "fe_init"));
   *out = c;
@@ -946,6 +996,7 @@ int fe_evaluate_async(fe_ctx* c, int B, int C, int M, int K, int L, const void* 
                       const int32_t* cand_idx, float* scores_out, int32_t* best_out, void* stream) {
   if (!c) return FE_ERR_INVALID_ARG;
   DeviceGuard g(c->device);
+  FE_RC(no_outstanding(c));
   FE_RC(check_shape(c, B, C, M, K, L));
   FE_RC(check_io(context, pool, cand_idx, scores_out, best_out, B, M, K, L));
   if (B == 0) {
@@ -954,7 +1005,7 @@ int fe_evaluate_async(fe_ctx* c, int B, int C, int M, int K, int L, const void* 
     return FE_OK;
   }
   Shape s{B, C, M, K, L};
-  IoPtrs io{context, pool, cand_idx, scores_out, best_out};
+  IoPtrs io{context, pool, cand_idx, scores_out, best_out, c->host_status};
   return launch_batch(c, s, io, (cudaStream_t)stream);
 }
 
@@ -974,6 +1025,7 @@ int fe_evaluate_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* c
                      const int32_t* cand_idx, float* scores_out, int32_t* best_out, void* stream) {
   if (!c) return FE_ERR_INVALID_ARG;
   DeviceGuard g(c->device);
+  FE_RC(no_outstanding(c));
   FE_RC(check_shape(c, B, C, M, K, L));
   if (B == 0) return FE_OK;
   if (!context || !best_out || (K > 0 && !scores_out) || (K * L > 0 && !cand_idx) || (K * L > 0 && M > 0 && !pool)) {
@@ -989,12 +1041,80 @@ int fe_evaluate_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* c
     FE_CK(cudaMemcpyAsync(c->in_pool, pool, (size_t)B * M * c->d * esz, cudaMemcpyHostToDevice, st));
   if (K * L > 0)
     FE_CK(cudaMemcpyAsync(c->in_idx, cand_idx, (size_t)B * K * L * sizeof(int32_t), cudaMemcpyHostToDevice, st));
-  IoPtrs io{c->in_ctx, c->in_pool, c->in_idx, c->out_scores, c->out_best};
+  IoPtrs io{c->in_ctx, c->in_pool, c->in_idx, c->out_scores, c->out_best, c->host_status};
   FE_RC(launch_batch(c, s, io, st));
   if (K > 0) FE_CK(cudaMemcpyAsync(scores_out, c->out_scores, (size_t)B * K * sizeof(float), cudaMemcpyDeviceToHost, st));
   FE_CK(cudaMemcpyAsync(best_out, c->out_best, (size_t)B * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   FE_CK(cudaEventRecord(c->done_ev, st));
   return wait_status(c);
+}
+
+int fe_submit_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* context, const void* pool,
+                   const int32_t* cand_idx, float* scores_out, int32_t* best_out) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  FE_RC(check_shape(c, B, C, M, K, L));
+  if (!context || !best_out || (K > 0 && !scores_out) || (K * L > 0 && !cand_idx) || (K * L > 0 && M > 0 && !pool)) {
+    g_msg = "null pointer";
+    return FE_ERR_INVALID_ARG;
+  }
+  if (c->n_outstanding >= 2) {
+    g_msg = "two host submissions are outstanding: call fe_wait_host first";
+    return FE_ERR_INVALID_ARG;
+  }
+  Shape s{B, C, M, K, L};
+  if (!fits(c, s)) {
+    if (c->n_outstanding > 0) {
+      g_msg = "a larger batch needs more workspace: wait for the outstanding submissions first";
+      return FE_ERR_INVALID_ARG;
+    }
+    FE_RC(reserve_impl(c, s));
+  }
+  const int k = c->next_slot;
+  HostSlot& hs = c->slots[k];
+  if (B == 0) {
+    *hs.hstatus = 0;
+    FE_CK(cudaEventRecord(hs.done_ev, c->sub_stream));
+  } else {
+    // copy-in on its own stream, once this slot's previous batch is complete
+    const size_t esz = c->cfg.io_dtype == FE_IO_F32 ? 4 : 2;
+    FE_CK(cudaStreamWaitEvent(c->copy_stream, hs.done_ev, 0));
+    FE_CK(cudaMemcpyAsync(hs.ctx, context, (size_t)B * C * c->d * esz, cudaMemcpyHostToDevice, c->copy_stream));
+    if (M > 0 && pool)
+      FE_CK(cudaMemcpyAsync(hs.pool, pool, (size_t)B * M * c->d * esz, cudaMemcpyHostToDevice, c->copy_stream));
+    if (K * L > 0)
+      FE_CK(cudaMemcpyAsync(hs.idx, cand_idx, (size_t)B * K * L * sizeof(int32_t), cudaMemcpyHostToDevice,
+                            c->copy_stream));
+    FE_CK(cudaEventRecord(hs.in_ev, c->copy_stream));
+    // the batch and the copy-out on the compute stream
+    FE_CK(cudaStreamWaitEvent(c->sub_stream, hs.in_ev, 0));
+    IoPtrs io{hs.ctx, hs.pool, hs.idx, hs.scores, hs.best, hs.hstatus};
+    FE_RC(launch_batch(c, s, io, c->sub_stream));
+    if (K > 0)
+      FE_CK(cudaMemcpyAsync(scores_out, hs.scores, (size_t)B * K * sizeof(float), cudaMemcpyDeviceToHost,
+                            c->sub_stream));
+    FE_CK(cudaMemcpyAsync(best_out, hs.best, (size_t)B * sizeof(int32_t), cudaMemcpyDeviceToHost, c->sub_stream));
+    FE_CK(cudaEventRecord(hs.done_ev, c->sub_stream));
+  }
+  c->n_outstanding += 1;
+  c->next_slot ^= 1;
+  return FE_OK;
+}
+
+int fe_wait_host(fe_ctx* c) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  if (c->n_outstanding == 0) {
+    g_msg = "no host submission outstanding";
+    return FE_ERR_INVALID_ARG;
+  }
+  // the oldest outstanding submission: slots are used alternately
+  const int k = (c->next_slot + 2 - c->n_outstanding) % 2;
+  HostSlot& hs = c->slots[k];
+  c->n_outstanding -= 1;
+  FE_CK(cudaEventSynchronize(hs.done_ev));
+  FE_CK(cudaGetLastError());
+  return status_to_rc(*hs.hstatus);
 }
 
 int fe_debug_layout(fe_ctx* c, int32_t* slot_out, int32_t* U_out) {
@@ -1161,6 +1281,14 @@ int fe_destroy(fe_ctx* c) {
     if (c->host_status) cudaFreeHost(c->host_status);
     if (c->done_ev) cudaEventDestroy(c->done_ev);
     if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+    for (HostSlot& hs : c->slots) {
+      if (hs.done_ev) cudaEventSynchronize(hs.done_ev);
+      if (hs.in_ev) cudaEventDestroy(hs.in_ev);
+      if (hs.done_ev) cudaEventDestroy(hs.done_ev);
+      if (hs.hstatus) cudaFreeHost(hs.hstatus);
+    }
+    if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+    if (c->sub_stream) cudaStreamDestroy(c->sub_stream);
   }
   delete c;
   return FE_OK;
