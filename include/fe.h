@@ -149,6 +149,26 @@ int fe_evaluate_host(fe_ctx* ctx, int B, int C, int M, int K, int L,
                      float* scores_out, int32_t* best_out, void* stream);
 
 /*
+ * The candidate-factorized evaluation E^ind of the same model and weights
+ * (Appendix A.3: every candidate scored as if on its own).  Same arguments
+ * and outputs as fe_evaluate_async (it returns after enqueueing; the batch
+ * status comes from fe_last_status), and the same scores: only the cost
+ * structure changes.  The context K/V are recomputed for every candidate
+ * sequence (B*K*C context rows instead of B*C) and every occurrence of an
+ * element is encoded on its own (B*K*L element rows instead of the B*|U(z)|
+ * distinct ones); the SeqEnc, cross-sequence and head steps are unchanged.
+ * Timing it against fe_evaluate on the same batch measures T_joint / T_ind
+ * (Section 5.2 relates it to 1/rho, rho = K*L / |U(z)|).  Requires d <= 128,
+ * bf16 inputs and weights and C a multiple of 128 (else FE_ERR_UNSUPPORTED);
+ * the workspace it reserves (K-fold context K/V) stays allocated.  The layout
+ * hook (fe_debug_layout) then reports U_b = K*L and the identity slots
+ * (-1 for rejected requests).
+ */
+int fe_evaluate_factorized(fe_ctx* ctx, int B, int C, int M, int K, int L,
+                           const void* context, const void* pool, const int32_t* cand_idx,
+                           float* scores_out, int32_t* best_out, void* stream);
+
+/*
  * Pipelined form of fe_evaluate_host for serving loops whose inputs arrive in
  * host memory.  fe_submit_host enqueues one batch and returns at once: the
  * inputs are copied to one of two library-owned device staging slots on the

@@ -28,7 +28,8 @@ FE_IO_BF16 = 0
 FE_IO_F32 = 1
 
 EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evaluate_async", "fe_last_status",
-           "fe_evaluate_host", "fe_submit_host", "fe_wait_host", "fe_debug_layout", "fe_debug_fetch", "fe_profile",
+           "fe_evaluate_host", "fe_evaluate_factorized", "fe_submit_host", "fe_wait_host", "fe_debug_layout",
+           "fe_debug_fetch", "fe_profile",
            "fe_profile_read",
            "fe_kernels_per_batch", "fe_distinct_layout_noalloc", "fe_destroy", "fe_strerror",
            "fe_last_error_message"]
@@ -64,7 +65,7 @@ def load_library(path: str = LIB_PATH):
     L.fe_init.restype = i32
     L.fe_reserve.argtypes = [vp, i32, i32, i32, i32, i32]
     L.fe_reserve.restype = i32
-    for name in ("fe_evaluate", "fe_evaluate_async", "fe_evaluate_host"):
+    for name in ("fe_evaluate", "fe_evaluate_async", "fe_evaluate_host", "fe_evaluate_factorized"):
         f = getattr(L, name)
         f.argtypes = [vp, i32, i32, i32, i32, i32, vp, vp, vp, vp, vp, vp]
         f.restype = i32
@@ -162,9 +163,11 @@ class Evaluator:
 
     # -- evaluation -------------------------------------------------------------
     def evaluate(self, context, pool, cand_idx, scores=None, best=None, stream=None, sync=True,
-                 allowed=(FE_OK, FE_ERR_INDEX, FE_ERR_NUMERIC)):
+                 allowed=(FE_OK, FE_ERR_INDEX, FE_ERR_NUMERIC), factorized=False):
         """context [B,C,d], pool [B,M,d] (bf16 or fp32 per the config), cand_idx [B,K,L]
-        int32, all CUDA tensors.  Returns (scores [B,K] fp32, best [B] int32)."""
+        int32, all CUDA tensors.  Returns (scores [B,K] fp32, best [B] int32).
+        factorized=True runs the candidate-factorized evaluation E^ind
+        (fe_evaluate_factorized): same outputs, per-sequence cost structure."""
         import torch
         B, C, _ = context.shape
         M = pool.shape[1]
@@ -185,9 +188,11 @@ class Evaluator:
         if stream is None:
             stream = torch.cuda.current_stream(dev).cuda_stream
         Lb = load_library()
-        fn = Lb.fe_evaluate if sync else Lb.fe_evaluate_async
+        fn = Lb.fe_evaluate_factorized if factorized else (Lb.fe_evaluate if sync else Lb.fe_evaluate_async)
         rc = fn(self._h, B, C, M, K, L, _ptr(context), _ptr(pool), _ptr(cand_idx), _ptr(scores), _ptr(best),
                 ctypes.c_void_p(stream))
+        if factorized and sync and rc == FE_OK:
+            rc = Lb.fe_last_status(self._h)
         self.last_status = _check(rc, allowed)
         return scores, best
 

@@ -168,7 +168,10 @@ int largest_bn(int N, int cap) {
 
 struct Shape {
   int B = 0, C = 0, M = 0, K = 0, L = 0;
-  bool operator==(const Shape& o) const { return B == o.B && C == o.C && M == o.M && K == o.K && L == o.L; }
+  bool fact = false;  // candidate-factorized evaluation (fe_evaluate_factorized)
+  bool operator==(const Shape& o) const {
+    return B == o.B && C == o.C && M == o.M && K == o.K && L == o.L && fact == o.fact;
+  }
 };
 
 struct IoPtrs {
@@ -225,7 +228,9 @@ struct fe_ctx {
   float *q0 = nullptr, *k0 = nullptr, *v0 = nullptr, *kP = nullptr, *vP = nullptr;
   // workspace
   Shape cap_shape;  // reserved maxima
-  int cap_rows = 0; // B * min(M, K*L) of the reservation
+  int cap_rows = 0; // element rows of the reservation: B * min(M, K*L), or B * K * L once factorized
+  bool cap_fact = false;      // the reservation covers candidate-factorized batches
+  long long kv_rows = 0;      // context K/V rows of the reservation: B * C, or B * K * C
   int *status = nullptr, *U = nullptr, *off = nullptr, *bad = nullptr, *slot = nullptr, *list = nullptr;
   unsigned* ticket = nullptr;
   Planes X, KV, xln, q, a, mid, kvI, o, cln, mids, z, qkv, ax, lncp;
@@ -452,7 +457,8 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   const int B = sh.B, C = sh.C, M = sh.M, K = sh.K, L = sh.L;
   const int d = c->d, Ly = c->Ly;
   const int io_f32 = c->cfg.io_dtype == FE_IO_F32;
-  const int cap = (M < K * L) ? M : K * L;
+  const bool fact = sh.fact;  // every occurrence its own element, one context K/V per sequence
+  const int cap = fact ? K * L : ((M < K * L) ? M : K * L);
   const int R = B * cap;
   const int S = B * K;
   c->launches_batch = 0;
@@ -464,8 +470,11 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   }
   const int* sumU = c->off + B;  // device: number of distinct elements of the batch
 
-  // (a0) distinct-element compaction of every request
-  {
+  // (a0) distinct-element compaction of every request (factorized: the identity layout)
+  if (fact) {
+    Prof pf(c, "layout", s);
+    FE_CK(fe::identity_layout_launch(io.idx, B, M, K * L, c->U, c->off, c->bad, c->slot, c->list, c->status, s));
+  } else {
     Prof pf(c, "compact", s);
     FE_CK(fe::compact_launch(io.idx, B, M, K, L, cap, c->U, c->off, c->bad, c->slot, c->list, c->status, c->ticket,
                            s));
@@ -475,11 +484,13 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     CUtensorMap tx{};
     FE_RC(encode_map(&tx, static_cast<const bf16*>(io.ctx), d, B * C, 128));
     fe::CtxKvParams p{};
-    p.rows = B * C;
+    p.rows = B * C * (fact ? K : 1);  // factorized: the context of every sequence
     p.d = d;
     p.N = 2 * Ly * d;
     p.eps = c->cfg.ln_eps;
     p.status = c->status;
+    p.C = C;
+    p.rep = fact ? K : 1;
     Prof pf(c, "ctx_ln_kv", s);
     FE_CK(fe::ctxkv_launch(&tx, &c->ctxkv_w, &c->KV.sh, c->dpad, p, s));
   } else {
@@ -503,11 +514,18 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
 
     fe::AttnParams ap{};
-    ap.n_segments = B;
+    if (fact) {  // segment = one sequence: its L occurrences over its own context K/V
+      ap.n_segments = B * K;
+      ap.max_q = L;
+      ap.q_stride = L;
+      ap.q_cnt_fixed = L;
+    } else {
+      ap.n_segments = B;
+      ap.max_q = cap;
+      ap.q_off_dev = c->off;
+      ap.q_cnt_dev = c->U;
+    }
     ap.n_heads = c->H;
-    ap.max_q = cap;
-    ap.q_off_dev = c->off;
-    ap.q_cnt_dev = c->U;
     ap.kv_stride = C;
     ap.kv_cnt = C;
     ap.q_col = 0;
@@ -679,17 +697,23 @@ int reserve_impl(fe_ctx* c, Shape s) {
   s.M = std::max(s.M, c->cap_shape.M);
   s.K = std::max(s.K, c->cap_shape.K);
   s.L = std::max(s.L, c->cap_shape.L);
+  const bool fact = s.fact || c->cap_fact;
+  if (fact && ((long long)s.B * s.K * s.L > (1ll << 30) || (long long)s.B * s.K * s.C > (1ll << 30))) {
+    g_msg = "batch too large for the factorized evaluation";
+    return FE_ERR_UNSUPPORTED;
+  }
   FE_CK(cudaDeviceSynchronize());
   clear_graphs(c);
   free_list(c->owned_ws);
   c->have_last = false;
   const int d = c->d, Ly = c->Ly;
   const long long capL = (long long)s.K * s.L;
-  const int cap = (int)((s.M < capL) ? s.M : capL);
+  const int cap = (int)(fact ? capL : ((s.M < capL) ? s.M : capL));
   const int B = s.B > 0 ? s.B : 1;
   const int R = B * (cap > 0 ? cap : 1);
   const int S = B * (s.K > 0 ? s.K : 1);
   const int BC = B * s.C;
+  const long long kv_rows = (long long)BC * (fact && s.K > 0 ? s.K : 1);
   auto dalloc = [&](void** p, size_t bytes) -> int {
     if (bytes == 0) bytes = 16;
     if (cudaMalloc(p, bytes) != cudaSuccess) {
@@ -728,7 +752,7 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->slots[1].scores, (size_t)S * sizeof(float)));
   FE_RC(dalloc((void**)&c->slots[1].best, (size_t)B * sizeof(int32_t)));
   if (!c->fused_ctxkv) FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
-  FE_RC(alloc_planes(c->KV, BC, 2 * Ly * d, false, c->owned_ws));
+  FE_RC(alloc_planes(c->KV, (int)kv_rows, 2 * Ly * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->xln, R, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->q, R, d, false, c->owned_ws));
   FE_RC(alloc_planes(c->a, R, c->dpad, true, c->owned_ws));
@@ -746,13 +770,16 @@ int reserve_impl(fe_ctx* c, Shape s) {
   for (Planes* p : {&c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->lncp}) FE_RC(map_out(*p));
   for (Planes* p : {&c->KV, &c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
   c->cap_shape = s;
+  c->cap_shape.fact = false;
   c->cap_rows = R;
+  c->cap_fact = fact;
+  c->kv_rows = kv_rows;
   return FE_OK;
 }
 
 bool fits(const fe_ctx* c, const Shape& s) {
   const Shape& r = c->cap_shape;
-  return r.B > 0 && s.B <= r.B && s.C <= r.C && s.M <= r.M && s.K <= r.K && s.L <= r.L;
+  return r.B > 0 && s.B <= r.B && s.C <= r.C && s.M <= r.M && s.K <= r.K && s.L <= r.L && (!s.fact || c->cap_fact);
 }
 
 int launch_batch(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t stream) {
@@ -1019,6 +1046,28 @@ int fe_evaluate(fe_ctx* c, int B, int C, int M, int K, int L, const void* contex
                 const int32_t* cand_idx, float* scores_out, int32_t* best_out, void* stream) {
   FE_RC(fe_evaluate_async(c, B, C, M, K, L, context, pool, cand_idx, scores_out, best_out, stream));
   return fe_last_status(c);
+}
+
+int fe_evaluate_factorized(fe_ctx* c, int B, int C, int M, int K, int L, const void* context, const void* pool,
+                           const int32_t* cand_idx, float* scores_out, int32_t* best_out, void* stream) {
+  if (!c) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  FE_RC(no_outstanding(c));
+  FE_RC(check_shape(c, B, C, M, K, L));
+  FE_RC(check_io(context, pool, cand_idx, scores_out, best_out, B, M, K, L));
+  if (!c->fused_ctxkv || C % 128 != 0) {
+    g_msg = "the factorized evaluation needs d <= 128, bf16 inputs and weights, and C a multiple of 128";
+    return FE_ERR_UNSUPPORTED;
+  }
+  // with no pool row every index is out of range: the joint evaluation gives the same outputs
+  Shape s{B, C, M, K, L, M > 0 && K * L > 0};
+  if (B == 0) {
+    *c->host_status = 0;
+    FE_CK(cudaEventRecord(c->done_ev, (cudaStream_t)stream));
+    return FE_OK;
+  }
+  IoPtrs io{context, pool, cand_idx, scores_out, best_out, c->host_status};
+  return launch_batch(c, s, io, (cudaStream_t)stream);
 }
 
 int fe_evaluate_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* context, const void* pool,

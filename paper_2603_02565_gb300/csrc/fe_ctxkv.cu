@@ -129,8 +129,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int rb = it & 1;
         if (it >= 2 && !mbar_wait_bounded(raw_empty + rb, ((it >> 1) - 1) & 1, p.status)) break;
         mbar_arrive_expect_tx(raw_full + rb, LY.raw_bytes);
+        // context row of this block (one K/V per candidate sequence: rep > 1)
+        const int r0 = t * BM;
+        const int in_row = p.rep > 1 ? ((r0 / p.C) / p.rep) * p.C + r0 % p.C : r0;
         for (int kb = 0; kb < NKB; ++kb)
-          tma_load_2d(sRaw + (size_t)rb * LY.raw_bytes + (size_t)kb * kPlane, &tX, kb * BK, t * BM, raw_full + rb);
+          tma_load_2d(sRaw + (size_t)rb * LY.raw_bytes + (size_t)kb * kPlane, &tX, kb * BK, in_row, raw_full + rb);
       }
     }
   } else if (warp == 1) {

@@ -121,6 +121,9 @@ struct CtxKvParams {
   int rows, d, N;
   float eps;
   int* status;
+  // output row r reads context row ((r / C) / rep) * C + r % C: rep = 1 for one
+  // K/V per request, rep = K for one per candidate sequence (C % 128 == 0)
+  int C, rep;
 };
 bool ctxkv_supported(int d, int d_pad, int N, int nb, int io_f32);
 cudaError_t ctxkv_prepare();
@@ -164,6 +167,12 @@ cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, cons
 cudaError_t misc_prepare();
 // Distinct-element compaction of every request: bitmap over the pool, ranks,
 // distinct list, |U(z_b)|, bad-request flags; the last CTA scans U into offsets.
+// Candidate-factorized layout (every occurrence its own element): per request b
+// U[b] = K*L, off[b] = b*K*L (off[B] = B*K*L), list[b*K*L + i] = cand[b, i],
+// slot[b, i] = i; a request with an index outside [0, M) gets bad[b] = 1,
+// slot -1, list entries 0 (in range for the gather; its scores become NaN).
+cudaError_t identity_layout_launch(const int32_t* cand, int B, int M, int KL, int* U, int* off, int* bad,
+                                   int* slot, int* list, int* status, cudaStream_t s);
 cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int cap, int* U, int* off,
                            int* bad, int* slot_local, int* list, int* status, unsigned* ticket,
                            cudaStream_t s);

@@ -242,6 +242,41 @@ cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int 
 }
 
 // ---------------------------------------------------------------------------
+// candidate-factorized layout: one CTA (256 threads) per request
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) identity_layout_kernel(const int32_t* __restrict__ cand, int B, int M, int KL,
+                                                              int* U, int* off, int* bad, int* slot, int* list,
+                                                              int* status) {
+  const int b = blockIdx.x;
+  pdl_wait();
+  pdl_trigger();
+  const int32_t* cb = cand + (size_t)b * KL;
+  int any_bad = 0;
+  for (int i = threadIdx.x; i < KL; i += blockDim.x) {
+    const int v = cb[i];
+    any_bad |= (v < 0 || v >= M);
+  }
+  any_bad = __syncthreads_or(any_bad);
+  for (int i = threadIdx.x; i < KL; i += blockDim.x) {
+    list[(size_t)b * KL + i] = any_bad ? 0 : cb[i];
+    slot[(size_t)b * KL + i] = any_bad ? -1 : i;
+  }
+  if (threadIdx.x == 0) {
+    U[b] = KL;
+    off[b] = b * KL;
+    bad[b] = any_bad;
+    if (any_bad) atomicOr(status, ST_INDEX);
+    if (b == B - 1) off[B] = B * KL;
+  }
+}
+
+cudaError_t identity_layout_launch(const int32_t* cand, int B, int M, int KL, int* U, int* off, int* bad,
+                                   int* slot, int* list, int* status, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  return launch_k(identity_layout_kernel, dim3(B), dim3(256), 0, s, cand, B, M, KL, U, off, bad, slot, list, status);
+}
+
+// ---------------------------------------------------------------------------
 // LN of context rows -> split planes (one warp per row)
 // ---------------------------------------------------------------------------
 template <int DPL, typename T>

@@ -221,3 +221,43 @@ def test_pipelined_host_entry(dev):
     with pytest.raises(FeError):
         ev.wait_host()                          # nothing outstanding
     check(w1, outs[0][0], outs[0][1])
+
+
+@pytest.mark.parametrize("name,kw", [("ksweep", dict(K=10, B=3)), ("ksweep", dict(K=100, B=2)),
+                                     ("serving", dict(B=3))])
+def test_factorized_matches_joint(dev, name, kw):
+    """fe_evaluate_factorized (context K/V per sequence, every occurrence encoded on
+    its own) gives the joint evaluation's scores: the same per-row arithmetic, only
+    more of it; against the oracle as well."""
+    w = wl.make_workload(name, **kw)
+    ev, gs, gb = run_gpu(w, dev)
+    ctx, pool, idx = to_dev(w, dev)
+    fs, fb = ev.evaluate(ctx, pool, idx, factorized=True)
+    fs, fb = fs.cpu().numpy(), fb.cpu().numpy()
+    np.testing.assert_allclose(fs, gs, rtol=1e-5, atol=1e-7)
+    np.testing.assert_array_equal(fb, gb)
+    check(w, fs, fb)
+    B, C, M, K, L = w.shape
+    sl, U = ev.layout(B, K, L)
+    np.testing.assert_array_equal(U, np.full(B, K * L))
+    np.testing.assert_array_equal(sl.reshape(B, -1), np.tile(np.arange(K * L), (B, 1)))
+    # the joint evaluation still works on the same context afterwards
+    gs2, gb2 = ev.evaluate(ctx, pool, idx)
+    np.testing.assert_array_equal(gs2.cpu().numpy(), gs)
+
+
+def test_factorized_bad_index(dev):
+    w = wl.make_workload("serving", B=4)
+    idx_bad = np.array(w.cand_idx)
+    idx_bad[1, 3, 2] = w.shape[2]  # == M: out of range
+    from paper_2603_02565_gb300.binding import Evaluator
+    ev = Evaluator(w.cfg, w.weights)
+    ctx, pool, _ = to_dev(w, dev)
+    idx = torch.from_numpy(np.ascontiguousarray(idx_bad)).to(dev)
+    fs, fb = ev.evaluate(ctx, pool, idx, factorized=True)
+    fs, fb = fs.cpu().numpy(), fb.cpu().numpy()
+    assert np.isnan(fs[1]).all() and fb[1] == -1
+    js, jb = ev.evaluate(ctx, pool, idx)
+    ok = [0, 2, 3]
+    np.testing.assert_allclose(fs[ok], js.cpu().numpy()[ok], rtol=1e-5, atol=1e-7)
+    np.testing.assert_array_equal(fb[ok], jb.cpu().numpy()[ok])
