@@ -108,6 +108,28 @@ int encode_map_t(CUtensorMap* m, CUtensorMapDataType dt, size_t esz, const void*
   return FE_OK;
 }
 
+// Head-major f16 blocks [blocks][rows][dh]: 3D map with box box_x x box_rows x 1.
+int encode_map_hm(CUtensorMap* m, const void* base, int dh, int rows, int blocks, int box_x, int box_rows,
+                  CUtensorMapSwizzle sw) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) {
+    g_msg = "cuTensorMapEncodeTiled is unavailable";
+    return FE_ERR_CUDA;
+  }
+  cuuint64_t dims[3] = {(cuuint64_t)dh, (cuuint64_t)rows, (cuuint64_t)blocks};
+  cuuint64_t strides[2] = {(cuuint64_t)dh * 2, (cuuint64_t)rows * dh * 2};
+  cuuint32_t box[3] = {(cuuint32_t)box_x, (cuuint32_t)box_rows, 1u};
+  cuuint32_t es[3] = {1u, 1u, 1u};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    g_msg = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+    return FE_ERR_CUDA;
+  }
+  return FE_OK;
+}
+
 // Operand tiles: 64 bf16 (128 B) x box_rows, 128-byte swizzle.
 int encode_map(CUtensorMap* m, const bf16* base, int cols, int rows, int box_rows) {
   return encode_map_t(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, cols, rows, 64, box_rows,
@@ -140,6 +162,17 @@ int map_attn(Planes& p, int dh) {
                         CU_TENSOR_MAP_SWIZZLE_64B);
   if (rc == FE_OK) rc = encode_map_t(&p.ah, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.h, p.ld, p.rows, dh, 128, sw);
   if (rc == FE_OK) rc = encode_map_t(&p.kh, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.h, p.ld, p.rows, dh, kv_rows, sw);
+  return rc;
+}
+
+// The fused context kernel's K/V, head-major [ld / dh blocks][rows][dh]: its
+// store map (32 x 32 boxes) and the attention kernel's key/value map, so that
+// every key chunk of one head is one contiguous block.
+int map_attn_hm(Planes& p, int dh) {
+  const CUtensorMapSwizzle sw = dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
+  const int kv_rows = dh == 32 ? 64 : 128;
+  int rc = encode_map_hm(&p.sh, p.h, dh, p.rows, p.ld / dh, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
+  if (rc == FE_OK) rc = encode_map_hm(&p.kh, p.h, dh, p.rows, p.ld / dh, dh, kv_rows, sw);
   return rc;
 }
 
@@ -487,6 +520,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.rows = B * C * (fact ? K : 1);  // factorized: the context of every sequence
     p.d = d;
     p.N = 2 * Ly * d;
+    p.dh = c->dh;
     p.eps = c->cfg.ln_eps;
     p.status = c->status;
     p.C = C;
@@ -531,6 +565,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.q_col = 0;
     ap.k_col = 2 * l * d;
     ap.v_col = (2 * l + 1) * d;
+    ap.kv3d = c->fused_ctxkv ? 1 : 0;
     ap.o_col = 0;
     ap.o_h = c->a.h;
     ap.o_l = c->a.l;
@@ -768,7 +803,8 @@ int reserve_impl(fe_ctx* c, Shape s) {
   if (!c->fused_ctxkv) FE_RC(map_act(c->X));
   for (Planes* p : {&c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp}) FE_RC(map_act(*p));
   for (Planes* p : {&c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->lncp}) FE_RC(map_out(*p));
-  for (Planes* p : {&c->KV, &c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
+  for (Planes* p : {&c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
+  FE_RC(c->fused_ctxkv ? map_attn_hm(c->KV, c->dh) : map_attn(c->KV, c->dh));
   c->cap_shape = s;
   c->cap_shape.fact = false;
   c->cap_rows = R;
@@ -1251,6 +1287,15 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
   }
   if (f32) {
     FE_CK(cudaMemcpy(dst, f32, rows * cols * sizeof(float), cudaMemcpyDeviceToHost));
+    return FE_OK;
+  }
+  if (pl == &c->KV && c->fused_ctxkv) {  // head-major [cols / dh][pl->rows][dh]
+    std::vector<uint16_t> hh((size_t)pl->rows * pl->ld);
+    FE_CK(cudaMemcpy(hh.data(), pl->h, hh.size() * 2, cudaMemcpyDeviceToHost));
+    const size_t dh = (size_t)c->dh;
+    for (size_t r = 0; r < rows; ++r)
+      for (size_t j = 0; j < cols; ++j)
+        dst[r * cols + j] = f16_to_float(hh[((j / dh) * pl->rows + r) * dh + j % dh]);
     return FE_OK;
   }
   std::vector<uint16_t> hh((size_t)rows * pl->ld), ll((size_t)rows * pl->ld);

@@ -11,13 +11,14 @@
 //   warp 0 lane 0 : TMA producer -- Q tile (two buffers, one per unit in
 //                   flight) and K/V chunks of CK keys (8 stages for d_h = 32,
 //                   4 for d_h = 64)
-//   warp 1 lane 0 : tcgen05.mma -- S_j = Q K_j^T into TMEM tile j % 2, then
+//   warp 1 lane 0 : tcgen05.mma -- S_j = Q K_j^T into TMEM tile j % 3, then
 //                   PV_j = P_j V_j with P_j read from that same TMEM tile
-//                   into PV buffer j % 2
-//   warps 2..     : online softmax from TMEM, one query row per lane; with
-//                   d_h = 64, warps w and w+4 share TMEM lane quadrant w % 4
-//                   and each take half of the chunk's keys and half of the
-//                   output columns.  P_j is written back over S_j as f16;
+//                   into PV buffer j % 2; three S/P tiles let S_{j+1} start
+//                   while PV_{j-1} still reads its tile
+//   warps 2..9    : online softmax from TMEM, one query row per lane; warps
+//                   w and w+4 share TMEM lane quadrant w % 4 and each take
+//                   half of the chunk's keys and half of the output columns
+//                   (row maxima and sums exchanged through shared memory).  P_j is written back over S_j as f16;
 //                   PV_{j-1} is folded into the register output after P_j is
 //                   handed over, so the softmax never waits for the PV
 //                   product of the chunk it has just finished
@@ -34,17 +35,20 @@ namespace {
 
 constexpr int BQ = 128;     // query rows per unit (TMEM lanes)
 
-// d_h = 32: 64-key chunks and 4 softmax warps, small enough for two CTAs per SM.
+// d_h = 32: 64-key chunks, 32 keys per softmax warp, small enough for two CTAs per SM.
 // d_h = 64: 128-key chunks and 8 softmax warps (two per TMEM lane quadrant).
 template <int DH>
 struct AttnCfg {
   static constexpr int CK = DH == 32 ? 64 : 128;                // keys per chunk
-  static constexpr int kSoftmaxWarps = DH == 32 ? 4 : 8;
+  static constexpr int kSoftmaxWarps = 8;
   static constexpr int kHalves = kSoftmaxWarps / 4;              // warps sharing one lane quadrant
+  static constexpr int KW = CK / kHalves;                        // keys per softmax warp and chunk
   static constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
   static constexpr int kCtasPerSM = DH == 32 ? 2 : 1;
-  // TMEM: S/P tiles at [0, CK) and [CK, 2CK), PV buffers at [2CK, 2CK + 2DH)
+  // TMEM: S/P tiles at [t CK, t CK + CK), t < 3; PV buffers at [3CK, 3CK + 2DH)
+  static constexpr int kTiles = 3;
   static constexpr uint32_t kTmemCols = DH == 32 ? 256 : 512;
+  static_assert(kTiles * CK + 2 * DH <= (int)kTmemCols, "TMEM budget");
   static constexpr uint32_t kRowBytes = DH * 2;                 // one row of a Q/K/V tile
   static constexpr uint32_t kQBytes = 128 * kRowBytes;          // Q tile: 128 rows
   static constexpr uint32_t kKVTile = CK * kRowBytes;           // K or V chunk: CK rows
@@ -66,8 +70,67 @@ __device__ __forceinline__ uint64_t desc_sw(uint32_t saddr, uint32_t sbo, uint32
   return d;
 }
 
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// maximum of 32 values as a tree of three-input maxima
+__device__ __forceinline__ float max32(const float* v) {
+  float a[11];
+#pragma unroll
+  for (int i = 0; i < 10; ++i) a[i] = max3f(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+  a[10] = fmaxf(v[30], v[31]);
+  return fmaxf(max3f(max3f(a[0], a[1], a[2]), max3f(a[3], a[4], a[5]), max3f(a[6], a[7], a[8])),
+               fmaxf(a[9], a[10]));
+}
+
 __device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// Unit cursor: unit u -> (segment b, head h, query tile); query tile fastest.
+// Every role walks its CTA's units u = blockIdx.x + i * gridDim.x and skips
+// tiles that start past their segment's end.  The segment count and offset
+// of the next candidate unit are loaded one unit ahead, so a role crossing
+// into its next unit does not wait on a global load.
+struct Cursor {
+  int u, b, h, q0, qcnt, qoff;
+  int pcnt, poff;  // q_cnt / q_off of unit u + gridDim.x
+};
+
+__device__ __forceinline__ void cur_fetch(const AttnParams& p, int u, int& cnt, int& off) {
+  const int b = u / (p.max_q_tiles * p.n_heads);
+  cnt = p.q_cnt_dev ? __ldg(p.q_cnt_dev + b) : p.q_cnt_fixed;
+  off = p.q_off_dev ? __ldg(p.q_off_dev + b) : b * p.q_stride;
+}
+
+// settle on the first unit at or after c.u whose tile holds query rows
+__device__ __forceinline__ void cur_settle(const AttnParams& p, int units, Cursor& c) {
+  while (c.u < units) {
+    c.b = c.u / (p.max_q_tiles * p.n_heads);
+    c.h = (c.u / p.max_q_tiles) % p.n_heads;
+    c.q0 = (c.u % p.max_q_tiles) * BQ;
+    if (c.q0 < c.qcnt) break;
+    c.u += gridDim.x;
+    if (c.u < units) cur_fetch(p, c.u, c.qcnt, c.qoff);
+  }
+  if (c.u < units && c.u + (int)gridDim.x < units) cur_fetch(p, c.u + gridDim.x, c.pcnt, c.poff);
+}
+
+__device__ __forceinline__ void cur_first(const AttnParams& p, int units, Cursor& c) {
+  c.u = blockIdx.x;
+  cur_fetch(p, c.u, c.qcnt, c.qoff);
+  cur_settle(p, units, c);
+}
+
+__device__ __forceinline__ void cur_next(const AttnParams& p, int units, Cursor& c) {
+  c.u += gridDim.x;
+  if (c.u >= units) return;
+  c.qcnt = c.pcnt;
+  c.qoff = c.poff;
+  cur_settle(p, units, c);
 }
 
 }  // namespace
@@ -88,10 +151,11 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   uint64_t* q_empty = bars + 2;   // [2]
   uint64_t* kv_full = bars + 4;   // [stages]
   uint64_t* kv_empty = bars + 12; // [stages]
-  uint64_t* s_full = bars + 20;   // [2] S_j complete in TMEM tile j % 2
-  uint64_t* p_full = bars + 22;   // [2] P_j written over S_j
-  uint64_t* pv_full = bars + 24;  // [2] PV_j complete in PV buffer j % 2
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 26);
+  uint64_t* s_full = bars + 20;     // [3] S_j complete in TMEM tile j % 3
+  uint64_t* p_full = bars + 23;     // [3] P_j written over S_j
+  uint64_t* tile_free = bars + 26;  // [3] PV_j has read P_j: tile j % 3 free again
+  uint64_t* pv_full = bars + 29;    // [2] PV_j complete in PV buffer j % 2
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 31);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // row-statistic exchange
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -104,9 +168,12 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     for (int i = 0; i < 2; ++i) {
       mbar_init(q_full + i, 1);
       mbar_init(q_empty + i, 1);
+      mbar_init(pv_full + i, 1);
+    }
+    for (int i = 0; i < Cfg::kTiles; ++i) {
       mbar_init(s_full + i, 1);
       mbar_init(p_full + i, 32 * Cfg::kSoftmaxWarps);
-      mbar_init(pv_full + i, 1);
+      mbar_init(tile_free + i, 1);
     }
     for (int i = 0; i < Cfg::kKVStages; ++i) {
       mbar_init(kv_full + i, 1);
@@ -127,42 +194,35 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   pdl_trigger();
   pdl_wait();
 
-  // unit u -> (segment, head, query tile); query tile fastest
-  auto unit_info = [&](int u, int& b, int& h, int& q0, int& qcnt, int& qoff) {
-    const int qt = u % qtiles;
-    h = (u / qtiles) % p.n_heads;
-    b = u / (qtiles * p.n_heads);
-    qcnt = p.q_cnt_dev ? p.q_cnt_dev[b] : p.q_cnt_fixed;
-    qoff = p.q_off_dev ? p.q_off_dev[b] : b * p.q_stride;
-    q0 = qt * BQ;
-  };
-
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer ----------------
       int ui = 0, gc = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        int b, h, q0, qcnt, qoff;
-        unit_info(u, b, h, q0, qcnt, qoff);
-        if (q0 >= qcnt) continue;
+      Cursor c;
+      for (cur_first(p, units, c); c.u < units && ok; cur_next(p, units, c)) {
         const int qb = ui & 1;
-        if (ui >= 2 && !mbar_wait_bounded(q_empty + qb, ((ui >> 1) - 1) & 1, p.status)) break;
+        if (ui >= 2 && !mbar_wait_compact(q_empty + qb, ((ui >> 1) - 1) & 1, p.status)) break;
         uint8_t* q = sQ + qb * Cfg::kQBytes;
         mbar_arrive_expect_tx(q_full + qb, Cfg::kQBytes);
-        tma_load_2d(q, &tQ, p.q_col + h * DH, qoff + q0, q_full + qb);
+        tma_load_2d(q, &tQ, p.q_col + c.h * DH, c.qoff + c.q0, q_full + qb);
         for (int j = 0; j < nch; ++j, ++gc) {
           const int ks = gc % Cfg::kKVStages;
           if (gc >= Cfg::kKVStages &&
-              !mbar_wait_bounded(kv_empty + ks, ((gc / Cfg::kKVStages) - 1) & 1, p.status)) {
+              !mbar_wait_compact(kv_empty + ks, ((gc / Cfg::kKVStages) - 1) & 1, p.status)) {
             ok = false;
             break;
           }
           uint8_t* kv = sKV + ks * Cfg::kKVBytes;
-          const int row = b * p.kv_stride + j * CK;
+          const int row = c.b * p.kv_stride + j * CK;
           mbar_arrive_expect_tx(kv_full + ks, Cfg::kKVBytes);
-          tma_load_2d(kv, &tK, p.k_col + h * DH, row, kv_full + ks);
-          tma_load_2d(kv + Cfg::kKVTile, &tV, p.v_col + h * DH, row, kv_full + ks);
+          if (p.kv3d) {  // head-major K/V: one contiguous block per head
+            tma_load_3d(kv, &tK, 0, row, (p.k_col + c.h * DH) / DH, kv_full + ks);
+            tma_load_3d(kv + Cfg::kKVTile, &tV, 0, row, (p.v_col + c.h * DH) / DH, kv_full + ks);
+          } else {
+            tma_load_2d(kv, &tK, p.k_col + c.h * DH, row, kv_full + ks);
+            tma_load_2d(kv + Cfg::kKVTile, &tV, p.v_col + c.h * DH, row, kv_full + ks);
+          }
         }
         ++ui;
       }
@@ -170,66 +230,70 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
+      // The chunks of all this CTA's units form one stream g = 0, 1, ...;
+      // S_{g+1} is issued before PV_g, across unit boundaries too, so the
+      // softmax finds the next unit's first S ready when it gets there.
       const uint32_t idesc_s = umma_idesc_f16(BQ, CK);
       const uint32_t idesc_pv = umma_idesc_f16(BQ, DH) | (1u << 16);  // B (V) is MN-major
-      int ui = 0, gc = 0;
-      bool ok = true;
-      // S = Q K^T of global chunk gcc into TMEM tile gcc % 2, the unit's Q in buffer qb
-      auto issue_s = [&](int qb, int gcc) -> bool {
-        // the tile is free once PV_{gcc-2}, which reads P_{gcc-2} from it, has completed
-        if (gcc >= 2 && !mbar_wait_bounded(pv_full + (gcc & 1), ((gcc - 2) >> 1) & 1, p.status)) return false;
-        const int ks = gcc % Cfg::kKVStages;
-        if (!mbar_wait_bounded(kv_full + ks, (gcc / Cfg::kKVStages) & 1, p.status)) return false;
+      Cursor sc;             // unit of the next S
+      int sj = 0, sui = 0;   // its chunk and its unit counter (Q buffer sui % 2)
+      int g_s = 0;           // S products issued
+      cur_first(p, units, sc);
+      // S = Q K^T of the chunk at the S cursor into TMEM tile g_s % 3, then advance the cursor
+      auto issue_next_s = [&]() -> bool {
+        if (sc.u >= units) return true;
+        const int qb = sui & 1;
+        if (sj == 0 && !mbar_wait_compact(q_full + qb, (sui >> 1) & 1, p.status)) return false;
+        const int t = g_s % Cfg::kTiles;
+        // the tile is free once PV_{g_s-3}, which reads P_{g_s-3} from it, has completed
+        if (g_s >= Cfg::kTiles && !mbar_wait_compact(tile_free + t, ((g_s / Cfg::kTiles) - 1) & 1, p.status))
+          return false;
+        const int ks = g_s % Cfg::kKVStages;
+        if (!mbar_wait_compact(kv_full + ks, (g_s / Cfg::kKVStages) & 1, p.status)) return false;
         tc_fence_after();
         const uint32_t q = smem_u32(sQ + qb * Cfg::kQBytes);
         const uint32_t k = smem_u32(sKV + ks * Cfg::kKVBytes);
-        const uint32_t dst = tmem + (uint32_t)((gcc & 1) * CK);
+        const uint32_t dst = tmem + (uint32_t)(t * CK);
         const uint64_t q0d = desc_sw(q, Cfg::kSbo, Cfg::kSwz), k0d = desc_sw(k, Cfg::kSbo, Cfg::kSwz);
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk)
           umma_bf16(dst, desc_adv(q0d, kk * 32), desc_adv(k0d, kk * 32), idesc_s, kk != 0 ? 1u : 0u);
-        umma_commit(s_full + (gcc & 1));
+        umma_commit(s_full + t);
+        ++g_s;
+        if (++sj == nch) {  // every S of this unit issued: its Q buffer frees on completion
+          umma_commit(q_empty + qb);
+          sj = 0;
+          ++sui;
+          cur_next(p, units, sc);
+        }
         return true;
       };
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        int b, h, q0, qcnt, qoff;
-        unit_info(u, b, h, q0, qcnt, qoff);
-        if (q0 >= qcnt) continue;
-        const int qb = ui & 1;
-        if (!mbar_wait_bounded(q_full + qb, (ui >> 1) & 1, p.status)) break;
-        for (int j = 0; j < nch; ++j, ++gc) {
-          // S_{j+1} is issued ahead so that it overlaps the softmax of chunk j
-          if ((j == 0 && !issue_s(qb, gc)) || (j + 1 < nch && !issue_s(qb, gc + 1))) {
-            ok = false;
-            break;
-          }
-          if (j + 1 == nch) umma_commit(q_empty + qb);  // every S of this unit issued: Q buffer frees on completion
-          if (!mbar_wait_bounded(p_full + (gc & 1), (gc >> 1) & 1, p.status)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          // PV_j: A = P_j from TMEM tile j % 2, each key block of 64 as 32
-          // columns of f16 pairs at the start of its 64 S columns
-          const int ks = gc % Cfg::kKVStages;
-          const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile);
-          const uint32_t pt = tmem + (uint32_t)((gc & 1) * CK);
-          const uint32_t dst = tmem + (uint32_t)(2 * CK + (gc & 1) * DH);
-          const uint64_t v0d = desc_sw(v, Cfg::kSbo, Cfg::kSwz);
+      bool ok = issue_next_s();
+      for (int g = 0; ok && g < g_s; ++g) {
+        if (!issue_next_s()) break;
+        const int t = g % Cfg::kTiles;
+        if (!mbar_wait_compact(p_full + t, (g / Cfg::kTiles) & 1, p.status)) break;
+        tc_fence_after();
+        // PV_g: A = P_g from TMEM tile g % 3, each softmax warp's KW keys as
+        // KW/2 columns of f16 pairs at the start of its KW S columns
+        const int ks = g % Cfg::kKVStages;
+        const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile);
+        const uint32_t pt = tmem + (uint32_t)(t * CK);
+        const uint32_t dst = tmem + (uint32_t)(Cfg::kTiles * CK + (g & 1) * DH);
+        const uint64_t v0d = desc_sw(v, Cfg::kSbo, Cfg::kSwz);
 #pragma unroll
-          for (int kk = 0; kk < CK / 16; ++kk)
-            umma_bf16_tmem_a(dst, pt + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8),
-                             desc_adv(v0d, (uint32_t)kk * 16 * Cfg::kRowBytes), idesc_pv, kk != 0 ? 1u : 0u);
-          umma_commit(pv_full + (gc & 1));
-          umma_commit(kv_empty + ks);
-        }
-        ++ui;
+        for (int kk = 0; kk < CK / 16; ++kk)
+          umma_bf16_tmem_a(dst, pt + (uint32_t)((kk / (Cfg::KW / 16)) * Cfg::KW + (kk % (Cfg::KW / 16)) * 8),
+                           desc_adv(v0d, (uint32_t)kk * 16 * Cfg::kRowBytes), idesc_pv, kk != 0 ? 1u : 0u);
+        umma_commit(pv_full + (g & 1));
+        umma_commit(tile_free + t);
+        umma_commit(kv_empty + ks);
       }
     }
   } else {
     // ---------------- softmax / output (warps 2..9) ----------------
     constexpr int DO = DH / Cfg::kHalves;  // output columns per warp
-    constexpr int KW = CK / Cfg::kHalves;  // keys per warp and chunk (64)
+    constexpr int KW = Cfg::KW;            // keys per warp and chunk (32 for d_h = 32, 64 for d_h = 64)
     const int sw = warp - 2;
     const int q4 = warp & 3;
     const int half = sw >> 2;     // keys [KW half, KW half + KW) of each chunk, output columns [DO half, DO half + DO)
@@ -240,10 +304,10 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q4) : "memory"); };
     // fold PV_g (PV buffer g % 2) into the register output: o = o * c + PV_g
     auto fold = [&](int g, float c, float* o) -> bool {
-      if (!mbar_wait_bounded(pv_full + (g & 1), (g >> 1) & 1, p.status)) return false;
+      if (!mbar_wait_compact(pv_full + (g & 1), (g >> 1) & 1, p.status)) return false;
       tc_fence_after();
       float pv[DO];
-      const uint32_t src = tmem + lane_off + (uint32_t)(2 * CK + (g & 1) * DH + half * DO);
+      const uint32_t src = tmem + lane_off + (uint32_t)(Cfg::kTiles * CK + (g & 1) * DH + half * DO);
       if (DO == 16) {
         tmem_ld16(src, pv);
       } else {
@@ -254,40 +318,71 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       for (int i = 0; i < DO; ++i) o[i] = o[i] * c + pv[i];
       return true;
     };
+    // the finished unit whose last PV is still to be folded and stored
+    struct Done {
+      int h, q0, qcnt, qoff, ui;
+      float l, corr;
+      bool active;
+    } dn{};
+    bool have_done = false;
+    float o[DO];
+    // fold the finished unit's last PV (chunk g), then O / l as a split pair
+    auto finish = [&](int g) -> bool {
+      if (dn.active && !fold(g, dn.corr, o)) return false;
+      float ltot = dn.l;
+      if (Cfg::kHalves == 2) {
+        float* rs = red_sum + (dn.ui & 1) * 256;
+        rs[half * 128 + r] = dn.l;
+        pair_sync();
+        ltot = rs[r] + rs[128 + r];
+      }
+      if (dn.q0 + r < dn.qcnt) {
+        const float inv = 1.f / ltot;
+        const size_t go = (size_t)(dn.qoff + dn.q0 + r) * p.ldo + p.o_col + dn.h * DH + half * DO;
+#pragma unroll
+        for (int c = 0; c < DO; c += 8) {
+          uint32_t hi[4], lo[4];
+#pragma unroll
+          for (int i = 0; i < 8; i += 2) split2(o[c + i] * inv, o[c + i + 1] * inv, hi[i / 2], lo[i / 2]);
+          *reinterpret_cast<uint4*>(p.o_h + go + c) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          *reinterpret_cast<uint4*>(p.o_l + go + c) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        }
+      }
+      return true;
+    };
     int gc = 0, ui = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-      int b, h, q0, qcnt, qoff;
-      unit_info(u, b, h, q0, qcnt, qoff);
-      if (q0 >= qcnt) continue;
-      float m = -INFINITY, l = 0.f, corr_prev = 1.f;
-      float o[DO];
-#pragma unroll
-      for (int i = 0; i < DO; ++i) o[i] = 0.f;
+    Cursor c;
+    for (cur_first(p, units, c); c.u < units && ok; cur_next(p, units, c)) {
+      float m = -INFINITY, l = 0.f, corr = 1.f;
       // a warp whose 32 query rows all lie past the segment's end only keeps
       // the barrier protocol; those rows of P and of the output are never used
-      const bool active = q0 + q4 * 32 < qcnt;
+      const bool active = c.q0 + q4 * 32 < c.qcnt;
       for (int j = 0; j < nch; ++j, ++gc) {
-        if (!mbar_wait_bounded(s_full + (gc & 1), (gc >> 1) & 1, p.status)) {
+        const int t = gc % Cfg::kTiles;
+        if (!mbar_wait_compact(s_full + t, (gc / Cfg::kTiles) & 1, p.status)) {
           ok = false;
           break;
         }
-        float corr = 1.f;
+        const float corr_prev = corr;
+        corr = 1.f;
         if (active) {
           tc_fence_after();
-          const uint32_t tile = tmem + lane_off + (uint32_t)((gc & 1) * CK + half * KW);
-          float v[64];
-          tmem_ld64(tile, v);
-          const int kvalid = p.kv_cnt - j * CK - half * KW;  // valid keys among this warp's 64
-          float mx = -INFINITY;
-          if (kvalid >= 64) {
+          const uint32_t tile = tmem + lane_off + (uint32_t)(t * CK + half * KW);
+          float v[KW];
+          if constexpr (KW == 64)
+            tmem_ld64(tile, v);
+          else
+            tmem_ld32(tile, v);
+          // keys past kv_cnt take no part: -inf gives them P = 0
+          const int kvalid = p.kv_cnt - j * CK - half * KW;  // valid keys among this warp's KW
+          if (kvalid < KW) {
 #pragma unroll
-            for (int i = 0; i < 64; ++i) mx = fmaxf(mx, v[i]);
-          } else {
-#pragma unroll
-            for (int i = 0; i < 64; ++i)
-              if (i < kvalid) mx = fmaxf(mx, v[i]);
+            for (int i = 0; i < KW; ++i)
+              if (i >= kvalid) v[i] = -INFINITY;
           }
+          float mx = max32(v);
+          if constexpr (KW == 64) mx = fmaxf(mx, max32(v + 32));
           mx *= p.scale_log2;
           if (Cfg::kHalves == 2) {
             float* rm = red_max + (gc & 1) * 256;
@@ -298,68 +393,61 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           const float mn = fmaxf(m, mx);
           corr = ex2_approx(m - mn);
           m = mn;
-          // P = 2^(s * scale - m) as f16 over the first 32 of this warp's 64
-          // S columns (all 64 already in registers): keys 2c, 2c+1 in column
-          // c; keys past kv_cnt get 0
+          // P = 2^(s * scale - m) as f16 over the first KW/2 of this warp's KW
+          // S columns (all of them already in registers): keys 2c, 2c+1 in
+          // column c
           const float sc = p.scale_log2, nm = -mn;
-          float sum = 0.f;
-          auto emit = [&](auto full) {
+          float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-            for (int hb = 0; hb < 2; ++hb) {
-              uint32_t pk[16];
+          for (int hb = 0; hb < KW / 32; ++hb) {
+            uint32_t pk[16];
 #pragma unroll
-              for (int i = 0; i < 32; i += 2) {
-                const int k = 32 * hb + i;
-                float p0 = ex2_approx(fmaf(v[k], sc, nm));
-                float p1 = ex2_approx(fmaf(v[k + 1], sc, nm));
-                if (!decltype(full)::value) {
-                  p0 = k < kvalid ? p0 : 0.f;
-                  p1 = k + 1 < kvalid ? p1 : 0.f;
-                }
-                sum += p0 + p1;
-                pk[i / 2] = pack_f16x2(p0, p1);
-              }
-              tmem_st16_nowait(tile + (uint32_t)(16 * hb), pk);
+            for (int i = 0; i < 32; i += 2) {
+              const int k = 32 * hb + i;
+              const float p0 = ex2_approx(fmaf(v[k], sc, nm));
+              const float p1 = ex2_approx(fmaf(v[k + 1], sc, nm));
+              s4[(i >> 1) & 3] += p0 + p1;
+              pk[i / 2] = pack_f16x2(p0, p1);
             }
-          };
-          if (kvalid >= 64) emit(std::true_type{});
-          else emit(std::false_type{});
+            tmem_st16_nowait(tile + (uint32_t)(16 * hb), pk);
+          }
+          const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
           l = l * corr + sum;
           tmem_st_wait();
           tc_fence_before();
         }
-        mbar_arrive1(p_full + (gc & 1));
-        // the previous chunk's PV is folded while PV_j runs
-        if (j > 0 && active && !fold(gc - 1, corr_prev, o)) {
-          ok = false;
-          break;
+        mbar_arrive1(p_full + t);
+        // the previous chunk's PV is folded while PV_j runs; at a unit's first
+        // chunk that is the last PV of the previous unit, which is then stored
+        if (j > 0) {
+          if (active && !fold(gc - 1, corr_prev, o)) {
+            ok = false;
+            break;
+          }
+        } else if (have_done) {
+          if (!finish(gc - 1)) {
+            ok = false;
+            break;
+          }
         }
-        corr_prev = corr;
+        if (j == 0) {
+#pragma unroll
+          for (int i = 0; i < DO; ++i) o[i] = 0.f;
+        }
       }
       if (!ok) break;
-      if (active && !fold(gc - 1, corr_prev, o)) break;
-      // row sum over both halves, then O / l as a split pair
-      float ltot = l;
-      if (Cfg::kHalves == 2) {
-        float* rs = red_sum + (ui & 1) * 256;
-        rs[half * 128 + r] = l;
-        pair_sync();
-        ltot = rs[r] + rs[128 + r];
-      }
+      dn.h = c.h;
+      dn.q0 = c.q0;
+      dn.qcnt = c.qcnt;
+      dn.qoff = c.qoff;
+      dn.ui = ui;
+      dn.l = l;
+      dn.corr = corr;
+      dn.active = active;
+      have_done = true;
       ++ui;
-      if (q0 + r < qcnt) {
-        const float inv = 1.f / ltot;
-        const size_t go = (size_t)(qoff + q0 + r) * p.ldo + p.o_col + h * DH + half * DO;
-#pragma unroll
-        for (int c = 0; c < DO; c += 8) {
-          uint32_t hi[4], lo[4];
-#pragma unroll
-          for (int i = 0; i < 8; i += 2) split2(o[c + i] * inv, o[c + i + 1] * inv, hi[i / 2], lo[i / 2]);
-          *reinterpret_cast<uint4*>(p.o_h + go + c) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-          *reinterpret_cast<uint4*>(p.o_l + go + c) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-        }
-      }
     }
+    if (ok && have_done) finish(gc - 1);
   }
 
   tc_fence_before();

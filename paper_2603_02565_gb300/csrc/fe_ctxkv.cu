@@ -259,7 +259,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_async_shared();
         __syncwarp();
         if (lane == 0) {
-          tma_store_2d(&tO, b, n_off + c, srow);  // rows past the tensor extent are clipped
+          // head-major K/V: column n_off + c is block (n_off + c) / dh, offset (n_off + c) % dh
+          tma_store_3d(&tO, b, (n_off + c) % p.dh, srow, (n_off + c) / p.dh);  // rows past the extent are clipped
           bulk_commit();
         }
         ++nstore;

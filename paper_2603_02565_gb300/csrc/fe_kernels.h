@@ -115,10 +115,11 @@ cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUt
 // bf16-exact weights, N = 2 * n_layers * d in {256, 512}).
 // x: raw context rows [rows, d] bf16, 64 x 128 boxes, 128-byte swizzle;
 // w: W^T [N, d_pad] bf16, 64 x 128 boxes, 128-byte swizzle;
-// o: the f16 K/V rows [rows, N], 32 x 32 boxes, 64-byte swizzle.
+// o: the f16 K/V, head-major: [N / dh blocks][rows][dh] (block = one head of
+// K_l or V_l), 3D map with 32 x 32 x 1 boxes, 64-byte swizzle.
 // ---------------------------------------------------------------------------
 struct CtxKvParams {
-  int rows, d, N;
+  int rows, d, N, dh;
   float eps;
   int* status;
   // output row r reads context row ((r / C) / rep) * C + r % C: rep = 1 for one
@@ -151,6 +152,7 @@ struct AttnParams {
   int kv_stride;
   int kv_cnt;
   int q_col, k_col, v_col, o_col;
+  int kv3d;              // K/V head-major (3D maps: x within the head, row, block = column / dh)
   bf16 *o_h, *o_l;
   int ldo;
   float scale_log2;      // log2(e) / sqrt(d_h)
