@@ -43,6 +43,12 @@ def make_workload(args, seed_offset=0):
     kw = {}
     if args.batch:
         kw["B"] = args.batch
+    if args.tasks != 1:
+        kw["n_tasks"] = args.tasks
+    if args.no_cross_seq:
+        kw["cross_seq"] = False
+    if (args.tasks != 1 or args.no_cross_seq) and args.workload not in ("serving", "ksweep", "stress"):
+        raise SystemExit("--tasks / --no-cross-seq apply to the recommendation workloads")
     if args.workload == "serving":
         return wl.serving(seed=1 + seed_offset, **kw)
     if args.workload == "ksweep":
@@ -69,6 +75,7 @@ def describe(w):
 # ----------------------------------------------------------------------------------------------
 def site_work(site, cfg, B, C, M, K, L, R):
     d, F, Ly = cfg.d, cfg.F, cfg.n_layers
+    T = int(getattr(cfg, "n_tasks", 1))
     S, n = B * K, B * C
     esz = 2 if cfg.io_bf16 else 4
     A = 4
@@ -94,7 +101,7 @@ def site_work(site, cfg, B, C, M, K, L, R):
         "gemm_cross_qkv": (6 * S * d * d, S * d * A + 3 * S * d * H),
         "attn_cross_seq": (4 * B * K * K * d, 3 * S * d * H + S * d * A),
         "gemm_cross_o_ln": (2 * S * d * d, S * d * (A + 8 + A)),
-        "gemm_head": (2 * S * d * d + 3 * S * d, S * d * A + 4 * S),
+        "gemm_head": (2 * S * d * d * T + 3 * S * d * T, S * d * A + 4 * S * (1 + (T if T > 1 else 0))),
         "select": (0, 4 * S + 4 * B),
     }
     return t.get(site, (0, 0))
@@ -416,7 +423,9 @@ def run_ours(args):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": describe(w), "global_batch": world * B, "K": K, "L": L,
                        "mode": ("candidate-factorized E^ind (fe_evaluate_factorized)" if args.factorized
-                                else "joint (fe_evaluate)"),
+                                else "joint (fe_evaluate)")
+                               + (f", {args.tasks} task heads + linear fusion" if args.tasks != 1 else "")
+                               + (", without cross-sequence interaction" if args.no_cross_seq else ""),
                        "parallelism": f"dp{world} (requests sharded, no collective)",
                        "precision": "bf16 MMA operands with activations split hi+lo bf16; attention Q, K, V, "
                                     "P single f16; fp32 accumulate, softmax, LayerNorm and residuals",
@@ -503,6 +512,10 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--factorized", action="store_true",
                     help="time the candidate-factorized evaluation E^ind (fe_evaluate_factorized) instead")
+    ap.add_argument("--tasks", type=int, default=1,
+                    help="task-specific prediction heads with a linear fusion (end of Section 4.4)")
+    ap.add_argument("--no-cross-seq", action="store_true",
+                    help="the variant without cross-sequence interaction (Appendix B.4)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args()

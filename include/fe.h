@@ -71,6 +71,11 @@ typedef struct fe_config {
   int32_t max_L;      /* rows of the position table P; sequences have L <= max_L     */
   int32_t io_dtype;   /* FE_IO_BF16 or FE_IO_F32 for context and pool                 */
   float   ln_eps;     /* LayerNorm epsilon (1e-5)                                     */
+  int32_t n_tasks;    /* task-specific prediction heads T (end of Section 4.4): 0 or 1
+                         is the single shared head; 2..4 add a fusion module
+                         s_k = sum_t fuse_w[t] s_{k,t} + fuse_b (T * d <= 512)      */
+  int32_t no_cross_seq; /* 1: the variant without cross-sequence interaction
+                         (Appendix B.4, "- CrossSeq"): C' = C; 0: the full model    */
 } fe_config;
 
 typedef struct fe_ctx fe_ctx;
@@ -83,8 +88,10 @@ typedef struct fe_ctx fe_ctx;
  *   for l in 0..n_layers-1:
  *     WQ_l[d,d] WK_l[d,d] WV_l[d,d] WO_l[d,d] W1_l[d,F] b1_l[F] W2_l[F,d] b2_l[d]
  *   P[max_L,d] cls[d] WQs[d,d] WKs[d,d] WVs[d,d] WOs[d,d] W1s[d,F] b1s[F] W2s[F,d] b2s[d]
- *   WQx[d,d] WKx[d,d] WVx[d,d] WOx[d,d]
- *   W1h[d,d] b1h[d] w2h[d] b2h[1]
+ *   WQx[d,d] WKx[d,d] WVx[d,d] WOx[d,d]          (absent when no_cross_seq = 1)
+ *   for t in 0..T-1 (T = max(n_tasks, 1)):
+ *     W1h_t[d,d] b1h_t[d] w2h_t[d] b2h_t[1]      (task t's head)
+ *   fuse_w[T] fuse_b[1]                          (only when T >= 2)
  */
 size_t fe_weight_count(const fe_config* cfg);
 
@@ -114,7 +121,8 @@ int fe_reserve(fe_ctx* ctx, int B, int C, int M, int K, int L);
  *   pool     [B, M, d]  io_dtype     candidate pools C(x), one row per element
  *   cand_idx [B, K, L]  int32        sequence k of request b is the pool rows
  *                                    cand_idx[b,k,0..L-1] (L_k of Section 3)
- *   scores_out [B, K]   float32      s_k of Section 4.4
+ *   scores_out [B, K]   float32      s_k of Section 4.4 (the fused score with
+ *                                    several task heads)
  *   best_out   [B]      int32        argmax_k s_k, smallest k on ties (Eq. 1)
  * The work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
  * stream) and the call waits for it, then returns the batch status:
@@ -213,7 +221,10 @@ int fe_debug_layout(fe_ctx* ctx, int32_t* slot_out, int32_t* U_out);
  *   "elem"    [sum U, d]    H, the final element representations, requests in
  *                           order, each request's elements in ascending pool index
  *   "seq"     [B*K, d]      c_k, the SeqEnc output
- *   "cross"   [B*K, d]      C', the cross-sequence output
+ *   "cross"   [B*K, d]      C', the cross-sequence output (FE_ERR_UNSUPPORTED
+ *                           when no_cross_seq = 1: C' = C is "seq")
+ *   "task_scores" [B*K, T]  every task head's score s_{k,t} before the fusion
+ *                           (T = 1: the score itself)
  * `max_floats` is the capacity of `dst`; *n_floats receives the element count
  * (also when dst is NULL).  Waits for the last call.
  */

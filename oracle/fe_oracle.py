@@ -22,6 +22,12 @@ s = Inter(c), then Eq. 1's argmax):
   s_k = ReLU(LN(C'_k) W1h + b1h) . w2h + b2h.
 * Selection (Eq. 1): the smallest k attaining max_k s_k (the smallest-index
   rule the paper uses for its listwise labels, Appendix B.1).
+* Multi-objective variant (end of Section 4.4): T task-specific heads of the
+  same shape read the shared C'_k, and a fusion module combines their scores.
+  The paper does not define the fusion module; the reading taken here is a
+  learned linear combination s_k = sum_t alpha_t s_{k,t} + beta.
+* Variant without cross-sequence interaction ("- CrossSeq", ablation of
+  Appendix B.4): C' = C, each sequence scored on its own representation.
 
 The paper leaves the block internals open (norm placement, FFN, pooling, head
 shape).  The readings taken here: pre-LN blocks with LayerNorm without affine
@@ -42,7 +48,7 @@ from __future__ import annotations
 import numpy as np
 
 __all__ = ["layer_norm", "softmax", "mha", "context_kv", "encode_elements",
-           "seq_encode", "cross_sequence", "score_head", "select_best",
+           "seq_encode", "cross_sequence", "score_head", "task_heads", "select_best",
            "distinct_layout", "evaluate_request", "evaluate"]
 
 
@@ -131,10 +137,20 @@ def cross_sequence(Cm, W, n_heads, eps):
     return Cm + a @ _w(W, "WOx")
 
 
-def score_head(Cp, W, eps):
-    """Shared prediction head s_k = ReLU(LN(C'_k) W1h + b1h) . w2h + b2h."""
-    f = _relu(layer_norm(Cp, eps) @ _w(W, "W1h") + _w(W, "b1h"))
-    return f @ _w(W, "w2h") + _w(W, "b2h")[0]
+def score_head(Cp, W, eps, suffix=""):
+    """Shared prediction head s_k = ReLU(LN(C'_k) W1h + b1h) . w2h + b2h
+    (the head's tensors named W1h, b1h, w2h, b2h followed by `suffix`)."""
+    f = _relu(layer_norm(Cp, eps) @ _w(W, "W1h" + suffix) + _w(W, "b1h" + suffix))
+    return f @ _w(W, "w2h" + suffix) + _w(W, "b2h" + suffix)[0]
+
+
+def task_heads(Cp, W, n_tasks, eps):
+    """Multi-objective heads (end of Section 4.4): task t's head, of the same
+    shape as the single head, with tensors W1h.t, b1h.t, w2h.t, b2h.t, then the
+    fusion s_k = sum_t fuse_w[t] s_{k,t} + fuse_b.  Returns (s [K], per-task
+    scores [K, T])."""
+    st = np.stack([score_head(Cp, W, eps, f".{t}") for t in range(n_tasks)], axis=1)
+    return st @ _w(W, "fuse_w") + _w(W, "fuse_b")[0], st
 
 
 def select_best(s):
@@ -157,8 +173,10 @@ def distinct_layout(cand_b):
 
 # -- whole evaluator ---------------------------------------------------------
 
-def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse"):
-    """Scores [K] of one request's K candidate sequences."""
+def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse", tasks_out=None):
+    """Scores [K] of one request's K candidate sequences.  With several task
+    heads the scores are the fused ones and, when tasks_out is a list, the
+    per-task scores [K, T] are appended to it."""
     H, Ly, eps = cfg.n_heads, cfg.n_layers, cfg.ln_eps
     K, L = cand_b.shape
     if mode == "reuse":
@@ -176,14 +194,24 @@ def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse"):
     else:
         raise ValueError(mode)
     Cm = np.vstack([seq_encode(rows[k], W, H, eps) for k in range(K)])
-    Cp = cross_sequence(Cm, W, H, eps)
-    return score_head(Cp, W, eps)
+    Cp = cross_sequence(Cm, W, H, eps) if getattr(cfg, "cross_seq", True) else Cm
+    T = int(getattr(cfg, "n_tasks", 1))
+    if T == 1:
+        s = score_head(Cp, W, eps)
+        if tasks_out is not None:
+            tasks_out.append(s[:, None])
+        return s
+    s, st = task_heads(Cp, W, T, eps)
+    if tasks_out is not None:
+        tasks_out.append(st)
+    return s
 
 
-def evaluate(context, pool, cand_idx, W, cfg, mode="reuse", requests=None):
+def evaluate(context, pool, cand_idx, W, cfg, mode="reuse", requests=None, with_tasks=False):
     """E_theta over a batch.  Returns (scores [B, K] float64, best [B] int32,
-    U [B] int32, slots [B, K, L] int32).  `requests` restricts the work to a
-    subset of request indices (the other rows stay NaN / -1)."""
+    U [B] int32, slots [B, K, L] int32), plus the per-task scores [B, K, T]
+    when with_tasks.  `requests` restricts the work to a subset of request
+    indices (the other rows stay NaN / -1)."""
     context = np.asarray(context)
     pool = np.asarray(pool)
     cand_idx = np.asarray(cand_idx)
@@ -193,6 +221,8 @@ def evaluate(context, pool, cand_idx, W, cfg, mode="reuse", requests=None):
     best = np.full(B, -1, dtype=np.int32)
     U = np.zeros(B, dtype=np.int32)
     slots = np.full((B, K, L), -1, dtype=np.int32)
+    T = int(getattr(cfg, "n_tasks", 1))
+    tasks = np.full((B, K, T), np.nan)
     for b in (range(B) if requests is None else requests):
         cb = cand_idx[b]
         if cb.size and (cb.min() < 0 or cb.max() >= M):
@@ -202,6 +232,10 @@ def evaluate(context, pool, cand_idx, W, cfg, mode="reuse", requests=None):
         slots[b] = sl
         if K == 0:
             continue
-        scores[b] = evaluate_request(context[b], pool[b], cb, W, cfg, mode)
+        out = []
+        scores[b] = evaluate_request(context[b], pool[b], cb, W, cfg, mode, tasks_out=out)
+        tasks[b] = out[0]
         best[b] = select_best(scores[b])
+    if with_tasks:
+        return scores, best, U, slots, tasks
     return scores, best, U, slots

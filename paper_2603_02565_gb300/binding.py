@@ -38,7 +38,7 @@ EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evalua
 class FeConfig(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("n_layers", ctypes.c_int32),
                 ("ffn_mult", ctypes.c_int32), ("max_L", ctypes.c_int32), ("io_dtype", ctypes.c_int32),
-                ("ln_eps", ctypes.c_float)]
+                ("ln_eps", ctypes.c_float), ("n_tasks", ctypes.c_int32), ("no_cross_seq", ctypes.c_int32)]
 
 
 class FeError(RuntimeError):
@@ -104,24 +104,41 @@ def _check(rc, allowed=(FE_OK,)):
     return rc
 
 
-def weight_order(n_layers: int):
+def weight_order(n_layers: int, n_tasks: int = 1, cross_seq: bool = True):
     """Tensor names in the order fe.h documents for fe_init."""
     names = []
     for l in range(n_layers):
         names += [f"WQ.{l}", f"WK.{l}", f"WV.{l}", f"WO.{l}", f"W1.{l}", f"b1.{l}", f"W2.{l}", f"b2.{l}"]
-    names += ["P", "cls", "WQs", "WKs", "WVs", "WOs", "W1s", "b1s", "W2s", "b2s",
-              "WQx", "WKx", "WVx", "WOx", "W1h", "b1h", "w2h", "b2h"]
+    names += ["P", "cls", "WQs", "WKs", "WVs", "WOs", "W1s", "b1s", "W2s", "b2s"]
+    if cross_seq:
+        names += ["WQx", "WKx", "WVx", "WOx"]
+    if n_tasks == 1:
+        names += ["W1h", "b1h", "w2h", "b2h"]
+    else:
+        for t in range(n_tasks):
+            names += [f"W1h.{t}", f"b1h.{t}", f"w2h.{t}", f"b2h.{t}"]
+        names += ["fuse_w", "fuse_b"]
     return names
 
 
+def _tasks(cfg):
+    return int(getattr(cfg, "n_tasks", 1))
+
+
+def _cross(cfg):
+    return bool(getattr(cfg, "cross_seq", True))
+
+
 def make_config(cfg) -> FeConfig:
-    """fe_config from any object with d, n_heads, n_layers, ffn_mult, max_L, io_bf16, ln_eps."""
+    """fe_config from any object with d, n_heads, n_layers, ffn_mult, max_L, io_bf16, ln_eps
+    (and optionally n_tasks, cross_seq)."""
     return FeConfig(cfg.d, cfg.n_heads, cfg.n_layers, cfg.ffn_mult, cfg.max_L,
-                    FE_IO_BF16 if cfg.io_bf16 else FE_IO_F32, cfg.ln_eps)
+                    FE_IO_BF16 if cfg.io_bf16 else FE_IO_F32, cfg.ln_eps, _tasks(cfg), 0 if _cross(cfg) else 1)
 
 
 def pack_weights(cfg, weights: dict) -> np.ndarray:
-    parts = [np.ascontiguousarray(weights[n], dtype=np.float32).ravel() for n in weight_order(cfg.n_layers)]
+    parts = [np.ascontiguousarray(weights[n], dtype=np.float32).ravel()
+             for n in weight_order(cfg.n_layers, _tasks(cfg), _cross(cfg))]
     return np.concatenate(parts)
 
 

@@ -258,6 +258,9 @@ struct fe_ctx {
   Weight ctx_kv;
   std::vector<Weight> wq, wo, w1, w2;
   Weight kvs, os, w1s, w2s, qkvx, ox, w1h;
+  int n_tasks = 1;                  // task heads T
+  float* head_vec = nullptr;        // b1 [head cols] | w2 [head cols] | b2 [T] | fuse_w [T] | fuse_b [1]
+  float* task_scores = nullptr;     // [S, T], every head's score of the last batch
   float *q0 = nullptr, *k0 = nullptr, *v0 = nullptr, *kP = nullptr, *vP = nullptr;
   // workspace
   Shape cap_shape;  // reserved maxima
@@ -357,7 +360,17 @@ bool config_ok(const fe_config* c) {
   if (c->max_L < 1 || c->max_L > 4096) return false;
   if (c->io_dtype != FE_IO_BF16 && c->io_dtype != FE_IO_F32) return false;
   if (!(c->ln_eps >= 0.f)) return false;
+  if (c->n_tasks < 0 || c->n_tasks > 4 || (c->n_tasks > 1 && c->n_tasks * d > 512)) return false;
+  if (c->no_cross_seq != 0 && c->no_cross_seq != 1) return false;
   return true;
+}
+
+// task heads T and the head product's width: T * d columns, padded to a
+// column tile the GEMM supports (at most 256, or 512)
+int n_tasks_of(const fe_config* c) { return c->n_tasks > 1 ? c->n_tasks : 1; }
+int head_cols(const fe_config* c) {
+  const int n = n_tasks_of(c) * c->d;
+  return n <= 256 ? n : 512;
 }
 
 // sizes of the weight tensors in fe_weight_count order
@@ -381,11 +394,18 @@ std::vector<size_t> weight_sizes(const fe_config* c) {
   s.push_back(F);                     // b1s
   s.push_back(F * d);                 // W2s
   s.push_back(d);                     // b2s
-  for (int i = 0; i < 4; ++i) s.push_back(d * d);  // WQx WKx WVx WOx
-  s.push_back(d * d);                 // W1h
-  s.push_back(d);                     // b1h
-  s.push_back(d);                     // w2h
-  s.push_back(1);                     // b2h
+  for (int i = 0; i < 4; ++i) s.push_back(c->no_cross_seq ? 0 : d * d);  // WQx WKx WVx WOx
+  const int T = n_tasks_of(c);
+  for (int t = 0; t < T; ++t) {
+    s.push_back(d * d);               // W1h_t
+    s.push_back(d);                   // b1h_t
+    s.push_back(d);                   // w2h_t
+    s.push_back(1);                   // b2h_t
+  }
+  if (T > 1) {
+    s.push_back((size_t)T);           // fuse_w
+    s.push_back(1);                   // fuse_b
+  }
   return s;
 }
 
@@ -398,6 +418,8 @@ enum { T_P = 0, T_CLS, T_WQS, T_WKS, T_WVS, T_WOS, T_W1S, T_B1S, T_W2S, T_B2S, T
 const float* wptr(const fe_ctx* c, int tensor) { return c->w32 + c->woff[tensor]; }
 const float* lw(const fe_ctx* c, int l, int i) { return wptr(c, T_PER_LAYER * l + i); }
 const float* tw(const fe_ctx* c, int i) { return wptr(c, t_tail(c, i)); }
+// task t's head tensor j (0 W1h, 1 b1h, 2 w2h, 3 b2h); the fusion weights follow the last head
+const float* hw(const fe_ctx* c, int t, int j) { return tw(c, T_W1H + 4 * t + j); }
 
 // Allocate the transposed weight [N, K_pad] and pick its tiling.
 int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
@@ -652,7 +674,8 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     }
   }
   // (a5) cross-sequence attention over the K sequence vectors of each request
-  {
+  // (absent in the variant without cross-sequence interaction: C' = C)
+  if (!c->cfg.no_cross_seq) {
     fe::GemmParams p{};
     p.out_f16 = 1;
     FE_RC(gemm(c, "gemm_cross_qkv", fe::EPI_STORE, c->z, c->qkvx, S, nullptr, p, &c->qkv, nullptr, s));
@@ -682,14 +705,22 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     po.ldr = d;
     FE_RC(gemm(c, "gemm_cross_o_ln", fe::EPI_RESID_LN, c->ax, c->ox, S, nullptr, po, &c->lncp, &c->cp, s));
   }
-  // (a6) score head and selection
+  // (a6) score heads (task heads and their fusion) and selection
   {
+    const int HN = c->w1h.N;
     fe::GemmParams p{};
-    p.bias = tw(c, T_B1H);
-    p.w2 = tw(c, T_W2H);
-    p.b2 = tw(c, T_B2H);
+    p.n_tasks = c->n_tasks;
+    p.head_d = d;
+    p.bias = c->head_vec;
+    p.w2 = c->head_vec + HN;
+    p.b2 = c->head_vec + 2 * HN;
+    p.fuse_w = c->head_vec + 2 * HN + c->n_tasks;
+    p.fuse_b = c->head_vec + 2 * HN + 2 * c->n_tasks;
     p.scores = io.scores;
-    FE_RC(gemm(c, "gemm_head", fe::EPI_HEAD, c->lncp, c->w1h, S, nullptr, p, nullptr, nullptr, s));
+    p.task_scores = c->task_scores;
+    // LN(C') from the cross-sequence block, or LN(C) = Z without it
+    const Planes& hin = c->cfg.no_cross_seq ? c->z : c->lncp;
+    FE_RC(gemm(c, "gemm_head", fe::EPI_HEAD, hin, c->w1h, S, nullptr, p, nullptr, nullptr, s));
   }
   {
     Prof pf(c, "select", s);
@@ -775,6 +806,7 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->in_idx, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int32_t)));
   FE_RC(dalloc((void**)&c->out_scores, (size_t)S * sizeof(float)));
   FE_RC(dalloc((void**)&c->out_best, (size_t)B * sizeof(int32_t)));
+  FE_RC(dalloc((void**)&c->task_scores, (size_t)S * c->n_tasks * sizeof(float)));
   // pipelined host entry: slot 0 uses the staging above, slot 1 its own copy
   c->slots[0].ctx = c->in_ctx;
   c->slots[0].pool = c->in_pool;
@@ -1004,14 +1036,39 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if (c->fused_ffn && (rc = map_fused_w1(c->w1s, c->nb > 1)) != FE_OK) return fail(rc);
   if ((rc = make_weight(c, c->w2s, d, F, 512)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w2s, tw(c, T_W2S), F, d, 0)) != FE_OK) return fail(rc);
-  if ((rc = make_weight(c, c->qkvx, 3 * d, d, 128)) != FE_OK) return fail(rc);
-  if ((rc = fill_weight(c->qkvx, tw(c, T_WQX), d, d, 0)) != FE_OK) return fail(rc);
-  if ((rc = fill_weight(c->qkvx, tw(c, T_WKX), d, d, d)) != FE_OK) return fail(rc);
-  if ((rc = fill_weight(c->qkvx, tw(c, T_WVX), d, d, 2 * d)) != FE_OK) return fail(rc);
-  if ((rc = make_weight(c, c->ox, d, d, 512)) != FE_OK) return fail(rc);
-  if ((rc = fill_weight(c->ox, tw(c, T_WOX), d, d, 0)) != FE_OK) return fail(rc);
-  if ((rc = make_weight(c, c->w1h, d, d, 512)) != FE_OK) return fail(rc);
-  if ((rc = fill_weight(c->w1h, tw(c, T_W1H), d, d, 0)) != FE_OK) return fail(rc);
+  if (!cfg->no_cross_seq) {
+    if ((rc = make_weight(c, c->qkvx, 3 * d, d, 128)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->qkvx, tw(c, T_WQX), d, d, 0)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->qkvx, tw(c, T_WKX), d, d, d)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->qkvx, tw(c, T_WVX), d, d, 2 * d)) != FE_OK) return fail(rc);
+    if ((rc = make_weight(c, c->ox, d, d, 512)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->ox, tw(c, T_WOX), d, d, 0)) != FE_OK) return fail(rc);
+  }
+  // the task heads' first layers as one product of head_cols(cfg) columns
+  // (task t in columns [t d, t d + d), padding columns zero), and their
+  // vectors gathered into one buffer
+  const int T = n_tasks_of(cfg), HN = head_cols(cfg);
+  c->n_tasks = T;
+  if ((rc = make_weight(c, c->w1h, HN, d, 512)) != FE_OK) return fail(rc);
+  for (int t = 0; t < T; ++t)
+    if ((rc = fill_weight(c->w1h, hw(c, t, 0), d, d, t * d)) != FE_OK) return fail(rc);
+  {
+    const size_t nv = 2 * (size_t)HN + 2 * T + 1;
+    if (cudaMalloc(&c->head_vec, nv * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+    c->owned_w.push_back(c->head_vec);
+    FE_CK(cudaMemset(c->head_vec, 0, nv * sizeof(float)));
+    for (int t = 0; t < T; ++t) {
+      FE_CK(cudaMemcpy(c->head_vec + t * d, hw(c, t, 1), d * sizeof(float), cudaMemcpyDeviceToDevice));
+      FE_CK(cudaMemcpy(c->head_vec + HN + t * d, hw(c, t, 2), d * sizeof(float), cudaMemcpyDeviceToDevice));
+      FE_CK(cudaMemcpy(c->head_vec + 2 * HN + t, hw(c, t, 3), sizeof(float), cudaMemcpyDeviceToDevice));
+    }
+    if (T > 1) {
+      FE_CK(cudaMemcpy(c->head_vec + 2 * HN + T, hw(c, T, 0), (T + 1) * sizeof(float), cudaMemcpyDeviceToDevice));
+    } else {
+      const float one = 1.f;  // a single head: its score is the score
+      FE_CK(cudaMemcpy(c->head_vec + 2 * HN + 1, &one, sizeof(float), cudaMemcpyHostToDevice));
+    }
+  }
   // weight-only products of SeqEnc: [CLS] W and P W
   const int mL = cfg->max_L;
   float* consts = nullptr;
@@ -1272,9 +1329,17 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
     rows = (size_t)s.B * s.K;
     cols = d;
   } else if (n == "cross") {
+    if (c->cfg.no_cross_seq) {
+      g_msg = "no cross-sequence block in this configuration (C' = C: fetch \"seq\")";
+      return FE_ERR_UNSUPPORTED;
+    }
     f32 = c->cp.p;
     rows = (size_t)s.B * s.K;
     cols = d;
+  } else if (n == "task_scores") {
+    f32 = c->task_scores;
+    rows = (size_t)s.B * s.K;
+    cols = (size_t)c->n_tasks;
   } else {
     g_msg = "unknown buffer name";
     return FE_ERR_INVALID_ARG;

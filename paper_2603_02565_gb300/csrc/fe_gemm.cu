@@ -422,19 +422,55 @@ __global__ void __launch_bounds__(kThreads, 1)
           stage_split(hi, lo, c, srow);
         }
       } else {  // EPI_HEAD
-        float accv = 0.f;
-        for (int c = 32 * half; c < BN; c += 64) {
+        // per task t: the dot product of ReLU(acc + b1) with w2 over its
+        // head_d columns (a 32-column block lies in one task, head_d % 32 == 0)
+        const int nt = p.n_tasks, ncol = nt * p.head_d;
+        float acc4[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int c = 32 * half; c < ncol; c += 64) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
+          float a = 0.f;
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
             const float x = fmaxf(v[i] + p.bias[c + i], 0.f);
-            accv = fmaf(x, p.w2[c + i], accv);
+            a = fmaf(x, p.w2[c + i], a);
+          }
+          const int t = c / p.head_d;
+#pragma unroll
+          for (int tt = 0; tt < 4; ++tt)
+            if (tt == t) acc4[tt] += a;
+        }
+        // both halves' partial sums, two tasks per exchange
+        float tot[4];
+#pragma unroll
+        for (int t0 = 0; t0 < 4; t0 += 2) {
+          if (t0 < nt) {
+            if (t0 > 0) pair_sync();  // the previous round's reads are done
+            red_sum[half * 128 + r] = acc4[t0];
+            red_var[half * 128 + r] = acc4[t0 + 1];
+            pair_sync();
+            tot[t0] = red_sum[r] + red_sum[128 + r];
+            tot[t0 + 1] = red_var[r] + red_var[128 + r];
           }
         }
-        red_sum[half * 128 + r] = accv;
-        pair_sync();
-        if (half == 0 && valid) p.scores[grow] = (red_sum[r] + red_sum[128 + r]) + p.b2[0];
+        if (half == 0 && valid) {
+          if (nt == 1) {
+            const float s0 = tot[0] + p.b2[0];
+            p.scores[grow] = s0;
+            if (p.task_scores) p.task_scores[grow] = s0;
+          } else {
+            float f = p.fuse_b[0];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              if (t < nt) {
+                const float st = tot[t] + p.b2[t];
+                if (p.task_scores) p.task_scores[(size_t)grow * nt + t] = st;
+                f = fmaf(p.fuse_w[t], st, f);
+              }
+            }
+            p.scores[grow] = f;
+          }
+        }
       }
       // every TMEM read of this accumulator has completed (tcgen05.wait::ld)
       tc_fence_before();

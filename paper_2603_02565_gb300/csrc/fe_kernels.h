@@ -48,7 +48,8 @@ inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
 enum GemmEpilogue : int {
   EPI_STORE = 0,    // out = [ReLU](acc + bias) as split planes
   EPI_RESID_LN = 1, // x = resid + acc + bias -> x_out (fp32) and LN(x) as split planes; BN == N
-  EPI_HEAD = 2,     // s = ReLU(acc + bias) . w2 + b2 -> scores (fp32); BN == N
+  EPI_HEAD = 2,     // task heads s_t = ReLU(acc_t + bias_t) . w2_t + b2_t over column blocks of
+                   // head_d, fused s = sum_t fuse_w[t] s_t + fuse_b (one task: s = s_0); BN == N
 };
 
 struct GemmParams {
@@ -68,9 +69,14 @@ struct GemmParams {
   int ldr;
   float eps;
   // EPI_HEAD
-  const float* w2;
-  const float* b2;
-  float* scores;
+  int n_tasks;          // 1..4 heads of head_d columns each (columns past n_tasks * head_d are padding)
+  int head_d;
+  const float* w2;      // [N]
+  const float* b2;      // [n_tasks]
+  const float* fuse_w;  // [n_tasks] (n_tasks > 1)
+  const float* fuse_b;  // [1] (n_tasks > 1)
+  float* scores;        // [rows]
+  float* task_scores;   // [rows, n_tasks] or null
   int* status;
 };
 

@@ -33,6 +33,8 @@ class ModelConfig:
     max_L: int = 64   # rows of the position-embedding table
     io_bf16: bool = True  # inputs are bf16-valued (False: plain fp32 inputs)
     ln_eps: float = 1e-5
+    n_tasks: int = 1      # task-specific prediction heads; > 1 adds the fusion module
+    cross_seq: bool = True  # False: the variant without cross-sequence interaction
 
     @property
     def F(self) -> int:
@@ -74,17 +76,28 @@ def param_shapes(cfg: ModelConfig):
                 (f"W2.{l}", (F, d)), (f"b2.{l}", (d,))]
     out += [("P", (cfg.max_L, d)), ("cls", (d,)),
             ("WQs", (d, d)), ("WKs", (d, d)), ("WVs", (d, d)), ("WOs", (d, d)),
-            ("W1s", (d, F)), ("b1s", (F,)), ("W2s", (F, d)), ("b2s", (d,)),
-            ("WQx", (d, d)), ("WKx", (d, d)), ("WVx", (d, d)), ("WOx", (d, d)),
-            ("W1h", (d, d)), ("b1h", (d,)), ("w2h", (d,)), ("b2h", (1,))]
+            ("W1s", (d, F)), ("b1s", (F,)), ("W2s", (F, d)), ("b2s", (d,))]
+    if cfg.cross_seq:
+        out += [("WQx", (d, d)), ("WKx", (d, d)), ("WVx", (d, d)), ("WOx", (d, d))]
+    if cfg.n_tasks == 1:
+        out += [("W1h", (d, d)), ("b1h", (d,)), ("w2h", (d,)), ("b2h", (1,))]
+    else:
+        for t in range(cfg.n_tasks):
+            out += [(f"W1h.{t}", (d, d)), (f"b1h.{t}", (d,)), (f"w2h.{t}", (d,)), (f"b2h.{t}", (1,))]
+        out += [("fuse_w", (cfg.n_tasks,)), ("fuse_b", (1,))]
     return out
 
 
 def make_weights(cfg: ModelConfig, rng: np.random.Generator, std: float = 0.02) -> dict:
-    """Every parameter (biases, position table and [CLS] included) ~ N(0, std)."""
+    """Every parameter (biases, position table and [CLS] included) ~ N(0, std),
+    except the fusion weights of a multi-task head, which are positive task
+    importances ~ U(0.5, 1.5)."""
     w = {}
     for name, shape in param_shapes(cfg):
-        a = rng.normal(0.0, std, size=shape).astype(np.float32)
+        if name == "fuse_w":
+            a = rng.uniform(0.5, 1.5, size=shape).astype(np.float32)
+        else:
+            a = rng.normal(0.0, std, size=shape).astype(np.float32)
         w[name] = round_to_bf16(a) if cfg.io_bf16 else a
     return w
 
@@ -125,8 +138,9 @@ def _normal(rng, shape, std, bf16):
 
 
 def _rec_workload(name, seed, B, C, d, H, Ly, M, K, L, zipf_s, ctx_std, pool_std,
-                  io_bf16=True, idx_seed=None, max_L=None):
-    cfg = ModelConfig(d=d, n_heads=H, n_layers=Ly, max_L=max_L or L, io_bf16=io_bf16)
+                  io_bf16=True, idx_seed=None, max_L=None, n_tasks=1, cross_seq=True):
+    cfg = ModelConfig(d=d, n_heads=H, n_layers=Ly, max_L=max_L or L, io_bf16=io_bf16,
+                      n_tasks=n_tasks, cross_seq=cross_seq)
     rng = np.random.default_rng(seed)
     weights = make_weights(cfg, rng)
     context = _normal(rng, (B, C, d), ctx_std, io_bf16)
