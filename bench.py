@@ -47,8 +47,13 @@ def make_workload(args, seed_offset=0):
         kw["n_tasks"] = args.tasks
     if args.no_cross_seq:
         kw["cross_seq"] = False
-    if (args.tasks != 1 or args.no_cross_seq) and args.workload not in ("serving", "ksweep", "stress"):
-        raise SystemExit("--tasks / --no-cross-seq apply to the recommendation workloads")
+    if args.elem_self_attn:
+        kw["elem_self_attn"] = True
+    if args.encode_pool:
+        kw["encode_pool"] = True
+    if kw.keys() - {"B"} and args.workload not in ("serving", "ksweep", "stress"):
+        raise SystemExit("--tasks / --no-cross-seq / --elem-self-attn / --encode-pool apply to the "
+                         "recommendation workloads")
     if args.workload == "serving":
         return wl.serving(seed=1 + seed_offset, **kw)
     if args.workload == "ksweep":
@@ -82,6 +87,10 @@ def site_work(site, cfg, B, C, M, K, L, R):
     H = 2
     t = {
         "compact": (0, 4 * B * K * L * 2 + 4 * R + 12 * B),
+        "pool_layout": (0, 4 * B * K * L * 2 + 4 * R + 12 * B),
+        "gemm_elem_qkv": (6 * R * d * d, R * d * A + 3 * R * d * H),
+        "attn_elem_self": (4 * R * (R / max(B, 1)) * d, 3 * R * d * H + R * d * A),
+        "gemm_elem_o_ln": (2 * R * d * d, R * d * (A + 8 + A)),
         "ctx_ln": (0, n * d * (esz + A)),
         "gemm_ctx_kv": (2 * n * d * 2 * Ly * d, n * d * A + n * 2 * Ly * d * H),
         "ctx_ln_kv": (2 * n * d * 2 * Ly * d, n * d * esz + n * 2 * Ly * d * H),
@@ -425,7 +434,9 @@ def run_ours(args):
                        "mode": ("candidate-factorized E^ind (fe_evaluate_factorized)" if args.factorized
                                 else "joint (fe_evaluate)")
                                + (f", {args.tasks} task heads + linear fusion" if args.tasks != 1 else "")
-                               + (", without cross-sequence interaction" if args.no_cross_seq else ""),
+                               + (", without cross-sequence interaction" if args.no_cross_seq else "")
+                               + (", element self-attention H^(1)" if args.elem_self_attn else "")
+                               + (", whole pool encoded (U = M)" if args.encode_pool else ""),
                        "parallelism": f"dp{world} (requests sharded, no collective)",
                        "precision": "bf16 MMA operands with activations split hi+lo bf16; attention Q, K, V, "
                                     "P single f16; fp32 accumulate, softmax, LayerNorm and residuals",
@@ -516,6 +527,10 @@ def main():
                     help="task-specific prediction heads with a linear fusion (end of Section 4.4)")
     ap.add_argument("--no-cross-seq", action="store_true",
                     help="the variant without cross-sequence interaction (Appendix B.4)")
+    ap.add_argument("--elem-self-attn", action="store_true",
+                    help="self-attention H^(1) over each request's element set (Section 4.2)")
+    ap.add_argument("--encode-pool", action="store_true",
+                    help="encode the whole pool (U(z) = C(x), U = M) instead of the distinct elements")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args()

@@ -76,6 +76,11 @@ typedef struct fe_config {
                          s_k = sum_t fuse_w[t] s_{k,t} + fuse_b (T * d <= 512)      */
   int32_t no_cross_seq; /* 1: the variant without cross-sequence interaction
                          (Appendix B.4, "- CrossSeq"): C' = C; 0: the full model    */
+  int32_t elem_self_attn; /* 1: self-attention over the request's element set before
+                         the cross-attention stack, H^(1) of Section 4.2:
+                         h += MHA(LN(h) WQe, LN(h) WKe, LN(h) WVe) WOe over the set  */
+  int32_t encode_pool;  /* 1: the element set is the whole pool (U(z) = C(x), U = M,
+                         Section 4.1) instead of the distinct sequence elements    */
 } fe_config;
 
 typedef struct fe_ctx fe_ctx;
@@ -92,6 +97,7 @@ typedef struct fe_ctx fe_ctx;
  *   for t in 0..T-1 (T = max(n_tasks, 1)):
  *     W1h_t[d,d] b1h_t[d] w2h_t[d] b2h_t[1]      (task t's head)
  *   fuse_w[T] fuse_b[1]                          (only when T >= 2)
+ *   WQe[d,d] WKe[d,d] WVe[d,d] WOe[d,d]          (only when elem_self_attn = 1)
  */
 size_t fe_weight_count(const fe_config* cfg);
 

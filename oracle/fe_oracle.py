@@ -28,6 +28,11 @@ s = Inter(c), then Eq. 1's argmax):
   learned linear combination s_k = sum_t alpha_t s_{k,t} + beta.
 * Variant without cross-sequence interaction ("- CrossSeq", ablation of
   Appendix B.4): C' = C, each sequence scored on its own representation.
+* Element self-attention H^(1) (Section 4.2), optional: before the
+  cross-attention stack, h += MHA(LN(h) W_Qe, LN(h) W_Ke, LN(h) W_Ve) W_Oe
+  over the request's element set (a pre-LN block with residual, like the
+  cross-sequence block).  The element set is U(z), or with encode_pool the
+  whole pool (U(z) = C(x), U = M, Section 4.1).
 
 The paper leaves the block internals open (norm placement, FFN, pooling, head
 shape).  The readings taken here: pre-LN blocks with LayerNorm without affine
@@ -47,9 +52,9 @@ from __future__ import annotations
 
 import numpy as np
 
-__all__ = ["layer_norm", "softmax", "mha", "context_kv", "encode_elements",
+__all__ = ["layer_norm", "softmax", "mha", "context_kv", "elem_self_attention", "encode_elements",
            "seq_encode", "cross_sequence", "score_head", "task_heads", "select_best",
-           "distinct_layout", "evaluate_request", "evaluate"]
+           "distinct_layout", "element_set", "evaluate_request", "evaluate"]
 
 
 # -- building blocks --------------------------------------------------------
@@ -99,6 +104,15 @@ def context_kv(context_b, W, n_layers, eps):
     [(K_1, V_1), ..., (K_Ly, V_Ly)], each [C, d]."""
     X = layer_norm(context_b, eps)
     return [(X @ _w(W, f"WK.{l}"), X @ _w(W, f"WV.{l}")) for l in range(n_layers)]
+
+
+def elem_self_attention(h, W, n_heads, eps):
+    """H^(1) of Section 4.2 over the rows of h, one request's element set:
+    h + MHA(Z W_Qe, Z W_Ke, Z W_Ve) W_Oe with Z = LN(h), every element
+    attending to every element of the set."""
+    h = np.asarray(h, dtype=np.float64)
+    Z = layer_norm(h, eps)
+    return h + mha(Z @ _w(W, "WQe"), Z @ _w(W, "WKe"), Z @ _w(W, "WVe"), n_heads) @ _w(W, "WOe")
 
 
 def encode_elements(h0, kv, W, n_heads, eps):
@@ -171,6 +185,15 @@ def distinct_layout(cand_b):
     return uniq.astype(np.int32), slots
 
 
+def element_set(cand_b, M, cfg):
+    """The element set a request encodes and every occurrence's slot in it:
+    U(z) (distinct_layout), or with cfg.encode_pool the whole pool
+    (U(z) = C(x), Section 4.1): rows 0..M-1, slot = the pool index."""
+    if getattr(cfg, "encode_pool", False):
+        return np.arange(M, dtype=np.int32), np.asarray(cand_b, dtype=np.int32).copy()
+    return distinct_layout(cand_b)
+
+
 # -- whole evaluator ---------------------------------------------------------
 
 def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse", tasks_out=None):
@@ -179,18 +202,28 @@ def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse", tasks_out=
     per-task scores [K, T] are appended to it."""
     H, Ly, eps = cfg.n_heads, cfg.n_layers, cfg.ln_eps
     K, L = cand_b.shape
+    pool_b = np.asarray(pool_b, np.float64)
+    uniq, slots = element_set(cand_b, pool_b.shape[0], cfg)
+    self_attn = getattr(cfg, "elem_self_attn", False)
     if mode == "reuse":
         kv = context_kv(context_b, W, Ly, eps)
-        uniq, slots = distinct_layout(cand_b)
-        Henc = encode_elements(np.asarray(pool_b, np.float64)[uniq], kv, W, H, eps)
+        h0 = pool_b[uniq]
+        if self_attn:
+            h0 = elem_self_attention(h0, W, H, eps)
+        Henc = encode_elements(h0, kv, W, H, eps)
         rows = [Henc[slots[k]] for k in range(K)]
     elif mode == "no_reuse":
         rows = []
         for k in range(K):
             kv = context_kv(context_b, W, Ly, eps)          # per sequence
-            r = np.vstack([encode_elements(np.asarray(pool_b, np.float64)[[m]], kv, W, H, eps)
-                           for m in cand_b[k]])             # per occurrence
-            rows.append(r)
+            r = []
+            for j, m in enumerate(cand_b[k]):               # per occurrence
+                if self_attn:                               # H^(1) over the set, recomputed
+                    h0 = elem_self_attention(pool_b[uniq], W, H, eps)[[slots[k, j]]]
+                else:
+                    h0 = pool_b[[m]]
+                r.append(encode_elements(h0, kv, W, H, eps))
+            rows.append(np.vstack(r))
     else:
         raise ValueError(mode)
     Cm = np.vstack([seq_encode(rows[k], W, H, eps) for k in range(K)])
@@ -227,7 +260,7 @@ def evaluate(context, pool, cand_idx, W, cfg, mode="reuse", requests=None, with_
         cb = cand_idx[b]
         if cb.size and (cb.min() < 0 or cb.max() >= M):
             continue
-        uniq, sl = distinct_layout(cb)
+        uniq, sl = element_set(cb, M, cfg)
         U[b] = len(uniq)
         slots[b] = sl
         if K == 0:

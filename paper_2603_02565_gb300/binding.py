@@ -38,7 +38,8 @@ EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evalua
 class FeConfig(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("n_layers", ctypes.c_int32),
                 ("ffn_mult", ctypes.c_int32), ("max_L", ctypes.c_int32), ("io_dtype", ctypes.c_int32),
-                ("ln_eps", ctypes.c_float), ("n_tasks", ctypes.c_int32), ("no_cross_seq", ctypes.c_int32)]
+                ("ln_eps", ctypes.c_float), ("n_tasks", ctypes.c_int32), ("no_cross_seq", ctypes.c_int32),
+                ("elem_self_attn", ctypes.c_int32), ("encode_pool", ctypes.c_int32)]
 
 
 class FeError(RuntimeError):
@@ -104,7 +105,7 @@ def _check(rc, allowed=(FE_OK,)):
     return rc
 
 
-def weight_order(n_layers: int, n_tasks: int = 1, cross_seq: bool = True):
+def weight_order(n_layers: int, n_tasks: int = 1, cross_seq: bool = True, elem_self_attn: bool = False):
     """Tensor names in the order fe.h documents for fe_init."""
     names = []
     for l in range(n_layers):
@@ -118,6 +119,8 @@ def weight_order(n_layers: int, n_tasks: int = 1, cross_seq: bool = True):
         for t in range(n_tasks):
             names += [f"W1h.{t}", f"b1h.{t}", f"w2h.{t}", f"b2h.{t}"]
         names += ["fuse_w", "fuse_b"]
+    if elem_self_attn:
+        names += ["WQe", "WKe", "WVe", "WOe"]
     return names
 
 
@@ -129,16 +132,21 @@ def _cross(cfg):
     return bool(getattr(cfg, "cross_seq", True))
 
 
+def _flag(cfg, name):
+    return 1 if getattr(cfg, name, False) else 0
+
+
 def make_config(cfg) -> FeConfig:
     """fe_config from any object with d, n_heads, n_layers, ffn_mult, max_L, io_bf16, ln_eps
-    (and optionally n_tasks, cross_seq)."""
+    (and optionally n_tasks, cross_seq, elem_self_attn, encode_pool)."""
     return FeConfig(cfg.d, cfg.n_heads, cfg.n_layers, cfg.ffn_mult, cfg.max_L,
-                    FE_IO_BF16 if cfg.io_bf16 else FE_IO_F32, cfg.ln_eps, _tasks(cfg), 0 if _cross(cfg) else 1)
+                    FE_IO_BF16 if cfg.io_bf16 else FE_IO_F32, cfg.ln_eps, _tasks(cfg), 0 if _cross(cfg) else 1,
+                    _flag(cfg, "elem_self_attn"), _flag(cfg, "encode_pool"))
 
 
 def pack_weights(cfg, weights: dict) -> np.ndarray:
     parts = [np.ascontiguousarray(weights[n], dtype=np.float32).ravel()
-             for n in weight_order(cfg.n_layers, _tasks(cfg), _cross(cfg))]
+             for n in weight_order(cfg.n_layers, _tasks(cfg), _cross(cfg), bool(_flag(cfg, "elem_self_attn")))]
     return np.concatenate(parts)
 
 

@@ -258,6 +258,7 @@ struct fe_ctx {
   Weight ctx_kv;
   std::vector<Weight> wq, wo, w1, w2;
   Weight kvs, os, w1s, w2s, qkvx, ox, w1h;
+  Weight qkve, oe;                  // element self-attention H^(1): [WQe | WKe | WVe], WOe
   int n_tasks = 1;                  // task heads T
   float* head_vec = nullptr;        // b1 [head cols] | w2 [head cols] | b2 [T] | fuse_w [T] | fuse_b [1]
   float* task_scores = nullptr;     // [S, T], every head's score of the last batch
@@ -269,7 +270,7 @@ struct fe_ctx {
   long long kv_rows = 0;      // context K/V rows of the reservation: B * C, or B * K * C
   int *status = nullptr, *U = nullptr, *off = nullptr, *bad = nullptr, *slot = nullptr, *list = nullptr;
   unsigned* ticket = nullptr;
-  Planes X, KV, xln, q, a, mid, kvI, o, cln, mids, z, qkv, ax, lncp;
+  Planes X, KV, xln, q, a, mid, kvI, o, cln, mids, z, qkv, ax, lncp, eqkv;  // eqkv: H^(1) Q | K | V
   F32Rows h, c, cp;
   void* in_ctx = nullptr;
   void* in_pool = nullptr;
@@ -362,6 +363,8 @@ bool config_ok(const fe_config* c) {
   if (!(c->ln_eps >= 0.f)) return false;
   if (c->n_tasks < 0 || c->n_tasks > 4 || (c->n_tasks > 1 && c->n_tasks * d > 512)) return false;
   if (c->no_cross_seq != 0 && c->no_cross_seq != 1) return false;
+  if (c->elem_self_attn != 0 && c->elem_self_attn != 1) return false;
+  if (c->encode_pool != 0 && c->encode_pool != 1) return false;
   return true;
 }
 
@@ -406,8 +409,13 @@ std::vector<size_t> weight_sizes(const fe_config* c) {
     s.push_back((size_t)T);           // fuse_w
     s.push_back(1);                   // fuse_b
   }
+  if (c->elem_self_attn)
+    for (int i = 0; i < 4; ++i) s.push_back(d * d);  // WQe WKe WVe WOe
   return s;
 }
+
+// element self-attention weight i (0 WQe, 1 WKe, 2 WVe, 3 WOe): the last four tensors
+const float* ew(const fe_ctx* c, int i);
 
 // tensor indices into weight_sizes()
 enum { T_WQ = 0, T_WK, T_WV, T_WO, T_W1, T_B1, T_W2, T_B2, T_PER_LAYER };
@@ -420,6 +428,7 @@ const float* lw(const fe_ctx* c, int l, int i) { return wptr(c, T_PER_LAYER * l 
 const float* tw(const fe_ctx* c, int i) { return wptr(c, t_tail(c, i)); }
 // task t's head tensor j (0 W1h, 1 b1h, 2 w2h, 3 b2h); the fusion weights follow the last head
 const float* hw(const fe_ctx* c, int t, int j) { return tw(c, T_W1H + 4 * t + j); }
+const float* ew(const fe_ctx* c, int i) { return wptr(c, (int)c->woff.size() - 4 + i); }
 
 // Allocate the transposed weight [N, K_pad] and pick its tiling.
 int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
@@ -513,7 +522,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   const int d = c->d, Ly = c->Ly;
   const int io_f32 = c->cfg.io_dtype == FE_IO_F32;
   const bool fact = sh.fact;  // every occurrence its own element, one context K/V per sequence
-  const int cap = fact ? K * L : ((M < K * L) ? M : K * L);
+  const int cap = fact ? K * L : (c->cfg.encode_pool ? M : ((M < K * L) ? M : K * L));
   const int R = B * cap;
   const int S = B * K;
   c->launches_batch = 0;
@@ -529,6 +538,9 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   if (fact) {
     Prof pf(c, "layout", s);
     FE_CK(fe::identity_layout_launch(io.idx, B, M, K * L, c->U, c->off, c->bad, c->slot, c->list, c->status, s));
+  } else if (c->cfg.encode_pool) {
+    Prof pf(c, "pool_layout", s);
+    FE_CK(fe::pool_layout_launch(io.idx, B, M, K * L, c->U, c->off, c->bad, c->slot, c->list, c->status, s));
   } else {
     Prof pf(c, "compact", s);
     FE_CK(fe::compact_launch(io.idx, B, M, K, L, cap, c->U, c->off, c->bad, c->slot, c->list, c->status, c->ticket,
@@ -563,6 +575,38 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     Prof pf(c, "gather_ln", s);
     FE_CK(fe::gather_ln_launch(io.pool, io_f32, B, M, d, cap, c->off, c->list, R, c->cfg.ln_eps, c->h.p, d, c->xln.h,
                              c->xln.l, c->xln.ld, s));
+  }
+  // (a2') element self-attention H^(1) over each request's element set
+  // (Section 4.2): h += MHA(LN(h) WQe, LN(h) WKe, LN(h) WVe) WOe, the keys and
+  // values of a request being its own element rows
+  if (c->cfg.elem_self_attn && !fact) {
+    fe::GemmParams p{};
+    p.out_f16 = 1;
+    FE_RC(gemm(c, "gemm_elem_qkv", fe::EPI_STORE, c->xln, c->qkve, R, sumU, p, &c->eqkv, nullptr, s));
+    fe::AttnParams ap{};
+    ap.n_segments = B;
+    ap.max_q = cap;
+    ap.q_off_dev = c->off;
+    ap.q_cnt_dev = c->U;
+    ap.kv_self = 1;
+    ap.n_heads = c->H;
+    ap.q_col = 0;
+    ap.k_col = d;
+    ap.v_col = 2 * d;
+    ap.o_col = 0;
+    ap.o_h = c->a.h;
+    ap.o_l = c->a.l;
+    ap.ldo = c->a.ld;
+    ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
+    ap.status = c->status;
+    {
+      Prof pf(c, "attn_elem_self", s);
+      FE_CK(fe::attn_launch(c->dh, &c->eqkv.ah, &c->eqkv.kh, &c->eqkv.kh, ap, s));
+    }
+    fe::GemmParams po{};
+    po.resid = c->h.p;
+    po.ldr = d;
+    FE_RC(gemm(c, "gemm_elem_o_ln", fe::EPI_RESID_LN, c->a, c->oe, R, sumU, po, &c->xln, &c->h, s));
   }
   for (int l = 0; l < Ly; ++l) {
     fe::GemmParams p{};
@@ -774,7 +818,10 @@ int reserve_impl(fe_ctx* c, Shape s) {
   c->have_last = false;
   const int d = c->d, Ly = c->Ly;
   const long long capL = (long long)s.K * s.L;
-  const int cap = (int)(fact ? capL : ((s.M < capL) ? s.M : capL));
+  // element rows per request: the distinct elements (at most min(M, K*L)),
+  // the whole pool (M), and K*L once the factorized evaluation is used
+  const long long cap_joint = c->cfg.encode_pool ? s.M : ((s.M < capL) ? s.M : capL);
+  const int cap = (int)std::max(cap_joint, fact ? capL : 0ll);
   const int B = s.B > 0 ? s.B : 1;
   const int R = B * (cap > 0 ? cap : 1);
   const int S = B * (s.K > 0 ? s.K : 1);
@@ -830,12 +877,14 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(alloc_planes(c->mids, S, c->Fpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->z, S, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->qkv, S, 3 * d, false, c->owned_ws));
+  if (c->cfg.elem_self_attn) FE_RC(alloc_planes(c->eqkv, R, 3 * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->ax, S, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->lncp, S, c->dpad, true, c->owned_ws));
   if (!c->fused_ctxkv) FE_RC(map_act(c->X));
   for (Planes* p : {&c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp}) FE_RC(map_act(*p));
   for (Planes* p : {&c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->lncp}) FE_RC(map_out(*p));
   for (Planes* p : {&c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
+  if (c->cfg.elem_self_attn) FE_RC(map_attn(c->eqkv, c->dh));
   FE_RC(c->fused_ctxkv ? map_attn_hm(c->KV, c->dh) : map_attn(c->KV, c->dh));
   c->cap_shape = s;
   c->cap_shape.fact = false;
@@ -1044,6 +1093,13 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     if ((rc = make_weight(c, c->ox, d, d, 512)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->ox, tw(c, T_WOX), d, d, 0)) != FE_OK) return fail(rc);
   }
+  if (cfg->elem_self_attn) {
+    if ((rc = make_weight(c, c->qkve, 3 * d, d, 128)) != FE_OK) return fail(rc);
+    for (int i = 0; i < 3; ++i)
+      if ((rc = fill_weight(c->qkve, ew(c, i), d, d, i * d)) != FE_OK) return fail(rc);
+    if ((rc = make_weight(c, c->oe, d, d, 512)) != FE_OK) return fail(rc);
+    if ((rc = fill_weight(c->oe, ew(c, 3), d, d, 0)) != FE_OK) return fail(rc);
+  }
   // the task heads' first layers as one product of head_cols(cfg) columns
   // (task t in columns [t d, t d + d), padding columns zero), and their
   // vectors gathered into one buffer
@@ -1150,6 +1206,11 @@ int fe_evaluate_factorized(fe_ctx* c, int B, int C, int M, int K, int L, const v
   FE_RC(check_io(context, pool, cand_idx, scores_out, best_out, B, M, K, L));
   if (!c->fused_ctxkv || C % 128 != 0) {
     g_msg = "the factorized evaluation needs d <= 128, bf16 inputs and weights, and C a multiple of 128";
+    return FE_ERR_UNSUPPORTED;
+  }
+  if (c->cfg.encode_pool || c->cfg.elem_self_attn) {
+    g_msg = "the factorized evaluation encodes every occurrence on its own; encode_pool and the element "
+            "self-attention over a set do not apply";
     return FE_ERR_UNSUPPORTED;
   }
   // with no pool row every index is out of range: the joint evaluation gives the same outputs

@@ -161,7 +161,11 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qtiles = p.max_q_tiles;
   const int units = p.n_segments * p.n_heads * qtiles;
-  const int nch = (p.kv_cnt + CK - 1) / CK;
+  // keys of a unit's segment: a fixed count at a fixed stride, or, for
+  // self-attention within segments, the segment's own query rows
+  auto kv_count = [&](const Cursor& c) { return p.kv_self ? c.qcnt : p.kv_cnt; };
+  auto kv_base = [&](const Cursor& c) { return p.kv_self ? c.qoff : c.b * p.kv_stride; };
+  auto chunks = [&](const Cursor& c) { return (kv_count(c) + CK - 1) / CK; };
   if ((int)blockIdx.x >= units) return;
 
   if (threadIdx.x == 0) {
@@ -206,6 +210,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         uint8_t* q = sQ + qb * Cfg::kQBytes;
         mbar_arrive_expect_tx(q_full + qb, Cfg::kQBytes);
         tma_load_2d(q, &tQ, p.q_col + c.h * DH, c.qoff + c.q0, q_full + qb);
+        const int nch = chunks(c);
         for (int j = 0; j < nch; ++j, ++gc) {
           const int ks = gc % Cfg::kKVStages;
           if (gc >= Cfg::kKVStages &&
@@ -214,7 +219,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
             break;
           }
           uint8_t* kv = sKV + ks * Cfg::kKVBytes;
-          const int row = c.b * p.kv_stride + j * CK;
+          const int row = kv_base(c) + j * CK;
           mbar_arrive_expect_tx(kv_full + ks, Cfg::kKVBytes);
           if (p.kv3d) {  // head-major K/V: one contiguous block per head
             tma_load_3d(kv, &tK, 0, row, (p.k_col + c.h * DH) / DH, kv_full + ks);
@@ -260,7 +265,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           umma_bf16(dst, desc_adv(q0d, kk * 32), desc_adv(k0d, kk * 32), idesc_s, kk != 0 ? 1u : 0u);
         umma_commit(s_full + t);
         ++g_s;
-        if (++sj == nch) {  // every S of this unit issued: its Q buffer frees on completion
+        if (++sj == chunks(sc)) {  // every S of this unit issued: its Q buffer frees on completion
           umma_commit(q_empty + qb);
           sj = 0;
           ++sui;
@@ -358,6 +363,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       // a warp whose 32 query rows all lie past the segment's end only keeps
       // the barrier protocol; those rows of P and of the output are never used
       const bool active = c.q0 + q4 * 32 < c.qcnt;
+      const int nch = chunks(c);
       for (int j = 0; j < nch; ++j, ++gc) {
         const int t = gc % Cfg::kTiles;
         if (!mbar_wait_compact(s_full + t, (gc / Cfg::kTiles) & 1, p.status)) {
@@ -375,7 +381,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           else
             tmem_ld32(tile, v);
           // keys past kv_cnt take no part: -inf gives them P = 0
-          const int kvalid = p.kv_cnt - j * CK - half * KW;  // valid keys among this warp's KW
+          const int kvalid = kv_count(c) - j * CK - half * KW;  // valid keys among this warp's KW
           if (kvalid < KW) {
 #pragma unroll
             for (int i = 0; i < KW; ++i)
@@ -474,7 +480,7 @@ cudaError_t attn_prepare() {
 
 cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, const CUtensorMap* v, const AttnParams& p0,
                         cudaStream_t s) {
-  if (p0.n_segments <= 0 || p0.max_q <= 0 || p0.kv_cnt <= 0) return cudaSuccess;
+  if (p0.n_segments <= 0 || p0.max_q <= 0 || (!p0.kv_self && p0.kv_cnt <= 0)) return cudaSuccess;
   AttnParams p = p0;
   p.max_q_tiles = (p.max_q + BQ - 1) / BQ;
   const long long units = (long long)p.n_segments * p.n_heads * p.max_q_tiles;

@@ -141,7 +141,8 @@ cudaError_t ctxkv_launch(const CUtensorMap* x, const CUtensorMap* w, const CUten
 // Flash-style multi-head attention over request segments (tcgen05, f16
 // operands, fp32 accumulation and softmax).  Segment b: query rows
 // [q_off(b), q_off(b) + q_cnt(b)), key and value rows
-// [b * kv_stride, b * kv_stride + kv_cnt).  Head h reads columns q_col + h*dh
+// [b * kv_stride, b * kv_stride + kv_cnt), or, with kv_self, the segment's
+// own rows [q_off(b), q_off(b) + q_cnt(b)) (self-attention within segments).  Head h reads columns q_col + h*dh
 // of Q, k_col + h*dh of K, v_col + h*dh of V (each one f16 plane) and writes
 // columns o_col + h*dh of the bf16 hi/lo output planes.  The Q map has boxes
 // of dh x 128, the K/V maps dh x (64 for dh = 32, else 128), with the 64-byte
@@ -159,6 +160,7 @@ struct AttnParams {
   int kv_cnt;
   int q_col, k_col, v_col, o_col;
   int kv3d;              // K/V head-major (3D maps: x within the head, row, block = column / dh)
+  int kv_self;           // keys / values are the segment's query rows (kv_stride, kv_cnt unused)
   bf16 *o_h, *o_l;
   int ldo;
   float scale_log2;      // log2(e) / sqrt(d_h)
@@ -179,6 +181,10 @@ cudaError_t misc_prepare();
 // U[b] = K*L, off[b] = b*K*L (off[B] = B*K*L), list[b*K*L + i] = cand[b, i],
 // slot[b, i] = i; a request with an index outside [0, M) gets bad[b] = 1,
 // slot -1, list entries 0 (in range for the gather; its scores become NaN).
+// Whole-pool layout: U[b] = M, off[b] = b*M, list[b*M + i] = i, slot[b, i] =
+// cand[b, i]; a request with an index outside [0, M) gets bad[b] = 1, slots -1.
+cudaError_t pool_layout_launch(const int32_t* cand, int B, int M, int KL, int* U, int* off, int* bad, int* slot,
+                               int* list, int* status, cudaStream_t s);
 cudaError_t identity_layout_launch(const int32_t* cand, int B, int M, int KL, int* U, int* off, int* bad,
                                    int* slot, int* list, int* status, cudaStream_t s);
 cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int cap, int* U, int* off,

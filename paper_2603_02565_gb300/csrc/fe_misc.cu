@@ -276,6 +276,39 @@ cudaError_t identity_layout_launch(const int32_t* cand, int B, int M, int KL, in
   return launch_k(identity_layout_kernel, dim3(B), dim3(256), 0, s, cand, B, M, KL, U, off, bad, slot, list, status);
 }
 
+// Whole-pool layout (Section 4.1's alternative U(z) = C(x), U = M): every pool
+// row of request b is an element, list[b*M + i] = i, slot[b, i] = cand[b, i];
+// a request with an index outside [0, M) gets bad[b] = 1 and slots -1.
+__global__ void __launch_bounds__(256) pool_layout_kernel(const int32_t* __restrict__ cand, int B, int M, int KL,
+                                                          int* U, int* off, int* bad, int* slot, int* list,
+                                                          int* status) {
+  const int b = blockIdx.x;
+  pdl_wait();
+  pdl_trigger();
+  const int32_t* cb = cand + (size_t)b * KL;
+  int any_bad = 0;
+  for (int i = threadIdx.x; i < KL; i += blockDim.x) {
+    const int v = cb[i];
+    any_bad |= (v < 0 || v >= M);
+  }
+  any_bad = __syncthreads_or(any_bad);
+  for (int i = threadIdx.x; i < KL; i += blockDim.x) slot[(size_t)b * KL + i] = any_bad ? -1 : cb[i];
+  for (int i = threadIdx.x; i < M; i += blockDim.x) list[(size_t)b * M + i] = i;
+  if (threadIdx.x == 0) {
+    U[b] = M;
+    off[b] = b * M;
+    bad[b] = any_bad;
+    if (any_bad) atomicOr(status, ST_INDEX);
+    if (b == B - 1) off[B] = B * M;
+  }
+}
+
+cudaError_t pool_layout_launch(const int32_t* cand, int B, int M, int KL, int* U, int* off, int* bad, int* slot,
+                               int* list, int* status, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  return launch_k(pool_layout_kernel, dim3(B), dim3(256), 0, s, cand, B, M, KL, U, off, bad, slot, list, status);
+}
+
 // ---------------------------------------------------------------------------
 // LN of context rows -> split planes (one warp per row)
 // ---------------------------------------------------------------------------

@@ -35,6 +35,8 @@ class ModelConfig:
     ln_eps: float = 1e-5
     n_tasks: int = 1      # task-specific prediction heads; > 1 adds the fusion module
     cross_seq: bool = True  # False: the variant without cross-sequence interaction
+    elem_self_attn: bool = False  # self-attention H^(1) over the element set
+    encode_pool: bool = False     # the element set is the whole pool (U = M)
 
     @property
     def F(self) -> int:
@@ -85,6 +87,8 @@ def param_shapes(cfg: ModelConfig):
         for t in range(cfg.n_tasks):
             out += [(f"W1h.{t}", (d, d)), (f"b1h.{t}", (d,)), (f"w2h.{t}", (d,)), (f"b2h.{t}", (1,))]
         out += [("fuse_w", (cfg.n_tasks,)), ("fuse_b", (1,))]
+    if cfg.elem_self_attn:
+        out += [("WQe", (d, d)), ("WKe", (d, d)), ("WVe", (d, d)), ("WOe", (d, d))]
     return out
 
 
@@ -138,9 +142,11 @@ def _normal(rng, shape, std, bf16):
 
 
 def _rec_workload(name, seed, B, C, d, H, Ly, M, K, L, zipf_s, ctx_std, pool_std,
-                  io_bf16=True, idx_seed=None, max_L=None, n_tasks=1, cross_seq=True):
+                  io_bf16=True, idx_seed=None, max_L=None, n_tasks=1, cross_seq=True,
+                  elem_self_attn=False, encode_pool=False):
     cfg = ModelConfig(d=d, n_heads=H, n_layers=Ly, max_L=max_L or L, io_bf16=io_bf16,
-                      n_tasks=n_tasks, cross_seq=cross_seq)
+                      n_tasks=n_tasks, cross_seq=cross_seq, elem_self_attn=elem_self_attn,
+                      encode_pool=encode_pool)
     rng = np.random.default_rng(seed)
     weights = make_weights(cfg, rng)
     context = _normal(rng, (B, C, d), ctx_std, io_bf16)
