@@ -51,9 +51,17 @@ def make_workload(args, seed_offset=0):
         kw["elem_self_attn"] = True
     if args.encode_pool:
         kw["encode_pool"] = True
-    if kw.keys() - {"B"} and args.workload not in ("serving", "ksweep", "stress"):
-        raise SystemExit("--tasks / --no-cross-seq / --elem-self-attn / --encode-pool apply to the "
-                         "recommendation workloads")
+    if args.linear_attn:
+        kw["linear_context_attn"] = True
+    if args.context:
+        kw["C"] = args.context
+    if args.online:
+        # the online deployment's shape (Appendix B.3): 1,000-interaction contexts,
+        # a pool of 60, K = 50 sequences of 6, embedding width 64
+        kw.update(C=1000, M=60, d=64, H=2)
+    if kw.keys() - {"B"} and args.workload not in ("serving", "ksweep", "stress") or (args.online and args.workload != "serving"):
+        raise SystemExit("--tasks / --no-cross-seq / --elem-self-attn / --encode-pool / --linear-attn / "
+                         "--context apply to the recommendation workloads")
     if args.workload == "serving":
         return wl.serving(seed=1 + seed_offset, **kw)
     if args.workload == "ksweep":
@@ -88,6 +96,8 @@ def site_work(site, cfg, B, C, M, K, L, R):
     t = {
         "compact": (0, 4 * B * K * L * 2 + 4 * R + 12 * B),
         "pool_layout": (0, 4 * B * K * L * 2 + 4 * R + 12 * B),
+        "lin_state": (4 * n * d * Ly * (d // cfg.n_heads), 2 * n * d * Ly * H + 4 * B * Ly * (d * (d // cfg.n_heads) + d)),
+        "lin_attn_item_ctx": (2 * R * d * (d // cfg.n_heads), R * d * (H + A) + 4 * B * (d * (d // cfg.n_heads) + d)),
         "gemm_elem_qkv": (6 * R * d * d, R * d * A + 3 * R * d * H),
         "attn_elem_self": (4 * R * (R / max(B, 1)) * d, 3 * R * d * H + R * d * A),
         "gemm_elem_o_ln": (2 * R * d * d, R * d * (A + 8 + A)),
@@ -436,7 +446,8 @@ def run_ours(args):
                                + (f", {args.tasks} task heads + linear fusion" if args.tasks != 1 else "")
                                + (", without cross-sequence interaction" if args.no_cross_seq else "")
                                + (", element self-attention H^(1)" if args.elem_self_attn else "")
-                               + (", whole pool encoded (U = M)" if args.encode_pool else ""),
+                               + (", whole pool encoded (U = M)" if args.encode_pool else "")
+                               + (", linear context attention" if args.linear_attn else ""),
                        "parallelism": f"dp{world} (requests sharded, no collective)",
                        "precision": "bf16 MMA operands with activations split hi+lo bf16; attention Q, K, V, "
                                     "P single f16; fp32 accumulate, softmax, LayerNorm and residuals",
@@ -531,6 +542,11 @@ def main():
                     help="self-attention H^(1) over each request's element set (Section 4.2)")
     ap.add_argument("--encode-pool", action="store_true",
                     help="encode the whole pool (U(z) = C(x), U = M) instead of the distinct elements")
+    ap.add_argument("--linear-attn", action="store_true",
+                    help="linear (kernelized) element -> context attention, as the online deployment (Appendix B.3)")
+    ap.add_argument("--context", type=int, default=0, help="override the context length C")
+    ap.add_argument("--online", action="store_true",
+                    help="the online deployment's shape: C=1000, M=60, d=64 (2 heads), K=50, L=6")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args()

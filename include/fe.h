@@ -81,6 +81,12 @@ typedef struct fe_config {
                          h += MHA(LN(h) WQe, LN(h) WKe, LN(h) WVe) WOe over the set  */
   int32_t encode_pool;  /* 1: the element set is the whole pool (U(z) = C(x), U = M,
                          Section 4.1) instead of the distinct sequence elements    */
+  int32_t linear_context_attn; /* 1: the element -> context attention is linear
+                         (kernelized) attention with phi(x) = elu(x) + 1, as the
+                         online deployment uses for long contexts (Appendix B.3):
+                         per request, layer and head the context is a d_h x d_h
+                         state S = phi(K)^T V with z = sum phi(K); an element
+                         reads phi(q) S / (phi(q) . z)                           */
 } fe_config;
 
 typedef struct fe_ctx fe_ctx;

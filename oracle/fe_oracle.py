@@ -33,6 +33,13 @@ s = Inter(c), then Eq. 1's argmax):
   over the request's element set (a pre-LN block with residual, like the
   cross-sequence block).  The element set is U(z), or with encode_pool the
   whole pool (U(z) = C(x), U = M, Section 4.1).
+* Linear-attention context module, optional (the online deployment of
+  Appendix B.3 uses linear attention for its 1,000-interaction contexts):
+  the element -> context cross-attention becomes kernelized attention with
+  the feature map phi(x) = elu(x) + 1 of Katharopoulos et al. (2020), non-causal
+  over the context; per request, layer and head the context reduces to the
+  state S = phi(K)^T V and z = sum_c phi(K_c), and an element query reads
+  phi(q) S / (phi(q) . z).
 
 The paper leaves the block internals open (norm placement, FFN, pooling, head
 shape).  The readings taken here: pre-LN blocks with LayerNorm without affine
@@ -52,7 +59,7 @@ from __future__ import annotations
 
 import numpy as np
 
-__all__ = ["layer_norm", "softmax", "mha", "context_kv", "elem_self_attention", "encode_elements",
+__all__ = ["layer_norm", "softmax", "mha", "elu_feature", "linear_attention", "context_kv", "elem_self_attention", "encode_elements",
            "seq_encode", "cross_sequence", "score_head", "task_heads", "select_best",
            "distinct_layout", "element_set", "evaluate_request", "evaluate"]
 
@@ -89,6 +96,30 @@ def mha(q, k, v, n_heads):
     return out
 
 
+def elu_feature(x):
+    """phi(x) = elu(x) + 1: x + 1 for x > 0, exp(x) otherwise (positive everywhere)."""
+    x = np.asarray(x, dtype=np.float64)
+    return np.where(x > 0, x + 1.0, np.exp(np.minimum(x, 0.0)))
+
+
+def linear_attention(q, k, v, n_heads):
+    """Kernelized (linear) attention of query rows q [n, d] over key rows k
+    [m, d] with values v [m, d], heads as contiguous column blocks: per head,
+    out = phi(q) S / (phi(q) . z) with the context state S = phi(k)^T v
+    [d_h, d_h] and z = sum over the keys of phi(k) [d_h]."""
+    n, d = q.shape
+    dh = d // n_heads
+    out = np.empty((n, d), dtype=np.float64)
+    for h in range(n_heads):
+        cols = slice(h * dh, (h + 1) * dh)
+        fk = elu_feature(k[:, cols])
+        S = fk.T @ np.asarray(v[:, cols], dtype=np.float64)
+        z = fk.sum(axis=0)
+        fq = elu_feature(q[:, cols])
+        out[:, cols] = (fq @ S) / (fq @ z)[:, None]
+    return out
+
+
 def _relu(x):
     return np.maximum(x, 0.0)
 
@@ -115,13 +146,15 @@ def elem_self_attention(h, W, n_heads, eps):
     return h + mha(Z @ _w(W, "WQe"), Z @ _w(W, "WKe"), Z @ _w(W, "WVe"), n_heads) @ _w(W, "WOe")
 
 
-def encode_elements(h0, kv, W, n_heads, eps):
+def encode_elements(h0, kv, W, n_heads, eps, linear=False):
     """Request-conditioned representation of each element row of h0 [n, d]:
-    the cross-attention stack over the context K/V, then a final LN."""
+    the cross-attention stack over the context K/V (softmax attention, or
+    linear attention when `linear`), then a final LN."""
     h = np.array(h0, dtype=np.float64)
+    attend = linear_attention if linear else mha
     for l, (Kl, Vl) in enumerate(kv):
         q = layer_norm(h, eps) @ _w(W, f"WQ.{l}")
-        h = h + mha(q, Kl, Vl, n_heads) @ _w(W, f"WO.{l}")
+        h = h + attend(q, Kl, Vl, n_heads) @ _w(W, f"WO.{l}")
         f = _relu(layer_norm(h, eps) @ _w(W, f"W1.{l}") + _w(W, f"b1.{l}"))
         h = h + f @ _w(W, f"W2.{l}") + _w(W, f"b2.{l}")
     return layer_norm(h, eps)
@@ -205,12 +238,13 @@ def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse", tasks_out=
     pool_b = np.asarray(pool_b, np.float64)
     uniq, slots = element_set(cand_b, pool_b.shape[0], cfg)
     self_attn = getattr(cfg, "elem_self_attn", False)
+    lin = getattr(cfg, "linear_context_attn", False)
     if mode == "reuse":
         kv = context_kv(context_b, W, Ly, eps)
         h0 = pool_b[uniq]
         if self_attn:
             h0 = elem_self_attention(h0, W, H, eps)
-        Henc = encode_elements(h0, kv, W, H, eps)
+        Henc = encode_elements(h0, kv, W, H, eps, linear=lin)
         rows = [Henc[slots[k]] for k in range(K)]
     elif mode == "no_reuse":
         rows = []
@@ -222,7 +256,7 @@ def evaluate_request(context_b, pool_b, cand_b, W, cfg, mode="reuse", tasks_out=
                     h0 = elem_self_attention(pool_b[uniq], W, H, eps)[[slots[k, j]]]
                 else:
                     h0 = pool_b[[m]]
-                r.append(encode_elements(h0, kv, W, H, eps))
+                r.append(encode_elements(h0, kv, W, H, eps, linear=lin))
             rows.append(np.vstack(r))
     else:
         raise ValueError(mode)

@@ -39,7 +39,8 @@ class FeConfig(ctypes.Structure):
     _fields_ = [("d", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("n_layers", ctypes.c_int32),
                 ("ffn_mult", ctypes.c_int32), ("max_L", ctypes.c_int32), ("io_dtype", ctypes.c_int32),
                 ("ln_eps", ctypes.c_float), ("n_tasks", ctypes.c_int32), ("no_cross_seq", ctypes.c_int32),
-                ("elem_self_attn", ctypes.c_int32), ("encode_pool", ctypes.c_int32)]
+                ("elem_self_attn", ctypes.c_int32), ("encode_pool", ctypes.c_int32),
+                ("linear_context_attn", ctypes.c_int32)]
 
 
 class FeError(RuntimeError):
@@ -138,10 +139,10 @@ def _flag(cfg, name):
 
 def make_config(cfg) -> FeConfig:
     """fe_config from any object with d, n_heads, n_layers, ffn_mult, max_L, io_bf16, ln_eps
-    (and optionally n_tasks, cross_seq, elem_self_attn, encode_pool)."""
+    (and optionally n_tasks, cross_seq, elem_self_attn, encode_pool, linear_context_attn)."""
     return FeConfig(cfg.d, cfg.n_heads, cfg.n_layers, cfg.ffn_mult, cfg.max_L,
                     FE_IO_BF16 if cfg.io_bf16 else FE_IO_F32, cfg.ln_eps, _tasks(cfg), 0 if _cross(cfg) else 1,
-                    _flag(cfg, "elem_self_attn"), _flag(cfg, "encode_pool"))
+                    _flag(cfg, "elem_self_attn"), _flag(cfg, "encode_pool"), _flag(cfg, "linear_context_attn"))
 
 
 def pack_weights(cfg, weights: dict) -> np.ndarray:

@@ -262,6 +262,7 @@ struct fe_ctx {
   int n_tasks = 1;                  // task heads T
   float* head_vec = nullptr;        // b1 [head cols] | w2 [head cols] | b2 [T] | fuse_w [T] | fuse_b [1]
   float* task_scores = nullptr;     // [S, T], every head's score of the last batch
+  float* lin_states = nullptr;      // linear-attention context states [segments][Ly][H][d_h^2 + d_h]
   float *q0 = nullptr, *k0 = nullptr, *v0 = nullptr, *kP = nullptr, *vP = nullptr;
   // workspace
   Shape cap_shape;  // reserved maxima
@@ -365,6 +366,7 @@ bool config_ok(const fe_config* c) {
   if (c->no_cross_seq != 0 && c->no_cross_seq != 1) return false;
   if (c->elem_self_attn != 0 && c->elem_self_attn != 1) return false;
   if (c->encode_pool != 0 && c->encode_pool != 1) return false;
+  if (c->linear_context_attn != 0 && c->linear_context_attn != 1) return false;
   return true;
 }
 
@@ -547,6 +549,8 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
                            s));
   }
   // (a1) context keys/values, once per request
+  const bool lin_fused = c->cfg.linear_context_attn && c->fused_ctxkv &&
+                         fe::ctxkv_state_supported(d, c->dpad, 2 * Ly * d, c->dh, C);
   if (c->fused_ctxkv) {
     CUtensorMap tx{};
     FE_RC(encode_map(&tx, static_cast<const bf16*>(io.ctx), d, B * C, 128));
@@ -559,7 +563,8 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.status = c->status;
     p.C = C;
     p.rep = fact ? K : 1;
-    Prof pf(c, "ctx_ln_kv", s);
+    if (lin_fused) p.states = c->lin_states;  // the context goes straight to its linear-attention states
+    Prof pf(c, lin_fused ? "ctx_ln_state" : "ctx_ln_kv", s);
     FE_CK(fe::ctxkv_launch(&tx, &c->ctxkv_w, &c->KV.sh, c->dpad, p, s));
   } else {
     {
@@ -569,6 +574,14 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     fe::GemmParams p{};
     p.out_f16 = 1;
     FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, &c->KV, nullptr, s));
+  }
+  // (a1') linear attention: the context of every request (sequence, once
+  // factorized) reduced to its per-layer, per-head states (unless the
+  // context kernel already did)
+  if (c->cfg.linear_context_attn && !lin_fused) {
+    Prof pf(c, "lin_state", s);
+    FE_CK(fe::lin_state_launch(c->KV.h, c->fused_ctxkv ? 1 : 0, c->KV.rows, c->KV.ld, fact ? B * K : B, C, d, c->dh,
+                               Ly, c->H, c->lin_states, s));
   }
   // (a2) distinct elements: gather + LN, then the cross-attention stack
   {
@@ -638,7 +651,11 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.ldo = c->a.ld;
     ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
     ap.status = c->status;
-    {
+    if (c->cfg.linear_context_attn) {
+      Prof pf(c, "lin_attn_item_ctx", s);
+      FE_CK(fe::lin_attn_launch(c->q.h, c->q.ld, c->lin_states, fact ? B * K : B, Ly, l, c->H, c->dh,
+                                fact ? nullptr : c->off, fact ? nullptr : c->U, L, L, c->a.h, c->a.l, c->a.ld, s));
+    } else {
       Prof pf(c, "attn_item_ctx", s);
       FE_CK(fe::attn_launch(c->dh, &c->q.ah, &c->KV.kh, &c->KV.kh, ap, s));
     }
@@ -854,6 +871,10 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->out_scores, (size_t)S * sizeof(float)));
   FE_RC(dalloc((void**)&c->out_best, (size_t)B * sizeof(int32_t)));
   FE_RC(dalloc((void**)&c->task_scores, (size_t)S * c->n_tasks * sizeof(float)));
+  if (c->cfg.linear_context_attn) {
+    const long long segs = s.C > 0 ? kv_rows / s.C : 1;  // requests, or sequences once factorized
+    FE_RC(dalloc((void**)&c->lin_states, (size_t)segs * Ly * c->H * (c->dh * c->dh + c->dh) * sizeof(float)));
+  }
   // pipelined host entry: slot 0 uses the staging above, slot 1 its own copy
   c->slots[0].ctx = c->in_ctx;
   c->slots[0].pool = c->in_pool;
@@ -1034,7 +1055,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   };
   int rc = FE_OK;
   if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess ||
-      fe::ffn_prepare() != cudaSuccess || fe::ctxkv_prepare() != cudaSuccess)
+      fe::ffn_prepare() != cudaSuccess || fe::ctxkv_prepare() != cudaSuccess || fe::linattn_prepare() != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "kernel attributes"));
   {
     size_t o = 0;
@@ -1376,6 +1397,11 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
     rows = (size_t)s.B * s.C;
     cols = d;
   } else if (n == "ctx_kv") {
+    if (c->cfg.linear_context_attn && c->fused_ctxkv &&
+        fe::ctxkv_state_supported(d, c->dpad, 2 * c->Ly * d, c->dh, s.C)) {
+      g_msg = "ctx_kv is not materialised: the context kernel reduces it to linear-attention states on chip";
+      return FE_ERR_UNSUPPORTED;
+    }
     pl = &c->KV;
     rows = (size_t)s.B * s.C;
     cols = 2 * c->Ly * d;

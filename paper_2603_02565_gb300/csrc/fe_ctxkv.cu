@@ -20,6 +20,16 @@
 //                   alternating 32-column chunks
 // Each context row is normalised once per column half; the raw rows are
 // bf16, so the second reading costs d * 2 bytes per row.
+//
+// Linear-attention state mode (STATE, two layers, C a multiple of 128): the
+// half of CTA c is layer c % 2, [K_l | V_l].  K/V never leave the chip: the
+// epilogue writes phi(K) (phi(x) = elu(x) + 1) and V of the 128-row tile as
+// MN-major 128-byte-swizzled operand tiles, sums phi(K) over its rows for z
+// (a warp reduce-scatter), and one epilogue thread issues phi(K)^T V
+// (M = N = 128, K = the tile's rows) into TMEM, accumulating over the C / 128
+// row blocks of the segment, which the CTA pair takes in a row; after the
+// last one each head's diagonal d_h x d_h block and z are stored.  The K/V
+// accumulator is single-buffered to leave TMEM for the state.
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -35,19 +45,41 @@ constexpr uint32_t kPlane = BM * BK * 2;                     // 16 KB: 128 rows 
 constexpr uint32_t kStage = 2048;                            // store staging: 32 rows x 32 f16, 64-byte swizzle
 constexpr size_t kSmemMaxBlock = 232448;
 
+constexpr uint32_t kStateTile = 2 * 16384;  // a 128 x 128 f16 MN-major operand: two 64-wide atoms of 128 rows
+
 struct CtxKvLayout {
-  uint32_t w_bytes, a_bytes, raw_bytes;
+  uint32_t w_bytes, a_bytes, raw_bytes, nraw, tail_bytes;
   size_t smem;
 };
 
-__host__ __device__ inline CtxKvLayout ctxkv_layout(int d_pad, int N) {
+// tail: the store staging (plain mode) or the phi(K) and V operand tiles of
+// the state product (state mode, which also keeps a single raw buffer)
+__host__ __device__ inline CtxKvLayout ctxkv_layout(int d_pad, int N, bool state) {
   CtxKvLayout L;
   L.w_bytes = (uint32_t)(d_pad / BK) * (uint32_t)(N / 2) * (BK * 2);  // [kb][N/2 rows x 128 B]
   L.a_bytes = (uint32_t)(d_pad / BK) * 2u * kPlane;                   // [kb][hi, lo]
   L.raw_bytes = (uint32_t)(d_pad / BK) * kPlane;                      // one raw block [kb]
-  L.smem = 1024 + (size_t)L.w_bytes + L.a_bytes + 2 * (size_t)L.raw_bytes + kEpiWarps * 2 * kStage + 256;
+  L.nraw = state ? 1u : 2u;
+  L.tail_bytes = state ? 2u * kStateTile : (uint32_t)kEpiWarps * 2u * kStage;
+  L.smem = 1024 + (size_t)L.w_bytes + L.a_bytes + L.nraw * (size_t)L.raw_bytes + L.tail_bytes + 256;
   return L;
 }
+
+// MN-major shared-memory descriptor, 128-byte swizzle: atoms of 64 elements
+// (M or N) x 8 rows (K); `lbo` = bytes between atoms along M/N, 1024 bytes
+// between 8-row groups along K
+__device__ __forceinline__ uint64_t desc_mn128(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// elu(x) + 1 (the linear-attention feature map)
+__device__ __forceinline__ float phi_elu1(float x) { return x > 0.f ? x + 1.f : __expf(x); }
 
 __device__ __forceinline__ void arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
@@ -57,7 +89,7 @@ __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v 
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 }  // namespace
 
-template <int NKB>
+template <int NKB, bool STATE>
 __global__ void __launch_bounds__(kThreads, 1)
     ctxkv_kernel(const __grid_constant__ CUtensorMap tX, const __grid_constant__ CUtensorMap tW,
                  const __grid_constant__ CUtensorMap tO, const CtxKvParams p) {
@@ -65,12 +97,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t raw_s = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
   const int Nh = p.N / 2, d = p.d;
-  const CtxKvLayout LY = ctxkv_layout(NKB * BK, p.N);
+  const CtxKvLayout LY = ctxkv_layout(NKB * BK, p.N, STATE);
+  constexpr int NRAW = STATE ? 1 : 2;                 // raw context buffers
+  constexpr int NACC = STATE ? 1 : 2;                 // K/V accumulators in TMEM
   uint8_t* sW = smem;                                 // [kb][Nh rows x 128 B]
   uint8_t* sA = sW + LY.w_bytes;                      // [kb][hi, lo]
-  uint8_t* sRaw = sA + LY.a_bytes;                    // [2 buffers][kb]
-  uint8_t* sStg = sRaw + 2 * (size_t)LY.raw_bytes;    // [epilogue warp][2][2 KB]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + kEpiWarps * 2 * kStage);
+  uint8_t* sRaw = sA + LY.a_bytes;                    // [NRAW buffers][kb]
+  uint8_t* sStg = sRaw + NRAW * (size_t)LY.raw_bytes;  // plain: [epilogue warp][2][2 KB]; state: phi(K) tile, V tile
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + LY.tail_bytes);
   uint64_t* w_full = bars;         // resident weight half loaded
   uint64_t* raw_full = bars + 1;   // [2] raw context block staged
   uint64_t* raw_empty = bars + 3;  // [2] the LayerNorm threads are done with it
@@ -78,7 +112,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* a_empty = bars + 6;    // the MMAs of the tile have read the A tile
   uint64_t* acc_full = bars + 7;   // [2] accumulator complete in TMEM
   uint64_t* acc_empty = bars + 9;  // [2] accumulator drained
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
+  uint64_t* st_full = bars + 11;   // state mode: the state product of the tile complete
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -91,24 +126,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(a_full, 32 * kLnWarps);
     mbar_init(a_empty, 1);
+    mbar_init(st_full, 1);
     fence_mbar_init();
     prefetch_tmap(&tX);
     prefetch_tmap(&tW);
     prefetch_tmap(&tO);
   }
-  // TMEM: accumulator i at columns [256 i, 256 i + Nh)
+  // TMEM: K/V accumulator i at columns [256 i, 256 i + Nh); state mode: one
+  // K/V accumulator at [0, Nh), the state product at [256, 384)
   if (warp == 0) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // CTA c: column half c % 2, row blocks c / 2, c / 2 + G, ... with G = gridDim.x / 2
+  // CTA c: column half c % 2, row blocks c / 2, c / 2 + G, ... with G = gridDim.x / 2;
+  // state mode: the row blocks of segments c / 2, c / 2 + G, ..., each segment's
+  // C / 128 blocks in a row, so its state accumulates in TMEM
   const int half = blockIdx.x & 1, G = gridDim.x >> 1;
   const int nblk = (p.rows + BM - 1) / BM;
   const int first = blockIdx.x >> 1;
+  const int Ts = STATE ? p.C / BM : 1;  // row blocks per segment
+  auto tile_at = [&](int i) -> int {    // this CTA's i-th row block, -1 past the last
+    const int seg = first + (i / Ts) * G;
+    const int t = seg * Ts + i % Ts;
+    return t < nblk ? t : -1;
+  };
   const int n_off = half * Nh;  // this CTA's output columns
   // the weight is a parameter: its load may start before the dependency wait
-  if (warp == 0 && lane == 0 && first < nblk) {
+  if (warp == 0 && lane == 0 && tile_at(0) >= 0) {
     mbar_arrive_expect_tx(w_full, LY.w_bytes);
     for (int kb = 0; kb < NKB; ++kb)
       for (int n0 = 0; n0 < Nh; n0 += BM)
@@ -116,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   pdl_trigger();
   pdl_wait();
-  if (first >= nblk) {
+  if (tile_at(0) < 0) {
     if (warp == 0) tmem_dealloc(tmem, 512);
     return;
   }
@@ -125,9 +170,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       // ---------------- TMA: raw context blocks ----------------
       int it = 0;
-      for (int t = first; t < nblk; t += G, ++it) {
-        const int rb = it & 1;
-        if (it >= 2 && !mbar_wait_bounded(raw_empty + rb, ((it >> 1) - 1) & 1, p.status)) break;
+      for (int t = tile_at(it); t >= 0; t = tile_at(++it)) {
+        const int rb = it % NRAW;
+        if (it >= NRAW && !mbar_wait_bounded(raw_empty + rb, ((it / NRAW) - 1) & 1, p.status)) break;
         mbar_arrive_expect_tx(raw_full + rb, LY.raw_bytes);
         // context row of this block (one K/V per candidate sequence: rep > 1)
         const int r0 = t * BM;
@@ -142,9 +187,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t idesc = umma_idesc_bf16(BM, Nh);
       bool ok = mbar_wait_bounded(w_full, 0, p.status);
       int it = 0;
-      for (int t = first; t < nblk && ok; t += G, ++it) {
-        const int ab = it & 1;
-        if (it >= 2 && !mbar_wait_bounded(acc_empty + ab, ((it >> 1) - 1) & 1, p.status)) break;
+      for (int t = tile_at(it); t >= 0 && ok; t = tile_at(++it)) {
+        const int ab = it % NACC;
+        if (it >= NACC && !mbar_wait_bounded(acc_empty + ab, ((it / NACC) - 1) & 1, p.status)) break;
         if (!mbar_wait_bounded(a_full, it & 1, p.status)) break;
         tc_fence_after();
         const uint32_t dst = tmem + (uint32_t)(256 * ab);
@@ -170,9 +215,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = (warp - 2) * 16 + (lane & 15), part = lane >> 4;
     constexpr int kPieces = 4 * NKB;  // 16-byte pieces (8 columns) per thread
     int it = 0;
-    for (int t = first; t < nblk; t += G, ++it) {
-      const int rb = it & 1;
-      if (!mbar_wait_bounded(raw_full + rb, (it >> 1) & 1, p.status)) break;
+    for (int t = tile_at(it); t >= 0; t = tile_at(++it)) {
+      const int rb = it % NRAW;
+      if (!mbar_wait_bounded(raw_full + rb, (it / NRAW) & 1, p.status)) break;
       const uint8_t* raw = sRaw + (size_t)rb * LY.raw_bytes;
       // piece j of this thread: global piece g = part * kPieces + j, column 8 g,
       // 128-byte-swizzled within its 64-column block
@@ -228,6 +273,120 @@ __global__ void __launch_bounds__(kThreads, 1)
       fence_async_shared();
       arrive(a_full);
     }
+  } else if constexpr (STATE) {
+    // ---------------- epilogue, state mode ----------------
+    const int ew = warp - 2 - kLnWarps;  // 0..7
+    const int q = warp & 3;              // TMEM lane quadrant: tile rows 32 q .. 32 q + 31
+    const int sub = ew >> 2;             // alternate 32-column chunks
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const int r = q * 32 + lane;         // this thread's row of the tile
+    const int d = p.d, dh = p.dh, H = p.d / p.dh, l = half;
+    const int SB = dh * dh + dh;
+    uint8_t* sPK = sStg;                 // phi(K)[row][feature]: MN-major, two 64-feature atoms
+    uint8_t* sPV = sStg + kStateTile;    // V[row][feature]
+    auto epi_sync = [&]() { asm volatile("bar.sync 5, 256;" ::: "memory"); };
+    // d = 64: features 64..127 of the phi(K) operand stay zero
+    if (d < 128) {
+      for (int i = (ew * 32 + lane) * 16; i < (int)kStateTile; i += 256 * 16)
+        if ((i / 16384) * 64 >= d) *reinterpret_cast<uint4*>(sPK + i) = make_uint4(0u, 0u, 0u, 0u);
+    }
+    // 16-byte piece of (row, feature m..m+7) in an MN-major tile
+    auto piece = [&](int m) {
+      return (uint32_t)(m >> 6) * 16384u + (uint32_t)r * 128u + ((((uint32_t)(m & 63) >> 3) ^ (uint32_t)(r & 7)) << 4);
+    };
+    const uint32_t idesc = umma_idesc_f16(BM, d) | (1u << 15) | (1u << 16);  // A and B MN-major
+    float zsum[2] = {0.f, 0.f};  // this lane's feature of each K chunk it handles: the segment's sum of phi(K)
+    int it = 0;
+    for (int t = tile_at(it); t >= 0; t = tile_at(++it)) {
+      const int pos = it % Ts;   // row block of the segment
+      if (!mbar_wait_bounded(acc_full, it & 1, p.status)) break;
+      tc_fence_after();
+      int kc = 0;
+      for (int c = 32 * sub; c < 2 * d; c += 64) {
+        float v[32];
+        tmem_ld32(tmem + lane_off + (uint32_t)c, v);
+        const bool isk = c < d;
+        const int m0 = isk ? c : c - d;
+        if (isk) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = phi_elu1(v[i]);
+          // z: this warp's 32 rows summed per feature; lane f ends with feature m0 + f
+          float a[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) a[i] = v[i];
+#pragma unroll
+          for (int o = 16; o >= 1; o >>= 1) {
+            const bool up = (lane & o) != 0;
+#pragma unroll
+            for (int i = 0; i < o; ++i) {
+              const float keep = up ? a[i + o] : a[i];
+              const float send = up ? a[i] : a[i + o];
+              a[i] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, o);
+            }
+          }
+          if (kc == 0) zsum[0] += a[0];
+          else zsum[1] += a[0];
+          ++kc;
+        }
+        // the previous row block's state product must be done reading the operand tiles
+        if (c < 64 && it > 0 && !mbar_wait_bounded(st_full, (it - 1) & 1, p.status)) break;
+        uint8_t* buf = isk ? sPK : sPV;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          *reinterpret_cast<uint4*>(buf + piece(m0 + 8 * j)) =
+              make_uint4(pack_f16x2(v[8 * j], v[8 * j + 1]), pack_f16x2(v[8 * j + 2], v[8 * j + 3]),
+                         pack_f16x2(v[8 * j + 4], v[8 * j + 5]), pack_f16x2(v[8 * j + 6], v[8 * j + 7]));
+      }
+      // the K/V accumulator is read: it may take the next tile
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) arrive(acc_empty);
+      fence_async_shared();  // the operand tiles, visible to the tensor core
+      epi_sync();
+      if (ew == 0 && lane == 0) {
+        tc_fence_after();
+        const uint64_t ad = desc_mn128(smem_u32(sPK), 16384u), bd = desc_mn128(smem_u32(sPV), 16384u);
+#pragma unroll
+        for (int kk = 0; kk < BM / 16; ++kk)
+          umma_bf16(tmem + 256u, desc_adv(ad, (uint32_t)kk * 16u * 128u), desc_adv(bd, (uint32_t)kk * 16u * 128u),
+                    idesc, (kk != 0 || pos != 0) ? 1u : 0u);  // accumulate over the segment's row blocks
+        umma_commit(st_full);
+      }
+      if (pos + 1 < Ts) continue;
+      // the segment's last row block: its state, S of each head from the
+      // diagonal blocks and z, stored (one segment per CTA pair: no atomics)
+      if (!mbar_wait_bounded(st_full, it & 1, p.status)) break;
+      tc_fence_after();
+      const int seg = (t * BM) / p.C;
+      float* st_seg = p.states + ((size_t)seg * 2 + l) * H * SB;
+      const int m = 32 * q + lane;  // this lane's feature of K
+      if (m < d && (sub == 0 || dh == 64)) {
+        const int h = m / dh, i = m % dh, j0 = dh == 64 ? 32 * sub : 0;
+        float sv[32];
+        tmem_ld32(tmem + lane_off + 256u + (uint32_t)(h * dh + j0), sv);
+        float* dst = st_seg + (size_t)h * SB + (size_t)i * dh + j0;
+#pragma unroll
+        for (int jj = 0; jj < 32; jj += 4)
+          *reinterpret_cast<float4*>(dst + jj) = make_float4(sv[jj], sv[jj + 1], sv[jj + 2], sv[jj + 3]);
+      }
+      // z: the four quadrant warps of each K chunk hold partial sums over
+      // their 32 rows; combined through the phi(K) tile, free now that the
+      // segment's last product is complete
+      tc_fence_before();
+      float* zsm = reinterpret_cast<float*>(sPK);  // [quadrant][128 features]
+      int kk2 = 0;
+      for (int c = 32 * sub; c < d; c += 64, ++kk2) zsm[q * 128 + c + lane] = kk2 == 0 ? zsum[0] : zsum[1];
+      epi_sync();
+      if (q == 0) {
+        for (int c = 32 * sub; c < d; c += 64) {
+          const int mz = c + lane;
+          st_seg[(size_t)(mz / dh) * SB + dh * dh + (mz % dh)] =
+              (zsm[mz] + zsm[128 + mz]) + (zsm[256 + mz] + zsm[384 + mz]);
+        }
+      }
+      zsum[0] = zsum[1] = 0.f;
+      epi_sync();  // the state accumulator is read before the next segment's first product
+    }
   } else {
     // ---------------- epilogue: TMEM -> f16 -> TMA stores ----------------
     const int ew = warp - 2 - kLnWarps;  // 0..7
@@ -237,7 +396,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* stg0 = sStg + (size_t)ew * 2 * kStage;
     int nstore = 0;
     int it = 0;
-    for (int t = first; t < nblk; t += G, ++it) {
+    for (int t = tile_at(it); t >= 0; t = tile_at(++it)) {
       const int ab = it & 1;
       if (!mbar_wait_bounded(acc_full + ab, (it >> 1) & 1, p.status)) break;
       tc_fence_after();
@@ -284,7 +443,15 @@ int g_ctxkv_sms = 0;
 bool ctxkv_supported(int d, int d_pad, int N, int nb, int io_f32) {
   if (io_f32 || nb != 1 || d > 128 || d % 32 || (d_pad != 64 && d_pad != 128)) return false;
   if (N % 256 || N > 512) return false;  // halves of 128 or 256 columns
-  return ctxkv_layout(d_pad, N).smem <= kSmemMaxBlock;
+  return ctxkv_layout(d_pad, N, false).smem <= kSmemMaxBlock;
+}
+
+bool ctxkv_state_supported(int d, int d_pad, int N, int dh, int C) {
+  if (d != 64 && d != 128) return false;
+  if (N != 4 * d) return false;  // two layers: each column half is one layer's [K | V]
+  if (dh != 32 && dh != 64) return false;
+  if (C <= 0 || C % BM) return false;  // a 128-row tile lies in one segment
+  return ctxkv_layout(d_pad, N, true).smem <= kSmemMaxBlock;
 }
 
 cudaError_t ctxkv_prepare() {
@@ -292,24 +459,32 @@ cudaError_t ctxkv_prepare() {
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_ctxkv_sms, cudaDevAttrMultiProcessorCount, dev);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(ctxkv_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+    e = cudaFuncSetAttribute(ctxkv_kernel<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(ctxkv_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+    e = cudaFuncSetAttribute(ctxkv_kernel<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(ctxkv_kernel<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(ctxkv_kernel<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemMaxBlock);
   return e;
 }
 
 cudaError_t ctxkv_launch(const CUtensorMap* x, const CUtensorMap* w, const CUtensorMap* o, int d_pad,
                          const CtxKvParams& p, cudaStream_t s) {
   if (p.rows <= 0) return cudaSuccess;
-  const CtxKvLayout LY = ctxkv_layout(d_pad, p.N);
+  const bool state = p.states != nullptr;
+  const CtxKvLayout LY = ctxkv_layout(d_pad, p.N, state);
   const long long nblk = (p.rows + BM - 1) / BM;
   // an even grid: CTA pairs (2i, 2i+1) take the two column halves of the same row blocks
   long long grid = g_ctxkv_sms > 0 ? g_ctxkv_sms : 148;
   if (grid > 2 * nblk) grid = 2 * nblk;
   grid &= ~1LL;
-  if (d_pad > BK)
-    return launch_k(ctxkv_kernel<2>, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *x, *w, *o, p);
-  return launch_k(ctxkv_kernel<1>, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *x, *w, *o, p);
+  const dim3 g((unsigned)grid), b(kThreads);
+  if (state)
+    return d_pad > BK ? launch_k(ctxkv_kernel<2, true>, g, b, LY.smem, s, *x, *w, *o, p)
+                      : launch_k(ctxkv_kernel<1, true>, g, b, LY.smem, s, *x, *w, *o, p);
+  return d_pad > BK ? launch_k(ctxkv_kernel<2, false>, g, b, LY.smem, s, *x, *w, *o, p)
+                    : launch_k(ctxkv_kernel<1, false>, g, b, LY.smem, s, *x, *w, *o, p);
 }
 
 }  // namespace fe

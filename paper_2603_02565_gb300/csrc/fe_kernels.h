@@ -131,8 +131,14 @@ struct CtxKvParams {
   // output row r reads context row ((r / C) / rep) * C + r % C: rep = 1 for one
   // K/V per request, rep = K for one per candidate sequence (C % 128 == 0)
   int C, rep;
+  // linear-attention state mode (non-null): no K/V is written; the states
+  // [segment = row / C][layer][head][dh*dh + dh] receive phi(K)^T V and
+  // sum phi(K) (feature map elu + 1) over the segment's rows
+  float* states;
 };
 bool ctxkv_supported(int d, int d_pad, int N, int nb, int io_f32);
+// whether the state mode applies: two layers (N = 4d), d in {64, 128}, dh in {32, 64}, C % 128 == 0
+bool ctxkv_state_supported(int d, int d_pad, int N, int dh, int C);
 cudaError_t ctxkv_prepare();
 cudaError_t ctxkv_launch(const CUtensorMap* x, const CUtensorMap* w, const CUtensorMap* o, int d_pad,
                          const CtxKvParams& p, cudaStream_t s);
@@ -169,6 +175,23 @@ struct AttnParams {
 cudaError_t attn_prepare();
 cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, const CUtensorMap* v, const AttnParams& p,
                         cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// Linear-attention context module (fe_linattn.cu): feature map elu(x) + 1.
+// lin_state: for segment s (context rows [s*C, s*C + C)), layer l, head h:
+//   states[((s * Ly + l) * H + h) * SB ...] = S [dh][dh] (row-major) | z [dh],
+//   SB = dh*dh + dh, S = sum_c phi(K_l[c,h]) V_l[c,h]^T, z = sum_c phi(K_l[c,h]);
+//   kv holds K_l | V_l column blocks (f16), head-major (hm: [col/dh][rows_alloc][dh])
+//   or row-major [rows][ld].
+// lin_attn: element rows [off(s), off(s) + cnt(s)) of segment s read layer l:
+//   out[row, h*dh + j] = (phi(q_h) S)_j / (phi(q_h) . z), written as a bf16 hi/lo pair.
+// ---------------------------------------------------------------------------
+cudaError_t linattn_prepare();
+cudaError_t lin_state_launch(const bf16* kv, int hm, int rows_alloc, int ld, int n_seg, int C, int d, int dh, int Ly,
+                             int H, float* states, cudaStream_t s);
+cudaError_t lin_attn_launch(const bf16* q, int ldq, const float* states, int n_seg, int Ly, int l, int H, int dh,
+                            const int* off_dev, const int* cnt_dev, int stride, int cnt_fixed, bf16* o_h, bf16* o_l,
+                            int ldo, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // element-wise / gather / selection kernels (fe_misc.cu)

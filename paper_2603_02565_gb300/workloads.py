@@ -37,6 +37,7 @@ class ModelConfig:
     cross_seq: bool = True  # False: the variant without cross-sequence interaction
     elem_self_attn: bool = False  # self-attention H^(1) over the element set
     encode_pool: bool = False     # the element set is the whole pool (U = M)
+    linear_context_attn: bool = False  # linear attention in the element -> context attention
 
     @property
     def F(self) -> int:
@@ -143,10 +144,10 @@ def _normal(rng, shape, std, bf16):
 
 def _rec_workload(name, seed, B, C, d, H, Ly, M, K, L, zipf_s, ctx_std, pool_std,
                   io_bf16=True, idx_seed=None, max_L=None, n_tasks=1, cross_seq=True,
-                  elem_self_attn=False, encode_pool=False):
+                  elem_self_attn=False, encode_pool=False, linear_context_attn=False):
     cfg = ModelConfig(d=d, n_heads=H, n_layers=Ly, max_L=max_L or L, io_bf16=io_bf16,
                       n_tasks=n_tasks, cross_seq=cross_seq, elem_self_attn=elem_self_attn,
-                      encode_pool=encode_pool)
+                      encode_pool=encode_pool, linear_context_attn=linear_context_attn)
     rng = np.random.default_rng(seed)
     weights = make_weights(cfg, rng)
     context = _normal(rng, (B, C, d), ctx_std, io_bf16)
