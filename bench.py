@@ -110,13 +110,14 @@ def site_work(site, cfg, B, C, M, K, L, R):
         "gemm_item_o_ln": (2 * R * d * d, R * d * (A + 8 + A)),
         "gemm_item_ffn1": (2 * R * d * F, R * d * A + R * F * A),
         "gemm_item_ffn2_ln": (2 * R * F * d, R * F * A + R * d * (8 + A)),
-        "ffn_item": (4 * R * d * F, R * d * (A + 8 + A)),
+        # attention output projection + FFN: A in, x0 in, x out, LN(x_out) out
+        "ffn_item": (2 * R * d * d + 4 * R * d * F, R * d * (A + 8 + A)),
         "gemm_item_seq_kv": (4 * R * d * d, R * d * A + 2 * R * d * A),
         "seq_cls_attn": (4 * S * (L + 1) * d, 2 * R * d * A + 4 * S * L + S * d * A),
         "gemm_seq_o_ln": (2 * S * d * d, S * d * (A + 4 + A)),
         "gemm_seq_ffn1": (2 * S * d * F, S * d * A + S * F * A),
         "gemm_seq_ffn2_ln": (2 * S * F * d, S * F * A + S * d * (8 + A)),
-        "ffn_seq": (4 * S * d * F, S * d * (A + 8 + A)),
+        "ffn_seq": (2 * S * d * d + 4 * S * d * F, S * d * (A + 4 + A)),  # x0: the [CLS] row
         "gemm_cross_qkv": (6 * S * d * d, S * d * A + 3 * S * d * H),
         "attn_cross_seq": (4 * B * K * K * d, 3 * S * d * H + S * d * A),
         "gemm_cross_o_ln": (2 * S * d * d, S * d * (A + 8 + A)),

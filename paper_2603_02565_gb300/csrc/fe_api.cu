@@ -491,8 +491,10 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   return FE_OK;
 }
 
-int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& W1, const Weight& W2, const float* b1,
-        const float* b2, const F32Rows& x, const Planes& ln_out, int rows, const int* rows_dev, cudaStream_t s) {
+// x = x0 + A W_O, then the FFN: x written to x (in place over x0 when x0_row is null), LN(x_out) to ln_out
+int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const Weight& W1, const Weight& W2,
+        const float* b1, const float* b2, const float* x0_row, const F32Rows& x, const Planes& ln_out, int rows,
+        const int* rows_dev, cudaStream_t s) {
   if (rows <= 0) return FE_OK;
   Prof pf(c, site, s);
   fe::FfnParams p{};
@@ -504,11 +506,13 @@ int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& W1, const We
   p.nb = c->nb;
   p.b1 = b1;
   p.b2 = b2;
-  p.resid = x.p;
-  p.ldr = x.ld;
+  p.x0 = x0_row ? nullptr : x.p;
+  p.ldx0 = x.ld;
+  p.x0_row = x0_row;
   p.eps = c->cfg.ln_eps;
   p.status = c->status;
-  FE_CK(fe::ffn_launch(&A.th, &A.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.sh, &ln_out.sl, &x.sx, p, s));
+  FE_CK(fe::ffn_launch(&A.th, &A.tl, &WO.p.th, &WO.p.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.sh, &ln_out.sl,
+                       &x.sx, p, s));
   return FE_OK;
 }
 
@@ -660,14 +664,15 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
       FE_CK(fe::attn_launch(c->dh, &c->q.ah, &c->KV.kh, &c->KV.kh, ap, s));
     }
 
-    fe::GemmParams po{};
-    po.resid = c->h.p;
-    po.ldr = d;
-    FE_RC(gemm(c, "gemm_item_o_ln", fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, &c->xln, &c->h, s));
-
     if (c->fused_ffn) {
-      FE_RC(ffn(c, "ffn_item", c->xln, c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), c->h, c->xln, R, sumU, s));
+      FE_RC(ffn(c, "ffn_item", c->a, c->wo[l], c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), nullptr, c->h,
+                c->xln, R, sumU, s));
     } else {
+      fe::GemmParams po{};
+      po.resid = c->h.p;
+      po.ldr = d;
+      FE_RC(gemm(c, "gemm_item_o_ln", fe::EPI_RESID_LN, c->a, c->wo[l], R, sumU, po, &c->xln, &c->h, s));
+
       fe::GemmParams p1{};
       p1.bias = lw(c, l, T_B1);
       p1.relu = 1;
@@ -711,15 +716,16 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     Prof pf(c, "seq_cls_attn", s);
     FE_CK(fe::cls_attn_launch(cp, s));
   }
-  {
-    fe::GemmParams p{};
-    p.resid = tw(c, T_CLS);
-    p.ldr = 0;
-    FE_RC(gemm(c, "gemm_seq_o_ln", fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, &c->cln, &c->c, s));
-  }
   if (c->fused_ffn) {
-    FE_RC(ffn(c, "ffn_seq", c->cln, c->w1s, c->w2s, tw(c, T_B1S), tw(c, T_B2S), c->c, c->z, S, nullptr, s));
+    FE_RC(ffn(c, "ffn_seq", c->o, c->os, c->w1s, c->w2s, tw(c, T_B1S), tw(c, T_B2S), tw(c, T_CLS), c->c, c->z, S,
+              nullptr, s));
   } else {
+    {
+      fe::GemmParams p{};
+      p.resid = tw(c, T_CLS);
+      p.ldr = 0;
+      FE_RC(gemm(c, "gemm_seq_o_ln", fe::EPI_RESID_LN, c->o, c->os, S, nullptr, p, &c->cln, &c->c, s));
+    }
     {
       fe::GemmParams p{};
       p.bias = tw(c, T_B1S);

@@ -1,26 +1,32 @@
-// Fused position-wise FFN block of the evaluator (element layers of Section
-// 4.2 and the SeqEnc block of Section 4.3):
-//     x_out = x + ReLU(LN(x) W1 + b1) W2 + b2,   also LN(x_out)
-// for rows of width d <= 128, without writing the F-wide intermediate to
-// memory.  A persistent CTA walks 128-row tiles, F in chunks of 128 columns:
-//   warp 0 lane 0 : TMA producer -- the LN(x) tile (hi/lo, held while FFN1
-//                   runs), a ring of weight slots in consumption order
-//                   W1_0, W1_1, W1_2, W2_0, W1_3, W2_1, ..., and, once every
-//                   FFN1 of the tile has completed, the fp32 residual tile x
-//                   into the space the LN(x) tile held
-//   warp 1 lane 0 : tcgen05.mma -- FFN1 chunk f (N = 128) into one of three
+// Attention output projection and position-wise FFN of one block of the
+// evaluator (element layers of Section 4.2, the SeqEnc block of Section 4.3),
+// in one kernel:
+//     x = x0 + A W_O,   x_out = x + ReLU(LN(x) W1 + b1) W2 + b2,   also LN(x_out)
+// (A the attention output, x0 the block's input rows, or one row broadcast
+// to every row) for rows of width d <= 128, without writing x, LN(x) or the
+// F-wide intermediate to memory.  A persistent CTA walks 128-row tiles, F in
+// chunks of 128 columns:
+//   warp 0 lane 0 : TMA producer -- the A tile (hi/lo) and a ring of weight
+//                   slots in consumption order W_O, W1_0, W1_1, W1_2, W2_0,
+//                   W1_3, W2_1, ...
+//   warp 1 lane 0 : tcgen05.mma -- A W_O into the d-column accumulator that
+//                   FFN2 uses; after the epilogue has put x there and LN(x)
+//                   in shared memory, FFN1 chunk f (N = 128) into one of three
 //                   TMEM buffers, two chunks ahead of FFN2 of chunk f-2, which
 //                   reads its A operand from that TMEM buffer and accumulates
-//                   every chunk into a d-column TMEM accumulator
-//   warps 2-9     : per chunk: bias + ReLU, split into hi/lo bf16 and written
-//                   back over the chunk's fp32 columns in TMEM; per tile:
-//                   residual + b2 + LayerNorm, stored with TMA tensor stores
-//                   staged in the residual tile's own 4 KB blocks
+//                   on top of x
+//   warps 2-9     : per tile: x0 rows read into registers while the A tile
+//                   arrives, x = x0 + A W_O written back into the
+//                   accumulator, LN(x) written over the A tile as FFN1's
+//                   operand; per chunk:
+//                   bias + ReLU, split into hi/lo bf16 and written back over
+//                   the chunk's fp32 columns in TMEM; per tile: x_out =
+//                   accumulator + b2, LayerNorm, stored with TMA tensor stores
+//                   staged in the tile's own 4 KB blocks
 // The MMA groups are 16 instructions of N >= 128 so that the tensor pipe has
-// queued work while the issuing thread polls its barriers; the residual
-// arrives by TMA rather than by register loads (global loads in flight hold up
-// the shared-memory and mbarrier operations of the other warps); the biases
-// sit in shared memory.
+// queued work while the issuing thread polls its barriers; x0 is read by the
+// epilogue warps before the projection completes, when they have nothing else
+// in flight; the biases sit in shared memory.
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -38,11 +44,11 @@ constexpr uint32_t kAPlane = BM * BK * 2;      // 16 KB: 128 rows x 64 bf16
 constexpr uint32_t kResBlock = 4096;           // residual block: 32 rows x 32 fp32, 128-byte swizzle
 constexpr size_t kSmemMaxBlock = 232448;
 constexpr int kMaxRing = 8;                    // weight slots
-constexpr uint32_t kBarBytes = 512;
+constexpr uint32_t kBarBytes = 512;  // 64 barriers
 constexpr uint32_t kRedBytes = 2 * 2 * 128 * 4;  // [sum|var][half][row]
 
 struct FfnLayout {
-  uint32_t a_bytes, slot_bytes, w1_chunk, w2_chunk, bias_bytes;
+  uint32_t a_bytes, slot_bytes, w1_chunk, w2_chunk, wo_bytes, bias_bytes;
   int ring;
   size_t smem;
 };
@@ -52,9 +58,10 @@ __host__ __device__ inline FfnLayout ffn_layout(int d, int d_pad, int F, int nb)
   L.a_bytes = (uint32_t)(d_pad / BK) * 2u * kAPlane;
   L.w1_chunk = (uint32_t)nb * (uint32_t)(d_pad / BK) * (FC * BK * 2);  // [kb][plane][128 rows x 64]
   L.w2_chunk = (uint32_t)nb * 2u * (uint32_t)d * (BK * 2);             // [plane][half][d rows x 64]
+  L.wo_bytes = (uint32_t)nb * (uint32_t)(d_pad / BK) * (uint32_t)d * (BK * 2);  // [kb][plane][d rows x 64]
   L.slot_bytes = L.w1_chunk > L.w2_chunk ? L.w1_chunk : L.w2_chunk;
   L.slot_bytes = (L.slot_bytes + 1023u) & ~1023u;
-  L.bias_bytes = ((uint32_t)(F + d) * 4u + 127u) & ~127u;
+  L.bias_bytes = ((uint32_t)(F + 2 * d) * 4u + 127u) & ~127u;  // b1, b2, the broadcast x0 row
   const size_t fixed = 1024 + L.a_bytes + L.bias_bytes + kBarBytes + kRedBytes;
   L.ring = fixed < kSmemMaxBlock ? (int)((kSmemMaxBlock - fixed) / L.slot_bytes) : 0;
   if (L.ring > kMaxRing) L.ring = kMaxRing;
@@ -72,6 +79,7 @@ __device__ __forceinline__ void mbar_arrive_one(uint64_t* bar) {
 template <int NKB, int NB>
 __global__ void __launch_bounds__(kThreads, 1)
     ffn_kernel(const __grid_constant__ CUtensorMap tA_h, const __grid_constant__ CUtensorMap tA_l,
+               const __grid_constant__ CUtensorMap tWo_h, const __grid_constant__ CUtensorMap tWo_l,
                const __grid_constant__ CUtensorMap tW1_h, const __grid_constant__ CUtensorMap tW1_l,
                const __grid_constant__ CUtensorMap tW2_h, const __grid_constant__ CUtensorMap tW2_l,
                const __grid_constant__ CUtensorMap tO_h, const __grid_constant__ CUtensorMap tO_l,
@@ -83,13 +91,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int d = p.d, F = p.F;
   const FfnLayout LY = ffn_layout(d, NKB * BK, F, nb);
   const int nf = F / FC;
-  uint8_t* sA = smem;  // LN(x) tile [kb][plane]; later the residual tile [32-column chunk][row quadrant][4 KB]
+  // the A tile [kb][plane], then LN(x) [kb][plane] in the same layout, then the
+  // output staging blocks [32-column chunk][row quadrant][4 KB]
+  uint8_t* sA = smem;
   uint8_t* sW = sA + LY.a_bytes;
   float* sB1 = reinterpret_cast<float*>(sW + (size_t)LY.ring * LY.slot_bytes);
   float* sB2 = sB1 + F;
+  float* sX0 = sB2 + d;  // the broadcast row x0, when there is one
   uint64_t* bars = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(sB1) + LY.bias_bytes);
-  uint64_t* a_full = bars;           // LN(x) tile loaded
-  uint64_t* a_empty = bars + 1;      // every FFN1 of the tile complete
+  uint64_t* a_full = bars;           // A tile loaded
+  uint64_t* o_done = bars + 1;       // A W_O complete in the accumulator (the A tile is read)
   uint64_t* w_full = bars + 2;       // [kMaxRing]
   uint64_t* w_empty = bars + 10;     // [kMaxRing]
   uint64_t* acc1_full = bars + 18;   // [NA1] FFN1 chunk complete in TMEM buffer
@@ -97,15 +108,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* mid_full = bars + 24;    // [NA1] hidden activation written over the buffer
   uint64_t* acc2_full = bars + 27;
   uint64_t* acc2_empty = bars + 28;
-  uint64_t* r_full = bars + 29;      // residual tile loaded
-  uint64_t* r_empty = bars + 30;     // residual blocks free again (their last store has read them)
+  uint64_t* ln_full = bars + 29;     // x back in the accumulator, LN(x) in sA
+  uint64_t* r_empty = bars + 30;     // staging blocks free again (their last store has read them)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 31);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + kBarBytes);  // [sum|var][half][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     mbar_init(a_full, 1);
-    mbar_init(a_empty, 1);
+    mbar_init(o_done, 1);
     for (int i = 0; i < kMaxRing; ++i) {
       mbar_init(w_full + i, 1);
       mbar_init(w_empty + i, 1);
@@ -117,23 +128,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(acc2_full, 1);
     mbar_init(acc2_empty, kEpiWarps);
-    mbar_init(r_full, 1);
+    mbar_init(ln_full, 32 * kEpiWarps);
     mbar_init(r_empty, kEpiWarps);
     fence_mbar_init();
     prefetch_tmap(&tA_h);
+    prefetch_tmap(&tWo_h);
     prefetch_tmap(&tW1_h);
     prefetch_tmap(&tW2_h);
-    prefetch_tmap(&tO_x);
   }
-  // biases are parameters, not outputs of an earlier kernel: read before the dependency wait
+  // biases and the broadcast row are parameters, not outputs of an earlier
+  // kernel: read before the dependency wait
   for (int i = threadIdx.x; i < F; i += kThreads) sB1[i] = p.b1[i];
-  for (int i = threadIdx.x; i < d; i += kThreads) sB2[i] = p.b2[i];
-  // TMEM: FFN1 chunk buffers at columns [128 i, 128 i + 128), i < 3; FFN2 accumulator at [384, 384 + d)
+  for (int i = threadIdx.x; i < d; i += kThreads) {
+    sB2[i] = p.b2[i];
+    sX0[i] = p.x0_row ? p.x0_row[i] : 0.f;
+  }
+  // TMEM: FFN1 chunk buffers at columns [128 i, 128 i + 128), i < 3; the
+  // d-column accumulator of A W_O, x and FFN2 at [384, 384 + d)
   if (warp == 0) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  const uint32_t acc2 = tmem + (uint32_t)(NA1 * FC);
   pdl_trigger();
   pdl_wait();
   int rows_valid = p.rows;
@@ -149,17 +166,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---------------- TMA producer ----------------
       int tl = 0, ws = 0;
       bool ok = true;
-      auto load_slot = [&](bool first, int f) -> bool {
+      // kind 0: W_O; 1: W1 rows [f*128, f*128+128); 2: W2 columns [f*128, f*128+128)
+      auto load_slot = [&](int kind, int f) -> bool {
         const int slot = ws % LY.ring;
         if (ws >= LY.ring && !mbar_wait_bounded(w_empty + slot, ((ws / LY.ring) - 1) & 1, p.status)) return false;
         uint8_t* dst = sW + (size_t)slot * LY.slot_bytes;
-        if (first) {  // W1 rows [f*128, f*128+128), every k block
+        if (kind == 0) {  // every d row, every k block: [kb][plane][d rows x 64]
+          mbar_arrive_expect_tx(w_full + slot, LY.wo_bytes);
+          for (int kb = 0; kb < nkb; ++kb)
+            for (int q = 0; q < nb; ++q)
+              tma_load_2d(dst + (size_t)(kb * nb + q) * d * (BK * 2), q ? &tWo_l : &tWo_h, kb * BK, 0, w_full + slot);
+        } else if (kind == 1) {  // every k block: [kb][plane][128 rows x 64]
           mbar_arrive_expect_tx(w_full + slot, LY.w1_chunk);
           for (int kb = 0; kb < nkb; ++kb)
             for (int q = 0; q < nb; ++q)
               tma_load_2d(dst + (size_t)(kb * nb + q) * (FC * BK * 2), q ? &tW1_l : &tW1_h, kb * BK, f * FC,
                           w_full + slot);
-        } else {  // W2 columns [f*128, f*128+128) as two 64-column halves, every d row
+        } else {  // two 64-column halves, every d row: [plane][half][d rows x 64]
           mbar_arrive_expect_tx(w_full + slot, LY.w2_chunk);
           for (int q = 0; q < nb; ++q)
             for (int hh = 0; hh < 2; ++hh)
@@ -170,25 +193,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         return true;
       };
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
-        // sA holds the previous tile's residual until that tile's stores have read it
+        // sA holds the previous tile's output staging until its stores have read it
         if (tl > 0 && !mbar_wait_bounded(r_empty, (tl - 1) & 1, p.status)) break;
         mbar_arrive_expect_tx(a_full, LY.a_bytes);
         for (int kb = 0; kb < nkb; ++kb) {
           tma_load_2d(sA + (size_t)(kb * 2) * kAPlane, &tA_h, kb * BK, t * BM, a_full);
           tma_load_2d(sA + (size_t)(kb * 2 + 1) * kAPlane, &tA_l, kb * BK, t * BM, a_full);
         }
+        if (!load_slot(0, 0)) break;
         for (int s = 0; s < nf + LA && ok; ++s) {
-          if (s < nf && !load_slot(true, s)) ok = false;
-          if (ok && s >= LA && !load_slot(false, s - LA)) ok = false;
+          if (s < nf && !load_slot(1, s)) ok = false;
+          if (ok && s >= LA && !load_slot(2, s - LA)) ok = false;
         }
-        if (!ok) break;
-        // residual x rows of the tile in 32 x 32 fp32 blocks, into sA once the
-        // last FFN1 has read it (rows past the tensor extent arrive as zeros)
-        if (!mbar_wait_bounded(a_empty, tl & 1, p.status)) break;
-        mbar_arrive_expect_tx(r_full, (uint32_t)(d / 32) * 4 * kResBlock);
-        for (int c = 0; c < d / 32; ++c)
-          for (int q = 0; q < 4; ++q)
-            tma_load_2d(sA + (size_t)(c * 4 + q) * kResBlock, &tO_x, 32 * c, t * BM + 32 * q, r_full);
       }
     }
   } else if (warp == 1) {
@@ -196,11 +212,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---------------- MMA issuer ----------------
       const uint32_t idesc1 = umma_idesc_bf16(BM, FC);
       const uint32_t idesc2 = umma_idesc_bf16(BM, d);
-      const uint32_t acc2 = tmem + (uint32_t)(NA1 * FC);
       int tl = 0, ws = 0, gf = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+        // ---- A W_O into the accumulator, once the previous tile's epilogue has read it
         if (!mbar_wait_bounded(a_full, tl & 1, p.status)) break;
+        {
+          const int slot = ws % LY.ring;
+          if (!mbar_wait_bounded(w_full + slot, (ws / LY.ring) & 1, p.status)) break;
+          if (tl > 0 && !mbar_wait_bounded(acc2_empty, (tl - 1) & 1, p.status)) break;
+          tc_fence_after();
+          const uint64_t a0 = umma_desc_sw128(smem_u32(sA));
+          const uint64_t w0 = umma_desc_sw128(smem_u32(sW + (size_t)slot * LY.slot_bytes));
+#pragma unroll
+          for (int kb = 0; kb < nkb; ++kb) {
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+              const uint64_t ah = desc_adv(a0, (uint32_t)(kb * 2) * kAPlane + kk * 32);
+              const uint64_t wh = desc_adv(w0, (uint32_t)(kb * nb) * (uint32_t)d * (BK * 2) + kk * 32);
+              umma_bf16(acc2, ah, wh, idesc2, (kb | kk) != 0 ? 1u : 0u);
+              umma_bf16(acc2, desc_adv(ah, kAPlane), wh, idesc2, 1u);
+              if (nb > 1) umma_bf16(acc2, ah, desc_adv(wh, (uint32_t)d * (BK * 2)), idesc2, 1u);
+            }
+          }
+          umma_commit(w_empty + slot);
+          umma_commit(o_done);
+          ++ws;
+        }
+        // ---- FFN1 / FFN2 once the epilogue has put x in the accumulator and LN(x) in sA
+        if (!mbar_wait_bounded(ln_full, tl & 1, p.status)) break;
         tc_fence_after();
         const int gf0 = gf;
         for (int s = 0; s < nf + LA && ok; ++s) {
@@ -234,15 +274,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_commit(w_empty + slot);
             umma_commit(acc1_full + b);
             ++ws;
-            if (s == nf - 1) umma_commit(a_empty);  // every FFN1 of this tile issued
           }
           if (s >= LA) {
             // FFN2 chunk c = s - LA: acc2 += mid(c) . W2 chunk c, mid(c) from TMEM buffer g % NA1
             const int c = s - LA, g = gf0 + c, b = g % NA1;
-            if (c == 0 && tl > 0 && !mbar_wait_bounded(acc2_empty, (tl - 1) & 1, p.status)) {
-              ok = false;
-              break;
-            }
             if (!mbar_wait_bounded(mid_full + b, (g / NA1) & 1, p.status)) {
               ok = false;
               break;
@@ -263,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const int hh = kk >> 2, k4 = kk & 3;
               const uint32_t mh = mt + (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1)), ml = mh + 16;
               const uint64_t wh = desc_adv(w0, (uint32_t)hh * (uint32_t)d * (BK * 2) + k4 * 32);
-              umma_bf16_tmem_a(acc2, mh, wh, idesc2, (c > 0 || kk > 0) ? 1u : 0u);
+              umma_bf16_tmem_a(acc2, mh, wh, idesc2, 1u);
               umma_bf16_tmem_a(acc2, ml, wh, idesc2, 1u);
               if (nb > 1) umma_bf16_tmem_a(acc2, mh, desc_adv(wh, 2u * (uint32_t)d * (BK * 2)), idesc2, 1u);
             }
@@ -306,6 +341,97 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int m0 = t * BM;
       const int srow = m0 + q * 32;
       const bool valid = m0 + r < rows_valid;
+      // ---- x = x0 + A W_O for this thread's row, columns 32 half + 64 ci + [0, 32)
+      // (x0 of rows past the valid count is 0); x goes back into the
+      // accumulator for FFN2 to add to, LN(x) into sA (which the projection
+      // has read) as FFN1's A tile.  The first 32 columns of x0 are read
+      // while the projection completes.
+      auto load_x0 = [&](int c, float* x) {
+        const float* src = p.x0_row ? nullptr : p.x0 + (size_t)(m0 + r) * p.ldx0 + c;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (p.x0_row)
+            v = *reinterpret_cast<const float4*>(sX0 + c + 4 * j);
+          else if (valid)
+            v = *reinterpret_cast<const float4*>(src + 4 * j);
+          x[4 * j] = v.x;
+          x[4 * j + 1] = v.y;
+          x[4 * j + 2] = v.z;
+          x[4 * j + 3] = v.w;
+        }
+      };
+      float xr[32];
+      load_x0(32 * half < d ? 32 * half : 0, xr);  // (unused when 32 half >= d)
+      if (!mbar_wait_bounded(o_done, tl & 1, p.status)) break;
+      tc_fence_after();
+      float sum = 0.f;
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        if (c < d) {
+          if (ci > 0) load_x0(c, xr);
+          float v[32];
+          tmem_ld32(acc2 + lane_off + (uint32_t)c, v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            v[j] += xr[j];
+            sum += v[j];
+          }
+          tmem_st32(acc2 + lane_off + (uint32_t)c, v);
+        }
+      }
+      red_sum[half * 128 + r] = sum;
+      pair_sync();
+      const float mean0 = (red_sum[r] + red_sum[128 + r]) / (float)d;
+      // x is read back from the accumulator rather than kept in registers
+      float var0 = 0.f;
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        if (c < d) {
+          float v[32];
+          tmem_ld32(acc2 + lane_off + (uint32_t)c, v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const float dv = v[j] - mean0;
+            var0 = fmaf(dv, dv, var0);
+          }
+        }
+      }
+      red_var[half * 128 + r] = var0;
+      pair_sync();
+      const float rstd0 = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)d + p.eps);
+      // row r of planes (kb, hi) and (kb, lo), 128-byte swizzle: this warp's
+      // four 16-byte pieces 4 half + jj; columns past d are zeros
+#pragma unroll
+      for (int ci = 0; ci < nkb; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        uint32_t hi[16], lo[16];
+        if (c < d) {
+          float v[32];
+          tmem_ld32(acc2 + lane_off + (uint32_t)c, v);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) split2((v[2 * j] - mean0) * rstd0, (v[2 * j + 1] - mean0) * rstd0, hi[j], lo[j]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            hi[j] = 0u;
+            lo[j] = 0u;
+          }
+        }
+        uint8_t* rowp = sA + (size_t)(ci * 2) * kAPlane + (size_t)r * 128u;
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+          const uint32_t o = (uint32_t)((4 * half + jj) ^ (r & 7)) << 4;
+          *reinterpret_cast<uint4*>(rowp + o) = make_uint4(hi[4 * jj], hi[4 * jj + 1], hi[4 * jj + 2], hi[4 * jj + 3]);
+          *reinterpret_cast<uint4*>(rowp + kAPlane + o) =
+              make_uint4(lo[4 * jj], lo[4 * jj + 1], lo[4 * jj + 2], lo[4 * jj + 3]);
+        }
+      }
+      fence_async_shared();
+      tc_fence_before();
+      mbar_arrive_one(ln_full);
       // ---- per chunk: mid = split(ReLU(acc1 + b1)) written back over this
       // warp's 64 columns of the chunk's TMEM buffer as FFN2's A operand
       for (int f = 0; f < nf; ++f, ++gf) {
@@ -337,34 +463,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive_one(mid_full + ba);
       }
       if (!ok) break;
-      // ---- final: x = resid + acc2 + b2, LayerNorm, stores
+      // ---- final: x_out = acc2 + b2 (acc2 = x + FFN2), LayerNorm, stores
       if (!mbar_wait_bounded(acc2_full, tl & 1, p.status)) break;
-      if (!mbar_wait_bounded(r_full, tl & 1, p.status)) break;
       tc_fence_after();
-      // this warp's residual blocks: column chunks half and half + 2 of row quadrant q
+      // this warp's staging blocks (every FFN1 has read the LN(x) tile they
+      // overlay): column chunks half and half + 2 of row quadrant q
       auto blk = [&](int ci) { return sA + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
       // row chunk of 32 fp32 in a block: 16-byte piece j of row `lane`, 128-byte swizzle
       auto xoff = [&](int j) { return (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4); };
-      // x = resid + acc2 + b2, written in place over the residual (rows past the
-      // valid count take resid = 0)
-      float sum = 0.f;
+      float sum2 = 0.f;
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
         if (c < d) {
           float v[32];
-          tmem_ld32(tmem + lane_off + (uint32_t)(NA1 * FC + c), v);
+          tmem_ld32(acc2 + lane_off + (uint32_t)c, v);
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            float4* px = reinterpret_cast<float4*>(blk(ci) + xoff(j));
-            float4 x = valid ? *px : make_float4(0.f, 0.f, 0.f, 0.f);
             const float4 bb = *reinterpret_cast<const float4*>(sB2 + c + 4 * j);
-            x.x += v[4 * j] + bb.x;
-            x.y += v[4 * j + 1] + bb.y;
-            x.z += v[4 * j + 2] + bb.z;
-            x.w += v[4 * j + 3] + bb.w;
-            sum += (x.x + x.y) + (x.z + x.w);
-            *px = x;
+            float4 x;
+            x.x = v[4 * j] + bb.x;
+            x.y = v[4 * j + 1] + bb.y;
+            x.z = v[4 * j + 2] + bb.z;
+            x.w = v[4 * j + 3] + bb.w;
+            sum2 += (x.x + x.y) + (x.z + x.w);
+            *reinterpret_cast<float4*>(blk(ci) + xoff(j)) = x;
           }
         }
       }
@@ -376,7 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int c = 32 * half + 64 * ci;
         if (c < d) issue(&tO_x, blk(ci), nullptr, nullptr, c, srow);
       }
-      red_sum[half * 128 + r] = sum;
+      red_sum[half * 128 + r] = sum2;
       pair_sync();
       const float mean = (red_sum[r] + red_sum[128 + r]) / (float)d;
       float var = 0.f;
@@ -425,7 +548,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       stores_read();
-      if (lane == 0) mbar_arrive_one(r_empty);  // sA may take the next tile's LN(x)
+      if (lane == 0) mbar_arrive_one(r_empty);  // sA may take the next tile's A
     }
     if (lane == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
   }
@@ -441,6 +564,7 @@ int g_ffn_sms = 0;
 
 bool ffn_supported(int d, int d_pad, int F, int nb) {
   if (d > 128 || d % 32 || F % FC || F < FC || NA1 * FC + d > 512) return false;
+  if (d_pad != (d > BK ? 2 * BK : BK)) return false;
   const FfnLayout L = ffn_layout(d, d_pad, F, nb);
   return L.ring >= 2 && L.smem <= kSmemMaxBlock;
 }
@@ -459,19 +583,21 @@ cudaError_t ffn_prepare() {
   return e;
 }
 
-cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* w1_h,
-                       const CUtensorMap* w1_l, const CUtensorMap* w2_h, const CUtensorMap* w2_l,
-                       const CUtensorMap* o_h, const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p,
-                       cudaStream_t s) {
+cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* wo_h,
+                       const CUtensorMap* wo_l, const CUtensorMap* w1_h, const CUtensorMap* w1_l,
+                       const CUtensorMap* w2_h, const CUtensorMap* w2_l, const CUtensorMap* o_h,
+                       const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p, cudaStream_t s) {
   if (p.rows <= 0) return cudaSuccess;
+  if (!p.x0_row && (!p.x0 || p.ldx0 < p.d || p.ldx0 % 4)) return cudaErrorInvalidValue;
   const FfnLayout LY = ffn_layout(p.d, p.d_pad, p.F, p.nb);
   const long long tiles = (p.rows + BM - 1) / BM;
   long long grid = g_ffn_sms > 0 ? g_ffn_sms : 148;
   if (grid > tiles) grid = tiles;
   auto kern = p.d_pad > BK ? (p.nb > 1 ? ffn_kernel<2, 2> : ffn_kernel<2, 1>)
                            : (p.nb > 1 ? ffn_kernel<1, 2> : ffn_kernel<1, 1>);
-  return launch_k(kern, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *a_h, *a_l, *w1_h,
-                  p.nb > 1 ? *w1_l : *w1_h, *w2_h, p.nb > 1 ? *w2_l : *w2_h, *o_h, *o_l, *o_x, p);
+  return launch_k(kern, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *a_h, *a_l, *wo_h,
+                  p.nb > 1 ? *wo_l : *wo_h, *w1_h, p.nb > 1 ? *w1_l : *w1_h, *w2_h, p.nb > 1 ? *w2_l : *w2_h, *o_h,
+                  *o_l, *o_x, p);
 }
 
 }  // namespace fe

@@ -92,11 +92,13 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l,
                         const CUtensorMap* o_x, const GemmParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
-// Fused FFN block for rows of width d <= 128 (fe_ffn.cu):
-//   x_out = x + ReLU(LN(x) W1 + b1) W2 + b2, and LN(x_out)
-// A: LN(x) planes (64 x 128 boxes, 128-byte swizzle); W1^T [F, d_pad] planes
-// with 64 x 64 boxes; W2^T [d, F_pad] planes with 64 x d boxes; outputs
-// through the same store descriptors as the GEMM epilogue.
+// Attention output projection + FFN block for rows of width d <= 128 (fe_ffn.cu):
+//   x = x0 + A W_O,   x_out = x + ReLU(LN(x) W1 + b1) W2 + b2, and LN(x_out)
+// A: attention output planes (64 x 128 boxes, 128-byte swizzle); W_O^T [d, d_pad]
+// and W2^T [d, F_pad] planes with 64 x d boxes; W1^T [F, d_pad] planes with
+// 64 x 128 boxes; outputs through the same store descriptors as the GEMM
+// epilogue.  x0 rows are fp32 [rows, ldx0] (o_x may write the same rows), or
+// one row x0_row added to every row.
 // ---------------------------------------------------------------------------
 struct FfnParams {
   int rows;             // row extent of the A descriptors
@@ -104,17 +106,18 @@ struct FfnParams {
   int d, d_pad, F, nb;
   const float* b1;      // [F]
   const float* b2;      // [d]
-  const float* resid;   // x rows
-  int ldr;
+  const float* x0;      // block input rows, unless x0_row is set
+  int ldx0;             // multiple of 4
+  const float* x0_row;  // [d], when set: the same input row for every row
   float eps;
   int* status;
 };
 bool ffn_supported(int d, int d_pad, int F, int nb);
 cudaError_t ffn_prepare();
-cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* w1_h,
-                       const CUtensorMap* w1_l, const CUtensorMap* w2_h, const CUtensorMap* w2_l,
-                       const CUtensorMap* o_h, const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p,
-                       cudaStream_t s);
+cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* wo_h,
+                       const CUtensorMap* wo_l, const CUtensorMap* w1_h, const CUtensorMap* w1_l,
+                       const CUtensorMap* w2_h, const CUtensorMap* w2_l, const CUtensorMap* o_h,
+                       const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Context LayerNorm + K/V projection in one kernel (d <= 128, bf16 inputs,
