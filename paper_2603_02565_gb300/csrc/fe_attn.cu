@@ -456,6 +456,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     if (ok && have_done) finish(gc - 1);
   }
 
+  __syncwarp();  // each warp arrives whole: single lanes ran the producer and MMA loops
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, Cfg::kTmemCols);

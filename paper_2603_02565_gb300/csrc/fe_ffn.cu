@@ -9,24 +9,23 @@
 //   warp 0 lane 0 : TMA producer -- the A tile (hi/lo) and a ring of weight
 //                   slots in consumption order W_O, W1_0, W1_1, W1_2, W2_0,
 //                   W1_3, W2_1, ...
-//   warp 1 lane 0 : tcgen05.mma -- A W_O into the d-column accumulator that
-//                   FFN2 uses; after the epilogue has put x there and LN(x)
-//                   in shared memory, FFN1 chunk f (N = 128) into one of three
-//                   TMEM buffers, two chunks ahead of FFN2 of chunk f-2, which
-//                   reads its A operand from that TMEM buffer and accumulates
-//                   on top of x
-//   warps 2-9     : per tile: x0 rows read into registers while the A tile
-//                   arrives, x = x0 + A W_O written back into the
-//                   accumulator, LN(x) written over the A tile as FFN1's
-//                   operand; per chunk:
+//   warp 1 lane 0 : tcgen05.mma -- A W_O into the TMEM buffer of FFN1 chunk
+//                   0; after the epilogue has written x into the d-column
+//                   accumulator and LN(x) in shared memory, FFN1 chunk f
+//                   (N = 128) into one of three TMEM buffers, two chunks ahead
+//                   of FFN2 of chunk f-2, which reads its A operand from that
+//                   TMEM buffer and accumulates on top of x
+//   warps 2-9     : per tile: x0 rows written into the accumulator while the
+//                   projection runs, then x = x0 + A W_O written there and
+//                   LN(x) written over the A tile as FFN1's operand; per chunk:
 //                   bias + ReLU, split into hi/lo bf16 and written back over
 //                   the chunk's fp32 columns in TMEM; per tile: x_out =
 //                   accumulator + b2, LayerNorm, stored with TMA tensor stores
 //                   staged in the tile's own 4 KB blocks
 // The MMA groups are 16 instructions of N >= 128 so that the tensor pipe has
 // queued work while the issuing thread polls its barriers; x0 is read by the
-// epilogue warps before the projection completes, when they have nothing else
-// in flight; the biases sit in shared memory.
+// epilogue warps while the A tile is in flight, when they have nothing else to
+// do; the biases sit in shared memory.
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -107,7 +106,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* acc1_empty = bars + 21;  // [NA1] FFN2 has read the buffer's hidden activation
   uint64_t* mid_full = bars + 24;    // [NA1] hidden activation written over the buffer
   uint64_t* acc2_full = bars + 27;
-  uint64_t* acc2_empty = bars + 28;
   uint64_t* ln_full = bars + 29;     // x back in the accumulator, LN(x) in sA
   uint64_t* r_empty = bars + 30;     // staging blocks free again (their last store has read them)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 31);
@@ -127,7 +125,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(mid_full + i, 32 * kEpiWarps);
     }
     mbar_init(acc2_full, 1);
-    mbar_init(acc2_empty, kEpiWarps);
     mbar_init(ln_full, 32 * kEpiWarps);
     mbar_init(r_empty, kEpiWarps);
     fence_mbar_init();
@@ -215,13 +212,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       int tl = 0, ws = 0, gf = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
-        // ---- A W_O into the accumulator, once the previous tile's epilogue has read it
+        // ---- A W_O into the FFN1 buffer that chunk 0 of this tile uses next
         if (!mbar_wait_bounded(a_full, tl & 1, p.status)) break;
         {
-          const int slot = ws % LY.ring;
+          const int slot = ws % LY.ring, bo = gf % NA1;
           if (!mbar_wait_bounded(w_full + slot, (ws / LY.ring) & 1, p.status)) break;
-          if (tl > 0 && !mbar_wait_bounded(acc2_empty, (tl - 1) & 1, p.status)) break;
+          if (gf >= NA1 && !mbar_wait_bounded(acc1_empty + bo, ((gf / NA1) - 1) & 1, p.status)) break;
           tc_fence_after();
+          const uint32_t dst = tmem + (uint32_t)(bo * FC);
           const uint64_t a0 = umma_desc_sw128(smem_u32(sA));
           const uint64_t w0 = umma_desc_sw128(smem_u32(sW + (size_t)slot * LY.slot_bytes));
 #pragma unroll
@@ -230,9 +228,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int kk = 0; kk < BK / 16; ++kk) {
               const uint64_t ah = desc_adv(a0, (uint32_t)(kb * 2) * kAPlane + kk * 32);
               const uint64_t wh = desc_adv(w0, (uint32_t)(kb * nb) * (uint32_t)d * (BK * 2) + kk * 32);
-              umma_bf16(acc2, ah, wh, idesc2, (kb | kk) != 0 ? 1u : 0u);
-              umma_bf16(acc2, desc_adv(ah, kAPlane), wh, idesc2, 1u);
-              if (nb > 1) umma_bf16(acc2, ah, desc_adv(wh, (uint32_t)d * (BK * 2)), idesc2, 1u);
+              umma_bf16(dst, ah, wh, idesc2, (kb | kk) != 0 ? 1u : 0u);
+              umma_bf16(dst, desc_adv(ah, kAPlane), wh, idesc2, 1u);
+              if (nb > 1) umma_bf16(dst, ah, desc_adv(wh, (uint32_t)d * (BK * 2)), idesc2, 1u);
             }
           }
           umma_commit(w_empty + slot);
@@ -247,7 +245,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (s < nf) {
             // FFN1 chunk s -> acc1 buffer (gf0 + s) % NA1
             const int g = gf0 + s, b = g % NA1;
-            if (g >= NA1 && !mbar_wait_bounded(acc1_empty + b, ((g / NA1) - 1) & 1, p.status)) {
+            // (chunk 0's buffer: waited for before the projection, read by the epilogue before ln_full)
+            if (s > 0 && g >= NA1 && !mbar_wait_bounded(acc1_empty + b, ((g / NA1) - 1) & 1, p.status)) {
               ok = false;
               break;
             }
@@ -342,10 +341,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int srow = m0 + q * 32;
       const bool valid = m0 + r < rows_valid;
       // ---- x = x0 + A W_O for this thread's row, columns 32 half + 64 ci + [0, 32)
-      // (x0 of rows past the valid count is 0); x goes back into the
-      // accumulator for FFN2 to add to, LN(x) into sA (which the projection
-      // has read) as FFN1's A tile.  The first 32 columns of x0 are read
-      // while the projection completes.
+      // (x0 of rows past the valid count is 0): x0 goes into the accumulator
+      // while the projection runs into the FFN1 buffer of chunk 0, x goes
+      // back into the accumulator for FFN2 to add to, and LN(x) into sA (which
+      // the projection has read) as FFN1's A tile.
       auto load_x0 = [&](int c, float* x) {
         const float* src = p.x0_row ? nullptr : p.x0 + (size_t)(m0 + r) * p.ldx0 + c;
 #pragma unroll
@@ -361,8 +360,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           x[4 * j + 3] = v.w;
         }
       };
-      float xr[32];
-      load_x0(32 * half < d ? 32 * half : 0, xr);  // (unused when 32 half >= d)
+      // x0 into the accumulator (this warp's lanes and columns, read by this
+      // warp in the previous tile's final phase) while the projection runs
+#pragma unroll
+      for (int ci = 0; ci < 2; ++ci) {
+        const int c = 32 * half + 64 * ci;
+        if (c < d) {
+          float xr[32];
+          load_x0(c, xr);
+          tmem_st32(acc2 + lane_off + (uint32_t)c, xr);
+        }
+      }
+      const uint32_t proj = tmem + (uint32_t)((gf % NA1) * FC);  // A W_O
       if (!mbar_wait_bounded(o_done, tl & 1, p.status)) break;
       tc_fence_after();
       float sum = 0.f;
@@ -370,12 +379,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
         if (c < d) {
-          if (ci > 0) load_x0(c, xr);
-          float v[32];
-          tmem_ld32(acc2 + lane_off + (uint32_t)c, v);
+          float v[32], w[32];
+          tmem_ld32(proj + lane_off + (uint32_t)c, v);
+          tmem_ld32(acc2 + lane_off + (uint32_t)c, w);
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            v[j] += xr[j];
+            v[j] += w[j];
             sum += v[j];
           }
           tmem_st32(acc2 + lane_off + (uint32_t)c, v);
@@ -466,9 +475,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---- final: x_out = acc2 + b2 (acc2 = x + FFN2), LayerNorm, stores
       if (!mbar_wait_bounded(acc2_full, tl & 1, p.status)) break;
       tc_fence_after();
-      // this warp's staging blocks (every FFN1 has read the LN(x) tile they
-      // overlay): column chunks half and half + 2 of row quadrant q
+      // this warp's staging blocks: column chunks half and half + 2 of row
+      // quadrant q; x_out in sA (every FFN1 has read the LN(x) tile there),
+      // LN(x_out) in the weight ring (every MMA of the tile has completed, and
+      // the producer loads nothing more before r_empty)
       auto blk = [&](int ci) { return sA + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
+      auto lblk = [&](int ci) { return sW + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
       // row chunk of 32 fp32 in a block: 16-byte piece j of row `lane`, 128-byte swizzle
       auto xoff = [&](int j) { return (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4); };
       float sum2 = 0.f;
@@ -491,9 +503,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_one(acc2_empty);  // accumulator read
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
@@ -523,7 +532,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       red_var[half * 128 + r] = var;
       pair_sync();
       const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)d + p.eps);
-      stores_read();  // the x stores have read the blocks
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
@@ -535,24 +543,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             split2((x.x - mean) * rstd, (x.y - mean) * rstd, hi[2 * j], lo[2 * j]);
             split2((x.z - mean) * rstd, (x.w - mean) * rstd, hi[2 * j + 1], lo[2 * j + 1]);
           }
-          __syncwarp();  // every row of the block is read before the planes overwrite it
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
-            *reinterpret_cast<uint4*>(blk(ci) + o) =
+            *reinterpret_cast<uint4*>(lblk(ci) + o) =
                 make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
-            *reinterpret_cast<uint4*>(blk(ci) + 2048 + o) =
+            *reinterpret_cast<uint4*>(lblk(ci) + 2048 + o) =
                 make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
           }
-          issue(&tO_h, blk(ci), &tO_l, blk(ci) + 2048, c, srow);
+          issue(&tO_h, lblk(ci), &tO_l, lblk(ci) + 2048, c, srow);
         }
       }
       stores_read();
-      if (lane == 0) mbar_arrive_one(r_empty);  // sA may take the next tile's A
+      if (lane == 0) mbar_arrive_one(r_empty);  // sA and the ring may take the next tile's loads
     }
     if (lane == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
   }
 
+  __syncwarp();  // each warp arrives whole: lane 0 of warps 0 and 1 ran the producer and MMA loops
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 512);
@@ -566,7 +574,8 @@ bool ffn_supported(int d, int d_pad, int F, int nb) {
   if (d > 128 || d % 32 || F % FC || F < FC || NA1 * FC + d > 512) return false;
   if (d_pad != (d > BK ? 2 * BK : BK)) return false;
   const FfnLayout L = ffn_layout(d, d_pad, F, nb);
-  return L.ring >= 2 && L.smem <= kSmemMaxBlock;
+  // the ring also stages LN(x_out): d / 32 column chunks x 4 row quadrants x 4 KB
+  return L.ring >= 2 && L.smem <= kSmemMaxBlock && (size_t)L.ring * L.slot_bytes >= (size_t)d * 512u;
 }
 
 cudaError_t ffn_prepare() {

@@ -480,6 +480,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
   }
 
+  __syncwarp();  // each warp arrives whole: single lanes ran the producer and MMA loops
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, ncols);
