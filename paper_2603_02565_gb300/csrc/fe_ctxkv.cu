@@ -3,23 +3,31 @@
 // d <= 128 with bf16 inputs and bf16-exact weights.  LN(context) never
 // reaches memory; K/V leave as one f16 plane (the attention operand).
 //
+// The LayerNorm has no affine parameters, so with mu and rstd the row's mean
+// and 1 / sqrt(var + eps),
+//     LN(x) W = rstd (x W) - rstd mu (1^T W):
+// the MMA multiplies the raw bf16 rows as they arrive (one exact bf16 plane,
+// no normalised operand tile), and the epilogue applies each row's rstd and
+// -rstd mu with the column sums of W before rounding to f16.
+//
 // The N = 2 * n_layers * d output columns are split in two halves; CTA c
 // owns half c % 2 (its slice of W^T stays resident in shared memory) and
 // walks 128-row blocks of context rows:
 //   warp 0 lane 0 : TMA -- the resident weight half once, then the raw
 //                   context block of every tile into one of two staging
 //                   buffers
-//   warp 1 lane 0 : tcgen05.mma -- X W_half (N/2 <= 256 columns) into one of
-//                   two TMEM accumulators, so the epilogue drains one tile
-//                   while the next is multiplied
-//   warps 2-9     : LayerNorm, two threads per context row (one 64-column
-//                   half each, partial sums exchanged by shuffle), from the
-//                   staged raw block into the split (hi/lo bf16) A operand tile
-//   warps 10-17   : epilogue -- TMEM -> f16 -> 32 x 32 staging blocks -> TMA
-//                   tensor stores; warps w and w+4 on TMEM lane quadrant w % 4,
-//                   alternating 32-column chunks
-// Each context row is normalised once per column half; the raw rows are
-// bf16, so the second reading costs d * 2 bytes per row.
+//   warp 1 lane 0 : tcgen05.mma -- X W_half (N/2 <= 256 columns) from the
+//                   staged raw block into one of two TMEM accumulators, so the
+//                   epilogue drains one tile while the next is multiplied
+//   warps 2-9     : LayerNorm statistics, two threads per context row (each
+//                   half of every 64-column k block, partial sums exchanged by
+//                   shuffle), from the staged raw block
+//   warps 10-17   : epilogue -- column sums of the weight half once; per tile
+//                   TMEM -> rstd acc - rstd mu colsum -> f16 -> 32 x 32 staging
+//                   blocks -> TMA tensor stores; warps w and w+4 on TMEM lane
+//                   quadrant w % 4, alternating 32-column chunks
+// The raw rows are bf16, so each column half's second reading of them costs
+// d * 2 bytes per row.
 //
 // Linear-attention state mode (STATE, two layers, C a multiple of 128): the
 // half of CTA c is layer c % 2, [K_l | V_l].  K/V never leave the chip: the
@@ -48,7 +56,7 @@ constexpr size_t kSmemMaxBlock = 232448;
 constexpr uint32_t kStateTile = 2 * 16384;  // a 128 x 128 f16 MN-major operand: two 64-wide atoms of 128 rows
 
 struct CtxKvLayout {
-  uint32_t w_bytes, a_bytes, raw_bytes, nraw, tail_bytes;
+  uint32_t w_bytes, aux_bytes, raw_bytes, nraw, tail_bytes;
   size_t smem;
 };
 
@@ -57,11 +65,11 @@ struct CtxKvLayout {
 __host__ __device__ inline CtxKvLayout ctxkv_layout(int d_pad, int N, bool state) {
   CtxKvLayout L;
   L.w_bytes = (uint32_t)(d_pad / BK) * (uint32_t)(N / 2) * (BK * 2);  // [kb][N/2 rows x 128 B]
-  L.a_bytes = (uint32_t)(d_pad / BK) * 2u * kPlane;                   // [kb][hi, lo]
+  L.aux_bytes = 4096;  // column sums of the weight half [256] fp32, row statistics [2][128] float2
   L.raw_bytes = (uint32_t)(d_pad / BK) * kPlane;                      // one raw block [kb]
   L.nraw = state ? 1u : 2u;
   L.tail_bytes = state ? 2u * kStateTile : (uint32_t)kEpiWarps * 2u * kStage;
-  L.smem = 1024 + (size_t)L.w_bytes + L.a_bytes + L.nraw * (size_t)L.raw_bytes + L.tail_bytes + 256;
+  L.smem = 1024 + (size_t)L.w_bytes + L.aux_bytes + L.nraw * (size_t)L.raw_bytes + L.tail_bytes + 256;
   return L;
 }
 
@@ -87,6 +95,22 @@ __device__ __forceinline__ void arrive(uint64_t* bar) {
 
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+
+// Column i of the weight half, summed over its rows (row i of the resident
+// W^T slice [kb][Nh rows x 128 B]; the swizzle only permutes a row's pieces).
+__device__ __forceinline__ float weight_colsum(const uint8_t* sW, int Nh, int nkb, int i) {
+  float s = 0.f;
+  for (int kb = 0; kb < nkb; ++kb) {
+    const uint8_t* row = sW + ((size_t)kb * Nh + i) * 128u;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const uint4 q = *reinterpret_cast<const uint4*>(row + 16 * j);
+      s += (bf16_lo(q.x) + bf16_hi(q.x)) + (bf16_lo(q.y) + bf16_hi(q.y)) + (bf16_lo(q.z) + bf16_hi(q.z)) +
+           (bf16_lo(q.w) + bf16_hi(q.w));
+    }
+  }
+  return s;
+}
 }  // namespace
 
 template <int NKB, bool STATE>
@@ -101,31 +125,30 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int NRAW = STATE ? 1 : 2;                 // raw context buffers
   constexpr int NACC = STATE ? 1 : 2;                 // K/V accumulators in TMEM
   uint8_t* sW = smem;                                 // [kb][Nh rows x 128 B]
-  uint8_t* sA = sW + LY.w_bytes;                      // [kb][hi, lo]
-  uint8_t* sRaw = sA + LY.a_bytes;                    // [NRAW buffers][kb]
+  float* wsum = reinterpret_cast<float*>(sW + LY.w_bytes);  // [Nh] column sums of the weight half
+  float2* stats = reinterpret_cast<float2*>(wsum + 256);    // [NACC][128] (rstd, -rstd mu) per row
+  uint8_t* sRaw = sW + LY.w_bytes + LY.aux_bytes;     // [NRAW buffers][kb]: the MMA's A operand
   uint8_t* sStg = sRaw + NRAW * (size_t)LY.raw_bytes;  // plain: [epilogue warp][2][2 KB]; state: phi(K) tile, V tile
   uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + LY.tail_bytes);
   uint64_t* w_full = bars;         // resident weight half loaded
   uint64_t* raw_full = bars + 1;   // [2] raw context block staged
-  uint64_t* raw_empty = bars + 3;  // [2] the LayerNorm threads are done with it
-  uint64_t* a_full = bars + 5;     // A tile written
-  uint64_t* a_empty = bars + 6;    // the MMAs of the tile have read the A tile
+  uint64_t* raw_empty = bars + 3;  // [2] the LayerNorm threads and the MMAs are done with it
   uint64_t* acc_full = bars + 7;   // [2] accumulator complete in TMEM
   uint64_t* acc_empty = bars + 9;  // [2] accumulator drained
   uint64_t* st_full = bars + 11;   // state mode: the state product of the tile complete
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  uint64_t* stats_full = bars + 12;  // [2] row statistics of the tile written
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     mbar_init(w_full, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(raw_full + i, 1);
-      mbar_init(raw_empty + i, 32 * kLnWarps);
+      mbar_init(raw_empty + i, 32 * kLnWarps + 1);  // + the MMA commit
+      mbar_init(stats_full + i, 32 * kLnWarps);
       mbar_init(acc_full + i, 1);
       mbar_init(acc_empty + i, kEpiWarps);
     }
-    mbar_init(a_full, 32 * kLnWarps);
-    mbar_init(a_empty, 1);
     mbar_init(st_full, 1);
     fence_mbar_init();
     prefetch_tmap(&tX);
@@ -190,28 +213,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int t = tile_at(it); t >= 0 && ok; t = tile_at(++it)) {
         const int ab = it % NACC;
         if (it >= NACC && !mbar_wait_bounded(acc_empty + ab, ((it / NACC) - 1) & 1, p.status)) break;
-        if (!mbar_wait_bounded(a_full, it & 1, p.status)) break;
+        const int rb = it % NRAW;
+        if (!mbar_wait_bounded(raw_full + rb, (it / NRAW) & 1, p.status)) break;
         tc_fence_after();
         const uint32_t dst = tmem + (uint32_t)(256 * ab);
-        const uint64_t a0 = umma_desc_sw128(smem_u32(sA));
+        const uint64_t a0 = umma_desc_sw128(smem_u32(sRaw + (size_t)rb * LY.raw_bytes));
         const uint64_t w0 = umma_desc_sw128(smem_u32(sW));
 #pragma unroll
         for (int kb = 0; kb < NKB; ++kb) {
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t ah = desc_adv(a0, (uint32_t)(kb * 2) * kPlane + kk * 32);
+            const uint64_t ah = desc_adv(a0, (uint32_t)kb * kPlane + kk * 32);
             const uint64_t wh = desc_adv(w0, (uint32_t)kb * (uint32_t)Nh * (BK * 2) + kk * 32);
             umma_bf16(dst, ah, wh, idesc, (kb | kk) != 0 ? 1u : 0u);
-            umma_bf16(dst, desc_adv(ah, kPlane), wh, idesc, 1u);
           }
         }
-        umma_commit(a_empty);  // the A tile frees once these MMAs complete
+        umma_commit(raw_empty + rb);  // the raw block frees once these MMAs (and the statistics) are done
         umma_commit(acc_full + ab);
       }
     }
   } else if (warp < 2 + kLnWarps) {
-    // ---------------- LayerNorm: two threads per row ----------------
-    // lanes l and l ^ 16 share row r; part 0 takes pieces [0, 8 NKB / 2), part 1 the rest
+    // ---------------- LayerNorm statistics: two threads per row ----------------
+    // lanes l and l ^ 16 share row r; of each 64-column k block part 0 takes
+    // the first four 16-byte pieces, part 1 the last four
     const int r = (warp - 2) * 16 + (lane & 15), part = lane >> 4;
     constexpr int kPieces = 4 * NKB;  // 16-byte pieces (8 columns) per thread
     int it = 0;
@@ -219,9 +243,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int rb = it % NRAW;
       if (!mbar_wait_bounded(raw_full + rb, (it / NRAW) & 1, p.status)) break;
       const uint8_t* raw = sRaw + (size_t)rb * LY.raw_bytes;
-      // piece j of this thread: global piece g = part * kPieces + j, column 8 g,
-      // 128-byte-swizzled within its 64-column block
-      auto gpiece = [&](int j) { return part * kPieces + j; };
+      // piece j of this thread: global piece g, column 8 g, 128-byte-swizzled
+      // within its 64-column block
+      auto gpiece = [&](int j) { return (j >> 2) * 8 + part * 4 + (j & 3); };
       auto piece_off = [&](int g) {
         return (size_t)(g >> 3) * kPlane + (uint32_t)r * 128u + ((uint32_t)((g & 7) ^ (r & 7)) << 4);
       };
@@ -251,27 +275,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       q2 += __shfl_xor_sync(0xffffffffu, q2, 16);
       const float rstd = 1.0f / sqrtf(q2 / (float)d + p.eps);
-      // the previous tile's MMAs must be done with the A tile
-      if (it > 0 && !mbar_wait_bounded(a_empty, (it - 1) & 1, p.status)) break;
-#pragma unroll
-      for (int j = 0; j < kPieces; ++j) {
-        const int g = gpiece(j);
-        uint32_t hi[4] = {0u, 0u, 0u, 0u}, lo[4] = {0u, 0u, 0u, 0u};
-        if (8 * g < d) {
-          const uint4 q = *reinterpret_cast<const uint4*>(raw + piece_off(g));
-          const uint32_t w[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-          for (int e = 0; e < 4; ++e)
-            split2((bf16_lo(w[e]) - mean) * rstd, (bf16_hi(w[e]) - mean) * rstd, hi[e], lo[e]);
-        }
-        // A planes: hi of k block g / 8 at (2 (g / 8)) * kPlane, lo one plane after
-        const size_t o = piece_off(g) + (size_t)(g >> 3) * kPlane;
-        *reinterpret_cast<uint4*>(sA + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-        *reinterpret_cast<uint4*>(sA + o + kPlane) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-      }
+      // the statistics slot: the epilogue must be done with the tile it held
+      const int sl = it % NACC;
+      if (it >= NACC && !mbar_wait_bounded(acc_empty + sl, ((it / NACC) - 1) & 1, p.status)) break;
+      if (part == 0) stats[sl * 128 + r] = make_float2(rstd, -mean * rstd);
+      arrive(stats_full + sl);
       arrive(raw_empty + rb);
-      fence_async_shared();
-      arrive(a_full);
     }
   } else if constexpr (STATE) {
     // ---------------- epilogue, state mode ----------------
@@ -296,15 +305,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     const uint32_t idesc = umma_idesc_f16(BM, d) | (1u << 15) | (1u << 16);  // A and B MN-major
     float zsum[2] = {0.f, 0.f};  // this lane's feature of each K chunk it handles: the segment's sum of phi(K)
+    const bool wok = mbar_wait_bounded(w_full, 0, p.status);
+    if (wok && ew * 32 + lane < Nh) wsum[ew * 32 + lane] = weight_colsum(sW, Nh, NKB, ew * 32 + lane);
+    epi_sync();
     int it = 0;
-    for (int t = tile_at(it); t >= 0; t = tile_at(++it)) {
+    for (int t = tile_at(it); t >= 0 && wok; t = tile_at(++it)) {
       const int pos = it % Ts;   // row block of the segment
       if (!mbar_wait_bounded(acc_full, it & 1, p.status)) break;
+      if (!mbar_wait_bounded(stats_full, it & 1, p.status)) break;
       tc_fence_after();
+      const float2 st = stats[r];  // rstd, -rstd mu of this thread's row
       int kc = 0;
       for (int c = 32 * sub; c < 2 * d; c += 64) {
         float v[32];
         tmem_ld32(tmem + lane_off + (uint32_t)c, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = fmaf(st.x, v[i], st.y * wsum[c + i]);  // LN(x) W
         const bool isk = c < d;
         const int m0 = isk ? c : c - d;
         if (isk) {
@@ -394,16 +410,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int sub = ew >> 2;             // alternate 32-column chunks
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     uint8_t* stg0 = sStg + (size_t)ew * 2 * kStage;
+    const int r = q * 32 + lane;  // this thread's row of the tile
+    const bool wok = mbar_wait_bounded(w_full, 0, p.status);
+    if (wok && ew * 32 + lane < Nh) wsum[ew * 32 + lane] = weight_colsum(sW, Nh, NKB, ew * 32 + lane);
+    asm volatile("bar.sync 5, 256;" ::: "memory");  // the eight epilogue warps: column sums written
     int nstore = 0;
     int it = 0;
-    for (int t = tile_at(it); t >= 0; t = tile_at(++it)) {
+    for (int t = tile_at(it); t >= 0 && wok; t = tile_at(++it)) {
       const int ab = it & 1;
       if (!mbar_wait_bounded(acc_full + ab, (it >> 1) & 1, p.status)) break;
+      if (!mbar_wait_bounded(stats_full + ab, (it >> 1) & 1, p.status)) break;
       tc_fence_after();
+      const float2 st = stats[ab * 128 + r];  // rstd, -rstd mu of this thread's row
       const int srow = t * BM + q * 32;
       for (int c = 32 * sub; c < Nh; c += 64) {
         float v[32];
         tmem_ld32(tmem + lane_off + (uint32_t)(256 * ab + c), v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = fmaf(st.x, v[i], st.y * wsum[c + i]);  // LN(x) W
         // alternate staging buffers; the one written two stores ago must be read
         uint8_t* b = stg0 + (size_t)(nstore & 1) * kStage;
         if (lane == 0 && nstore >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
