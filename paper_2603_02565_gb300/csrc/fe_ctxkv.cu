@@ -51,6 +51,7 @@ constexpr int kEpiWarps = 8;
 constexpr int kThreads = 32 * (2 + kLnWarps + kEpiWarps);  // 576
 constexpr uint32_t kPlane = BM * BK * 2;                     // 16 KB: 128 rows x 64 bf16
 constexpr uint32_t kStage = 2048;                            // store staging: 32 rows x 32 f16, 64-byte swizzle
+constexpr int kStgBufs = 4;                                  // staging buffers per epilogue warp (stores in flight)
 constexpr size_t kSmemMaxBlock = 232448;
 
 constexpr uint32_t kStateTile = 2 * 16384;  // a 128 x 128 f16 MN-major operand: two 64-wide atoms of 128 rows
@@ -68,7 +69,7 @@ __host__ __device__ inline CtxKvLayout ctxkv_layout(int d_pad, int N, bool state
   L.aux_bytes = 4096;  // column sums of the weight half [256] fp32, row statistics [2][128] float2
   L.raw_bytes = (uint32_t)(d_pad / BK) * kPlane;                      // one raw block [kb]
   L.nraw = state ? 1u : 2u;
-  L.tail_bytes = state ? 2u * kStateTile : (uint32_t)kEpiWarps * 2u * kStage;
+  L.tail_bytes = state ? 2u * kStateTile : (uint32_t)kEpiWarps * (uint32_t)kStgBufs * kStage;
   L.smem = 1024 + (size_t)L.w_bytes + L.aux_bytes + L.nraw * (size_t)L.raw_bytes + L.tail_bytes + 256;
   return L;
 }
@@ -128,7 +129,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* wsum = reinterpret_cast<float*>(sW + LY.w_bytes);  // [Nh] column sums of the weight half
   float2* stats = reinterpret_cast<float2*>(wsum + 256);    // [NACC][128] (rstd, -rstd mu) per row
   uint8_t* sRaw = sW + LY.w_bytes + LY.aux_bytes;     // [NRAW buffers][kb]: the MMA's A operand
-  uint8_t* sStg = sRaw + NRAW * (size_t)LY.raw_bytes;  // plain: [epilogue warp][2][2 KB]; state: phi(K) tile, V tile
+  uint8_t* sStg = sRaw + NRAW * (size_t)LY.raw_bytes;  // plain: [epilogue warp][kStgBufs][2 KB]; state: phi(K) tile, V tile
   uint64_t* bars = reinterpret_cast<uint64_t*>(sStg + LY.tail_bytes);
   uint64_t* w_full = bars;         // resident weight half loaded
   uint64_t* raw_full = bars + 1;   // [2] raw context block staged
@@ -409,7 +410,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;              // TMEM lane quadrant this warp may access
     const int sub = ew >> 2;             // alternate 32-column chunks
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    uint8_t* stg0 = sStg + (size_t)ew * 2 * kStage;
+    uint8_t* stg0 = sStg + (size_t)ew * kStgBufs * kStage;
     const int r = q * 32 + lane;  // this thread's row of the tile
     const bool wok = mbar_wait_bounded(w_full, 0, p.status);
     if (wok && ew * 32 + lane < Nh) wsum[ew * 32 + lane] = weight_colsum(sW, Nh, NKB, ew * 32 + lane);
@@ -428,9 +429,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32(tmem + lane_off + (uint32_t)(256 * ab + c), v);
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = fmaf(st.x, v[i], st.y * wsum[c + i]);  // LN(x) W
-        // alternate staging buffers; the one written two stores ago must be read
-        uint8_t* b = stg0 + (size_t)(nstore & 1) * kStage;
-        if (lane == 0 && nstore >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+        // rotating staging buffers: the one written kStgBufs stores ago must have been read
+        uint8_t* b = stg0 + (size_t)(nstore % kStgBufs) * kStage;
+        if (lane == 0 && nstore >= kStgBufs)
+          asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(kStgBufs - 1) : "memory");
         __syncwarp();
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
