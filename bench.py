@@ -86,8 +86,11 @@ def describe(w):
 # algorithmic work per launch site (flops, bytes); split activations are 4 B/element, the
 # single-plane f16 attention operands (context K/V, element Q, cross Q/K/V) 2 B/element
 # ----------------------------------------------------------------------------------------------
-def site_work(site, cfg, B, C, M, K, L, R):
+def site_work(site, cfg, B, C, M, K, L, R, per_step=None):
+    """per_step: launches per step of every site (tells whether the element-layer
+    FFN launches also ran the next layer's Q and SeqEnc's element K/V)."""
     d, F, Ly = cfg.d, cfg.F, cfg.n_layers
+    per_step = per_step or {}
     T = int(getattr(cfg, "n_tasks", 1))
     S, n = B * K, B * C
     esz = 2 if cfg.io_bf16 else 4
@@ -110,7 +113,8 @@ def site_work(site, cfg, B, C, M, K, L, R):
         "gemm_item_o_ln": (2 * R * d * d, R * d * (A + 8 + A)),
         "gemm_item_ffn1": (2 * R * d * F, R * d * A + R * F * A),
         "gemm_item_ffn2_ln": (2 * R * F * d, R * F * A + R * d * (8 + A)),
-        # attention output projection + FFN: A in, x0 in, x out, LN(x_out) out
+        # attention output projection + FFN: A in, x0 in, x out, LN(x_out) out (averaged over the
+        # layers below when the launches also carry the tail products)
         "ffn_item": (2 * R * d * d + 4 * R * d * F, R * d * (A + 8 + A)),
         "gemm_item_seq_kv": (4 * R * d * d, R * d * A + 2 * R * d * A),
         "seq_cls_attn": (4 * S * (L + 1) * d, 2 * R * d * A + 4 * S * L + S * d * A),
@@ -124,6 +128,20 @@ def site_work(site, cfg, B, C, M, K, L, R):
         "gemm_head": (2 * S * d * d * T + 3 * S * d * T, S * d * A + 4 * S * (1 + (T if T > 1 else 0))),
         "select": (0, 4 * S + 4 * B),
     }
+    if site == "ffn_item" and per_step:
+        # tails: layers < Ly-1 write the next layer's Q (f16) instead of LN(x_out); the last
+        # layer also writes the element K/V (split pair); averaged per launch
+        tq = Ly > 1 and per_step.get("gemm_item_q", Ly) < Ly
+        tkv = "gemm_item_seq_kv" not in per_step
+        fl, by = t["ffn_item"]
+        fl_tot, by_tot = Ly * fl, Ly * by
+        if tq:
+            fl_tot += (Ly - 1) * 2 * R * d * d
+            by_tot += (Ly - 1) * R * d * (H - A)
+        if tkv:
+            fl_tot += 4 * R * d * d
+            by_tot += 2 * R * d * A
+        return fl_tot / Ly, by_tot / Ly
     return t.get(site, (0, 0))
 
 
@@ -363,16 +381,17 @@ def run_ours(args):
     peaks, peak_src = load_peaks()
     kern = []
     step_total = sum(s[2] for s in sites) / n_prof
+    per_step = {name: nl / n_prof for name, nl, tot in sites}
     for name, nl, tot in sites:
         per_launch_ms = tot / nl
-        flops, byts = site_work(name, cfg, B, C, M, K, L, sumU)
+        flops, byts = site_work(name, cfg, B, C, M, K, L, sumU, per_step)
         kern.append({"site": name, "launches_per_step": nl / n_prof, "us_per_launch": per_launch_ms * 1e3,
                      "share": (tot / n_prof) / step_total if step_total else 0.0,
                      "gbs": byts / (per_launch_ms * 1e-3) / 1e9 if byts else 0.0,
                      "tflops": flops / (per_launch_ms * 1e-3) / 1e12 if flops else 0.0})
     roof = None
     dom = max(kern, key=lambda k: k["share"])
-    flops, byts = site_work(dom["site"], cfg, B, C, M, K, L, sumU)
+    flops, byts = site_work(dom["site"], cfg, B, C, M, K, L, sumU, per_step)
     t_launch = dom["us_per_launch"] * 1e-6
     tensor_bound = flops / (peaks["bf16_tflops"] * 1e12) > byts / (peaks["hbm_gbs"] * 1e9)
     if args.factorized:

@@ -190,7 +190,7 @@ int alloc_f32(F32Rows& f, int rows, int ld, std::vector<void*>& owned) {
 struct Weight {
   Planes p;
   int N = 0, K_pad = 0, BN = 0, stages = 0;
-  CUtensorMap fh{}, fl{};  // W1 of the fused FFN: 64 x 128 boxes
+  CUtensorMap fh{}, fl{};  // W1 of the fused FFN: 64 x 128 boxes; a fused FFN's tail weight: 64 x N
 };
 
 int largest_bn(int N, int cap) {
@@ -248,6 +248,8 @@ struct fe_ctx {
   int device = 0;
   int d = 0, H = 0, dh = 0, Ly = 0, F = 0, dpad = 0, Fpad = 0, nb = 1;
   bool fused_ffn = false;  // FFN1 + FFN2 in one kernel (d <= 128)
+  bool tail_q = false;     // the fused FFN of layer l also projects the next layer's Q
+  bool tail_kv = false;    // the fused FFN of the last layer also projects [WKs | WVs]
   bool fused_ctxkv = false;  // context LN + K/V projection in one kernel (d <= 128, bf16 inputs)
   CUtensorMap ctxkv_w{};     // W^T of the K/V projection, 64 x 128 boxes, for the fused kernel
   std::vector<void*> owned_w;  // weight allocations
@@ -450,6 +452,13 @@ int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
   return rc;
 }
 
+// The weight of a fused FFN's tail product: 64 x N boxes (N <= 256).
+int map_tail(Weight& w, bool two) {
+  int rc = encode_map(&w.fh, w.p.h, w.p.ld, w.p.rows, w.N);
+  if (rc == FE_OK) rc = encode_map(&w.fl, two ? w.p.l : w.p.h, w.p.ld, w.p.rows, w.N);
+  return rc;
+}
+
 int map_fused_w1(Weight& w, bool two) {
   int rc = encode_map(&w.fh, w.p.h, w.p.ld, w.p.rows, 128);
   if (rc == FE_OK) rc = encode_map(&w.fl, two ? w.p.l : w.p.h, w.p.ld, w.p.rows, 128);
@@ -491,10 +500,12 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   return FE_OK;
 }
 
-// x = x0 + A W_O, then the FFN: x written to x (in place over x0 when x0_row is null), LN(x_out) to ln_out
+// x = x0 + A W_O, then the FFN: x written to x (in place over x0 when x0_row is null), LN(x_out) to
+// ln_out when store_ln, and with a tail weight WT the product LN(x_out) WT to tail_out (f16 when tail_f16)
 int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const Weight& W1, const Weight& W2,
         const float* b1, const float* b2, const float* x0_row, const F32Rows& x, const Planes& ln_out, int rows,
-        const int* rows_dev, cudaStream_t s) {
+        const int* rows_dev, cudaStream_t s, int store_ln = 1, const Weight* WT = nullptr,
+        const Planes* tail_out = nullptr, int tail_f16 = 0) {
   if (rows <= 0) return FE_OK;
   Prof pf(c, site, s);
   fe::FfnParams p{};
@@ -509,10 +520,14 @@ int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const We
   p.x0 = x0_row ? nullptr : x.p;
   p.ldx0 = x.ld;
   p.x0_row = x0_row;
+  p.tail_n = WT ? WT->N : 0;
+  p.tail_f16 = tail_f16;
+  p.store_ln = store_ln;
   p.eps = c->cfg.ln_eps;
   p.status = c->status;
-  FE_CK(fe::ffn_launch(&A.th, &A.tl, &WO.p.th, &WO.p.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.sh, &ln_out.sl,
-                       &x.sx, p, s));
+  FE_CK(fe::ffn_launch(&A.th, &A.tl, &WO.p.th, &WO.p.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.th, &ln_out.tl,
+                       &x.sx, WT ? &WT->fh : nullptr, WT ? &WT->fl : nullptr, tail_out ? &tail_out->sh : nullptr,
+                       tail_out ? &tail_out->sl : nullptr, p, s));
   return FE_OK;
 }
 
@@ -626,9 +641,11 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     FE_RC(gemm(c, "gemm_elem_o_ln", fe::EPI_RESID_LN, c->a, c->oe, R, sumU, po, &c->xln, &c->h, s));
   }
   for (int l = 0; l < Ly; ++l) {
-    fe::GemmParams p{};
-    p.out_f16 = 1;
-    FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
+    if (l == 0 || !c->tail_q) {  // (otherwise the previous layer's fused FFN wrote Q)
+      fe::GemmParams p{};
+      p.out_f16 = 1;
+      FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
+    }
 
     fe::AttnParams ap{};
     if (fact) {  // segment = one sequence: its L occurrences over its own context K/V
@@ -665,8 +682,13 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     }
 
     if (c->fused_ffn) {
+      // the tail: the next layer's Q (f16), or after the last layer SeqEnc's element K/V (split);
+      // LN(x_out) itself is stored when something else reads it (the last layer's: the element encodings)
+      const bool last = l == Ly - 1;
+      const Weight* WT = !last ? (c->tail_q ? &c->wq[l + 1] : nullptr) : (c->tail_kv ? &c->kvs : nullptr);
+      const Planes* TO = !last ? &c->q : &c->kvI;
       FE_RC(ffn(c, "ffn_item", c->a, c->wo[l], c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), nullptr, c->h,
-                c->xln, R, sumU, s));
+                c->xln, R, sumU, s, (last || !c->tail_q) ? 1 : 0, WT, WT ? TO : nullptr, last ? 0 : 1));
     } else {
       fe::GemmParams po{};
       po.resid = c->h.p;
@@ -685,8 +707,8 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
       FE_RC(gemm(c, "gemm_item_ffn2_ln", fe::EPI_RESID_LN, c->mid, c->w2[l], R, sumU, p2, &c->xln, &c->h, s));
     }
   }
-  // element projections of SeqEnc: H WKs | H WVs
-  {
+  // element projections of SeqEnc: H WKs | H WVs (unless the last fused FFN did them)
+  if (!(c->fused_ffn && c->tail_kv)) {
     fe::GemmParams p{};
     FE_RC(gemm(c, "gemm_item_seq_kv", fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, &c->kvI, nullptr, s));
   }
@@ -1110,6 +1132,12 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if ((rc = make_weight(c, c->w1s, F, d, 128)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w1s, tw(c, T_W1S), d, F, 0)) != FE_OK) return fail(rc);
   if (c->fused_ffn && (rc = map_fused_w1(c->w1s, c->nb > 1)) != FE_OK) return fail(rc);
+  c->tail_q = c->fused_ffn && Ly > 1 && fe::ffn_tail_supported(d, c->dpad, F, c->nb, d, 1);
+  c->tail_kv = c->fused_ffn && fe::ffn_tail_supported(d, c->dpad, F, c->nb, 2 * d, 0);
+  if (c->tail_q)
+    for (int l = 1; l < Ly; ++l)
+      if ((rc = map_tail(c->wq[l], c->nb > 1)) != FE_OK) return fail(rc);
+  if (c->tail_kv && (rc = map_tail(c->kvs, c->nb > 1)) != FE_OK) return fail(rc);
   if ((rc = make_weight(c, c->w2s, d, F, 512)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w2s, tw(c, T_W2S), F, d, 0)) != FE_OK) return fail(rc);
   if (!cfg->no_cross_seq) {

@@ -82,7 +82,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                const __grid_constant__ CUtensorMap tW1_h, const __grid_constant__ CUtensorMap tW1_l,
                const __grid_constant__ CUtensorMap tW2_h, const __grid_constant__ CUtensorMap tW2_l,
                const __grid_constant__ CUtensorMap tO_h, const __grid_constant__ CUtensorMap tO_l,
-               const __grid_constant__ CUtensorMap tO_x, const FfnParams p) {
+               const __grid_constant__ CUtensorMap tO_x, const __grid_constant__ CUtensorMap tT_h,
+               const __grid_constant__ CUtensorMap tT_l, const __grid_constant__ CUtensorMap tTo_h,
+               const __grid_constant__ CUtensorMap tTo_l, const FfnParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_s = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
@@ -90,10 +92,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int d = p.d, F = p.F;
   const FfnLayout LY = ffn_layout(d, NKB * BK, F, nb);
   const int nf = F / FC;
-  // the A tile [kb][plane], then LN(x) [kb][plane] in the same layout, then the
-  // output staging blocks [32-column chunk][row quadrant][4 KB]
+  // sA: the A tile [kb][plane], then LN(x) [kb][plane] in the same layout,
+  // then LN(x_out) the same way (stored from there, and the tail's A operand).
+  // sW: the weight ring; at the end of a tile the x_out staging blocks
+  // [32-column chunk][row quadrant][4 KB] at its start, then the tail weight
+  // [kb][plane][tail_n rows x 128 B], later the tail's output staging.
   uint8_t* sA = smem;
   uint8_t* sW = sA + LY.a_bytes;
+  const int tail_n = p.tail_n;
+  uint8_t* sT = sW + (size_t)d * 512u;
   float* sB1 = reinterpret_cast<float*>(sW + (size_t)LY.ring * LY.slot_bytes);
   float* sB2 = sB1 + F;
   float* sX0 = sB2 + d;  // the broadcast row x0, when there is one
@@ -108,7 +115,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* acc2_full = bars + 27;
   uint64_t* ln_full = bars + 29;     // x back in the accumulator, LN(x) in sA
   uint64_t* r_empty = bars + 30;     // staging blocks free again (their last store has read them)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 31);
+  uint64_t* tail_a = bars + 31;      // LN(x_out) written in sA
+  uint64_t* wt_full = bars + 32;     // tail weight loaded
+  uint64_t* tail_full = bars + 33;   // tail product complete in TMEM
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 40);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + kBarBytes);  // [sum|var][half][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -127,6 +137,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(acc2_full, 1);
     mbar_init(ln_full, 32 * kEpiWarps);
     mbar_init(r_empty, kEpiWarps);
+    mbar_init(tail_a, 32 * kEpiWarps);
+    mbar_init(wt_full, 1);
+    mbar_init(tail_full, 1);
     fence_mbar_init();
     prefetch_tmap(&tA_h);
     prefetch_tmap(&tWo_h);
@@ -201,6 +214,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int s = 0; s < nf + LA && ok; ++s) {
           if (s < nf && !load_slot(1, s)) ok = false;
           if (ok && s >= LA && !load_slot(2, s - LA)) ok = false;
+        }
+        if (ok && tail_n > 0) {
+          // the tail weight, past the x_out staging, once every FFN MMA of the
+          // tile (the last readers of the ring) has completed
+          if (!mbar_wait_bounded(acc2_full, tl & 1, p.status)) break;
+          mbar_arrive_expect_tx(wt_full, (uint32_t)nkb * nb * (uint32_t)tail_n * (BK * 2));
+          for (int kb = 0; kb < nkb; ++kb)
+            for (int q = 0; q < nb; ++q)
+              tma_load_2d(sT + (size_t)(kb * nb + q) * tail_n * (BK * 2), q ? &tT_l : &tT_h, kb * BK, 0, wt_full);
         }
       }
     }
@@ -308,6 +330,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         gf = gf0 + nf;
+        if (ok && tail_n > 0) {
+          // tail: LN(x_out) . W_t into TMEM columns [0, tail_n) (every FFN1
+          // buffer is free once the FFN2 of the tile has completed)
+          if (!mbar_wait_bounded(tail_a, tl & 1, p.status)) break;
+          if (!mbar_wait_bounded(wt_full, tl & 1, p.status)) break;
+          tc_fence_after();
+          const uint32_t idesc3 = umma_idesc_bf16(BM, tail_n);
+          const uint64_t a0 = umma_desc_sw128(smem_u32(sA));
+          const uint64_t w0 = umma_desc_sw128(smem_u32(sT));
+#pragma unroll
+          for (int kb = 0; kb < nkb; ++kb) {
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk) {
+              const uint64_t ah = desc_adv(a0, (uint32_t)(kb * 2) * kAPlane + kk * 32);
+              const uint64_t wh = desc_adv(w0, (uint32_t)(kb * nb) * (uint32_t)tail_n * (BK * 2) + kk * 32);
+              umma_bf16(tmem, ah, wh, idesc3, (kb | kk) != 0 ? 1u : 0u);
+              umma_bf16(tmem, desc_adv(ah, kAPlane), wh, idesc3, 1u);
+              if (nb > 1) umma_bf16(tmem, ah, desc_adv(wh, (uint32_t)tail_n * (BK * 2)), idesc3, 1u);
+            }
+          }
+          umma_commit(tail_full);
+        }
       }
     }
   } else {
@@ -475,12 +519,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---- final: x_out = acc2 + b2 (acc2 = x + FFN2), LayerNorm, stores
       if (!mbar_wait_bounded(acc2_full, tl & 1, p.status)) break;
       tc_fence_after();
-      // this warp's staging blocks: column chunks half and half + 2 of row
-      // quadrant q; x_out in sA (every FFN1 has read the LN(x) tile there),
-      // LN(x_out) in the weight ring (every MMA of the tile has completed, and
-      // the producer loads nothing more before r_empty)
-      auto blk = [&](int ci) { return sA + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
-      auto lblk = [&](int ci) { return sW + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
+      // this warp's x_out staging blocks at the start of the weight ring (every
+      // MMA of the tile has completed, and before r_empty the producer loads
+      // only the tail weight, past them): column chunks half and half + 2 of
+      // row quadrant q
+      auto blk = [&](int ci) { return sW + (size_t)((half + 2 * ci) * 4 + q) * kResBlock; };
       // row chunk of 32 fp32 in a block: 16-byte piece j of row `lane`, 128-byte swizzle
       auto xoff = [&](int j) { return (uint32_t)lane * 128u + ((uint32_t)(j ^ (lane & 7)) << 4); };
       float sum2 = 0.f;
@@ -532,27 +575,82 @@ __global__ void __launch_bounds__(kThreads, 1)
       red_var[half * 128 + r] = var;
       pair_sync();
       const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)d + p.eps);
+      // LN(x_out) as the split tile [kb][plane] in sA, 128-byte swizzle (every
+      // FFN1 has read the LN(x) tile there): row r, this warp's four 16-byte
+      // pieces 4 half + jj of each plane; columns past d are zeros
 #pragma unroll
-      for (int ci = 0; ci < 2; ++ci) {
+      for (int ci = 0; ci < nkb; ++ci) {
         const int c = 32 * half + 64 * ci;
+        uint32_t hi[16], lo[16];
         if (c < d) {
-          uint32_t hi[16], lo[16];
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const float4 x = *reinterpret_cast<const float4*>(blk(ci) + xoff(j));
             split2((x.x - mean) * rstd, (x.y - mean) * rstd, hi[2 * j], lo[2 * j]);
             split2((x.z - mean) * rstd, (x.w - mean) * rstd, hi[2 * j + 1], lo[2 * j + 1]);
           }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            hi[j] = 0u;
+            lo[j] = 0u;
+          }
+        }
+        uint8_t* rowp = sA + (size_t)(ci * 2) * kAPlane + (size_t)r * 128u;
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+          const uint32_t o = (uint32_t)((4 * half + jj) ^ (r & 7)) << 4;
+          *reinterpret_cast<uint4*>(rowp + o) = make_uint4(hi[4 * jj], hi[4 * jj + 1], hi[4 * jj + 2], hi[4 * jj + 3]);
+          *reinterpret_cast<uint4*>(rowp + kAPlane + o) =
+              make_uint4(lo[4 * jj], lo[4 * jj + 1], lo[4 * jj + 2], lo[4 * jj + 3]);
+        }
+      }
+      fence_async_shared();
+      if (tail_n > 0) mbar_arrive_one(tail_a);
+      if (p.store_ln) {
+        asm volatile("bar.sync 5, 256;" ::: "memory");  // every row of the tile written
+        if (ew == 0 && lane == 0) {
+          for (int kb = 0; kb < nkb; ++kb) {
+            tma_store_2d(&tO_h, sA + (size_t)(kb * 2) * kAPlane, kb * BK, m0);
+            tma_store_2d(&tO_l, sA + (size_t)(kb * 2 + 1) * kAPlane, kb * BK, m0);
+          }
+          bulk_commit();
+        }
+        __syncwarp();
+      }
+      if (tail_n > 0) {
+        // tail output: 32-column chunks half, half + 2, ... of this warp's row
+        // quadrant, f16 (one 2 KB block) or a split pair (two), through two
+        // rotating staging buffers of this warp where the tail weight was
+        if (!mbar_wait_bounded(tail_full, tl & 1, p.status)) break;
+        tc_fence_after();
+        const uint32_t tb = p.tail_f16 ? 2048u : 4096u;
+        uint8_t* stg = sT + (size_t)ew * 2u * tb;
+        int k = 0;
+        for (int c = 32 * half; c < tail_n; c += 64, ++k) {
+          float v[32];
+          tmem_ld32(tmem + lane_off + (uint32_t)c, v);
+          uint8_t* b = stg + (size_t)(k & 1) * tb;
+          if (lane == 0 && k >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+          __syncwarp();
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
-            *reinterpret_cast<uint4*>(lblk(ci) + o) =
-                make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
-            *reinterpret_cast<uint4*>(lblk(ci) + 2048 + o) =
-                make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
+            if (p.tail_f16) {
+              *reinterpret_cast<uint4*>(b + o) =
+                  make_uint4(pack_f16x2(v[8 * j], v[8 * j + 1]), pack_f16x2(v[8 * j + 2], v[8 * j + 3]),
+                             pack_f16x2(v[8 * j + 4], v[8 * j + 5]), pack_f16x2(v[8 * j + 6], v[8 * j + 7]));
+            } else {
+              uint32_t hi[4], lo[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) split2(v[8 * j + 2 * e], v[8 * j + 2 * e + 1], hi[e], lo[e]);
+              *reinterpret_cast<uint4*>(b + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+              *reinterpret_cast<uint4*>(b + 2048 + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            }
           }
-          issue(&tO_h, lblk(ci), &tO_l, lblk(ci) + 2048, c, srow);
+          issue(&tTo_h, b, p.tail_f16 ? nullptr : &tTo_l, b + 2048, c, srow);
         }
+        tc_fence_before();  // TMEM read before r_empty lets the next tile's projection in
       }
       stores_read();
       if (lane == 0) mbar_arrive_one(r_empty);  // sA and the ring may take the next tile's loads
@@ -574,8 +672,18 @@ bool ffn_supported(int d, int d_pad, int F, int nb) {
   if (d > 128 || d % 32 || F % FC || F < FC || NA1 * FC + d > 512) return false;
   if (d_pad != (d > BK ? 2 * BK : BK)) return false;
   const FfnLayout L = ffn_layout(d, d_pad, F, nb);
-  // the ring also stages LN(x_out): d / 32 column chunks x 4 row quadrants x 4 KB
+  // the ring also stages x_out: d / 32 column chunks x 4 row quadrants x 4 KB
   return L.ring >= 2 && L.smem <= kSmemMaxBlock && (size_t)L.ring * L.slot_bytes >= (size_t)d * 512u;
+}
+
+bool ffn_tail_supported(int d, int d_pad, int F, int nb, int tail_n, int tail_f16) {
+  if (!ffn_supported(d, d_pad, F, nb)) return false;
+  if (tail_n < 32 || tail_n > 256 || tail_n % 32) return false;
+  const FfnLayout L = ffn_layout(d, d_pad, F, nb);
+  // past the x_out staging: the tail weight, then the tail staging (8 warps x 2 buffers)
+  const size_t wt = (size_t)(d_pad / BK) * nb * tail_n * (BK * 2);
+  const size_t stg = (size_t)kEpiWarps * 2u * (tail_f16 ? 2048u : 4096u);
+  return (size_t)d * 512u + (wt > stg ? wt : stg) <= (size_t)L.ring * L.slot_bytes;
 }
 
 cudaError_t ffn_prepare() {
@@ -595,18 +703,28 @@ cudaError_t ffn_prepare() {
 cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* wo_h,
                        const CUtensorMap* wo_l, const CUtensorMap* w1_h, const CUtensorMap* w1_l,
                        const CUtensorMap* w2_h, const CUtensorMap* w2_l, const CUtensorMap* o_h,
-                       const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p, cudaStream_t s) {
+                       const CUtensorMap* o_l, const CUtensorMap* o_x, const CUtensorMap* t_h,
+                       const CUtensorMap* t_l, const CUtensorMap* to_h, const CUtensorMap* to_l,
+                       const FfnParams& p, cudaStream_t s) {
   if (p.rows <= 0) return cudaSuccess;
   if (!p.x0_row && (!p.x0 || p.ldx0 < p.d || p.ldx0 % 4)) return cudaErrorInvalidValue;
+  if (p.tail_n > 0 && (!t_h || !to_h || (!p.tail_f16 && !to_l) ||
+                       !ffn_tail_supported(p.d, p.d_pad, p.F, p.nb, p.tail_n, p.tail_f16)))
+    return cudaErrorInvalidValue;
   const FfnLayout LY = ffn_layout(p.d, p.d_pad, p.F, p.nb);
   const long long tiles = (p.rows + BM - 1) / BM;
   long long grid = g_ffn_sms > 0 ? g_ffn_sms : 148;
   if (grid > tiles) grid = tiles;
   auto kern = p.d_pad > BK ? (p.nb > 1 ? ffn_kernel<2, 2> : ffn_kernel<2, 1>)
                            : (p.nb > 1 ? ffn_kernel<1, 2> : ffn_kernel<1, 1>);
+  // without a tail its maps are never read: any valid descriptor stands in
+  const CUtensorMap* th = p.tail_n > 0 ? t_h : o_h;
+  const CUtensorMap* tl = p.tail_n > 0 && p.nb > 1 ? t_l : th;
+  const CUtensorMap* toh = p.tail_n > 0 ? to_h : o_h;
+  const CUtensorMap* tol = p.tail_n > 0 && !p.tail_f16 ? to_l : toh;
   return launch_k(kern, dim3((unsigned)grid), dim3(kThreads), LY.smem, s, *a_h, *a_l, *wo_h,
                   p.nb > 1 ? *wo_l : *wo_h, *w1_h, p.nb > 1 ? *w1_l : *w1_h, *w2_h, p.nb > 1 ? *w2_l : *w2_h, *o_h,
-                  *o_l, *o_x, p);
+                  *o_l, *o_x, *th, *tl, *toh, *tol, p);
 }
 
 }  // namespace fe

@@ -93,12 +93,16 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l,
 
 // ---------------------------------------------------------------------------
 // Attention output projection + FFN block for rows of width d <= 128 (fe_ffn.cu):
-//   x = x0 + A W_O,   x_out = x + ReLU(LN(x) W1 + b1) W2 + b2, and LN(x_out)
+//   x = x0 + A W_O,   x_out = x + ReLU(LN(x) W1 + b1) W2 + b2, and LN(x_out),
+// optionally followed by a tail product LN(x_out) W_t (N = tail_n <= 256).
 // A: attention output planes (64 x 128 boxes, 128-byte swizzle); W_O^T [d, d_pad]
 // and W2^T [d, F_pad] planes with 64 x d boxes; W1^T [F, d_pad] planes with
-// 64 x 128 boxes; outputs through the same store descriptors as the GEMM
-// epilogue.  x0 rows are fp32 [rows, ldx0] (o_x may write the same rows), or
-// one row x0_row added to every row.
+// 64 x 128 boxes; W_t^T [tail_n, d_pad] planes with 64 x tail_n boxes.  o_x:
+// x_out (fp32, 32 x 32 boxes); o_h / o_l: LN(x_out) planes with 64 x 128
+// boxes and the 128-byte swizzle (stored when store_ln); to_h / to_l: the tail
+// output, one f16 plane (tail_f16) or a split pair, 32 x 32 boxes with the
+// 64-byte swizzle.  x0 rows are fp32 [rows, ldx0] (o_x may write the same
+// rows), or one row x0_row added to every row.
 // ---------------------------------------------------------------------------
 struct FfnParams {
   int rows;             // row extent of the A descriptors
@@ -109,15 +113,21 @@ struct FfnParams {
   const float* x0;      // block input rows, unless x0_row is set
   int ldx0;             // multiple of 4
   const float* x0_row;  // [d], when set: the same input row for every row
+  int tail_n;           // 0: no tail product
+  int tail_f16;         // tail output as one f16 plane (else a split pair)
+  int store_ln;         // store LN(x_out)
   float eps;
   int* status;
 };
 bool ffn_supported(int d, int d_pad, int F, int nb);
+bool ffn_tail_supported(int d, int d_pad, int F, int nb, int tail_n, int tail_f16);
 cudaError_t ffn_prepare();
 cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* wo_h,
                        const CUtensorMap* wo_l, const CUtensorMap* w1_h, const CUtensorMap* w1_l,
                        const CUtensorMap* w2_h, const CUtensorMap* w2_l, const CUtensorMap* o_h,
-                       const CUtensorMap* o_l, const CUtensorMap* o_x, const FfnParams& p, cudaStream_t s);
+                       const CUtensorMap* o_l, const CUtensorMap* o_x, const CUtensorMap* t_h,
+                       const CUtensorMap* t_l, const CUtensorMap* to_h, const CUtensorMap* to_l,
+                       const FfnParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Context LayerNorm + K/V projection in one kernel (d <= 128, bf16 inputs,
