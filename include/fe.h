@@ -191,15 +191,18 @@ int fe_evaluate_factorized(fe_ctx* ctx, int B, int C, int M, int K, int L,
 /*
  * Pipelined form of fe_evaluate_host for serving loops whose inputs arrive in
  * host memory.  fe_submit_host enqueues one batch and returns at once: the
- * inputs are copied to one of two library-owned device staging slots on the
- * library's own copy stream, the batch runs on the library's own compute
+ * inputs are copied to one of three library-owned device staging slots on
+ * the library's own copy stream, the batch runs on the library's own compute
  * stream once its copy is complete, and scores/best are copied back into the
  * caller's host buffers.  The copy of one batch therefore overlaps the
- * evaluation of the previous one; every batch still moves its own inputs and
+ * evaluation of the previous ones; every batch still moves its own inputs and
  * results across the host link.  fe_wait_host waits for the oldest
  * outstanding submission and returns its batch status (as fe_evaluate).
- * At most two submissions may be outstanding (a third returns
- * FE_ERR_INVALID_ARG); the host buffers of a submission must stay valid and
+ * At most three submissions may be outstanding (a fourth returns
+ * FE_ERR_INVALID_ARG); with three, a slot's next copy may start as soon as
+ * the batch two submissions back has completed, so the host's wake-up and
+ * submission latency stays off the device's critical path.  The host
+ * buffers of a submission must stay valid and
  * unchanged until its fe_wait_host returns (page-locked buffers for overlap).
  * While submissions are outstanding, fe_evaluate, fe_evaluate_async and
  * fe_evaluate_host return FE_ERR_INVALID_ARG (they share the workspace), and a

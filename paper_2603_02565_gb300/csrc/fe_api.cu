@@ -283,10 +283,11 @@ struct fe_ctx {
   int* host_status = nullptr;  // page-locked
   cudaEvent_t done_ev = nullptr;
   cudaStream_t cap_stream = nullptr;
-  // pipelined host entry: two slots, a copy-in stream and a compute stream
-  HostSlot slots[2];
+  // pipelined host entry: kHostSlots slots, a copy-in stream and a compute stream
+  static constexpr int kHostSlots = 3;
+  HostSlot slots[kHostSlots];
   cudaStream_t copy_stream = nullptr, sub_stream = nullptr;
-  int next_slot = 0;       // slot of the next submission; slots alternate
+  int next_slot = 0;       // slot of the next submission; slots are used in turn
   int n_outstanding = 0;   // submissions not yet waited for (the oldest is next_slot - n_outstanding)
   std::vector<GraphEntry> graphs;
   unsigned long long use_clock = 0;
@@ -903,17 +904,19 @@ int reserve_impl(fe_ctx* c, Shape s) {
     const long long segs = s.C > 0 ? kv_rows / s.C : 1;  // requests, or sequences once factorized
     FE_RC(dalloc((void**)&c->lin_states, (size_t)segs * Ly * c->H * (c->dh * c->dh + c->dh) * sizeof(float)));
   }
-  // pipelined host entry: slot 0 uses the staging above, slot 1 its own copy
+  // pipelined host entry: slot 0 uses the staging above, the others their own copies
   c->slots[0].ctx = c->in_ctx;
   c->slots[0].pool = c->in_pool;
   c->slots[0].idx = c->in_idx;
   c->slots[0].scores = c->out_scores;
   c->slots[0].best = c->out_best;
-  FE_RC(dalloc(&c->slots[1].ctx, (size_t)BC * d * esz));
-  FE_RC(dalloc(&c->slots[1].pool, (size_t)B * (s.M > 0 ? s.M : 1) * d * esz));
-  FE_RC(dalloc((void**)&c->slots[1].idx, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int32_t)));
-  FE_RC(dalloc((void**)&c->slots[1].scores, (size_t)S * sizeof(float)));
-  FE_RC(dalloc((void**)&c->slots[1].best, (size_t)B * sizeof(int32_t)));
+  for (int k = 1; k < fe_ctx::kHostSlots; ++k) {
+    FE_RC(dalloc(&c->slots[k].ctx, (size_t)BC * d * esz));
+    FE_RC(dalloc(&c->slots[k].pool, (size_t)B * (s.M > 0 ? s.M : 1) * d * esz));
+    FE_RC(dalloc((void**)&c->slots[k].idx, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int32_t)));
+    FE_RC(dalloc((void**)&c->slots[k].scores, (size_t)S * sizeof(float)));
+    FE_RC(dalloc((void**)&c->slots[k].best, (size_t)B * sizeof(int32_t)));
+  }
   if (!c->fused_ctxkv) FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->KV, (int)kv_rows, 2 * Ly * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->xln, R, c->dpad, true, c->owned_ws));
@@ -1316,8 +1319,8 @@ int fe_submit_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* con
     g_msg = "null pointer";
     return FE_ERR_INVALID_ARG;
   }
-  if (c->n_outstanding >= 2) {
-    g_msg = "two host submissions are outstanding: call fe_wait_host first";
+  if (c->n_outstanding >= fe_ctx::kHostSlots) {
+    g_msg = "three host submissions are outstanding: call fe_wait_host first";
     return FE_ERR_INVALID_ARG;
   }
   Shape s{B, C, M, K, L};
@@ -1355,7 +1358,7 @@ int fe_submit_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* con
     FE_CK(cudaEventRecord(hs.done_ev, c->sub_stream));
   }
   c->n_outstanding += 1;
-  c->next_slot ^= 1;
+  c->next_slot = (c->next_slot + 1) % fe_ctx::kHostSlots;
   return FE_OK;
 }
 
@@ -1366,8 +1369,8 @@ int fe_wait_host(fe_ctx* c) {
     g_msg = "no host submission outstanding";
     return FE_ERR_INVALID_ARG;
   }
-  // the oldest outstanding submission: slots are used alternately
-  const int k = (c->next_slot + 2 - c->n_outstanding) % 2;
+  // the oldest outstanding submission: slots are used in turn
+  const int k = (c->next_slot + fe_ctx::kHostSlots - c->n_outstanding) % fe_ctx::kHostSlots;
   HostSlot& hs = c->slots[k];
   c->n_outstanding -= 1;
   FE_CK(cudaEventSynchronize(hs.done_ev));

@@ -193,26 +193,29 @@ def test_stress_full_batch_sampled(dev):
 
 
 def test_pipelined_host_entry(dev):
-    """fe_submit_host / fe_wait_host: two different batches in flight give the
+    """fe_submit_host / fe_wait_host: three different batches in flight give the
     same results as the synchronous entry; other calls are refused meanwhile."""
     from paper_2603_02565_gb300.binding import Evaluator, FeError
     w1 = wl.make_workload("serving", B=4)
     w2 = wl.make_workload("serving", B=4, seed=11)
+    w3 = wl.make_workload("serving", B=4, seed=12)
     ev = Evaluator(w1.cfg, w1.weights)
     dt = torch.bfloat16
     host = []
-    for w in (w1, w2):
+    for w in (w1, w2, w3):
         host.append((torch.from_numpy(w.context).to(dt).pin_memory(), torch.from_numpy(w.pool).to(dt).pin_memory(),
                      torch.from_numpy(np.ascontiguousarray(w.cand_idx)).pin_memory()))
     ref = [ev.evaluate_host(*h) for h in host]
-    outs = [(np.full((4, w1.shape[3]), -1.0, np.float32), np.full(4, -7, np.int32)) for _ in range(2)]
+    outs = [(np.full((4, w1.shape[3]), -1.0, np.float32), np.full(4, -7, np.int32)) for _ in range(3)]
     for rep in range(2):
         ev.submit_host(*host[0], *outs[0])
         ev.submit_host(*host[1], *outs[1])
+        ev.submit_host(*host[2], *outs[2])
         with pytest.raises(FeError):
-            ev.submit_host(*host[0], *outs[0])  # a third outstanding submission
+            ev.submit_host(*host[0], *outs[0])  # a fourth outstanding submission
         with pytest.raises(FeError):
             ev.evaluate_host(*host[0])          # the workspace is in use
+        ev.wait_host()
         ev.wait_host()
         ev.wait_host()
         for (s_ref, b_ref), (s, b) in zip(ref, outs):
