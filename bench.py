@@ -126,7 +126,7 @@ def site_work(site, cfg, B, C, M, K, L, R, per_step=None):
         "attn_cross_seq": (4 * B * K * K * d, 3 * S * d * H + S * d * A),
         "gemm_cross_o_ln": (2 * S * d * d, S * d * (A + 8 + A)),
         "gemm_head": (2 * S * d * d * T + 3 * S * d * T, S * d * A + 4 * S * (1 + (T if T > 1 else 0))),
-        "select": (0, 4 * S + 4 * B),
+        "select": (0, 4 * S + 4 * B),  # (fused into gemm_head: the argmax of Eq. 1)
     }
     if site == "ffn_item" and per_step:
         # tails: layers < Ly-1 write the next layer's Q (f16) instead of LN(x_out); the last

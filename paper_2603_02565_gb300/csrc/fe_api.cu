@@ -248,6 +248,12 @@ struct fe_ctx {
   int device = 0;
   int d = 0, H = 0, dh = 0, Ly = 0, F = 0, dpad = 0, Fpad = 0, nb = 1;
   bool fused_ffn = false;  // FFN1 + FFN2 in one kernel (d <= 128)
+  // the argmax fused into the score head: [keys: B_cap x 8 B][NaN flags: B_cap x 4 B][ticket]
+  unsigned long long* sel_keys = nullptr;
+  int* sel_nan = nullptr;
+  unsigned* sel_ticket = nullptr;
+  size_t sel_bytes = 0;
+  bool sel_dirty = false;  // a batch stopped before its score head: clear the words before the next one
   bool tail_q = false;     // the fused FFN of layer l also projects the next layer's Q
   bool tail_kv = false;    // the fused FFN of the last layer also projects [WKs | WVs]
   bool fused_ctxkv = false;  // context LN + K/V projection in one kernel (d <= 128, bf16 inputs)
@@ -548,8 +554,10 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   const int R = B * cap;
   const int S = B * K;
   c->launches_batch = 0;
-  FE_CK(cudaMemsetAsync(c->status, 0, sizeof(int), s));
+  // The status word and the fused argmax's words are zero here: the score
+  // head's last CTA clears them after copying the status to io.hstatus.
   if (K == 0) {
+    FE_CK(cudaMemsetAsync(c->status, 0, sizeof(int), s));
     FE_CK(cudaMemsetAsync(io.best, 0xFF, (size_t)B * sizeof(int32_t), s));
     FE_CK(cudaMemcpyAsync(io.hstatus, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
     return FE_OK;
@@ -808,15 +816,19 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.fuse_b = c->head_vec + 2 * HN + 2 * c->n_tasks;
     p.scores = io.scores;
     p.task_scores = c->task_scores;
+    // (a6) Eq. 1's argmax over each request's K scores, in the same launch
+    p.sel_keys = c->sel_keys;
+    p.sel_nan = c->sel_nan;
+    p.sel_ticket = c->sel_ticket;
+    p.sel_bad = c->bad;
+    p.sel_best = io.best;
+    p.sel_B = B;
+    p.sel_K = K;
+    p.host_status = io.hstatus;
     // LN(C') from the cross-sequence block, or LN(C) = Z without it
     const Planes& hin = c->cfg.no_cross_seq ? c->z : c->lncp;
     FE_RC(gemm(c, "gemm_head", fe::EPI_HEAD, hin, c->w1h, S, nullptr, p, nullptr, nullptr, s));
   }
-  {
-    Prof pf(c, "select", s);
-    FE_CK(fe::select_launch(io.scores, B, K, c->bad, io.best, c->status, s));
-  }
-  FE_CK(cudaMemcpyAsync(io.hstatus, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
   c->launches_last = c->launches_batch;
   return FE_OK;
 }
@@ -888,6 +900,10 @@ int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(dalloc((void**)&c->U, (size_t)B * sizeof(int)));
   FE_RC(dalloc((void**)&c->off, (size_t)(B + 1) * sizeof(int)));
   FE_RC(dalloc((void**)&c->bad, (size_t)B * sizeof(int)));
+  c->sel_bytes = (size_t)B * (sizeof(unsigned long long) + sizeof(int)) + sizeof(unsigned);
+  FE_RC(dalloc((void**)&c->sel_keys, c->sel_bytes));
+  c->sel_nan = reinterpret_cast<int*>(c->sel_keys + B);
+  c->sel_ticket = reinterpret_cast<unsigned*>(c->sel_nan + B);
   FE_RC(dalloc((void**)&c->slot, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int)));
   FE_RC(dalloc((void**)&c->list, (size_t)R * sizeof(int)));
   FE_RC(alloc_f32(c->h, R, d, c->owned_ws));
@@ -951,7 +967,22 @@ bool fits(const fe_ctx* c, const Shape& s) {
   return r.B > 0 && s.B <= r.B && s.C <= r.C && s.M <= r.M && s.K <= r.K && s.L <= r.L && (!s.fact || c->cap_fact);
 }
 
+int launch_batch_impl(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t stream);
+
+// A batch normally ends with its score head clearing the status word and the
+// fused argmax's words; after a launch that stopped early they are cleared here.
 int launch_batch(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t stream) {
+  if (c->sel_dirty && c->sel_keys) {
+    FE_CK(cudaMemsetAsync(c->status, 0, sizeof(int), stream));
+    FE_CK(cudaMemsetAsync(c->sel_keys, 0, c->sel_bytes, stream));
+    c->sel_dirty = false;
+  }
+  const int rc = launch_batch_impl(c, s, io, stream);
+  if (rc != FE_OK) c->sel_dirty = true;
+  return rc;
+}
+
+int launch_batch_impl(fe_ctx* c, const Shape& s, const IoPtrs& io, cudaStream_t stream) {
   if (!fits(c, s)) FE_RC(reserve_impl(c, s));
   c->last_shape = s;
   c->have_last = true;

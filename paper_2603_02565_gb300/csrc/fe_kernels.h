@@ -77,6 +77,22 @@ struct GemmParams {
   const float* fuse_b;  // [1] (n_tasks > 1)
   float* scores;        // [rows]
   float* task_scores;   // [rows, n_tasks] or null
+  // EPI_HEAD with sel_keys: the per-request argmax of Eq. 1 (the best
+  // candidate sequence) fused into the epilogue.  Row s is sequence k = s % sel_K
+  // of request b = s / sel_K; a rejected request (sel_bad[b]) gets NaN scores
+  // and best -1; a NaN score makes best -1 and sets ST_NUMERIC; ties go to the
+  // smaller k.  sel_keys, sel_nan and sel_ticket are zero at launch; the last
+  // CTA to finish writes sel_best.
+  unsigned long long* sel_keys;  // [sel_B] max of (order-preserving score bits << 32 | ~k)
+  int* sel_nan;                  // [sel_B]
+  unsigned* sel_ticket;          // CTAs done
+  const int* sel_bad;            // [sel_B]
+  int32_t* sel_best;             // [sel_B]
+  int sel_B, sel_K;
+  // with sel_keys: the batch status word, copied by the last CTA into this
+  // page-locked host word (device-accessible) once the batch is decided, after
+  // which status, keys, flags and ticket are cleared for the next batch
+  int* host_status;
   int* status;
 };
 
@@ -248,9 +264,6 @@ struct ClsParams {
   float scale;                // 1 / sqrt(d_h)
 };
 cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s);
-// argmax with smallest-index ties; NaN / bad requests -> -1 (+ status bits)
-cudaError_t select_launch(float* scores, int B, int K, const int* bad, int32_t* best, int* status,
-                          cudaStream_t s);
 // weight preparation: out[(row0 + n) * ldo + k] = split(W[k * N + n]) for k < Kin, n < N
 cudaError_t transpose_split_launch(const float* W, int Kin, int N, bf16* out_h, bf16* out_l, int ldo,
                                    int row0, cudaStream_t s);

@@ -490,56 +490,6 @@ cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s) {
 }
 
 // ---------------------------------------------------------------------------
-// Eq. 1 selection: one warp per request; first maximal index; NaN -> -1
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) select_kernel(float* scores, int B, int K, const int* bad, int32_t* best,
-                                                     int* status) {
-  const int lane = threadIdx.x & 31;
-  const int b = blockIdx.x * 8 + (threadIdx.x >> 5);
-  pdl_wait();
-  pdl_trigger();
-  if (b >= B) return;
-  float* sb = scores + (size_t)b * K;
-  if (bad[b]) {
-    for (int k = lane; k < K; k += 32) sb[k] = __int_as_float(0x7fc00000);
-    if (lane == 0) best[b] = -1;
-    return;
-  }
-  float bv = -INFINITY;
-  int bi = INT_MAX;
-  bool nan = false;
-  for (int k = lane; k < K; k += 32) {
-    const float v = sb[k];
-    if (v != v)
-      nan = true;
-    else if (bi == INT_MAX || v > bv) {
-      bv = v;
-      bi = k;
-    }
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-    if (oi != INT_MAX && (bi == INT_MAX || ov > bv || (ov == bv && oi < bi))) {
-      bv = ov;
-      bi = oi;
-    }
-  }
-  nan = __any_sync(0xffffffffu, nan);
-  if (lane == 0) {
-    best[b] = nan ? -1 : bi;
-    if (nan) atomicOr(status, ST_NUMERIC);
-  }
-}
-
-cudaError_t select_launch(float* scores, int B, int K, const int* bad, int32_t* best, int* status,
-                          cudaStream_t s) {
-  if (B <= 0) return cudaSuccess;
-  return launch_k(select_kernel, dim3((unsigned)((B + 7) / 8)), dim3(256), 0, s, scores, B, K, bad, best, status);
-}
-
-// ---------------------------------------------------------------------------
 // init-time weight preparation
 // ---------------------------------------------------------------------------
 __global__ void transpose_split_kernel(const float* __restrict__ W, int Kin, int N, bf16* out_h, bf16* out_l,
