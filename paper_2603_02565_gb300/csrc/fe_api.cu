@@ -230,6 +230,7 @@ struct HostSlot {
   int32_t* best = nullptr;
   int* hstatus = nullptr;      // page-locked
   cudaEvent_t in_ev = nullptr;   // inputs copied in
+  cudaEvent_t run_ev = nullptr;  // batch evaluated (its results may be copied out)
   cudaEvent_t done_ev = nullptr; // batch and copy-out complete (the slot is free again)
 };
 
@@ -292,7 +293,7 @@ struct fe_ctx {
   // pipelined host entry: kHostSlots slots, a copy-in stream and a compute stream
   static constexpr int kHostSlots = 3;
   HostSlot slots[kHostSlots];
-  cudaStream_t copy_stream = nullptr, sub_stream = nullptr;
+  cudaStream_t copy_stream = nullptr, sub_stream = nullptr, out_stream = nullptr;  // host entry: copy-in, batches, copy-out
   int next_slot = 0;       // slot of the next submission; slots are used in turn
   int n_outstanding = 0;   // submissions not yet waited for (the oldest is next_slot - n_outstanding)
   std::vector<GraphEntry> graphs;
@@ -1235,12 +1236,14 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if (cudaEventCreateWithFlags(&c->done_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&c->sub_stream, cudaStreamNonBlocking) != cudaSuccess)
+      cudaStreamCreateWithFlags(&c->sub_stream, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&c->out_stream, cudaStreamNonBlocking) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "stream/event"));
   for (HostSlot& hs : c->slots) {
     if (cudaMallocHost(&hs.hstatus, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
     *hs.hstatus = 0;
     if (cudaEventCreateWithFlags(&hs.in_ev, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&hs.run_ev, cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&hs.done_ev, cudaEventDisableTiming) != cudaSuccess)
       return fail(set_cuda_err(cudaGetLastError(), "stream/event"));
   }
@@ -1378,15 +1381,18 @@ int fe_submit_host(fe_ctx* c, int B, int C, int M, int K, int L, const void* con
       FE_CK(cudaMemcpyAsync(hs.idx, cand_idx, (size_t)B * K * L * sizeof(int32_t), cudaMemcpyHostToDevice,
                             c->copy_stream));
     FE_CK(cudaEventRecord(hs.in_ev, c->copy_stream));
-    // the batch and the copy-out on the compute stream
+    // the batch on the compute stream; its copy-out on a stream of its own, so
+    // that the next batch follows this one on the compute stream at once
     FE_CK(cudaStreamWaitEvent(c->sub_stream, hs.in_ev, 0));
     IoPtrs io{hs.ctx, hs.pool, hs.idx, hs.scores, hs.best, hs.hstatus};
     FE_RC(launch_batch(c, s, io, c->sub_stream));
+    FE_CK(cudaEventRecord(hs.run_ev, c->sub_stream));
+    FE_CK(cudaStreamWaitEvent(c->out_stream, hs.run_ev, 0));
     if (K > 0)
       FE_CK(cudaMemcpyAsync(scores_out, hs.scores, (size_t)B * K * sizeof(float), cudaMemcpyDeviceToHost,
-                            c->sub_stream));
-    FE_CK(cudaMemcpyAsync(best_out, hs.best, (size_t)B * sizeof(int32_t), cudaMemcpyDeviceToHost, c->sub_stream));
-    FE_CK(cudaEventRecord(hs.done_ev, c->sub_stream));
+                            c->out_stream));
+    FE_CK(cudaMemcpyAsync(best_out, hs.best, (size_t)B * sizeof(int32_t), cudaMemcpyDeviceToHost, c->out_stream));
+    FE_CK(cudaEventRecord(hs.done_ev, c->out_stream));
   }
   c->n_outstanding += 1;
   c->next_slot = (c->next_slot + 1) % fe_ctx::kHostSlots;
@@ -1598,11 +1604,13 @@ int fe_destroy(fe_ctx* c) {
     for (HostSlot& hs : c->slots) {
       if (hs.done_ev) cudaEventSynchronize(hs.done_ev);
       if (hs.in_ev) cudaEventDestroy(hs.in_ev);
+      if (hs.run_ev) cudaEventDestroy(hs.run_ev);
       if (hs.done_ev) cudaEventDestroy(hs.done_ev);
       if (hs.hstatus) cudaFreeHost(hs.hstatus);
     }
     if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
     if (c->sub_stream) cudaStreamDestroy(c->sub_stream);
+    if (c->out_stream) cudaStreamDestroy(c->out_stream);
   }
   delete c;
   return FE_OK;
