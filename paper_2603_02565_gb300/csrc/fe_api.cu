@@ -545,6 +545,21 @@ int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const We
     if (rc_ != FE_OK) return rc_; \
   } while (0)
 
+// The fused argmax of Eq. 1 for a batch (fe_select.cuh).
+fe::SelArgs sel_args(fe_ctx* c, int B, int K, const IoPtrs& io) {
+  fe::SelArgs a{};
+  a.keys = c->sel_keys;
+  a.nan = c->sel_nan;
+  a.ticket = c->sel_ticket;
+  a.bad = c->bad;
+  a.best = io.best;
+  a.B = B;
+  a.K = K;
+  a.status = c->status;
+  a.host_status = io.hstatus;
+  return a;
+}
+
 // The whole evaluation of one batch, enqueued on s (captured into a graph by the caller).
 int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) {
   const int B = sh.B, C = sh.C, M = sh.M, K = sh.K, L = sh.L;
@@ -818,14 +833,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     p.scores = io.scores;
     p.task_scores = c->task_scores;
     // (a6) Eq. 1's argmax over each request's K scores, in the same launch
-    p.sel_keys = c->sel_keys;
-    p.sel_nan = c->sel_nan;
-    p.sel_ticket = c->sel_ticket;
-    p.sel_bad = c->bad;
-    p.sel_best = io.best;
-    p.sel_B = B;
-    p.sel_K = K;
-    p.host_status = io.hstatus;
+    p.sel = sel_args(c, B, K, io);
     // LN(C') from the cross-sequence block, or LN(C) = Z without it
     const Planes& hin = c->cfg.no_cross_seq ? c->z : c->lncp;
     FE_RC(gemm(c, "gemm_head", fe::EPI_HEAD, hin, c->w1h, S, nullptr, p, nullptr, nullptr, s));

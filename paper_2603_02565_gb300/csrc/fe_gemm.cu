@@ -17,6 +17,7 @@
 // A_hi W_hi + A_lo W_hi (+ A_hi W_lo when the weights carry a lo plane).
 #include "fe_common.cuh"
 #include "fe_kernels.h"
+#include "fe_select.cuh"
 
 namespace fe {
 
@@ -59,45 +60,6 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
 
 // NB: weight planes (1 when the weights are exact in bf16, else 2); a
 // compile-time constant so that the MMA issue sequence has no branches
-// Order-preserving map of a (non-NaN) float to 32 bits: a > b iff key(a) > key(b).
-__device__ __forceinline__ uint32_t ordered_bits(float f) {
-  const uint32_t u = __float_as_uint(f);
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
-
-// The fused argmax's last step, by the last CTA to finish: best index per
-// request, then the batch status to the host, and every word of the argmax
-// and the status cleared for the next batch.
-static __device__ void select_finish(const GemmParams& p) {
-  __threadfence();
-  for (int b = threadIdx.x; b < p.sel_B; b += blockDim.x) {
-    const unsigned long long key = atomicExch(p.sel_keys + b, 0ull);  // through L2
-    const int nan = atomicExch(p.sel_nan + b, 0);
-    int best = -1;
-    if (!p.sel_bad[b] && !nan && key != 0ull) best = (int)(0xFFFFFFFFu - (uint32_t)(key & 0xFFFFFFFFull));
-    if (!p.sel_bad[b] && nan) atomicOr(p.status, ST_NUMERIC);
-    p.sel_best[b] = best;
-  }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const int st = atomicExch(p.status, 0);
-    *p.sel_ticket = 0u;
-    *reinterpret_cast<volatile int*>(p.host_status) = st;
-    __threadfence_system();
-  }
-}
-
-// Every CTA of a head launch with the fused argmax counts itself done; the
-// last one finishes.  `flag`: a shared word the CTA no longer uses.
-static __device__ void select_ticket(const GemmParams& p, volatile uint32_t* flag) {
-  __threadfence();  // this thread's score atomics before the count
-  __syncthreads();
-  if (threadIdx.x == 0) *flag = atomicAdd(p.sel_ticket, 1u) == gridDim.x - 1 ? 1u : 0u;
-  __syncthreads();
-  if (*flag) select_finish(p);
-}
-
 template <int EPI, int NB>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tA_h, const __grid_constant__ CUtensorMap tA_l,
@@ -156,7 +118,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tiles = ((rows_valid + BM - 1) / BM) * nt;
   if ((int)blockIdx.x >= tiles) {  // nothing for this CTA (uniform)
     if (warp == 0) tmem_dealloc(tmem, ncols);
-    if (EPI == EPI_HEAD && p.sel_keys) select_ticket(p, tmem_slot);  // (the slot is free once deallocated)
+    if (EPI == EPI_HEAD && p.sel.keys) sel_ticket(p.sel, tmem_slot);  // (the slot is free once deallocated)
     return;
   }
 
@@ -509,16 +471,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               }
             }
           }
-          if (p.sel_keys) {  // the argmax over the request's K sequences
-            const int b = grow / p.sel_K, k = grow - b * p.sel_K;
-            if (p.sel_bad[b])
-              f = __int_as_float(0x7fc00000);  // rejected request: NaN scores
-            else if (f != f)
-              atomicOr(p.sel_nan + b, 1);
-            else
-              atomicMax(p.sel_keys + b,
-                        ((unsigned long long)ordered_bits(f) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)k));
-          }
+          if (p.sel.keys) sel_fold(p.sel, grow, f);  // the argmax over the request's K sequences
           p.scores[grow] = f;
         }
       }
@@ -534,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, ncols);
-  if (EPI == EPI_HEAD && p.sel_keys) select_ticket(p, tmem_slot);
+  if (EPI == EPI_HEAD && p.sel.keys) sel_ticket(p.sel, tmem_slot);
 }
 
 template <int EPI, int NB>

@@ -45,6 +45,18 @@ inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
 // B: weights transposed, [N, K_pad], one or two bf16 planes (hi[, lo])
 // Persistent CTAs walk 128 x BN tiles; BN <= 512 (two N=256 MMAs above 256).
 // ---------------------------------------------------------------------------
+// Eq. 1's argmax fused into the kernel that computes the scores (fe_select.cuh).
+struct SelArgs {
+  unsigned long long* keys;  // [B], zero at launch
+  int* nan;                  // [B], zero at launch
+  unsigned* ticket;          // zero at launch
+  const int* bad;            // [B]
+  int32_t* best;             // [B]
+  int B, K;
+  int* status;               // the batch status word
+  int* host_status;          // page-locked host word (device-accessible)
+};
+
 enum GemmEpilogue : int {
   EPI_STORE = 0,    // out = [ReLU](acc + bias) as split planes
   EPI_RESID_LN = 1, // x = resid + acc + bias -> x_out (fp32) and LN(x) as split planes; BN == N
@@ -77,22 +89,8 @@ struct GemmParams {
   const float* fuse_b;  // [1] (n_tasks > 1)
   float* scores;        // [rows]
   float* task_scores;   // [rows, n_tasks] or null
-  // EPI_HEAD with sel_keys: the per-request argmax of Eq. 1 (the best
-  // candidate sequence) fused into the epilogue.  Row s is sequence k = s % sel_K
-  // of request b = s / sel_K; a rejected request (sel_bad[b]) gets NaN scores
-  // and best -1; a NaN score makes best -1 and sets ST_NUMERIC; ties go to the
-  // smaller k.  sel_keys, sel_nan and sel_ticket are zero at launch; the last
-  // CTA to finish writes sel_best.
-  unsigned long long* sel_keys;  // [sel_B] max of (order-preserving score bits << 32 | ~k)
-  int* sel_nan;                  // [sel_B]
-  unsigned* sel_ticket;          // CTAs done
-  const int* sel_bad;            // [sel_B]
-  int32_t* sel_best;             // [sel_B]
-  int sel_B, sel_K;
-  // with sel_keys: the batch status word, copied by the last CTA into this
-  // page-locked host word (device-accessible) once the batch is decided, after
-  // which status, keys, flags and ticket are cleared for the next batch
-  int* host_status;
+  // EPI_HEAD with sel.keys: the argmax of Eq. 1 fused into the epilogue (fe_select.cuh)
+  SelArgs sel;
   int* status;
 };
 
