@@ -455,24 +455,26 @@ __global__ void __launch_bounds__(kThreads, 1)
             tot[t0 + 1] = red_var[r] + red_var[128 + r];
           }
         }
-        if (half == 0 && valid) {
-          float f;
-          if (nt == 1) {
-            f = tot[0] + p.b2[0];
-            if (p.task_scores) p.task_scores[grow] = f;
-          } else {
-            f = p.fuse_b[0];
+        if (half == 0) {  // (uniform per warp: the warps of the first column half write the scores)
+          float f = 0.f;
+          if (valid) {
+            if (nt == 1) {
+              f = tot[0] + p.b2[0];
+              if (p.task_scores) p.task_scores[grow] = f;
+            } else {
+              f = p.fuse_b[0];
 #pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              if (t < nt) {
-                const float st = tot[t] + p.b2[t];
-                if (p.task_scores) p.task_scores[(size_t)grow * nt + t] = st;
-                f = fmaf(p.fuse_w[t], st, f);
+              for (int t = 0; t < 4; ++t) {
+                if (t < nt) {
+                  const float st = tot[t] + p.b2[t];
+                  if (p.task_scores) p.task_scores[(size_t)grow * nt + t] = st;
+                  f = fmaf(p.fuse_w[t], st, f);
+                }
               }
             }
           }
-          if (p.sel.keys) sel_fold(p.sel, grow, f);  // the argmax over the request's K sequences
-          p.scores[grow] = f;
+          if (p.sel.keys) sel_fold_warp(p.sel, grow, f, valid);  // the argmax over the request's K sequences
+          if (valid) p.scores[grow] = f;
         }
       }
       // every TMEM read of this accumulator has completed (tcgen05.wait::ld)

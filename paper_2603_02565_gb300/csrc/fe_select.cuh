@@ -24,16 +24,31 @@ __device__ __forceinline__ uint32_t sel_ordered_bits(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Row `row`'s score f: folded into its request's maximum (NaN for a rejected request).
-__device__ __forceinline__ void sel_fold(const SelArgs& s, int row, float& f) {
-  const int b = row / s.K, k = row - b * s.K;
-  if (s.bad[b])
-    f = __int_as_float(0x7fc00000);
-  else if (f != f)
-    atomicOr(s.nan + b, 1);
-  else
-    atomicMax(s.keys + b,
-              ((unsigned long long)sel_ordered_bits(f) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)k));
+// Row `row`'s score f folded into its request's maximum (NaN for a rejected
+// request), for the 32 rows of a warp (all lanes call it, `valid` per lane):
+// lanes of the same request (contiguous rows) first take their maximum by a
+// segmented shuffle reduction, so that each request sees one atomic per warp.
+__device__ __forceinline__ void sel_fold_warp(const SelArgs& s, int row, float& f, bool valid) {
+  const int lane = threadIdx.x & 31;
+  const int b = valid ? row / s.K : -1;
+  unsigned long long key = 0ull;
+  if (valid) {
+    const int k = row - b * s.K;
+    if (s.bad[b])
+      f = __int_as_float(0x7fc00000);
+    else if (f != f)
+      atomicOr(s.nan + b, 1);
+    else
+      key = ((unsigned long long)sel_ordered_bits(f) << 32) | (unsigned long long)(0xFFFFFFFFu - (uint32_t)k);
+  }
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {  // lane i: maximum over [i, i + 2 off) within its request
+    const unsigned long long ok = __shfl_down_sync(0xffffffffu, key, off);
+    const int ob = __shfl_down_sync(0xffffffffu, b, off);
+    if (lane + off < 32 && ob == b && ok > key) key = ok;
+  }
+  const int pb = __shfl_up_sync(0xffffffffu, b, 1);
+  if (valid && key != 0ull && (lane == 0 || pb != b)) atomicMax(s.keys + b, key);  // the request's first lane
 }
 
 static __device__ void sel_finish(const SelArgs& s) {
