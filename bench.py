@@ -108,6 +108,7 @@ def site_work(site, cfg, B, C, M, K, L, R, per_step=None):
         "gemm_ctx_kv": (2 * n * d * 2 * Ly * d, n * d * A + n * 2 * Ly * d * H),
         "ctx_ln_kv": (2 * n * d * 2 * Ly * d, n * d * esz + n * 2 * Ly * d * H),
         "gather_ln": (0, R * d * (esz + 4 + A)),
+        "embed_q": (2 * R * d * d, R * d * (esz + 4 + H)),  # gather + LN + layer-0 Q: pool row in, h and Q out
         "gemm_item_q": (2 * R * d * d, R * d * A + R * d * H),
         "attn_item_ctx": (4 * R * C * d, R * d * (H + A) + 2 * n * d * H),
         "gemm_item_o_ln": (2 * R * d * d, R * d * (A + 8 + A)),

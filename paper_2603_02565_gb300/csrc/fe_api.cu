@@ -255,6 +255,7 @@ struct fe_ctx {
   unsigned* sel_ticket = nullptr;
   size_t sel_bytes = 0;
   bool sel_dirty = false;  // a batch stopped before its score head: clear the words before the next one
+  bool fused_embed = false;  // gather + LN + the first layer's Q projection in one kernel
   bool tail_q = false;     // the fused FFN of layer l also projects the next layer's Q
   bool tail_kv = false;    // the fused FFN of the last layer also projects [WKs | WVs]
   bool fused_ctxkv = false;  // context LN + K/V projection in one kernel (d <= 128, bf16 inputs)
@@ -627,8 +628,25 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     FE_CK(fe::lin_state_launch(c->KV.h, c->fused_ctxkv ? 1 : 0, c->KV.rows, c->KV.ld, fact ? B * K : B, C, d, c->dh,
                                Ly, c->H, c->lin_states, s));
   }
-  // (a2) distinct elements: gather + LN, then the cross-attention stack
-  {
+  // (a2) distinct elements: gather + LN (+ the first layer's Q), then the cross-attention stack
+  if (c->fused_embed) {
+    fe::EmbedParams ep{};
+    ep.pool = static_cast<const bf16*>(io.pool);
+    ep.B = B;
+    ep.M = M;
+    ep.cap = cap;
+    ep.off = c->off;
+    ep.list = c->list;
+    ep.rows = R;
+    ep.d = d;
+    ep.d_pad = c->dpad;
+    ep.eps = c->cfg.ln_eps;
+    ep.h = c->h.p;
+    ep.ldh = c->h.ld;
+    ep.status = c->status;
+    Prof pf(c, "embed_q", s);
+    FE_CK(fe::embed_q_launch(&c->wq[0].p.th, &c->q.sh, ep, s));
+  } else {
     Prof pf(c, "gather_ln", s);
     FE_CK(fe::gather_ln_launch(io.pool, io_f32, B, M, d, cap, c->off, c->list, R, c->cfg.ln_eps, c->h.p, d, c->xln.h,
                              c->xln.l, c->xln.ld, s));
@@ -666,7 +684,8 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     FE_RC(gemm(c, "gemm_elem_o_ln", fe::EPI_RESID_LN, c->a, c->oe, R, sumU, po, &c->xln, &c->h, s));
   }
   for (int l = 0; l < Ly; ++l) {
-    if (l == 0 || !c->tail_q) {  // (otherwise the previous layer's fused FFN wrote Q)
+    // (otherwise the embedding kernel or the previous layer's fused FFN wrote Q)
+    if ((l == 0 && !c->fused_embed) || (l > 0 && !c->tail_q)) {
       fe::GemmParams p{};
       p.out_f16 = 1;
       FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
@@ -1126,7 +1145,8 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   };
   int rc = FE_OK;
   if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess ||
-      fe::ffn_prepare() != cudaSuccess || fe::ctxkv_prepare() != cudaSuccess || fe::linattn_prepare() != cudaSuccess)
+      fe::ffn_prepare() != cudaSuccess || fe::ctxkv_prepare() != cudaSuccess || fe::linattn_prepare() != cudaSuccess ||
+      fe::embed_q_prepare() != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "kernel attributes"));
   {
     size_t o = 0;
@@ -1176,6 +1196,8 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if ((rc = fill_weight(c->w1s, tw(c, T_W1S), d, F, 0)) != FE_OK) return fail(rc);
   if (c->fused_ffn && (rc = map_fused_w1(c->w1s, c->nb > 1)) != FE_OK) return fail(rc);
   c->tail_q = c->fused_ffn && Ly > 1 && fe::ffn_tail_supported(d, c->dpad, F, c->nb, d, 1);
+  c->fused_embed = fe::embed_q_supported(d, c->dpad, c->nb, cfg->io_dtype == FE_IO_F32 ? 1 : 0) &&
+                   !cfg->elem_self_attn && c->wq[0].N == d && c->wq[0].BN == d;
   c->tail_kv = c->fused_ffn && fe::ffn_tail_supported(d, c->dpad, F, c->nb, 2 * d, 0);
   if (c->tail_q)
     for (int l = 1; l < Ly; ++l)

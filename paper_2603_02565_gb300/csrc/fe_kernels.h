@@ -144,6 +144,29 @@ cudaError_t ffn_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUt
                        const FfnParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
+// Distinct-element gather + LayerNorm + the first layer's Q projection in one
+// kernel (fe_embed.cu), for d <= 128, bf16 pool rows and bf16-exact WQ:
+//   h[r] = pool[b M + list[b cap + r - off[b]]] (fp32), Q[r] = LN(h[r]) WQ (f16)
+// w: WQ^T [d, d_pad] bf16, 64 x d boxes, 128-byte swizzle; q_out: Q's f16
+// store map (32 x 32 boxes, 64-byte swizzle).  Rows past off[B] are not written.
+// ---------------------------------------------------------------------------
+struct EmbedParams {
+  const bf16* pool;     // [B * M, d]
+  int B, M, cap;
+  const int* off;       // [B + 1] row offsets of the requests' distinct elements
+  const int* list;      // [B, cap] the distinct elements' pool rows within their request
+  int rows;             // row extent of h and Q
+  int d, d_pad;
+  float eps;
+  float* h;             // [rows, ldh] fp32
+  int ldh;
+  int* status;
+};
+bool embed_q_supported(int d, int d_pad, int nb, int io_f32);
+cudaError_t embed_q_prepare();
+cudaError_t embed_q_launch(const CUtensorMap* w, const CUtensorMap* q_out, const EmbedParams& p, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
 // Context LayerNorm + K/V projection in one kernel (d <= 128, bf16 inputs,
 // bf16-exact weights, N = 2 * n_layers * d in {256, 512}).
 // x: raw context rows [rows, d] bf16, 64 x 128 boxes, 128-byte swizzle;
