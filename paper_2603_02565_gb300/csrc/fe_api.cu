@@ -581,17 +581,15 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   }
   const int* sumU = c->off + B;  // device: number of distinct elements of the batch
 
-  // (a0) distinct-element compaction of every request (factorized: the identity layout)
+  // (a0) the distinct-element layout of every request: the identity layout
+  // (factorized) and the whole pool here; the compaction after the context
+  // kernel, beside which it runs
   if (fact) {
     Prof pf(c, "layout", s);
     FE_CK(fe::identity_layout_launch(io.idx, B, M, K * L, c->U, c->off, c->bad, c->slot, c->list, c->status, s));
   } else if (c->cfg.encode_pool) {
     Prof pf(c, "pool_layout", s);
     FE_CK(fe::pool_layout_launch(io.idx, B, M, K * L, c->U, c->off, c->bad, c->slot, c->list, c->status, s));
-  } else {
-    Prof pf(c, "compact", s);
-    FE_CK(fe::compact_launch(io.idx, B, M, K, L, cap, c->U, c->off, c->bad, c->slot, c->list, c->status, c->ticket,
-                           s));
   }
   // (a1) context keys/values, once per request
   const bool lin_fused = c->cfg.linear_context_attn && c->fused_ctxkv &&
@@ -619,6 +617,11 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     fe::GemmParams p{};
     p.out_f16 = 1;
     FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_STORE, c->X, c->ctx_kv, B * C, nullptr, p, &c->KV, nullptr, s));
+  }
+  if (!fact && !c->cfg.encode_pool) {
+    Prof pf(c, "compact", s);
+    FE_CK(fe::compact_launch(io.idx, B, M, K, L, cap, c->U, c->off, c->bad, c->slot, c->list, c->status, c->ticket,
+                           s));
   }
   // (a1') linear attention: the context of every request (sequence, once
   // factorized) reduced to its per-layer, per-head states (unless the

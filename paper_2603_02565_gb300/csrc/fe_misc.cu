@@ -144,7 +144,11 @@ __device__ __forceinline__ void warp_layer_norm(float* x, int d, float eps) {
 }  // namespace
 
 // ---------------------------------------------------------------------------
-// distinct-element compaction, one CTA (256 threads) per request
+// distinct-element compaction, one CTA (256 threads) per request.  It reads
+// only the batch's candidate indices and writes only the layout, so it waits
+// for the kernel before it (the context kernel) at its end rather than its
+// start: it runs beside that kernel, and still completes after it, so the
+// kernels after it see both.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) compact_kernel(const int32_t* __restrict__ cand, int B, int M, int K,
                                                       int L, int cap, int* U, int* off, int* bad, int* slot_local,
@@ -158,7 +162,6 @@ __global__ void __launch_bounds__(256) compact_kernel(const int32_t* __restrict_
   const int b = blockIdx.x, tid = threadIdx.x;
   const int n = K * L;
   const int32_t* cb = cand + (size_t)b * n;
-  pdl_wait();
   pdl_trigger();
 
   for (int w = tid; w < W; w += 256) bits[w] = 0u;
@@ -231,6 +234,7 @@ __global__ void __launch_bounds__(256) compact_kernel(const int32_t* __restrict_
       *ticket = 0u;
     }
   }
+  pdl_wait();  // complete no earlier than the kernel before this one
 }
 
 cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int cap, int* U, int* off,
