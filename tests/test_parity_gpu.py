@@ -73,6 +73,17 @@ def test_serving_small_batches(dev, B):
     check_layout(ev, w, o_U, o_sl)
 
 
+@pytest.mark.parametrize("d,H", [(32, 1), (64, 2)])
+def test_serving_narrow(dev, d, H):
+    """Narrow bf16 rows: the fused embedding and FFN kernels with one 64-column
+    k block (d = 32 leaves half of it as zero padding), the FFN tails, and at
+    d = 32 the unfused context path (N = 2 Ly d = 128 < 256)."""
+    w = wl.make_workload("serving", B=5, d=d, H=H)
+    ev, gs, gb = run_gpu(w, dev)
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb)
+    check_layout(ev, w, o_U, o_sl)
+
+
 def context_kv_rows(w, nreq):
     """Oracle [K_0 | V_0 | K_1 | V_1 ...] rows of the first nreq requests."""
     cfg = w.cfg
