@@ -130,6 +130,30 @@ int encode_map_hm(CUtensorMap* m, const void* base, int dh, int rows, int blocks
   return FE_OK;
 }
 
+// f16 rows grouped in segments of seg_rows, [segments][seg_rows][cols]: 3D map
+// with box box_x x box_rows x 1, so that a box reaching past its segment's end
+// reads zeros there (the cross-sequence attention's V).
+int encode_map_seg(CUtensorMap* m, const void* base, int cols, int seg_rows, int segments, int box_x, int box_rows,
+                   CUtensorMapSwizzle sw) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) {
+    g_msg = "cuTensorMapEncodeTiled is unavailable";
+    return FE_ERR_CUDA;
+  }
+  cuuint64_t dims[3] = {(cuuint64_t)cols, (cuuint64_t)seg_rows, (cuuint64_t)segments};
+  cuuint64_t strides[2] = {(cuuint64_t)cols * 2, (cuuint64_t)seg_rows * cols * 2};
+  cuuint32_t box[3] = {(cuuint32_t)box_x, (cuuint32_t)box_rows, 1u};
+  cuuint32_t es[3] = {1u, 1u, 1u};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    g_msg = "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")";
+    return FE_ERR_CUDA;
+  }
+  return FE_OK;
+}
+
 // Operand tiles: 64 bf16 (128 B) x box_rows, 128-byte swizzle.
 int encode_map(CUtensorMap* m, const bf16* base, int cols, int rows, int box_rows) {
   return encode_map_t(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, cols, rows, 64, box_rows,
@@ -832,9 +856,14 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.ldo = c->ax.ld;
     ap.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
     ap.status = c->status;
+    // V as [request][K][3d], so that a key chunk reaching past K reads zeros, not the next request's rows
+    CUtensorMap vseg;
+    FE_RC(encode_map_seg(&vseg, c->qkv.h, c->qkv.ld, K, B, c->dh, c->dh == 32 ? 64 : 128,
+                         c->dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B));
+    ap.kv_seg = 1;
     {
       Prof pf(c, "attn_cross_seq", s);
-      FE_CK(fe::attn_launch(c->dh, &c->qkv.ah, &c->qkv.kh, &c->qkv.kh, ap, s));
+      FE_CK(fe::attn_launch(c->dh, &c->qkv.ah, &c->qkv.kh, &vseg, ap, s));
     }
     fe::GemmParams po{};
     po.resid = c->c.p;

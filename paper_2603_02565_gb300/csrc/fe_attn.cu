@@ -135,6 +135,13 @@ __device__ __forceinline__ void cur_next(const AttnParams& p, int units, Cursor&
 
 }  // namespace
 
+// Zero bytes [o0, end) of a shared-memory tile (one thread, 16-byte stores),
+// then order the writes before this thread's next tensor-core operations.
+__device__ __noinline__ void zero_tail(uint8_t* t, int o0, int end) {
+  for (int o = o0; o < end; o += 16) *reinterpret_cast<uint4*>(t + o) = make_uint4(0u, 0u, 0u, 0u);
+  fence_async_shared();
+}
+
 template <int DH>
 __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM)
     attn_kernel(const __grid_constant__ CUtensorMap tQ, const __grid_constant__ CUtensorMap tK,
@@ -226,7 +233,10 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
             tma_load_3d(kv + Cfg::kKVTile, &tV, 0, row, (p.v_col + c.h * DH) / DH, kv_full + ks);
           } else {
             tma_load_2d(kv, &tK, p.k_col + c.h * DH, row, kv_full + ks);
-            tma_load_2d(kv + Cfg::kKVTile, &tV, p.v_col + c.h * DH, row, kv_full + ks);
+            if (p.kv_seg)  // rows past the segment's kv_cnt keys are outside the map: zeros
+              tma_load_3d(kv + Cfg::kKVTile, &tV, p.v_col + c.h * DH, j * CK, c.b, kv_full + ks);
+            else
+              tma_load_2d(kv + Cfg::kKVTile, &tV, p.v_col + c.h * DH, row, kv_full + ks);
           }
         }
         ++ui;
@@ -240,6 +250,9 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       // softmax finds the next unit's first S ready when it gets there.
       const uint32_t idesc_s = umma_idesc_f16(BQ, CK);
       const uint32_t idesc_pv = umma_idesc_f16(BQ, DH) | (1u << 16);  // B (V) is MN-major
+      // only a variable key count or one that is not a multiple of CK leaves a
+      // partial chunk, whose V rows a segmented map already reads as zeros
+      const bool pad_v = p.kv_self || (p.kv_cnt % CK != 0 && !p.kv_seg);
       Cursor sc;             // unit of the next S
       int sj = 0, sui = 0;   // its chunk and its unit counter (Q buffer sui % 2)
       int g_s = 0;           // S products issued
@@ -264,6 +277,13 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         for (int kk = 0; kk < DH / 16; ++kk)
           umma_bf16(dst, desc_adv(q0d, kk * 32), desc_adv(k0d, kk * 32), idesc_s, kk != 0 ? 1u : 0u);
         umma_commit(s_full + t);
+        // The V rows of a partial chunk past the key count belong to the next
+        // segment: their P is 0, but 0 x NaN is NaN, so they are zeroed here
+        // (the chunk has landed; PV_{g_s}, issued later by this thread, reads them)
+        if (pad_v) {
+          const int kval = kv_count(sc) - sj * CK;
+          if (kval < CK) zero_tail(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile, kval * (int)Cfg::kRowBytes, (int)Cfg::kKVTile);
+        }
         ++g_s;
         if (++sj == chunks(sc)) {  // every S of this unit issued: its Q buffer frees on completion
           umma_commit(q_empty + qb);

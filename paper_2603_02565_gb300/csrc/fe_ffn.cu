@@ -31,6 +31,14 @@
 
 namespace fe {
 
+// ReLU that keeps a NaN (max.NaN): a NaN activation reaches the score, and so
+// the argmax's NaN flag, instead of becoming 0 as with fmaxf.
+__device__ __forceinline__ float relu_nan(float x) {
+  float r;
+  asm("max.NaN.f32 %0, %1, 0f00000000;" : "=f"(r) : "f"(x));
+  return r;
+}
+
 namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;
@@ -506,7 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const float2 bb = *reinterpret_cast<const float2*>(bias + 2 * j);
-            split2_trunc(fmaxf(v[2 * j] + bb.x, 0.f), fmaxf(v[2 * j + 1] + bb.y, 0.f), hi[j], lo[j]);
+            split2_trunc(relu_nan(v[2 * j] + bb.x), relu_nan(v[2 * j + 1] + bb.y), hi[j], lo[j]);
           }
           tmem_st16_nowait(col, hi);
           tmem_st16_nowait(col + 16, lo);

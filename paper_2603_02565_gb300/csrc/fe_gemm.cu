@@ -21,6 +21,14 @@
 
 namespace fe {
 
+// ReLU that keeps a NaN (max.NaN): a NaN activation reaches the score, and so
+// the argmax's NaN flag, instead of becoming 0 as with fmaxf.
+__device__ __forceinline__ float relu_nan(float x) {
+  float r;
+  asm("max.NaN.f32 %0, %1, 0f00000000;" : "=f"(r) : "f"(x));
+  return r;
+}
+
 namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;                               // one 128-byte swizzle row of bf16
@@ -279,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (p.relu) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = fmaxf(v[i], 0.f);
+            for (int i = 0; i < 32; ++i) v[i] = relu_nan(v[i]);
           }
           if (p.out_f16) {
             // one f16 plane (an attention operand)
@@ -434,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           float a = 0.f;
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const float x = fmaxf(v[i] + p.bias[c + i], 0.f);
+            const float x = relu_nan(v[i] + p.bias[c + i]);
             a = fmaf(x, p.w2[c + i], a);
           }
           const int t = c / p.head_d;

@@ -217,6 +217,7 @@ struct AttnParams {
   int q_col, k_col, v_col, o_col;
   int kv3d;              // K/V head-major (3D maps: x within the head, row, block = column / dh)
   int kv_self;           // keys / values are the segment's query rows (kv_stride, kv_cnt unused)
+  int kv_seg;            // V through a 3D map [segment][kv_cnt][col]: rows past kv_cnt read as zeros
   bf16 *o_h, *o_l;
   int ldo;
   float scale_log2;      // log2(e) / sqrt(d_h)

@@ -295,6 +295,22 @@ def test_bad_index_isolates_request():
     np.testing.assert_allclose(s[0], O.evaluate(ctx, pool, cand, W, cfg)[0][0], rtol=1e-13)
 
 
+def test_nan_input_isolates_request():
+    """A NaN in one request's pool row or context row: that request's scores are
+    NaN (the cross-sequence attention mixes every candidate) and Eq. 1 selects
+    nothing (-1); the other request is untouched."""
+    cfg, W, ctx, pool, cand = micro_case(23, K=3, L=2, M=5)
+    for where in ("pool", "context"):
+        ctx2, pool2, cand2 = (np.concatenate([a, a]) for a in (ctx, pool, cand))
+        if where == "pool":
+            pool2[1, cand2[1, 0, 0], 0] = np.nan
+        else:
+            ctx2[1, 0, 0] = np.nan
+        s, best, U, slots = O.evaluate(ctx2, pool2, cand2, W, cfg)
+        assert np.isnan(s[1]).all() and best[1] == -1 and U[1] == U[0]
+        np.testing.assert_allclose(s[0], O.evaluate(ctx, pool, cand, W, cfg)[0][0], rtol=1e-13)
+
+
 # -- the whole evaluator against stock torch.nn layers -----------------------------
 
 @pytest.mark.parametrize("seed", range(40))

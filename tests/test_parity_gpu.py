@@ -160,6 +160,39 @@ def test_bad_index_isolated(dev):
     check(w, gs, gb, requests=[0, 1])
 
 
+def test_nan_request_isolated(dev):
+    """A NaN input value leaves Eq. 1 without a maximum for its request: that
+    request's scores are NaN and its best index -1 (FE_ERR_NUMERIC, the NaN
+    flags of the fused argmax), the other requests are unaffected, and the next
+    batch starts clean, through the device entry and the pipelined host entry."""
+    from paper_2603_02565_gb300 import binding
+    w = wl.make_workload("serving", B=4)
+    clean = wl.make_workload("serving", B=4)   # the same weights and inputs, without the NaNs
+    w.pool, w.context = w.pool.copy(), w.context.copy()
+    w.pool[1, int(w.cand_idx[1, 0, 0]), 3] = np.nan   # one element of request 1
+    w.context[3, 5, 0] = np.nan                        # one context row of request 3
+    ev, gs, gb = run_gpu(w, dev)
+    for b in (1, 3):
+        assert np.isnan(gs[b]).all() and gb[b] == -1
+    assert ev.last_status == binding.FE_ERR_NUMERIC
+    check(w, gs, gb, requests=[0, 2])
+    _, cs, cb = run_gpu(clean, dev, ev)
+    assert ev.last_status == binding.FE_OK
+    check(clean, cs, cb)
+    dt = torch.bfloat16
+    host = [(torch.from_numpy(x.context).to(dt).pin_memory(), torch.from_numpy(x.pool).to(dt).pin_memory(),
+             torch.from_numpy(np.ascontiguousarray(x.cand_idx)).pin_memory()) for x in (w, clean)]
+    outs = [(np.zeros((4, w.shape[3]), np.float32), np.zeros(4, np.int32)) for _ in range(2)]
+    ev.submit_host(*host[0], *outs[0])
+    ev.submit_host(*host[1], *outs[1])
+    assert ev.wait_host() == binding.FE_ERR_NUMERIC
+    assert ev.wait_host() == binding.FE_OK
+    np.testing.assert_array_equal(outs[0][0], gs)
+    np.testing.assert_array_equal(outs[0][1], gb)
+    np.testing.assert_array_equal(outs[1][0], cs)
+    np.testing.assert_array_equal(outs[1][1], cb)
+
+
 def test_edge_shapes(dev):
     """K = 1, L = 1, M = 1, and a sequence repeating one element."""
     for kw in [dict(K=1), dict(L=1), dict(M=1, L=1, K=3), dict(K=2, L=3, M=3)]:
