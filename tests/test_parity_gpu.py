@@ -193,6 +193,26 @@ def test_nan_request_isolated(dev):
     np.testing.assert_array_equal(outs[1][1], cb)
 
 
+@pytest.mark.parametrize("kw,where", [
+    (dict(B=3, C=100), "context"),
+    (dict(B=3, C=128, M=60, K=20, L=5, elem_self_attn=True, encode_pool=True, seed=32), "pool")])
+def test_nan_isolated_across_partial_chunks(dev, kw, where):
+    """Request 0's last key chunk reaches into request 1's rows: context rows
+    100-127 of a 100-row context, element rows 60-63 of the element
+    self-attention over 60 elements. A NaN there stays in request 1."""
+    from paper_2603_02565_gb300 import binding
+    w = wl.make_workload("serving", **kw)
+    w.pool, w.context = w.pool.copy(), w.context.copy()
+    if where == "context":
+        w.context[1, 3, 0] = np.nan   # key row 103 of request 0's second chunk
+    else:
+        w.pool[1, 2, 0] = np.nan      # element row 62 of request 0's only chunk
+    ev, gs, gb = run_gpu(w, dev)
+    assert np.isnan(gs[1]).all() and gb[1] == -1
+    assert ev.last_status == binding.FE_ERR_NUMERIC
+    check(w, gs, gb, requests=[0, 2])
+
+
 def test_edge_shapes(dev):
     """K = 1, L = 1, M = 1, and a sequence repeating one element."""
     for kw in [dict(K=1), dict(L=1), dict(M=1, L=1, K=3), dict(K=2, L=3, M=3)]:
