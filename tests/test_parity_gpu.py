@@ -213,6 +213,22 @@ def test_nan_isolated_across_partial_chunks(dev, kw, where):
     check(w, gs, gb, requests=[0, 2])
 
 
+def test_empty_batches(dev):
+    """K = 0 leaves Eq. 1 without candidates: best -1 for every request with
+    status FE_OK, as in the oracle; B = 0 does nothing; a normal batch on the
+    same context afterwards is unaffected."""
+    from paper_2603_02565_gb300 import binding
+    w = wl.make_workload("serving", B=3, K=0)
+    ev, gs, gb = run_gpu(w, dev)
+    assert gs.shape == (3, 0) and ev.last_status == binding.FE_OK
+    np.testing.assert_array_equal(gb, O.evaluate(w.context, w.pool, w.cand_idx, w.weights, w.cfg)[1])
+    _, gs0, gb0 = run_gpu(wl.make_workload("serving", B=0), dev, ev)
+    assert gs0.shape == (0, 50) and gb0.shape == (0,) and ev.last_status == binding.FE_OK
+    w1 = wl.make_workload("serving", B=2)
+    _, gs1, gb1 = run_gpu(w1, dev, ev)
+    check(w1, gs1, gb1)
+
+
 def test_edge_shapes(dev):
     """K = 1, L = 1, M = 1, and a sequence repeating one element."""
     for kw in [dict(K=1), dict(L=1), dict(M=1, L=1, K=3), dict(K=2, L=3, M=3)]:
