@@ -119,6 +119,30 @@ size_t fe_weight_count(const fe_config* cfg);
 int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx** out);
 
 /*
+ * Weight blob: the parameters theta of the evaluator E_theta (Section 3)
+ * together with their configuration, as one self-describing buffer (a file
+ * on disk, for example).  The paper defines no storage format; this one is
+ * the library's.  Layout, every field little-endian:
+ *   bytes  0..3    magic "FEW1"
+ *   bytes  4..7    uint32 version, 1
+ *   bytes  8..55   the twelve fe_config fields in declaration order, 4 bytes
+ *                  each (int32, except ln_eps: IEEE-754 float32)
+ *   bytes 56..63   uint64 n = fe_weight_count(config)
+ *   bytes 64..     n float32 weights in the order fe_weight_count documents
+ * fe_blob_parse checks a blob on the host (no CUDA call): magic, version,
+ * configuration, n and the total size, which must be exactly 64 + 4 n bytes.
+ * On success it writes the configuration to *cfg_out and n to *n_floats_out
+ * (when not NULL).  Errors: FE_ERR_INVALID_ARG (null pointer, wrong magic,
+ * n or size), FE_ERR_UNSUPPORTED (a version other than 1, or a configuration
+ * that fe_init refuses).
+ * fe_init_blob is fe_blob_parse followed by fe_init with the blob's weights;
+ * the blob stays caller-owned and may be freed when the call returns.  Same
+ * errors as both.
+ */
+int fe_blob_parse(const void* blob, size_t bytes, fe_config* cfg_out, size_t* n_floats_out);
+int fe_init_blob(const void* blob, size_t bytes, fe_ctx** out);
+
+/*
  * Size the device workspace for batches up to (B, C, M, K, L) and build the
  * TMA descriptors for it.  Optional: fe_evaluate grows the workspace itself
  * when a call exceeds the reserved shape (that call then allocates).
@@ -292,6 +316,33 @@ int fe_kernels_per_batch(fe_ctx* ctx);
  */
 int fe_distinct_layout_noalloc(const int32_t* cand_idx, int B, int M, int K, int L,
                                int32_t* U_out, int32_t* slot_out, void* stream);
+
+/*
+ * Test hook for the allocation-failure path (no counterpart in the paper).
+ * fail_at > 0 makes the fail_at-th device or page-locked allocation that the
+ * library makes from now on fail as if the device were out of memory: the
+ * entry point making it returns FE_ERR_OOM after releasing what it had
+ * allocated (fe_init leaves no context; a failed workspace grow leaves the
+ * context with no workspace, and its next call reserves again).  0 disarms
+ * the hook; a negative value leaves it as it is.  *live_out, when not NULL,
+ * receives the number of the library's allocations that are live, over all
+ * contexts.  The setting is process-wide; host only; returns FE_OK.
+ */
+int fe_debug_alloc_hook(int fail_at, int64_t* live_out);
+
+/*
+ * Test hook for the bounded device-side waits (no counterpart in the paper).
+ * Enqueues on `stream` one thread that waits, through the batch kernels' own
+ * bounded mbarrier wait, on a barrier that nothing arrives on, with a limit of
+ * limit_us microseconds (1..1000000) instead of the batch kernels' one
+ * second; no copy or tensor-core work is in flight.  The status word then
+ * reaches the host as a batch's does (copied to the page-locked word and
+ * cleared), so the call waits and returns FE_ERR_TIMEOUT; the context stays
+ * usable for the next batch.  Reserves a minimal workspace when the context
+ * has none.  Errors: FE_ERR_INVALID_ARG (null context, limit out of range,
+ * host submissions outstanding), FE_ERR_CUDA.
+ */
+int fe_debug_wait_probe(fe_ctx* ctx, uint32_t limit_us, void* stream);
 
 /* Release every device resource owned by ctx (waits for its work first). */
 int fe_destroy(fe_ctx* ctx);

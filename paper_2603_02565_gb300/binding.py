@@ -32,7 +32,8 @@ EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evalua
            "fe_debug_fetch", "fe_profile",
            "fe_profile_read",
            "fe_kernels_per_batch", "fe_distinct_layout_noalloc", "fe_destroy", "fe_strerror",
-           "fe_last_error_message"]
+           "fe_last_error_message", "fe_blob_parse", "fe_init_blob", "fe_debug_alloc_hook",
+           "fe_debug_wait_probe"]
 
 
 class FeConfig(ctypes.Structure):
@@ -65,6 +66,14 @@ def load_library(path: str = LIB_PATH):
     L.fe_weight_count.restype = sz
     L.fe_init.argtypes = [ctypes.POINTER(FeConfig), ctypes.POINTER(ctypes.c_float), sz, ctypes.POINTER(vp)]
     L.fe_init.restype = i32
+    L.fe_blob_parse.argtypes = [vp, sz, ctypes.POINTER(FeConfig), ctypes.POINTER(sz)]
+    L.fe_blob_parse.restype = i32
+    L.fe_init_blob.argtypes = [vp, sz, ctypes.POINTER(vp)]
+    L.fe_init_blob.restype = i32
+    L.fe_debug_alloc_hook.argtypes = [i32, ctypes.POINTER(ctypes.c_int64)]
+    L.fe_debug_alloc_hook.restype = i32
+    L.fe_debug_wait_probe.argtypes = [vp, ctypes.c_uint32, vp]
+    L.fe_debug_wait_probe.restype = i32
     L.fe_reserve.argtypes = [vp, i32, i32, i32, i32, i32]
     L.fe_reserve.restype = i32
     for name in ("fe_evaluate", "fe_evaluate_async", "fe_evaluate_host", "fe_evaluate_factorized"):
@@ -151,12 +160,74 @@ def pack_weights(cfg, weights: dict) -> np.ndarray:
     return np.concatenate(parts)
 
 
+BLOB_MAGIC = b"FEW1"
+BLOB_VERSION = 1
+
+
+def weights_blob(cfg, weights: dict) -> bytes:
+    """The weight blob of fe.h (magic, version, the fe_config fields, the
+    weight count, then the fp32 weights in fe_init's order), little-endian."""
+    import struct
+    c = make_config(cfg)
+    flat = pack_weights(cfg, weights).astype("<f4", copy=False)
+    head = BLOB_MAGIC + struct.pack("<I", BLOB_VERSION)
+    head += struct.pack("<6if5i", c.d, c.n_heads, c.n_layers, c.ffn_mult, c.max_L, c.io_dtype, c.ln_eps, c.n_tasks,
+                        c.no_cross_seq, c.elem_self_attn, c.encode_pool, c.linear_context_attn)
+    head += struct.pack("<Q", flat.size)
+    return head + flat.tobytes()
+
+
+def save_blob(path: str, cfg, weights: dict) -> None:
+    with open(path, "wb") as f:
+        f.write(weights_blob(cfg, weights))
+
+
+class BlobConfig:
+    """The configuration read from a weight blob by fe_blob_parse, with the
+    attribute names the rest of this module uses."""
+
+    def __init__(self, c: FeConfig):
+        self.d, self.n_heads, self.n_layers = c.d, c.n_heads, c.n_layers
+        self.ffn_mult, self.max_L, self.ln_eps = c.ffn_mult, c.max_L, c.ln_eps
+        self.io_bf16 = c.io_dtype == FE_IO_BF16
+        self.n_tasks = max(c.n_tasks, 1)
+        self.cross_seq = c.no_cross_seq == 0
+        self.elem_self_attn = bool(c.elem_self_attn)
+        self.encode_pool = bool(c.encode_pool)
+        self.linear_context_attn = bool(c.linear_context_attn)
+        self.F = c.ffn_mult * c.d
+
+
+def parse_blob(blob: bytes):
+    """(BlobConfig, weight count) of a blob, checked by the library's parser."""
+    L = load_library()
+    c = FeConfig()
+    n = ctypes.c_size_t()
+    buf = ctypes.create_string_buffer(bytes(blob), len(blob))
+    _check(L.fe_blob_parse(buf, len(blob), ctypes.byref(c), ctypes.byref(n)))
+    return BlobConfig(c), n.value
+
+
 def _ptr(t):
     return ctypes.c_void_p(0 if t is None else t.data_ptr())
 
 
 class Evaluator:
     """One library context: weights on the device plus a reusable workspace."""
+
+    @classmethod
+    def from_blob(cls, blob: bytes):
+        """A context from a weight blob (fe_init_blob); the configuration is the blob's."""
+        L = load_library()
+        cfg, _ = parse_blob(blob)
+        self = cls.__new__(cls)
+        self.cfg = cfg
+        buf = ctypes.create_string_buffer(bytes(blob), len(blob))
+        h = ctypes.c_void_p()
+        _check(L.fe_init_blob(buf, len(blob), ctypes.byref(h)))
+        self._h = h
+        self.last_status = FE_OK
+        return self
 
     def __init__(self, cfg, weights: dict):
         L = load_library()

@@ -1,6 +1,7 @@
 // C-ABI of the joint evaluator: weights, workspace, TMA descriptors, the
 // launch sequence of one evaluation and its CUDA-graph cache.
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <limits>
 #include <cstdio>
@@ -21,6 +22,54 @@ thread_local std::string g_msg;
 int set_cuda_err(cudaError_t e, const char* what) {
   g_msg = std::string(what) + ": " + cudaGetErrorString(e);
   return FE_ERR_CUDA;
+}
+
+// Every device and page-locked allocation of the library goes through
+// dev_alloc / host_alloc: they count the live allocations and, for tests
+// (fe_debug_alloc_hook), can make a chosen allocation fail as if the device
+// were out of memory.
+std::atomic<long long> g_live_allocs{0};
+std::atomic<int> g_fail_countdown{0};  // > 0: the allocation that takes it to 0 fails
+
+bool injected_failure() {
+  int n = g_fail_countdown.load();
+  while (n > 0)
+    if (g_fail_countdown.compare_exchange_weak(n, n - 1)) return n == 1;
+  return false;
+}
+
+cudaError_t dev_alloc(void** p, size_t bytes) {
+  *p = nullptr;
+  if (injected_failure()) return cudaErrorMemoryAllocation;
+  const cudaError_t e = cudaMalloc(p, bytes);
+  if (e == cudaSuccess) {
+    ++g_live_allocs;
+  } else {
+    *p = nullptr;
+    cudaGetLastError();  // an allocation failure must not surface as a later call's CUDA error
+  }
+  return e;
+}
+
+void dev_free(void* p) {
+  if (p && cudaFree(p) == cudaSuccess) --g_live_allocs;
+}
+
+cudaError_t host_alloc(void** p, size_t bytes) {
+  *p = nullptr;
+  if (injected_failure()) return cudaErrorMemoryAllocation;
+  const cudaError_t e = cudaMallocHost(p, bytes);
+  if (e == cudaSuccess) {
+    ++g_live_allocs;
+  } else {
+    *p = nullptr;
+    cudaGetLastError();
+  }
+  return e;
+}
+
+void host_free(void* p) {
+  if (p && cudaFreeHost(p) == cudaSuccess) --g_live_allocs;
 }
 
 #define FE_CK(call)                                                     \
@@ -77,11 +126,11 @@ int alloc_planes(Planes& p, int rows, int ld, bool two, std::vector<void*>& owne
   p.rows = rows < 128 ? 128 : rows;  // TMA boxes of 128 rows stay inside every allocation
   p.ld = ld;
   const size_t bytes = (size_t)p.rows * ld * sizeof(bf16);
-  if (cudaMalloc(&p.h, bytes) != cudaSuccess) return FE_ERR_OOM;
+  if (dev_alloc((void**)&p.h, bytes) != cudaSuccess) return FE_ERR_OOM;
   owned.push_back(p.h);
   FE_CK(cudaMemset(p.h, 0, bytes));
   if (two) {
-    if (cudaMalloc(&p.l, bytes) != cudaSuccess) return FE_ERR_OOM;
+    if (dev_alloc((void**)&p.l, bytes) != cudaSuccess) return FE_ERR_OOM;
     owned.push_back(p.l);
     FE_CK(cudaMemset(p.l, 0, bytes));
   }
@@ -204,7 +253,7 @@ int alloc_f32(F32Rows& f, int rows, int ld, std::vector<void*>& owned) {
   f.rows = rows < 128 ? 128 : rows;
   f.ld = ld;
   const size_t bytes = (size_t)f.rows * ld * sizeof(float);
-  if (cudaMalloc(&f.p, bytes) != cudaSuccess) return FE_ERR_OOM;
+  if (dev_alloc((void**)&f.p, bytes) != cudaSuccess) return FE_ERR_OOM;
   owned.push_back(f.p);
   FE_CK(cudaMemset(f.p, 0, bytes));
   return encode_map_t(&f.sx, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, f.p, ld, f.rows, 32, 32, CU_TENSOR_MAP_SWIZZLE_128B);
@@ -504,7 +553,7 @@ int fill_weight(Weight& w, const float* W, int Kin, int N, int row0) {
 }
 
 void free_list(std::vector<void*>& v) {
-  for (void* p : v) cudaFree(p);
+  for (void* p : v) dev_free(p);
   v.clear();
 }
 
@@ -917,6 +966,13 @@ int check_shape(const fe_ctx* c, int B, int C, int M, int K, int L) {
   return FE_OK;
 }
 
+int reserve_body(fe_ctx* c, const Shape& s, bool fact);
+
+// Sizes the workspace for shape s (growing monotonically).  Shapes outside
+// the limits are refused before anything changes.  Otherwise the old
+// workspace is released first; when an allocation of the new one fails,
+// whatever was allocated is released too and the reservation is left empty,
+// so the context holds no stale buffer and the next call reserves again.
 int reserve_impl(fe_ctx* c, Shape s) {
   FE_RC(check_shape(c, s.B, s.C, s.M, s.K, s.L));
   // grow monotonically
@@ -930,6 +986,23 @@ int reserve_impl(fe_ctx* c, Shape s) {
     g_msg = "batch too large for the factorized evaluation";
     return FE_ERR_UNSUPPORTED;
   }
+  const int rc = reserve_body(c, s, fact);
+  if (rc != FE_OK) {
+    cudaDeviceSynchronize();
+    free_list(c->owned_ws);
+    c->cap_shape = Shape{};
+    c->cap_rows = 0;
+    c->cap_fact = false;
+    c->kv_rows = 0;
+    c->have_last = false;
+    c->status = nullptr;  // the next reservation allocates these zeroed
+    c->sel_keys = nullptr;
+    c->sel_dirty = false;
+  }
+  return rc;
+}
+
+int reserve_body(fe_ctx* c, const Shape& s, const bool fact) {
   FE_CK(cudaDeviceSynchronize());
   clear_graphs(c);
   free_list(c->owned_ws);
@@ -947,7 +1020,7 @@ int reserve_impl(fe_ctx* c, Shape s) {
   const long long kv_rows = (long long)BC * (fact && s.K > 0 ? s.K : 1);
   auto dalloc = [&](void** p, size_t bytes) -> int {
     if (bytes == 0) bytes = 16;
-    if (cudaMalloc(p, bytes) != cudaSuccess) {
+    if (dev_alloc(p, bytes) != cudaSuccess) {
       g_msg = "cudaMalloc of " + std::to_string(bytes) + " bytes failed";
       return FE_ERR_OOM;
     }
@@ -1187,7 +1260,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
       o += s;
     }
   }
-  if (cudaMalloc(&c->w32, n_floats * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+  if (dev_alloc((void**)&c->w32, n_floats * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
   c->owned_w.push_back(c->w32);
   if (cudaMemcpy(c->w32, weights, n_floats * sizeof(float), cudaMemcpyHostToDevice) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "weight copy"));
@@ -1262,7 +1335,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     if ((rc = fill_weight(c->w1h, hw(c, t, 0), d, d, t * d)) != FE_OK) return fail(rc);
   {
     const size_t nv = 2 * (size_t)HN + 2 * T + 1;
-    if (cudaMalloc(&c->head_vec, nv * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+    if (dev_alloc((void**)&c->head_vec, nv * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
     c->owned_w.push_back(c->head_vec);
     FE_CK(cudaMemset(c->head_vec, 0, nv * sizeof(float)));
     for (int t = 0; t < T; ++t) {
@@ -1280,7 +1353,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   // weight-only products of SeqEnc: [CLS] W and P W
   const int mL = cfg->max_L;
   float* consts = nullptr;
-  if (cudaMalloc(&consts, (size_t)(3 + 2 * mL) * d * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+  if (dev_alloc((void**)&consts, (size_t)(3 + 2 * mL) * d * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
   c->owned_w.push_back(consts);
   c->q0 = consts;
   c->k0 = consts + d;
@@ -1293,7 +1366,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
       fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WKS), d, c->kP, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WVS), d, c->vP, 0) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "SeqEnc constants"));
-  if (cudaMallocHost(&c->host_status, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
+  if (host_alloc((void**)&c->host_status, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
   *c->host_status = 0;
   if (cudaEventCreateWithFlags(&c->done_ev, cudaEventDisableTiming) != cudaSuccess ||
       cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking) != cudaSuccess ||
@@ -1302,7 +1375,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
       cudaStreamCreateWithFlags(&c->out_stream, cudaStreamNonBlocking) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "stream/event"));
   for (HostSlot& hs : c->slots) {
-    if (cudaMallocHost(&hs.hstatus, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
+    if (host_alloc((void**)&hs.hstatus, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
     *hs.hstatus = 0;
     if (cudaEventCreateWithFlags(&hs.in_ev, cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&hs.run_ev, cudaEventDisableTiming) != cudaSuccess ||
@@ -1313,6 +1386,116 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   if (e != cudaSuccess) return fail(set_cuda_err(e, "fe_init"));
   *out = c;
   return FE_OK;
+}
+
+namespace {
+
+constexpr size_t kBlobHeader = 64;
+
+uint32_t rd_u32(const unsigned char* p) {
+  return (uint32_t)p[0] | ((uint32_t)p[1] << 8) | ((uint32_t)p[2] << 16) | ((uint32_t)p[3] << 24);
+}
+
+int32_t rd_i32(const unsigned char* p) {
+  const uint32_t u = rd_u32(p);
+  int32_t v;
+  std::memcpy(&v, &u, 4);
+  return v;
+}
+
+}  // namespace
+
+int fe_blob_parse(const void* blob, size_t bytes, fe_config* cfg_out, size_t* n_floats_out) {
+  if (!blob || !cfg_out) {
+    g_msg = "null argument";
+    return FE_ERR_INVALID_ARG;
+  }
+  const unsigned char* b = static_cast<const unsigned char*>(blob);
+  if (bytes < kBlobHeader) {
+    g_msg = "blob shorter than its 64-byte header";
+    return FE_ERR_INVALID_ARG;
+  }
+  if (std::memcmp(b, "FEW1", 4) != 0) {
+    g_msg = "not a weight blob (magic is not FEW1)";
+    return FE_ERR_INVALID_ARG;
+  }
+  const uint32_t version = rd_u32(b + 4);
+  if (version != 1) {
+    g_msg = "weight blob version " + std::to_string(version) + " (this library reads version 1)";
+    return FE_ERR_UNSUPPORTED;
+  }
+  fe_config c{};
+  c.d = rd_i32(b + 8);
+  c.n_heads = rd_i32(b + 12);
+  c.n_layers = rd_i32(b + 16);
+  c.ffn_mult = rd_i32(b + 20);
+  c.max_L = rd_i32(b + 24);
+  c.io_dtype = rd_i32(b + 28);
+  const uint32_t eps_bits = rd_u32(b + 32);
+  std::memcpy(&c.ln_eps, &eps_bits, 4);
+  c.n_tasks = rd_i32(b + 36);
+  c.no_cross_seq = rd_i32(b + 40);
+  c.elem_self_attn = rd_i32(b + 44);
+  c.encode_pool = rd_i32(b + 48);
+  c.linear_context_attn = rd_i32(b + 52);
+  const uint64_t n = (uint64_t)rd_u32(b + 56) | ((uint64_t)rd_u32(b + 60) << 32);
+  if (!config_ok(&c)) {
+    g_msg = "the blob's configuration is not supported";
+    return FE_ERR_UNSUPPORTED;
+  }
+  const size_t need = fe_weight_count(&c);
+  if (n != need) {
+    g_msg = "the blob holds " + std::to_string(n) + " weights, its configuration needs " + std::to_string(need);
+    return FE_ERR_INVALID_ARG;
+  }
+  if (bytes != kBlobHeader + 4 * need) {
+    g_msg = "blob size " + std::to_string(bytes) + " != 64 + 4 * " + std::to_string(need);
+    return FE_ERR_INVALID_ARG;
+  }
+  *cfg_out = c;
+  if (n_floats_out) *n_floats_out = need;
+  return FE_OK;
+}
+
+int fe_init_blob(const void* blob, size_t bytes, fe_ctx** out) {
+  if (!out) {
+    g_msg = "null argument";
+    return FE_ERR_INVALID_ARG;
+  }
+  *out = nullptr;
+  fe_config cfg{};
+  size_t n = 0;
+  FE_RC(fe_blob_parse(blob, bytes, &cfg, &n));
+  const unsigned char* w = static_cast<const unsigned char*>(blob) + kBlobHeader;
+  if (reinterpret_cast<uintptr_t>(w) % alignof(float) == 0)
+    return fe_init(&cfg, reinterpret_cast<const float*>(w), n, out);
+  std::vector<float> aligned(n);
+  std::memcpy(aligned.data(), w, n * sizeof(float));
+  return fe_init(&cfg, aligned.data(), n, out);
+}
+
+int fe_debug_alloc_hook(int fail_at, int64_t* live_out) {
+  if (fail_at >= 0) g_fail_countdown.store(fail_at);
+  if (live_out) *live_out = g_live_allocs.load();
+  return FE_OK;
+}
+
+int fe_debug_wait_probe(fe_ctx* c, uint32_t limit_us, void* stream) {
+  if (!c || limit_us == 0 || limit_us > 1000000u) {
+    g_msg = "null context or limit outside 1..1000000 us";
+    return FE_ERR_INVALID_ARG;
+  }
+  DeviceGuard g(c->device);
+  FE_RC(no_outstanding(c));
+  if (!c->status) FE_RC(reserve_impl(c, Shape{1, 1, 1, 1, 1}));
+  cudaStream_t s = (cudaStream_t)stream;
+  // the status word's way to the host is the batch's: copied to the
+  // page-locked word, then cleared for the next batch
+  FE_CK(fe::wait_probe_launch(c->status, (uint64_t)limit_us * 1000ull, s));
+  FE_CK(cudaMemcpyAsync(c->host_status, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+  FE_CK(cudaMemsetAsync(c->status, 0, sizeof(int), s));
+  FE_CK(cudaEventRecord(c->done_ev, s));
+  return wait_status(c);
 }
 
 int fe_reserve(fe_ctx* c, int B, int C, int M, int K, int L) {
@@ -1660,7 +1843,7 @@ int fe_destroy(fe_ctx* c) {
     }
     free_list(c->owned_ws);
     free_list(c->owned_w);
-    if (c->host_status) cudaFreeHost(c->host_status);
+    host_free(c->host_status);
     if (c->done_ev) cudaEventDestroy(c->done_ev);
     if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
     for (HostSlot& hs : c->slots) {
@@ -1668,7 +1851,7 @@ int fe_destroy(fe_ctx* c) {
       if (hs.in_ev) cudaEventDestroy(hs.in_ev);
       if (hs.run_ev) cudaEventDestroy(hs.run_ev);
       if (hs.done_ev) cudaEventDestroy(hs.done_ev);
-      if (hs.hstatus) cudaFreeHost(hs.hstatus);
+      host_free(hs.hstatus);
     }
     if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
     if (c->sub_stream) cudaStreamDestroy(c->sub_stream);

@@ -100,19 +100,25 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Wait for the completion of the phase with the given parity.  Gives up after
-// kWaitLimitNs, sets ST_TIMEOUT in *status and returns false.
+// limit_ns of %globaltimer, sets ST_TIMEOUT in *status and returns false.
 // Also gives up at once when another CTA of the batch has already timed out.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, int* status) {
+__device__ __forceinline__ bool mbar_wait_bounded_ns(uint64_t* bar, uint32_t parity, int* status,
+                                                     uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 255u) == 0u && (*reinterpret_cast<volatile int*>(status) & ST_TIMEOUT)) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
       atomicOr(status, ST_TIMEOUT);
       return false;
     }
   }
+}
+
+// The batch kernels' wait: limit kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, int* status) {
+  return mbar_wait_bounded_ns(bar, parity, status, kWaitLimitNs);
 }
 
 // The same wait with its loop out of line, for kernels with many wait sites

@@ -249,6 +249,8 @@ cudaError_t lin_attn_launch(const bf16* q, int ldq, const float* states, int n_s
 // ---------------------------------------------------------------------------
 // Raises the dynamic shared-memory limit of the compaction kernel (once per device).
 cudaError_t misc_prepare();
+// A bounded wait that nothing completes (test hook): sets ST_TIMEOUT in *status after limit_ns.
+cudaError_t wait_probe_launch(int* status, uint64_t limit_ns, cudaStream_t s);
 // Distinct-element compaction of every request: bitmap over the pool, ranks,
 // distinct list, |U(z_b)|, bad-request flags; the last CTA scans U into offsets.
 // Candidate-factorized layout (every occurrence its own element): per request b

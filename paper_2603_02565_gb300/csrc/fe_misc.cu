@@ -532,6 +532,24 @@ cudaError_t small_matmul_launch(const float* X, int R, int Kd, const float* W, i
   return cudaGetLastError();
 }
 
+// A bounded wait that nothing completes: one thread initialises an mbarrier
+// with an arrival count of one, never arrives on it and waits for its first
+// phase through the batch kernels' bounded wait, with a limit of limit_ns.
+// No copy and no tensor-core work is in flight, so giving up is always safe.
+// Launched only by the wait test hook (fe_debug_wait_probe).
+__global__ void wait_probe_kernel(int* status, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_mbar_init();
+  mbar_wait_bounded_ns(&bar, 0, status, limit_ns);
+}
+
+cudaError_t wait_probe_launch(int* status, uint64_t limit_ns, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(status, limit_ns);
+  return cudaGetLastError();
+}
+
 bool pdl_enabled() {
   static const bool on = [] {
     const char* v = std::getenv("FE_NO_PDL");
