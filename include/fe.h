@@ -262,6 +262,9 @@ int fe_debug_layout(fe_ctx* ctx, int32_t* slot_out, int32_t* U_out);
  *   "seq"     [B*K, d]      c_k, the SeqEnc output
  *   "cross"   [B*K, d]      C', the cross-sequence output (FE_ERR_UNSUPPORTED
  *                           when no_cross_seq = 1: C' = C is "seq")
+ *                           (both FE_ERR_UNSUPPORTED when the sequence-stage
+ *                           kernel kept them on chip: see
+ *                           fe_debug_keep_intermediates)
  *   "task_scores" [B*K, T]  every task head's score s_{k,t} before the fusion
  *                           (T = 1: the score itself)
  * `max_floats` is the capacity of `dst`; *n_floats receives the element count
@@ -269,6 +272,15 @@ int fe_debug_layout(fe_ctx* ctx, int32_t* slot_out, int32_t* U_out);
  */
 int fe_debug_fetch(fe_ctx* ctx, const char* name, float* dst, size_t max_floats,
                    size_t* n_floats);
+
+/*
+ * Test hook: with on = 1, later batches also store the SeqEnc output c and the
+ * cross-sequence output C' ("seq" and "cross" of fe_debug_fetch) where the
+ * sequence-stage kernel otherwise keeps them on chip (d = 128, K <= 128,
+ * L <= 31, one score head, bf16-exact weights); on = 0 stops it.  The extra
+ * stores cost time.  Errors: FE_ERR_INVALID_ARG, FE_ERR_CUDA.
+ */
+int fe_debug_keep_intermediates(fe_ctx* ctx, int on);
 
 /*
  * Tracing.  fe_profile(ctx, 1) makes later evaluations launch kernel by kernel

@@ -33,7 +33,7 @@ EXPORTS = ["fe_weight_count", "fe_init", "fe_reserve", "fe_evaluate", "fe_evalua
            "fe_profile_read",
            "fe_kernels_per_batch", "fe_distinct_layout_noalloc", "fe_destroy", "fe_strerror",
            "fe_last_error_message", "fe_blob_parse", "fe_init_blob", "fe_debug_alloc_hook",
-           "fe_debug_wait_probe"]
+           "fe_debug_wait_probe", "fe_debug_keep_intermediates"]
 
 
 class FeConfig(ctypes.Structure):
@@ -74,6 +74,8 @@ def load_library(path: str = LIB_PATH):
     L.fe_debug_alloc_hook.restype = i32
     L.fe_debug_wait_probe.argtypes = [vp, ctypes.c_uint32, vp]
     L.fe_debug_wait_probe.restype = i32
+    L.fe_debug_keep_intermediates.argtypes = [vp, i32]
+    L.fe_debug_keep_intermediates.restype = i32
     L.fe_reserve.argtypes = [vp, i32, i32, i32, i32, i32]
     L.fe_reserve.restype = i32
     for name in ("fe_evaluate", "fe_evaluate_async", "fe_evaluate_host", "fe_evaluate_factorized"):
@@ -361,6 +363,11 @@ class Evaluator:
             nm = raw[32 * i:32 * (i + 1)].split(b"\0", 1)[0].decode()
             out.append((nm, int(launches[i]), float(total[i])))
         return out
+
+    def keep_intermediates(self, on: bool = True):
+        """Store c and C' for fetch("seq") / fetch("cross") in later batches even
+        where the sequence-stage kernel keeps them on chip (a test hook)."""
+        _check(load_library().fe_debug_keep_intermediates(self._h, 1 if on else 0))
 
     def kernels_per_batch(self) -> int:
         return int(load_library().fe_kernels_per_batch(self._h))

@@ -332,6 +332,10 @@ struct fe_ctx {
   bool tail_q = false;     // the fused FFN of layer l also projects the next layer's Q
   bool tail_kv = false;    // the fused FFN of the last layer also projects [WKs | WVs]
   bool fused_ctxkv = false;  // context LN + K/V projection in one kernel (d <= 128, bf16 inputs)
+  bool seq_ok = false;       // the sequence stage can run as one kernel (fe_seq.cu) for suitable K, L
+  bool keep_inter = false;   // store c and C' even where the sequence-stage kernel keeps them on chip
+  int n_sms = 148;
+  float* elog = nullptr;     // [rows, d / 32] the elements' [CLS] logit partials (sequence-stage kernel)
   CUtensorMap ctxkv_w{};     // W^T of the K/V projection, 64 x 128 boxes, for the fused kernel
   std::vector<void*> owned_w;  // weight allocations
   std::vector<void*> owned_ws; // workspace allocations
@@ -587,7 +591,7 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
 int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const Weight& W1, const Weight& W2,
         const float* b1, const float* b2, const float* x0_row, const F32Rows& x, const Planes& ln_out, int rows,
         const int* rows_dev, cudaStream_t s, int store_ln = 1, const Weight* WT = nullptr,
-        const Planes* tail_out = nullptr, int tail_f16 = 0) {
+        const Planes* tail_out = nullptr, int tail_f16 = 0, float* tail_logits = nullptr) {
   if (rows <= 0) return FE_OK;
   Prof pf(c, site, s);
   fe::FfnParams p{};
@@ -607,6 +611,8 @@ int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const We
   p.store_ln = store_ln;
   p.eps = c->cfg.ln_eps;
   p.status = c->status;
+  p.tail_q0 = tail_logits ? c->q0 : nullptr;
+  p.tail_logits = tail_logits;
   FE_CK(fe::ffn_launch(&A.th, &A.tl, &WO.p.th, &WO.p.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.th, &ln_out.tl,
                        &x.sx, WT ? &WT->fh : nullptr, WT ? &WT->fl : nullptr, tail_out ? &tail_out->sh : nullptr,
                        tail_out ? &tail_out->sl : nullptr, p, s));
@@ -634,6 +640,12 @@ fe::SelArgs sel_args(fe_ctx* c, int B, int K, const IoPtrs& io) {
   return a;
 }
 
+// Whether a batch of K sequences of length L runs its sequence stage (assembly
+// to argmax) as one kernel.
+bool seq_fused(const fe_ctx* c, int K, int L) {
+  return c->seq_ok && fe::seq_supported(c->d, c->dh, c->F, c->nb, c->n_tasks, K, L);
+}
+
 // The whole evaluation of one batch, enqueued on s (captured into a graph by the caller).
 int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) {
   const int B = sh.B, C = sh.C, M = sh.M, K = sh.K, L = sh.L;
@@ -643,6 +655,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   const int cap = fact ? K * L : (c->cfg.encode_pool ? M : ((M < K * L) ? M : K * L));
   const int R = B * cap;
   const int S = B * K;
+  const bool use_seq = seq_fused(c, K, L);
   c->launches_batch = 0;
   // The status word and the fused argmax's words are zero here: the score
   // head's last CTA clears them after copying the status to io.hstatus.
@@ -808,7 +821,8 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
       const Weight* WT = !last ? (c->tail_q ? &c->wq[l + 1] : nullptr) : (c->tail_kv ? &c->kvs : nullptr);
       const Planes* TO = !last ? &c->q : &c->kvI;
       FE_RC(ffn(c, "ffn_item", c->a, c->wo[l], c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), nullptr, c->h,
-                c->xln, R, sumU, s, (last || !c->tail_q) ? 1 : 0, WT, WT ? TO : nullptr, last ? 0 : 1));
+                c->xln, R, sumU, s, (last || !c->tail_q) ? 1 : 0, WT, WT ? TO : nullptr,
+                (!last || (use_seq && WT)) ? 1 : 0, (last && use_seq && WT) ? c->elog : nullptr));
     } else {
       fe::GemmParams po{};
       po.resid = c->h.p;
@@ -831,6 +845,50 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   if (!(c->fused_ffn && c->tail_kv)) {
     fe::GemmParams p{};
     FE_RC(gemm(c, "gemm_item_seq_kv", fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, &c->kvI, nullptr, s));
+  }
+  if (use_seq) {
+    // (a3 - a6) in one kernel: assembly + [CLS] attention, SeqEnc, the
+    // cross-sequence block, the head and the argmax, G whole requests per tile
+    const int HN = c->w1h.N;
+    fe::SeqParams sp{};
+    sp.B = B;
+    sp.K = K;
+    sp.L = L;
+    sp.H = c->H;
+    sp.dh = c->dh;
+    sp.F = c->F;
+    const int per_sm = (B + c->n_sms - 1) / c->n_sms;
+    sp.G = std::max(1, std::min(128 / K, per_sm));
+    sp.off = c->off;
+    sp.bad = c->bad;
+    sp.slot = c->slot;
+    sp.elog = c->elog;
+    sp.v_h = c->kvI.h;
+    sp.ldv = c->kvI.ld;
+    sp.voff = d;
+    sp.q0 = c->q0;
+    sp.k0 = c->k0;
+    sp.v0 = c->v0;
+    sp.kP = c->kP;
+    sp.vP = c->vP;
+    sp.cls = tw(c, T_CLS);
+    sp.b1s = tw(c, T_B1S);
+    sp.b2s = tw(c, T_B2S);
+    sp.b1h = c->head_vec;
+    sp.w2h = c->head_vec + HN;
+    sp.b2h = c->head_vec + 2 * HN;
+    sp.cross = c->cfg.no_cross_seq ? 0 : 1;
+    sp.eps = c->cfg.ln_eps;
+    sp.scale_log2 = 1.4426950408889634f / sqrtf((float)c->dh);
+    sp.scores = io.scores;
+    sp.task_scores = c->task_scores;
+    sp.c_out = c->keep_inter ? c->c.p : nullptr;
+    sp.cp_out = c->keep_inter && !c->cfg.no_cross_seq ? c->cp.p : nullptr;
+    sp.sel = sel_args(c, B, K, io);
+    Prof pf(c, "seq_stage", s);
+    FE_CK(fe::seq_launch(&c->os.p.th, &c->w1s.fh, &c->w2s.p.th, &c->qkvx.p.th, &c->ox.p.th, &c->w1h.p.th, sp, s));
+    c->launches_last = c->launches_batch;
+    return FE_OK;
   }
   // (a3, a4) index-based assembly + [CLS] attention, then c = cls + o WOs, FFN
   {
@@ -1039,6 +1097,7 @@ int reserve_body(fe_ctx* c, const Shape& s, const bool fact) {
   c->sel_ticket = reinterpret_cast<unsigned*>(c->sel_nan + B);
   FE_RC(dalloc((void**)&c->slot, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int)));
   FE_RC(dalloc((void**)&c->list, (size_t)R * sizeof(int)));
+  if (c->seq_ok) FE_RC(dalloc((void**)&c->elog, (size_t)R * (size_t)(d / 32) * sizeof(float)));
   FE_RC(alloc_f32(c->h, R, d, c->owned_ws));
   FE_RC(alloc_f32(c->c, S, d, c->owned_ws));
   FE_RC(alloc_f32(c->cp, S, d, c->owned_ws));
@@ -1251,7 +1310,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   int rc = FE_OK;
   if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess ||
       fe::ffn_prepare() != cudaSuccess || fe::ctxkv_prepare() != cudaSuccess || fe::linattn_prepare() != cudaSuccess ||
-      fe::embed_q_prepare() != cudaSuccess)
+      fe::embed_q_prepare() != cudaSuccess || fe::seq_prepare() != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "kernel attributes"));
   {
     size_t o = 0;
@@ -1308,6 +1367,9 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     for (int l = 1; l < Ly; ++l)
       if ((rc = map_tail(c->wq[l], c->nb > 1)) != FE_OK) return fail(rc);
   if (c->tail_kv && (rc = map_tail(c->kvs, c->nb > 1)) != FE_OK) return fail(rc);
+  c->seq_ok = c->fused_ffn && c->tail_kv && fe::seq_supported(d, c->dh, F, c->nb, n_tasks_of(cfg), 1, 1);
+  if (cudaDeviceGetAttribute(&c->n_sms, cudaDevAttrMultiProcessorCount, c->device) != cudaSuccess)
+    return fail(set_cuda_err(cudaGetLastError(), "device attribute"));
   if ((rc = make_weight(c, c->w2s, d, F, 512)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w2s, tw(c, T_W2S), F, d, 0)) != FE_OK) return fail(rc);
   if (!cfg->no_cross_seq) {
@@ -1731,12 +1793,20 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
     rows = (size_t)sum;
     cols = d;
   } else if (n == "seq") {
+    if (seq_fused(c, s.K, s.L) && !c->keep_inter) {
+      g_msg = "seq is kept on chip by the sequence-stage kernel (fe_debug_keep_intermediates stores it)";
+      return FE_ERR_UNSUPPORTED;
+    }
     f32 = c->c.p;
     rows = (size_t)s.B * s.K;
     cols = d;
   } else if (n == "cross") {
     if (c->cfg.no_cross_seq) {
       g_msg = "no cross-sequence block in this configuration (C' = C: fetch \"seq\")";
+      return FE_ERR_UNSUPPORTED;
+    }
+    if (seq_fused(c, s.K, s.L) && !c->keep_inter) {
+      g_msg = "cross is kept on chip by the sequence-stage kernel (fe_debug_keep_intermediates stores it)";
       return FE_ERR_UNSUPPORTED;
     }
     f32 = c->cp.p;
@@ -1785,6 +1855,17 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
       std::memcpy(&fb, &b, 4);
       dst[r * cols + j] = fa + fb;
     }
+  return FE_OK;
+}
+
+int fe_debug_keep_intermediates(fe_ctx* c, int on) {
+  if (!c || (on != 0 && on != 1)) return FE_ERR_INVALID_ARG;
+  DeviceGuard g(c->device);
+  if (c->keep_inter != (on == 1)) {
+    FE_CK(cudaDeviceSynchronize());
+    clear_graphs(c);
+    c->keep_inter = on == 1;
+  }
   return FE_OK;
 }
 

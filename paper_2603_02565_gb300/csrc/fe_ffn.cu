@@ -635,9 +635,24 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t tb = p.tail_f16 ? 2048u : 4096u;
         uint8_t* stg = sT + (size_t)ew * 2u * tb;
         int k = 0;
-        for (int c = 32 * half; c < tail_n; c += 64, ++k) {
+        for (int c = 32 * half; c < tail_n; c += 64) {
           float v[32];
           tmem_ld32(tmem + lane_off + (uint32_t)c, v);
+          if (p.tail_q0 && c < d) {
+            // a key group of SeqEnc: only its [CLS] logit partial q0 . k leaves the SM
+            float acc = 0.f;
+            const float4* q = reinterpret_cast<const float4*>(p.tail_q0 + c);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 qq = __ldg(q + j);
+              acc = fmaf(v[4 * j], qq.x, acc);
+              acc = fmaf(v[4 * j + 1], qq.y, acc);
+              acc = fmaf(v[4 * j + 2], qq.z, acc);
+              acc = fmaf(v[4 * j + 3], qq.w, acc);
+            }
+            if (valid) p.tail_logits[(size_t)(m0 + r) * (size_t)(d / 32) + (size_t)(c / 32)] = acc;
+            continue;
+          }
           uint8_t* b = stg + (size_t)(k & 1) * tb;
           if (lane == 0 && k >= 2) asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
           __syncwarp();
@@ -657,6 +672,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           issue(&tTo_h, b, p.tail_f16 ? nullptr : &tTo_l, b + 2048, c, srow);
+          ++k;
         }
         tc_fence_before();  // TMEM read before r_empty lets the next tile's projection in
       }

@@ -132,6 +132,12 @@ struct FfnParams {
   int store_ln;         // store LN(x_out)
   float eps;
   int* status;
+  // With tail_q0 set (a split-pair tail of 2d columns, keys | values of SeqEnc):
+  // the key columns are not stored; each 32-column group g of them is reduced
+  // with q0 (the [CLS] query cls WQs, fp32 [d]) and written to
+  // tail_logits[row * (d / 32) + g] (fp32); the value columns are stored as usual.
+  const float* tail_q0;
+  float* tail_logits;
 };
 bool ffn_supported(int d, int d_pad, int F, int nb);
 bool ffn_tail_supported(int d, int d_pad, int F, int nb, int tail_n, int tail_f16);
@@ -288,6 +294,44 @@ struct ClsParams {
   float scale;                // 1 / sqrt(d_h)
 };
 cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// The sequence stage in one kernel (fe_seq.cu), for d = 128, d_h in {32, 64},
+// K <= 128, L <= 31, one score head and bf16-exact weights: index-based
+// assembly and the [CLS] attention of SeqEnc (Section 4.3), SeqEnc's output
+// projection and FFN, the cross-sequence block (Section 4.4), the score head
+// and the argmax of Eq. 1.  A tile holds G whole requests (G K <= 128 rows,
+// row = request-local sequence), so the cross-sequence attention and the
+// argmax never leave the CTA.
+// Weight maps: W^T planes with 64 x 128 boxes and the 128-byte swizzle:
+// WOs [d, d], W1s [F, d], W2s [d, F], [WQx | WKx | WVx] [3d, d], WOx [d, d],
+// W1h [d, d].
+// ---------------------------------------------------------------------------
+struct SeqParams {
+  int B, K, L, H, dh, F;
+  int G;                     // requests per tile
+  const int* off;            // [B + 1] element row offsets
+  const int* bad;            // [B]
+  const int* slot;           // [B, K, L] request-local slots
+  const float* elog;         // [rows, d / 32] per-32-column [CLS] logit partials q0 . (H WKs)
+  const bf16* v_h;           // element values H WVs, one f16 plane (bits), row stride ldv, at column voff
+  int ldv, voff;
+  const float *q0, *k0, *v0, *kP, *vP;  // [CLS] WQs / WKs / WVs, P WKs, P WVs
+  const float *cls, *b1s, *b2s, *b1h, *w2h, *b2h;
+  int cross;                 // 0: no cross-sequence block (C' = C)
+  float eps;
+  float scale_log2;          // log2(e) / sqrt(d_h)
+  float* scores;             // [B, K]
+  float* task_scores;        // [B, K] the single head's score again (the per-task scores of one task), or null
+  float* c_out;              // [B K, d] c (SeqEnc output), or null
+  float* cp_out;             // [B K, d] C', or null
+  SelArgs sel;               // best, status, host status, ticket (keys / nan unused)
+};
+bool seq_supported(int d, int dh, int F, int nb, int n_tasks, int K, int L);
+cudaError_t seq_prepare();
+cudaError_t seq_launch(const CUtensorMap* wos, const CUtensorMap* w1s, const CUtensorMap* w2s,
+                       const CUtensorMap* qkvx, const CUtensorMap* wox, const CUtensorMap* w1h, const SeqParams& p,
+                       cudaStream_t s);
 // weight preparation: out[(row0 + n) * ldo + k] = split(W[k * N + n]) for k < Kin, n < N
 cudaError_t transpose_split_launch(const float* W, int Kin, int N, bf16* out_h, bf16* out_l, int ldo,
                                    int row0, cudaStream_t s);

@@ -1,0 +1,1034 @@
+// The sequence stage of the evaluator in one kernel, for rows of width
+// d = 128: index-based assembly with position embeddings and the [CLS]
+// attention of SeqEnc (Section 4.3), SeqEnc's output projection, residual on
+// [CLS] and FFN, the cross-sequence self-attention block (Section 4.4), the
+// shared score head and the argmax of Eq. 1.
+//
+// A tile is 128 rows holding G whole requests (row = lr K + k: sequence k of
+// the tile's request lr), so everything a request needs -- its K sequence
+// vectors for the cross-sequence attention and its K scores for the argmax --
+// stays in one CTA; nothing of the stage goes to memory but the scores and
+// best indices.  Per tile:
+//   A  (epilogue warps) for every sequence: the [CLS] logits of its L element
+//      rows come precomputed per element (q0 . (H WKs), q0 = cls WQs, from the
+//      last element layer's tail), plus q0 . (P WKs) per position; softmax
+//      over [CLS; L tokens] per head; o = p_cls v0 + sum_j p_j (H_j WVs +
+//      P_j WVs) with the value rows gathered by 8-byte loads; o -> shared
+//      memory as the split operand tile
+//   B  c = cls + o WOs; c += W2s ReLU(W1s LN(c) + b1s) + b2s  (the FFN in
+//      128-column chunks, the hidden activation in TMEM, as fe_ffn.cu)
+//   C  Z = LN(c); Q | K | V = Z [WQx | WKx | WVx] (f16 tiles in shared
+//      memory); per head S = Q K^T over the tile's 128 rows with the
+//      block-diagonal request mask, softmax, P (f16, in TMEM) V
+//   D  C' = c + A WOx; LN(C')
+//   E  s = ReLU(LN(C') W1h + b1h) . w2h + b2h; per request the smallest k
+//      attaining the maximum
+// Roles: warp 0 lane 0 streams the weights (32 KB chunks in consumption order
+// through a ring of three slots, by TMA), warp 1 lane 0 issues tcgen05.mma,
+// warps 2-9 run the gathers, softmaxes and epilogues (two warps per TMEM lane
+// quadrant, each owning half of a row's columns).  Products take split
+// bf16 activations (hi + lo) times exact bf16 weights with fp32 accumulation;
+// the attention operands Q, K, V, P are single f16 planes; LayerNorm,
+// softmax and residuals are fp32.
+#include "fe_common.cuh"
+#include "fe_kernels.h"
+
+namespace fe {
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int D = 128;
+constexpr int BK = 64;
+constexpr int FC = 128;  // FFN columns per chunk
+constexpr int NA1 = 3;   // TMEM buffers for FFN1 chunks
+constexpr int LA = 2;    // FFN1 chunks issued ahead of the FFN2 that consumes them
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
+constexpr int kMaxL = 31;
+constexpr int kMaxF = 1024;
+constexpr uint32_t kAPlane = BM * BK * 2;  // 16 KB: 128 rows x 64 bf16
+constexpr uint32_t kChunk = 2 * kAPlane;   // a weight chunk: two 128-row x 64-column boxes
+constexpr int kRing = 3;
+constexpr uint32_t kOffV = 4 * kAPlane;               // 64 KB: the split A tile [kb][plane]
+constexpr uint32_t kOffRing = kOffV + 32768;          // the V tiles, one per head
+constexpr uint32_t kOffMisc = kOffRing + kRing * kChunk;
+// misc: b1s [kMaxF], b2s, cls, b1h, w2h [D], q0.kP [32][4], q0.k0 [4], row-statistic
+// exchange [4][2][128], scores [128], request flags [128], barriers, TMEM slot
+constexpr uint32_t kMiscB1 = 0;
+constexpr uint32_t kMiscB2 = kMiscB1 + kMaxF * 4;
+constexpr uint32_t kMiscCls = kMiscB2 + D * 4;
+constexpr uint32_t kMiscB1h = kMiscCls + D * 4;
+constexpr uint32_t kMiscW2h = kMiscB1h + D * 4;
+constexpr uint32_t kMiscQkP = kMiscW2h + D * 4;
+constexpr uint32_t kMiscQk0 = kMiscQkP + 32 * 4 * 4;
+constexpr uint32_t kMiscRed = kMiscQk0 + 64;
+constexpr uint32_t kMiscSc = kMiscRed + 4 * 2 * 128 * 4;
+constexpr uint32_t kMiscFlag = kMiscSc + 128 * 4;
+constexpr uint32_t kMiscBars = kMiscFlag + 128 * 4;
+constexpr uint32_t kMiscBytes = kMiscBars + 64 * 8 + 64;
+constexpr size_t kSmem = 1024 + kOffMisc + kMiscBytes;
+
+__device__ __forceinline__ float relu_keep_nan(float x) {
+  float r;
+  asm("max.NaN.f32 %0, %1, 0f00000000;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+__device__ __forceinline__ void arrive1(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ uint64_t desc_swz(uint32_t saddr, uint32_t sbo, uint32_t swz) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(sbo >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)swz << 61;
+  return d;
+}
+
+// The weight chunk the tile consumes i-th: its map and box origin.  Order: WOs,
+// then FFN1 chunk s and FFN2 chunk s - LA interleaved as the MMA issuer takes
+// them, then WQx, WKx, WVx, WOx (with the cross-sequence block), then W1h.
+struct ChunkSrc {
+  int kind;  // 0 WOs, 1 W1s, 2 W2s, 3 QKVx, 4 WOx, 5 W1h
+  int idx;
+};
+
+__device__ __forceinline__ ChunkSrc chunk_of(int i, int nf, int cross) {
+  if (i == 0) return {0, 0};
+  int r = i - 1;
+  for (int s = 0; s < nf + LA; ++s) {
+    if (s < nf) {
+      if (r == 0) return {1, s};
+      --r;
+    }
+    if (s >= LA) {
+      if (r == 0) return {2, s - LA};
+      --r;
+    }
+  }
+  if (cross) {
+    if (r < 3) return {3, r};
+    if (r == 3) return {4, 0};
+    r -= 4;
+  }
+  return {5, 0};
+}
+
+// Two 32-column pieces of this warp's 32 TMEM lanes (row = lane) into
+// registers, one wait for both.
+__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, float* va, float* vb) {
+  uint32_t a[32], b[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
+      "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7]),
+        "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]), "=r"(a[14]), "=r"(a[15]),
+        "=r"(a[16]), "=r"(a[17]), "=r"(a[18]), "=r"(a[19]), "=r"(a[20]), "=r"(a[21]), "=r"(a[22]), "=r"(a[23]),
+        "=r"(a[24]), "=r"(a[25]), "=r"(a[26]), "=r"(a[27]), "=r"(a[28]), "=r"(a[29]), "=r"(a[30]), "=r"(a[31]),
+        "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7]),
+        "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]), "=r"(b[14]), "=r"(b[15]),
+        "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]), "=r"(b[21]), "=r"(b[22]), "=r"(b[23]),
+        "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]), "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
+      : "r"(ta), "r"(tb)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    va[i] = __uint_as_float(a[i]);
+    vb[i] = __uint_as_float(b[i]);
+  }
+}
+
+// 32 lanes x 32 columns from registers, no wait (tmem_st_wait completes it)
+__device__ __forceinline__ void tmem_st32_nw(uint32_t taddr, const float* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15])), "r"(__float_as_uint(v[16])), "r"(__float_as_uint(v[17])),
+      "r"(__float_as_uint(v[18])), "r"(__float_as_uint(v[19])), "r"(__float_as_uint(v[20])),
+      "r"(__float_as_uint(v[21])), "r"(__float_as_uint(v[22])), "r"(__float_as_uint(v[23])),
+      "r"(__float_as_uint(v[24])), "r"(__float_as_uint(v[25])), "r"(__float_as_uint(v[26])),
+      "r"(__float_as_uint(v[27])), "r"(__float_as_uint(v[28])), "r"(__float_as_uint(v[29])),
+      "r"(__float_as_uint(v[30])), "r"(__float_as_uint(v[31]))
+      : "memory");
+}
+
+// This thread's 64 columns of row r (32 half + 64 ci + [0, 32), ci < 2) as a
+// split bf16 pair into the A tile (128-byte swizzle, [kb][plane]).
+__device__ __forceinline__ void store_split64(uint8_t* sA, int r, int half, const float* v) {
+#pragma unroll
+  for (int ci = 0; ci < 2; ++ci) {
+    uint32_t hi[16], lo[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) split2(v[32 * ci + 2 * j], v[32 * ci + 2 * j + 1], hi[j], lo[j]);
+    uint8_t* rowp = sA + (size_t)(ci * 2) * kAPlane + (size_t)r * 128u;
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+      const uint32_t o = (uint32_t)((4 * half + jj) ^ (r & 7)) << 4;
+      *reinterpret_cast<uint4*>(rowp + o) = make_uint4(hi[4 * jj], hi[4 * jj + 1], hi[4 * jj + 2], hi[4 * jj + 3]);
+      *reinterpret_cast<uint4*>(rowp + kAPlane + o) =
+          make_uint4(lo[4 * jj], lo[4 * jj + 1], lo[4 * jj + 2], lo[4 * jj + 3]);
+    }
+  }
+}
+
+// The residual step shared by SeqEnc and the cross-sequence block (one copy
+// of the code for its three uses): x = acc [+ add] [+ bias] (this thread's 64
+// columns of row r; written back to the accumulator when anything was added,
+// and to out_row when given), then LN(x) as the split A tile.  acc_t and add_t
+// are TMEM addresses of the thread's lane quadrant (add: whether add_t is
+// added); the row statistics are exchanged with the partner warp of the quadrant.
+__device__ __noinline__ void epi_resid_ln(uint8_t* sA, float* red, uint32_t acc_t, bool add, uint32_t add_t,
+                                          const float* bias, float* out_row, int r, int q, int half, float eps) {
+  float v[64];
+  tmem_ld32x2(acc_t + (uint32_t)(32 * half), acc_t + (uint32_t)(32 * half + 64), v, v + 32);
+  if (add) {
+    float w[64];
+    tmem_ld32x2(add_t + (uint32_t)(32 * half), add_t + (uint32_t)(32 * half + 64), w, w + 32);
+#pragma unroll
+    for (int j = 0; j < 64; ++j) v[j] += w[j];
+  }
+  if (bias) {
+#pragma unroll
+    for (int ci = 0; ci < 2; ++ci)
+#pragma unroll
+      for (int j = 0; j < 32; j += 4) {
+        const float4 b = *reinterpret_cast<const float4*>(bias + 32 * half + 64 * ci + j);
+        v[32 * ci + j] += b.x;
+        v[32 * ci + j + 1] += b.y;
+        v[32 * ci + j + 2] += b.z;
+        v[32 * ci + j + 3] += b.w;
+      }
+  }
+  if (add || bias) {
+    tmem_st32_nw(acc_t + (uint32_t)(32 * half), v);
+    tmem_st32_nw(acc_t + (uint32_t)(32 * half + 64), v + 32);
+  }
+  if (out_row) {
+#pragma unroll
+    for (int ci = 0; ci < 2; ++ci)
+#pragma unroll
+      for (int j = 0; j < 32; j += 4)
+        *reinterpret_cast<float4*>(out_row + 32 * half + 64 * ci + j) =
+            make_float4(v[32 * ci + j], v[32 * ci + j + 1], v[32 * ci + j + 2], v[32 * ci + j + 3]);
+  }
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < 64; ++j) sum += v[j];
+  red[half * 128 + r] = sum;
+  asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+  const float mean = (red[r] + red[128 + r]) * (1.f / (float)D);
+  float var = 0.f;
+#pragma unroll
+  for (int j = 0; j < 64; ++j) {
+    const float dv = v[j] - mean;
+    var = fmaf(dv, dv, var);
+  }
+  red[256 + half * 128 + r] = var;
+  asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+  const float rstd = 1.0f / sqrtf((red[256 + r] + red[256 + 128 + r]) * (1.f / (float)D) + eps);
+#pragma unroll
+  for (int j = 0; j < 64; ++j) v[j] = (v[j] - mean) * rstd;
+  store_split64(sA, r, half, v);
+  if (add || bias) tmem_st_wait();
+}
+
+// D = (split A tile at sA) . (weight chunk at w)^T, N = 128, K = 128: the
+// products of every weight chunk but FFN2's (one copy of the issue code).
+__device__ __noinline__ void mma_tile(uint32_t dst, uint32_t sa, uint32_t w, uint32_t idesc) {
+  const uint64_t a0 = umma_desc_sw128(sa);
+  const uint64_t w0 = umma_desc_sw128(w);
+#pragma unroll
+  for (int kb = 0; kb < 2; ++kb) {
+#pragma unroll
+    for (int kk = 0; kk < BK / 16; ++kk) {
+      const uint64_t ah = desc_adv(a0, (uint32_t)(kb * 2) * kAPlane + kk * 32);
+      const uint64_t wh = desc_adv(w0, (uint32_t)kb * kAPlane + kk * 32);
+      umma_bf16(dst, ah, wh, idesc, (kb | kk) != 0 ? 1u : 0u);
+      umma_bf16(dst, desc_adv(ah, kAPlane), wh, idesc, 1u);
+    }
+  }
+}
+
+}  // namespace
+
+template <int DH>
+__global__ void __launch_bounds__(kThreads, 1)
+    seq_kernel(const __grid_constant__ CUtensorMap tWOs, const __grid_constant__ CUtensorMap tW1s,
+               const __grid_constant__ CUtensorMap tW2s, const __grid_constant__ CUtensorMap tQKV,
+               const __grid_constant__ CUtensorMap tWOx, const __grid_constant__ CUtensorMap tW1h,
+               const SeqParams p) {
+  constexpr int H = D / DH;
+  constexpr uint32_t kVRow = DH * 2;                 // bytes per row of a V tile
+  constexpr uint32_t kVTile = BM * kVRow;            // one head's V tile: 128 keys x DH
+  constexpr uint32_t kVSbo = 8 * kVRow;
+  constexpr uint32_t kVSwz = DH == 32 ? 4u : 2u;     // 64-byte / 128-byte swizzle
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_s = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
+  uint8_t* sA = smem;
+  uint8_t* sV = smem + kOffV;
+  uint8_t* sR = smem + kOffRing;
+  uint8_t* misc = smem + kOffMisc;
+  float* sB1 = reinterpret_cast<float*>(misc + kMiscB1);
+  float* sB2 = reinterpret_cast<float*>(misc + kMiscB2);
+  float* sCls = reinterpret_cast<float*>(misc + kMiscCls);
+  float* sB1h = reinterpret_cast<float*>(misc + kMiscB1h);
+  float* sW2h = reinterpret_cast<float*>(misc + kMiscW2h);
+  float* sQkP = reinterpret_cast<float*>(misc + kMiscQkP);  // [j][4]: q0 . kP[j] per head
+  float* sQk0 = reinterpret_cast<float*>(misc + kMiscQk0);  // [4]: q0 . k0 per head
+  float* red = reinterpret_cast<float*>(misc + kMiscRed);   // [slot][half][row]
+  float* sSc = reinterpret_cast<float*>(misc + kMiscSc);
+  int* sFlag = reinterpret_cast<int*>(misc + kMiscFlag);    // request of the tile has a non-finite value row
+  int* sErow = reinterpret_cast<int*>(sV);                  // during the gathers: [row][32] element rows,
+                                                            // then the token weights at sV + 16 KB
+  uint64_t* bars = reinterpret_cast<uint64_t*>(misc + kMiscBars);
+  uint64_t* w_full = bars;            // [kRing]
+  uint64_t* w_empty = bars + 3;       // [kRing]
+  uint64_t* a_full = bars + 6;        // o written in sA
+  uint64_t* o_done = bars + 7;        // o WOs complete
+  uint64_t* ln_full = bars + 8;       // x in the accumulator, LN(x) in sA
+  uint64_t* acc1_full = bars + 9;     // [NA1]
+  uint64_t* acc1_empty = bars + 12;   // [NA1]
+  uint64_t* mid_full = bars + 15;     // [NA1]
+  uint64_t* acc2_full = bars + 18;    // the FFN complete
+  uint64_t* z_full = bars + 19;       // c in the accumulator, LN(c) in sA
+  uint64_t* qkv_full = bars + 20;     // the Q | K | V product complete
+  uint64_t* qkv_ready = bars + 21;    // Q, K in sA and V in sV
+  uint64_t* s_full = bars + 22;       // [2]
+  uint64_t* p_full = bars + 24;       // [2]
+  uint64_t* s_free = bars + 26;       // [2] PV has read the S/P buffer
+  uint64_t* o_full = bars + 28;       // every head's PV complete
+  uint64_t* a2_full = bars + 29;      // attention output in sA
+  uint64_t* ox_full = bars + 30;      // A WOx complete
+  uint64_t* lnc_full = bars + 31;     // LN(C') in sA
+  uint64_t* head_full = bars + 32;    // the head product complete
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 40);
+  volatile uint32_t* last_flag = reinterpret_cast<volatile uint32_t*>(bars + 41);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int K = p.K, L = p.L, G = p.G, F = p.F;
+  const int nf = F / FC;
+  const int tiles = (p.B + G - 1) / G;
+  const int nch = 1 + 2 * nf + (p.cross ? 4 : 0) + 1;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kRing; ++i) {
+      mbar_init(w_full + i, 1);
+      mbar_init(w_empty + i, 1);
+    }
+    for (int i = 0; i < NA1; ++i) {
+      mbar_init(acc1_full + i, 1);
+      mbar_init(acc1_empty + i, 1);
+      mbar_init(mid_full + i, 32 * kEpiWarps);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(s_full + i, 1);
+      mbar_init(p_full + i, 32 * kEpiWarps);
+      mbar_init(s_free + i, 1);
+    }
+    mbar_init(a_full, 32 * kEpiWarps);
+    mbar_init(o_done, 1);
+    mbar_init(ln_full, 32 * kEpiWarps);
+    mbar_init(acc2_full, 1);
+    mbar_init(z_full, 32 * kEpiWarps);
+    mbar_init(qkv_full, 1);
+    mbar_init(qkv_ready, 32 * kEpiWarps);
+    mbar_init(o_full, 1);
+    mbar_init(a2_full, 32 * kEpiWarps);
+    mbar_init(ox_full, 1);
+    mbar_init(lnc_full, 32 * kEpiWarps);
+    mbar_init(head_full, 1);
+    fence_mbar_init();
+    prefetch_tmap(&tWOs);
+    prefetch_tmap(&tW1s);
+    prefetch_tmap(&tW2s);
+    prefetch_tmap(&tQKV);
+    prefetch_tmap(&tWOx);
+    prefetch_tmap(&tW1h);
+  }
+  // parameters (not outputs of an earlier kernel): read before the dependency wait
+  for (int i = threadIdx.x; i < F; i += kThreads) sB1[i] = p.b1s[i];
+  for (int i = threadIdx.x; i < D; i += kThreads) {
+    sB2[i] = p.b2s[i];
+    sCls[i] = p.cls[i];
+    sB1h[i] = p.b1h[i];
+    sW2h[i] = p.w2h[i];
+  }
+  // the [CLS] query's logits against [CLS] itself and against each position
+  // embedding's key part, per head (unscaled)
+  for (int i = threadIdx.x; i < (L + 1) * H; i += kThreads) {
+    const int j = i / H, h = i - j * H;
+    const float* kv = j < L ? p.kP + (size_t)j * D : p.k0;
+    float acc = 0.f;
+    for (int c = h * DH; c < h * DH + DH; ++c) acc = fmaf(p.q0[c], kv[c], acc);
+    if (j < L)
+      sQkP[j * 4 + h] = acc;
+    else
+      sQk0[h] = acc;
+  }
+  // TMEM: FFN1 chunk buffers [128 i, 128 i + 128), i < 3 (later Q | K | V, then the
+  // S/P buffers [0, 256) with the attention output at [256, 384), then A WOx at
+  // [0, 128) and the head product at [128, 256)); the d-column accumulator of
+  // x, c and C' at [384, 512)
+  if (warp == 0) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t acc2 = tmem + (uint32_t)(NA1 * FC);
+  pdl_trigger();
+  pdl_wait();
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer: the weight chunks of every tile ----------------
+      int ws = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
+        for (int i = 0; i < nch; ++i, ++ws) {
+          const int slot = ws % kRing;
+          if (ws >= kRing && !mbar_wait_compact(w_empty + slot, ((ws / kRing) - 1) & 1, p.sel.status)) {
+            ok = false;
+            break;
+          }
+          const ChunkSrc cs = chunk_of(i, nf, p.cross);
+          const CUtensorMap* m = &tWOs;
+          int x0 = 0, x1 = BK, y = 0;
+          if (cs.kind == 1) {
+            m = &tW1s;
+            y = cs.idx * FC;
+          } else if (cs.kind == 2) {
+            m = &tW2s;
+            x0 = cs.idx * FC;
+            x1 = x0 + BK;
+          } else if (cs.kind == 3) {
+            m = &tQKV;
+            y = cs.idx * D;
+          } else if (cs.kind == 4) {
+            m = &tWOx;
+          } else if (cs.kind == 5) {
+            m = &tW1h;
+          }
+          uint8_t* dst = sR + (size_t)slot * kChunk;
+          mbar_arrive_expect_tx(w_full + slot, kChunk);
+          tma_load_2d(dst, m, x0, y, w_full + slot);
+          tma_load_2d(dst + kAPlane, m, x1, y, w_full + slot);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      const uint32_t idesc = umma_idesc_bf16(BM, FC);
+      const uint32_t idesc_s = umma_idesc_f16(BM, BM);
+      const uint32_t idesc_pv = umma_idesc_f16(BM, DH) | (1u << 16);  // V is MN-major
+      int ws = 0, gf = 0, tl = 0;
+      bool ok = true;
+      auto wait = [&](uint64_t* bar, uint32_t par) -> bool {
+        if (!mbar_wait_compact(bar, par, p.sel.status)) ok = false;
+        return ok;
+      };
+      // the next weight chunk landed: its slot
+      auto next_slot = [&]() -> int {
+        const int slot = ws % kRing;
+        if (!wait(w_full + slot, (ws / kRing) & 1)) return -1;
+        tc_fence_after();
+        return slot;
+      };
+      // dst = (split A tile in sA) . (weight chunk in `slot`)^T, N = 128, K = 128
+      auto mma_sa = [&](uint32_t dst, int slot) {
+        mma_tile(dst, smem_u32(sA), smem_u32(sR + (size_t)slot * kChunk), idesc);
+        umma_commit(w_empty + slot);
+        ++ws;
+      };
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+        // ---- B: o WOs into the FFN1 buffer that chunk 0 of this tile uses next
+        if (!wait(a_full, tl & 1)) break;
+        {
+          const int bo = gf % NA1;
+          const int slot = next_slot();
+          if (slot < 0) break;
+          if (gf >= NA1 && !wait(acc1_empty + bo, ((gf / NA1) - 1) & 1)) break;
+          tc_fence_after();
+          mma_sa(tmem + (uint32_t)(bo * FC), slot);
+          umma_commit(o_done);
+        }
+        // ---- B: FFN1 / FFN2 once x is in the accumulator and LN(x) in sA
+        if (!wait(ln_full, tl & 1)) break;
+        tc_fence_after();
+        const int gf0 = gf;
+        for (int s = 0; s < nf + LA && ok; ++s) {
+          if (s < nf) {
+            const int g = gf0 + s, b = g % NA1;
+            if (s > 0 && g >= NA1 && !wait(acc1_empty + b, ((g / NA1) - 1) & 1)) break;
+            const int slot = next_slot();
+            if (slot < 0) break;
+            mma_sa(tmem + (uint32_t)(b * FC), slot);
+            umma_commit(acc1_full + b);
+          }
+          if (s >= LA) {
+            const int c = s - LA, g = gf0 + c, b = g % NA1;
+            if (!wait(mid_full + b, (g / NA1) & 1)) break;
+            const int slot = next_slot();
+            if (slot < 0) break;
+            // each 32-column piece of the buffer: 32 hidden units as the hi plane
+            // (16 columns of bf16 pairs) then the lo plane; the W2s chunk holds two
+            // 64-column halves of the chunk's hidden units, 128 output rows each
+            const uint32_t mt = tmem + (uint32_t)(b * FC);
+            const uint64_t w0 = umma_desc_sw128(smem_u32(sR + (size_t)slot * kChunk));
+#pragma unroll
+            for (int kk = 0; kk < FC / 16; ++kk) {
+              const int hh = kk >> 2, k4 = kk & 3;
+              const uint32_t mh = mt + (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1)), ml = mh + 16;
+              const uint64_t wh = desc_adv(w0, (uint32_t)hh * kAPlane + k4 * 32);
+              umma_bf16_tmem_a(acc2, mh, wh, idesc, 1u);
+              umma_bf16_tmem_a(acc2, ml, wh, idesc, 1u);
+            }
+            umma_commit(w_empty + slot);
+            ++ws;
+            umma_commit(acc1_empty + b);
+            if (c == nf - 1) umma_commit(acc2_full);
+          }
+        }
+        if (!ok) break;
+        gf = gf0 + nf;
+        if (!wait(z_full, tl & 1)) break;
+        tc_fence_after();
+        if (p.cross) {
+          // ---- C: Q | K | V = Z [WQx | WKx | WVx] into TMEM [0, 384)
+          for (int i = 0; i < 3 && ok; ++i) {
+            const int slot = next_slot();
+            if (slot < 0) break;
+            mma_sa(tmem + (uint32_t)(i * 128), slot);
+          }
+          if (!ok) break;
+          umma_commit(qkv_full);
+          if (!wait(qkv_ready, tl & 1)) break;
+          tc_fence_after();
+          // S_h = Q_h K_h^T over the tile's 128 rows into S/P buffer (tl H + h) % 2
+          auto issue_s = [&](int h) -> bool {
+            const int g = tl * H + h, buf = g & 1;
+            if (g >= 2 && !wait(s_free + buf, ((g - 2) >> 1) & 1)) return false;
+            tc_fence_after();
+            const int c0 = h * DH;
+            const uint64_t qd = umma_desc_sw128(smem_u32(sA + (uint32_t)(c0 / BK) * kAPlane));
+            const uint64_t kd = umma_desc_sw128(smem_u32(sA + (uint32_t)(2 + c0 / BK) * kAPlane));
+#pragma unroll
+            for (int kk = 0; kk < DH / 16; ++kk) {
+              const uint32_t o = (uint32_t)(c0 % BK) * 2u + (uint32_t)kk * 32u;
+              umma_bf16(tmem + (uint32_t)(buf * 128), desc_adv(qd, o), desc_adv(kd, o), idesc_s, kk != 0 ? 1u : 0u);
+            }
+            umma_commit(s_full + buf);
+            return true;
+          };
+          if (!issue_s(0)) break;
+          if (H > 1 && !issue_s(1)) break;
+          for (int h = 0; h < H && ok; ++h) {
+            const int g = tl * H + h, buf = g & 1;
+            if (!wait(p_full + buf, (g >> 1) & 1)) break;
+            tc_fence_after();
+            // PV_h: A = P_h from the S/P buffer (each half-row warp's 64 keys as 32
+            // columns of f16 pairs at the start of its 64 S columns), B = V_h
+            const uint32_t pt = tmem + (uint32_t)(buf * 128);
+            const uint64_t vd = desc_swz(smem_u32(sV + (uint32_t)h * kVTile), kVSbo, kVSwz);
+#pragma unroll
+            for (int kk = 0; kk < BM / 16; ++kk)
+              umma_bf16_tmem_a(tmem + 256u + (uint32_t)(h * DH), pt + (uint32_t)((kk >> 2) * 64 + (kk & 3) * 8),
+                               desc_adv(vd, (uint32_t)kk * 16u * kVRow), idesc_pv, kk != 0 ? 1u : 0u);
+            umma_commit(s_free + buf);
+            if (h + 2 < H && !issue_s(h + 2)) break;
+          }
+          if (!ok) break;
+          umma_commit(o_full);
+          // ---- D: A WOx into [0, 128)
+          if (!wait(a2_full, tl & 1)) break;
+          {
+            const int slot = next_slot();
+            if (slot < 0) break;
+            mma_sa(tmem, slot);
+            umma_commit(ox_full);
+          }
+          if (!wait(lnc_full, tl & 1)) break;
+          tc_fence_after();
+        }
+        // ---- E: the head's first layer into [128, 256)
+        {
+          const int slot = next_slot();
+          if (slot < 0) break;
+          mma_sa(tmem + 128u, slot);
+          umma_commit(head_full);
+        }
+      }
+    }
+  } else {
+    // ---------------- gathers, softmax and epilogues (warps 2..9) ----------------
+    const int ew = warp - 2, q = warp & 3, half = ew >> 2;
+    const int et = threadIdx.x - 64;
+    const int r = q * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const float sl2 = p.scale_log2;
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory"); };
+    auto epi_sync = [&]() { asm volatile("bar.sync 5, 256;" ::: "memory"); };
+    bool ok = true;
+    auto wait = [&](uint64_t* bar, uint32_t par) -> bool {
+      if (!mbar_wait_compact(bar, par, p.sel.status)) ok = false;
+      return ok;
+    };
+    int tl = 0, gf = 0;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+      const int b0 = t * G;
+      const int Gv = min(G, p.B - b0);
+      const int rows_v = Gv * K;
+      const bool rvalid = r < rows_v;
+      const int lr = r / K;
+      // ================= A: assembly and the [CLS] attention =================
+      // element row of every occurrence of the tile (-1 for a rejected request)
+      for (int i = et; i < rows_v * L; i += 32 * kEpiWarps) {
+        const int rr = i / L, j = i - rr * L;
+        const int b = b0 + rr / K;
+        int e = -1;
+        if (!p.bad[b]) e = p.off[b] + p.slot[(size_t)(b0 * K + rr) * L + j];
+        sErow[rr * 32 + j] = e;
+      }
+      if (et < G) sFlag[et] = 0;
+      epi_sync();
+      {
+        // lane group g = lane / 8 takes the sequence of row ew + 8 (g0 + g), four
+        // sequences per warp at a time; lane li = lane % 8 of the group owns columns
+        // 16 li .. 16 li + 15 (head hc) and tokens li, li + 8, ... for the softmax
+        const int g = lane >> 3, li = lane & 7;
+        const int hc = (16 * li) / DH;
+#pragma unroll 1
+        for (int g0 = 0; g0 < 16; g0 += 4) {
+          const int rr = ew + 8 * (g0 + g);
+          const bool live = rr < rows_v && sErow[rr * 32] >= 0;  // not a rejected request
+          const bool dead = rr < rows_v && !live;
+          float o[16];
+          // a rejected request's scores become NaN; o = v0 keeps its rows finite
+#pragma unroll
+          for (int i = 0; i < 16; i += 4) {
+            const float4 v0 = dead ? __ldg(reinterpret_cast<const float4*>(p.v0 + 16 * li + i)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            o[i] = v0.x;
+            o[i + 1] = v0.y;
+            o[i + 2] = v0.z;
+            o[i + 3] = v0.w;
+          }
+          // logits of tokens li + 8 t (t < 4), per head, in the log2 domain
+          float sc[4][4];
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const int j = li + 8 * t;
+            float4 pt = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (live && j < L) pt = *reinterpret_cast<const float4*>(p.elog + (size_t)sErow[rr * 32 + j] * 4);
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              const float lg = DH == 32 ? (h == 0 ? pt.x : h == 1 ? pt.y : h == 2 ? pt.z : pt.w)
+                                        : (h == 0 ? pt.x + pt.y : pt.z + pt.w);
+              sc[t][h] = (live && h < H && j < L) ? (lg + sQkP[j * 4 + h]) * sl2 : -INFINITY;
+            }
+          }
+          // softmax over [CLS; L tokens] per head within the group: p[t][h], and [CLS]'s weight for head hc
+          float pw[4][4];
+          float pc = 0.f;
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const float s0 = sQk0[h < H ? h : 0] * sl2;
+            float m = fmaxf(fmaxf(sc[0][h], sc[1][h]), fmaxf(sc[2][h], sc[3][h]));
+            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
+            m = fmaxf(m, s0);
+            float sum = 0.f;
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+              pw[t][h] = ex2_approx(sc[t][h] - m);  // 0 for tokens past L
+              sum += pw[t][h];
+            }
+            sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+            sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+            sum += __shfl_xor_sync(0xffffffffu, sum, 4);
+            const float e0 = ex2_approx(s0 - m);
+            const float inv = 1.f / (sum + e0);
+#pragma unroll
+            for (int t = 0; t < 4; ++t) pw[t][h] *= inv;
+            if (h == hc) pc = e0 * inv;
+          }
+          // the weights through shared memory: [warp][group][token][head]
+          float* pwg = reinterpret_cast<float*>(sV + 16384) + (size_t)(ew * 4 + g) * 128;
+#pragma unroll
+          for (int t = 0; t < 4; ++t)
+            *reinterpret_cast<float4*>(pwg + (li + 8 * t) * 4) = make_float4(pw[t][0], pw[t][1], pw[t][2], pw[t][3]);
+          __syncwarp();
+          if (live) {
+#pragma unroll
+            for (int i = 0; i < 16; i += 4) {
+              const float4 v0 = __ldg(reinterpret_cast<const float4*>(p.v0 + 16 * li + i));
+              o[i] = pc * v0.x;
+              o[i + 1] = pc * v0.y;
+              o[i + 2] = pc * v0.z;
+              o[i + 3] = pc * v0.w;
+            }
+          }
+          // o += sum_j p_j (H_j WVs + P_j WVs): the value rows of four tokens in flight
+          // at a time (f16, 32 bytes per lane)
+#pragma unroll 1
+          for (int j0 = 0; j0 < L; j0 += 4) {
+            uint4 va[4], vb[4];
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+              va[jj] = make_uint4(0u, 0u, 0u, 0u);
+              vb[jj] = va[jj];
+              if (live && j0 + jj < L) {
+                const uint4* src = reinterpret_cast<const uint4*>(
+                    p.v_h + (size_t)sErow[rr * 32 + j0 + jj] * p.ldv + p.voff + 16 * li);
+                va[jj] = src[0];
+                vb[jj] = src[1];
+              }
+            }
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+              const int j = j0 + jj;
+              if (!(live && j < L)) continue;
+              const float w = pwg[j * 4 + hc];
+              const float4* vp = reinterpret_cast<const float4*>(p.vP + (size_t)j * D + 16 * li);
+              const uint32_t wv[8] = {va[jj].x, va[jj].y, va[jj].z, va[jj].w, vb[jj].x, vb[jj].y, vb[jj].z, vb[jj].w};
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const float4 pp = __ldg(vp + i);
+                const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i]));
+                const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i + 1]));
+                o[4 * i] = fmaf(w, a.x + pp.x, o[4 * i]);
+                o[4 * i + 1] = fmaf(w, a.y + pp.y, o[4 * i + 1]);
+                o[4 * i + 2] = fmaf(w, b.x + pp.z, o[4 * i + 2]);
+                o[4 * i + 3] = fmaf(w, b.y + pp.w, o[4 * i + 3]);
+              }
+            }
+          }
+          __syncwarp();  // every lane has read the weights before the next group writes them
+          // o -> row rr of the split tile: columns 16 li .. 16 li + 15 are 16-byte
+          // pieces 2 (li % 4) and 2 (li % 4) + 1 of plane li / 4
+          {
+            uint32_t hi[8], lo[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) split2(o[2 * i], o[2 * i + 1], hi[i], lo[i]);
+            uint8_t* rowp = sA + (size_t)((li >> 2) * 2) * kAPlane + (size_t)rr * 128u;
+            const uint32_t o0 = (uint32_t)((2 * (li & 3)) ^ (rr & 7)) << 4;
+            const uint32_t o1 = (uint32_t)((2 * (li & 3) + 1) ^ (rr & 7)) << 4;
+            *reinterpret_cast<uint4*>(rowp + o0) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+            *reinterpret_cast<uint4*>(rowp + o1) = make_uint4(hi[4], hi[5], hi[6], hi[7]);
+            *reinterpret_cast<uint4*>(rowp + kAPlane + o0) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            *reinterpret_cast<uint4*>(rowp + kAPlane + o1) = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+          }
+        }
+      }
+      // x0 = [CLS] into the accumulator (read by this thread in the previous tile's last phase)
+      tmem_st32_nw(acc2 + lane_off + (uint32_t)(32 * half), sCls + 32 * half);
+      tmem_st32_nw(acc2 + lane_off + (uint32_t)(32 * half + 64), sCls + 32 * half + 64);
+      tmem_st_wait();
+      fence_async_shared();
+      tc_fence_before();
+      arrive1(a_full);
+      // ================= B: c = cls + o WOs, FFN =================
+      {
+        const uint32_t proj = tmem + (uint32_t)((gf % NA1) * FC);
+        if (!wait(o_done, tl & 1)) break;
+        tc_fence_after();
+        epi_resid_ln(sA, red, acc2 + lane_off, true, proj + lane_off, nullptr, nullptr, r, q, half, p.eps);
+        fence_async_shared();
+        tc_fence_before();
+        arrive1(ln_full);
+      }
+      for (int f = 0; f < nf; ++f, ++gf) {
+        const int ba = gf % NA1;
+        if (!wait(acc1_full + ba, (gf / NA1) & 1)) break;
+        tc_fence_after();
+        {
+          const uint32_t col = tmem + lane_off + (uint32_t)(ba * FC + 64 * half);
+          const float* bias = sB1 + f * FC + 64 * half;
+          float v[64];
+          tmem_ld64(col, v);
+#pragma unroll
+          for (int hp = 0; hp < 2; ++hp) {
+            uint32_t hi[16], lo[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+              split2_trunc(relu_keep_nan(v[32 * hp + 2 * j] + bias[32 * hp + 2 * j]),
+                           relu_keep_nan(v[32 * hp + 2 * j + 1] + bias[32 * hp + 2 * j + 1]), hi[j], lo[j]);
+            tmem_st16_nowait(col + (uint32_t)(32 * hp), hi);
+            tmem_st16_nowait(col + (uint32_t)(32 * hp + 16), lo);
+          }
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        arrive1(mid_full + ba);
+      }
+      if (!ok) break;
+      // c = acc2 + b2s; Z = LN(c) (the cross-sequence block's input, or the head's)
+      if (!wait(acc2_full, tl & 1)) break;
+      tc_fence_after();
+      epi_resid_ln(sA, red, acc2 + lane_off, false, 0u, sB2, (p.c_out && rvalid) ? p.c_out + (size_t)(b0 * K + r) * D : nullptr,
+                   r, q, half, p.eps);
+      fence_async_shared();
+      tc_fence_before();
+      arrive1(z_full);
+      if (p.cross) {
+        // ================= C: cross-sequence attention =================
+        if (!wait(qkv_full, tl & 1)) break;
+        tc_fence_after();
+        // Q and K as f16 K-major tiles [kb][128 rows x 128 B] at sA and sA + 32 KB;
+        // V per head as an MN-major tile [128 keys x DH] in sV; a V row with a
+        // non-finite value is written as zeros (P = 0 for other requests' rows
+        // must not meet 0 x NaN) and marks its request
+        bool bad_v = false;
+#pragma unroll 1
+        for (int pc = 0; pc < 6; ++pc) {
+          const int part = pc >> 1, ci = pc & 1;
+          {
+            const int c = 32 * half + 64 * ci;
+            float v[32];
+            tmem_ld32(tmem + lane_off + (uint32_t)(part * 128 + c), v);
+            uint32_t w[16];
+            bool fin = true;
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              if (part == 2) fin = fin && isfinite(v[2 * j]) && isfinite(v[2 * j + 1]);
+              w[j] = pack_f16x2(v[2 * j], v[2 * j + 1]);
+            }
+            if (part < 2) {
+              uint8_t* rowp = sA + (size_t)(part * 2 + c / BK) * kAPlane + (size_t)r * 128u;
+#pragma unroll
+              for (int jj = 0; jj < 4; ++jj) {
+                const uint32_t o = (uint32_t)(((c % BK) / 8 + jj) ^ (r & 7)) << 4;
+                *reinterpret_cast<uint4*>(rowp + o) = make_uint4(w[4 * jj], w[4 * jj + 1], w[4 * jj + 2], w[4 * jj + 3]);
+              }
+            } else {
+              if (!fin) {
+                bad_v = true;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) w[j] = 0u;
+              }
+              const int h = c / DH, cc = c % DH;
+              uint8_t* rowp = sV + (size_t)h * kVTile + (size_t)r * kVRow;
+#pragma unroll
+              for (int jj = 0; jj < 4; ++jj) {
+                const int j16 = cc / 8 + jj;
+                const int sw = DH == 32 ? (j16 ^ ((r >> 1) & 3)) : (j16 ^ (r & 7));
+                *reinterpret_cast<uint4*>(rowp + ((uint32_t)sw << 4)) =
+                    make_uint4(w[4 * jj], w[4 * jj + 1], w[4 * jj + 2], w[4 * jj + 3]);
+              }
+            }
+          }
+        }
+        if (bad_v && rvalid) sFlag[lr] = 1;
+        fence_async_shared();
+        tc_fence_before();
+        arrive1(qkv_ready);
+        // per head: softmax over the row's own request's K keys (keys of other
+        // requests and padding rows take no part: -inf)
+        const int klo = rvalid ? lr * K : 0, khi = rvalid ? lr * K + K : 0;
+        float lh[4] = {1.f, 1.f, 1.f, 1.f};
+        float* rmax = red + 512;  // [half][row]
+        float* rsum = red + 768;
+#pragma unroll 1
+        for (int h = 0; h < H; ++h) {
+          const int g = tl * H + h, buf = g & 1;
+          if (!wait(s_full + buf, (g >> 1) & 1)) break;
+          tc_fence_after();
+          const uint32_t tile = tmem + lane_off + (uint32_t)(buf * 128 + 64 * half);
+          float v[64];
+          tmem_ld64(tile, v);
+          float mx = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < 64; ++i) {
+            const int key = 64 * half + i;
+            if (key < klo || key >= khi) v[i] = -INFINITY;
+            mx = fmaxf(mx, v[i]);
+          }
+          rmax[half * 128 + r] = mx;
+          pair_sync();
+          float m = fmaxf(rmax[r], rmax[128 + r]) * sl2;
+          if (m == -INFINITY) m = 0.f;  // a padding row: every P is 0
+          float s4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int hb = 0; hb < 2; ++hb) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 32; i += 2) {
+              const int k = 32 * hb + i;
+              const float p0 = ex2_approx(fmaf(v[k], sl2, -m));
+              const float p1 = ex2_approx(fmaf(v[k + 1], sl2, -m));
+              s4[(i >> 1) & 3] += p0 + p1;
+              pk[i / 2] = pack_f16x2(p0, p1);
+            }
+            tmem_st16_nowait(tile + (uint32_t)(16 * hb), pk);
+          }
+          rsum[half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+          tmem_st_wait();
+          tc_fence_before();
+          arrive1(p_full + buf);
+          pair_sync();
+          const float lt = rsum[r] + rsum[128 + r];
+          const float lv = lt == 0.f ? 1.f : lt;  // 0 only for a padding row (a NaN stays NaN)
+          lh[0] = h == 0 ? lv : lh[0];
+          lh[1] = h == 1 ? lv : lh[1];
+          lh[2] = h == 2 ? lv : lh[2];
+          lh[3] = h == 3 ? lv : lh[3];
+        }
+        if (!ok) break;
+        // the attention output O_h / l_h as the split A tile of the output projection
+        if (!wait(o_full, tl & 1)) break;
+        tc_fence_after();
+        {
+          float v[64];
+          tmem_ld32x2(tmem + lane_off + 256u + (uint32_t)(32 * half), tmem + lane_off + 256u + (uint32_t)(32 * half + 64),
+                      v, v + 32);
+#pragma unroll
+          for (int ci = 0; ci < 2; ++ci) {
+            const int hh = (32 * half + 64 * ci) / DH;
+            const float inv = 1.f / (hh == 0 ? lh[0] : hh == 1 ? lh[1] : hh == 2 ? lh[2] : lh[3]);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[32 * ci + j] *= inv;
+          }
+          store_split64(sA, r, half, v);
+        }
+        fence_async_shared();
+        tc_fence_before();
+        arrive1(a2_full);
+        // ================= D: C' = c + A WOx, LN(C') =================
+        if (!wait(ox_full, tl & 1)) break;
+        tc_fence_after();
+        epi_resid_ln(sA, red, acc2 + lane_off, true, tmem + lane_off, nullptr,
+                     (p.cp_out && rvalid) ? p.cp_out + (size_t)(b0 * K + r) * D : nullptr, r, q, half, p.eps);
+        fence_async_shared();
+        tc_fence_before();
+        arrive1(lnc_full);
+      }
+      // ================= E: score head and the argmax of Eq. 1 =================
+      if (!wait(head_full, tl & 1)) break;
+      tc_fence_after();
+      {
+        float part = 0.f;
+        {
+          float v[64];
+          tmem_ld32x2(tmem + 128u + lane_off + (uint32_t)(32 * half), tmem + 128u + lane_off + (uint32_t)(32 * half + 64),
+                      v, v + 32);
+#pragma unroll
+          for (int ci = 0; ci < 2; ++ci) {
+            const int c = 32 * half + 64 * ci;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) part = fmaf(relu_keep_nan(v[32 * ci + j] + sB1h[c + j]), sW2h[c + j], part);
+          }
+        }
+        tc_fence_before();
+        red[half * 128 + r] = part;
+        pair_sync();
+        float s = red[r] + red[128 + r] + p.b2h[0];
+        if (rvalid) {
+          const int b = b0 + lr;
+          if (p.bad[b] || sFlag[lr]) s = __int_as_float(0x7fc00000);
+          p.scores[(size_t)(b0 * K + r)] = s;
+          if (p.task_scores) p.task_scores[(size_t)(b0 * K + r)] = s;
+          sSc[r] = s;
+        }
+      }
+      epi_sync();
+      if (et < Gv) {
+        // request et of the tile: the smallest k attaining the maximum; -1 for a
+        // rejected request or a NaN score (the latter also flags the batch)
+        const int b = b0 + et;
+        int best = -1;
+        if (!p.bad[b]) {
+          float mx = -INFINITY;
+          bool nan = false;
+          for (int k = 0; k < K; ++k) {
+            const float v = sSc[et * K + k];
+            if (v != v) {
+              nan = true;
+            } else if (v > mx || best < 0) {
+              mx = v;
+              best = k;
+            }
+          }
+          if (nan) {
+            best = -1;
+            atomicOr(p.sel.status, ST_NUMERIC);
+          }
+        }
+        p.sel.best[b] = best;
+      }
+      epi_sync();
+    }
+  }
+
+  __syncwarp();  // each warp arrives whole: single lanes ran the producer and MMA loops
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(tmem, 512);
+  // the last CTA to finish hands the batch status to the host word and clears
+  // the status and the ticket for the next batch
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) *last_flag = atomicAdd(p.sel.ticket, 1u) == gridDim.x - 1 ? 1u : 0u;
+  __syncthreads();
+  if (*last_flag && threadIdx.x == 0) {
+    __threadfence();
+    const int st = atomicExch(p.sel.status, 0);
+    *p.sel.ticket = 0u;
+    *reinterpret_cast<volatile int*>(p.sel.host_status) = st;
+    __threadfence_system();
+  }
+}
+
+namespace {
+int g_seq_sms = 0;
+}
+
+bool seq_supported(int d, int dh, int F, int nb, int n_tasks, int K, int L) {
+  return d == D && (dh == 32 || dh == 64) && F % FC == 0 && F >= FC && F <= kMaxF && nb == 1 && n_tasks <= 1 &&
+         K >= 1 && K <= BM && L >= 1 && L <= kMaxL;
+}
+
+cudaError_t seq_prepare() {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_seq_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(seq_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(seq_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+  return e;
+}
+
+cudaError_t seq_launch(const CUtensorMap* wos, const CUtensorMap* w1s, const CUtensorMap* w2s,
+                       const CUtensorMap* qkvx, const CUtensorMap* wox, const CUtensorMap* w1h, const SeqParams& p0,
+                       cudaStream_t s) {
+  if (p0.B <= 0 || p0.K <= 0) return cudaSuccess;
+  if (!seq_supported(D, p0.dh, p0.F, 1, 1, p0.K, p0.L) || p0.H * p0.dh != D || p0.G < 1 || p0.G * p0.K > BM)
+    return cudaErrorInvalidValue;
+  const long long tiles = (p0.B + p0.G - 1) / p0.G;
+  long long grid = g_seq_sms > 0 ? g_seq_sms : 148;
+  if (grid > tiles) grid = tiles;
+  // without the cross-sequence block its maps are never read
+  const CUtensorMap* qk = p0.cross ? qkvx : wos;
+  const CUtensorMap* wx = p0.cross ? wox : wos;
+  if (p0.dh == 32)
+    return launch_k(seq_kernel<32>, dim3((unsigned)grid), dim3(kThreads), kSmem, s, *wos, *w1s, *w2s, *qk, *wx, *w1h,
+                    p0);
+  return launch_k(seq_kernel<64>, dim3((unsigned)grid), dim3(kThreads), kSmem, s, *wos, *w1s, *w2s, *qk, *wx, *w1h,
+                  p0);
+}
+
+}  // namespace fe

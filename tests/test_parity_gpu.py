@@ -104,9 +104,11 @@ KV_RTOL, KV_ATOL = 1e-3, 1e-5
 def test_stagewise_serving(dev):
     """Intermediates: context K/V, element cache, SeqEnc and cross-sequence outputs
     (serving runs the fused context kernel, so LN(context) is not materialised)."""
-    from paper_2603_02565_gb300.binding import FeError
+    from paper_2603_02565_gb300.binding import Evaluator, FeError
     w = wl.make_workload("serving", B=2)
-    ev, gs, gb = run_gpu(w, dev)
+    ev = Evaluator(w.cfg, w.weights)
+    ev.keep_intermediates(True)  # c and C' are otherwise kept on chip by the sequence-stage kernel
+    ev, gs, gb = run_gpu(w, dev, ev)
     cfg, W = w.cfg, w.weights
     eps = cfg.ln_eps
     np.testing.assert_allclose(ev.fetch("ctx_kv", cols=2 * cfg.n_layers * cfg.d), context_kv_rows(w, 2),
@@ -123,8 +125,11 @@ def test_stagewise_serving(dev):
         seq.append(Cm)
         cross.append(O.cross_sequence(Cm, W, cfg.n_heads, eps))
     np.testing.assert_allclose(ev.fetch("elem"), np.vstack(elem), rtol=0, atol=2e-4)
-    np.testing.assert_allclose(ev.fetch("seq"), np.vstack(seq), rtol=1e-3, atol=2e-5)
-    np.testing.assert_allclose(ev.fetch("cross"), np.vstack(cross), rtol=1e-3, atol=2e-5)
+    # c and C' come from the [CLS] attention, whose value rows are single f16 planes
+    # like every attention operand (unit roundoff 2^-11 on values of magnitude up to
+    # ~0.2): an absolute error of up to ~1e-4 on c, rtol 1e-3 elsewhere
+    np.testing.assert_allclose(ev.fetch("seq"), np.vstack(seq), rtol=1e-3, atol=1e-4)
+    np.testing.assert_allclose(ev.fetch("cross"), np.vstack(cross), rtol=1e-3, atol=1e-4)
 
 
 @pytest.mark.parametrize("K", [10, 100, 1000])
