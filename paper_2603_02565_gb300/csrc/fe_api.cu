@@ -336,6 +336,7 @@ struct fe_ctx {
   bool keep_inter = false;   // store c and C' even where the sequence-stage kernel keeps them on chip
   int n_sms = 148;
   float* elog = nullptr;     // [rows, d / 32] the elements' [CLS] logit partials (sequence-stage kernel)
+  Planes vI16;               // [rows, d] the elements' SeqEnc value rows H WVs, one f16 plane (sequence-stage kernel)
   CUtensorMap ctxkv_w{};     // W^T of the K/V projection, 64 x 128 boxes, for the fused kernel
   std::vector<void*> owned_w;  // weight allocations
   std::vector<void*> owned_ws; // workspace allocations
@@ -351,6 +352,7 @@ struct fe_ctx {
   float* task_scores = nullptr;     // [S, T], every head's score of the last batch
   float* lin_states = nullptr;      // linear-attention context states [segments][Ly][H][d_h^2 + d_h]
   float *q0 = nullptr, *k0 = nullptr, *v0 = nullptr, *kP = nullptr, *vP = nullptr;
+  float* qk = nullptr;  // [max_L + 1][4]: q0 . kP[j] and q0 . k0 per head (the sequence-stage kernel)
   // workspace
   Shape cap_shape;  // reserved maxima
   int cap_rows = 0; // element rows of the reservation: B * min(M, K*L), or B * K * L once factorized
@@ -613,6 +615,7 @@ int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const We
   p.status = c->status;
   p.tail_q0 = tail_logits ? c->q0 : nullptr;
   p.tail_logits = tail_logits;
+  p.tail_col0 = tail_logits ? c->d : 0;  // the value columns go to their own [rows, d] buffer
   FE_CK(fe::ffn_launch(&A.th, &A.tl, &WO.p.th, &WO.p.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.th, &ln_out.tl,
                        &x.sx, WT ? &WT->fh : nullptr, WT ? &WT->fl : nullptr, tail_out ? &tail_out->sh : nullptr,
                        tail_out ? &tail_out->sl : nullptr, p, s));
@@ -819,7 +822,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
       // LN(x_out) itself is stored when something else reads it (the last layer's: the element encodings)
       const bool last = l == Ly - 1;
       const Weight* WT = !last ? (c->tail_q ? &c->wq[l + 1] : nullptr) : (c->tail_kv ? &c->kvs : nullptr);
-      const Planes* TO = !last ? &c->q : &c->kvI;
+      const Planes* TO = !last ? &c->q : (use_seq ? &c->vI16 : &c->kvI);
       FE_RC(ffn(c, "ffn_item", c->a, c->wo[l], c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), nullptr, c->h,
                 c->xln, R, sumU, s, (last || !c->tail_q) ? 1 : 0, WT, WT ? TO : nullptr,
                 (!last || (use_seq && WT)) ? 1 : 0, (last && use_seq && WT) ? c->elog : nullptr));
@@ -863,14 +866,11 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     sp.bad = c->bad;
     sp.slot = c->slot;
     sp.elog = c->elog;
-    sp.v_h = c->kvI.h;
-    sp.ldv = c->kvI.ld;
-    sp.voff = d;
-    sp.q0 = c->q0;
-    sp.k0 = c->k0;
+    sp.v_h = c->vI16.h;
     sp.v0 = c->v0;
-    sp.kP = c->kP;
     sp.vP = c->vP;
+    sp.qkP = c->qk;
+    sp.qk0 = c->qk + (size_t)c->cfg.max_L * 4;
     sp.cls = tw(c, T_CLS);
     sp.b1s = tw(c, T_B1S);
     sp.b2s = tw(c, T_B2S);
@@ -1097,7 +1097,12 @@ int reserve_body(fe_ctx* c, const Shape& s, const bool fact) {
   c->sel_ticket = reinterpret_cast<unsigned*>(c->sel_nan + B);
   FE_RC(dalloc((void**)&c->slot, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int)));
   FE_RC(dalloc((void**)&c->list, (size_t)R * sizeof(int)));
-  if (c->seq_ok) FE_RC(dalloc((void**)&c->elog, (size_t)R * (size_t)(d / 32) * sizeof(float)));
+  if (c->seq_ok) {
+    FE_RC(dalloc((void**)&c->elog, (size_t)R * (size_t)(d / 32) * sizeof(float)));
+    FE_RC(alloc_planes(c->vI16, R, d, false, c->owned_ws));
+    FE_RC(encode_map_t(&c->vI16.sh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->vI16.h, d, c->vI16.rows, 32, 32,
+                       CU_TENSOR_MAP_SWIZZLE_64B));
+  }
   FE_RC(alloc_f32(c->h, R, d, c->owned_ws));
   FE_RC(alloc_f32(c->c, S, d, c->owned_ws));
   FE_RC(alloc_f32(c->cp, S, d, c->owned_ws));
@@ -1415,18 +1420,21 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   // weight-only products of SeqEnc: [CLS] W and P W
   const int mL = cfg->max_L;
   float* consts = nullptr;
-  if (dev_alloc((void**)&consts, (size_t)(3 + 2 * mL) * d * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+  if (dev_alloc((void**)&consts, ((size_t)(3 + 2 * mL) * d + (size_t)(mL + 1) * 4) * sizeof(float)) != cudaSuccess)
+    return fail(FE_ERR_OOM);
   c->owned_w.push_back(consts);
   c->q0 = consts;
   c->k0 = consts + d;
   c->v0 = consts + 2 * d;
   c->kP = consts + 3 * d;
   c->vP = consts + (size_t)(3 + mL) * d;
+  c->qk = consts + (size_t)(3 + 2 * mL) * d;
   if (fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WQS), d, c->q0, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WKS), d, c->k0, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WVS), d, c->v0, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WKS), d, c->kP, 0) != cudaSuccess ||
-      fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WVS), d, c->vP, 0) != cudaSuccess)
+      fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WVS), d, c->vP, 0) != cudaSuccess ||
+      fe::seq_consts_launch(c->q0, c->k0, c->kP, mL, d, c->dh, c->qk, 0) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "SeqEnc constants"));
   if (host_alloc((void**)&c->host_status, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
   *c->host_status = 0;

@@ -671,7 +671,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               *reinterpret_cast<uint4*>(b + 2048 + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
             }
           }
-          issue(&tTo_h, b, p.tail_f16 ? nullptr : &tTo_l, b + 2048, c, srow);
+          issue(&tTo_h, b, p.tail_f16 ? nullptr : &tTo_l, b + 2048, c - p.tail_col0, srow);
           ++k;
         }
         tc_fence_before();  // TMEM read before r_empty lets the next tile's projection in

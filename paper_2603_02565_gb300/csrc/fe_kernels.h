@@ -138,6 +138,7 @@ struct FfnParams {
   // tail_logits[row * (d / 32) + g] (fp32); the value columns are stored as usual.
   const float* tail_q0;
   float* tail_logits;
+  int tail_col0;        // tail output column c is stored at column c - tail_col0 of the output map
 };
 bool ffn_supported(int d, int d_pad, int F, int nb);
 bool ffn_tail_supported(int d, int d_pad, int F, int nb, int tail_n, int tail_f16);
@@ -314,9 +315,9 @@ struct SeqParams {
   const int* bad;            // [B]
   const int* slot;           // [B, K, L] request-local slots
   const float* elog;         // [rows, d / 32] per-32-column [CLS] logit partials q0 . (H WKs)
-  const bf16* v_h;           // element values H WVs, one f16 plane (bits), row stride ldv, at column voff
-  int ldv, voff;
-  const float *q0, *k0, *v0, *kP, *vP;  // [CLS] WQs / WKs / WVs, P WKs, P WVs
+  const bf16* v_h;           // element values H WVs, one f16 plane (bits), [rows, d] row-major
+  const float *v0, *vP;      // [CLS] WVs, P WVs [max_L, d]
+  const float *qkP, *qk0;    // q0 . (P WKs)_j per head [j][4] and q0 . ([CLS] WKs) per head [4], q0 = [CLS] WQs
   const float *cls, *b1s, *b2s, *b1h, *w2h, *b2h;
   int cross;                 // 0: no cross-sequence block (C' = C)
   float eps;
@@ -328,6 +329,10 @@ struct SeqParams {
   SelArgs sel;               // best, status, host status, ticket (keys / nan unused)
 };
 bool seq_supported(int d, int dh, int F, int nb, int n_tasks, int K, int L);
+// the weight-only [CLS] logits of the kernel: out[j * 4 + h] = q0 . kP[j] over head h
+// (j < max_L), out[max_L * 4 + h] = q0 . k0 over head h
+cudaError_t seq_consts_launch(const float* q0, const float* k0, const float* kP, int max_L, int d, int dh, float* out,
+                              cudaStream_t s);
 cudaError_t seq_prepare();
 cudaError_t seq_launch(const CUtensorMap* wos, const CUtensorMap* w1s, const CUtensorMap* w2s,
                        const CUtensorMap* qkvx, const CUtensorMap* wox, const CUtensorMap* w1h, const SeqParams& p,

@@ -23,8 +23,8 @@
 //   D  C' = c + A WOx; LN(C')
 //   E  s = ReLU(LN(C') W1h + b1h) . w2h + b2h; per request the smallest k
 //      attaining the maximum
-// Roles: warp 0 lane 0 streams the weights (32 KB chunks in consumption order
-// through a ring of three slots, by TMA), warp 1 lane 0 issues tcgen05.mma,
+// Roles: warp 0 lane 0 streams the weights (16 KB boxes, two per 128 x 128
+// chunk, in consumption order through a ring of seven slots, by TMA), warp 1 lane 0 issues tcgen05.mma,
 // warps 2-9 run the gathers, softmaxes and epilogues (two warps per TMEM lane
 // quadrant, each owning half of a row's columns).  Products take split
 // bf16 activations (hi + lo) times exact bf16 weights with fp32 accumulation;
@@ -48,11 +48,14 @@ constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
 constexpr int kMaxL = 31;
 constexpr int kMaxF = 1024;
 constexpr uint32_t kAPlane = BM * BK * 2;  // 16 KB: 128 rows x 64 bf16
-constexpr uint32_t kChunk = 2 * kAPlane;   // a weight chunk: two 128-row x 64-column boxes
-constexpr int kRing = 3;
+constexpr uint32_t kBox = kAPlane;         // a weight box: 128 rows x 64 columns (a chunk is two)
+constexpr int kRing = 7;                   // weight box slots
+constexpr int kStageSlot = 2;              // slots 2..6 also stage the tile's element rows during the gathers
+constexpr int NST = 240;                   // element rows staged: f16 values (256 B) + logit partials (16 B),
+                                           // then the L rows of P WVs (fp32, 512 B each)
 constexpr uint32_t kOffV = 4 * kAPlane;               // 64 KB: the split A tile [kb][plane]
 constexpr uint32_t kOffRing = kOffV + 32768;          // the V tiles, one per head
-constexpr uint32_t kOffMisc = kOffRing + kRing * kChunk;
+constexpr uint32_t kOffMisc = kOffRing + kRing * kBox;
 // misc: b1s [kMaxF], b2s, cls, b1h, w2h [D], q0.kP [32][4], q0.k0 [4], row-statistic
 // exchange [4][2][128], scores [128], request flags [128], barriers, TMEM slot
 constexpr uint32_t kMiscB1 = 0;
@@ -63,7 +66,8 @@ constexpr uint32_t kMiscW2h = kMiscB1h + D * 4;
 constexpr uint32_t kMiscQkP = kMiscW2h + D * 4;
 constexpr uint32_t kMiscQk0 = kMiscQkP + 32 * 4 * 4;
 constexpr uint32_t kMiscRed = kMiscQk0 + 64;
-constexpr uint32_t kMiscSc = kMiscRed + 4 * 2 * 128 * 4;
+constexpr uint32_t kMiscV0 = kMiscRed + 4 * 2 * 128 * 4;   // [CLS] WVs [D], then b2h
+constexpr uint32_t kMiscSc = kMiscV0 + D * 4 + 16;
 constexpr uint32_t kMiscFlag = kMiscSc + 128 * 4;
 constexpr uint32_t kMiscBars = kMiscFlag + 128 * 4;
 constexpr uint32_t kMiscBytes = kMiscBars + 64 * 8 + 64;
@@ -116,6 +120,15 @@ __device__ __forceinline__ ChunkSrc chunk_of(int i, int nf, int cross) {
     r -= 4;
   }
   return {5, 0};
+}
+
+// Contiguous bytes global -> shared by the copy engine, completion on an mbarrier
+// (16-byte aligned addresses, a multiple of 16 bytes).
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
 }
 
 // Two 32-column pieces of this warp's 32 TMEM lanes (row = lane) into
@@ -247,20 +260,18 @@ __device__ __noinline__ void epi_resid_ln(uint8_t* sA, float* red, uint32_t acc_
   if (add || bias) tmem_st_wait();
 }
 
-// D = (split A tile at sA) . (weight chunk at w)^T, N = 128, K = 128: the
-// products of every weight chunk but FFN2's (one copy of the issue code).
-__device__ __noinline__ void mma_tile(uint32_t dst, uint32_t sa, uint32_t w, uint32_t idesc) {
+// D (+)= (64-column block of the split A tile: hi plane at sa, lo plane at
+// sa + 16 KB) . (weight box at w)^T, N = 128: eight products, one copy of the
+// issue code for every weight chunk but FFN2's.
+__device__ __noinline__ void mma_half(uint32_t dst, uint32_t sa, uint32_t w, uint32_t idesc, bool acc) {
   const uint64_t a0 = umma_desc_sw128(sa);
   const uint64_t w0 = umma_desc_sw128(w);
 #pragma unroll
-  for (int kb = 0; kb < 2; ++kb) {
-#pragma unroll
-    for (int kk = 0; kk < BK / 16; ++kk) {
-      const uint64_t ah = desc_adv(a0, (uint32_t)(kb * 2) * kAPlane + kk * 32);
-      const uint64_t wh = desc_adv(w0, (uint32_t)kb * kAPlane + kk * 32);
-      umma_bf16(dst, ah, wh, idesc, (kb | kk) != 0 ? 1u : 0u);
-      umma_bf16(dst, desc_adv(ah, kAPlane), wh, idesc, 1u);
-    }
+  for (int kk = 0; kk < BK / 16; ++kk) {
+    const uint64_t ah = desc_adv(a0, kk * 32);
+    const uint64_t wh = desc_adv(w0, kk * 32);
+    umma_bf16(dst, ah, wh, idesc, (acc || kk != 0) ? 1u : 0u);
+    umma_bf16(dst, desc_adv(ah, kAPlane), wh, idesc, 1u);
   }
 }
 
@@ -293,32 +304,34 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* sQk0 = reinterpret_cast<float*>(misc + kMiscQk0);  // [4]: q0 . k0 per head
   float* red = reinterpret_cast<float*>(misc + kMiscRed);   // [slot][half][row]
   float* sSc = reinterpret_cast<float*>(misc + kMiscSc);
+  float* sV0 = reinterpret_cast<float*>(misc + kMiscV0);
   int* sFlag = reinterpret_cast<int*>(misc + kMiscFlag);    // request of the tile has a non-finite value row
   int* sErow = reinterpret_cast<int*>(sV);                  // during the gathers: [row][32] element rows,
                                                             // then the token weights at sV + 16 KB
   uint64_t* bars = reinterpret_cast<uint64_t*>(misc + kMiscBars);
   uint64_t* w_full = bars;            // [kRing]
-  uint64_t* w_empty = bars + 3;       // [kRing]
-  uint64_t* a_full = bars + 6;        // o written in sA
-  uint64_t* o_done = bars + 7;        // o WOs complete
-  uint64_t* ln_full = bars + 8;       // x in the accumulator, LN(x) in sA
-  uint64_t* acc1_full = bars + 9;     // [NA1]
-  uint64_t* acc1_empty = bars + 12;   // [NA1]
-  uint64_t* mid_full = bars + 15;     // [NA1]
-  uint64_t* acc2_full = bars + 18;    // the FFN complete
-  uint64_t* z_full = bars + 19;       // c in the accumulator, LN(c) in sA
-  uint64_t* qkv_full = bars + 20;     // the Q | K | V product complete
-  uint64_t* qkv_ready = bars + 21;    // Q, K in sA and V in sV
-  uint64_t* s_full = bars + 22;       // [2]
-  uint64_t* p_full = bars + 24;       // [2]
-  uint64_t* s_free = bars + 26;       // [2] PV has read the S/P buffer
-  uint64_t* o_full = bars + 28;       // every head's PV complete
-  uint64_t* a2_full = bars + 29;      // attention output in sA
-  uint64_t* ox_full = bars + 30;      // A WOx complete
-  uint64_t* lnc_full = bars + 31;     // LN(C') in sA
-  uint64_t* head_full = bars + 32;    // the head product complete
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 40);
-  volatile uint32_t* last_flag = reinterpret_cast<volatile uint32_t*>(bars + 41);
+  uint64_t* w_empty = bars + 8;       // [kRing]
+  uint64_t* a_full = bars + 16;       // o written in sA
+  uint64_t* o_done = bars + 17;       // o WOs complete
+  uint64_t* ln_full = bars + 18;      // x in the accumulator, LN(x) in sA
+  uint64_t* acc1_full = bars + 19;    // [NA1]
+  uint64_t* acc1_empty = bars + 22;   // [NA1]
+  uint64_t* mid_full = bars + 25;     // [NA1]
+  uint64_t* acc2_full = bars + 28;    // the FFN complete
+  uint64_t* z_full = bars + 29;       // c in the accumulator, LN(c) in sA
+  uint64_t* qkv_full = bars + 30;     // the Q | K | V product complete
+  uint64_t* qkv_ready = bars + 31;    // Q, K in sA and V in sV
+  uint64_t* s_full = bars + 32;       // [2]
+  uint64_t* p_full = bars + 34;       // [2]
+  uint64_t* s_free = bars + 36;       // [2] PV has read the S/P buffer
+  uint64_t* o_full = bars + 38;       // every head's PV complete
+  uint64_t* a2_full = bars + 39;      // attention output in sA
+  uint64_t* ox_full = bars + 40;      // A WOx complete
+  uint64_t* lnc_full = bars + 41;     // LN(C') in sA
+  uint64_t* head_full = bars + 42;    // the head product complete
+  uint64_t* st_full = bars + 43;      // the tile's element rows staged
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 48);
+  volatile uint32_t* last_flag = reinterpret_cast<volatile uint32_t*>(bars + 49);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = p.K, L = p.L, G = p.G, F = p.F;
@@ -353,6 +366,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(ox_full, 1);
     mbar_init(lnc_full, 32 * kEpiWarps);
     mbar_init(head_full, 1);
+    mbar_init(st_full, 1);
     fence_mbar_init();
     prefetch_tmap(&tWOs);
     prefetch_tmap(&tW1s);
@@ -368,19 +382,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     sCls[i] = p.cls[i];
     sB1h[i] = p.b1h[i];
     sW2h[i] = p.w2h[i];
+    sV0[i] = p.v0[i];
   }
-  // the [CLS] query's logits against [CLS] itself and against each position
-  // embedding's key part, per head (unscaled)
-  for (int i = threadIdx.x; i < (L + 1) * H; i += kThreads) {
-    const int j = i / H, h = i - j * H;
-    const float* kv = j < L ? p.kP + (size_t)j * D : p.k0;
-    float acc = 0.f;
-    for (int c = h * DH; c < h * DH + DH; ++c) acc = fmaf(p.q0[c], kv[c], acc);
-    if (j < L)
-      sQkP[j * 4 + h] = acc;
-    else
-      sQk0[h] = acc;
-  }
+  if (threadIdx.x == 0) sV0[D] = p.b2h[0];
+  // the [CLS] query's logits against each position embedding's key part and
+  // against [CLS] itself, per head (unscaled; weight-only constants)
+  for (int i = threadIdx.x; i < L * 4; i += kThreads) sQkP[i] = p.qkP[i];
+  if (threadIdx.x < 4) sQk0[threadIdx.x] = p.qk0[threadIdx.x];
   // TMEM: FFN1 chunk buffers [128 i, 128 i + 128), i < 3 (later Q | K | V, then the
   // S/P buffers [0, 256) with the attention output at [256, 384), then A WOx at
   // [0, 128) and the head product at [128, 256)); the d-column accumulator of
@@ -397,11 +405,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer: the weight chunks of every tile ----------------
-      int ws = 0;
+      int ws = 0, tl = 0;
       bool ok = true;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        for (int i = 0; i < nch; ++i, ++ws) {
+      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
+        bool gathered = false;  // the tile's gathers are done: the staging slots are weight slots again
+        for (int ib = 0; ib < 2 * nch; ++ib, ++ws) {
+          const int i = ib >> 1, box = ib & 1;
           const int slot = ws % kRing;
+          if (slot >= kStageSlot && !gathered) {
+            if (!mbar_wait_compact(a_full, tl & 1, p.sel.status)) {
+              ok = false;
+              break;
+            }
+            gathered = true;
+          }
           if (ws >= kRing && !mbar_wait_compact(w_empty + slot, ((ws / kRing) - 1) & 1, p.sel.status)) {
             ok = false;
             break;
@@ -424,10 +441,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           } else if (cs.kind == 5) {
             m = &tW1h;
           }
-          uint8_t* dst = sR + (size_t)slot * kChunk;
-          mbar_arrive_expect_tx(w_full + slot, kChunk);
-          tma_load_2d(dst, m, x0, y, w_full + slot);
-          tma_load_2d(dst + kAPlane, m, x1, y, w_full + slot);
+          mbar_arrive_expect_tx(w_full + slot, kBox);
+          tma_load_2d(sR + (size_t)slot * kBox, m, box ? x1 : x0, y, w_full + slot);
         }
       }
     }
@@ -443,29 +458,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait_compact(bar, par, p.sel.status)) ok = false;
         return ok;
       };
-      // the next weight chunk landed: its slot
-      auto next_slot = [&]() -> int {
+      // the next weight box landed: its shared-memory address (0 on a timeout)
+      auto next_box = [&]() -> uint32_t {
         const int slot = ws % kRing;
-        if (!wait(w_full + slot, (ws / kRing) & 1)) return -1;
+        if (!wait(w_full + slot, (ws / kRing) & 1)) return 0u;
         tc_fence_after();
-        return slot;
+        return smem_u32(sR + (size_t)slot * kBox);
       };
-      // dst = (split A tile in sA) . (weight chunk in `slot`)^T, N = 128, K = 128
-      auto mma_sa = [&](uint32_t dst, int slot) {
-        mma_tile(dst, smem_u32(sA), smem_u32(sR + (size_t)slot * kChunk), idesc);
-        umma_commit(w_empty + slot);
+      // the box's slot is free once the products issued so far complete
+      auto release_box = [&]() {
+        umma_commit(w_empty + ws % kRing);
         ++ws;
+      };
+      // dst = (split A tile in sA) . (the next weight chunk)^T, N = 128, K = 128,
+      // box by box: each box's slot is released after its eight products
+      auto mma_sa = [&](uint32_t dst) -> bool {
+        for (int kb = 0; kb < 2; ++kb) {
+          const uint32_t w = next_box();
+          if (!w) return false;
+          mma_half(dst, smem_u32(sA) + (uint32_t)(kb * 2) * kAPlane, w, idesc, kb != 0);
+          release_box();
+        }
+        return true;
       };
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
         // ---- B: o WOs into the FFN1 buffer that chunk 0 of this tile uses next
         if (!wait(a_full, tl & 1)) break;
         {
           const int bo = gf % NA1;
-          const int slot = next_slot();
-          if (slot < 0) break;
           if (gf >= NA1 && !wait(acc1_empty + bo, ((gf / NA1) - 1) & 1)) break;
           tc_fence_after();
-          mma_sa(tmem + (uint32_t)(bo * FC), slot);
+          if (!mma_sa(tmem + (uint32_t)(bo * FC))) break;
           umma_commit(o_done);
         }
         // ---- B: FFN1 / FFN2 once x is in the accumulator and LN(x) in sA
@@ -476,31 +499,35 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (s < nf) {
             const int g = gf0 + s, b = g % NA1;
             if (s > 0 && g >= NA1 && !wait(acc1_empty + b, ((g / NA1) - 1) & 1)) break;
-            const int slot = next_slot();
-            if (slot < 0) break;
-            mma_sa(tmem + (uint32_t)(b * FC), slot);
+            if (!mma_sa(tmem + (uint32_t)(b * FC))) break;
             umma_commit(acc1_full + b);
           }
           if (s >= LA) {
             const int c = s - LA, g = gf0 + c, b = g % NA1;
             if (!wait(mid_full + b, (g / NA1) & 1)) break;
-            const int slot = next_slot();
-            if (slot < 0) break;
             // each 32-column piece of the buffer: 32 hidden units as the hi plane
-            // (16 columns of bf16 pairs) then the lo plane; the W2s chunk holds two
-            // 64-column halves of the chunk's hidden units, 128 output rows each
+            // (16 columns of bf16 pairs) then the lo plane; the W2s chunk's two boxes
+            // are 64-column halves of the chunk's hidden units, 128 output rows each
             const uint32_t mt = tmem + (uint32_t)(b * FC);
-            const uint64_t w0 = umma_desc_sw128(smem_u32(sR + (size_t)slot * kChunk));
+            bool got = true;
+            for (int hh = 0; hh < 2; ++hh) {
+              const uint32_t w = next_box();
+              if (!w) {
+                got = false;
+                break;
+              }
+              const uint64_t w0 = umma_desc_sw128(w);
 #pragma unroll
-            for (int kk = 0; kk < FC / 16; ++kk) {
-              const int hh = kk >> 2, k4 = kk & 3;
-              const uint32_t mh = mt + (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1)), ml = mh + 16;
-              const uint64_t wh = desc_adv(w0, (uint32_t)hh * kAPlane + k4 * 32);
-              umma_bf16_tmem_a(acc2, mh, wh, idesc, 1u);
-              umma_bf16_tmem_a(acc2, ml, wh, idesc, 1u);
+              for (int k4 = 0; k4 < 4; ++k4) {
+                const int kk = 4 * hh + k4;
+                const uint32_t mh = mt + (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1)), ml = mh + 16;
+                const uint64_t wh = desc_adv(w0, (uint32_t)k4 * 32);
+                umma_bf16_tmem_a(acc2, mh, wh, idesc, 1u);
+                umma_bf16_tmem_a(acc2, ml, wh, idesc, 1u);
+              }
+              release_box();
             }
-            umma_commit(w_empty + slot);
-            ++ws;
+            if (!got) break;
             umma_commit(acc1_empty + b);
             if (c == nf - 1) umma_commit(acc2_full);
           }
@@ -511,11 +538,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         if (p.cross) {
           // ---- C: Q | K | V = Z [WQx | WKx | WVx] into TMEM [0, 384)
-          for (int i = 0; i < 3 && ok; ++i) {
-            const int slot = next_slot();
-            if (slot < 0) break;
-            mma_sa(tmem + (uint32_t)(i * 128), slot);
-          }
+          for (int i = 0; i < 3 && ok; ++i)
+            if (!mma_sa(tmem + (uint32_t)(i * 128))) break;
           if (!ok) break;
           umma_commit(qkv_full);
           if (!wait(qkv_ready, tl & 1)) break;
@@ -557,22 +581,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           umma_commit(o_full);
           // ---- D: A WOx into [0, 128)
           if (!wait(a2_full, tl & 1)) break;
-          {
-            const int slot = next_slot();
-            if (slot < 0) break;
-            mma_sa(tmem, slot);
-            umma_commit(ox_full);
-          }
+          if (!mma_sa(tmem)) break;
+          umma_commit(ox_full);
           if (!wait(lnc_full, tl & 1)) break;
           tc_fence_after();
         }
         // ---- E: the head's first layer into [128, 256)
-        {
-          const int slot = next_slot();
-          if (slot < 0) break;
-          mma_sa(tmem + 128u, slot);
-          umma_commit(head_full);
-        }
+        if (!mma_sa(tmem + 128u)) break;
+        umma_commit(head_full);
       }
     }
   } else {
@@ -597,6 +613,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool rvalid = r < rows_v;
       const int lr = r / K;
       // ================= A: assembly and the [CLS] attention =================
+      // the tile's element rows [e0, e0 + nst) to shared memory by two bulk copies
+      // (values, logit partials), over weight slots 2..6, which the producer
+      // leaves alone until the gathers are done; rows past NST are read from memory
+      uint8_t* sStage = sR + (size_t)kStageSlot * kBox;
+      const int e0 = p.off[b0];
+      const int nst = min(p.off[b0 + Gv] - e0, NST);
+      const float* sVP = reinterpret_cast<const float*>(sStage + NST * 272);
+      if (et == 0) {
+        mbar_arrive_expect_tx(st_full, (uint32_t)nst * 272u + (uint32_t)L * (D * 4));
+        if (nst > 0) {
+          bulk_g2s(sStage, p.v_h + (size_t)e0 * D, (uint32_t)nst * 256u, st_full);
+          bulk_g2s(sStage + NST * 256, p.elog + (size_t)e0 * 4, (uint32_t)nst * 16u, st_full);
+        }
+        bulk_g2s(sStage + NST * 272, p.vP, (uint32_t)L * (D * 4), st_full);
+      }
       // element row of every occurrence of the tile (-1 for a rejected request)
       for (int i = et; i < rows_v * L; i += 32 * kEpiWarps) {
         const int rr = i / L, j = i - rr * L;
@@ -605,14 +636,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!p.bad[b]) e = p.off[b] + p.slot[(size_t)(b0 * K + rr) * L + j];
         sErow[rr * 32 + j] = e;
       }
-      if (et < G) sFlag[et] = 0;
+      if (et < G) sFlag[et] = (et < Gv && p.bad[b0 + et]) ? 2 : 0;  // bit 1: a rejected request
       epi_sync();
+      if (!wait(st_full, tl & 1)) break;
       {
         // lane group g = lane / 8 takes the sequence of row ew + 8 (g0 + g), four
         // sequences per warp at a time; lane li = lane % 8 of the group owns columns
         // 16 li .. 16 li + 15 (head hc) and tokens li, li + 8, ... for the softmax
         const int g = lane >> 3, li = lane & 7;
         const int hc = (16 * li) / DH;
+        // this lane's 16 value columns of element row e: staged, or in memory
+        auto vrow = [&](int e) -> const uint4* {
+          const int er = e - e0;
+          return (unsigned)er < (unsigned)nst ? reinterpret_cast<const uint4*>(sStage + (size_t)er * 256 + 32 * li)
+                                              : reinterpret_cast<const uint4*>(p.v_h + (size_t)e * D + 16 * li);
+        };
 #pragma unroll 1
         for (int g0 = 0; g0 < 16; g0 += 4) {
           const int rr = ew + 8 * (g0 + g);
@@ -622,27 +660,49 @@ __global__ void __launch_bounds__(kThreads, 1)
           // a rejected request's scores become NaN; o = v0 keeps its rows finite
 #pragma unroll
           for (int i = 0; i < 16; i += 4) {
-            const float4 v0 = dead ? __ldg(reinterpret_cast<const float4*>(p.v0 + 16 * li + i)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 v0 = dead ? *reinterpret_cast<const float4*>(sV0 + 16 * li + i) : make_float4(0.f, 0.f, 0.f, 0.f);
             o[i] = v0.x;
             o[i + 1] = v0.y;
             o[i + 2] = v0.z;
             o[i + 3] = v0.w;
           }
-          // logits of tokens li + 8 t (t < 4), per head, in the log2 domain
+          // every load of the group first: the logit partials of tokens li + 8 t
+          // (t < 4) and the value rows of tokens 0 .. 7 (f16, 32 bytes per lane)
+          float4 pt[4];
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const int j = li + 8 * t;
+            pt[t] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (live && j < L) {
+              const int e = sErow[rr * 32 + j], er = e - e0;
+              pt[t] = *((unsigned)er < (unsigned)nst ? reinterpret_cast<const float4*>(sStage + NST * 256 + er * 16)
+                                                    : reinterpret_cast<const float4*>(p.elog + (size_t)e * 4));
+            }
+          }
+          uint4 va[8], vb[8];
+#pragma unroll
+          for (int jj = 0; jj < 8; ++jj) {
+            va[jj] = make_uint4(0u, 0u, 0u, 0u);
+            vb[jj] = va[jj];
+            if (live && jj < L) {
+              const uint4* src = vrow(sErow[rr * 32 + jj]);
+              va[jj] = src[0];
+              vb[jj] = src[1];
+            }
+          }
+          // logits per head, in the log2 domain
           float sc[4][4];
 #pragma unroll
           for (int t = 0; t < 4; ++t) {
             const int j = li + 8 * t;
-            float4 pt = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (live && j < L) pt = *reinterpret_cast<const float4*>(p.elog + (size_t)sErow[rr * 32 + j] * 4);
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
-              const float lg = DH == 32 ? (h == 0 ? pt.x : h == 1 ? pt.y : h == 2 ? pt.z : pt.w)
-                                        : (h == 0 ? pt.x + pt.y : pt.z + pt.w);
+              const float lg = DH == 32 ? (h == 0 ? pt[t].x : h == 1 ? pt[t].y : h == 2 ? pt[t].z : pt[t].w)
+                                        : (h == 0 ? pt[t].x + pt[t].y : pt[t].z + pt[t].w);
               sc[t][h] = (live && h < H && j < L) ? (lg + sQkP[j * 4 + h]) * sl2 : -INFINITY;
             }
           }
-          // softmax over [CLS; L tokens] per head within the group: p[t][h], and [CLS]'s weight for head hc
+          // softmax over [CLS; L tokens] per head within the group: pw[t][h], and [CLS]'s weight for head hc
           float pw[4][4];
           float pc = 0.f;
 #pragma unroll
@@ -677,46 +737,49 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (live) {
 #pragma unroll
             for (int i = 0; i < 16; i += 4) {
-              const float4 v0 = __ldg(reinterpret_cast<const float4*>(p.v0 + 16 * li + i));
+              const float4 v0 = *reinterpret_cast<const float4*>(sV0 + 16 * li + i);
               o[i] = pc * v0.x;
               o[i + 1] = pc * v0.y;
               o[i + 2] = pc * v0.z;
               o[i + 3] = pc * v0.w;
             }
           }
-          // o += sum_j p_j (H_j WVs + P_j WVs): the value rows of four tokens in flight
-          // at a time (f16, 32 bytes per lane)
-#pragma unroll 1
-          for (int j0 = 0; j0 < L; j0 += 4) {
-            uint4 va[4], vb[4];
+          // o += sum_j p_j (H_j WVs + P_j WVs): tokens 0 .. 7 from the loads above,
+          // longer sequences four further tokens at a time
+          auto accumulate = [&](int j, const uint4& a4, const uint4& b4) {
+            const float w = pwg[j * 4 + hc];
+            const float4* vp = reinterpret_cast<const float4*>(sVP + (size_t)j * D + 16 * li);
+            const uint32_t wv[8] = {a4.x, a4.y, a4.z, a4.w, b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
-            for (int jj = 0; jj < 4; ++jj) {
-              va[jj] = make_uint4(0u, 0u, 0u, 0u);
-              vb[jj] = va[jj];
-              if (live && j0 + jj < L) {
-                const uint4* src = reinterpret_cast<const uint4*>(
-                    p.v_h + (size_t)sErow[rr * 32 + j0 + jj] * p.ldv + p.voff + 16 * li);
-                va[jj] = src[0];
-                vb[jj] = src[1];
-              }
+            for (int i = 0; i < 4; ++i) {
+              const float4 pp = vp[i];
+              const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i]));
+              const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i + 1]));
+              o[4 * i] = fmaf(w, a.x + pp.x, o[4 * i]);
+              o[4 * i + 1] = fmaf(w, a.y + pp.y, o[4 * i + 1]);
+              o[4 * i + 2] = fmaf(w, b.x + pp.z, o[4 * i + 2]);
+              o[4 * i + 3] = fmaf(w, b.y + pp.w, o[4 * i + 3]);
             }
+          };
+          if (live) {
 #pragma unroll
-            for (int jj = 0; jj < 4; ++jj) {
-              const int j = j0 + jj;
-              if (!(live && j < L)) continue;
-              const float w = pwg[j * 4 + hc];
-              const float4* vp = reinterpret_cast<const float4*>(p.vP + (size_t)j * D + 16 * li);
-              const uint32_t wv[8] = {va[jj].x, va[jj].y, va[jj].z, va[jj].w, vb[jj].x, vb[jj].y, vb[jj].z, vb[jj].w};
+            for (int jj = 0; jj < 8; ++jj)
+              if (jj < L) accumulate(jj, va[jj], vb[jj]);
+#pragma unroll 1
+            for (int j0 = 8; j0 < L; j0 += 4) {
 #pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                const float4 pp = __ldg(vp + i);
-                const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i]));
-                const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i + 1]));
-                o[4 * i] = fmaf(w, a.x + pp.x, o[4 * i]);
-                o[4 * i + 1] = fmaf(w, a.y + pp.y, o[4 * i + 1]);
-                o[4 * i + 2] = fmaf(w, b.x + pp.z, o[4 * i + 2]);
-                o[4 * i + 3] = fmaf(w, b.y + pp.w, o[4 * i + 3]);
+              for (int jj = 0; jj < 4; ++jj) {
+                va[jj] = make_uint4(0u, 0u, 0u, 0u);
+                vb[jj] = va[jj];
+                if (j0 + jj < L) {
+                  const uint4* src = vrow(sErow[rr * 32 + j0 + jj]);
+                  va[jj] = src[0];
+                  vb[jj] = src[1];
+                }
               }
+#pragma unroll
+              for (int jj = 0; jj < 4; ++jj)
+                if (j0 + jj < L) accumulate(j0 + jj, va[jj], vb[jj]);
             }
           }
           __syncwarp();  // every lane has read the weights before the next group writes them
@@ -834,7 +897,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        if (bad_v && rvalid) sFlag[lr] = 1;
+        if (bad_v && rvalid) atomicOr(sFlag + lr, 1);  // bit 0: a non-finite value row
         fence_async_shared();
         tc_fence_before();
         arrive1(qkv_ready);
@@ -937,39 +1000,47 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         red[half * 128 + r] = part;
         pair_sync();
-        float s = red[r] + red[128 + r] + p.b2h[0];
+        float s = red[r] + red[128 + r] + sV0[D];
         if (rvalid) {
-          const int b = b0 + lr;
-          if (p.bad[b] || sFlag[lr]) s = __int_as_float(0x7fc00000);
+          if (sFlag[lr]) s = __int_as_float(0x7fc00000);
           p.scores[(size_t)(b0 * K + r)] = s;
           if (p.task_scores) p.task_scores[(size_t)(b0 * K + r)] = s;
           sSc[r] = s;
         }
       }
       epi_sync();
-      if (et < Gv) {
-        // request et of the tile: the smallest k attaining the maximum; -1 for a
-        // rejected request or a NaN score (the latter also flags the batch)
-        const int b = b0 + et;
-        int best = -1;
-        if (!p.bad[b]) {
-          float mx = -INFINITY;
-          bool nan = false;
-          for (int k = 0; k < K; ++k) {
-            const float v = sSc[et * K + k];
-            if (v != v) {
-              nan = true;
-            } else if (v > mx || best < 0) {
-              mx = v;
-              best = k;
-            }
-          }
-          if (nan) {
-            best = -1;
-            atomicOr(p.sel.status, ST_NUMERIC);
+      // request lr2 of the tile, one warp each: the smallest k attaining the
+      // maximum; -1 for a rejected request or a NaN score (the latter also flags
+      // the batch)
+      for (int lr2 = ew; lr2 < Gv; lr2 += kEpiWarps) {
+        float mx = -INFINITY;
+        int bk = 0x7FFFFFFF;
+        bool nan = false;
+        for (int k = lane; k < K; k += 32) {
+          const float v = sSc[lr2 * K + k];
+          if (v != v)
+            nan = true;
+          else if (v > mx || bk == 0x7FFFFFFF) {
+            mx = v;
+            bk = k;
           }
         }
-        p.sel.best[b] = best;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float om = __shfl_xor_sync(0xffffffffu, mx, o);
+          const int ok2 = __shfl_xor_sync(0xffffffffu, bk, o);
+          if (ok2 != 0x7FFFFFFF && (bk == 0x7FFFFFFF || om > mx || (om == mx && ok2 < bk))) {
+            mx = om;
+            bk = ok2;
+          }
+        }
+        nan = __any_sync(0xffffffffu, nan);
+        if (lane == 0) {
+          const bool rejected = (sFlag[lr2] & 2) != 0;
+          const int best = (nan || rejected) ? -1 : bk;
+          if (nan && !rejected) atomicOr(p.sel.status, ST_NUMERIC);
+          p.sel.best[b0 + lr2] = best;
+        }
       }
       epi_sync();
     }
@@ -992,6 +1063,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     *reinterpret_cast<volatile int*>(p.sel.host_status) = st;
     __threadfence_system();
   }
+}
+
+// q0 . kP[j] per head (out[j * 4 + h], j < max_L) and q0 . k0 per head
+// (out[max_L * 4 + h]); heads past H are 0.  Init time.
+__global__ void seq_consts_kernel(const float* q0, const float* k0, const float* kP, int max_L, int d, int dh,
+                                  float* out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (max_L + 1) * 4) return;
+  const int j = i / 4, h = i % 4;
+  float acc = 0.f;
+  if (h * dh < d) {
+    const float* kv = j < max_L ? kP + (size_t)j * d : k0;
+    for (int c = h * dh; c < h * dh + dh; ++c) acc = fmaf(q0[c], kv[c], acc);
+  }
+  out[i] = acc;
+}
+
+cudaError_t seq_consts_launch(const float* q0, const float* k0, const float* kP, int max_L, int d, int dh, float* out,
+                              cudaStream_t s) {
+  const int n = (max_L + 1) * 4;
+  seq_consts_kernel<<<(n + 127) / 128, 128, 0, s>>>(q0, k0, kP, max_L, d, dh, out);
+  return cudaGetLastError();
 }
 
 namespace {
