@@ -239,19 +239,21 @@ __device__ __noinline__ void epi_resid_ln(uint8_t* sA, float* red, uint32_t acc_
         *reinterpret_cast<float4*>(out_row + 32 * half + 64 * ci + j) =
             make_float4(v[32 * ci + j], v[32 * ci + j + 1], v[32 * ci + j + 2], v[32 * ci + j + 3]);
   }
-  float sum = 0.f;
+  // four independent partial sums per statistic (short dependency chains)
+  float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-  for (int j = 0; j < 64; ++j) sum += v[j];
-  red[half * 128 + r] = sum;
+  for (int j = 0; j < 64; ++j) s4[j & 3] += v[j];
+  red[half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
   asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
   const float mean = (red[r] + red[128 + r]) * (1.f / (float)D);
-  float var = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) s4[i] = 0.f;
 #pragma unroll
   for (int j = 0; j < 64; ++j) {
     const float dv = v[j] - mean;
-    var = fmaf(dv, dv, var);
+    s4[j & 3] = fmaf(dv, dv, s4[j & 3]);
   }
-  red[256 + half * 128 + r] = var;
+  red[256 + half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
   asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
   const float rstd = 1.0f / sqrtf((red[256 + r] + red[256 + 128 + r]) * (1.f / (float)D) + eps);
 #pragma unroll
@@ -276,6 +278,113 @@ __device__ __noinline__ void mma_half(uint32_t dst, uint32_t sa, uint32_t w, uin
 }
 
 }  // namespace
+
+// Phase A for one lane of the epilogue warps: rows rr_k = ew + 8 (4 k + g),
+// k < 4 (g = lane / 8), of which the lane owns value columns 16 li .. 16 li + 15
+// (li = lane % 8; head hc).  Per row, for head hc: the [CLS] query's logits
+// against [CLS] and the L assembled tokens (the element's partial plus the
+// position part), their softmax, and o = p_cls v0 + sum_j p_j (v_j + vP_j)
+// over the lane's columns, written into the split A tile.  Both lanes that own
+// columns of head hc compute its softmax (no exchange between lanes); the four
+// rows go through the token loop together so that their loads overlap.
+// kStaged: every element row of the tile is in the staging area, so every
+// load is a shared-memory load; otherwise rows past the staged ones are read
+// from memory.
+template <int DH, bool kStaged>
+__device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const uint8_t* sStage, const float* sVP,
+                                         const float* sQkP, const float* sQk0, const float* sV0, const bf16* v_h,
+                                         const float* elog, int e0, int nst, int rows_v, int L, float sl2, int ew,
+                                         int lane) {
+  const int g = lane >> 3, li = lane & 7;
+  const int hc = (16 * li) / DH;
+  int rrow[4];
+  bool live[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    rrow[k] = ew + 8 * (4 * k + g);
+    live[k] = rrow[k] < rows_v && sErow[rrow[k] * 32] >= 0;  // not padding, not a rejected request
+  }
+  // the element part of the logit of element row e for head hc (unscaled)
+  auto part = [&](int e) -> float {
+    const int er = e - e0;
+    const float* src = (kStaged || (unsigned)er < (unsigned)nst)
+                           ? reinterpret_cast<const float*>(sStage + NST * 256 + er * 16)
+                           : elog + (size_t)e * 4;
+    return DH == 32 ? src[hc] : src[2 * hc] + src[2 * hc + 1];
+  };
+  const float s0 = sQk0[hc] * sl2;
+  float m[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) m[k] = s0;
+#pragma unroll 1
+  for (int j = 0; j < L; ++j) {
+    const float qp = sQkP[j * 4 + hc];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (live[k]) m[k] = fmaxf(m[k], (part(sErow[rrow[k] * 32 + j]) + qp) * sl2);
+  }
+  float sum[4], o[4][16];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    sum[k] = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) o[k][i] = 0.f;
+  }
+#pragma unroll 1
+  for (int j = 0; j < L; ++j) {
+    const float qp = sQkP[j * 4 + hc];
+    const float4* vp = reinterpret_cast<const float4*>(sVP + (size_t)j * D + 16 * li);
+    const float4 pp[4] = {vp[0], vp[1], vp[2], vp[3]};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if (!live[k]) continue;
+      const int e = sErow[rrow[k] * 32 + j];
+      const int er = e - e0;
+      const uint4* src = (kStaged || (unsigned)er < (unsigned)nst)
+                             ? reinterpret_cast<const uint4*>(sStage + (size_t)er * 256 + 32 * li)
+                             : reinterpret_cast<const uint4*>(v_h + (size_t)e * D + 16 * li);
+      const uint4 a4 = src[0], b4 = src[1];
+      const float w = ex2_approx((part(e) + qp) * sl2 - m[k]);
+      sum[k] += w;
+      const uint32_t wv[8] = {a4.x, a4.y, a4.z, a4.w, b4.x, b4.y, b4.z, b4.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i]));
+        const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i + 1]));
+        o[k][4 * i] = fmaf(w, a.x + pp[i].x, o[k][4 * i]);
+        o[k][4 * i + 1] = fmaf(w, a.y + pp[i].y, o[k][4 * i + 1]);
+        o[k][4 * i + 2] = fmaf(w, b.x + pp[i].z, o[k][4 * i + 2]);
+        o[k][4 * i + 3] = fmaf(w, b.y + pp[i].w, o[k][4 * i + 3]);
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int rr = rrow[k];
+    if (live[k]) {
+      const float pc = ex2_approx(s0 - m[k]);
+      const float inv = 1.f / (sum[k] + pc);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) o[k][i] = fmaf(pc, sV0[16 * li + i], o[k][i]) * inv;
+    } else if (rr < rows_v) {
+      // a rejected request's scores become NaN; o = v0 keeps its rows finite
+#pragma unroll
+      for (int i = 0; i < 16; ++i) o[k][i] = sV0[16 * li + i];
+    }
+    // o -> row rr of the split tile: columns 16 li .. 16 li + 15 are 16-byte
+    // pieces 2 (li % 4) and 2 (li % 4) + 1 of plane li / 4
+    uint32_t hi[8], lo[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) split2(o[k][2 * i], o[k][2 * i + 1], hi[i], lo[i]);
+    uint8_t* rowp = sA + (size_t)((li >> 2) * 2) * kAPlane + (size_t)rr * 128u;
+    const uint32_t o0 = (uint32_t)((2 * (li & 3)) ^ (rr & 7)) << 4;
+    const uint32_t o1 = (uint32_t)((2 * (li & 3) + 1) ^ (rr & 7)) << 4;
+    *reinterpret_cast<uint4*>(rowp + o0) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    *reinterpret_cast<uint4*>(rowp + o1) = make_uint4(hi[4], hi[5], hi[6], hi[7]);
+    *reinterpret_cast<uint4*>(rowp + kAPlane + o0) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    *reinterpret_cast<uint4*>(rowp + kAPlane + o1) = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+  }
+}
 
 template <int DH>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -639,166 +748,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (et < G) sFlag[et] = (et < Gv && p.bad[b0 + et]) ? 2 : 0;  // bit 1: a rejected request
       epi_sync();
       if (!wait(st_full, tl & 1)) break;
-      {
-        // lane group g = lane / 8 takes the sequence of row ew + 8 (g0 + g), four
-        // sequences per warp at a time; lane li = lane % 8 of the group owns columns
-        // 16 li .. 16 li + 15 (head hc) and tokens li, li + 8, ... for the softmax
-        const int g = lane >> 3, li = lane & 7;
-        const int hc = (16 * li) / DH;
-        // this lane's 16 value columns of element row e: staged, or in memory
-        auto vrow = [&](int e) -> const uint4* {
-          const int er = e - e0;
-          return (unsigned)er < (unsigned)nst ? reinterpret_cast<const uint4*>(sStage + (size_t)er * 256 + 32 * li)
-                                              : reinterpret_cast<const uint4*>(p.v_h + (size_t)e * D + 16 * li);
-        };
-#pragma unroll 1
-        for (int g0 = 0; g0 < 16; g0 += 4) {
-          const int rr = ew + 8 * (g0 + g);
-          const bool live = rr < rows_v && sErow[rr * 32] >= 0;  // not a rejected request
-          const bool dead = rr < rows_v && !live;
-          float o[16];
-          // a rejected request's scores become NaN; o = v0 keeps its rows finite
-#pragma unroll
-          for (int i = 0; i < 16; i += 4) {
-            const float4 v0 = dead ? *reinterpret_cast<const float4*>(sV0 + 16 * li + i) : make_float4(0.f, 0.f, 0.f, 0.f);
-            o[i] = v0.x;
-            o[i + 1] = v0.y;
-            o[i + 2] = v0.z;
-            o[i + 3] = v0.w;
-          }
-          // every load of the group first: the logit partials of tokens li + 8 t
-          // (t < 4) and the value rows of tokens 0 .. 7 (f16, 32 bytes per lane)
-          float4 pt[4];
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            const int j = li + 8 * t;
-            pt[t] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (live && j < L) {
-              const int e = sErow[rr * 32 + j], er = e - e0;
-              pt[t] = *((unsigned)er < (unsigned)nst ? reinterpret_cast<const float4*>(sStage + NST * 256 + er * 16)
-                                                    : reinterpret_cast<const float4*>(p.elog + (size_t)e * 4));
-            }
-          }
-          uint4 va[8], vb[8];
-#pragma unroll
-          for (int jj = 0; jj < 8; ++jj) {
-            va[jj] = make_uint4(0u, 0u, 0u, 0u);
-            vb[jj] = va[jj];
-            if (live && jj < L) {
-              const uint4* src = vrow(sErow[rr * 32 + jj]);
-              va[jj] = src[0];
-              vb[jj] = src[1];
-            }
-          }
-          // logits per head, in the log2 domain
-          float sc[4][4];
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            const int j = li + 8 * t;
-#pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              const float lg = DH == 32 ? (h == 0 ? pt[t].x : h == 1 ? pt[t].y : h == 2 ? pt[t].z : pt[t].w)
-                                        : (h == 0 ? pt[t].x + pt[t].y : pt[t].z + pt[t].w);
-              sc[t][h] = (live && h < H && j < L) ? (lg + sQkP[j * 4 + h]) * sl2 : -INFINITY;
-            }
-          }
-          // softmax over [CLS; L tokens] per head within the group: pw[t][h], and [CLS]'s weight for head hc
-          float pw[4][4];
-          float pc = 0.f;
-#pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const float s0 = sQk0[h < H ? h : 0] * sl2;
-            float m = fmaxf(fmaxf(sc[0][h], sc[1][h]), fmaxf(sc[2][h], sc[3][h]));
-            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
-            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
-            m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
-            m = fmaxf(m, s0);
-            float sum = 0.f;
-#pragma unroll
-            for (int t = 0; t < 4; ++t) {
-              pw[t][h] = ex2_approx(sc[t][h] - m);  // 0 for tokens past L
-              sum += pw[t][h];
-            }
-            sum += __shfl_xor_sync(0xffffffffu, sum, 1);
-            sum += __shfl_xor_sync(0xffffffffu, sum, 2);
-            sum += __shfl_xor_sync(0xffffffffu, sum, 4);
-            const float e0 = ex2_approx(s0 - m);
-            const float inv = 1.f / (sum + e0);
-#pragma unroll
-            for (int t = 0; t < 4; ++t) pw[t][h] *= inv;
-            if (h == hc) pc = e0 * inv;
-          }
-          // the weights through shared memory: [warp][group][token][head]
-          float* pwg = reinterpret_cast<float*>(sV + 16384) + (size_t)(ew * 4 + g) * 128;
-#pragma unroll
-          for (int t = 0; t < 4; ++t)
-            *reinterpret_cast<float4*>(pwg + (li + 8 * t) * 4) = make_float4(pw[t][0], pw[t][1], pw[t][2], pw[t][3]);
-          __syncwarp();
-          if (live) {
-#pragma unroll
-            for (int i = 0; i < 16; i += 4) {
-              const float4 v0 = *reinterpret_cast<const float4*>(sV0 + 16 * li + i);
-              o[i] = pc * v0.x;
-              o[i + 1] = pc * v0.y;
-              o[i + 2] = pc * v0.z;
-              o[i + 3] = pc * v0.w;
-            }
-          }
-          // o += sum_j p_j (H_j WVs + P_j WVs): tokens 0 .. 7 from the loads above,
-          // longer sequences four further tokens at a time
-          auto accumulate = [&](int j, const uint4& a4, const uint4& b4) {
-            const float w = pwg[j * 4 + hc];
-            const float4* vp = reinterpret_cast<const float4*>(sVP + (size_t)j * D + 16 * li);
-            const uint32_t wv[8] = {a4.x, a4.y, a4.z, a4.w, b4.x, b4.y, b4.z, b4.w};
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const float4 pp = vp[i];
-              const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i]));
-              const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&wv[2 * i + 1]));
-              o[4 * i] = fmaf(w, a.x + pp.x, o[4 * i]);
-              o[4 * i + 1] = fmaf(w, a.y + pp.y, o[4 * i + 1]);
-              o[4 * i + 2] = fmaf(w, b.x + pp.z, o[4 * i + 2]);
-              o[4 * i + 3] = fmaf(w, b.y + pp.w, o[4 * i + 3]);
-            }
-          };
-          if (live) {
-#pragma unroll
-            for (int jj = 0; jj < 8; ++jj)
-              if (jj < L) accumulate(jj, va[jj], vb[jj]);
-#pragma unroll 1
-            for (int j0 = 8; j0 < L; j0 += 4) {
-#pragma unroll
-              for (int jj = 0; jj < 4; ++jj) {
-                va[jj] = make_uint4(0u, 0u, 0u, 0u);
-                vb[jj] = va[jj];
-                if (j0 + jj < L) {
-                  const uint4* src = vrow(sErow[rr * 32 + j0 + jj]);
-                  va[jj] = src[0];
-                  vb[jj] = src[1];
-                }
-              }
-#pragma unroll
-              for (int jj = 0; jj < 4; ++jj)
-                if (j0 + jj < L) accumulate(j0 + jj, va[jj], vb[jj]);
-            }
-          }
-          __syncwarp();  // every lane has read the weights before the next group writes them
-          // o -> row rr of the split tile: columns 16 li .. 16 li + 15 are 16-byte
-          // pieces 2 (li % 4) and 2 (li % 4) + 1 of plane li / 4
-          {
-            uint32_t hi[8], lo[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) split2(o[2 * i], o[2 * i + 1], hi[i], lo[i]);
-            uint8_t* rowp = sA + (size_t)((li >> 2) * 2) * kAPlane + (size_t)rr * 128u;
-            const uint32_t o0 = (uint32_t)((2 * (li & 3)) ^ (rr & 7)) << 4;
-            const uint32_t o1 = (uint32_t)((2 * (li & 3) + 1) ^ (rr & 7)) << 4;
-            *reinterpret_cast<uint4*>(rowp + o0) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-            *reinterpret_cast<uint4*>(rowp + o1) = make_uint4(hi[4], hi[5], hi[6], hi[7]);
-            *reinterpret_cast<uint4*>(rowp + kAPlane + o0) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-            *reinterpret_cast<uint4*>(rowp + kAPlane + o1) = make_uint4(lo[4], lo[5], lo[6], lo[7]);
-          }
-        }
-      }
+      if (nst == p.off[b0 + Gv] - e0)
+        cls_rows<DH, true>(sA, sErow, sStage, sVP, sQkP, sQk0, sV0, p.v_h, p.elog, e0, nst, rows_v, L, sl2, ew, lane);
+      else
+        cls_rows<DH, false>(sA, sErow, sStage, sVP, sQkP, sQk0, sV0, p.v_h, p.elog, e0, nst, rows_v, L, sl2, ew, lane);
       // x0 = [CLS] into the accumulator (read by this thread in the previous tile's last phase)
       tmem_st32_nw(acc2 + lane_off + (uint32_t)(32 * half), sCls + 32 * half);
       tmem_st32_nw(acc2 + lane_off + (uint32_t)(32 * half + 64), sCls + 32 * half + 64);
