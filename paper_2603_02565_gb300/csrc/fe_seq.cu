@@ -83,6 +83,16 @@ __device__ __forceinline__ void arrive1(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
+// One arrival per warp, on a barrier whose count is the number of arriving
+// warps: the lanes synchronise first, which orders every lane's earlier
+// (fenced) writes before the single arrival.  Lanes that left the tile loop
+// on a timed-out wait take no part.
+__device__ __forceinline__ void warp_arrive(uint64_t* bar) {
+  const unsigned m = __activemask();
+  __syncwarp(m);
+  if ((int)(threadIdx.x & 31) == __ffs(m) - 1) arrive1(bar);
+}
+
 __device__ __forceinline__ uint64_t desc_swz(uint32_t saddr, uint32_t sbo, uint32_t swz) {
   uint64_t d = 0;
   d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
@@ -456,24 +466,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < NA1; ++i) {
       mbar_init(acc1_full + i, 1);
       mbar_init(acc1_empty + i, 1);
-      mbar_init(mid_full + i, 32 * kEpiWarps);
+      mbar_init(mid_full + i, kEpiWarps);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(s_full + i, 1);
-      mbar_init(p_full + i, 32 * kEpiWarps);
+      mbar_init(p_full + i, kEpiWarps);
       mbar_init(s_free + i, 1);
     }
-    mbar_init(a_full, 32 * kEpiWarps);
+    mbar_init(a_full, kEpiWarps);
     mbar_init(o_done, 1);
-    mbar_init(ln_full, 32 * kEpiWarps);
+    mbar_init(ln_full, kEpiWarps);
     mbar_init(acc2_full, 1);
-    mbar_init(z_full, 32 * kEpiWarps);
+    mbar_init(z_full, kEpiWarps);
     mbar_init(qkv_full, 1);
-    mbar_init(qkv_ready, 32 * kEpiWarps);
+    mbar_init(qkv_ready, kEpiWarps);
     mbar_init(o_full, 1);
-    mbar_init(a2_full, 32 * kEpiWarps);
+    mbar_init(a2_full, kEpiWarps);
     mbar_init(ox_full, 1);
-    mbar_init(lnc_full, 32 * kEpiWarps);
+    mbar_init(lnc_full, kEpiWarps);
     mbar_init(head_full, 1);
     mbar_init(st_full, 1);
     fence_mbar_init();
@@ -758,7 +768,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_st_wait();
       fence_async_shared();
       tc_fence_before();
-      arrive1(a_full);
+      warp_arrive(a_full);
       // ================= B: c = cls + o WOs, FFN =================
       {
         const uint32_t proj = tmem + (uint32_t)((gf % NA1) * FC);
@@ -767,7 +777,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         epi_resid_ln(sA, red, acc2 + lane_off, true, proj + lane_off, nullptr, nullptr, r, q, half, p.eps);
         fence_async_shared();
         tc_fence_before();
-        arrive1(ln_full);
+        warp_arrive(ln_full);
       }
       for (int f = 0; f < nf; ++f, ++gf) {
         const int ba = gf % NA1;
@@ -791,7 +801,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_st_wait();
         tc_fence_before();
-        arrive1(mid_full + ba);
+        warp_arrive(mid_full + ba);
       }
       if (!ok) break;
       // c = acc2 + b2s; Z = LN(c) (the cross-sequence block's input, or the head's)
@@ -801,7 +811,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                    r, q, half, p.eps);
       fence_async_shared();
       tc_fence_before();
-      arrive1(z_full);
+      warp_arrive(z_full);
       if (p.cross) {
         // ================= C: cross-sequence attention =================
         if (!wait(qkv_full, tl & 1)) break;
@@ -853,7 +863,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (bad_v && rvalid) atomicOr(sFlag + lr, 1);  // bit 0: a non-finite value row
         fence_async_shared();
         tc_fence_before();
-        arrive1(qkv_ready);
+        warp_arrive(qkv_ready);
         // per head: softmax over the row's own request's K keys (keys of other
         // requests and padding rows take no part: -inf)
         const int klo = rvalid ? lr * K : 0, khi = rvalid ? lr * K + K : 0;
@@ -896,7 +906,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           rsum[half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
           tmem_st_wait();
           tc_fence_before();
-          arrive1(p_full + buf);
+          warp_arrive(p_full + buf);
           pair_sync();
           const float lt = rsum[r] + rsum[128 + r];
           const float lv = lt == 0.f ? 1.f : lt;  // 0 only for a padding row (a NaN stays NaN)
@@ -924,7 +934,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         fence_async_shared();
         tc_fence_before();
-        arrive1(a2_full);
+        warp_arrive(a2_full);
         // ================= D: C' = c + A WOx, LN(C') =================
         if (!wait(ox_full, tl & 1)) break;
         tc_fence_after();
@@ -932,7 +942,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                      (p.cp_out && rvalid) ? p.cp_out + (size_t)(b0 * K + r) * D : nullptr, r, q, half, p.eps);
         fence_async_shared();
         tc_fence_before();
-        arrive1(lnc_full);
+        warp_arrive(lnc_full);
       }
       // ================= E: score head and the argmax of Eq. 1 =================
       if (!wait(head_full, tl & 1)) break;
