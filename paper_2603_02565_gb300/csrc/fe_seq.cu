@@ -25,8 +25,8 @@
 //      attaining the maximum
 // Roles: warp 0 lane 0 streams the weights (16 KB boxes, two per 128 x 128
 // chunk, in consumption order through a ring of seven slots, by TMA), warp 1 lane 0 issues tcgen05.mma,
-// warps 2-9 run the gathers, softmaxes and epilogues (two warps per TMEM lane
-// quadrant, each owning half of a row's columns).  Products take split
+// warps 2-17 run the gathers, softmaxes and epilogues (four warps per TMEM lane
+// quadrant, each owning a quarter of a row's columns).  Products take split
 // bf16 activations (hi + lo) times exact bf16 weights with fp32 accumulation;
 // the attention operands Q, K, V, P are single f16 planes; LayerNorm,
 // softmax and residuals are fp32.
@@ -43,8 +43,8 @@ constexpr int BK = 64;
 constexpr int FC = 128;  // FFN columns per chunk
 constexpr int NA1 = 3;   // TMEM buffers for FFN1 chunks
 constexpr int LA = 2;    // FFN1 chunks issued ahead of the FFN2 that consumes them
-constexpr int kEpiWarps = 8;
-constexpr int kThreads = 64 + 32 * kEpiWarps;  // 320
+constexpr int kEpiWarps = 16;
+constexpr int kThreads = 64 + 32 * kEpiWarps;  // 576
 constexpr int kMaxL = 31;
 constexpr int kMaxF = 1024;
 constexpr uint32_t kAPlane = BM * BK * 2;  // 16 KB: 128 rows x 64 bf16
@@ -57,7 +57,7 @@ constexpr uint32_t kOffV = 4 * kAPlane;               // 64 KB: the split A tile
 constexpr uint32_t kOffRing = kOffV + 32768;          // the V tiles, one per head
 constexpr uint32_t kOffMisc = kOffRing + kRing * kBox;
 // misc: b1s [kMaxF], b2s, cls, b1h, w2h [D], q0.kP [32][4], q0.k0 [4], row-statistic
-// exchange [4][2][128], scores [128], request flags [128], barriers, TMEM slot
+// exchange [2][4][128], scores [128], request flags [128], barriers, TMEM slot
 constexpr uint32_t kMiscB1 = 0;
 constexpr uint32_t kMiscB2 = kMiscB1 + kMaxF * 4;
 constexpr uint32_t kMiscCls = kMiscB2 + D * 4;
@@ -141,35 +141,6 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
                : "memory");
 }
 
-// Two 32-column pieces of this warp's 32 TMEM lanes (row = lane) into
-// registers, one wait for both.
-__device__ __forceinline__ void tmem_ld32x2(uint32_t ta, uint32_t tb, float* va, float* vb) {
-  uint32_t a[32], b[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
-      "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
-      "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3]), "=r"(a[4]), "=r"(a[5]), "=r"(a[6]), "=r"(a[7]),
-        "=r"(a[8]), "=r"(a[9]), "=r"(a[10]), "=r"(a[11]), "=r"(a[12]), "=r"(a[13]), "=r"(a[14]), "=r"(a[15]),
-        "=r"(a[16]), "=r"(a[17]), "=r"(a[18]), "=r"(a[19]), "=r"(a[20]), "=r"(a[21]), "=r"(a[22]), "=r"(a[23]),
-        "=r"(a[24]), "=r"(a[25]), "=r"(a[26]), "=r"(a[27]), "=r"(a[28]), "=r"(a[29]), "=r"(a[30]), "=r"(a[31]),
-        "=r"(b[0]), "=r"(b[1]), "=r"(b[2]), "=r"(b[3]), "=r"(b[4]), "=r"(b[5]), "=r"(b[6]), "=r"(b[7]),
-        "=r"(b[8]), "=r"(b[9]), "=r"(b[10]), "=r"(b[11]), "=r"(b[12]), "=r"(b[13]), "=r"(b[14]), "=r"(b[15]),
-        "=r"(b[16]), "=r"(b[17]), "=r"(b[18]), "=r"(b[19]), "=r"(b[20]), "=r"(b[21]), "=r"(b[22]), "=r"(b[23]),
-        "=r"(b[24]), "=r"(b[25]), "=r"(b[26]), "=r"(b[27]), "=r"(b[28]), "=r"(b[29]), "=r"(b[30]), "=r"(b[31])
-      : "r"(ta), "r"(tb)
-      : "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) {
-    va[i] = __uint_as_float(a[i]);
-    vb[i] = __uint_as_float(b[i]);
-  }
-}
-
 // 32 lanes x 32 columns from registers, no wait (tmem_st_wait completes it)
 __device__ __forceinline__ void tmem_st32_nw(uint32_t taddr, const float* v) {
   asm volatile(
@@ -190,85 +161,76 @@ __device__ __forceinline__ void tmem_st32_nw(uint32_t taddr, const float* v) {
       : "memory");
 }
 
-// This thread's 64 columns of row r (32 half + 64 ci + [0, 32), ci < 2) as a
-// split bf16 pair into the A tile (128-byte swizzle, [kb][plane]).
-__device__ __forceinline__ void store_split64(uint8_t* sA, int r, int half, const float* v) {
+// This thread's 32 columns of row r (32 qt .. 32 qt + 31) as a split bf16
+// pair into the A tile (128-byte swizzle, [kb][plane]).
+__device__ __forceinline__ void store_split32(uint8_t* sA, int r, int qt, const float* v) {
+  uint32_t hi[16], lo[16];
 #pragma unroll
-  for (int ci = 0; ci < 2; ++ci) {
-    uint32_t hi[16], lo[16];
+  for (int j = 0; j < 16; ++j) split2(v[2 * j], v[2 * j + 1], hi[j], lo[j]);
+  uint8_t* rowp = sA + (size_t)((qt >> 1) * 2) * kAPlane + (size_t)r * 128u;
 #pragma unroll
-    for (int j = 0; j < 16; ++j) split2(v[32 * ci + 2 * j], v[32 * ci + 2 * j + 1], hi[j], lo[j]);
-    uint8_t* rowp = sA + (size_t)(ci * 2) * kAPlane + (size_t)r * 128u;
-#pragma unroll
-    for (int jj = 0; jj < 4; ++jj) {
-      const uint32_t o = (uint32_t)((4 * half + jj) ^ (r & 7)) << 4;
-      *reinterpret_cast<uint4*>(rowp + o) = make_uint4(hi[4 * jj], hi[4 * jj + 1], hi[4 * jj + 2], hi[4 * jj + 3]);
-      *reinterpret_cast<uint4*>(rowp + kAPlane + o) =
-          make_uint4(lo[4 * jj], lo[4 * jj + 1], lo[4 * jj + 2], lo[4 * jj + 3]);
-    }
+  for (int jj = 0; jj < 4; ++jj) {
+    const uint32_t o = (uint32_t)((4 * (qt & 1) + jj) ^ (r & 7)) << 4;
+    *reinterpret_cast<uint4*>(rowp + o) = make_uint4(hi[4 * jj], hi[4 * jj + 1], hi[4 * jj + 2], hi[4 * jj + 3]);
+    *reinterpret_cast<uint4*>(rowp + kAPlane + o) = make_uint4(lo[4 * jj], lo[4 * jj + 1], lo[4 * jj + 2], lo[4 * jj + 3]);
   }
 }
 
 // The residual step shared by SeqEnc and the cross-sequence block (one copy
-// of the code for its three uses): x = acc [+ add] [+ bias] (this thread's 64
-// columns of row r; written back to the accumulator when anything was added,
-// and to out_row when given), then LN(x) as the split A tile.  acc_t and add_t
-// are TMEM addresses of the thread's lane quadrant (add: whether add_t is
-// added); the row statistics are exchanged with the partner warp of the quadrant.
+// of the code for its three uses): x = acc [+ add] [+ bias] (this thread's 32
+// columns 32 qt .. 32 qt + 31 of row r; written back to the accumulator when
+// anything was added, and to out_row when given), then LN(x) as the split A
+// tile.  acc_t and add_t are TMEM addresses of the thread's lane quadrant (add:
+// whether add_t is added); the row statistics are exchanged with the other three
+// warps of the quadrant.
 __device__ __noinline__ void epi_resid_ln(uint8_t* sA, float* red, uint32_t acc_t, bool add, uint32_t add_t,
-                                          const float* bias, float* out_row, int r, int q, int half, float eps) {
-  float v[64];
-  tmem_ld32x2(acc_t + (uint32_t)(32 * half), acc_t + (uint32_t)(32 * half + 64), v, v + 32);
+                                          const float* bias, float* out_row, int r, int q, int qt, float eps) {
+  const uint32_t c = (uint32_t)(32 * qt);
+  float v[32];
+  tmem_ld32(acc_t + c, v);
   if (add) {
-    float w[64];
-    tmem_ld32x2(add_t + (uint32_t)(32 * half), add_t + (uint32_t)(32 * half + 64), w, w + 32);
+    float w[32];
+    tmem_ld32(add_t + c, w);
 #pragma unroll
-    for (int j = 0; j < 64; ++j) v[j] += w[j];
+    for (int j = 0; j < 32; ++j) v[j] += w[j];
   }
   if (bias) {
 #pragma unroll
-    for (int ci = 0; ci < 2; ++ci)
-#pragma unroll
-      for (int j = 0; j < 32; j += 4) {
-        const float4 b = *reinterpret_cast<const float4*>(bias + 32 * half + 64 * ci + j);
-        v[32 * ci + j] += b.x;
-        v[32 * ci + j + 1] += b.y;
-        v[32 * ci + j + 2] += b.z;
-        v[32 * ci + j + 3] += b.w;
-      }
+    for (int j = 0; j < 32; j += 4) {
+      const float4 b = *reinterpret_cast<const float4*>(bias + c + j);
+      v[j] += b.x;
+      v[j + 1] += b.y;
+      v[j + 2] += b.z;
+      v[j + 3] += b.w;
+    }
   }
-  if (add || bias) {
-    tmem_st32_nw(acc_t + (uint32_t)(32 * half), v);
-    tmem_st32_nw(acc_t + (uint32_t)(32 * half + 64), v + 32);
-  }
+  if (add || bias) tmem_st32_nw(acc_t + c, v);
   if (out_row) {
 #pragma unroll
-    for (int ci = 0; ci < 2; ++ci)
-#pragma unroll
-      for (int j = 0; j < 32; j += 4)
-        *reinterpret_cast<float4*>(out_row + 32 * half + 64 * ci + j) =
-            make_float4(v[32 * ci + j], v[32 * ci + j + 1], v[32 * ci + j + 2], v[32 * ci + j + 3]);
+    for (int j = 0; j < 32; j += 4)
+      *reinterpret_cast<float4*>(out_row + c + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
   }
   // four independent partial sums per statistic (short dependency chains)
   float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-  for (int j = 0; j < 64; ++j) s4[j & 3] += v[j];
-  red[half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
-  asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
-  const float mean = (red[r] + red[128 + r]) * (1.f / (float)D);
+  for (int j = 0; j < 32; ++j) s4[j & 3] += v[j];
+  red[qt * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+  asm volatile("bar.sync %0, 128;" ::"r"(1 + q) : "memory");
+  const float mean = ((red[r] + red[128 + r]) + (red[256 + r] + red[384 + r])) * (1.f / (float)D);
 #pragma unroll
   for (int i = 0; i < 4; ++i) s4[i] = 0.f;
 #pragma unroll
-  for (int j = 0; j < 64; ++j) {
+  for (int j = 0; j < 32; ++j) {
     const float dv = v[j] - mean;
     s4[j & 3] = fmaf(dv, dv, s4[j & 3]);
   }
-  red[256 + half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
-  asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
-  const float rstd = 1.0f / sqrtf((red[256 + r] + red[256 + 128 + r]) * (1.f / (float)D) + eps);
+  red[512 + qt * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+  asm volatile("bar.sync %0, 128;" ::"r"(1 + q) : "memory");
+  const float rstd =
+      1.0f / sqrtf(((red[512 + r] + red[640 + r]) + (red[768 + r] + red[896 + r])) * (1.f / (float)D) + eps);
 #pragma unroll
-  for (int j = 0; j < 64; ++j) v[j] = (v[j] - mean) * rstd;
-  store_split64(sA, r, half, v);
+  for (int j = 0; j < 32; ++j) v[j] = (v[j] - mean) * rstd;
+  store_split32(sA, r, qt, v);
   if (add || bias) tmem_st_wait();
 }
 
@@ -289,13 +251,13 @@ __device__ __noinline__ void mma_half(uint32_t dst, uint32_t sa, uint32_t w, uin
 
 }  // namespace
 
-// Phase A for one lane of the epilogue warps: rows rr_k = ew + 8 (4 k + g),
-// k < 4 (g = lane / 8), of which the lane owns value columns 16 li .. 16 li + 15
+// Phase A for one lane of the epilogue warps: rows rr_k = ew + kEpiWarps (4 k + g),
+// k < NR = 128 / (4 kEpiWarps) (g = lane / 8), of which the lane owns value columns 16 li .. 16 li + 15
 // (li = lane % 8; head hc).  Per row, for head hc: the [CLS] query's logits
 // against [CLS] and the L assembled tokens (the element's partial plus the
 // position part), their softmax, and o = p_cls v0 + sum_j p_j (v_j + vP_j)
 // over the lane's columns, written into the split A tile.  Both lanes that own
-// columns of head hc compute its softmax (no exchange between lanes); the four
+// columns of head hc compute its softmax (no exchange between lanes); the NR
 // rows go through the token loop together so that their loads overlap.
 // kStaged: every element row of the tile is in the staging area, so every
 // load is a shared-memory load; otherwise rows past the staged ones are read
@@ -305,13 +267,14 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
                                          const float* sQkP, const float* sQk0, const float* sV0, const bf16* v_h,
                                          const float* elog, int e0, int nst, int rows_v, int L, float sl2, int ew,
                                          int lane) {
+  constexpr int NR = BM / (4 * kEpiWarps);
   const int g = lane >> 3, li = lane & 7;
   const int hc = (16 * li) / DH;
-  int rrow[4];
-  bool live[4];
+  int rrow[NR];
+  bool live[NR];
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    rrow[k] = ew + 8 * (4 * k + g);
+  for (int k = 0; k < NR; ++k) {
+    rrow[k] = ew + kEpiWarps * (4 * k + g);
     live[k] = rrow[k] < rows_v && sErow[rrow[k] * 32] >= 0;  // not padding, not a rejected request
   }
   // the element part of the logit of element row e for head hc (unscaled)
@@ -323,19 +286,19 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
     return DH == 32 ? src[hc] : src[2 * hc] + src[2 * hc + 1];
   };
   const float s0 = sQk0[hc] * sl2;
-  float m[4];
+  float m[NR];
 #pragma unroll
-  for (int k = 0; k < 4; ++k) m[k] = s0;
+  for (int k = 0; k < NR; ++k) m[k] = s0;
 #pragma unroll 1
   for (int j = 0; j < L; ++j) {
     const float qp = sQkP[j * 4 + hc];
 #pragma unroll
-    for (int k = 0; k < 4; ++k)
+    for (int k = 0; k < NR; ++k)
       if (live[k]) m[k] = fmaxf(m[k], (part(sErow[rrow[k] * 32 + j]) + qp) * sl2);
   }
-  float sum[4], o[4][16];
+  float sum[NR], o[NR][16];
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
+  for (int k = 0; k < NR; ++k) {
     sum[k] = 0.f;
 #pragma unroll
     for (int i = 0; i < 16; ++i) o[k][i] = 0.f;
@@ -346,7 +309,7 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
     const float4* vp = reinterpret_cast<const float4*>(sVP + (size_t)j * D + 16 * li);
     const float4 pp[4] = {vp[0], vp[1], vp[2], vp[3]};
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
+    for (int k = 0; k < NR; ++k) {
       if (!live[k]) continue;
       const int e = sErow[rrow[k] * 32 + j];
       const int er = e - e0;
@@ -369,7 +332,7 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
     }
   }
 #pragma unroll
-  for (int k = 0; k < 4; ++k) {
+  for (int k = 0; k < NR; ++k) {
     const int rr = rrow[k];
     if (live[k]) {
       const float pc = ex2_approx(s0 - m[k]);
@@ -421,7 +384,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* sW2h = reinterpret_cast<float*>(misc + kMiscW2h);
   float* sQkP = reinterpret_cast<float*>(misc + kMiscQkP);  // [j][4]: q0 . kP[j] per head
   float* sQk0 = reinterpret_cast<float*>(misc + kMiscQk0);  // [4]: q0 . k0 per head
-  float* red = reinterpret_cast<float*>(misc + kMiscRed);   // [slot][half][row]
+  float* red = reinterpret_cast<float*>(misc + kMiscRed);   // [statistic][quarter][row]
   float* sSc = reinterpret_cast<float*>(misc + kMiscSc);
   float* sV0 = reinterpret_cast<float*>(misc + kMiscV0);
   int* sFlag = reinterpret_cast<int*>(misc + kMiscFlag);    // request of the tile has a non-finite value row
@@ -712,13 +675,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ---------------- gathers, softmax and epilogues (warps 2..9) ----------------
-    const int ew = warp - 2, q = warp & 3, half = ew >> 2;
+    const int ew = warp - 2, q = warp & 3, qt = ew >> 2;  // lane quadrant, column quarter
     const int et = threadIdx.x - 64;
     const int r = q * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const float sl2 = p.scale_log2;
-    auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory"); };
-    auto epi_sync = [&]() { asm volatile("bar.sync 5, 256;" ::: "memory"); };
+    auto pair_sync = [&]() { asm volatile("bar.sync %0, 128;" ::"r"(1 + q) : "memory"); };  // the quadrant's 4 warps
+    auto epi_sync = [&]() { asm volatile("bar.sync 5, %0;" ::"n"(32 * kEpiWarps) : "memory"); };
     bool ok = true;
     auto wait = [&](uint64_t* bar, uint32_t par) -> bool {
       if (!mbar_wait_compact(bar, par, p.sel.status)) ok = false;
@@ -763,8 +726,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       else
         cls_rows<DH, false>(sA, sErow, sStage, sVP, sQkP, sQk0, sV0, p.v_h, p.elog, e0, nst, rows_v, L, sl2, ew, lane);
       // x0 = [CLS] into the accumulator (read by this thread in the previous tile's last phase)
-      tmem_st32_nw(acc2 + lane_off + (uint32_t)(32 * half), sCls + 32 * half);
-      tmem_st32_nw(acc2 + lane_off + (uint32_t)(32 * half + 64), sCls + 32 * half + 64);
+      tmem_st32_nw(acc2 + lane_off + (uint32_t)(32 * qt), sCls + 32 * qt);
       tmem_st_wait();
       fence_async_shared();
       tc_fence_before();
@@ -774,7 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t proj = tmem + (uint32_t)((gf % NA1) * FC);
         if (!wait(o_done, tl & 1)) break;
         tc_fence_after();
-        epi_resid_ln(sA, red, acc2 + lane_off, true, proj + lane_off, nullptr, nullptr, r, q, half, p.eps);
+        epi_resid_ln(sA, red, acc2 + lane_off, true, proj + lane_off, nullptr, nullptr, r, q, qt, p.eps);
         fence_async_shared();
         tc_fence_before();
         warp_arrive(ln_full);
@@ -784,20 +746,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!wait(acc1_full + ba, (gf / NA1) & 1)) break;
         tc_fence_after();
         {
-          const uint32_t col = tmem + lane_off + (uint32_t)(ba * FC + 64 * half);
-          const float* bias = sB1 + f * FC + 64 * half;
-          float v[64];
-          tmem_ld64(col, v);
+          // this thread's 32 hidden units: the hi plane (16 columns of bf16
+          // pairs) then the lo plane over the same 32 TMEM columns
+          const uint32_t col = tmem + lane_off + (uint32_t)(ba * FC + 32 * qt);
+          const float* bias = sB1 + f * FC + 32 * qt;
+          float v[32];
+          tmem_ld32(col, v);
+          uint32_t hi[16], lo[16];
 #pragma unroll
-          for (int hp = 0; hp < 2; ++hp) {
-            uint32_t hi[16], lo[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j)
-              split2_trunc(relu_keep_nan(v[32 * hp + 2 * j] + bias[32 * hp + 2 * j]),
-                           relu_keep_nan(v[32 * hp + 2 * j + 1] + bias[32 * hp + 2 * j + 1]), hi[j], lo[j]);
-            tmem_st16_nowait(col + (uint32_t)(32 * hp), hi);
-            tmem_st16_nowait(col + (uint32_t)(32 * hp + 16), lo);
-          }
+          for (int j = 0; j < 16; ++j)
+            split2_trunc(relu_keep_nan(v[2 * j] + bias[2 * j]), relu_keep_nan(v[2 * j + 1] + bias[2 * j + 1]), hi[j],
+                         lo[j]);
+          tmem_st16_nowait(col, hi);
+          tmem_st16_nowait(col + 16u, lo);
         }
         tmem_st_wait();
         tc_fence_before();
@@ -808,7 +769,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!wait(acc2_full, tl & 1)) break;
       tc_fence_after();
       epi_resid_ln(sA, red, acc2 + lane_off, false, 0u, sB2, (p.c_out && rvalid) ? p.c_out + (size_t)(b0 * K + r) * D : nullptr,
-                   r, q, half, p.eps);
+                   r, q, qt, p.eps);
       fence_async_shared();
       tc_fence_before();
       warp_arrive(z_full);
@@ -822,10 +783,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // must not meet 0 x NaN) and marks its request
         bool bad_v = false;
 #pragma unroll 1
-        for (int pc = 0; pc < 6; ++pc) {
-          const int part = pc >> 1, ci = pc & 1;
+        for (int part = 0; part < 3; ++part) {
           {
-            const int c = 32 * half + 64 * ci;
+            const int c = 32 * qt;
             float v[32];
             tmem_ld32(tmem + lane_off + (uint32_t)(part * 128 + c), v);
             uint32_t w[16];
@@ -868,47 +828,44 @@ __global__ void __launch_bounds__(kThreads, 1)
         // requests and padding rows take no part: -inf)
         const int klo = rvalid ? lr * K : 0, khi = rvalid ? lr * K + K : 0;
         float lh[4] = {1.f, 1.f, 1.f, 1.f};
-        float* rmax = red + 512;  // [half][row]
-        float* rsum = red + 768;
+        float* rmax = red;  // [quarter][row] (the LayerNorm statistics are consumed by now)
+        float* rsum = red + 512;
 #pragma unroll 1
         for (int h = 0; h < H; ++h) {
           const int g = tl * H + h, buf = g & 1;
           if (!wait(s_full + buf, (g >> 1) & 1)) break;
           tc_fence_after();
-          const uint32_t tile = tmem + lane_off + (uint32_t)(buf * 128 + 64 * half);
-          float v[64];
-          tmem_ld64(tile, v);
+          const uint32_t tile = tmem + lane_off + (uint32_t)(buf * 128);
+          float v[32];
+          tmem_ld32(tile + (uint32_t)(32 * qt), v);  // keys 32 qt .. 32 qt + 31
           float mx = -INFINITY;
 #pragma unroll
-          for (int i = 0; i < 64; ++i) {
-            const int key = 64 * half + i;
+          for (int i = 0; i < 32; ++i) {
+            const int key = 32 * qt + i;
             if (key < klo || key >= khi) v[i] = -INFINITY;
             mx = fmaxf(mx, v[i]);
           }
-          rmax[half * 128 + r] = mx;
-          pair_sync();
-          float m = fmaxf(rmax[r], rmax[128 + r]) * sl2;
+          rmax[qt * 128 + r] = mx;
+          pair_sync();  // also: every warp of the quadrant has read its S columns before P overwrites them
+          float m = fmaxf(fmaxf(rmax[r], rmax[128 + r]), fmaxf(rmax[256 + r], rmax[384 + r])) * sl2;
           if (m == -INFINITY) m = 0.f;  // a padding row: every P is 0
           float s4[4] = {0.f, 0.f, 0.f, 0.f};
+          uint32_t pk[16];
 #pragma unroll
-          for (int hb = 0; hb < 2; ++hb) {
-            uint32_t pk[16];
-#pragma unroll
-            for (int i = 0; i < 32; i += 2) {
-              const int k = 32 * hb + i;
-              const float p0 = ex2_approx(fmaf(v[k], sl2, -m));
-              const float p1 = ex2_approx(fmaf(v[k + 1], sl2, -m));
-              s4[(i >> 1) & 3] += p0 + p1;
-              pk[i / 2] = pack_f16x2(p0, p1);
-            }
-            tmem_st16_nowait(tile + (uint32_t)(16 * hb), pk);
+          for (int i = 0; i < 32; i += 2) {
+            const float p0 = ex2_approx(fmaf(v[i], sl2, -m));
+            const float p1 = ex2_approx(fmaf(v[i + 1], sl2, -m));
+            s4[(i >> 1) & 3] += p0 + p1;
+            pk[i / 2] = pack_f16x2(p0, p1);
           }
-          rsum[half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+          // P of keys 64 k + 32 j + [0, 32) in f16 pairs at columns 64 k + 16 j + [0, 16)
+          tmem_st16_nowait(tile + (uint32_t)(64 * (qt >> 1) + 16 * (qt & 1)), pk);
+          rsum[qt * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
           tmem_st_wait();
           tc_fence_before();
           warp_arrive(p_full + buf);
           pair_sync();
-          const float lt = rsum[r] + rsum[128 + r];
+          const float lt = (rsum[r] + rsum[128 + r]) + (rsum[256 + r] + rsum[384 + r]);
           const float lv = lt == 0.f ? 1.f : lt;  // 0 only for a padding row (a NaN stays NaN)
           lh[0] = h == 0 ? lv : lh[0];
           lh[1] = h == 1 ? lv : lh[1];
@@ -920,17 +877,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!wait(o_full, tl & 1)) break;
         tc_fence_after();
         {
-          float v[64];
-          tmem_ld32x2(tmem + lane_off + 256u + (uint32_t)(32 * half), tmem + lane_off + 256u + (uint32_t)(32 * half + 64),
-                      v, v + 32);
+          float v[32];
+          tmem_ld32(tmem + lane_off + 256u + (uint32_t)(32 * qt), v);
+          const int hh = (32 * qt) / DH;
+          const float inv = 1.f / (hh == 0 ? lh[0] : hh == 1 ? lh[1] : hh == 2 ? lh[2] : lh[3]);
 #pragma unroll
-          for (int ci = 0; ci < 2; ++ci) {
-            const int hh = (32 * half + 64 * ci) / DH;
-            const float inv = 1.f / (hh == 0 ? lh[0] : hh == 1 ? lh[1] : hh == 2 ? lh[2] : lh[3]);
-#pragma unroll
-            for (int j = 0; j < 32; ++j) v[32 * ci + j] *= inv;
-          }
-          store_split64(sA, r, half, v);
+          for (int j = 0; j < 32; ++j) v[j] *= inv;
+          store_split32(sA, r, qt, v);
         }
         fence_async_shared();
         tc_fence_before();
@@ -939,7 +892,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!wait(ox_full, tl & 1)) break;
         tc_fence_after();
         epi_resid_ln(sA, red, acc2 + lane_off, true, tmem + lane_off, nullptr,
-                     (p.cp_out && rvalid) ? p.cp_out + (size_t)(b0 * K + r) * D : nullptr, r, q, half, p.eps);
+                     (p.cp_out && rvalid) ? p.cp_out + (size_t)(b0 * K + r) * D : nullptr, r, q, qt, p.eps);
         fence_async_shared();
         tc_fence_before();
         warp_arrive(lnc_full);
@@ -950,20 +903,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       {
         float part = 0.f;
         {
-          float v[64];
-          tmem_ld32x2(tmem + 128u + lane_off + (uint32_t)(32 * half), tmem + 128u + lane_off + (uint32_t)(32 * half + 64),
-                      v, v + 32);
+          float v[32];
+          tmem_ld32(tmem + 128u + lane_off + (uint32_t)(32 * qt), v);
+          const int c = 32 * qt;
 #pragma unroll
-          for (int ci = 0; ci < 2; ++ci) {
-            const int c = 32 * half + 64 * ci;
-#pragma unroll
-            for (int j = 0; j < 32; ++j) part = fmaf(relu_keep_nan(v[32 * ci + j] + sB1h[c + j]), sW2h[c + j], part);
-          }
+          for (int j = 0; j < 32; ++j) part = fmaf(relu_keep_nan(v[j] + sB1h[c + j]), sW2h[c + j], part);
         }
         tc_fence_before();
-        red[half * 128 + r] = part;
+        red[qt * 128 + r] = part;
         pair_sync();
-        float s = red[r] + red[128 + r] + sV0[D];
+        float s = (red[r] + red[128 + r]) + (red[256 + r] + red[384 + r]) + sV0[D];
         if (rvalid) {
           if (sFlag[lr]) s = __int_as_float(0x7fc00000);
           p.scores[(size_t)(b0 * K + r)] = s;
