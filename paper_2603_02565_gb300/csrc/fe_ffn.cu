@@ -140,12 +140,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < NA1; ++i) {
       mbar_init(acc1_full + i, 1);
       mbar_init(acc1_empty + i, 1);
-      mbar_init(mid_full + i, 32 * kEpiWarps);
+      mbar_init(mid_full + i, kEpiWarps);
     }
     mbar_init(acc2_full, 1);
-    mbar_init(ln_full, 32 * kEpiWarps);
+    mbar_init(ln_full, kEpiWarps);
     mbar_init(r_empty, kEpiWarps);
-    mbar_init(tail_a, 32 * kEpiWarps);
+    mbar_init(tail_a, kEpiWarps);
     mbar_init(wt_full, 1);
     mbar_init(tail_full, 1);
     fence_mbar_init();
@@ -386,6 +386,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) bulk_wait_read0();
       __syncwarp();
     };
+    // one arrival per warp on barriers counted in warps (the lanes synchronise first)
+    auto warp_arrive = [&](uint64_t* bar) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive_one(bar);
+    };
     int tl = 0, gf = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++tl) {
@@ -492,7 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       fence_async_shared();
       tc_fence_before();
-      mbar_arrive_one(ln_full);
+      warp_arrive(ln_full);
       // ---- per chunk: mid = split(ReLU(acc1 + b1)) written back over this
       // warp's 64 columns of the chunk's TMEM buffer as FFN2's A operand
       for (int f = 0; f < nf; ++f, ++gf) {
@@ -521,7 +526,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tmem_st_wait();
         tc_fence_before();
-        mbar_arrive_one(mid_full + ba);
+        warp_arrive(mid_full + ba);
       }
       if (!ok) break;
       // ---- final: x_out = acc2 + b2 (acc2 = x + FFN2), LayerNorm, stores
@@ -614,7 +619,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       fence_async_shared();
-      if (tail_n > 0) mbar_arrive_one(tail_a);
+      if (tail_n > 0) warp_arrive(tail_a);
       if (p.store_ln) {
         asm volatile("bar.sync 5, 256;" ::: "memory");  // every row of the tile written
         if (ew == 0 && lane == 0) {
