@@ -35,7 +35,8 @@ constexpr uint32_t kWBytes = 2 * 128 * BK * 2; // WQ^T: up to 2 k blocks of 128 
 constexpr uint32_t kABytes = 2 * kPlane;       // operand tile: up to 2 k blocks
 constexpr uint32_t kStage = 2048;              // store staging: 32 rows x 32 f16, 64-byte swizzle
 constexpr uint32_t kStgBytes = kGWarps * 2 * kStage;
-constexpr size_t kSmem = 1024 + kWBytes + kABytes + kStgBytes + 128 * 4 + 128 * 8 + 256;
+constexpr int kMaxOff = 4096;                  // request offsets staged in shared memory (B < kMaxOff)
+constexpr size_t kSmem = 1024 + kWBytes + kABytes + kStgBytes + 128 * 4 + 128 * 8 + 256 + 4 * kMaxOff;
 
 __device__ __forceinline__ void arrive1(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
@@ -81,6 +82,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* acc_full = bars + 2;  // product complete in TMEM
   uint64_t* acc_empty = bars + 3; // product read by the epilogue
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 4);
+  int* sOff = reinterpret_cast<int*>(bars + 32);  // [B + 1] request offsets (when B < kMaxOff)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -148,6 +150,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     uint8_t* stg = sStg + (size_t)gw * 2 * kStage;
     // column sums of WQ: row i of the resident WQ^T (the swizzle only permutes a row's pieces)
+    // the request offsets to shared memory: each row's request is found by a
+    // binary search over them, which would otherwise be a chain of dependent
+    // global loads
+    const bool off_staged = p.B < kMaxOff;
+    if (off_staged)
+      for (int i = gw * 32 + lane; i <= p.B; i += 32 * kGWarps) sOff[i] = p.off[i];
     bool ok = mbar_wait_bounded(w_full, 0, p.status);
     {
       const int i = gw * 32 + lane;
@@ -178,12 +186,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < kPieces; ++j) pc[j] = make_uint4(0u, 0u, 0u, 0u);
       if (valid) {
         int lo = 0, hi = p.B - 1;  // largest b with off[b] <= row
-        while (lo < hi) {
-          const int mid = (lo + hi + 1) >> 1;
-          if (p.off[mid] <= row)
-            lo = mid;
-          else
-            hi = mid - 1;
+        if (off_staged) {
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (sOff[mid] <= row)
+              lo = mid;
+            else
+              hi = mid - 1;
+          }
+        } else {
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (p.off[mid] <= row)
+              lo = mid;
+            else
+              hi = mid - 1;
+          }
         }
         const int m = p.list[(size_t)lo * p.cap + (row - p.off[lo])];
         const bf16* src = p.pool + ((size_t)lo * p.M + m) * d;

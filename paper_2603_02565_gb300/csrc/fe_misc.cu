@@ -345,13 +345,17 @@ __global__ void __launch_bounds__(256) gather_ln_kernel(const T* __restrict__ po
   pdl_wait();
   pdl_trigger();
   if (r >= max_rows || r >= off[B]) return;
-  int lo = 0, hi = B - 1;  // largest b with off[b] <= r
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (off[mid] <= r)
-      lo = mid;
-    else
-      hi = mid - 1;
+  // the largest b with off[b] <= r, by the warp: each round the 32 lanes probe
+  // 32 evenly spaced candidates of the range [lo, hi) (off[lo] <= r holds) and
+  // keep the span after the last one that passes, so that B = 1024 takes two
+  // rounds of loads instead of ten dependent ones
+  int lo = 0, hi = B;
+  while (hi - lo > 1) {
+    const int step = (hi - lo + 31) / 32;
+    const int idx = lo + lane * step;
+    const unsigned pass = __ballot_sync(0xffffffffu, idx < hi && off[idx] <= r);
+    lo += (31 - __clz(pass)) * step;
+    hi = min(lo + step, hi);
   }
   const int b = lo;
   const int m = list[(size_t)b * cap + (r - off[b])];
