@@ -12,16 +12,18 @@
 //                   flight) and K/V chunks of CK keys (8 stages for d_h = 32,
 //                   4 for d_h = 64)
 //   warp 1 lane 0 : tcgen05.mma -- S_j = Q K_j^T into TMEM tile j % 3, then
-//                   PV_j = P_j V_j with P_j read from that same TMEM tile
-//                   into PV buffer j % 2; three S/P tiles let S_{j+1} start
-//                   while PV_{j-1} still reads its tile
+//                   PV_j = P_j V_j with P_j read from that same TMEM tile,
+//                   accumulated into the unit's output accumulator in TMEM
+//                   (two, alternating by unit); three S/P tiles let S_{j+1}
+//                   start while PV_{j-1} still reads its tile
 //   warps 2..9    : online softmax from TMEM, one query row per lane; warps
 //                   w and w+4 share TMEM lane quadrant w % 4 and each take
 //                   half of the chunk's keys and half of the output columns
-//                   (row maxima and sums exchanged through shared memory).  P_j is written back over S_j as f16;
-//                   PV_{j-1} is folded into the register output after P_j is
-//                   handed over, so the softmax never waits for the PV
-//                   product of the chunk it has just finished
+//                   (row maxima and sums exchanged through shared memory).  P_j is written back over S_j as f16
+//                   against a running maximum that moves only when a chunk
+//                   exceeds it by more than 2^8, when the output accumulator
+//                   is rescaled in TMEM; otherwise the softmax never reads
+//                   the PV products until the unit's output is stored
 // Q, K, V and P are single f16 planes (unit roundoff 2^-11; Q and K come
 // from LayerNorm'd rows times weights of magnitude well inside the f16
 // range, P lies in [0, 1]); accumulation, softmax statistics and the output
@@ -45,7 +47,8 @@ struct AttnCfg {
   static constexpr int KW = CK / kHalves;                        // keys per softmax warp and chunk
   static constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
   static constexpr int kCtasPerSM = DH == 32 ? 2 : 1;
-  // TMEM: S/P tiles at [t CK, t CK + CK), t < 3; PV buffers at [3CK, 3CK + 2DH)
+  // TMEM: S/P tiles at [t CK, t CK + CK), t < 3; the output accumulators of
+  // consecutive units (alternating) at [3CK, 3CK + 2DH)
   static constexpr int kTiles = 3;
   static constexpr uint32_t kTmemCols = DH == 32 ? 256 : 512;
   static_assert(kTiles * CK + 2 * DH <= (int)kTmemCols, "TMEM budget");
@@ -256,6 +259,9 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       Cursor sc;             // unit of the next S
       int sj = 0, sui = 0;   // its chunk and its unit counter (Q buffer sui % 2)
       int g_s = 0;           // S products issued
+      // per chunk g (g % 4; at most two chunks separate S and PV): its unit
+      // counter's parity (the output accumulator) and whether it opens the unit
+      uint32_t pv_info = 0;
       cur_first(p, units, sc);
       // S = Q K^T of the chunk at the S cursor into TMEM tile g_s % 3, then advance the cursor
       auto issue_next_s = [&]() -> bool {
@@ -277,6 +283,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         for (int kk = 0; kk < DH / 16; ++kk)
           umma_bf16(dst, desc_adv(q0d, kk * 32), desc_adv(k0d, kk * 32), idesc_s, kk != 0 ? 1u : 0u);
         umma_commit(s_full + t);
+        pv_info = (pv_info & ~(3u << (2 * (g_s & 3)))) | ((uint32_t)(((sui & 1) << 1) | (sj == 0 ? 1 : 0)) << (2 * (g_s & 3)));
         // The V rows of a partial chunk past the key count belong to the next
         // segment: their P is 0, but 0 x NaN is NaN, so they are zeroed here
         // (the chunk has landed; PV_{g_s}, issued later by this thread, reads them)
@@ -304,12 +311,15 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         const int ks = g % Cfg::kKVStages;
         const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile);
         const uint32_t pt = tmem + (uint32_t)(t * CK);
-        const uint32_t dst = tmem + (uint32_t)(Cfg::kTiles * CK + (g & 1) * DH);
+        // PV accumulates into the unit's output accumulator (unit parity), from zero at its first chunk
+        const uint32_t info = (pv_info >> (2 * (g & 3))) & 3u;
+        const uint32_t dst = tmem + (uint32_t)(Cfg::kTiles * CK + (int)(info >> 1) * DH);
         const uint64_t v0d = desc_sw(v, Cfg::kSbo, Cfg::kSwz);
 #pragma unroll
         for (int kk = 0; kk < CK / 16; ++kk)
           umma_bf16_tmem_a(dst, pt + (uint32_t)((kk / (Cfg::KW / 16)) * Cfg::KW + (kk % (Cfg::KW / 16)) * 8),
-                           desc_adv(v0d, (uint32_t)kk * 16 * Cfg::kRowBytes), idesc_pv, kk != 0 ? 1u : 0u);
+                           desc_adv(v0d, (uint32_t)kk * 16 * Cfg::kRowBytes), idesc_pv,
+                           (kk != 0 || !(info & 1u)) ? 1u : 0u);
         umma_commit(pv_full + (g & 1));
         umma_commit(tile_free + t);
         umma_commit(kv_empty + ks);
@@ -327,33 +337,27 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     float* red_max = red;         // [parity][half][128]
     float* red_sum = red + 512;
     auto pair_sync = [&]() { asm volatile("bar.sync %0, 64;" ::"r"(1 + q4) : "memory"); };
-    // fold PV_g (PV buffer g % 2) into the register output: o = o * c + PV_g
-    auto fold = [&](int g, float c, float* o) -> bool {
-      if (!mbar_wait_compact(pv_full + (g & 1), (g >> 1) & 1, p.status)) return false;
-      tc_fence_after();
-      float pv[DO];
-      const uint32_t src = tmem + lane_off + (uint32_t)(Cfg::kTiles * CK + (g & 1) * DH + half * DO);
-      if (DO == 16) {
-        tmem_ld16(src, pv);
-      } else {
-#pragma unroll
-        for (int cc = 0; cc < DO; cc += 32) tmem_ld32(src + (uint32_t)cc, pv + cc);
-      }
-#pragma unroll
-      for (int i = 0; i < DO; ++i) o[i] = o[i] * c + pv[i];
-      return true;
+    // this warp's DO columns of the output accumulator of unit counter ui
+    auto o_cols = [&](int ui) {
+      return tmem + lane_off + (uint32_t)(Cfg::kTiles * CK + (ui & 1) * DH + half * DO);
     };
-    // the finished unit whose last PV is still to be folded and stored
+    // o (this warp's DO columns, DO = 16 or 32) from / to TMEM
+    auto o_load = [&](uint32_t a, float* o) {
+      if constexpr (DO == 16)
+        tmem_ld16(a, o);
+      else
+        tmem_ld32(a, o);
+    };
+    // the finished unit whose output is still to be normalised and stored
     struct Done {
-      int h, q0, qcnt, qoff, ui;
-      float l, corr;
+      int h, q0, qcnt, qoff, ui, g;  // g: its last chunk
+      float l;
       bool active;
     } dn{};
     bool have_done = false;
-    float o[DO];
-    // fold the finished unit's last PV (chunk g), then O / l as a split pair
-    auto finish = [&](int g) -> bool {
-      if (dn.active && !fold(g, dn.corr, o)) return false;
+    // once the unit's last PV has completed: O / l (l summed over both key
+    // halves) as a split pair
+    auto finish = [&]() -> bool {
       float ltot = dn.l;
       if (Cfg::kHalves == 2) {
         float* rs = red_sum + (dn.ui & 1) * 256;
@@ -361,6 +365,11 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         pair_sync();
         ltot = rs[r] + rs[128 + r];
       }
+      if (!dn.active) return true;
+      if (!mbar_wait_compact(pv_full + (dn.g & 1), (dn.g >> 1) & 1, p.status)) return false;
+      tc_fence_after();
+      float o[DO];
+      o_load(o_cols(dn.ui), o);
       if (dn.q0 + r < dn.qcnt) {
         const float inv = 1.f / ltot;
         const size_t go = (size_t)(dn.qoff + dn.q0 + r) * p.ldo + p.o_col + dn.h * DH + half * DO;
@@ -379,7 +388,12 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     bool ok = true;
     Cursor c;
     for (cur_first(p, units, c); c.u < units && ok; cur_next(p, units, c)) {
-      float m = -INFINITY, l = 0.f, corr = 1.f;
+      // the running maximum m that P is taken against moves only when a chunk's
+      // maximum exceeds it by more than kSlack (log2 units; P <= 2^kSlack stays
+      // far inside f16), and then the unit's output accumulator in TMEM is
+      // rescaled: most chunks need no correction at all
+      constexpr float kSlack = 8.f;
+      float m = -INFINITY, l = 0.f;
       // a warp whose 32 query rows all lie past the segment's end only keeps
       // the barrier protocol; those rows of P and of the output are never used
       const bool active = c.q0 + q4 * 32 < c.qcnt;
@@ -390,8 +404,6 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           ok = false;
           break;
         }
-        const float corr_prev = corr;
-        corr = 1.f;
         if (active) {
           tc_fence_after();
           const uint32_t tile = tmem + lane_off + (uint32_t)(t * CK + half * KW);
@@ -416,13 +428,39 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
             pair_sync();
             mx = fmaxf(rm[r], rm[128 + r]);
           }
-          const float mn = fmaxf(m, mx);
-          corr = ex2_approx(m - mn);
-          m = mn;
+          if (j == 0) {
+            m = mx;  // the unit's first PV overwrites the accumulator
+          } else {
+            const bool up = mx > m + kSlack;
+            if (__any_sync(0xffffffffu, up)) {
+              // the accumulator holds PV up to chunk gc - 1: scale it (and l) to the new maximum
+              if (!mbar_wait_compact(pv_full + ((gc - 1) & 1), ((gc - 1) >> 1) & 1, p.status)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const float corr = up ? ex2_approx(m - mx) : 1.f;
+              if (up) m = mx;
+              l *= corr;
+              float o[DO];
+              const uint32_t oa = o_cols(ui);
+              o_load(oa, o);
+#pragma unroll
+              for (int i = 0; i < DO; ++i) o[i] *= corr;
+              if constexpr (DO == 16) {
+                uint32_t ou[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) ou[i] = __float_as_uint(o[i]);
+                tmem_st16_nowait(oa, ou);
+              } else {
+                tmem_st32(oa, o);
+              }
+            }
+          }
           // P = 2^(s * scale - m) as f16 over the first KW/2 of this warp's KW
           // S columns (all of them already in registers): keys 2c, 2c+1 in
           // column c
-          const float sc = p.scale_log2, nm = -mn;
+          const float sc = p.scale_log2, nm = -m;
           float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
           for (int hb = 0; hb < KW / 32; ++hb) {
@@ -437,28 +475,16 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
             }
             tmem_st16_nowait(tile + (uint32_t)(16 * hb), pk);
           }
-          const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
-          l = l * corr + sum;
+          l += (s4[0] + s4[1]) + (s4[2] + s4[3]);
           tmem_st_wait();
           tc_fence_before();
         }
         mbar_arrive1(p_full + t);
-        // the previous chunk's PV is folded while PV_j runs; at a unit's first
-        // chunk that is the last PV of the previous unit, which is then stored
-        if (j > 0) {
-          if (active && !fold(gc - 1, corr_prev, o)) {
-            ok = false;
-            break;
-          }
-        } else if (have_done) {
-          if (!finish(gc - 1)) {
-            ok = false;
-            break;
-          }
-        }
-        if (j == 0) {
-#pragma unroll
-          for (int i = 0; i < DO; ++i) o[i] = 0.f;
+        // at a unit's first chunk, the previous unit's output is stored (its
+        // last PV has completed or is about to)
+        if (j == 0 && have_done && !finish()) {
+          ok = false;
+          break;
         }
       }
       if (!ok) break;
@@ -467,13 +493,13 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       dn.qcnt = c.qcnt;
       dn.qoff = c.qoff;
       dn.ui = ui;
+      dn.g = gc - 1;
       dn.l = l;
-      dn.corr = corr;
       dn.active = active;
       have_done = true;
       ++ui;
     }
-    if (ok && have_done) finish(gc - 1);
+    if (ok && have_done) finish();
   }
 
   __syncwarp();  // each warp arrives whole: single lanes ran the producer and MMA loops
