@@ -18,7 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG, "_build")
 LIB_PATH = os.path.join(PKG, "libfe.so")
 SOURCES = ["fe_api.cu", "fe_gemm.cu", "fe_attn.cu", "fe_ffn.cu", "fe_ctxkv.cu", "fe_misc.cu", "fe_noalloc.cu",
-           "fe_linattn.cu", "fe_embed.cu", "fe_seq.cu"]
+           "fe_linattn.cu", "fe_embed.cu", "fe_seq.cu", "fe_ffn256.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
 

@@ -264,6 +264,7 @@ struct Weight {
   Planes p;
   int N = 0, K_pad = 0, BN = 0, stages = 0;
   CUtensorMap fh{}, fl{};  // W1 of the fused FFN: 64 x 128 boxes; a fused FFN's tail weight: 64 x N
+  CUtensorMap b128{};      // the d = 256 FFN kernel's boxes: 64 x 128 of the (single) plane
 };
 
 int largest_bn(int N, int cap) {
@@ -330,6 +331,7 @@ struct fe_ctx {
   bool sel_dirty = false;  // a batch stopped before its score head: clear the words before the next one
   bool fused_embed = false;  // gather + LN + the first layer's Q projection in one kernel
   bool tail_q = false;     // the fused FFN of layer l also projects the next layer's Q
+  bool ffn_w = false;      // d = 256: the output projection and FFN in one kernel (fe_ffn256.cu), with the Q tail
   bool tail_kv = false;    // the fused FFN of the last layer also projects [WKs | WVs]
   bool fused_ctxkv = false;  // context LN + K/V projection in one kernel (d <= 128, bf16 inputs)
   bool seq_ok = false;       // the sequence stage can run as one kernel (fe_seq.cu) for suitable K, L
@@ -622,6 +624,34 @@ int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const We
   return FE_OK;
 }
 
+// The d = 256 output projection + FFN block (fe_ffn256.cu): x0 rows are x
+// itself unless x0_row is given; x_out goes to x; LN(x_out) to ln_out when
+// store_ln; with WQ the next layer's Q (f16) to q_out.
+int ffn256(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const Weight& W1, const Weight& W2,
+           const float* b1, const float* b2, const float* x0_row, const F32Rows& x, const Planes& ln_out, int rows,
+           const int* rows_dev, cudaStream_t s, int store_ln, const Weight* WQ = nullptr, Planes* q_out = nullptr) {
+  if (rows <= 0) return FE_OK;
+  Prof pf(c, site, s);
+  fe::Ffn256Params p{};
+  p.rows = rows;
+  p.rows_dev = rows_dev;
+  p.F = c->F;
+  p.b1 = b1;
+  p.b2 = b2;
+  p.x = x.p;
+  p.ldx = x.ld;
+  p.x0_row = x0_row;
+  p.store_ln = store_ln;
+  p.tail = WQ ? 1 : 0;
+  p.q_out = q_out ? q_out->h : nullptr;
+  p.ldq = q_out ? q_out->ld : 0;
+  p.eps = c->cfg.ln_eps;
+  p.status = c->status;
+  FE_CK(fe::ffn256_launch(&A.th, &A.tl, &WO.b128, &W1.b128, &W2.b128, WQ ? &WQ->b128 : nullptr, &ln_out.th,
+                          &ln_out.tl, p, s));
+  return FE_OK;
+}
+
 #define FE_RC(call)              \
   do {                           \
     int rc_ = (call);            \
@@ -777,7 +807,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   }
   for (int l = 0; l < Ly; ++l) {
     // (otherwise the embedding kernel or the previous layer's fused FFN wrote Q)
-    if ((l == 0 && !c->fused_embed) || (l > 0 && !c->tail_q)) {
+    if ((l == 0 && !c->fused_embed) || (l > 0 && !c->tail_q && !c->ffn_w)) {
       fe::GemmParams p{};
       p.out_f16 = 1;
       FE_RC(gemm(c, "gemm_item_q", fe::EPI_STORE, c->xln, c->wq[l], R, sumU, p, &c->q, nullptr, s));
@@ -826,6 +856,12 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
       FE_RC(ffn(c, "ffn_item", c->a, c->wo[l], c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), nullptr, c->h,
                 c->xln, R, sumU, s, (last || !c->tail_q) ? 1 : 0, WT, WT ? TO : nullptr,
                 (!last || (use_seq && WT)) ? 1 : 0, (last && use_seq && WT) ? c->elog : nullptr));
+    } else if (c->ffn_w) {
+      // d = 256: the next layer's Q as the tail; LN(x_out) stored after the last
+      // layer (the element encodings, which SeqEnc's projection reads)
+      const bool last = l == Ly - 1;
+      FE_RC(ffn256(c, "ffn_item", c->a, c->wo[l], c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), nullptr, c->h,
+                   c->xln, R, sumU, s, last ? 1 : 0, last ? nullptr : &c->wq[l + 1], last ? nullptr : &c->q));
     } else {
       fe::GemmParams po{};
       po.resid = c->h.p;
@@ -919,6 +955,9 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   if (c->fused_ffn) {
     FE_RC(ffn(c, "ffn_seq", c->o, c->os, c->w1s, c->w2s, tw(c, T_B1S), tw(c, T_B2S), tw(c, T_CLS), c->c, c->z, S,
               nullptr, s));
+  } else if (c->ffn_w) {
+    FE_RC(ffn256(c, "ffn_seq", c->o, c->os, c->w1s, c->w2s, tw(c, T_B1S), tw(c, T_B2S), tw(c, T_CLS), c->c, c->z, S,
+                 nullptr, s, 1));
   } else {
     {
       fe::GemmParams p{};
@@ -1315,7 +1354,7 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   int rc = FE_OK;
   if (fe::gemm_prepare() != cudaSuccess || fe::attn_prepare() != cudaSuccess || fe::misc_prepare() != cudaSuccess ||
       fe::ffn_prepare() != cudaSuccess || fe::ctxkv_prepare() != cudaSuccess || fe::linattn_prepare() != cudaSuccess ||
-      fe::embed_q_prepare() != cudaSuccess || fe::seq_prepare() != cudaSuccess)
+      fe::embed_q_prepare() != cudaSuccess || fe::seq_prepare() != cudaSuccess || fe::ffn256_prepare() != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "kernel attributes"));
   {
     size_t o = 0;
@@ -1356,6 +1395,12 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     for (int l = 0; l < Ly; ++l)
       if ((rc = map_fused_w1(c->w1[l], c->nb > 1)) != FE_OK) return fail(rc);
   }
+  c->ffn_w = !c->fused_ffn && fe::ffn256_supported(d, F, c->nb);
+  if (c->ffn_w) {
+    for (int l = 0; l < Ly; ++l)
+      for (Weight* w : {&c->wq[l], &c->wo[l], &c->w1[l], &c->w2[l]})
+        if ((rc = encode_map(&w->b128, w->p.h, w->p.ld, w->p.rows, 128)) != FE_OK) return fail(rc);
+  }
   if ((rc = make_weight(c, c->kvs, 2 * d, d, 128)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->kvs, tw(c, T_WKS), d, d, 0)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->kvs, tw(c, T_WVS), d, d, d)) != FE_OK) return fail(rc);
@@ -1377,6 +1422,9 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
     return fail(set_cuda_err(cudaGetLastError(), "device attribute"));
   if ((rc = make_weight(c, c->w2s, d, F, 512)) != FE_OK) return fail(rc);
   if ((rc = fill_weight(c->w2s, tw(c, T_W2S), F, d, 0)) != FE_OK) return fail(rc);
+  if (c->ffn_w)
+    for (Weight* w : {&c->os, &c->w1s, &c->w2s})
+      if ((rc = encode_map(&w->b128, w->p.h, w->p.ld, w->p.rows, 128)) != FE_OK) return fail(rc);
   if (!cfg->no_cross_seq) {
     if ((rc = make_weight(c, c->qkvx, 3 * d, d, 128)) != FE_OK) return fail(rc);
     if ((rc = fill_weight(c->qkvx, tw(c, T_WQX), d, d, 0)) != FE_OK) return fail(rc);

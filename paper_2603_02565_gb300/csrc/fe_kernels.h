@@ -140,6 +140,33 @@ struct FfnParams {
   float* tail_logits;
   int tail_col0;        // tail output column c is stored at column c - tail_col0 of the output map
 };
+// The same block for rows of width d = 256 (fe_ffn256.cu): x0 + A W_O, the
+// FFN, x_out (fp32, in place over x when x0_row is null), LN(x_out) (split
+// pair, by TMA through o_h / o_l, when store_ln), and with tail the next
+// layer's Q = LN(x_out) W_Q as f16 rows.  Weights are bf16-exact transposed
+// planes read through 64 x 128 boxes: W_O^T and W_Q^T [256, 256], W1^T
+// [F, 256], W2^T [256, F].
+struct Ffn256Params {
+  int rows;             // row extent of the A descriptors
+  const int* rows_dev;  // when set: number of valid rows, read on the device
+  int F;
+  const float* b1;      // [F]
+  const float* b2;      // [256]
+  float* x;             // [rows, ldx]: x0 in (unless x0_row), x_out out
+  int ldx;              // multiple of 4
+  const float* x0_row;  // [256], when set: the same input row for every row
+  int store_ln;
+  int tail;
+  bf16* q_out;          // [rows, ldq] f16 bits (tail)
+  int ldq;              // multiple of 8
+  float eps;
+  int* status;
+};
+bool ffn256_supported(int d, int F, int nb);
+cudaError_t ffn256_prepare();
+cudaError_t ffn256_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* wo, const CUtensorMap* w1,
+                          const CUtensorMap* w2, const CUtensorMap* wt, const CUtensorMap* o_h, const CUtensorMap* o_l,
+                          const Ffn256Params& p, cudaStream_t s);
 bool ffn_supported(int d, int d_pad, int F, int nb);
 bool ffn_tail_supported(int d, int d_pad, int F, int nb, int tail_n, int tail_f16);
 cudaError_t ffn_prepare();
