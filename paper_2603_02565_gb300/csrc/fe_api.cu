@@ -643,12 +643,10 @@ int ffn256(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const
   p.x0_row = x0_row;
   p.store_ln = store_ln;
   p.tail = WQ ? 1 : 0;
-  p.q_out = q_out ? q_out->h : nullptr;
-  p.ldq = q_out ? q_out->ld : 0;
   p.eps = c->cfg.ln_eps;
   p.status = c->status;
   FE_CK(fe::ffn256_launch(&A.th, &A.tl, &WO.b128, &W1.b128, &W2.b128, WQ ? &WQ->b128 : nullptr, &ln_out.th,
-                          &ln_out.tl, p, s));
+                          &ln_out.tl, &x.sx, q_out ? &q_out->th : nullptr, p, s));
   return FE_OK;
 }
 
@@ -1188,6 +1186,7 @@ int reserve_body(fe_ctx* c, const Shape& s, const bool fact) {
   for (Planes* p : {&c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp}) FE_RC(map_act(*p));
   for (Planes* p : {&c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->lncp}) FE_RC(map_out(*p));
   for (Planes* p : {&c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
+  if (c->ffn_w) FE_RC(encode_map(&c->q.th, c->q.h, c->q.ld, c->q.rows, 128));  // the d = 256 FFN's Q stores
   if (c->cfg.elem_self_attn) FE_RC(map_attn(c->eqkv, c->dh));
   FE_RC(c->fused_ctxkv ? map_attn_hm(c->KV, c->dh) : map_attn(c->KV, c->dh));
   c->cap_shape = s;

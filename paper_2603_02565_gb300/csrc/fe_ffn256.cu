@@ -21,8 +21,9 @@
 // 2-9 (two per TMEM lane quadrant, each owning 128 of a row's 256 columns)
 // run the epilogues: x0 + projection, LayerNorm statistics exchanged with the
 // partner warp, LN(x) as the split operand tile over the A tile, bias + ReLU
-// + split per chunk, x_out + b2 to memory, LN(x_out) over the A tile (stored
-// by TMA), and the tail's f16 output.  Products take split bf16 activations
+// + split per chunk, x_out + b2 (staged over the A tile and stored by TMA),
+// LN(x_out) over the A tile (stored by TMA), and the tail's f16 output (over
+// the A tile, stored by TMA).  Products take split bf16 activations
 // (hi + lo) times exact bf16 weights with fp32 accumulation; LayerNorm and
 // residuals are fp32.
 #include "fe_common.cuh"
@@ -100,6 +101,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                   const __grid_constant__ CUtensorMap tWO, const __grid_constant__ CUtensorMap tW1,
                   const __grid_constant__ CUtensorMap tW2, const __grid_constant__ CUtensorMap tT,
                   const __grid_constant__ CUtensorMap tO_h, const __grid_constant__ CUtensorMap tO_l,
+                  const __grid_constant__ CUtensorMap tX, const __grid_constant__ CUtensorMap tQ,
                   const Ffn256Params p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_s = smem_u32(smem_raw);
@@ -431,16 +433,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         warp_arrive(mid_full + ba);
       }
       if (!ok) break;
-      // ---- x_out = acc2 + b2 to memory; LN(x_out) over the A tile (every FFN1
-      // has read LN(x) there)
+      // ---- x_out = acc2 + b2 to memory, staged in this warp's 16 KB of sA (every
+      // FFN1 has read LN(x) there) as four 32 x 32 blocks (128-byte swizzle)
+      // and stored by TMA; then LN(x_out) over the A tile
       if (!wait(acc2_full, tl & 1)) break;
       tc_fence_after();
+      uint8_t* xst = sA + (size_t)ew * 16384u;
 #pragma unroll
       for (int k = 0; k < 4; ++k) s4[k] = 0.f;
       for (int i = 0; i < 4; ++i) {
         const int c = c0 + 32 * i;
         float v[32];
         tmem_ld32(acc2 + lane_off + (uint32_t)c, v);
+        uint8_t* blk = xst + (size_t)i * 4096u + (uint32_t)lane * 128u;
 #pragma unroll
         for (int j = 0; j < 32; j += 4) {
           const float4 bb = *reinterpret_cast<const float4*>(sB2 + c + j);
@@ -452,8 +457,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           s4[1] += v[j + 1];
           s4[2] += v[j + 2];
           s4[3] += v[j + 3];
-          if (valid) *reinterpret_cast<float4*>(xrow + c + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+          *reinterpret_cast<float4*>(blk + ((uint32_t)((j >> 2) ^ (lane & 7)) << 4)) =
+              make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
         }
+      }
+      fence_async_shared();
+      __syncwarp();
+      if (lane == 0) {
+        for (int i = 0; i < 4; ++i) tma_store_2d(&tX, xst + (size_t)i * 4096u, c0 + 32 * i, m0 + 32 * q);
+        bulk_commit();
       }
       const float mean = pair_mean((s4[0] + s4[1]) + (s4[2] + s4[3]));
 #pragma unroll
@@ -469,6 +481,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       const float rstd = pair_rstd((s4[0] + s4[1]) + (s4[2] + s4[3]));
+      if (lane == 0) bulk_wait_read0();
+      epi_sync();  // every warp's x_out staging read: sA takes LN(x_out)
       for (int i = 0; i < 4; ++i) {
         const int c = c0 + 32 * i;
         float v[32];
@@ -490,7 +504,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           bulk_commit();
         }
       }
-      // ---- the tail: Q = LN(x_out) W_Q as f16, this thread's 128 columns
+      // ---- the tail: Q = LN(x_out) W_Q as f16 over sA (the tail product has read
+      // LN(x_out)): this thread's 128 columns of row r as 128-byte-swizzled
+      // [kb][128 rows x 64] tiles, stored by TMA
       if (p.tail) {
         if (!wait(tail_full, tl & 1)) break;
         tc_fence_after();
@@ -498,22 +514,26 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int c = c0 + 32 * i;
           float v[32];
           tmem_ld32(tmem + lane_off + (uint32_t)c, v);
-          if (valid) {
-            uint4* dst = reinterpret_cast<uint4*>(p.q_out + (size_t)(m0 + r) * p.ldq + c);
+          uint8_t* rowp = sA + (size_t)(c >> 6) * kBox + (size_t)r * 128u;
+          const int u0 = (c & 63) >> 3;
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-              dst[j] = make_uint4(pack_f16x2(v[8 * j], v[8 * j + 1]), pack_f16x2(v[8 * j + 2], v[8 * j + 3]),
-                                  pack_f16x2(v[8 * j + 4], v[8 * j + 5]), pack_f16x2(v[8 * j + 6], v[8 * j + 7]));
-          }
+          for (int j = 0; j < 4; ++j)
+            *reinterpret_cast<uint4*>(rowp + ((uint32_t)((u0 + j) ^ (r & 7)) << 4)) =
+                make_uint4(pack_f16x2(v[8 * j], v[8 * j + 1]), pack_f16x2(v[8 * j + 2], v[8 * j + 3]),
+                           pack_f16x2(v[8 * j + 4], v[8 * j + 5]), pack_f16x2(v[8 * j + 6], v[8 * j + 7]));
         }
         tc_fence_before();
+        fence_async_shared();
+        epi_sync();  // every row of Q written
+        if (et == 0) {
+          for (int kb = 0; kb < NKB; ++kb) tma_store_2d(&tQ, sA + (size_t)kb * kBox, kb * BK, m0);
+          bulk_commit();
+        }
       }
       // ---- sA and the TMEM columns [0, 256) may take the next tile once the
       // stores have read sA
-      if (p.store_ln) {
-        if (et == 0) bulk_wait_read0();
-        epi_sync();
-      }
+      if (et == 0) bulk_wait_read0();
+      epi_sync();
       warp_arrive(a_free);
     }
     if (et == 0) bulk_wait0();  // output tensor stores complete before the CTA retires
@@ -541,15 +561,14 @@ cudaError_t ffn256_prepare() {
 
 cudaError_t ffn256_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* wo, const CUtensorMap* w1,
                           const CUtensorMap* w2, const CUtensorMap* wt, const CUtensorMap* o_h, const CUtensorMap* o_l,
-                          const Ffn256Params& p, cudaStream_t s) {
+                          const CUtensorMap* x_st, const CUtensorMap* q_st, const Ffn256Params& p, cudaStream_t s) {
   if (p.rows <= 0) return cudaSuccess;
-  if (!ffn256_supported(D, p.F, 1) || !p.x || p.ldx < D || p.ldx % 4 || (p.tail && (!wt || !p.q_out || p.ldq % 8)))
-    return cudaErrorInvalidValue;
+  if (!ffn256_supported(D, p.F, 1) || !x_st || (p.tail && !wt) || (p.tail && !q_st)) return cudaErrorInvalidValue;
   const long long tiles = (p.rows + BM - 1) / BM;
   long long grid = g_ffn256_sms > 0 ? g_ffn256_sms : 148;
   if (grid > tiles) grid = tiles;
   return launch_k(ffn256_kernel, dim3((unsigned)grid), dim3(kThreads), kSmem, s, *a_h, *a_l, *wo, *w1, *w2,
-                  p.tail ? *wt : *wo, *o_h, *o_l, p);
+                  p.tail ? *wt : *wo, *o_h, *o_l, *x_st, p.tail ? *q_st : *o_h, p);
 }
 
 }  // namespace fe

@@ -157,16 +157,15 @@ struct Ffn256Params {
   const float* x0_row;  // [256], when set: the same input row for every row
   int store_ln;
   int tail;
-  bf16* q_out;          // [rows, ldq] f16 bits (tail)
-  int ldq;              // multiple of 8
   float eps;
   int* status;
 };
 bool ffn256_supported(int d, int F, int nb);
 cudaError_t ffn256_prepare();
+// x_st: fp32 x rows, 32 x 32 boxes (128-byte swizzle); q_st: Q rows, 64 x 128 boxes (128-byte swizzle)
 cudaError_t ffn256_launch(const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* wo, const CUtensorMap* w1,
                           const CUtensorMap* w2, const CUtensorMap* wt, const CUtensorMap* o_h, const CUtensorMap* o_l,
-                          const Ffn256Params& p, cudaStream_t s);
+                          const CUtensorMap* x_st, const CUtensorMap* q_st, const Ffn256Params& p, cudaStream_t s);
 bool ffn_supported(int d, int d_pad, int F, int nb);
 bool ffn_tail_supported(int d, int d_pad, int F, int nb, int tail_n, int tail_f16);
 cudaError_t ffn_prepare();
