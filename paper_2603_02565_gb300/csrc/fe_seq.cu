@@ -270,6 +270,10 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
   constexpr int NR = BM / (4 * kEpiWarps);
   const int g = lane >> 3, li = lane & 7;
   const int hc = (16 * li) / DH;
+  // lanes 4-7 of a group hold their two 8-column halves in the other order
+  // (register i <-> column 16 li + ((i + 8 rot) mod 16)), so that each 16-byte
+  // load of a staged row and of a position row touches distinct banks
+  const int rot = (li >> 2) & 1;
   int rrow[NR];
   bool live[NR];
 #pragma unroll
@@ -307,7 +311,7 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
   for (int j = 0; j < L; ++j) {
     const float qp = sQkP[j * 4 + hc];
     const float4* vp = reinterpret_cast<const float4*>(sVP + (size_t)j * D + 16 * li);
-    const float4 pp[4] = {vp[0], vp[1], vp[2], vp[3]};
+    const float4 pp[4] = {vp[(2 * rot) & 3], vp[(1 + 2 * rot) & 3], vp[(2 + 2 * rot) & 3], vp[(3 + 2 * rot) & 3]};
 #pragma unroll
     for (int k = 0; k < NR; ++k) {
       if (!live[k]) continue;
@@ -316,7 +320,7 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
       const uint4* src = (kStaged || (unsigned)er < (unsigned)nst)
                              ? reinterpret_cast<const uint4*>(sStage + (size_t)er * 256 + 32 * li)
                              : reinterpret_cast<const uint4*>(v_h + (size_t)e * D + 16 * li);
-      const uint4 a4 = src[0], b4 = src[1];
+      const uint4 a4 = src[rot], b4 = src[rot ^ 1];
       const float w = ex2_approx((part(e) + qp) * sl2 - m[k]);
       sum[k] += w;
       const uint32_t wv[8] = {a4.x, a4.y, a4.z, a4.w, b4.x, b4.y, b4.z, b4.w};
@@ -338,20 +342,20 @@ __device__ __forceinline__ void cls_rows(uint8_t* sA, const int* sErow, const ui
       const float pc = ex2_approx(s0 - m[k]);
       const float inv = 1.f / (sum[k] + pc);
 #pragma unroll
-      for (int i = 0; i < 16; ++i) o[k][i] = fmaf(pc, sV0[16 * li + i], o[k][i]) * inv;
+      for (int i = 0; i < 16; ++i) o[k][i] = fmaf(pc, sV0[16 * li + ((i + 8 * rot) & 15)], o[k][i]) * inv;
     } else if (rr < rows_v) {
       // a rejected request's scores become NaN; o = v0 keeps its rows finite
 #pragma unroll
-      for (int i = 0; i < 16; ++i) o[k][i] = sV0[16 * li + i];
+      for (int i = 0; i < 16; ++i) o[k][i] = sV0[16 * li + ((i + 8 * rot) & 15)];
     }
-    // o -> row rr of the split tile: columns 16 li .. 16 li + 15 are 16-byte
-    // pieces 2 (li % 4) and 2 (li % 4) + 1 of plane li / 4
+    // o -> row rr of the split tile: registers 0-7 (columns 16 li + 8 rot ..) are
+    // 16-byte piece 2 (li % 4) + rot of plane li / 4, registers 8-15 the other piece
     uint32_t hi[8], lo[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) split2(o[k][2 * i], o[k][2 * i + 1], hi[i], lo[i]);
     uint8_t* rowp = sA + (size_t)((li >> 2) * 2) * kAPlane + (size_t)rr * 128u;
-    const uint32_t o0 = (uint32_t)((2 * (li & 3)) ^ (rr & 7)) << 4;
-    const uint32_t o1 = (uint32_t)((2 * (li & 3) + 1) ^ (rr & 7)) << 4;
+    const uint32_t o0 = (uint32_t)((2 * (li & 3) + rot) ^ (rr & 7)) << 4;
+    const uint32_t o1 = (uint32_t)((2 * (li & 3) + (rot ^ 1)) ^ (rr & 7)) << 4;
     *reinterpret_cast<uint4*>(rowp + o0) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
     *reinterpret_cast<uint4*>(rowp + o1) = make_uint4(hi[4], hi[5], hi[6], hi[7]);
     *reinterpret_cast<uint4*>(rowp + kAPlane + o0) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
