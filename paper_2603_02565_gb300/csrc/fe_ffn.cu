@@ -431,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t proj = tmem + (uint32_t)((gf % NA1) * FC);  // A W_O
       if (!mbar_wait_bounded(o_done, tl & 1, p.status)) break;
       tc_fence_after();
-      float sum = 0.f;
+      float s4[4] = {0.f, 0.f, 0.f, 0.f};  // four independent partial sums per statistic
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
@@ -442,16 +442,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             v[j] += w[j];
-            sum += v[j];
+            s4[j & 3] += v[j];
           }
           tmem_st32(acc2 + lane_off + (uint32_t)c, v);
         }
       }
-      red_sum[half * 128 + r] = sum;
+      red_sum[half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
       pair_sync();
       const float mean0 = (red_sum[r] + red_sum[128 + r]) / (float)d;
       // x is read back from the accumulator rather than kept in registers
-      float var0 = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) s4[i] = 0.f;
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         const int c = 32 * half + 64 * ci;
@@ -461,11 +462,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             const float dv = v[j] - mean0;
-            var0 = fmaf(dv, dv, var0);
+            s4[j & 3] = fmaf(dv, dv, s4[j & 3]);
           }
         }
       }
-      red_var[half * 128 + r] = var0;
+      red_var[half * 128 + r] = (s4[0] + s4[1]) + (s4[2] + s4[3]);
       pair_sync();
       const float rstd0 = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)d + p.eps);
       // row r of planes (kb, hi) and (kb, lo), 128-byte swizzle: this warp's
@@ -567,25 +568,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       red_sum[half * 128 + r] = sum2;
       pair_sync();
       const float mean = (red_sum[r] + red_sum[128 + r]) / (float)d;
-      float var = 0.f;
+      float v4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int ci = 0; ci < 2; ++ci) {
         if (32 * half + 64 * ci < d) {
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const float4 x = *reinterpret_cast<const float4*>(blk(ci) + xoff(j));
-            float dv = x.x - mean;
-            var = fmaf(dv, dv, var);
-            dv = x.y - mean;
-            var = fmaf(dv, dv, var);
-            dv = x.z - mean;
-            var = fmaf(dv, dv, var);
-            dv = x.w - mean;
-            var = fmaf(dv, dv, var);
+            const float d0 = x.x - mean, d1 = x.y - mean, d2 = x.z - mean, d3 = x.w - mean;
+            v4[0] = fmaf(d0, d0, v4[0]);
+            v4[1] = fmaf(d1, d1, v4[1]);
+            v4[2] = fmaf(d2, d2, v4[2]);
+            v4[3] = fmaf(d3, d3, v4[3]);
           }
         }
       }
-      red_var[half * 128 + r] = var;
+      red_var[half * 128 + r] = (v4[0] + v4[1]) + (v4[2] + v4[3]);
       pair_sync();
       const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)d + p.eps);
       // LN(x_out) as the split tile [kb][plane] in sA, 128-byte swizzle (every
