@@ -265,6 +265,9 @@ struct Weight {
   int N = 0, K_pad = 0, BN = 0, stages = 0;
   CUtensorMap fh{}, fl{};  // W1 of the fused FFN: 64 x 128 boxes; a fused FFN's tail weight: 64 x N
   CUtensorMap b128{};      // the d = 256 FFN kernel's boxes: 64 x 128 of the (single) plane
+  // RESID_LN with clusters, N = cs x 128 or cs x 64: boxes of 64 x 128 / 64 x 64 on both planes
+  CUtensorMap c128h{}, c128l{}, c64h{}, c64l{};
+  bool cmaps = false;
 };
 
 int largest_bn(int N, int cap) {
@@ -539,6 +542,14 @@ int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
   const int box = w.BN > 256 ? 256 : w.BN;
   rc = encode_map(&w.p.th, w.p.h, w.p.ld, w.p.rows, box);
   if (rc == FE_OK) rc = encode_map(&w.p.tl, c->nb > 1 ? w.p.l : w.p.h, w.p.ld, w.p.rows, box);
+  if (rc == FE_OK && N >= 256 && N % 128 == 0) {
+    const bf16* lo = c->nb > 1 ? w.p.l : w.p.h;
+    rc = encode_map(&w.c128h, w.p.h, w.p.ld, w.p.rows, 128);
+    if (rc == FE_OK) rc = encode_map(&w.c128l, lo, w.p.ld, w.p.rows, 128);
+    if (rc == FE_OK) rc = encode_map(&w.c64h, w.p.h, w.p.ld, w.p.rows, 64);
+    if (rc == FE_OK) rc = encode_map(&w.c64l, lo, w.p.ld, w.p.rows, 64);
+    w.cmaps = rc == FE_OK;
+  }
   return rc;
 }
 
@@ -583,9 +594,29 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   p.nb = c->nb;
   p.stages = 0;  // chosen by gemm_launch
   p.nacc = 0;
+  p.cs = 1;
   p.status = c->status;
   p.eps = c->cfg.ln_eps;
-  FE_CK(fe::gemm_launch(epi, &A.th, &A.tl, &W.p.th, &W.p.tl, out ? &out->sh : nullptr, out ? &out->sl : nullptr,
+  const CUtensorMap *bh = &W.p.th, *bl = &W.p.tl;
+  // LayerNorm rows wider than 128 columns with fewer row tiles than SMs: a
+  // cluster of cs CTAs shares each row tile, 128 (or, with very few tiles, 64)
+  // columns per CTA, and exchanges the row statistics through distributed
+  // shared memory, so that more SMs multiply and the epilogue is split cs ways
+  if (epi == fe::EPI_RESID_LN && W.cmaps) {
+    const int mtiles = (rows + 127) / 128;
+    int cs = W.N / 128, bn = 128;
+    if (mtiles * cs * 4 <= c->n_sms && cs * 2 <= 8) {
+      cs *= 2;
+      bn = 64;
+    }
+    if (mtiles < c->n_sms && cs <= 8 && fe::gemm_cluster_capacity(cs) > 0) {
+      p.cs = cs;
+      p.BN = bn;
+      bh = bn == 128 ? &W.c128h : &W.c64h;
+      bl = bn == 128 ? &W.c128l : &W.c64l;
+    }
+  }
+  FE_CK(fe::gemm_launch(epi, &A.th, &A.tl, bh, bl, out ? &out->sh : nullptr, out ? &out->sl : nullptr,
                         xout ? &xout->sx : nullptr, p, s));
   return FE_OK;
 }

@@ -15,6 +15,8 @@
 //                    alternate 32-column chunks
 // The activation is a split pair (hi + lo bf16); the product is
 // A_hi W_hi + A_lo W_hi (+ A_hi W_lo when the weights carry a lo plane).
+#include <cstdlib>
+
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 #include "fe_select.cuh"
@@ -38,7 +40,8 @@ constexpr size_t kSmemMaxBlock = 232448;             // 227 KB opt-in per block
 constexpr int kEpiWarps = 8;                         // two per TMEM lane quadrant, alternating 32-column chunks
 constexpr uint32_t kStageOut = 4096;                 // one staging buffer: 32 rows x 128 B
 constexpr uint32_t kRedBytes = 4 * 2 * 128 * 4;      // row-reduction exchange: [parity][sum|var][half][128]
-constexpr size_t kSmemExtra = 1024 + 256 + 1024 + kEpiWarps * 2 * kStageOut + kRedBytes;
+// alignment slack, barriers, staging; then the row-reduction area (red_bytes)
+constexpr size_t kSmemFixed = 1024 + 256 + 1024 + kEpiWarps * 2 * kStageOut;
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kMaxStages = 8;
 
@@ -47,23 +50,78 @@ int g_num_sms = 0;
 __host__ __device__ inline uint32_t pow2_cols(int n) {
   return n <= 32 ? 32u : n <= 64 ? 64u : n <= 128 ? 128u : n <= 256 ? 256u : 512u;
 }
+
+// Row-reduction area: the pair exchange within a CTA, or with clusters of cs > 1
+// the partial row sums of every CTA of the cluster, [sum|var][cs][half][128].
+__host__ __device__ inline uint32_t red_bytes(int cs) { return cs > 1 ? (uint32_t)cs * 2048u : kRedBytes; }
+constexpr int kMaxCluster = 8;
+int g_cluster_cap[2][kMaxCluster + 1] = {};  // resident clusters of size cs with one / two CTAs per SM
+int g_cluster_limit = -1;                 // FE_GEMM_CLUSTERS: 0 disables clusters, n > 0 caps clusters per launch
+bool g_two_per_sm[3][2] = {};             // [EPI][NB - 1]: two CTAs fit on an SM (registers) at half the shared memory
 }  // namespace
 
-size_t gemm_smem_bytes(int BN, int nb, int stages) {
+size_t gemm_smem_bytes(int BN, int nb, int stages, int cs) {
   const size_t stage = 2 * (size_t)kATile + (size_t)nb * BN * BK * 2;
-  return (size_t)stages * stage + kSmemExtra;
+  return (size_t)stages * stage + kSmemFixed + red_bytes(cs);
 }
 
-int gemm_max_stages(int BN, int nb, int K_pad) {
+int gemm_max_stages(int BN, int nb, int K_pad, int cs) {
   (void)K_pad;  // stages run ahead across tiles, so the ring is not capped by one tile's k blocks
   const size_t stage = 2 * (size_t)kATile + (size_t)nb * BN * BK * 2;
-  int s = (int)((kSmemMaxBlock - kSmemExtra) / stage);
+  int s = (int)((kSmemMaxBlock - kSmemFixed - red_bytes(cs)) / stage);
   if (s > kMaxStages) s = kMaxStages;
   return s < 1 ? 1 : s;
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// ---- thread-block cluster helpers (the RESID_LN row exchange) ----
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// every thread of every CTA of the cluster; orders the barrier initialisation
+// before any remote access, and keeps each CTA's shared memory alive until the
+// cluster's last remote store to it
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t map_peer(uint32_t local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+// 4-byte store into a peer CTA's shared memory, counted on the peer's mbarrier
+__device__ __forceinline__ void st_async_peer(uint32_t addr, float v, uint32_t bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(addr),
+               "r"(__float_as_uint(v)), "r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// bounded like mbar_wait_bounded, acquiring at cluster scope (the peers' stores)
+__device__ __noinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity, int* status) {
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if ((it & 255u) == 255u && (*reinterpret_cast<volatile int*>(status) & ST_TIMEOUT)) return false;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      atomicOr(status, ST_TIMEOUT);
+      return false;
+    }
+  }
 }
 
 // NB: weight planes (1 when the weights are exact in bf16, else 2); a
@@ -81,13 +139,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int nb = NB;
   const int BN = p.BN, S = p.stages;
   const int nacc = p.nacc;
+  const int cs = p.cs > 1 ? p.cs : 1;  // (uniform) CTAs of a cluster sharing each row tile
   const uint32_t b_bytes = (uint32_t)BN * BK * 2;
   const uint32_t stage_bytes = 2 * kATile + (uint32_t)nb * b_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;  // [2] accumulator ready for the epilogue
   uint64_t* tempty = tfull + 2; // [2] accumulator drained by the epilogue
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  uint64_t* xbar = tempty + 2;  // [2] cluster row exchange: partial sums / partial variances received
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(xbar + 2);
   // output staging: two 4 KB buffers per epilogue warp, 1024-byte aligned; then
   // the row-reduction exchange of the two warps sharing a lane quadrant
   uint8_t* stg_base = smem + (((size_t)S * stage_bytes + 256 + 1023) & ~(size_t)1023);
@@ -106,6 +166,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(tfull + a, 1);
       mbar_init(tempty + a, kEpiWarps);  // one arrival per epilogue warp
     }
+    if (cs > 1) {
+      mbar_init(xbar, 1);  // the local expect_tx; the peers' stores complete the bytes
+      mbar_init(xbar + 1, 1);
+    }
     fence_mbar_init();
     prefetch_tmap(&tA_h);
     prefetch_tmap(&tA_l);
@@ -115,6 +179,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) tmem_alloc(tmem_slot, ncols);
   tc_fence_before();
   __syncthreads();
+  if (cs > 1) cluster_sync_all();  // the peers' barriers exist before any store to them
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int nk = p.K_pad / BK;
@@ -122,6 +187,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();
   int rows_valid = p.rows;
   if (p.rows_dev) rows_valid = min(*p.rows_dev, p.rows);
+  // With clusters nt == cs and the grid is a multiple of cs: CTA rank k of a
+  // cluster always takes column tile k, and the cluster's CTAs walk the same
+  // row tiles in the same order (and leave together below).
   const int nt = p.N / BN;
   const int tiles = ((rows_valid + BM - 1) / BM) * nt;
   if ((int)blockIdx.x >= tiles) {  // nothing for this CTA (uniform)
@@ -238,7 +306,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       issue(&tO_h, b, &tO_l, b + 2048, col, row);
     };
 
+    // Clusters (EPI_RESID_LN, cs > 1): each CTA holds BN columns of the rows; the
+    // row sums and then the sums of squared deviations of every warp are stored
+    // into all cs CTAs' exchange areas ([cs][half][128] per kind) with st.async,
+    // which counts the bytes on the receiver's xbar[kind]; one local thread
+    // posts the expected cs * 1 KB.  Each CTA adds the 2 * cs partials of a row
+    // in the same order, so the cluster's CTAs use identical statistics.  A
+    // peer stores the next tile's partials of one kind only after it received
+    // this CTA's partials of the other kind, which each warp sends after it read
+    // the current ones, so one area per kind suffices.
     int tl = 0;
+    const uint32_t my_rank = cs > 1 ? cluster_rank() : 0u;
+    auto row_xchg = [&](int kind, float v, float& tot) -> bool {
+      float* xs = red + (size_t)kind * cs * 256;
+      const uint32_t slot = smem_u32(xs + (my_rank * 2 + half) * 128 + r);
+      const uint32_t bar = smem_u32(xbar + kind);
+      for (int k = 0; k < cs; ++k) st_async_peer(map_peer(slot, (uint32_t)k), v, map_peer(bar, (uint32_t)k));
+      if (ew == 0 && lane == 0) mbar_arrive_expect_tx(xbar + kind, (uint32_t)cs * 1024u);
+      if (!mbar_wait_cluster(xbar + kind, (uint32_t)tl & 1u, p.status)) return false;
+      float a = 0.f;
+      for (int k = 0; k < cs; ++k) a += xs[(2 * k) * 128 + r] + xs[(2 * k + 1) * 128 + r];
+      tot = a;
+      return true;
+    };
+
     float xr[64];  // EPI_RESID_LN with BN <= 128: this warp's chunks of the row
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tl) {
       const int acc = tl % nacc, use = tl / nacc;
@@ -254,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             float4 qv = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (valid && c < BN) qv = reinterpret_cast<const float4*>(rrow + c)[j];
+            if (valid && c < BN) qv = reinterpret_cast<const float4*>(rrow + n0 + c)[j];
             xr[32 * ci + 4 * j] = qv.x;
             xr[32 * ci + 4 * j + 1] = qv.y;
             xr[32 * ci + 4 * j + 2] = qv.z;
@@ -321,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 32; ++i) xr[32 * ci + i] += v[i];
             if (p.bias) {
-              const float4* b4 = reinterpret_cast<const float4*>(p.bias + c);
+              const float4* b4 = reinterpret_cast<const float4*>(p.bias + n0 + c);
 #pragma unroll
               for (int j = 0; j < 8; ++j) {
                 const float4 bb = __ldg(b4 + j);
@@ -342,12 +433,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                   make_float4(xr[32 * ci + 4 * j], xr[32 * ci + 4 * j + 1], xr[32 * ci + 4 * j + 2],
                               xr[32 * ci + 4 * j + 3]);
             }
-            issue(&tO_x, b, nullptr, nullptr, c, srow);
+            issue(&tO_x, b, nullptr, nullptr, n0 + c, srow);
           }
         }
-        red_sum[half * 128 + r] = sum;
-        pair_sync();
-        const float mean = (red_sum[r] + red_sum[128 + r]) / (float)BN;
+        float mean, rstd, tot = 0.f;
+        if (cs > 1) {
+          if (!row_xchg(0, sum, tot)) break;
+          mean = tot / (float)p.N;
+        } else {
+          red_sum[half * 128 + r] = sum;
+          pair_sync();
+          mean = (red_sum[r] + red_sum[128 + r]) / (float)BN;
+        }
         float var = 0.f;
 #pragma unroll
         for (int ci = 0; ci < 2; ++ci) {
@@ -359,9 +456,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
         }
-        red_var[half * 128 + r] = var;
-        pair_sync();
-        const float rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)BN + p.eps);
+        if (cs > 1) {
+          if (!row_xchg(1, var, tot)) break;
+          rstd = 1.0f / sqrtf(tot / (float)p.N + p.eps);
+        } else {
+          red_var[half * 128 + r] = var;
+          pair_sync();
+          rstd = 1.0f / sqrtf((red_var[r] + red_var[128 + r]) / (float)BN + p.eps);
+        }
 #pragma unroll
         for (int ci = 0; ci < 2; ++ci) {
           const int c = 32 * half + 64 * ci;
@@ -370,7 +472,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 32; i += 2)
               split2((xr[32 * ci + i] - mean) * rstd, (xr[32 * ci + i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
-            stage_split(hi, lo, c, srow);
+            stage_split(hi, lo, n0 + c, srow);
           }
         }
       } else if (EPI == EPI_RESID_LN) {
@@ -496,6 +598,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncwarp();  // each warp arrives whole: single lanes ran the producer and MMA loops
   tc_fence_before();
   __syncthreads();
+  if (cs > 1) cluster_sync_all();  // no peer still stores into this CTA's exchange area
   if (warp == 0) tmem_dealloc(tmem, ncols);
   if (EPI == EPI_HEAD && p.sel.keys) sel_ticket(p.sel, tmem_slot);
 }
@@ -505,6 +608,8 @@ static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, cons
                             const CUtensorMap* b_l, const CUtensorMap* o_h, const CUtensorMap* o_l,
                             const CUtensorMap* o_x, const GemmParams& p0, cudaStream_t s) {
   GemmParams p = p0;
+  const int cs = (EPI == EPI_RESID_LN && p.cs > 1) ? p.cs : 1;
+  p.cs = cs;
   const int sms = g_num_sms > 0 ? g_num_sms : 148;
   const long long tiles = (long long)((p.rows + BM - 1) / BM) * (p.N / p.BN);
   const size_t stage = 2 * (size_t)kATile + (size_t)p.nb * p.BN * BK * 2;
@@ -512,22 +617,34 @@ static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, cons
   // co-resident CTAs overlap each other's loads, MMAs and epilogues.
   // Otherwise: one persistent CTA per SM with a double-buffered accumulator.
   int per_sm = 1;
-  const int st2 = (int)((kSmemPerSM / 2 - 1024 - kSmemExtra) / stage);
-  if (tiles <= 2LL * sms && st2 >= 1 && 2 * pow2_cols(p.BN) <= 512) {
+  const int st2 = (int)((kSmemPerSM / 2 - 1024 - kSmemFixed - red_bytes(cs)) / stage);
+  if (tiles <= 2LL * sms && st2 >= 1 && 2 * pow2_cols(p.BN) <= 512 && g_two_per_sm[EPI][NB - 1]) {
     per_sm = 2;
     p.nacc = 1;
     p.stages = st2 < kMaxStages ? st2 : kMaxStages;
   } else {
     p.nacc = 2 * p.BN <= 512 ? 2 : 1;
-    p.stages = gemm_max_stages(p.BN, p.nb, p.K_pad);
+    p.stages = gemm_max_stages(p.BN, p.nb, p.K_pad, cs);
   }
-  size_t smem = gemm_smem_bytes(p.BN, p.nb, p.stages);
+  size_t smem = gemm_smem_bytes(p.BN, p.nb, p.stages, cs);
   // (CTAs resident per SM) x (TMEM columns per CTA) <= 512: no CTA ever waits in
   // tcgen05.alloc for a co-resident one
   const size_t max_ctas = 512 / pow2_cols(p.nacc * p.BN);
   const size_t floor_bytes = kSmemPerSM / (max_ctas + 1) + 1;
   if (smem < floor_bytes) smem = floor_bytes;
   if (smem > kSmemMaxBlock) smem = kSmemMaxBlock;
+  if (cs > 1) {
+    // as many whole clusters as can be resident at once (the CTAs of a cluster
+    // share a GPC), persistent over the row tiles; tiles is a multiple of cs
+    if (p.N != cs * p.BN || p.BN > 128 || cs > kMaxCluster) return cudaErrorInvalidValue;
+    long long nclu = g_cluster_cap[per_sm - 1][cs];
+    if (nclu < 1) return cudaErrorInvalidConfiguration;
+    if (g_cluster_limit > 0 && nclu > g_cluster_limit) nclu = g_cluster_limit;
+    long long grid = nclu * cs;
+    if (grid > tiles) grid = tiles;
+    return launch_kc(gemm_kernel<EPI, NB>, dim3((unsigned)grid), dim3(kThreads), smem, s, cs, *a_h, *a_l, *b_h,
+                     *b_l, o_h ? *o_h : *a_h, o_l ? *o_l : *a_l, o_x ? *o_x : *a_h, p);
+  }
   long long grid = (long long)sms * per_sm;
   if (grid > tiles) grid = tiles;
   return launch_k(gemm_kernel<EPI, NB>, dim3((unsigned)grid), dim3(kThreads), smem, s, *a_h, *a_l, *b_h, *b_l,
@@ -547,7 +664,53 @@ cudaError_t gemm_prepare() {
   attr((const void*)gemm_kernel<EPI_RESID_LN, 2>);
   attr((const void*)gemm_kernel<EPI_HEAD, 1>);
   attr((const void*)gemm_kernel<EPI_HEAD, 2>);
+  auto two_fit = [&](const void* f) {
+    int n = 0;
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, f, kThreads, kSmemPerSM / 2 - 1024);
+    return n >= 2;
+  };
+  g_two_per_sm[EPI_STORE][0] = two_fit((const void*)gemm_kernel<EPI_STORE, 1>);
+  g_two_per_sm[EPI_STORE][1] = two_fit((const void*)gemm_kernel<EPI_STORE, 2>);
+  g_two_per_sm[EPI_RESID_LN][0] = two_fit((const void*)gemm_kernel<EPI_RESID_LN, 1>);
+  g_two_per_sm[EPI_RESID_LN][1] = two_fit((const void*)gemm_kernel<EPI_RESID_LN, 2>);
+  g_two_per_sm[EPI_HEAD][0] = two_fit((const void*)gemm_kernel<EPI_HEAD, 1>);
+  g_two_per_sm[EPI_HEAD][1] = two_fit((const void*)gemm_kernel<EPI_HEAD, 2>);
+  if (g_cluster_limit < 0) {
+    const char* v = std::getenv("FE_GEMM_CLUSTERS");
+    g_cluster_limit = v && *v ? std::atoi(v) : 0x7fffffff;
+  }
+  // resident clusters per size, for one CTA per SM (all the shared memory) and two
+  for (int two = 0; two < 2 && e == cudaSuccess; ++two) {
+    for (int cs = 2; cs <= kMaxCluster; cs *= 2) {
+      int n1 = 0, n2 = 0;
+      for (int nbv = 1; nbv <= 2; ++nbv) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)cs);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = two ? kSmemPerSM / 2 - 1024 : kSmemMaxBlock;
+        cudaLaunchAttribute a[1];
+        a[0].id = cudaLaunchAttributeClusterDimension;
+        a[0].val.clusterDim.x = (unsigned)cs;
+        a[0].val.clusterDim.y = 1;
+        a[0].val.clusterDim.z = 1;
+        cfg.attrs = a;
+        cfg.numAttrs = 1;
+        int n = 0;
+        const void* f = nbv == 1 ? (const void*)gemm_kernel<EPI_RESID_LN, 1> : (const void*)gemm_kernel<EPI_RESID_LN, 2>;
+        if (cudaOccupancyMaxActiveClusters(&n, f, &cfg) != cudaSuccess) {
+          (void)cudaGetLastError();
+          n = 0;
+        }
+        (nbv == 1 ? n1 : n2) = n;
+      }
+      g_cluster_cap[two][cs] = g_cluster_limit == 0 ? 0 : (n1 < n2 ? n1 : n2);
+    }
+  }
   return e;
+}
+
+int gemm_cluster_capacity(int cs) {
+  return (cs >= 2 && cs <= kMaxCluster) ? g_cluster_cap[0][cs] : 0;
 }
 
 cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l, const CUtensorMap* b_h,

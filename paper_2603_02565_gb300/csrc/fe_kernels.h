@@ -39,6 +39,27 @@ inline cudaError_t launch_k(void (*kern)(KArgs...), dim3 grid, dim3 block, size_
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// The same launch with thread-block clusters of cs CTAs along x (cs > 1).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_kc(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, int cs,
+                             Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)cs;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cs > 1 ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // ---------------------------------------------------------------------------
 // tcgen05 GEMM:  D[r, n] = sum over planes  A_p[r, :] . B_q[n, :]
 // A: activation as two bf16 planes (hi, lo), row-major [rows, K_pad]
@@ -73,6 +94,7 @@ struct GemmParams {
   int nb;               // weight planes: 1 (exact bf16) or 2 (hi + lo)
   int stages;           // shared-memory pipeline depth (chosen by gemm_launch)
   int nacc;             // TMEM accumulators, 1 or 2 (chosen by gemm_launch)
+  int cs;               // EPI_RESID_LN: CTAs per cluster sharing one row tile (N = cs * BN, BN <= 128), 0/1: none
   const float* bias;    // [N] or null
   int relu;
   int out_f16;          // EPI_STORE: one f16 plane through o_h (attention operands) instead of bf16 hi/lo
@@ -96,8 +118,11 @@ struct GemmParams {
 
 // Raises the dynamic shared-memory limit of the GEMM kernels (call once per device, outside capture).
 cudaError_t gemm_prepare();
-size_t gemm_smem_bytes(int BN, int nb, int stages);
-int gemm_max_stages(int BN, int nb, int K_pad);
+size_t gemm_smem_bytes(int BN, int nb, int stages, int cs = 1);
+int gemm_max_stages(int BN, int nb, int K_pad, int cs = 1);
+// Clusters of cs CTAs (2, 4 or 8) that can be resident at once for the EPI_RESID_LN kernels (0 when
+// such clusters cannot be scheduled, or when FE_GEMM_CLUSTERS=0); valid after gemm_prepare.
+int gemm_cluster_capacity(int cs);
 // o_h / o_l: output bf16 planes (EPI_STORE: the product, EPI_RESID_LN: LN(x)), tensor maps with
 // 32 x 32 boxes and the 64-byte swizzle; o_x: the fp32 x_out rows of EPI_RESID_LN, 32 x 32 boxes,
 // 128-byte swizzle.  Unused maps may be null.
