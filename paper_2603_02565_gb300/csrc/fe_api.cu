@@ -358,6 +358,7 @@ struct fe_ctx {
   float* lin_states = nullptr;      // linear-attention context states [segments][Ly][H][d_h^2 + d_h]
   float *q0 = nullptr, *k0 = nullptr, *v0 = nullptr, *kP = nullptr, *vP = nullptr;
   float* qk = nullptr;  // [max_L + 1][4]: q0 . kP[j] and q0 . k0 per head (the sequence-stage kernel)
+  float* qkH = nullptr;  // [max_L + 1][H]: the same per head for any H (the [CLS] attention kernel)
   // workspace
   Shape cap_shape;  // reserved maxima
   int cap_rows = 0; // element rows of the reservation: B * min(M, K*L), or B * K * L once factorized
@@ -648,7 +649,9 @@ int ffn(fe_ctx* c, const char* site, const Planes& A, const Weight& WO, const We
   p.status = c->status;
   p.tail_q0 = tail_logits ? c->q0 : nullptr;
   p.tail_logits = tail_logits;
-  p.tail_col0 = tail_logits ? c->d : 0;  // the value columns go to their own [rows, d] buffer
+  // with logits the key columns are not stored: the value columns go to column 0 of a
+  // [rows, d] buffer, or stay at column d of a [rows, 2d] one
+  p.tail_col0 = (tail_logits && tail_out && tail_out->ld < 2 * c->d) ? c->d : 0;
   FE_CK(fe::ffn_launch(&A.th, &A.tl, &WO.p.th, &WO.p.tl, &W1.fh, &W1.fl, &W2.p.th, &W2.p.tl, &ln_out.th, &ln_out.tl,
                        &x.sx, WT ? &WT->fh : nullptr, WT ? &WT->fl : nullptr, tail_out ? &tail_out->sh : nullptr,
                        tail_out ? &tail_out->sl : nullptr, p, s));
@@ -884,7 +887,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
       const Planes* TO = !last ? &c->q : (use_seq ? &c->vI16 : &c->kvI);
       FE_RC(ffn(c, "ffn_item", c->a, c->wo[l], c->w1[l], c->w2[l], lw(c, l, T_B1), lw(c, l, T_B2), nullptr, c->h,
                 c->xln, R, sumU, s, (last || !c->tail_q) ? 1 : 0, WT, WT ? TO : nullptr,
-                (!last || (use_seq && WT)) ? 1 : 0, (last && use_seq && WT) ? c->elog : nullptr));
+                (!last || (use_seq && WT)) ? 1 : 0, (last && WT) ? c->elog : nullptr));
     } else if (c->ffn_w) {
       // d = 256: the next layer's Q as the tail; LN(x_out) stored after the last
       // layer (the element encodings, which SeqEnc's projection reads)
@@ -911,7 +914,12 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   }
   // element projections of SeqEnc: H WKs | H WVs (unless the last fused FFN did them)
   if (!(c->fused_ffn && c->tail_kv)) {
+    // the key half leaves as the [CLS] logit partials only
     fe::GemmParams p{};
+    p.lq = c->q0;
+    p.lq_n = d;
+    p.logits = c->elog;
+    p.ld_logit = d / 32;
     FE_RC(gemm(c, "gemm_item_seq_kv", fe::EPI_STORE, c->xln, c->kvs, R, sumU, p, &c->kvI, nullptr, s));
   }
   if (use_seq) {
@@ -969,10 +977,10 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     cp.kv_h = c->kvI.h;
     cp.kv_l = c->kvI.l;
     cp.ldkv = c->kvI.ld;
-    cp.q0 = c->q0;
-    cp.k0 = c->k0;
+    cp.elog = c->elog;
+    cp.qkP = c->qkH;
+    cp.qk0 = c->qkH + (size_t)c->cfg.max_L * c->H;
     cp.v0 = c->v0;
-    cp.kP = c->kP;
     cp.vP = c->vP;
     cp.o_h = c->o.h;
     cp.o_l = c->o.l;
@@ -1165,8 +1173,8 @@ int reserve_body(fe_ctx* c, const Shape& s, const bool fact) {
   c->sel_ticket = reinterpret_cast<unsigned*>(c->sel_nan + B);
   FE_RC(dalloc((void**)&c->slot, (size_t)B * (size_t)(capL > 0 ? capL : 1) * sizeof(int)));
   FE_RC(dalloc((void**)&c->list, (size_t)R * sizeof(int)));
+  FE_RC(dalloc((void**)&c->elog, (size_t)R * (size_t)(d / 32) * sizeof(float)));
   if (c->seq_ok) {
-    FE_RC(dalloc((void**)&c->elog, (size_t)R * (size_t)(d / 32) * sizeof(float)));
     FE_RC(alloc_planes(c->vI16, R, d, false, c->owned_ws));
     FE_RC(encode_map_t(&c->vI16.sh, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->vI16.h, d, c->vI16.rows, 32, 32,
                        CU_TENSOR_MAP_SWIZZLE_64B));
@@ -1498,7 +1506,8 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   // weight-only products of SeqEnc: [CLS] W and P W
   const int mL = cfg->max_L;
   float* consts = nullptr;
-  if (dev_alloc((void**)&consts, ((size_t)(3 + 2 * mL) * d + (size_t)(mL + 1) * 4) * sizeof(float)) != cudaSuccess)
+  if (dev_alloc((void**)&consts, ((size_t)(3 + 2 * mL) * d + (size_t)(mL + 1) * (4 + c->H)) * sizeof(float)) !=
+      cudaSuccess)
     return fail(FE_ERR_OOM);
   c->owned_w.push_back(consts);
   c->q0 = consts;
@@ -1507,12 +1516,14 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   c->kP = consts + 3 * d;
   c->vP = consts + (size_t)(3 + mL) * d;
   c->qk = consts + (size_t)(3 + 2 * mL) * d;
+  c->qkH = c->qk + (size_t)(mL + 1) * 4;
   if (fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WQS), d, c->q0, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WKS), d, c->k0, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_CLS), 1, d, tw(c, T_WVS), d, c->v0, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WKS), d, c->kP, 0) != cudaSuccess ||
       fe::small_matmul_launch(tw(c, T_P), mL, d, tw(c, T_WVS), d, c->vP, 0) != cudaSuccess ||
-      fe::seq_consts_launch(c->q0, c->k0, c->kP, mL, d, c->dh, c->qk, 0) != cudaSuccess)
+      fe::seq_consts_launch(c->q0, c->k0, c->kP, mL, d, c->dh, c->qk, 0) != cudaSuccess ||
+      fe::cls_consts_launch(c->q0, c->k0, c->kP, mL, d, c->H, c->qkH, 0) != cudaSuccess)
     return fail(set_cuda_err(cudaGetLastError(), "SeqEnc constants"));
   if (host_alloc((void**)&c->host_status, sizeof(int)) != cudaSuccess) return fail(FE_ERR_OOM);
   *c->host_status = 0;

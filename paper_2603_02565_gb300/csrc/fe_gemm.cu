@@ -380,6 +380,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = relu_nan(v[i]);
           }
+          if (col < p.lq_n) {
+            // a key chunk of SeqEnc: only its [CLS] logit partial leaves the SM
+            const float4* q4 = reinterpret_cast<const float4*>(p.lq + col);
+            float a = 0.f;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 qq = __ldg(q4 + j);
+              a = fmaf(v[4 * j], qq.x, a);
+              a = fmaf(v[4 * j + 1], qq.y, a);
+              a = fmaf(v[4 * j + 2], qq.z, a);
+              a = fmaf(v[4 * j + 3], qq.w, a);
+            }
+            if (valid) p.logits[(size_t)grow * p.ld_logit + (size_t)(col / 32)] = a;
+            continue;
+          }
           if (p.out_f16) {
             // one f16 plane (an attention operand)
             uint8_t* b = next_stage();

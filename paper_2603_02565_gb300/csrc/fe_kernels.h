@@ -98,6 +98,12 @@ struct GemmParams {
   const float* bias;    // [N] or null
   int relu;
   int out_f16;          // EPI_STORE: one f16 plane through o_h (attention operands) instead of bf16 hi/lo
+  // EPI_STORE: output columns below lq_n are not stored; each 32-column chunk c of such a row r leaves
+  // as the partial dot product logits[r * ld_logit + c / 32] = sum_i out[r, c + i] lq[c + i]
+  const float* lq;
+  int lq_n;
+  float* logits;
+  int ld_logit;
   // EPI_RESID_LN (outputs through the o_x / o_h / o_l tensor maps)
   const float* resid;   // residual rows (ldr == 0: one row broadcast to every row)
   int ldr;
@@ -337,14 +343,20 @@ struct ClsParams {
   const int* off;
   const int* bad;
   const int* slot_local;  // [B, K, L]
-  const bf16 *kv_h, *kv_l;  // element projections [rows, 2d]: keys | values
+  const float* elog;      // [rows, d / 32] element [CLS] logit partials q0 . (H WKs) per 32-column chunk
+  const bf16 *kv_h, *kv_l;  // element projections [rows, 2d]: values in columns d .. 2d - 1
   int ldkv;
-  const float *q0, *k0, *v0;  // [CLS] WQs, [CLS] WKs, [CLS] WVs
-  const float *kP, *vP;       // P WKs, P WVs  [max_L, d]
+  const float* qkP;       // [max_L, H] q0 . (P WKs) per head
+  const float* qk0;       // [H] q0 . ([CLS] WKs) per head
+  const float* v0;        // [CLS] WVs
+  const float* vP;        // P WVs  [max_L, d]
   bf16 *o_h, *o_l;
   int ldo;
-  float scale;                // 1 / sqrt(d_h)
+  float scale;            // 1 / sqrt(d_h)
 };
+// qk[j * H + h] = q0 . kP[j] over head h's columns for j < max_L, and qk[max_L * H + h] = q0 . k0
+cudaError_t cls_consts_launch(const float* q0, const float* k0, const float* kP, int max_L, int d, int H, float* qk,
+                              cudaStream_t s);
 cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s);
 
 // ---------------------------------------------------------------------------

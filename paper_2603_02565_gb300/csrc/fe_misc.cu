@@ -421,79 +421,165 @@ cudaError_t gather_ln_launch(const void* pool, int io_f32, int B, int M, int d, 
 }
 
 // ---------------------------------------------------------------------------
-// SeqEnc [CLS] attention: one warp per sequence (b, k).  Tokens are [CLS]
-// (key/value = [CLS] WKs / WVs) and the L indexed elements, whose keys/values
-// are the cached element projections plus the position projections
-// (x_j W = H[i] W + P[j-1] W; positions added after indexing).
+// SeqEnc [CLS] attention: W = 1, 2, 4 or 8 warps per sequence (b, k) and 8 / W
+// sequences per CTA.  Tokens are [CLS] and the L indexed elements, whose keys
+// and values are the cached element projections plus the position projections
+// (x_j W = H[i] W + P[j-1] W; positions added after indexing).  Only the [CLS]
+// query is needed, so a key enters through its logit
+//   q0 . (H[i] WKs + P[j-1] WKs) = sum of the element's per-chunk partials
+//                                  q0 . (H[i] WKs) + a per-position constant,
+// and a key costs its value row (and the position's value row) only.  Warp w of
+// a sequence takes the keys j = w, w + W, ... with its own running maximum and
+// sum per head and its own output row; with W > 1 the W partial results are
+// merged in shared memory (softmax over all keys = the partial sums rescaled to
+// the largest partial maximum), so that few long sequences still give every SM
+// several warps.  Short position tables (L d <= kVpStage) are staged in shared
+// memory once per CTA.
 // ---------------------------------------------------------------------------
+constexpr int kVpStage = 6144;  // floats
+
 template <int DPL>
-__global__ void __launch_bounds__(256) cls_attn_kernel(const ClsParams p) {
-  const int lane = threadIdx.x & 31;
-  const int seq = blockIdx.x * 8 + (threadIdx.x >> 5);
-  pdl_wait();
-  pdl_trigger();
-  if (seq >= p.B * p.K) return;
-  const int b = seq / p.K;
+__global__ void __launch_bounds__(256) cls_attn_kernel(const ClsParams p, int W) {
+  extern __shared__ float cls_sm[];  // W > 1: [8][d] partial rows, [8][32] maxima, [8][32] sums; then P WVs
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int seq = blockIdx.x * (8 / W) + warp / W;
+  const int wi = warp % W;  // this warp's share of the keys
   const int d = p.d;
   const int lph = 32 / p.H;  // lanes per head
+  const int hd = lane / lph;  // this lane's head
+  const int cph = (d / p.H) / 32;  // logit chunks per head (1 or 2)
+  const int nch = d / 32;
   const int d0 = lane * DPL;
-  float q[DPL], kx[DPL], vx[DPL], o[DPL];
-  load_vec<DPL>(p.q0 + d0, q);
-  load_vec<DPL>(p.k0 + d0, kx);
-  load_vec<DPL>(p.v0 + d0, vx);
-  // token 0: [CLS]
-  float s = 0.f;
-#pragma unroll
-  for (int i = 0; i < DPL; ++i) s = fmaf(q[i], kx[i], s);
-  for (int o2 = 1; o2 < lph; o2 <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o2);
-  float m = s * p.scale, l = 1.f;
-#pragma unroll
-  for (int i = 0; i < DPL; ++i) o[i] = vx[i];
-  const int L = p.bad[b] ? 0 : p.L;
-  const int base = p.off[b];
-  const int* sl = p.slot_local + (size_t)seq * p.L;
-  // lane j holds slot j (one load for the first 32 keys), so a key's rows are
-  // requested without first waiting for its slot index
-  const int my_slot = lane < L ? sl[lane] : 0;
-  for (int j = 0; j < L; ++j) {
-    const int slot = j < 32 ? __shfl_sync(0xffffffffu, my_slot, j) : sl[j];
-    const size_t row = (size_t)(base + slot) * p.ldkv;
-    float kp[DPL], vp[DPL];
-    load_split<DPL>(p.kv_h + row + d0, p.kv_l + row + d0, kx);
-    load_split<DPL>(p.kv_h + row + d + d0, p.kv_l + row + d + d0, vx);
-    load_vec<DPL>(p.kP + (size_t)j * d + d0, kp);
-    load_vec<DPL>(p.vP + (size_t)j * d + d0, vp);
-    s = 0.f;
-#pragma unroll
-    for (int i = 0; i < DPL; ++i) s = fmaf(q[i], kx[i] + kp[i], s);
-    for (int o2 = 1; o2 < lph; o2 <<= 1) s += __shfl_xor_sync(0xffffffffu, s, o2);
-    s *= p.scale;
-    const float mn = fmaxf(m, s);
-    const float c = expf(m - mn);
-    const float e = expf(s - mn);
-    l = l * c + e;
-#pragma unroll
-    for (int i = 0; i < DPL; ++i) o[i] = o[i] * c + e * (vx[i] + vp[i]);
-    m = mn;
+  // P WVs rows are parameters: staged before the programmatic wait
+  const bool vp_smem = p.L * d <= kVpStage;
+  float* svp = cls_sm + (W > 1 ? 8 * d + 512 : 0);
+  if (vp_smem) {
+    const float4* src = reinterpret_cast<const float4*>(p.vP);
+    for (int i = threadIdx.x; i < p.L * d / 4; i += blockDim.x) reinterpret_cast<float4*>(svp)[i] = src[i];
   }
-  const float inv = 1.f / l;
+  const float* vpb = vp_smem ? svp : p.vP;
+  pdl_wait();
+  pdl_trigger();
+  if (vp_smem) __syncthreads();
+  const bool live = seq < p.B * p.K;
+  float o[DPL];
+  float m = -INFINITY, l = 0.f;
 #pragma unroll
-  for (int i = 0; i < DPL; ++i) o[i] *= inv;
-  store_split<DPL>(o, p.o_h + (size_t)seq * p.ldo + d0, p.o_l + (size_t)seq * p.ldo + d0);
+  for (int i = 0; i < DPL; ++i) o[i] = 0.f;
+  if (live) {
+    const int b = seq / p.K;
+    if (wi == 0) {  // token 0: [CLS]
+      m = p.qk0[hd] * p.scale;
+      l = 1.f;
+      load_vec<DPL>(p.v0 + d0, o);
+    }
+    const int L = p.bad[b] ? 0 : p.L;
+    const int base = p.off[b];
+    const int* sl = p.slot_local + (size_t)seq * p.L;
+    const int nk = L > wi ? (L - wi + W - 1) / W : 0;  // keys of this warp
+    // lane i holds the slot of the warp's key i (one load for its first 32 keys),
+    // so a key's rows are requested without first waiting for its slot index
+    const int my_slot = lane < nk ? sl[wi + lane * W] : 0;
+    for (int i = 0; i < nk; ++i) {
+      const int j = wi + i * W;
+      const int slot = i < 32 ? __shfl_sync(0xffffffffu, my_slot, i) : sl[j];
+      const size_t er = (size_t)(base + slot);
+      const float* lg = p.elog + er * nch + (size_t)(hd * cph);
+      float s = lg[0];
+      if (cph > 1) s += lg[1];
+      s = (s + p.qkP[j * p.H + hd]) * p.scale;
+      float vx[DPL], vp[DPL];
+      load_split<DPL>(p.kv_h + er * p.ldkv + d + d0, p.kv_l + er * p.ldkv + d + d0, vx);
+      load_vec<DPL>(vpb + (size_t)j * d + d0, vp);
+      const float mn = fmaxf(m, s);
+      const float c = expf(m - mn);  // 0 while m is -inf (a warp's first key)
+      const float e = expf(s - mn);
+      l = l * c + e;
+#pragma unroll
+      for (int t = 0; t < DPL; ++t) o[t] = o[t] * c + e * (vx[t] + vp[t]);
+      m = mn;
+    }
+  }
+  if (W == 1) {
+    if (live) {
+      const float inv = 1.f / l;
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) o[i] *= inv;
+      store_split<DPL>(o, p.o_h + (size_t)seq * p.ldo + d0, p.o_l + (size_t)seq * p.ldo + d0);
+    }
+    return;
+  }
+  float* so = cls_sm;             // [8][d]
+  float* sm = cls_sm + 8 * d;     // [8][32]
+  float* ss = sm + 256;           // [8][32]
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) so[warp * d + d0 + i] = o[i];
+  sm[warp * 32 + lane] = m;
+  ss[warp * 32 + lane] = l;
+  __syncthreads();
+  if (!live) return;
+  // the sequence's W warps merge its row, two adjacent columns per thread; a
+  // column's maximum and sum are those of the lane that owns it (equal on all
+  // lanes of a head); warp 0 of the sequence holds [CLS], so the maximum is finite
+  const int g0 = warp - wi;
+  for (int c = 2 * (wi * 32 + lane); c < d; c += 64 * W) {
+    float r[2];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int ln = (c + u) / DPL;
+      float M = -INFINITY;
+      for (int w = 0; w < W; ++w) M = fmaxf(M, sm[(g0 + w) * 32 + ln]);
+      float sum = 0.f, acc = 0.f;
+      for (int w = 0; w < W; ++w) {
+        const float e = expf(sm[(g0 + w) * 32 + ln] - M);
+        sum = fmaf(ss[(g0 + w) * 32 + ln], e, sum);
+        acc = fmaf(so[(g0 + w) * d + c + u], e, acc);
+      }
+      r[u] = acc / sum;
+    }
+    uint32_t hw, lw;
+    split2(r[0], r[1], hw, lw);
+    *reinterpret_cast<uint32_t*>(p.o_h + (size_t)seq * p.ldo + c) = hw;
+    *reinterpret_cast<uint32_t*>(p.o_l + (size_t)seq * p.ldo + c) = lw;
+  }
 }
 
 cudaError_t cls_attn_launch(const ClsParams& p, cudaStream_t s) {
   const int n = p.B * p.K;
   if (n <= 0) return cudaSuccess;
-  const unsigned g = (unsigned)((n + 7) / 8);
+  // warps per sequence: enough warps in flight (about 4096) for the latency of
+  // the gathered rows, at least two keys per warp
+  int W = 1;
+  while (W < 8 && 2 * W <= p.L && (long long)n * W < 4096) W *= 2;
+  const unsigned g = (unsigned)((n + 8 / W - 1) / (8 / W));
+  const size_t smem = ((W > 1 ? (size_t)(8 * p.d + 512) : 0) + (p.L * p.d <= kVpStage ? (size_t)p.L * p.d : 0)) *
+                      sizeof(float);
   switch (p.d) {
-    case 32: return launch_k(cls_attn_kernel<1>, dim3(g), dim3(256), 0, s, p);
-    case 64: return launch_k(cls_attn_kernel<2>, dim3(g), dim3(256), 0, s, p);
-    case 128: return launch_k(cls_attn_kernel<4>, dim3(g), dim3(256), 0, s, p);
-    case 256: return launch_k(cls_attn_kernel<8>, dim3(g), dim3(256), 0, s, p);
-    case 512: return launch_k(cls_attn_kernel<16>, dim3(g), dim3(256), 0, s, p);
+    case 32: return launch_k(cls_attn_kernel<1>, dim3(g), dim3(256), smem, s, p, W);
+    case 64: return launch_k(cls_attn_kernel<2>, dim3(g), dim3(256), smem, s, p, W);
+    case 128: return launch_k(cls_attn_kernel<4>, dim3(g), dim3(256), smem, s, p, W);
+    case 256: return launch_k(cls_attn_kernel<8>, dim3(g), dim3(256), smem, s, p, W);
+    case 512: return launch_k(cls_attn_kernel<16>, dim3(g), dim3(256), smem, s, p, W);
     default: return cudaErrorInvalidValue;
   }
+  return cudaGetLastError();
+}
+
+__global__ void cls_consts_kernel(const float* q0, const float* k0, const float* kP, int max_L, int d, int H,
+                                  float* out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (max_L + 1) * H) return;
+  const int j = i / H, h = i % H, dh = d / H;
+  const float* kv = j < max_L ? kP + (size_t)j * d : k0;
+  float acc = 0.f;
+  for (int c = h * dh; c < h * dh + dh; ++c) acc = fmaf(q0[c], kv[c], acc);
+  out[i] = acc;
+}
+
+cudaError_t cls_consts_launch(const float* q0, const float* k0, const float* kP, int max_L, int d, int H, float* qk,
+                              cudaStream_t s) {
+  const int n = (max_L + 1) * H;
+  cls_consts_kernel<<<(n + 127) / 128, 128, 0, s>>>(q0, k0, kP, max_L, d, H, qk);
   return cudaGetLastError();
 }
 
