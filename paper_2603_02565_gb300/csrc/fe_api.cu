@@ -337,6 +337,9 @@ struct fe_ctx {
   bool ffn_w = false;      // d = 256: the output projection and FFN in one kernel (fe_ffn256.cu), with the Q tail
   bool tail_kv = false;    // the fused FFN of the last layer also projects [WKs | WVs]
   bool fused_ctxkv = false;  // context LN + K/V projection in one kernel (d <= 128, bf16 inputs)
+  bool ctx_fold = false;     // otherwise with bf16 inputs: the GEMM multiplies the raw rows and folds the LN in
+  float2* ctx_stats = nullptr;  // [B C] (mean, rstd) of the context rows (ctx_fold)
+  float* kv_colsum = nullptr;   // [2 Ly d] column sums of the K/V weight (ctx_fold)
   bool seq_ok = false;       // the sequence stage can run as one kernel (fe_seq.cu) for suitable K, L
   bool keep_inter = false;   // store c and C' even where the sequence-stage kernel keeps them on chip
   int n_sms = 148;
@@ -590,7 +593,7 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   p.rows = rows;
   p.rows_dev = rows_dev;
   p.N = W.N;
-  p.BN = (epi == fe::EPI_STORE) ? W.BN : W.N;
+  p.BN = (epi == fe::EPI_STORE || epi == fe::EPI_LN_FOLD) ? W.BN : W.N;
   p.K_pad = W.K_pad;
   p.nb = c->nb;
   p.stages = 0;  // chosen by gemm_launch
@@ -760,6 +763,23 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     if (lin_fused) p.states = c->lin_states;  // the context goes straight to its linear-attention states
     Prof pf(c, lin_fused ? "ctx_ln_state" : "ctx_ln_kv", s);
     FE_CK(fe::ctxkv_launch(&tx, &c->ctxkv_w, &c->KV.sh, c->dpad, p, s));
+  } else if (c->ctx_fold) {
+    // LN(x) W = rstd (x W) - mu rstd colsum(W): the GEMM multiplies the raw bf16
+    // context rows (one exact plane) and applies the row statistics in its epilogue
+    {
+      Prof pf(c, "ctx_stats", s);
+      FE_CK(fe::row_stats_launch(static_cast<const bf16*>(io.ctx), B * C, d, c->cfg.ln_eps, c->ctx_stats, s));
+    }
+    Planes raw;
+    raw.h = static_cast<bf16*>(const_cast<void*>(io.ctx));
+    raw.ld = d;
+    raw.rows = B * C;
+    FE_RC(encode_map(&raw.th, raw.h, d, B * C, 128));
+    raw.tl = raw.th;
+    fe::GemmParams p{};
+    p.row_stats = c->ctx_stats;
+    p.colsum = c->kv_colsum;
+    FE_RC(gemm(c, "gemm_ctx_kv", fe::EPI_LN_FOLD, raw, c->ctx_kv, B * C, nullptr, p, &c->KV, nullptr, s));
   } else {
     {
       Prof pf(c, "ctx_ln", s);
@@ -1206,7 +1226,8 @@ int reserve_body(fe_ctx* c, const Shape& s, const bool fact) {
     FE_RC(dalloc((void**)&c->slots[k].scores, (size_t)S * sizeof(float)));
     FE_RC(dalloc((void**)&c->slots[k].best, (size_t)B * sizeof(int32_t)));
   }
-  if (!c->fused_ctxkv) FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
+  if (!c->fused_ctxkv && !c->ctx_fold) FE_RC(alloc_planes(c->X, BC, c->dpad, true, c->owned_ws));
+  if (c->ctx_fold) FE_RC(dalloc((void**)&c->ctx_stats, (size_t)BC * sizeof(float2)));
   FE_RC(alloc_planes(c->KV, (int)kv_rows, 2 * Ly * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->xln, R, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->q, R, d, false, c->owned_ws));
@@ -1221,7 +1242,7 @@ int reserve_body(fe_ctx* c, const Shape& s, const bool fact) {
   if (c->cfg.elem_self_attn) FE_RC(alloc_planes(c->eqkv, R, 3 * d, false, c->owned_ws));
   FE_RC(alloc_planes(c->ax, S, c->dpad, true, c->owned_ws));
   FE_RC(alloc_planes(c->lncp, S, c->dpad, true, c->owned_ws));
-  if (!c->fused_ctxkv) FE_RC(map_act(c->X));
+  if (!c->fused_ctxkv && !c->ctx_fold) FE_RC(map_act(c->X));
   for (Planes* p : {&c->xln, &c->a, &c->mid, &c->o, &c->cln, &c->mids, &c->z, &c->ax, &c->lncp}) FE_RC(map_act(*p));
   for (Planes* p : {&c->xln, &c->mid, &c->kvI, &c->cln, &c->mids, &c->z, &c->lncp}) FE_RC(map_out(*p));
   for (Planes* p : {&c->q, &c->qkv}) FE_RC(map_attn(*p, c->dh));
@@ -1414,6 +1435,14 @@ int fe_init(const fe_config* cfg, const float* weights, size_t n_floats, fe_ctx*
   c->fused_ctxkv = fe::ctxkv_supported(d, c->dpad, 2 * Ly * d, c->nb, c->cfg.io_dtype == FE_IO_F32);
   if (c->fused_ctxkv && (rc = encode_map(&c->ctxkv_w, c->ctx_kv.p.h, c->ctx_kv.p.ld, c->ctx_kv.p.rows, 128)) != FE_OK)
     return fail(rc);
+  c->ctx_fold = !c->fused_ctxkv && c->cfg.io_dtype != FE_IO_F32 && d % 64 == 0;
+  if (c->ctx_fold) {
+    if (dev_alloc((void**)&c->kv_colsum, (size_t)c->ctx_kv.N * sizeof(float)) != cudaSuccess) return fail(FE_ERR_OOM);
+    c->owned_w.push_back(c->kv_colsum);
+    if (fe::colsum_launch(c->ctx_kv.p.h, c->nb > 1 ? c->ctx_kv.p.l : nullptr, c->ctx_kv.p.ld, c->ctx_kv.N, d,
+                          c->kv_colsum, 0) != cudaSuccess)
+      return fail(set_cuda_err(cudaGetLastError(), "K/V weight column sums"));
+  }
   c->wq.resize(Ly);
   c->wo.resize(Ly);
   c->w1.resize(Ly);
@@ -1867,8 +1896,8 @@ int fe_debug_fetch(fe_ctx* c, const char* name, float* dst, size_t max_floats, s
   size_t rows = 0, cols = 0;
   const std::string n(name);
   if (n == "ctx_ln") {
-    if (c->fused_ctxkv) {
-      g_msg = "ctx_ln is not materialised: the fused context kernel keeps LN(context) on chip";
+    if (c->fused_ctxkv || c->ctx_fold) {
+      g_msg = "ctx_ln is not materialised: the context K/V product folds the LayerNorm into its epilogue";
       return FE_ERR_UNSUPPORTED;
     }
     pl = &c->X;

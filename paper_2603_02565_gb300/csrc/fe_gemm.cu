@@ -57,17 +57,17 @@ __host__ __device__ inline uint32_t red_bytes(int cs) { return cs > 1 ? (uint32_
 constexpr int kMaxCluster = 8;
 int g_cluster_cap[2][kMaxCluster + 1] = {};  // resident clusters of size cs with one / two CTAs per SM
 int g_cluster_limit = -1;                 // FE_GEMM_CLUSTERS: 0 disables clusters, n > 0 caps clusters per launch
-bool g_two_per_sm[3][2] = {};             // [EPI][NB - 1]: two CTAs fit on an SM (registers) at half the shared memory
+bool g_two_per_sm[4][2] = {};             // [EPI][NB - 1]: two CTAs fit on an SM (registers) at half the shared memory
 }  // namespace
 
-size_t gemm_smem_bytes(int BN, int nb, int stages, int cs) {
-  const size_t stage = 2 * (size_t)kATile + (size_t)nb * BN * BK * 2;
+size_t gemm_smem_bytes(int BN, int nb, int stages, int cs, int na) {
+  const size_t stage = (size_t)na * kATile + (size_t)nb * BN * BK * 2;
   return (size_t)stages * stage + kSmemFixed + red_bytes(cs);
 }
 
-int gemm_max_stages(int BN, int nb, int K_pad, int cs) {
+int gemm_max_stages(int BN, int nb, int K_pad, int cs, int na) {
   (void)K_pad;  // stages run ahead across tiles, so the ring is not capped by one tile's k blocks
-  const size_t stage = 2 * (size_t)kATile + (size_t)nb * BN * BK * 2;
+  const size_t stage = (size_t)na * kATile + (size_t)nb * BN * BK * 2;
   int s = (int)((kSmemMaxBlock - kSmemFixed - red_bytes(cs)) / stage);
   if (s > kMaxStages) s = kMaxStages;
   return s < 1 ? 1 : s;
@@ -141,7 +141,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nacc = p.nacc;
   const int cs = p.cs > 1 ? p.cs : 1;  // (uniform) CTAs of a cluster sharing each row tile
   const uint32_t b_bytes = (uint32_t)BN * BK * 2;
-  const uint32_t stage_bytes = 2 * kATile + (uint32_t)nb * b_bytes;
+  // activation planes: the split pair, or one exact bf16 plane (raw rows of EPI_LN_FOLD)
+  constexpr int NA = EPI == EPI_LN_FOLD ? 1 : 2;
+  const uint32_t stage_bytes = NA * kATile + (uint32_t)nb * b_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * stage_bytes);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;  // [2] accumulator ready for the epilogue
@@ -214,11 +216,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint8_t* st = smem + (size_t)s * stage_bytes;
           mbar_arrive_expect_tx(full + s, stage_bytes);
           tma_load_2d(st, &tA_h, kb * BK, m0, full + s);
-          tma_load_2d(st + kATile, &tA_l, kb * BK, m0, full + s);
+          if (NA > 1) tma_load_2d(st + kATile, &tA_l, kb * BK, m0, full + s);
           for (int q = 0; q < nb; ++q) {
             const CUtensorMap* tb = q ? &tB_l : &tB_h;
             for (int h = 0; h < BN; h += 256)
-              tma_load_2d(st + 2 * kATile + q * b_bytes + (uint32_t)h * BK * 2, tb, kb * BK, n0 + h, full + s);
+              tma_load_2d(st + NA * kATile + q * b_bytes + (uint32_t)h * BK * 2, tb, kb * BK, n0 + h, full + s);
           }
         }
       }
@@ -245,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t st = smem_u32(smem + (size_t)s * stage_bytes);
           // descriptors built once per stage; the k steps only add 32-byte offsets
           const uint64_t ah0 = umma_desc_sw128(st), al0 = umma_desc_sw128(st + kATile);
-          const uint64_t bh0 = umma_desc_sw128(st + 2 * kATile), bl0 = umma_desc_sw128(st + 2 * kATile + b_bytes);
+          const uint64_t bh0 = umma_desc_sw128(st + NA * kATile), bl0 = umma_desc_sw128(st + NA * kATile + b_bytes);
           for (int h = 0; h < BN; h += 256) {
             const uint32_t hb = (uint32_t)h * BK * 2;
 #pragma unroll
@@ -254,7 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const uint64_t ah = desc_adv(ah0, kk * 32), al = desc_adv(al0, kk * 32);
               const uint64_t bh = desc_adv(bh0, hb + kk * 32);
               umma_bf16(dst + (uint32_t)h, ah, bh, idesc, (kb | kk) != 0 ? 1u : 0u);
-              umma_bf16(dst + (uint32_t)h, al, bh, idesc, 1u);
+              if (NA > 1) umma_bf16(dst + (uint32_t)h, al, bh, idesc, 1u);
               if (nb > 1) umma_bf16(dst + (uint32_t)h, ah, desc_adv(bl0, hb + kk * 32), idesc, 1u);
             }
           }
@@ -548,6 +550,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             split2((v[i] - mean) * rstd, (v[i + 1] - mean) * rstd, hi[i / 2], lo[i / 2]);
           stage_split(hi, lo, c, srow);
         }
+      } else if (EPI == EPI_LN_FOLD) {
+        // LN(x) W = rstd (x W) - mu rstd colsum(W) from the raw rows' product,
+        // rounded to one f16 plane (an attention operand)
+        float2 ms = make_float2(0.f, 0.f);
+        if (valid) ms = __ldg(p.row_stats + grow);
+        const float nmr = -ms.x * ms.y;
+        for (int c = 32 * half; c < BN; c += 64) {
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
+          const int col = n0 + c;
+          const float4* cw = reinterpret_cast<const float4*>(p.colsum + col);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float4 cc = __ldg(cw + j);
+            v[4 * j] = fmaf(v[4 * j], ms.y, nmr * cc.x);
+            v[4 * j + 1] = fmaf(v[4 * j + 1], ms.y, nmr * cc.y);
+            v[4 * j + 2] = fmaf(v[4 * j + 2], ms.y, nmr * cc.z);
+            v[4 * j + 3] = fmaf(v[4 * j + 3], ms.y, nmr * cc.w);
+          }
+          uint8_t* b = next_stage();
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const uint32_t o = (uint32_t)lane * 64u + ((uint32_t)(j ^ ((lane >> 1) & 3)) << 4);
+            *reinterpret_cast<uint4*>(b + o) =
+                make_uint4(pack_f16x2(v[8 * j], v[8 * j + 1]), pack_f16x2(v[8 * j + 2], v[8 * j + 3]),
+                           pack_f16x2(v[8 * j + 4], v[8 * j + 5]), pack_f16x2(v[8 * j + 6], v[8 * j + 7]));
+          }
+          issue(&tO_h, b, nullptr, nullptr, col, srow);
+        }
       } else {  // EPI_HEAD
         // per task t: the dot product of ReLU(acc + b1) with w2 over its
         // head_d columns (a 32-column block lies in one task, head_d % 32 == 0)
@@ -627,7 +658,8 @@ static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, cons
   p.cs = cs;
   const int sms = g_num_sms > 0 ? g_num_sms : 148;
   const long long tiles = (long long)((p.rows + BM - 1) / BM) * (p.N / p.BN);
-  const size_t stage = 2 * (size_t)kATile + (size_t)p.nb * p.BN * BK * 2;
+  constexpr int NA = EPI == EPI_LN_FOLD ? 1 : 2;
+  const size_t stage = (size_t)NA * kATile + (size_t)p.nb * p.BN * BK * 2;
   // At most two waves of tiles: two CTAs per SM, one accumulator each, so the
   // co-resident CTAs overlap each other's loads, MMAs and epilogues.
   // Otherwise: one persistent CTA per SM with a double-buffered accumulator.
@@ -639,9 +671,9 @@ static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, cons
     p.stages = st2 < kMaxStages ? st2 : kMaxStages;
   } else {
     p.nacc = 2 * p.BN <= 512 ? 2 : 1;
-    p.stages = gemm_max_stages(p.BN, p.nb, p.K_pad, cs);
+    p.stages = gemm_max_stages(p.BN, p.nb, p.K_pad, cs, NA);
   }
-  size_t smem = gemm_smem_bytes(p.BN, p.nb, p.stages, cs);
+  size_t smem = gemm_smem_bytes(p.BN, p.nb, p.stages, cs, NA);
   // (CTAs resident per SM) x (TMEM columns per CTA) <= 512: no CTA ever waits in
   // tcgen05.alloc for a co-resident one
   const size_t max_ctas = 512 / pow2_cols(p.nacc * p.BN);
@@ -679,6 +711,8 @@ cudaError_t gemm_prepare() {
   attr((const void*)gemm_kernel<EPI_RESID_LN, 2>);
   attr((const void*)gemm_kernel<EPI_HEAD, 1>);
   attr((const void*)gemm_kernel<EPI_HEAD, 2>);
+  attr((const void*)gemm_kernel<EPI_LN_FOLD, 1>);
+  attr((const void*)gemm_kernel<EPI_LN_FOLD, 2>);
   auto two_fit = [&](const void* f) {
     int n = 0;
     if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, f, kThreads, kSmemPerSM / 2 - 1024);
@@ -690,6 +724,8 @@ cudaError_t gemm_prepare() {
   g_two_per_sm[EPI_RESID_LN][1] = two_fit((const void*)gemm_kernel<EPI_RESID_LN, 2>);
   g_two_per_sm[EPI_HEAD][0] = two_fit((const void*)gemm_kernel<EPI_HEAD, 1>);
   g_two_per_sm[EPI_HEAD][1] = two_fit((const void*)gemm_kernel<EPI_HEAD, 2>);
+  g_two_per_sm[EPI_LN_FOLD][0] = two_fit((const void*)gemm_kernel<EPI_LN_FOLD, 1>);
+  g_two_per_sm[EPI_LN_FOLD][1] = two_fit((const void*)gemm_kernel<EPI_LN_FOLD, 2>);
   if (g_cluster_limit < 0) {
     const char* v = std::getenv("FE_GEMM_CLUSTERS");
     g_cluster_limit = v && *v ? std::atoi(v) : 0x7fffffff;
@@ -740,6 +776,9 @@ cudaError_t gemm_launch(int epi, const CUtensorMap* a_h, const CUtensorMap* a_l,
     case EPI_RESID_LN:
       return two ? launch_t<EPI_RESID_LN, 2>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s)
                  : launch_t<EPI_RESID_LN, 1>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
+    case EPI_LN_FOLD:
+      return two ? launch_t<EPI_LN_FOLD, 2>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s)
+                 : launch_t<EPI_LN_FOLD, 1>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);
     default:
       return two ? launch_t<EPI_HEAD, 2>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s)
                  : launch_t<EPI_HEAD, 1>(a_h, a_l, b_h, b_l, o_h, o_l, o_x, p, s);

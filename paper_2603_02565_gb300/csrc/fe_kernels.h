@@ -81,8 +81,11 @@ struct SelArgs {
 enum GemmEpilogue : int {
   EPI_STORE = 0,    // out = [ReLU](acc + bias) as split planes
   EPI_RESID_LN = 1, // x = resid + acc + bias -> x_out (fp32) and LN(x) as split planes; BN == N
+                   // (or N = cs BN over a cluster)
   EPI_HEAD = 2,     // task heads s_t = ReLU(acc_t + bias_t) . w2_t + b2_t over column blocks of
                    // head_d, fused s = sum_t fuse_w[t] s_t + fuse_b (one task: s = s_0); BN == N
+  EPI_LN_FOLD = 3,  // LN(x) W from the raw rows x: out = rstd (acc - mu colsum(W)) as one f16 plane;
+                   // A is ONE exact bf16 plane (a_l unused), (mu, rstd) per row in row_stats
 };
 
 struct GemmParams {
@@ -108,6 +111,9 @@ struct GemmParams {
   const float* resid;   // residual rows (ldr == 0: one row broadcast to every row)
   int ldr;
   float eps;
+  // EPI_LN_FOLD
+  const float2* row_stats;  // [rows] (mean, rstd) of the raw rows
+  const float* colsum;      // [N] column sums of W
   // EPI_HEAD
   int n_tasks;          // 1..4 heads of head_d columns each (columns past n_tasks * head_d are padding)
   int head_d;
@@ -124,8 +130,8 @@ struct GemmParams {
 
 // Raises the dynamic shared-memory limit of the GEMM kernels (call once per device, outside capture).
 cudaError_t gemm_prepare();
-size_t gemm_smem_bytes(int BN, int nb, int stages, int cs = 1);
-int gemm_max_stages(int BN, int nb, int K_pad, int cs = 1);
+size_t gemm_smem_bytes(int BN, int nb, int stages, int cs = 1, int na = 2);
+int gemm_max_stages(int BN, int nb, int K_pad, int cs = 1, int na = 2);
 // Clusters of cs CTAs (2, 4 or 8) that can be resident at once for the EPI_RESID_LN kernels (0 when
 // such clusters cannot be scheduled, or when FE_GEMM_CLUSTERS=0); valid after gemm_prepare.
 int gemm_cluster_capacity(int cs);
@@ -331,6 +337,10 @@ cudaError_t compact_launch(const int32_t* cand, int B, int M, int K, int L, int 
                            int* bad, int* slot_local, int* list, int* status, unsigned* ticket,
                            cudaStream_t s);
 // Per-row LN of the context -> split planes [rows, ldo]
+// (mean, rstd) of each bf16 row of d columns (LayerNorm without affine parameters, biased variance)
+cudaError_t row_stats_launch(const bf16* x, int rows, int d, float eps, float2* out, cudaStream_t s);
+// out[n] = sum_k (W_h[n, k] + W_l[n, k]) over k < K of the transposed weight planes (W_l may be null)
+cudaError_t colsum_launch(const bf16* w_h, const bf16* w_l, int ld, int N, int K, float* out, cudaStream_t s);
 cudaError_t ctx_ln_launch(const void* x, int io_f32, int rows, int d, float eps, bf16* out_h, bf16* out_l,
                           int ldo, cudaStream_t s);
 // Gather distinct pool rows of every request -> residual stream h (fp32) and LN(h) planes

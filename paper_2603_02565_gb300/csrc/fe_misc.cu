@@ -382,6 +382,65 @@ static cudaError_t ctx_ln_t(const T* x, int rows, int d, float eps, bf16* oh, bf
   return cudaGetLastError();
 }
 
+// (mean, rstd) of a row, one warp per row, two passes over the row in registers
+template <int DPL>
+__global__ void __launch_bounds__(256) row_stats_kernel(const bf16* __restrict__ x, int rows, float eps,
+                                                        float2* __restrict__ out) {
+  constexpr int d = DPL * 32;
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  pdl_wait();
+  pdl_trigger();
+  if (r >= rows) return;
+  float v[DPL];
+  load_vec<DPL>(x + (size_t)r * d + lane * DPL, v);
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) s += v[i];
+  const float mean = warp_sum(s) / (float)d;
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < DPL; ++i) {
+    const float t = v[i] - mean;
+    q = fmaf(t, t, q);
+  }
+  const float rstd = 1.0f / sqrtf(warp_sum(q) / (float)d + eps);
+  if (lane == 0) out[r] = make_float2(mean, rstd);
+}
+
+cudaError_t row_stats_launch(const bf16* x, int rows, int d, float eps, float2* out, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  const unsigned g = (unsigned)((rows + 7) / 8);
+  switch (d) {
+    case 32: return launch_k(row_stats_kernel<1>, dim3(g), dim3(256), 0, s, x, rows, eps, out);
+    case 64: return launch_k(row_stats_kernel<2>, dim3(g), dim3(256), 0, s, x, rows, eps, out);
+    case 128: return launch_k(row_stats_kernel<4>, dim3(g), dim3(256), 0, s, x, rows, eps, out);
+    case 256: return launch_k(row_stats_kernel<8>, dim3(g), dim3(256), 0, s, x, rows, eps, out);
+    case 512: return launch_k(row_stats_kernel<16>, dim3(g), dim3(256), 0, s, x, rows, eps, out);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+// column sums of a weight (init time): one warp per output column n
+__global__ void colsum_kernel(const bf16* w_h, const bf16* w_l, int ld, int N, int K, float* out) {
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (n >= N) return;
+  float a = 0.f;
+  for (int k = lane; k < K; k += 32) {
+    a += __bfloat162float(w_h[(size_t)n * ld + k]);
+    if (w_l) a += __bfloat162float(w_l[(size_t)n * ld + k]);
+  }
+  a = warp_sum(a);
+  if (lane == 0) out[n] = a;
+}
+
+cudaError_t colsum_launch(const bf16* w_h, const bf16* w_l, int ld, int N, int K, float* out, cudaStream_t s) {
+  if (N <= 0) return cudaSuccess;
+  colsum_kernel<<<(N + 7) / 8, 256, 0, s>>>(w_h, w_l, ld, N, K, out);
+  return cudaGetLastError();
+}
+
 cudaError_t ctx_ln_launch(const void* x, int io_f32, int rows, int d, float eps, bf16* out_h, bf16* out_l,
                           int ldo, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;

@@ -101,6 +101,23 @@ def context_kv_rows(w, nreq):
 KV_RTOL, KV_ATOL = 1e-3, 1e-5
 
 
+@pytest.mark.parametrize("kind,B", [("stress", 2), ("summarisation", 2)])
+def test_context_kv_ln_folded(dev, kind, B):
+    """d = 256 and d = 512 with bf16 inputs: the K/V product multiplies the raw
+    context rows and applies the row statistics in its epilogue,
+    rstd (x W) - mu rstd colsum(W); LN(context) is not materialised."""
+    from paper_2603_02565_gb300.binding import Evaluator, FeError
+    w = wl.summarisation(B=B) if kind == "summarisation" else wl.make_workload(kind, B=B)
+    ev = Evaluator(w.cfg, w.weights)
+    ev, gs, gb = run_gpu(w, dev, ev)
+    np.testing.assert_allclose(ev.fetch("ctx_kv", cols=2 * w.cfg.n_layers * w.cfg.d), context_kv_rows(w, B),
+                               rtol=KV_RTOL, atol=KV_ATOL)
+    with pytest.raises(FeError):
+        ev.fetch("ctx_ln")
+    if kind == "stress":  # (the summarisation scores: test_summarisation_small)
+        check(w, gs, gb)
+
+
 def test_stagewise_serving(dev):
     """Intermediates: context K/V, element cache, SeqEnc and cross-sequence outputs
     (serving runs the fused context kernel, so LN(context) is not materialised)."""
