@@ -339,33 +339,58 @@ __global__ void __launch_bounds__(256) gather_ln_kernel(const T* __restrict__ po
                                                         const int* __restrict__ off, const int* __restrict__ list,
                                                         int max_rows, float eps, float* h, int ldh, bf16* ln_h,
                                                         bf16* ln_l, int ldln) {
-  constexpr int d = DPL * 32;
+  constexpr int d = DPL * 32, RPW = 4;  // four consecutive rows per warp, their loads issued together
   const int lane = threadIdx.x & 31;
-  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int r0 = (blockIdx.x * 8 + (threadIdx.x >> 5)) * RPW;
   pdl_wait();
   pdl_trigger();
-  if (r >= max_rows || r >= off[B]) return;
-  // the largest b with off[b] <= r, by the warp: each round the 32 lanes probe
-  // 32 evenly spaced candidates of the range [lo, hi) (off[lo] <= r holds) and
+  const int nrow = min(max_rows, off[B]);
+  if (r0 >= nrow) return;
+  // the largest b with off[b] <= r0, by the warp: each round the 32 lanes probe
+  // 32 evenly spaced candidates of the range [lo, hi) (off[lo] <= r0 holds) and
   // keep the span after the last one that passes, so that B = 1024 takes two
   // rounds of loads instead of ten dependent ones
   int lo = 0, hi = B;
   while (hi - lo > 1) {
     const int step = (hi - lo + 31) / 32;
     const int idx = lo + lane * step;
-    const unsigned pass = __ballot_sync(0xffffffffu, idx < hi && off[idx] <= r);
+    const unsigned pass = __ballot_sync(0xffffffffu, idx < hi && off[idx] <= r0);
     lo += (31 - __clz(pass)) * step;
     hi = min(lo + step, hi);
   }
-  const int b = lo;
-  const int m = list[(size_t)b * cap + (r - off[b])];
-  float v[DPL];
-  load_vec<DPL>(pool + ((size_t)b * M + m) * d + lane * DPL, v);
-  float* hr = h + (size_t)r * ldh + lane * DPL;
+  // the following rows: the same request, or a later one
+  int bs[RPW], ms[RPW];
+  int b = lo, b_end = off[b + 1];
 #pragma unroll
-  for (int i = 0; i < DPL; ++i) hr[i] = v[i];
-  warp_layer_norm<DPL>(v, d, eps);
-  store_split<DPL>(v, ln_h + (size_t)r * ldln + lane * DPL, ln_l + (size_t)r * ldln + lane * DPL);
+  for (int u = 0; u < RPW; ++u) {
+    const int r = r0 + u;
+    bs[u] = -1;
+    if (r < nrow) {
+      while (b_end <= r) b_end = off[++b + 1];
+      bs[u] = b;
+      ms[u] = list[(size_t)b * cap + (r - off[b])];
+    }
+  }
+  float v[RPW][DPL];
+#pragma unroll
+  for (int u = 0; u < RPW; ++u)
+    if (bs[u] >= 0) load_vec<DPL>(pool + ((size_t)bs[u] * M + ms[u]) * d + lane * DPL, v[u]);
+#pragma unroll
+  for (int u = 0; u < RPW; ++u) {
+    if (bs[u] < 0) break;
+    const int r = r0 + u;
+    float* hr = h + (size_t)r * ldh + lane * DPL;
+    if constexpr (DPL % 4 == 0) {
+#pragma unroll
+      for (int i = 0; i < DPL; i += 4)
+        *reinterpret_cast<float4*>(hr + i) = make_float4(v[u][i], v[u][i + 1], v[u][i + 2], v[u][i + 3]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) hr[i] = v[u][i];
+    }
+    warp_layer_norm<DPL>(v[u], d, eps);
+    store_split<DPL>(v[u], ln_h + (size_t)r * ldln + lane * DPL, ln_l + (size_t)r * ldln + lane * DPL);
+  }
 }
 
 template <typename T>
@@ -382,35 +407,47 @@ static cudaError_t ctx_ln_t(const T* x, int rows, int d, float eps, bf16* oh, bf
   return cudaGetLastError();
 }
 
-// (mean, rstd) of a row, one warp per row, two passes over the row in registers
+// (mean, rstd) of a row: four rows per warp, their loads issued together, then
+// two passes over each row in registers
 template <int DPL>
 __global__ void __launch_bounds__(256) row_stats_kernel(const bf16* __restrict__ x, int rows, float eps,
                                                         float2* __restrict__ out) {
-  constexpr int d = DPL * 32;
+  constexpr int d = DPL * 32, RPW = 4;
   const int lane = threadIdx.x & 31;
-  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int r0 = (blockIdx.x * 8 + (threadIdx.x >> 5)) * RPW;
   pdl_wait();
   pdl_trigger();
-  if (r >= rows) return;
-  float v[DPL];
-  load_vec<DPL>(x + (size_t)r * d + lane * DPL, v);
-  float s = 0.f;
+  if (r0 >= rows) return;
+  float v[RPW][DPL];
 #pragma unroll
-  for (int i = 0; i < DPL; ++i) s += v[i];
-  const float mean = warp_sum(s) / (float)d;
-  float q = 0.f;
+  for (int u = 0; u < RPW; ++u) {
+    if (r0 + u < rows) {
+      load_vec<DPL>(x + (size_t)(r0 + u) * d + lane * DPL, v[u]);
+    } else {
 #pragma unroll
-  for (int i = 0; i < DPL; ++i) {
-    const float t = v[i] - mean;
-    q = fmaf(t, t, q);
+      for (int i = 0; i < DPL; ++i) v[u][i] = 0.f;
+    }
   }
-  const float rstd = 1.0f / sqrtf(warp_sum(q) / (float)d + eps);
-  if (lane == 0) out[r] = make_float2(mean, rstd);
+#pragma unroll
+  for (int u = 0; u < RPW; ++u) {
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < DPL; ++i) s += v[u][i];
+    const float mean = warp_sum(s) / (float)d;
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < DPL; ++i) {
+      const float t = v[u][i] - mean;
+      q = fmaf(t, t, q);
+    }
+    const float rstd = 1.0f / sqrtf(warp_sum(q) / (float)d + eps);
+    if (lane == 0 && r0 + u < rows) out[r0 + u] = make_float2(mean, rstd);
+  }
 }
 
 cudaError_t row_stats_launch(const bf16* x, int rows, int d, float eps, float2* out, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  const unsigned g = (unsigned)((rows + 7) / 8);
+  const unsigned g = (unsigned)((rows + 31) / 32);
   switch (d) {
     case 32: return launch_k(row_stats_kernel<1>, dim3(g), dim3(256), 0, s, x, rows, eps, out);
     case 64: return launch_k(row_stats_kernel<2>, dim3(g), dim3(256), 0, s, x, rows, eps, out);
@@ -452,7 +489,7 @@ template <typename T>
 static cudaError_t gather_t(const T* pool, int B, int M, int d, int cap, const int* off, const int* list,
                             int max_rows, float eps, float* h, int ldh, bf16* lh, bf16* ll, int ldln,
                             cudaStream_t s) {
-  const unsigned g = (unsigned)((max_rows + 7) / 8);
+  const unsigned g = (unsigned)((max_rows + 31) / 32);
 #define FE_GATHER(DPL)                                                                                      \
   return launch_k(gather_ln_kernel<DPL, T>, dim3(g), dim3(256), 0, s, pool, B, M, cap, off, list, max_rows, eps, h, \
                   ldh, lh, ll, ldln)
