@@ -268,6 +268,9 @@ struct Weight {
   // RESID_LN with clusters, N = cs x 128 or cs x 64: boxes of 64 x 128 / 64 x 64 on both planes
   CUtensorMap c128h{}, c128l{}, c64h{}, c64l{};
   bool cmaps = false;
+  // products with many row tiles, N % 256 == 0: 256-column tiles (boxes of 64 x 256 on both planes)
+  CUtensorMap c256h{}, c256l{};
+  bool wide = false;
 };
 
 int largest_bn(int N, int cap) {
@@ -554,6 +557,11 @@ int make_weight(fe_ctx* c, Weight& w, int N, int Kin, int bn_cap) {
     if (rc == FE_OK) rc = encode_map(&w.c64l, lo, w.p.ld, w.p.rows, 64);
     w.cmaps = rc == FE_OK;
   }
+  if (rc == FE_OK && N % 256 == 0) {
+    rc = encode_map(&w.c256h, w.p.h, w.p.ld, w.p.rows, 256);
+    if (rc == FE_OK) rc = encode_map(&w.c256l, c->nb > 1 ? w.p.l : w.p.h, w.p.ld, w.p.rows, 256);
+    w.wide = rc == FE_OK;
+  }
   return rc;
 }
 
@@ -602,6 +610,14 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   p.status = c->status;
   p.eps = c->cfg.ln_eps;
   const CUtensorMap *bh = &W.p.th, *bl = &W.p.tl;
+  // 256-column tiles when they still fill every SM: each stage then feeds MMAs of
+  // N = 256, twice the work per wait of the issuing thread
+  if ((epi == fe::EPI_STORE || epi == fe::EPI_LN_FOLD) && W.wide && p.BN < 256 &&
+      (long long)((rows + 127) / 128) * (W.N / 256) >= c->n_sms) {
+    p.BN = 256;
+    bh = &W.c256h;
+    bl = &W.c256l;
+  }
   // LayerNorm rows wider than 128 columns with fewer row tiles than SMs: a
   // cluster of cs CTAs shares each row tile, 128 (or, with very few tiles, 64)
   // columns per CTA, and exchanges the row statistics through distributed
