@@ -621,11 +621,12 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
     bh = &W.c256h;
     bl = &W.c256l;
   }
-  // LayerNorm rows wider than 128 columns with fewer row tiles than SMs: a
-  // cluster of cs CTAs shares each row tile, 128 (or, with very few tiles, 64)
-  // columns per CTA, and exchanges the row statistics through distributed
-  // shared memory, so that more SMs multiply and the epilogue is split cs ways
-  if (epi == fe::EPI_RESID_LN && W.cmaps) {
+  // LayerNorm (or score-head) rows wider than 128 columns with fewer row tiles
+  // than SMs: a cluster of cs CTAs shares each row tile, 128 (or, with very few
+  // tiles, 64) columns per CTA, and exchanges the row statistics (the head's
+  // partial dot products) through distributed shared memory, so that more SMs
+  // multiply and the epilogue is split cs ways
+  if ((epi == fe::EPI_RESID_LN || (epi == fe::EPI_HEAD && p.n_tasks <= 2)) && W.cmaps) {
     const int mtiles = (rows + 127) / 128;
     int cs = W.N / 128, bn = 128;
     if (mtiles * cs * 4 <= c->n_sms && cs * 2 <= 8) {

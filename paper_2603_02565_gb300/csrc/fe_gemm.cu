@@ -582,36 +582,46 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else {  // EPI_HEAD
         // per task t: the dot product of ReLU(acc + b1) with w2 over its
         // head_d columns (a 32-column block lies in one task, head_d % 32 == 0)
+        // (with a cluster, this CTA's BN columns from n0 on; at most two tasks)
         const int nt = p.n_tasks, ncol = nt * p.head_d;
         float acc4[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int c = 32 * half; c < ncol; c += 64) {
+        for (int c = 32 * half; c < BN && n0 + c < ncol; c += 64) {
+          const int gc = n0 + c;
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
           float a = 0.f;
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const float x = relu_nan(v[i] + p.bias[c + i]);
-            a = fmaf(x, p.w2[c + i], a);
+            const float x = relu_nan(v[i] + p.bias[gc + i]);
+            a = fmaf(x, p.w2[gc + i], a);
           }
-          const int t = c / p.head_d;
+          const int t = gc / p.head_d;
 #pragma unroll
           for (int tt = 0; tt < 4; ++tt)
             if (tt == t) acc4[tt] += a;
         }
-        // both halves' partial sums, two tasks per exchange
-        float tot[4];
+        float tot[4] = {0.f, 0.f, 0.f, 0.f};
+        if (cs > 1) {
+          // every warp's partial dot of task 0 (and 1) into every CTA of the cluster
+          if (!row_xchg(0, acc4[0], tot[0])) break;
+          if (nt > 1 && !row_xchg(1, acc4[1], tot[1])) break;
+        } else {
+          // both halves' partial sums, two tasks per exchange
 #pragma unroll
-        for (int t0 = 0; t0 < 4; t0 += 2) {
-          if (t0 < nt) {
-            if (t0 > 0) pair_sync();  // the previous round's reads are done
-            red_sum[half * 128 + r] = acc4[t0];
-            red_var[half * 128 + r] = acc4[t0 + 1];
-            pair_sync();
-            tot[t0] = red_sum[r] + red_sum[128 + r];
-            tot[t0 + 1] = red_var[r] + red_var[128 + r];
+          for (int t0 = 0; t0 < 4; t0 += 2) {
+            if (t0 < nt) {
+              if (t0 > 0) pair_sync();  // the previous round's reads are done
+              red_sum[half * 128 + r] = acc4[t0];
+              red_var[half * 128 + r] = acc4[t0 + 1];
+              pair_sync();
+              tot[t0] = red_sum[r] + red_sum[128 + r];
+              tot[t0 + 1] = red_var[r] + red_var[128 + r];
+            }
           }
         }
-        if (half == 0) {  // (uniform per warp: the warps of the first column half write the scores)
+        // (uniform per warp: the warps of the first column half of the cluster's
+        // first CTA write the scores)
+        if (half == 0 && my_rank == 0) {
           float f = 0.f;
           if (valid) {
             if (nt == 1) {
@@ -654,7 +664,7 @@ static cudaError_t launch_t(const CUtensorMap* a_h, const CUtensorMap* a_l, cons
                             const CUtensorMap* b_l, const CUtensorMap* o_h, const CUtensorMap* o_l,
                             const CUtensorMap* o_x, const GemmParams& p0, cudaStream_t s) {
   GemmParams p = p0;
-  const int cs = (EPI == EPI_RESID_LN && p.cs > 1) ? p.cs : 1;
+  const int cs = ((EPI == EPI_RESID_LN || EPI == EPI_HEAD) && p.cs > 1) ? p.cs : 1;
   p.cs = cs;
   const int sms = g_num_sms > 0 ? g_num_sms : 148;
   const long long tiles = (long long)((p.rows + BM - 1) / BM) * (p.N / p.BN);
@@ -747,12 +757,16 @@ cudaError_t gemm_prepare() {
         cfg.attrs = a;
         cfg.numAttrs = 1;
         int n = 0;
+        // the LayerNorm and head instantiations: the smaller capacity
         const void* f = nbv == 1 ? (const void*)gemm_kernel<EPI_RESID_LN, 1> : (const void*)gemm_kernel<EPI_RESID_LN, 2>;
-        if (cudaOccupancyMaxActiveClusters(&n, f, &cfg) != cudaSuccess) {
+        const void* fh = nbv == 1 ? (const void*)gemm_kernel<EPI_HEAD, 1> : (const void*)gemm_kernel<EPI_HEAD, 2>;
+        int nh = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, f, &cfg) != cudaSuccess ||
+            cudaOccupancyMaxActiveClusters(&nh, fh, &cfg) != cudaSuccess) {
           (void)cudaGetLastError();
-          n = 0;
+          n = nh = 0;
         }
-        (nbv == 1 ? n1 : n2) = n;
+        (nbv == 1 ? n1 : n2) = n < nh ? n : nh;
       }
       g_cluster_cap[two][cs] = g_cluster_limit == 0 ? 0 : (n1 < n2 ? n1 : n2);
     }
