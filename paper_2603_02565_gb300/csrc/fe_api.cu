@@ -230,7 +230,7 @@ int map_out(Planes& p) {
 // store map and the attention kernel's Q and K/V head-slice maps.
 int map_attn(Planes& p, int dh) {
   const CUtensorMapSwizzle sw = dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
-  const int kv_rows = dh == 32 ? 64 : 128;
+  const int kv_rows = fe::attn_chunk_keys(dh);
   int rc = encode_map_t(&p.sh, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.h, p.ld, p.rows, 32, 32,
                         CU_TENSOR_MAP_SWIZZLE_64B);
   if (rc == FE_OK) rc = encode_map_t(&p.ah, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, p.h, p.ld, p.rows, dh, 128, sw);
@@ -243,7 +243,7 @@ int map_attn(Planes& p, int dh) {
 // every key chunk of one head is one contiguous block.
 int map_attn_hm(Planes& p, int dh) {
   const CUtensorMapSwizzle sw = dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B;
-  const int kv_rows = dh == 32 ? 64 : 128;
+  const int kv_rows = fe::attn_chunk_keys(dh);
   int rc = encode_map_hm(&p.sh, p.h, dh, p.rows, p.ld / dh, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
   if (rc == FE_OK) rc = encode_map_hm(&p.kh, p.h, dh, p.rows, p.ld / dh, dh, kv_rows, sw);
   return rc;
@@ -1091,7 +1091,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     ap.status = c->status;
     // V as [request][K][3d], so that a key chunk reaching past K reads zeros, not the next request's rows
     CUtensorMap vseg;
-    FE_RC(encode_map_seg(&vseg, c->qkv.h, c->qkv.ld, K, B, c->dh, c->dh == 32 ? 64 : 128,
+    FE_RC(encode_map_seg(&vseg, c->qkv.h, c->qkv.ld, K, B, c->dh, fe::attn_chunk_keys(c->dh),
                          c->dh == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B));
     ap.kv_seg = 1;
     {

@@ -525,6 +525,8 @@ cudaError_t attn_prepare() {
   return e;
 }
 
+int attn_chunk_keys(int dh) { return dh == 32 ? AttnCfg<32>::CK : AttnCfg<64>::CK; }
+
 cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, const CUtensorMap* v, const AttnParams& p0,
                         cudaStream_t s) {
   if (p0.n_segments <= 0 || p0.max_q <= 0 || (!p0.kv_self && p0.kv_cnt <= 0)) return cudaSuccess;

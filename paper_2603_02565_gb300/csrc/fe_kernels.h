@@ -294,6 +294,9 @@ struct AttnParams {
   int* status;
 };
 cudaError_t attn_prepare();
+// Keys per chunk of the attention kernel for head size dh: the row count of the
+// key/value tensor-map boxes (tK, tV) that attn_launch expects.
+int attn_chunk_keys(int dh);
 cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, const CUtensorMap* v, const AttnParams& p,
                         cudaStream_t s);
 
