@@ -149,7 +149,7 @@ def test_stagewise_serving(dev):
     np.testing.assert_allclose(ev.fetch("cross"), np.vstack(cross), rtol=1e-3, atol=1e-4)
 
 
-@pytest.mark.parametrize("K", [10, 100, 1000])
+@pytest.mark.parametrize("K", [1, 10, 50, 100, 129, 400, 1000])
 def test_ksweep_small(dev, K):
     w = wl.make_workload("ksweep", K=K, B=3)
     ev, gs, gb = run_gpu(w, dev)
@@ -290,6 +290,18 @@ def test_stress_full_batch_sampled(dev):
     w = wl.make_workload("stress")
     ev, gs, gb = run_gpu(w, dev)
     rq = [0, 1, 511, 777, 1022, 1023]
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb, requests=rq)
+    check_layout(ev, w, o_U, o_sl, requests=rq)
+
+
+def test_summarisation_full_batch_sampled(dev):
+    """The summarisation batch at the benchmark's size (B=32, C=1024, d=512, K=16,
+    L=64): clustered LayerNorm GEMMs and score head, the folded context K/V and the
+    several-warps [CLS] attention at their launch sizes; the first and last
+    requests checked."""
+    w = wl.summarisation()
+    ev, gs, gb = run_gpu(w, dev)
+    rq = [0, w.shape[0] - 1]
     o_s, o_b, o_U, o_sl, err = check(w, gs, gb, requests=rq)
     check_layout(ev, w, o_U, o_sl, requests=rq)
 
