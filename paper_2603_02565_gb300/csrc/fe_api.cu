@@ -769,7 +769,9 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
   // the first element layer), so that they run beside the compaction and the
   // element gather, which do not read them
   cudaStream_t sc = s;
-  if (c->fork_ctx) {
+  // (small batches keep one stream: the fork's event edges cost more than it overlaps)
+  const bool fork = c->fork_ctx && (long long)B * C >= 8192;
+  if (fork) {
     FE_CK(cudaEventRecord(c->fork_ev, s));
     FE_CK(cudaStreamWaitEvent(c->ctx_stream, c->fork_ev, 0));
     sc = c->ctx_stream;
@@ -830,7 +832,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     FE_CK(fe::lin_state_launch(c->KV.h, c->fused_ctxkv ? 1 : 0, c->KV.rows, c->KV.ld, fact ? B * K : B, C, d, c->dh,
                                Ly, c->H, c->lin_states, sc));
   }
-  if (c->fork_ctx) FE_CK(cudaEventRecord(c->kv_ev, sc));
+  if (fork) FE_CK(cudaEventRecord(c->kv_ev, sc));
   // (a2) distinct elements: gather + LN (+ the first layer's Q), then the cross-attention stack
   if (c->fused_embed) {
     fe::EmbedParams ep{};
@@ -886,7 +888,7 @@ int enqueue_batch(fe_ctx* c, const Shape& sh, const IoPtrs& io, cudaStream_t s) 
     po.ldr = d;
     FE_RC(gemm(c, "gemm_elem_o_ln", fe::EPI_RESID_LN, c->a, c->oe, R, sumU, po, &c->xln, &c->h, s));
   }
-  if (c->fork_ctx) FE_CK(cudaStreamWaitEvent(s, c->kv_ev, 0));  // the context K/V (or states) are complete
+  if (fork) FE_CK(cudaStreamWaitEvent(s, c->kv_ev, 0));  // the context K/V (or states) are complete
   for (int l = 0; l < Ly; ++l) {
     // (otherwise the embedding kernel or the previous layer's fused FFN wrote Q)
     if ((l == 0 && !c->fused_embed) || (l > 0 && !c->tail_q && !c->ffn_w)) {
