@@ -176,11 +176,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---------------- TMA producer ----------------
       int ws = 0, tl = 0;
       bool ok = true;
+      // every CTA re-reads the same weight boxes while the activation tiles
+      // stream past once: keep the weights in L2, let the activations go first
+      const uint64_t keep = l2_policy_evict_last(), pass = l2_policy_evict_first();
       auto load = [&](const CUtensorMap* m, int x, int y) -> bool {
         const int slot = ws % kRing;
         if (ws >= kRing && !mbar_wait_compact(w_empty + slot, ((ws / kRing) - 1) & 1, p.status)) return false;
         mbar_arrive_expect_tx(w_full + slot, kBox);
-        tma_load_2d(sR + (size_t)slot * kBox, m, x, y, w_full + slot);
+        tma_load_2d_hint(sR + (size_t)slot * kBox, m, x, y, w_full + slot, keep);
         ++ws;
         return true;
       };
@@ -195,8 +198,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             mbar_arrive_expect_tx(a_full, kABytes);
             for (int kb = 0; kb < NKB; ++kb) {
-              tma_load_2d(sA + (size_t)(kb * 2) * kBox, &tA_h, kb * BK, t * BM, a_full);
-              tma_load_2d(sA + (size_t)(kb * 2 + 1) * kBox, &tA_l, kb * BK, t * BM, a_full);
+              tma_load_2d_hint(sA + (size_t)(kb * 2) * kBox, &tA_h, kb * BK, t * BM, a_full, pass);
+              tma_load_2d_hint(sA + (size_t)(kb * 2 + 1) * kBox, &tA_l, kb * BK, t * BM, a_full, pass);
             }
           }
           if (!load(&tWO, (i >> 1) * BK, (i & 1) * 128)) ok = false;
