@@ -284,14 +284,14 @@ def blas_threads():
     return os.cpu_count() or 1
 
 
-def oracle_requests_per_s(w, budget_s=12.0, max_requests=None):
+def oracle_requests_per_s(w, budget_s=12.0, max_requests=None, mode="reuse"):
     import oracle.fe_oracle as O
     B = w.shape[0]
     t0 = time.perf_counter()
     n = 0
     while True:
         b = n % B
-        O.evaluate(w.context[b:b + 1], w.pool[b:b + 1], w.cand_idx[b:b + 1], w.weights, w.cfg)
+        O.evaluate(w.context[b:b + 1], w.pool[b:b + 1], w.cand_idx[b:b + 1], w.weights, w.cfg, mode=mode)
         n += 1
         el = time.perf_counter() - t0
         if el >= budget_s or (max_requests and n >= max_requests):
@@ -525,6 +525,11 @@ def run_ours(args):
         cpu = {"value": rps, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
                "sample": f"{n} requests of the {w.name} batch, one at a time (float64 numpy, reuse mode), "
                          f"{el:.1f} s"}
+        # the same oracle without reuse (context K/V per sequence, every occurrence
+        # encoded on its own: the candidate-factorized evaluation), a shorter sample
+        rps_nr, n_nr, el_nr = oracle_requests_per_s(w, budget_s=args.cpu_seconds / 3, mode="no_reuse")
+        cpu["no_reuse"] = {"value": rps_nr, "unit": UNIT,
+                           "sample": f"{n_nr} requests, one at a time (float64 numpy, no-reuse mode), {el_nr:.1f} s"}
 
     if rank == 0:
         out = {
