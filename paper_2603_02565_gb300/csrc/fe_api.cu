@@ -613,6 +613,14 @@ int gemm(fe_ctx* c, const char* site, int epi, const Planes& A, const Weight& W,
   p.status = c->status;
   p.eps = c->cfg.ln_eps;
   const CUtensorMap *bh = &W.p.th, *bl = &W.p.tl;
+  // stored products with fewer 128-column tiles than half the SMs (the sequence
+  // side of wide shapes): 64-column tiles, twice the CTAs
+  if (epi == fe::EPI_STORE && W.cmaps && p.BN == 128 &&
+      2LL * ((rows + 127) / 128) * (W.N / 128) < c->n_sms) {
+    p.BN = 64;
+    bh = &W.c64h;
+    bl = &W.c64l;
+  }
   // 256-column tiles when they still fill every SM: each stage then feeds MMAs of
   // N = 256, twice the work per wait of the issuing thread
   if ((epi == fe::EPI_STORE || epi == fe::EPI_LN_FOLD) && W.wide && p.BN < 256 &&
