@@ -294,6 +294,17 @@ def test_stress_full_batch_sampled(dev):
     check_layout(ev, w, o_U, o_sl, requests=rq)
 
 
+def test_stress_mid_batch_sampled(dev):
+    """Stress width at B=24: the cross-sequence LayerNorm GEMM and the score head
+    (4800 sequence rows, 38 row tiles) over clusters of two CTAs of 128 columns;
+    three sampled requests checked."""
+    w = wl.make_workload("stress", B=24)
+    ev, gs, gb = run_gpu(w, dev)
+    rq = [0, 11, 23]
+    o_s, o_b, o_U, o_sl, err = check(w, gs, gb, requests=rq)
+    check_layout(ev, w, o_U, o_sl, requests=rq)
+
+
 def test_summarisation_full_batch_sampled(dev):
     """The summarisation batch at the benchmark's size (B=32, C=1024, d=512, K=16,
     L=64): clustered LayerNorm GEMMs and score head, the folded context K/V and the
