@@ -32,9 +32,10 @@
 // Linear-attention state mode (STATE, two layers, C a multiple of 128): the
 // half of CTA c is layer c % 2, [K_l | V_l].  K/V never leave the chip: the
 // epilogue writes phi(K) (phi(x) = elu(x) + 1) and V of the 128-row tile as
-// MN-major 128-byte-swizzled operand tiles, sums phi(K) over its rows for z
-// (a warp reduce-scatter), and one epilogue thread issues phi(K)^T V
-// (M = N = 128, K = the tile's rows) into TMEM, accumulating over the C / 128
+// MN-major 128-byte-swizzled operand tiles, V followed by 16 columns of ones,
+// and one epilogue thread issues phi(K)^T [V | 1] (M = 128, N = d + 16, K = the
+// tile's rows) into TMEM, so that the ones columns accumulate z = sum of
+// phi(K) over the rows, accumulating over the C / 128
 // row blocks of the segment, which the CTA pair takes in a row; after the
 // last one each head's diagonal d_h x d_h block and z are stored.  The K/V
 // accumulator is single-buffered to leave TMEM for the state.
@@ -69,7 +70,8 @@ __host__ __device__ inline CtxKvLayout ctxkv_layout(int d_pad, int N, bool state
   L.aux_bytes = 4096;  // column sums of the weight half [256] fp32, row statistics [2][128] float2
   L.raw_bytes = (uint32_t)(d_pad / BK) * kPlane;                      // one raw block [kb]
   L.nraw = state ? 1u : 2u;
-  L.tail_bytes = state ? 2u * kStateTile : (uint32_t)kEpiWarps * (uint32_t)kStgBufs * kStage;
+  // (state mode: the V tile has a third 64-feature atom for the ones columns of z)
+  L.tail_bytes = state ? 2u * kStateTile + 16384u : (uint32_t)kEpiWarps * (uint32_t)kStgBufs * kStage;
   L.smem = 1024 + (size_t)L.w_bytes + L.aux_bytes + L.nraw * (size_t)L.raw_bytes + L.tail_bytes + 256;
   return L;
 }
@@ -293,7 +295,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int d = p.d, dh = p.dh, H = p.d / p.dh, l = half;
     const int SB = dh * dh + dh;
     uint8_t* sPK = sStg;                 // phi(K)[row][feature]: MN-major, two 64-feature atoms
-    uint8_t* sPV = sStg + kStateTile;    // V[row][feature]
+    uint8_t* sPV = sStg + kStateTile;    // V[row][feature], then 16 feature columns of ones
     auto epi_sync = [&]() { asm volatile("bar.sync 5, 256;" ::: "memory"); };
     // d = 64: features 64..127 of the phi(K) operand stay zero
     if (d < 128) {
@@ -304,8 +306,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto piece = [&](int m) {
       return (uint32_t)(m >> 6) * 16384u + (uint32_t)r * 128u + ((((uint32_t)(m & 63) >> 3) ^ (uint32_t)(r & 7)) << 4);
     };
-    const uint32_t idesc = umma_idesc_f16(BM, d) | (1u << 15) | (1u << 16);  // A and B MN-major
-    float zsum[2] = {0.f, 0.f};  // this lane's feature of each K chunk it handles: the segment's sum of phi(K)
+    // V features d .. d + 15 are ones (f16 1.0), so the state product's columns
+    // d .. d + 15 accumulate z = sum over rows of phi(K), on the tensor core and
+    // from the same f16 phi(K) as S
+    if (sub == 0) {
+      *reinterpret_cast<uint4*>(sPV + piece(d)) = make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);
+      *reinterpret_cast<uint4*>(sPV + piece(d + 8)) = make_uint4(0x3C003C00u, 0x3C003C00u, 0x3C003C00u, 0x3C003C00u);
+    }
+    const uint32_t idesc = umma_idesc_f16(BM, d + 16) | (1u << 15) | (1u << 16);  // A and B MN-major
     const bool wok = mbar_wait_bounded(w_full, 0, p.status);
     if (wok && ew * 32 + lane < Nh) wsum[ew * 32 + lane] = weight_colsum(sW, Nh, NKB, ew * 32 + lane);
     epi_sync();
@@ -316,7 +324,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait_bounded(stats_full, it & 1, p.status)) break;
       tc_fence_after();
       const float2 st = stats[r];  // rstd, -rstd mu of this thread's row
-      int kc = 0;
       for (int c = 32 * sub; c < 2 * d; c += 64) {
         float v[32];
         tmem_ld32(tmem + lane_off + (uint32_t)c, v);
@@ -327,23 +334,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (isk) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = phi_elu1(v[i]);
-          // z: this warp's 32 rows summed per feature; lane f ends with feature m0 + f
-          float a[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) a[i] = v[i];
-#pragma unroll
-          for (int o = 16; o >= 1; o >>= 1) {
-            const bool up = (lane & o) != 0;
-#pragma unroll
-            for (int i = 0; i < o; ++i) {
-              const float keep = up ? a[i + o] : a[i];
-              const float send = up ? a[i] : a[i + o];
-              a[i] = keep + __shfl_xor_sync(0xFFFFFFFFu, send, o);
-            }
-          }
-          if (kc == 0) zsum[0] += a[0];
-          else zsum[1] += a[0];
-          ++kc;
         }
         // the previous row block's state product must be done reading the operand tiles
         if (c < 64 && it > 0 && !mbar_wait_bounded(st_full, (it - 1) & 1, p.status)) break;
@@ -386,22 +376,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int jj = 0; jj < 32; jj += 4)
           *reinterpret_cast<float4*>(dst + jj) = make_float4(sv[jj], sv[jj + 1], sv[jj + 2], sv[jj + 3]);
       }
-      // z: the four quadrant warps of each K chunk hold partial sums over
-      // their 32 rows; combined through the phi(K) tile, free now that the
-      // segment's last product is complete
-      tc_fence_before();
-      float* zsm = reinterpret_cast<float*>(sPK);  // [quadrant][128 features]
-      int kk2 = 0;
-      for (int c = 32 * sub; c < d; c += 64, ++kk2) zsm[q * 128 + c + lane] = kk2 == 0 ? zsum[0] : zsum[1];
-      epi_sync();
-      if (q == 0) {
-        for (int c = 32 * sub; c < d; c += 64) {
-          const int mz = c + lane;
-          st_seg[(size_t)(mz / dh) * SB + dh * dh + (mz % dh)] =
-              (zsm[mz] + zsm[128 + mz]) + (zsm[256 + mz] + zsm[384 + mz]);
-        }
+      // z of feature m: column d of the state accumulator (any of the ones columns)
+      if (sub == 0 && 32 * q < d) {
+        float zz[16];
+        tmem_ld16(tmem + lane_off + 256u + (uint32_t)d, zz);
+        st_seg[(size_t)(m / dh) * SB + dh * dh + (m % dh)] = zz[0];
       }
-      zsum[0] = zsum[1] = 0.f;
+      tc_fence_before();
       epi_sync();  // the state accumulator is read before the next segment's first product
     }
   } else {
