@@ -15,7 +15,11 @@
 //                   PV_j = P_j V_j with P_j read from that same TMEM tile,
 //                   accumulated into the unit's output accumulator in TMEM
 //                   (two, alternating by unit); three S/P tiles let S_{j+1}
-//                   start while PV_{j-1} still reads its tile
+//                   start while PV_{j-1} still reads its tile.  One commit per
+//                   PV_j, on the K/V stage's empty barrier, tells every role
+//                   that PV_j is complete: the producer may refill the stage,
+//                   the issuer may write S_{j+3} over P_j, the softmax may
+//                   rescale or read the output accumulator
 //   warps 2..9    : online softmax from TMEM, one query row per lane; warps
 //                   w and w+4 share TMEM lane quadrant w % 4 and each take
 //                   half of the chunk's keys and half of the output columns
@@ -89,6 +93,25 @@ __device__ __forceinline__ float max32(const float* v) {
                fmaxf(a[9], a[10]));
 }
 
+// Non-blocking probe of an mbarrier phase, for waits that are normally
+// already satisfied when reached (the issuer's K/V and tile checks).
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_ready(uint64_t* bar, uint32_t parity, int* status) {
+  if (mbar_test(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, status);
+}
+
 __device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
@@ -160,12 +183,10 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   uint64_t* q_full = bars;        // [2]
   uint64_t* q_empty = bars + 2;   // [2]
   uint64_t* kv_full = bars + 4;   // [stages]
-  uint64_t* kv_empty = bars + 12; // [stages]
+  uint64_t* kv_empty = bars + 12; // [stages] PV_j (and everything issued before it) complete
   uint64_t* s_full = bars + 20;     // [3] S_j complete in TMEM tile j % 3
   uint64_t* p_full = bars + 23;     // [3] P_j written over S_j
-  uint64_t* tile_free = bars + 26;  // [3] PV_j has read P_j: tile j % 3 free again
-  uint64_t* pv_full = bars + 29;    // [2] PV_j complete in PV buffer j % 2
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 31);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 26);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // row-statistic exchange
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -182,12 +203,10 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     for (int i = 0; i < 2; ++i) {
       mbar_init(q_full + i, 1);
       mbar_init(q_empty + i, 1);
-      mbar_init(pv_full + i, 1);
     }
     for (int i = 0; i < Cfg::kTiles; ++i) {
       mbar_init(s_full + i, 1);
       mbar_init(p_full + i, 32 * Cfg::kSoftmaxWarps);
-      mbar_init(tile_free + i, 1);
     }
     for (int i = 0; i < Cfg::kKVStages; ++i) {
       mbar_init(kv_full + i, 1);
@@ -250,39 +269,49 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
       // ---------------- MMA issuer ----------------
       // The chunks of all this CTA's units form one stream g = 0, 1, ...;
       // S_{g+1} is issued before PV_g, across unit boundaries too, so the
-      // softmax finds the next unit's first S ready when it gets there.
+      // softmax finds the next unit's first S ready when it gets there.  The
+      // loop is this one thread's serial path and sets the pace of the
+      // kernel: running indices instead of divisions, descriptors as a base
+      // plus an offset, and one commit per product.
+      constexpr int NS = Cfg::kKVStages;
+      static_assert((NS & (NS - 1)) == 0, "K/V stages: a power of two");
       const uint32_t idesc_s = umma_idesc_f16(BQ, CK);
       const uint32_t idesc_pv = umma_idesc_f16(BQ, DH) | (1u << 16);  // B (V) is MN-major
       // only a variable key count or one that is not a multiple of CK leaves a
       // partial chunk, whose V rows a segmented map already reads as zeros
       const bool pad_v = p.kv_self || (p.kv_cnt % CK != 0 && !p.kv_seg);
+      const uint64_t qd0 = desc_sw(smem_u32(sQ), Cfg::kSbo, Cfg::kSwz);
+      const uint64_t kd0 = desc_sw(smem_u32(sKV), Cfg::kSbo, Cfg::kSwz);
       Cursor sc;             // unit of the next S
       int sj = 0, sui = 0;   // its chunk and its unit counter (Q buffer sui % 2)
+      int s_nch = 0;         // that unit's chunk count
       int g_s = 0;           // S products issued
+      int t_s = 0;           // TMEM tile of the next S (g_s % 3)
       // per chunk g (g % 4; at most two chunks separate S and PV): its unit
       // counter's parity (the output accumulator) and whether it opens the unit
       uint32_t pv_info = 0;
       cur_first(p, units, sc);
-      // S = Q K^T of the chunk at the S cursor into TMEM tile g_s % 3, then advance the cursor
+      if (sc.u < units) s_nch = chunks(sc);
+      // S = Q K^T of the chunk at the S cursor into TMEM tile t_s, then advance the cursor
       auto issue_next_s = [&]() -> bool {
         if (sc.u >= units) return true;
         const int qb = sui & 1;
         if (sj == 0 && !mbar_wait_compact(q_full + qb, (sui >> 1) & 1, p.status)) return false;
-        const int t = g_s % Cfg::kTiles;
         // the tile is free once PV_{g_s-3}, which reads P_{g_s-3} from it, has completed
-        if (g_s >= Cfg::kTiles && !mbar_wait_compact(tile_free + t, ((g_s / Cfg::kTiles) - 1) & 1, p.status))
-          return false;
-        const int ks = g_s % Cfg::kKVStages;
-        if (!mbar_wait_compact(kv_full + ks, (g_s / Cfg::kKVStages) & 1, p.status)) return false;
+        if (g_s >= Cfg::kTiles) {
+          const int gp = g_s - Cfg::kTiles;
+          if (!mbar_wait_ready(kv_empty + (gp & (NS - 1)), (uint32_t)(gp / NS) & 1u, p.status)) return false;
+        }
+        const int ks = g_s & (NS - 1);
+        if (!mbar_wait_ready(kv_full + ks, (uint32_t)(g_s / NS) & 1u, p.status)) return false;
         tc_fence_after();
-        const uint32_t q = smem_u32(sQ + qb * Cfg::kQBytes);
-        const uint32_t k = smem_u32(sKV + ks * Cfg::kKVBytes);
-        const uint32_t dst = tmem + (uint32_t)(t * CK);
-        const uint64_t q0d = desc_sw(q, Cfg::kSbo, Cfg::kSwz), k0d = desc_sw(k, Cfg::kSbo, Cfg::kSwz);
+        const uint32_t dst = tmem + (uint32_t)(t_s * CK);
+        const uint64_t qd = qd0 + (uint64_t)((qb * Cfg::kQBytes) >> 4);
+        const uint64_t kd = kd0 + (uint64_t)((ks * Cfg::kKVBytes) >> 4);
 #pragma unroll
         for (int kk = 0; kk < DH / 16; ++kk)
-          umma_bf16(dst, desc_adv(q0d, kk * 32), desc_adv(k0d, kk * 32), idesc_s, kk != 0 ? 1u : 0u);
-        umma_commit(s_full + t);
+          umma_bf16(dst, qd + (uint64_t)(kk * 2), kd + (uint64_t)(kk * 2), idesc_s, kk != 0 ? 1u : 0u);
+        umma_commit(s_full + t_s);
         pv_info = (pv_info & ~(3u << (2 * (g_s & 3)))) | ((uint32_t)(((sui & 1) << 1) | (sj == 0 ? 1 : 0)) << (2 * (g_s & 3)));
         // The V rows of a partial chunk past the key count belong to the next
         // segment: their P is 0, but 0 x NaN is NaN, so they are zeroed here
@@ -292,37 +321,41 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
           if (kval < CK) zero_tail(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile, kval * (int)Cfg::kRowBytes, (int)Cfg::kKVTile);
         }
         ++g_s;
-        if (++sj == chunks(sc)) {  // every S of this unit issued: its Q buffer frees on completion
+        t_s = t_s == Cfg::kTiles - 1 ? 0 : t_s + 1;
+        if (++sj == s_nch) {  // every S of this unit issued: its Q buffer frees on completion
           umma_commit(q_empty + qb);
           sj = 0;
           ++sui;
           cur_next(p, units, sc);
+          if (sc.u < units) s_nch = chunks(sc);
         }
         return true;
       };
       bool ok = issue_next_s();
+      int t = 0;
+      uint32_t p_par = 0;  // parity of P_g's phase on p_full[t]: (g / 3) & 1
       for (int g = 0; ok && g < g_s; ++g) {
         if (!issue_next_s()) break;
-        const int t = g % Cfg::kTiles;
-        if (!mbar_wait_compact(p_full + t, (g / Cfg::kTiles) & 1, p.status)) break;
+        if (!mbar_wait_compact(p_full + t, p_par, p.status)) break;
         tc_fence_after();
         // PV_g: A = P_g from TMEM tile g % 3, each softmax warp's KW keys as
         // KW/2 columns of f16 pairs at the start of its KW S columns
-        const int ks = g % Cfg::kKVStages;
-        const uint32_t v = smem_u32(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile);
+        const int ks = g & (NS - 1);
+        const uint64_t vd = kd0 + (uint64_t)((ks * Cfg::kKVBytes + Cfg::kKVTile) >> 4);
         const uint32_t pt = tmem + (uint32_t)(t * CK);
         // PV accumulates into the unit's output accumulator (unit parity), from zero at its first chunk
         const uint32_t info = (pv_info >> (2 * (g & 3))) & 3u;
         const uint32_t dst = tmem + (uint32_t)(Cfg::kTiles * CK + (int)(info >> 1) * DH);
-        const uint64_t v0d = desc_sw(v, Cfg::kSbo, Cfg::kSwz);
 #pragma unroll
         for (int kk = 0; kk < CK / 16; ++kk)
           umma_bf16_tmem_a(dst, pt + (uint32_t)((kk / (Cfg::KW / 16)) * Cfg::KW + (kk % (Cfg::KW / 16)) * 8),
-                           desc_adv(v0d, (uint32_t)kk * 16 * Cfg::kRowBytes), idesc_pv,
+                           vd + (uint64_t)((kk * 16 * Cfg::kRowBytes) >> 4), idesc_pv,
                            (kk != 0 || !(info & 1u)) ? 1u : 0u);
-        umma_commit(pv_full + (g & 1));
-        umma_commit(tile_free + t);
         umma_commit(kv_empty + ks);
+        if (++t == Cfg::kTiles) {
+          t = 0;
+          p_par ^= 1u;
+        }
       }
     }
   } else {
@@ -366,7 +399,8 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         ltot = rs[r] + rs[128 + r];
       }
       if (!dn.active) return true;
-      if (!mbar_wait_compact(pv_full + (dn.g & 1), (dn.g >> 1) & 1, p.status)) return false;
+      if (!mbar_wait_compact(kv_empty + (dn.g % Cfg::kKVStages), (uint32_t)(dn.g / Cfg::kKVStages) & 1u, p.status))
+        return false;
       tc_fence_after();
       float o[DO];
       o_load(o_cols(dn.ui), o);
@@ -434,7 +468,8 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
             const bool up = mx > m + kSlack;
             if (__any_sync(0xffffffffu, up)) {
               // the accumulator holds PV up to chunk gc - 1: scale it (and l) to the new maximum
-              if (!mbar_wait_compact(pv_full + ((gc - 1) & 1), ((gc - 1) >> 1) & 1, p.status)) {
+              if (!mbar_wait_compact(kv_empty + ((gc - 1) % Cfg::kKVStages), (uint32_t)((gc - 1) / Cfg::kKVStages) & 1u,
+                                     p.status)) {
                 ok = false;
                 break;
               }
