@@ -11,16 +11,17 @@
 //   warp 0 lane 0 : TMA producer -- Q tile (two buffers, one per unit in
 //                   flight) and K/V chunks of CK keys (8 stages for d_h = 32,
 //                   4 for d_h = 64)
-//   warp 1 lane 0 : tcgen05.mma -- S_j = Q K_j^T into TMEM tile j % 3, then
-//                   PV_j = P_j V_j with P_j read from that same TMEM tile,
-//                   accumulated into the unit's output accumulator in TMEM
-//                   (two, alternating by unit); three S/P tiles let S_{j+1}
-//                   start while PV_{j-1} still reads its tile.  One commit per
-//                   PV_j, on the K/V stage's empty barrier, tells every role
-//                   that PV_j is complete: the producer may refill the stage,
-//                   the issuer may write S_{j+3} over P_j, the softmax may
-//                   rescale or read the output accumulator
-//   warps 2..9    : online softmax from TMEM, one query row per lane; warps
+//   tcgen05.mma   : S_j = Q K_j^T into TMEM tile j % 3 (three S/P tiles let
+//                   S_{j+1} and S_{j+2} run ahead of PV_j), and PV_j = P_j V_j
+//                   with P_j read from the same TMEM tile, accumulated into the
+//                   unit's output accumulator in TMEM (two, alternating by
+//                   unit).  One commit per PV_j, on the K/V stage's empty
+//                   barrier, tells every role that PV_j is complete.  Each
+//                   tcgen05.mma costs its issuing thread a fixed latency
+//                   (about 45 ns, whatever N), so a CTA that walks many chunks
+//                   issues S from warp 1 and PV from warp 2 (SPLIT); a short
+//                   launch keeps one issuer (warp 1) and one warp fewer
+//   the other 8   : online softmax from TMEM, one query row per lane; warps
 //                   w and w+4 share TMEM lane quadrant w % 4 and each take
 //                   half of the chunk's keys and half of the output columns
 //                   (row maxima and sums exchanged through shared memory).  P_j is written back over S_j as f16
@@ -32,6 +33,8 @@
 // from LayerNorm'd rows times weights of magnitude well inside the f16
 // range, P lies in [0, 1]); accumulation, softmax statistics and the output
 // are fp32, the output leaves as a bf16 hi/lo pair.
+#include <cstdlib>
+
 #include "fe_common.cuh"
 #include "fe_kernels.h"
 
@@ -48,8 +51,8 @@ struct AttnCfg {
   static constexpr int CK = DH == 32 ? 64 : 128;                // keys per chunk
   static constexpr int kSoftmaxWarps = 8;
   static constexpr int kHalves = kSoftmaxWarps / 4;              // warps sharing one lane quadrant
+  static_assert(kHalves == 2, "two softmax warps per TMEM lane quadrant");
   static constexpr int KW = CK / kHalves;                        // keys per softmax warp and chunk
-  static constexpr int kThreads = 64 + 32 * kSoftmaxWarps;
   static constexpr int kCtasPerSM = DH == 32 ? 2 : 1;
   // TMEM: S/P tiles at [t CK, t CK + CK), t < 3; the output accumulators of
   // consecutive units (alternating) at [3CK, 3CK + 2DH)
@@ -64,7 +67,13 @@ struct AttnCfg {
   static constexpr uint32_t kKVBytes = 2 * kKVTile;             // K, V
   static constexpr int kKVStages = DH == 32 ? 8 : 4;
   static constexpr uint32_t kRed = 2 * 2 * 2 * 128 * 4;       // [max|sum][parity][half][row]
-  static constexpr size_t kSmem = 1024 + 2 * kQBytes + kKVStages * kKVBytes + 256 + kRed;
+  // output staging for d_h = 64, per TMEM lane quadrant: [plane hi|lo][32 rows][NC 16-byte chunks]
+  // (for d_h = 32 the direct stores measured faster: 32-byte row pieces, and
+  // the unit's end waits on its last PV anyway)
+  static constexpr bool kStageOut = DH == 64;
+  static constexpr int NC = DH / 8;                            // 16-byte chunks in a row of one plane
+  static constexpr uint32_t kStageQuad = kStageOut ? 2 * 32 * NC * 16 : 0;
+  static constexpr size_t kSmem = 1024 + 2 * kQBytes + kKVStages * kKVBytes + 256 + kRed + 4 * kStageQuad;
 };
 
 __device__ __forceinline__ uint64_t desc_sw(uint32_t saddr, uint32_t sbo, uint32_t swz) {
@@ -168,8 +177,15 @@ __device__ __noinline__ void zero_tail(uint8_t* t, int o0, int end) {
   fence_async_shared();
 }
 
-template <int DH>
-__global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM)
+// Warps ahead of the softmax warps: the producer and one MMA issuer, or the
+// producer and separate S and PV issuers.
+template <bool SPLIT>
+__host__ __device__ constexpr int attn_role_warps() { return SPLIT ? 3 : 2; }
+template <int DH, bool SPLIT>
+__host__ __device__ constexpr int attn_threads() { return 32 * (attn_role_warps<SPLIT>() + AttnCfg<DH>::kSoftmaxWarps); }
+
+template <int DH, bool SPLIT>
+__global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasPerSM)
     attn_kernel(const __grid_constant__ CUtensorMap tQ, const __grid_constant__ CUtensorMap tK,
                 const __grid_constant__ CUtensorMap tV, const AttnParams p) {
   using Cfg = AttnCfg<DH>;
@@ -188,6 +204,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
   uint64_t* p_full = bars + 23;     // [3] P_j written over S_j
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 26);
   float* red = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // row-statistic exchange
+  uint8_t* stage = reinterpret_cast<uint8_t*>(bars) + 256 + Cfg::kRed;             // output staging
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qtiles = p.max_q_tiles;
@@ -264,7 +281,7 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         ++ui;
       }
     }
-  } else if (warp == 1) {
+  } else if (!SPLIT && warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
       // The chunks of all this CTA's units form one stream g = 0, 1, ...;
@@ -358,11 +375,115 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
         }
       }
     }
+  } else if (SPLIT && warp == 1) {
+    if (lane == 0) {
+      // ---------------- S issuer ----------------
+      // The chunks of all this CTA's units form one stream g = 0, 1, ...; S_g
+      // goes into TMEM tile g % 3 as soon as its K chunk has landed and PV_{g-3}
+      // has released the tile, across unit boundaries too, so the softmax finds
+      // the next S ready when it gets there.  Running indices and descriptors
+      // as a base plus an offset keep this thread's serial path short.
+      constexpr int NS = Cfg::kKVStages;
+      static_assert((NS & (NS - 1)) == 0, "K/V stages: a power of two");
+      const uint32_t idesc_s = umma_idesc_f16(BQ, CK);
+      const uint64_t qd0 = desc_sw(smem_u32(sQ), Cfg::kSbo, Cfg::kSwz);
+      const uint64_t kd0 = desc_sw(smem_u32(sKV), Cfg::kSbo, Cfg::kSwz);
+      int g_s = 0, t_s = 0, sui = 0;
+      Cursor sc;
+      bool ok = true;
+      for (cur_first(p, units, sc); sc.u < units && ok; cur_next(p, units, sc)) {
+        const int qb = sui & 1;
+        if (!mbar_wait_compact(q_full + qb, (sui >> 1) & 1, p.status)) break;
+        const uint64_t qd = qd0 + (uint64_t)((qb * Cfg::kQBytes) >> 4);
+        const int nch = chunks(sc);
+        for (int j = 0; j < nch; ++j) {
+          // the tile is free once PV_{g_s-3}, which reads P_{g_s-3} from it, has completed
+          if (g_s >= Cfg::kTiles) {
+            const int gp = g_s - Cfg::kTiles;
+            if (!mbar_wait_ready(kv_empty + (gp & (NS - 1)), (uint32_t)(gp / NS) & 1u, p.status)) {
+              ok = false;
+              break;
+            }
+          }
+          const int ks = g_s & (NS - 1);
+          if (!mbar_wait_ready(kv_full + ks, (uint32_t)(g_s / NS) & 1u, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t dst = tmem + (uint32_t)(t_s * CK);
+          const uint64_t kd = kd0 + (uint64_t)((ks * Cfg::kKVBytes) >> 4);
+#pragma unroll
+          for (int kk = 0; kk < DH / 16; ++kk)
+            umma_bf16(dst, qd + (uint64_t)(kk * 2), kd + (uint64_t)(kk * 2), idesc_s, kk != 0 ? 1u : 0u);
+          umma_commit(s_full + t_s);
+          ++g_s;
+          t_s = t_s == Cfg::kTiles - 1 ? 0 : t_s + 1;
+        }
+        if (!ok) break;
+        umma_commit(q_empty + qb);  // every S of this unit issued: its Q buffer frees on completion
+        ++sui;
+      }
+    }
+  } else if (SPLIT && warp == 2) {
+    if (lane == 0) {
+      // ---------------- PV issuer ----------------
+      // PV_g = P_g V_g, P_g read from TMEM tile g % 3 once the softmax has
+      // written it, accumulated into the unit's output accumulator (two,
+      // alternating by unit), from zero at the unit's first chunk.  One commit
+      // per product, on the K/V stage's empty barrier, tells every role that
+      // PV_g is complete: the producer may refill the stage, the S issuer may
+      // write S_{g+3} over P_g, the softmax may rescale or read the output.
+      constexpr int NS = Cfg::kKVStages;
+      const uint32_t idesc_pv = umma_idesc_f16(BQ, DH) | (1u << 16);  // B (V) is MN-major
+      // only a variable key count or one that is not a multiple of CK leaves a
+      // partial chunk, whose V rows a segmented map already reads as zeros
+      const bool pad_v = p.kv_self || (p.kv_cnt % CK != 0 && !p.kv_seg);
+      const uint64_t vd0 = desc_sw(smem_u32(sKV + Cfg::kKVTile), Cfg::kSbo, Cfg::kSwz);
+      int g = 0, t = 0, ui = 0;
+      uint32_t p_par = 0;  // parity of P_g's phase on p_full[t]: (g / 3) & 1
+      Cursor c;
+      bool ok = true;
+      for (cur_first(p, units, c); c.u < units && ok; cur_next(p, units, c)) {
+        const uint32_t dst = tmem + (uint32_t)(Cfg::kTiles * CK + (ui & 1) * DH);
+        const int nch = chunks(c);
+        for (int j = 0; j < nch; ++j, ++g) {
+          if (!mbar_wait_compact(p_full + t, p_par, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const int ks = g & (NS - 1);
+          // The V rows of a partial chunk past the key count belong to the
+          // next segment: their P is 0, but 0 x NaN is NaN, so they are zeroed
+          // (the chunk landed before S_g, which P_g follows)
+          if (pad_v) {
+            const int kval = kv_count(c) - j * CK;
+            if (kval < CK) zero_tail(sKV + ks * Cfg::kKVBytes + Cfg::kKVTile, kval * (int)Cfg::kRowBytes, (int)Cfg::kKVTile);
+          }
+          // A = P_g from the tile: each softmax warp's KW keys as KW/2 columns
+          // of f16 pairs at the start of its KW S columns
+          const uint64_t vd = vd0 + (uint64_t)((ks * Cfg::kKVBytes) >> 4);
+          const uint32_t pt = tmem + (uint32_t)(t * CK);
+#pragma unroll
+          for (int kk = 0; kk < CK / 16; ++kk)
+            umma_bf16_tmem_a(dst, pt + (uint32_t)((kk / (Cfg::KW / 16)) * Cfg::KW + (kk % (Cfg::KW / 16)) * 8),
+                             vd + (uint64_t)((kk * 16 * Cfg::kRowBytes) >> 4), idesc_pv,
+                             (kk != 0 || j != 0) ? 1u : 0u);
+          umma_commit(kv_empty + ks);
+          if (++t == Cfg::kTiles) {
+            t = 0;
+            p_par ^= 1u;
+          }
+        }
+        ++ui;
+      }
+    }
   } else {
     // ---------------- softmax / output (warps 2..9) ----------------
     constexpr int DO = DH / Cfg::kHalves;  // output columns per warp
     constexpr int KW = Cfg::KW;            // keys per warp and chunk (32 for d_h = 32, 64 for d_h = 64)
-    const int sw = warp - 2;
+    const int sw = warp - attn_role_warps<SPLIT>();
     const int q4 = warp & 3;
     const int half = sw >> 2;     // keys [KW half, KW half + KW) of each chunk, output columns [DO half, DO half + DO)
     const int r = q4 * 32 + lane; // query row of the tile = TMEM lane
@@ -389,34 +510,75 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
     } dn{};
     bool have_done = false;
     // once the unit's last PV has completed: O / l (l summed over both key
-    // halves) as a split pair
+    // halves) as a split pair.  Each lane holds one query row.  For d_h = 64
+    // the two warps of a lane quadrant stage their halves of the quadrant's
+    // 32 rows in shared memory (16-byte chunks XOR-swizzled by row: no bank
+    // conflicts on either side) and then each stores one plane, a lane per
+    // chunk, so that a warp instruction writes whole 128-byte rows instead of
+    // touching 32 rows
+    constexpr int NC = Cfg::NC;
+    auto swz = [](int row) { return NC == 8 ? (row & 7) : ((row >> 1) & 3); };
     auto finish = [&]() -> bool {
-      float ltot = dn.l;
-      if (Cfg::kHalves == 2) {
-        float* rs = red_sum + (dn.ui & 1) * 256;
-        rs[half * 128 + r] = dn.l;
-        pair_sync();
-        ltot = rs[r] + rs[128 + r];
-      }
+      float* rs = red_sum + (dn.ui & 1) * 256;
+      rs[half * 128 + r] = dn.l;
+      pair_sync();
+      const float ltot = rs[r] + rs[128 + r];
       if (!dn.active) return true;
-      if (!mbar_wait_compact(kv_empty + (dn.g % Cfg::kKVStages), (uint32_t)(dn.g / Cfg::kKVStages) & 1u, p.status))
-        return false;
-      tc_fence_after();
-      float o[DO];
-      o_load(o_cols(dn.ui), o);
-      if (dn.q0 + r < dn.qcnt) {
-        const float inv = 1.f / ltot;
-        const size_t go = (size_t)(dn.qoff + dn.q0 + r) * p.ldo + p.o_col + dn.h * DH + half * DO;
+      // with staging, both warps of the pair meet at the second barrier below, also after a timed-out wait
+      const bool okw = mbar_wait_compact(kv_empty + (dn.g % Cfg::kKVStages),
+                                         (uint32_t)(dn.g / Cfg::kKVStages) & 1u, p.status);
+      if constexpr (!Cfg::kStageOut) {
+        if (!okw) return false;
+        tc_fence_after();
+        float o[DO];
+        o_load(o_cols(dn.ui), o);
+        if (dn.q0 + r < dn.qcnt) {
+          const float inv = 1.f / ltot;
+          const size_t go = (size_t)(dn.qoff + dn.q0 + r) * p.ldo + p.o_col + dn.h * DH + half * DO;
 #pragma unroll
-        for (int c = 0; c < DO; c += 8) {
-          uint32_t hi[4], lo[4];
+          for (int c = 0; c < DO; c += 8) {
+            uint32_t hi[4], lo[4];
 #pragma unroll
-          for (int i = 0; i < 8; i += 2) split2(o[c + i] * inv, o[c + i + 1] * inv, hi[i / 2], lo[i / 2]);
-          *reinterpret_cast<uint4*>(p.o_h + go + c) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-          *reinterpret_cast<uint4*>(p.o_l + go + c) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            for (int i = 0; i < 8; i += 2) split2(o[c + i] * inv, o[c + i + 1] * inv, hi[i / 2], lo[i / 2]);
+            *reinterpret_cast<uint4*>(p.o_h + go + c) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+            *reinterpret_cast<uint4*>(p.o_l + go + c) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+          }
         }
+        return true;
+      } else {
+        uint8_t* st = stage + q4 * Cfg::kStageQuad;
+        if (okw) {
+          tc_fence_after();
+          float o[DO];
+          o_load(o_cols(dn.ui), o);
+          const float inv = 1.f / ltot;
+#pragma unroll
+          for (int c = 0; c < DO; c += 8) {
+            uint32_t hi[4], lo[4];
+#pragma unroll
+            for (int i = 0; i < 8; i += 2) split2(o[c + i] * inv, o[c + i + 1] * inv, hi[i / 2], lo[i / 2]);
+            const int pc = (half * (DO / 8) + c / 8) ^ swz(lane);
+            *reinterpret_cast<uint4*>(st + (lane * NC + pc) * 16) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+            *reinterpret_cast<uint4*>(st + ((32 + lane) * NC + pc) * 16) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+          }
+        }
+        pair_sync();
+        if (!okw) return false;
+        // warp `half` stores plane `half` (hi, lo) of the quadrant's rows
+        const uint8_t* src = st + half * 32 * NC * 16;
+        bf16* dst = half ? p.o_l : p.o_h;
+        const int row0 = dn.q0 + q4 * 32;
+#pragma unroll
+        for (int i = 0; i < NC; ++i) {
+          const int idx = i * 32 + lane;
+          const int row = idx / NC, ch = idx % NC;
+          if (row0 + row < dn.qcnt) {
+            const uint4 v = *reinterpret_cast<const uint4*>(src + (row * NC + (ch ^ swz(row))) * 16);
+            *reinterpret_cast<uint4*>(dst + (size_t)(dn.qoff + row0 + row) * p.ldo + p.o_col + dn.h * DH + ch * 8) = v;
+          }
+        }
+        return true;
       }
-      return true;
     };
     int gc = 0, ui = 0;
     bool ok = true;
@@ -545,17 +707,27 @@ __global__ void __launch_bounds__(AttnCfg<DH>::kThreads, AttnCfg<DH>::kCtasPerSM
 
 namespace {
 int g_attn_sms = 0;
+// a launch whose CTAs each walk at least this many key chunks takes the split issuers
+constexpr long long kSplitChunks = 32;
+int g_attn_split = -1;  // FE_ATTN_SPLIT for d_h = 32: 0 one issuer, 1 split issuers, unset by chunks per CTA
 }
 
 cudaError_t attn_prepare() {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&g_attn_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (g_attn_split < 0) {
+    const char* v = std::getenv("FE_ATTN_SPLIT");
+    g_attn_split = v && *v ? (std::atoi(v) != 0 ? 1 : 0) : 2;
+  }
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(attn_kernel<32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)AttnCfg<32>::kSmem);
   if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(attn_kernel<32, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)AttnCfg<32>::kSmem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(attn_kernel<64, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)AttnCfg<64>::kSmem);
   return e;
 }
@@ -569,14 +741,20 @@ cudaError_t attn_launch(int dh, const CUtensorMap* q, const CUtensorMap* k, cons
   p.max_q_tiles = (p.max_q + BQ - 1) / BQ;
   const long long units = (long long)p.n_segments * p.n_heads * p.max_q_tiles;
   const long long sms = g_attn_sms > 0 ? g_attn_sms : 148;
+  const int ck = attn_chunk_keys(dh);
+  const long long grid_max = sms * (dh == 32 ? AttnCfg<32>::kCtasPerSM : AttnCfg<64>::kCtasPerSM);
+  const long long grid = units < grid_max ? units : grid_max;
+  // key chunks per CTA: the split issuers pay off once each CTA walks many
+  const long long keys = p.kv_self ? p.max_q : p.kv_cnt;
+  const long long per_cta = units * ((keys + ck - 1) / ck) / grid;
+  const bool split = g_attn_split == 2 ? per_cta >= kSplitChunks : g_attn_split == 1;  // d_h = 64 always splits
+  const dim3 g((unsigned)grid);
   if (dh == 32) {
-    const long long grid = units < sms * AttnCfg<32>::kCtasPerSM ? units : sms * AttnCfg<32>::kCtasPerSM;
-    return launch_k(attn_kernel<32>, dim3((unsigned)grid), dim3(AttnCfg<32>::kThreads), AttnCfg<32>::kSmem, s, *q, *k,
-                    *v, p);
+    if (split)
+      return launch_k(attn_kernel<32, true>, g, dim3(attn_threads<32, true>()), AttnCfg<32>::kSmem, s, *q, *k, *v, p);
+    return launch_k(attn_kernel<32, false>, g, dim3(attn_threads<32, false>()), AttnCfg<32>::kSmem, s, *q, *k, *v, p);
   }
-  const long long grid = units < sms * AttnCfg<64>::kCtasPerSM ? units : sms * AttnCfg<64>::kCtasPerSM;
-  return launch_k(attn_kernel<64>, dim3((unsigned)grid), dim3(AttnCfg<64>::kThreads), AttnCfg<64>::kSmem, s, *q, *k,
-                  *v, p);
+  return launch_k(attn_kernel<64, true>, g, dim3(attn_threads<64, true>()), AttnCfg<64>::kSmem, s, *q, *k, *v, p);
 }
 
 }  // namespace fe
