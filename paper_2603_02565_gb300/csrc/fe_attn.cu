@@ -127,14 +127,13 @@ __device__ __forceinline__ void mbar_arrive1(uint64_t* bar) {
 
 // Unit cursor: unit u -> (segment b, head h, query tile t); query tile fastest.
 // Every role walks its CTA's units u = blockIdx.x + i * gridDim.x and skips
-// tiles that start past their segment's end.  With INC the position of
-// u + gridDim.x follows from that of u by adding gridDim.x's digits in the
-// same mixed radix (tiles, heads), kept in shared memory, so that a role moving
-// to its next unit does not divide (the one-issuer form, where the issuer's
-// serial path sets the pace); otherwise the position is divided out of u (the
-// split form, whose register budget is the tighter constraint).  The segment
-// count and offset of the next candidate unit are loaded one unit ahead, so a
-// role crossing into its next unit does not wait on a global load.
+// tiles that start past their segment's end.  The position of u + gridDim.x
+// follows from that of u by adding gridDim.x's digits in the same mixed radix
+// (tiles, heads), kept in shared memory, so that a role moving to its next
+// unit does not divide (an integer division is a long serial chain on the
+// issuing thread, whose pace sets the kernel's).  The segment count and offset
+// of the next candidate unit are loaded one unit ahead, so a role crossing into
+// its next unit does not wait on a global load.
 struct Cursor {
   int u, b, h, q0, qcnt, qoff;
   int pcnt, poff;  // q_cnt / q_off of unit u + gridDim.x
@@ -164,49 +163,35 @@ __device__ __forceinline__ void cur_fetch(const AttnParams& p, int b, int& cnt, 
 
 // settle on the first unit at or after c.u whose tile holds query rows, then
 // load the counts of the unit after it
-template <bool INC>
 __device__ __forceinline__ void cur_settle(const AttnParams& p, const int* step, int units, Cursor& c) {
-  if constexpr (INC) {
-    while (c.u < units && c.q0 >= c.qcnt) {
-      c.u += gridDim.x;
-      if (c.u < units) {
-        pos_add(p, step, c.b, c.h, c.q0);
-        cur_fetch(p, c.b, c.qcnt, c.qoff);
-      }
+  while (c.u < units && c.q0 >= c.qcnt) {
+    c.u += gridDim.x;
+    if (c.u < units) {
+      pos_add(p, step, c.b, c.h, c.q0);
+      cur_fetch(p, c.b, c.qcnt, c.qoff);
     }
-    if (c.u < units && c.u + (int)gridDim.x < units) {
-      int nb = c.b, nh = c.h, nq = c.q0;
-      pos_add(p, step, nb, nh, nq);
-      cur_fetch(p, nb, c.pcnt, c.poff);
-    }
-  } else {
-    while (c.u < units) {
-      pos_of(p, c.u, c.b, c.h, c.q0);
-      if (c.q0 < c.qcnt) break;
-      c.u += gridDim.x;
-      if (c.u < units) cur_fetch(p, c.u / (p.max_q_tiles * p.n_heads), c.qcnt, c.qoff);
-    }
-    if (c.u < units && c.u + (int)gridDim.x < units)
-      cur_fetch(p, (c.u + (int)gridDim.x) / (p.max_q_tiles * p.n_heads), c.pcnt, c.poff);
+  }
+  if (c.u < units && c.u + (int)gridDim.x < units) {
+    int nb = c.b, nh = c.h, nq = c.q0;
+    pos_add(p, step, nb, nh, nq);
+    cur_fetch(p, nb, c.pcnt, c.poff);
   }
 }
 
-template <bool INC>
 __device__ __forceinline__ void cur_first(const AttnParams& p, const int* step, int units, Cursor& c) {
   c.u = blockIdx.x;
-  if constexpr (INC) pos_of(p, c.u, c.b, c.h, c.q0);
-  cur_fetch(p, c.u / (p.max_q_tiles * p.n_heads), c.qcnt, c.qoff);
-  cur_settle<INC>(p, step, units, c);
+  pos_of(p, c.u, c.b, c.h, c.q0);
+  cur_fetch(p, c.b, c.qcnt, c.qoff);
+  cur_settle(p, step, units, c);
 }
 
-template <bool INC>
 __device__ __forceinline__ void cur_next(const AttnParams& p, const int* step, int units, Cursor& c) {
   c.u += gridDim.x;
   if (c.u >= units) return;
-  if constexpr (INC) pos_add(p, step, c.b, c.h, c.q0);
+  pos_add(p, step, c.b, c.h, c.q0);
   c.qcnt = c.pcnt;
   c.qoff = c.poff;
-  cur_settle<INC>(p, step, units, c);
+  cur_settle(p, step, units, c);
 }
 
 }  // namespace
@@ -272,7 +257,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
       mbar_init(kv_empty + i, 1);
     }
     fence_mbar_init();
-    if (!SPLIT) pos_of(p, (int)gridDim.x, step[0], step[1], step[2]);
+    pos_of(p, (int)gridDim.x, step[0], step[1], step[2]);
     prefetch_tmap(&tQ);
     prefetch_tmap(&tK);
     prefetch_tmap(&tV);
@@ -293,7 +278,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
       int ui = 0, gc = 0;
       bool ok = true;
       Cursor c;
-      for (cur_first<!SPLIT>(p, step, units, c); c.u < units && ok; cur_next<!SPLIT>(p, step, units, c)) {
+      for (cur_first(p, step, units, c); c.u < units && ok; cur_next(p, step, units, c)) {
         const int qb = ui & 1;
         if (ui >= 2 && !mbar_wait_compact(q_empty + qb, ((ui >> 1) - 1) & 1, p.status)) break;
         uint8_t* q = sQ + qb * Cfg::kQBytes;
@@ -350,7 +335,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
       // per chunk g (g % 4; at most two chunks separate S and PV): its unit
       // counter's parity (the output accumulator) and whether it opens the unit
       uint32_t pv_info = 0;
-      cur_first<!SPLIT>(p, step, units, sc);
+      cur_first(p, step, units, sc);
       if (sc.u < units) s_nch = chunks(sc);
       // S = Q K^T of the chunk at the S cursor into TMEM tile t_s, then advance the cursor
       auto issue_next_s = [&]() -> bool {
@@ -386,7 +371,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
           umma_commit(q_empty + qb);
           sj = 0;
           ++sui;
-          cur_next<!SPLIT>(p, step, units, sc);
+          cur_next(p, step, units, sc);
           if (sc.u < units) s_nch = chunks(sc);
         }
         return true;
@@ -434,7 +419,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
       int g_s = 0, t_s = 0, sui = 0;
       Cursor sc;
       bool ok = true;
-      for (cur_first<!SPLIT>(p, step, units, sc); sc.u < units && ok; cur_next<!SPLIT>(p, step, units, sc)) {
+      for (cur_first(p, step, units, sc); sc.u < units && ok; cur_next(p, step, units, sc)) {
         const int qb = sui & 1;
         if (!mbar_wait_compact(q_full + qb, (sui >> 1) & 1, p.status)) break;
         const uint64_t qd = qd0 + (uint64_t)((qb * Cfg::kQBytes) >> 4);
@@ -487,7 +472,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
       uint32_t p_par = 0;  // parity of P_g's phase on p_full[t]: (g / 3) & 1
       Cursor c;
       bool ok = true;
-      for (cur_first<!SPLIT>(p, step, units, c); c.u < units && ok; cur_next<!SPLIT>(p, step, units, c)) {
+      for (cur_first(p, step, units, c); c.u < units && ok; cur_next(p, step, units, c)) {
         const uint32_t dst = tmem + (uint32_t)(Cfg::kTiles * CK + (ui & 1) * DH);
         const int nch = chunks(c);
         for (int j = 0; j < nch; ++j, ++g) {
@@ -626,7 +611,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
     int gc = 0, ui = 0;
     bool ok = true;
     Cursor c;
-    for (cur_first<!SPLIT>(p, step, units, c); c.u < units && ok; cur_next<!SPLIT>(p, step, units, c)) {
+    for (cur_first(p, step, units, c); c.u < units && ok; cur_next(p, step, units, c)) {
       // the running maximum m that P is taken against moves only when a chunk's
       // maximum exceeds it by more than kSlack (log2 units; P <= 2^kSlack stays
       // far inside f16), and then the unit's output accumulator in TMEM is
