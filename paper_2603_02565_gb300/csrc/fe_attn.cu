@@ -24,14 +24,17 @@
 //   the other 8   : online softmax from TMEM, one query row per lane; warps
 //                   w and w+4 share TMEM lane quadrant w % 4 and each take
 //                   half of the chunk's keys and half of the output columns
-//                   (row maxima and sums exchanged through shared memory).  P_j is written back over S_j as f16
-//                   against a running maximum that moves only when a chunk
-//                   exceeds it by more than 2^8, when the output accumulator
-//                   is rescaled in TMEM; otherwise the softmax never reads
-//                   the PV products until the unit's output is stored
+//                   (row maxima and sums exchanged through shared memory).
+//                   P_j is written back over S_j as f16 against a running
+//                   maximum that moves only when a chunk exceeds it by more
+//                   than 8 (log2 units), when the output accumulator is
+//                   rescaled in TMEM; otherwise the softmax never reads the PV
+//                   products until the unit's output is stored (for d_h = 64
+//                   staged through shared memory, so that the stores write
+//                   whole rows)
 // Q, K, V and P are single f16 planes (unit roundoff 2^-11; Q and K come
 // from LayerNorm'd rows times weights of magnitude well inside the f16
-// range, P lies in [0, 1]); accumulation, softmax statistics and the output
+// range, P lies in [0, 2^8]); accumulation, softmax statistics and the output
 // are fp32, the output leaves as a bf16 hi/lo pair.
 #include <cstdlib>
 
@@ -508,7 +511,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
       }
     }
   } else {
-    // ---------------- softmax / output (warps 2..9) ----------------
+    // ---------------- softmax / output (the last eight warps) ----------------
     constexpr int DO = DH / Cfg::kHalves;  // output columns per warp
     constexpr int KW = Cfg::KW;            // keys per warp and chunk (32 for d_h = 32, 64 for d_h = 64)
     const int sw = warp - attn_role_warps<SPLIT>();
