@@ -275,7 +275,14 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
   pdl_trigger();
   pdl_wait();
 
-  if (warp == 0) {
+  // Two CTAs share an SM in the d_h = 32 launches, and a grid of two per SM
+  // places the second half of the grid second on each SM: there the one-issuer
+  // form swaps the producer and issuer warps, so that the two CTAs' issuing
+  // threads sit on different SM sub-partitions (warp w runs on sub-partition
+  // w % 4) instead of competing for one's issue slots
+  const bool swap_roles = !SPLIT && Cfg::kCtasPerSM == 2 && (int)blockIdx.x >= (int)(gridDim.x >> 1);
+  const int w_prod = swap_roles ? 1 : 0, w_mma = swap_roles ? 0 : 1;
+  if (warp == w_prod) {
     if (lane == 0) {
       // ---------------- TMA producer ----------------
       int ui = 0, gc = 0;
@@ -312,7 +319,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
         ++ui;
       }
     }
-  } else if (!SPLIT && warp == 1) {
+  } else if (!SPLIT && warp == w_mma) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
       // The chunks of all this CTA's units form one stream g = 0, 1, ...;
