@@ -276,12 +276,15 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
   pdl_wait();
 
   // Two CTAs share an SM in the d_h = 32 launches, and a grid of two per SM
-  // places the second half of the grid second on each SM: there the one-issuer
-  // form swaps the producer and issuer warps, so that the two CTAs' issuing
-  // threads sit on different SM sub-partitions (warp w runs on sub-partition
-  // w % 4) instead of competing for one's issue slots
-  const bool swap_roles = !SPLIT && Cfg::kCtasPerSM == 2 && (int)blockIdx.x >= (int)(gridDim.x >> 1);
-  const int w_prod = swap_roles ? 1 : 0, w_mma = swap_roles ? 0 : 1;
+  // places the second half of the grid second on each SM: there the role warps
+  // rotate (one issuer: producer and issuer swap; two issuers: producer, S and
+  // PV issuers move to warps 2, 0, 1), so that the two CTAs' issuing threads
+  // sit on different SM sub-partitions (warp w runs on sub-partition w % 4)
+  // instead of competing for one's issue slots
+  const bool second = Cfg::kCtasPerSM == 2 && (int)blockIdx.x >= (int)(gridDim.x >> 1);
+  const int w_prod = second ? (SPLIT ? 2 : 1) : 0;
+  const int w_mma = second ? 0 : 1;             // one issuer; with two, the S issuer
+  const int w_pv = second ? 1 : 2;              // two issuers: the PV issuer
   if (warp == w_prod) {
     if (lane == 0) {
       // ---------------- TMA producer ----------------
@@ -413,7 +416,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
         }
       }
     }
-  } else if (SPLIT && warp == 1) {
+  } else if (SPLIT && warp == w_mma) {
     if (lane == 0) {
       // ---------------- S issuer ----------------
       // The chunks of all this CTA's units form one stream g = 0, 1, ...; S_g
@@ -463,7 +466,7 @@ __global__ void __launch_bounds__(attn_threads<DH, SPLIT>(), AttnCfg<DH>::kCtasP
         ++sui;
       }
     }
-  } else if (SPLIT && warp == 2) {
+  } else if (SPLIT && warp == w_pv) {
     if (lane == 0) {
       // ---------------- PV issuer ----------------
       // PV_g = P_g V_g, P_g read from TMEM tile g % 3 once the softmax has
